@@ -1,0 +1,387 @@
+/*
+ * pmpe_oracle.c -- plain CPU oracle for the policy-masked sparse-MoE layer
+ * forward of "Policy-Masked Private Experts" (arXiv 2608.06690).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the slow, obviously-correct
+ * definition that the GPU path is checked against.  Only the test suite,
+ * the smoke check and the benchmark's CPU-baseline leg may load it.  It
+ * shares no code, header, table or helper with the CUDA library; the two
+ * only meet in the seeded input generator, which holds none of the method's
+ * arithmetic.
+ *
+ * Arithmetic: every dot product accumulates in double (fp64) from the BF16
+ * operands.  Three rounding points are part of the reading of the method, not
+ * of any kernel:
+ *   - router logits are rounded to fp32 before the top-k decision (the
+ *     routing decision is taken on fp32 logits on both sides);
+ *   - the SwiGLU activation silu(g)*u is rounded to BF16, because it is the
+ *     BF16 operand of the down projection in a BF16 model;
+ *   - the layer output is rounded once to BF16 (round to nearest even).
+ * Everything else (g, u, y, the weighted sum) stays in double.
+ *
+ * Parity status: the values are pinned by closed forms, special cases that
+ * reduce to a textbook SwiGLU MLP / softmax / sort, brute force on tiny
+ * inputs and the audit invariants of Sec. 2.2 (Eq. 1, G1).  The paper prints
+ * no worked numeric example of the layer, so no printed value pins it; the
+ * hand-worked fixtures under tests/golden/ are derived from the definitions.
+ *
+ * Method passages followed (paper sections / equations):
+ *   - Sec. 2.1 (threat model) and App. B.1 (policy resolution): missing,
+ *     malformed or non-Boolean authorisation resolves to tau = 0.  As a byte
+ *     per token: only 0x01 is ALLOW; NULL means every token is DENY.
+ *   - Sec. 3.1, Eq. 4 (the mask m_{l,e}(tau)) and the sentence after it: top-k
+ *     is taken over z_l(h) + m_l(tau), m = 0 on the eligible pool and -inf on
+ *     the other one; public ids 0..E_pub-1, private ids E_pub..E_pub+E_priv-1
+ *     (the concatenated public/private pool of Sec. 4.2).
+ *   - App. B.1 fail-closed procedure, steps 2, 4, 5: resolve, mask then
+ *     top-k, record the route.
+ *   - Sec. 3.1 / Sec. 4.2: private experts copy the public expert
+ *     architecture (gate, up, down projections: a SwiGLU MLP).
+ *   - Sec. 5.2 / App. F.1: independent execution counts observed at the
+ *     expert modules themselves, separate from the route log.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+typedef struct {
+    int T, H, I, E_pub, E_priv, E_sh, k;
+    int renormalize;                 /* 1: softmax renormalised over the top-k; 0: pool softmax probs */
+    const uint16_t *hidden;          /* [T][H] BF16 bits */
+    const uint8_t *policy;           /* [T] bytes, or NULL */
+    const uint16_t *router_pub;      /* [E_pub][H] */
+    const uint16_t *router_priv;     /* [E_priv][H] */
+    const uint16_t *gate_pub, *up_pub, *down_pub;     /* [E_pub][I][H], [E_pub][I][H], [E_pub][H][I] */
+    const uint16_t *gate_priv, *up_priv, *down_priv;  /* [E_priv][I][H], ..., [E_priv][H][I] */
+    const uint16_t *gate_sh, *up_sh, *down_sh;        /* [E_sh][I][H], ..., [E_sh][H][I]; NULL if E_sh == 0 */
+} oracle_layer;
+
+/* ---------------------------------------------------------------- BF16 -- */
+
+static double bf16_value(uint16_t b)
+{
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* Round a double to the nearest BF16 value, ties to even.  BF16 keeps
+ * 8 significant bits; for |x| in [2^(e-1), 2^e) the spacing is 2^(e-8),
+ * and below the smallest normal (2^-126) it is 2^-133. */
+uint16_t oracle_bf16_round(double x)
+{
+    if (isnan(x)) return 0x7FC0;
+    uint16_t sign = signbit(x) ? 0x8000 : 0;
+    double a = fabs(x);
+    if (a == 0.0) return sign;
+    if (isinf(a)) return sign | 0x7F80;
+    int e;
+    frexp(a, &e);                     /* a = m * 2^e with m in [0.5, 1) */
+    int q_exp = (e - 1 < -126) ? -133 : e - 8;
+    double q = nearbyint(ldexp(a, -q_exp));   /* default mode: ties to even */
+    double r = ldexp(q, q_exp);
+    if (r > 0x1.FEp127) return sign | 0x7F80; /* beyond the largest finite BF16 */
+    float f = (float)r;               /* exact: r is a BF16 value */
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    return sign | (uint16_t)(u >> 16);
+}
+
+double oracle_bf16_value(uint16_t b) { return bf16_value(b); }
+
+/* ------------------------------------------------------ policy resolve -- */
+
+/* tau_t = 1 only for the trusted byte 0x01; NULL policy -> all 0. */
+void oracle_resolve(const uint8_t *policy, int T, uint8_t *tau)
+{
+    for (int t = 0; t < T; ++t)
+        tau[t] = (policy != NULL && policy[t] == 0x01) ? 1 : 0;
+}
+
+/* ------------------------------------------------------------- routing -- */
+
+/* The row of the concatenated router for global expert id e. */
+static const uint16_t *router_row(const oracle_layer *L, int e)
+{
+    return e < L->E_pub ? L->router_pub + (size_t)e * L->H
+                        : L->router_priv + (size_t)(e - L->E_pub) * L->H;
+}
+
+/* Route one token: z_e over the concatenated pool, s = z + m(tau), top-k of s
+ * (descending, ties to the lower id), weights from the softmax of s.
+ * Writes idx[k], w[k], and the gap s_(k) - s_(k+1) inside the visible pool
+ * (+inf when k equals the pool size). */
+static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, double *gap,
+                        double *s /* scratch [E] */, char *taken /* scratch [E] */)
+{
+    const int E = L->E_pub + L->E_priv;
+    const int tau = (L->policy != NULL && L->policy[t] == 0x01);
+    const uint16_t *h = L->hidden + (size_t)t * L->H;
+
+    for (int e = 0; e < E; ++e) {
+        const uint16_t *wr = router_row(L, e);
+        double z = 0.0;
+        for (int c = 0; c < L->H; ++c) z += bf16_value(h[c]) * bf16_value(wr[c]);
+        const int eligible = tau ? (e >= L->E_pub) : (e < L->E_pub);
+        s[e] = eligible ? (double)(float)z : -INFINITY;   /* z + m(tau), z rounded to fp32 */
+        taken[e] = 0;
+    }
+    /* top-k by repeated selection: largest s, lower id on ties */
+    for (int j = 0; j < L->k; ++j) {
+        int best = -1;
+        for (int e = 0; e < E; ++e) {
+            if (taken[e] || s[e] == -INFINITY) continue;
+            if (best < 0 || s[e] > s[best]) best = e;
+        }
+        idx[j] = best;
+        taken[best] = 1;
+    }
+    /* (k+1)-th best in the visible pool, for the gap rule */
+    int next = -1;
+    for (int e = 0; e < E; ++e) {
+        if (taken[e] || s[e] == -INFINITY) continue;
+        if (next < 0 || s[e] > s[next]) next = e;
+    }
+    *gap = next < 0 ? INFINITY : s[idx[L->k - 1]] - s[next];
+
+    /* softmax over the masked logits (exp(-inf) = 0 drops the other pool) */
+    const double smax = s[idx[0]];
+    double denom_pool = 0.0;
+    for (int e = 0; e < E; ++e) denom_pool += exp(s[e] - smax);
+    double sel = 0.0;
+    for (int j = 0; j < L->k; ++j) {
+        w[j] = exp(s[idx[j]] - smax) / denom_pool;     /* p_e of the pool softmax */
+        sel += w[j];
+    }
+    if (L->renormalize)
+        for (int j = 0; j < L->k; ++j) w[j] /= sel;     /* renormalise over the top-k */
+}
+
+/* ------------------------------------------------------------- experts -- */
+
+/* One SwiGLU expert on one token: g = Wg h, u = Wu h, a = bf16(silu(g) u),
+ * y = Wd a.  Wg, Wu: [I][H]; Wd: [H][I].  Every call adds one row to
+ * *exec_counter: the execution count is observed here, where the expert
+ * runs, not copied from the route log. */
+static void swiglu_expert(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int I,
+                          const double *h, double *y, double *a, uint32_t *exec_counter)
+{
+    for (int i = 0; i < I; ++i) {
+        const uint16_t *rg = Wg + (size_t)i * H, *ru = Wu + (size_t)i * H;
+        double g = 0.0, u = 0.0;
+        for (int c = 0; c < H; ++c) {
+            g += h[c] * bf16_value(rg[c]);
+            u += h[c] * bf16_value(ru[c]);
+        }
+        const double silu = g / (1.0 + exp(-g));
+        a[i] = bf16_value(oracle_bf16_round(silu * u));
+    }
+    for (int o = 0; o < H; ++o) {
+        const uint16_t *rd = Wd + (size_t)o * I;
+        double acc = 0.0;
+        for (int i = 0; i < I; ++i) acc += a[i] * bf16_value(rd[i]);
+        y[o] = acc;
+    }
+    *exec_counter += 1;
+}
+
+static void routed_expert_weights(const oracle_layer *L, int e, const uint16_t **g, const uint16_t **u,
+                                  const uint16_t **d)
+{
+    const size_t ih = (size_t)L->I * L->H;
+    if (e < L->E_pub) {
+        *g = L->gate_pub + e * ih; *u = L->up_pub + e * ih; *d = L->down_pub + e * ih;
+    } else {
+        const int p = e - L->E_pub;
+        *g = L->gate_priv + p * ih; *u = L->up_priv + p * ih; *d = L->down_priv + p * ih;
+    }
+}
+
+/* ---------------------------------------------------------- public API -- */
+
+static int check_layer(const oracle_layer *L)
+{
+    if (!L || L->T < 0 || L->H <= 0 || L->I <= 0 || L->E_pub < 0 || L->E_priv < 0 || L->E_sh < 0) return -1;
+    if (L->k < 1 || L->k > L->E_pub || L->k > L->E_priv) return -1;
+    if (L->T > 0 && !L->hidden) return -1;
+    if (!L->router_pub || !L->router_priv) return -1;
+    return 0;
+}
+
+/* Routing only, for the tokens in `tokens` (NULL = all T).  Outputs are
+ * indexed by position in the list. */
+int oracle_route(const oracle_layer *L, const int32_t *tokens, int n, int32_t *idx, double *w, double *gap,
+                 int nthreads)
+{
+    if (check_layer(L)) return -1;
+    const int E = L->E_pub + L->E_priv;
+    if (!tokens) n = L->T;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+#pragma omp parallel
+    {
+        double *s = (double *)malloc(sizeof(double) * E);
+        char *taken = (char *)malloc(E);
+#pragma omp for schedule(dynamic, 4)
+        for (int p = 0; p < n; ++p) {
+            const int t = tokens ? tokens[p] : p;
+            route_token(L, t, idx + (size_t)p * L->k, w + (size_t)p * L->k, gap + p, s, taken);
+        }
+        free(s);
+        free(taken);
+    }
+    return 0;
+}
+
+/* One routed expert (global id e) or, with shared = 1, shared expert e, on a
+ * single BF16 hidden row.  y: [H] doubles. */
+int oracle_expert(const oracle_layer *L, int e, int shared, const uint16_t *h_row, double *y)
+{
+    if (!L || !h_row || !y) return -1;
+    const uint16_t *g, *u, *d;
+    if (shared) {
+        if (e < 0 || e >= L->E_sh) return -1;
+        const size_t ih = (size_t)L->I * L->H;
+        g = L->gate_sh + e * ih; u = L->up_sh + e * ih; d = L->down_sh + e * ih;
+    } else {
+        if (e < 0 || e >= L->E_pub + L->E_priv) return -1;
+        routed_expert_weights(L, e, &g, &u, &d);
+    }
+    double *h = (double *)malloc(sizeof(double) * L->H);
+    double *a = (double *)malloc(sizeof(double) * L->I);
+    for (int c = 0; c < L->H; ++c) h[c] = bf16_value(h_row[c]);
+    uint32_t dummy = 0;
+    swiglu_expert(g, u, d, L->H, L->I, h, y, a, &dummy);
+    free(h);
+    free(a);
+    return 0;
+}
+
+/* Full layer forward for the tokens in `tokens` (NULL = all T).
+ *   out_bf16 [n][H], out_f64 [n][H] (may be NULL), idx [n][k], w [n][k], gap [n]
+ *   route_count [E], route_priv_rows [n]      -- the route log
+ *   exec_rows [E], exec_priv_rows [n]         -- counted where the experts run
+ *   shared_rows [1]                           -- shared-expert executions
+ * Counters are overwritten (not accumulated). */
+int oracle_forward(const oracle_layer *L, const int32_t *tokens, int n, uint16_t *out_bf16, double *out_f64,
+                   int32_t *idx, double *w, double *gap, uint32_t *route_count, uint32_t *route_priv_rows,
+                   uint32_t *exec_rows, uint32_t *exec_priv_rows, uint32_t *shared_rows, int nthreads)
+{
+    if (check_layer(L)) return -1;
+    if (L->E_sh > 0 && (!L->gate_sh || !L->up_sh || !L->down_sh)) return -1;
+    const int E = L->E_pub + L->E_priv, H = L->H, I = L->I, k = L->k;
+    if (!tokens) n = L->T;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+    const int nt = omp_get_max_threads();
+#else
+    (void)nthreads;
+    const int nt = 1;
+#endif
+    /* per-thread execution counters, reduced in a fixed order afterwards */
+    uint32_t *exec_local = (uint32_t *)calloc((size_t)nt * (E + 1), sizeof(uint32_t));
+    uint32_t *exec_priv_local = (uint32_t *)calloc((size_t)n > 0 ? (size_t)n : 1, sizeof(uint32_t));
+
+#pragma omp parallel
+    {
+#ifdef _OPENMP
+        const int tid = omp_get_thread_num();
+#else
+        const int tid = 0;
+#endif
+        uint32_t *my_exec = exec_local + (size_t)tid * (E + 1);
+        double *s = (double *)malloc(sizeof(double) * E);
+        char *taken = (char *)malloc(E);
+        double *h = (double *)malloc(sizeof(double) * H);
+        double *y = (double *)malloc(sizeof(double) * H);
+        double *acc = (double *)malloc(sizeof(double) * H);
+        double *a = (double *)malloc(sizeof(double) * I);
+#pragma omp for schedule(dynamic, 1)
+        for (int p = 0; p < n; ++p) {
+            const int t = tokens ? tokens[p] : p;
+            int32_t *ti = idx + (size_t)p * k;
+            double *tw = w + (size_t)p * k;
+            route_token(L, t, ti, tw, gap + p, s, taken);
+
+            const uint16_t *hr = L->hidden + (size_t)t * H;
+            for (int c = 0; c < H; ++c) { h[c] = bf16_value(hr[c]); acc[c] = 0.0; }
+            for (int j = 0; j < k; ++j) {
+                const int e = ti[j];
+                const uint16_t *g, *u, *d;
+                routed_expert_weights(L, e, &g, &u, &d);
+                uint32_t before = my_exec[e];
+                swiglu_expert(g, u, d, H, I, h, y, a, &my_exec[e]);
+                if (e >= L->E_pub) exec_priv_local[p] += my_exec[e] - before;
+                for (int c = 0; c < H; ++c) acc[c] += tw[j] * y[c];
+            }
+            const size_t ih = (size_t)I * H;
+            for (int sidx = 0; sidx < L->E_sh; ++sidx) {
+                swiglu_expert(L->gate_sh + sidx * ih, L->up_sh + sidx * ih, L->down_sh + sidx * ih, H, I, h, y, a,
+                              &my_exec[E]);
+                for (int c = 0; c < H; ++c) acc[c] += y[c];
+            }
+            for (int c = 0; c < H; ++c) {
+                out_bf16[(size_t)p * H + c] = oracle_bf16_round(acc[c]);
+                if (out_f64) out_f64[(size_t)p * H + c] = acc[c];
+            }
+        }
+        free(s); free(taken); free(h); free(y); free(acc); free(a);
+    }
+
+    /* route log, from the routing decisions */
+    for (int e = 0; e < E; ++e) route_count[e] = 0;
+    for (int p = 0; p < n; ++p) {
+        route_priv_rows[p] = 0;
+        for (int j = 0; j < k; ++j) {
+            const int e = idx[(size_t)p * k + j];
+            route_count[e] += 1;
+            if (e >= L->E_pub) route_priv_rows[p] += 1;
+        }
+    }
+    /* execution log, from the expert calls */
+    for (int e = 0; e < E; ++e) exec_rows[e] = 0;
+    *shared_rows = 0;
+    for (int tid = 0; tid < nt; ++tid) {
+        for (int e = 0; e < E; ++e) exec_rows[e] += exec_local[(size_t)tid * (E + 1) + e];
+        *shared_rows += exec_local[(size_t)tid * (E + 1) + E];
+    }
+    for (int p = 0; p < n; ++p) exec_priv_rows[p] = exec_priv_local[p];
+    free(exec_local);
+    free(exec_priv_local);
+    return 0;
+}
+
+/* Dispatch order of the routed rows (the permutation any grouped expert
+ * execution needs): rows are grouped by expert id, and inside an expert by
+ * token then rank.  counts[e] = #{(t,j): idx[t][j] = e}; offsets = exclusive
+ * prefix sum of counts (E+1 entries); slot_of[t][j] = the row's position;
+ * tok_of_slot[slot] = t.  Returns -1 on an id outside [0, E). */
+int oracle_permute(const int32_t *idx, int T, int k, int E, uint32_t *counts, uint32_t *offsets, int32_t *slot_of,
+                   int32_t *tok_of_slot)
+{
+    for (int e = 0; e < E; ++e) counts[e] = 0;
+    for (size_t r = 0; r < (size_t)T * k; ++r) {
+        if (idx[r] < 0 || idx[r] >= E) return -1;
+        counts[idx[r]] += 1;
+    }
+    offsets[0] = 0;
+    for (int e = 0; e < E; ++e) offsets[e + 1] = offsets[e] + counts[e];
+    uint32_t next = 0;
+    for (int e = 0; e < E; ++e)
+        for (int t = 0; t < T; ++t)
+            for (int j = 0; j < k; ++j)
+                if (idx[(size_t)t * k + j] == e) {
+                    slot_of[(size_t)t * k + j] = (int32_t)next;
+                    tok_of_slot[next] = t;
+                    next += 1;
+                }
+    return 0;
+}

@@ -1,0 +1,303 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: an
+exhaustive enumeration, a closed form, a brute-force sort, a library routine
+(torch.nn.functional in fp64, torch's BF16 conversion) or a hand-worked
+fixture.  A plausible mistake in the oracle (a dropped mask, a wrong sign, a
+transposed weight, swapped gate/up, a wrong softmax denominator, a wrong tie
+break, an off-by-one in the dispatch order) fails at least one of them.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle
+from paper_2608_06690_gb300.inputs import LayerShape
+from pmpe_testlib import make_layer, oracle_layer, bits_to_f64
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "hand_worked.json")
+
+
+# ------------------------------------------------------------------ BF16
+
+def test_bf16_round_matches_torch_on_float32_values():
+    """The oracle's double->BF16 rounding equals torch's float32->BF16
+    round-to-nearest-even on values that are exact in float32 (so no double
+    rounding is involved), including ties, subnormals and overflow."""
+    g = torch.Generator().manual_seed(1)
+    x = torch.randn(20000, generator=g) * torch.exp(torch.randn(20000, generator=g) * 8)
+    ties = torch.tensor([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -(1.0 + 2.0 ** -8), 2.0 ** -130, 3.0 * 2.0 ** -134,
+                         3.3895e38, 3.4e38, -0.0, 0.0, 1e-45, 2.0 ** -126, 65504.0], dtype=torch.float32)
+    x = torch.cat([x.float(), ties])
+    want = x.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    got = np.array([oracle.bf16_round(float(v)) for v in x.tolist()], dtype=np.uint16)
+    assert np.array_equal(got, want)
+
+
+# ---------------------------------------------------------------- resolve
+
+def test_resolve_exhaustive_over_all_bytes():
+    """Sec. 2.1 / App. B.1: only the trusted ALLOW value gives tau = 1;
+    every other byte fails closed."""
+    pol = np.arange(256, dtype=np.uint8)
+    tau = oracle.resolve(pol, 256)
+    assert tau[1] == 1 and tau.sum() == 1
+
+
+def test_resolve_missing_metadata_is_deny():
+    assert oracle.resolve(None, 37).sum() == 0
+
+
+# ---------------------------------------------------------------- routing
+
+def _expected_topk(s_row, k):
+    """Brute force: sort (score desc, id asc), keep the first k finite."""
+    order = sorted(range(len(s_row)), key=lambda e: (-s_row[e], e))
+    order = [e for e in order if s_row[e] != -math.inf]
+    return order[:k], order
+
+
+@pytest.mark.parametrize("renorm", [True, False])
+def test_route_one_hot_rows_closed_form(renorm):
+    """With h = one-hot(c), z_e = W_router[e, c] exactly; the oracle's top-k
+    equals a brute-force sort of the eligible pool and its weights equal the
+    softmax computed with math.exp."""
+    s = LayerShape(T=96, H=64, I=16, E_pub=12, E_priv=6, E_sh=0, k=3, renormalize=renorm)
+    w, _, pol = make_layer(s, seed=3)
+    g = torch.Generator().manual_seed(5)
+    cols = torch.randint(0, s.H, (s.T,), generator=g)
+    h = torch.zeros(s.T, s.H)
+    h[torch.arange(s.T), cols] = 1.0
+    h = h.to(torch.bfloat16)
+    L = oracle_layer(s, w, h, pol)
+    idx, wt, gap = oracle.route(L)
+    R = torch.cat([w["router_pub"], w["router_priv"]]).float().numpy()
+    for t in range(s.T):
+        allow = int(pol[t]) == 1
+        srow = [float(R[e, cols[t]]) if ((e >= s.E_pub) == allow) else -math.inf for e in range(s.E)]
+        top, order = _expected_topk(srow, s.k)
+        assert list(idx[t]) == top
+        m = srow[top[0]]
+        ex = {e: math.exp(srow[e] - m) for e in order}
+        denom = sum(ex[e] for e in (top if renorm else order))
+        np.testing.assert_allclose(wt[t], [ex[e] / denom for e in top], rtol=1e-12)
+        nxt = order[s.k] if len(order) > s.k else None
+        assert gap[t] == (math.inf if nxt is None else srow[top[-1]] - srow[nxt])
+
+
+def test_route_random_rows_brute_force_sort():
+    """Random h: logits from numpy's float64 matmul rounded to fp32, masked,
+    then a full sort -- equals the oracle's selection."""
+    s = LayerShape(T=200, H=128, I=16, E_pub=20, E_priv=8, E_sh=0, k=4, renormalize=True)
+    w, h, pol = make_layer(s, seed=11)
+    L = oracle_layer(s, w, h, pol)
+    idx, _, _ = oracle.route(L)
+    R = torch.cat([w["router_pub"], w["router_priv"]]).double().numpy()
+    Z = (h.double().numpy() @ R.T).astype(np.float32).astype(np.float64)
+    for t in range(s.T):
+        allow = int(pol[t]) == 1
+        srow = [Z[t, e] if ((e >= s.E_pub) == allow) else -math.inf for e in range(s.E)]
+        assert list(idx[t]) == _expected_topk(srow, s.k)[0]
+
+
+@pytest.mark.parametrize("renorm", [True, False])
+def test_route_equal_logits_tie_break_and_uniform_weights(renorm):
+    """h = 0 makes every logit 0: the top-k are the k lowest ids of the pool
+    and the weights are 1/k (renormalised) or 1/|pool| (pool softmax)."""
+    s = LayerShape(T=4, H=32, I=8, E_pub=10, E_priv=5, E_sh=0, k=3, renormalize=renorm)
+    w, _, _ = make_layer(s, seed=2)
+    h = torch.zeros(s.T, s.H, dtype=torch.bfloat16)
+    pol = torch.tensor([0, 1, 7, 1], dtype=torch.uint8)
+    idx, wt, gap = oracle.route(oracle_layer(s, w, h, pol))
+    assert idx.tolist() == [[0, 1, 2], [10, 11, 12], [0, 1, 2], [10, 11, 12]]
+    for t in range(4):
+        pool = s.E_priv if pol[t] == 1 else s.E_pub
+        np.testing.assert_allclose(wt[t], [1 / s.k if renorm else 1 / pool] * s.k, rtol=1e-15)
+    assert np.all(gap == 0.0)
+
+
+def test_route_k_equals_pool_selects_whole_pool():
+    s = LayerShape(T=16, H=32, I=8, E_pub=4, E_priv=4, E_sh=0, k=4, renormalize=False)
+    w, h, pol = make_layer(s, seed=4)
+    idx, wt, gap = oracle.route(oracle_layer(s, w, h, pol))
+    for t in range(s.T):
+        pool = set(range(4, 8)) if pol[t] == 1 else set(range(4))
+        assert set(idx[t].tolist()) == pool
+    np.testing.assert_allclose(wt.sum(1), 1.0, rtol=1e-12)   # pool softmax over the whole pool
+    assert np.all(np.isinf(gap))
+
+
+def test_route_k1_argmax_weight_one():
+    s = LayerShape(T=50, H=64, I=8, E_pub=8, E_priv=3, E_sh=0, k=1, renormalize=True)
+    w, h, pol = make_layer(s, seed=6)
+    idx, wt, _ = oracle.route(oracle_layer(s, w, h, pol))
+    assert np.all(wt == 1.0)
+
+
+def test_weights_sum_rules():
+    """Renormalised weights sum to 1; pool-softmax weights are each <= 1 and
+    sum to at most 1."""
+    for renorm in (True, False):
+        s = LayerShape(T=64, H=64, I=8, E_pub=16, E_priv=8, E_sh=0, k=5, renormalize=renorm)
+        w, h, pol = make_layer(s, seed=8)
+        _, wt, _ = oracle.route(oracle_layer(s, w, h, pol))
+        if renorm:
+            np.testing.assert_allclose(wt.sum(1), 1.0, rtol=1e-12)
+        else:
+            assert np.all(wt <= 1.0) and np.all(wt.sum(1) <= 1.0 + 1e-12) and np.all(wt > 0)
+        assert np.all(np.diff(wt, axis=1) <= 1e-15)               # descending score order
+
+
+def test_mask_holds_against_adversarial_hidden_states():
+    """Prompt content cannot change the pool (Sec. 3.1; App. F.1 Table 7):
+    hidden states built to maximise the *other* pool's logits still route
+    inside the pool the policy selects."""
+    s = LayerShape(T=8, H=64, I=8, E_pub=6, E_priv=4, E_sh=0, k=2, renormalize=True)
+    w, _, _ = make_layer(s, seed=9)
+    priv_dir = w["router_priv"].float().sum(0)
+    pub_dir = w["router_pub"].float().sum(0)
+    h = torch.stack([priv_dir * 50 * (i + 1) for i in range(4)] + [pub_dir * 50 * (i + 1) for i in range(4)])
+    pol = torch.tensor([0, 0x7F, 0xFF, 2, 1, 1, 1, 1], dtype=torch.uint8)
+    idx, _, _ = oracle.route(oracle_layer(s, w, h.to(torch.bfloat16), pol))
+    assert np.all(idx[:4] < s.E_pub)
+    assert np.all(idx[4:] >= s.E_pub)
+
+
+# ---------------------------------------------------------------- experts
+
+def _torch_mlp(h, g, u, d):
+    """Textbook SwiGLU MLP in fp64 with the activation rounded to BF16."""
+    a = (F.silu(F.linear(h, g)) * F.linear(h, u)).float().to(torch.bfloat16).double()
+    return F.linear(a, d)
+
+
+def test_expert_matches_textbook_swiglu():
+    s = LayerShape(T=6, H=96, I=40, E_pub=3, E_priv=2, E_sh=2, k=1, renormalize=True)
+    w, h, pol = make_layer(s, seed=10)
+    L = oracle_layer(s, w, h, pol)
+    for e in range(s.E):
+        pool, j = ("pub", e) if e < s.E_pub else ("priv", e - s.E_pub)
+        for t in range(s.T):
+            y = oracle.expert(L, e, h[t])
+            ref = _torch_mlp(h[t].double(), w[f"gate_{pool}"][j].double(), w[f"up_{pool}"][j].double(),
+                             w[f"down_{pool}"][j].double()).numpy()
+            np.testing.assert_allclose(y, ref, rtol=0, atol=1e-5 * np.abs(ref).max())
+    for sidx in range(s.E_sh):
+        y = oracle.expert(L, sidx, h[0], shared=True)
+        ref = _torch_mlp(h[0].double(), w["gate_sh"][sidx].double(), w["up_sh"][sidx].double(),
+                         w["down_sh"][sidx].double()).numpy()
+        np.testing.assert_allclose(y, ref, rtol=0, atol=1e-5 * np.abs(ref).max())
+
+
+def test_forward_single_expert_pools_reduce_to_dense_mlp():
+    """E_pub = E_priv = k = 1 (renormalised): the layer is the dense SwiGLU
+    MLP of the public expert under DENY and of the private one under ALLOW."""
+    s = LayerShape(T=24, H=64, I=48, E_pub=1, E_priv=1, E_sh=0, k=1, renormalize=True)
+    w, h, pol = make_layer(s, seed=12)
+    r = oracle.forward(oracle_layer(s, w, h, pol))
+    for t in range(s.T):
+        pool = "priv" if pol[t] == 1 else "pub"
+        ref = _torch_mlp(h[t].double(), w[f"gate_{pool}"][0].double(), w[f"up_{pool}"][0].double(),
+                         w[f"down_{pool}"][0].double())
+        np.testing.assert_allclose(r["out_f64"][t], ref.numpy(), rtol=0, atol=1e-5 * ref.abs().max().item())
+        assert np.array_equal(r["out"][t], ref.float().to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16))
+
+
+def test_forward_identical_experts_give_the_mlp():
+    """If every routed expert has the same weights, the renormalised weights
+    sum to 1 and the layer output is that one MLP, whatever the routing."""
+    s = LayerShape(T=20, H=64, I=32, E_pub=6, E_priv=4, E_sh=0, k=3, renormalize=True)
+    w, h, pol = make_layer(s, seed=13)
+    for name in ("gate", "up", "down"):
+        base = w[f"{name}_pub"][0]
+        w[f"{name}_pub"] = base.expand(s.E_pub, *base.shape).contiguous()
+        w[f"{name}_priv"] = base.expand(s.E_priv, *base.shape).contiguous()
+    r = oracle.forward(oracle_layer(s, w, h, pol))
+    ref = _torch_mlp(h.double(), w["gate_pub"][0].double(), w["up_pub"][0].double(), w["down_pub"][0].double())
+    np.testing.assert_allclose(r["out_f64"], ref.numpy(), rtol=0, atol=1e-9 * ref.abs().max().item())
+
+
+def test_forward_is_weighted_sum_of_routed_plus_shared_experts():
+    """out = bf16(sum_j w_j MLP_{idx_j}(h) + sum_s MLP_s(h)) with the MLPs
+    from torch.nn.functional; pins the combine order-free up to fp64."""
+    s = LayerShape(T=12, H=64, I=32, E_pub=8, E_priv=4, E_sh=2, k=3, renormalize=False)
+    w, h, pol = make_layer(s, seed=14)
+    r = oracle.forward(oracle_layer(s, w, h, pol))
+    for t in range(s.T):
+        acc = torch.zeros(s.H, dtype=torch.float64)
+        for j in range(s.k):
+            e = int(r["idx"][t, j])
+            pool, i = ("pub", e) if e < s.E_pub else ("priv", e - s.E_pub)
+            acc += r["w"][t, j] * _torch_mlp(h[t].double(), w[f"gate_{pool}"][i].double(),
+                                             w[f"up_{pool}"][i].double(), w[f"down_{pool}"][i].double())
+        for sidx in range(s.E_sh):
+            acc += _torch_mlp(h[t].double(), w["gate_sh"][sidx].double(), w["up_sh"][sidx].double(),
+                              w["down_sh"][sidx].double())
+        np.testing.assert_allclose(r["out_f64"][t], acc.numpy(), rtol=0, atol=1e-9 * acc.abs().max().item())
+
+
+# ------------------------------------------------------------------ audit
+
+@pytest.mark.parametrize("policy", ["iid", "allow", "deny", "none"])
+def test_audit_invariants(policy):
+    """G1 (Sec. 2.2 Eq. 1) and the hook audit (Sec. 5.2, App. F.1): no
+    private row executes for a token whose policy is not ALLOW; execution
+    counts observed at the experts equal the route log; closed-form totals."""
+    s = LayerShape(T=40, H=64, I=16, E_pub=10, E_priv=5, E_sh=1, k=2, renormalize=True)
+    w, h, pol = make_layer(s, seed=15, policy=policy)
+    r = oracle.forward(oracle_layer(s, w, h, pol))
+    tau = oracle.resolve(None if pol is None else pol.numpy(), s.T)
+    assert r["route_count"].sum() == s.T * s.k
+    assert r["route_count"][s.E_pub:].sum() == s.k * tau.sum()
+    assert r["route_count"][:s.E_pub].sum() == s.k * (s.T - tau.sum())
+    assert np.array_equal(r["exec_rows"], r["route_count"])
+    assert np.array_equal(r["route_priv_rows"], s.k * tau.astype(np.uint32))
+    assert np.array_equal(r["exec_priv_rows"], r["route_priv_rows"])
+    assert np.all(r["exec_priv_rows"][tau == 0] == 0)
+    assert r["shared_rows"][0] == s.T * s.E_sh
+
+
+# ---------------------------------------------------------------- permute
+
+def test_permute_matches_brute_force_sort():
+    g = torch.Generator().manual_seed(21)
+    T, k, E = 57, 3, 11
+    idx = np.stack([torch.randperm(E, generator=g)[:k].numpy() for _ in range(T)]).astype(np.int32)
+    idx[5] = [0, 1, 2]                            # make sure some experts are hot
+    counts, offsets, slot_of, tok_of_slot = oracle.permute(idx, E)
+    rows = sorted(((int(idx[t, j]), t, j) for t in range(T) for j in range(k)))
+    for slot, (e, t, j) in enumerate(rows):
+        assert slot_of[t, j] == slot and tok_of_slot[slot] == t
+    assert np.array_equal(counts, np.bincount(idx.reshape(-1), minlength=E))
+    assert offsets[0] == 0 and np.array_equal(np.diff(offsets.astype(np.int64)), counts)
+
+
+def test_permute_rejects_out_of_range_ids():
+    with pytest.raises(ValueError):
+        oracle.permute(np.array([[0, 5]], np.int32), 5)
+
+
+# ----------------------------------------------------------------- golden
+
+def _golden_layer(c):
+    s = LayerShape(**c["shape"])
+    bf = lambda v: torch.tensor(v, dtype=torch.float32).to(torch.bfloat16)
+    t = {n: bf(c[n]) for n in ("hidden", "router_pub", "router_priv", "gate_pub", "up_pub", "down_pub",
+                               "gate_priv", "up_priv", "down_priv")}
+    for n in t:
+        assert torch.equal(t[n].float(), torch.tensor(c[n], dtype=torch.float32)), "fixture not BF16-exact"
+    return s, oracle.Layer(s, t, np.array(c["policy"], np.uint8))
+
+
+@pytest.mark.parametrize("case", json.load(open(GOLDEN))["cases"], ids=lambda c: c["name"])
+def test_golden_hand_worked(case):
+    s, L = _golden_layer(case)
+    r = oracle.forward(L)
+    assert r["idx"].tolist() == case["expected_idx"]
+    np.testing.assert_allclose(r["w"], case["expected_w"], rtol=1e-15)
+    assert bits_to_f64(r["out"]).tolist() == case["expected_out"]
