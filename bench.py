@@ -1,0 +1,363 @@
+"""Benchmark of the policy-masked MoE layer forward on GB300.
+
+python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+A step is one full layer forward (resolve, masked router + top-k, dispatch,
+grouped gate/up GEMM + SwiGLU, grouped down GEMM, combine) over one batch of
+the named workload (default: the Qwen3-30B-A3B-shaped prefill layer, 4096
+tokens, mixed ALLOW/DENY requests).  Prints one JSON line on rank 0.
+
+Multi-GPU: independent replicas (the layer is token-parallel with no
+exchange step); each rank runs the same workload on its own GPU, and value =
+tokens processed by all ranks / max over ranks of the timed duration.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_06690_gb300 import inputs as inp  # noqa: E402
+from paper_2608_06690_gb300.configs import CONFIGS  # noqa: E402
+
+METRIC = "MoE-layer tokens/s (mixed allow/deny)"
+L2_FLUSH_BYTES = 512 << 20   # > 129 MB L2
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p.get("bf16_tflops_sustained", p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def build_workload(cfg, device, seed_offset=0):
+    s = cfg.shape
+    w = inp.make_weights(s, cfg.seed + seed_offset, device=device, skew=cfg.skew)
+    h = inp.make_hidden(s, cfg.seed + seed_offset, device=device, skew=cfg.skew)
+    pol = cfg.policy(s.T).to(device)
+    return w, h, pol
+
+
+def algorithmic_work(s, counts: np.ndarray):
+    """FLOPs of the two grouped GEMMs and the byte counts of the HBM-bound
+    stages, for one forward with the given per-expert row counts."""
+    R = s.T * s.k
+    f_gateup = 2.0 * R * s.H * 2 * s.I + 2.0 * s.T * s.H * 2 * s.E_sh * s.I
+    f_down = 2.0 * R * s.I * s.H + 2.0 * s.T * s.E_sh * s.I * s.H
+    touched = int((counts > 0).sum())
+    expert_w = 3 * s.I * s.H * 2
+    gemm_weight_bytes = touched * expert_w + s.E_sh * expert_w
+    b_gateup = touched * 2 * s.I * s.H * 2 + s.E_sh * 2 * s.I * s.H * 2 + R * s.H * 2 + R * s.I * 2 \
+        + (s.T * s.H * 2 + s.T * s.E_sh * s.I * 2 if s.E_sh else 0)
+    b_down = touched * s.I * s.H * 2 + s.E_sh * s.I * s.H * 2 + R * s.I * 2 + R * s.H * 2 \
+        + (s.T * s.E_sh * s.I * 2 + s.T * s.H * 2 if s.E_sh else 0)
+    b_route = s.T * s.H * 2 + (s.E_pub + s.E_priv) * s.H * 2 + s.T * s.k * 8 + s.T
+    b_permute = R * s.H * 2 * 2 + R * 16
+    b_combine = R * s.H * 2 + s.T * s.H * 2 + (s.T * s.H * 2 if s.E_sh else 0)
+    return dict(flops_gateup=f_gateup, flops_down=f_down, bytes_gateup=b_gateup, bytes_down=b_down,
+                bytes_route=b_route, bytes_permute=b_permute, bytes_combine=b_combine,
+                touched_experts=touched, gemm_weight_bytes=gemm_weight_bytes)
+
+
+def cpu_baseline(cfg, w, h, pol, budget_s=12.0, max_tokens=4096):
+    """The CPU oracle, as it stands, on a bounded sample of the workload's
+    tokens (the first n tokens of each request, spread evenly)."""
+    import oracle
+    s = cfg.shape
+    wc = {k: (None if v is None else v.cpu()) for k, v in w.items()}
+    L = oracle.Layer(s, dict(wc, hidden=h.cpu()), pol.cpu().numpy())
+    cores = len(os.sched_getaffinity(0))
+    per_req = s.T // cfg.n_requests
+
+    def sample(n):
+        take = max(1, n // cfg.n_requests)
+        toks = [r * per_req + i for r in range(cfg.n_requests) for i in range(min(take, per_req))]
+        return np.array(toks[:max(n, 1)], dtype=np.int32)
+
+    n = min(32, s.T)
+    t0 = time.perf_counter()
+    oracle.forward(L, tokens=sample(n), nthreads=cores)
+    dt = time.perf_counter() - t0
+    n2 = int(min(max_tokens, s.T, max(n, n * budget_s / max(dt, 1e-3))))
+    toks = sample(n2)
+    t0 = time.perf_counter()
+    oracle.forward(L, tokens=toks, nthreads=cores)
+    dt = time.perf_counter() - t0
+    return {"value": len(toks) / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{len(toks)} of {s.T} tokens of {cfg.name} (spread over its {cfg.n_requests} requests), "
+                      f"full layer forward in fp64, OpenMP over tokens, {dt:.1f} s"}
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle, timed as it stands on the host cores,
+    each step a bounded sample of the workload."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    import oracle
+    cfg = CONFIGS[args.config]
+    s = cfg.shape
+    w, h, pol = build_workload(cfg, "cpu")
+    L = oracle.Layer(s, dict(w, hidden=h), pol.numpy())
+    cores = len(os.sched_getaffinity(0))
+    per_req = s.T // cfg.n_requests
+    n_tok = max(1, min(s.T, args.ref_tokens))
+    take = max(1, n_tok // cfg.n_requests)
+    toks = np.array([r * per_req + i for r in range(cfg.n_requests) for i in range(min(take, per_req))][:n_tok],
+                    dtype=np.int32)
+    for _ in range(args.warmup):
+        oracle.forward(L, tokens=toks[:max(1, len(toks) // 8)], nthreads=cores)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.forward(L, tokens=toks, nthreads=cores)
+    dt = time.perf_counter() - t0
+    value = len(toks) * args.steps / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": cfg.name, "tokens_per_step": len(toks), "layer_tokens": s.T},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{len(toks)} of {s.T} tokens of {cfg.name} per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    from paper_2608_06690_gb300 import pmpe
+    ws, rank, local = _dist()
+    if ws > 1:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg = CONFIGS[args.config]
+    s = cfg.shape
+    w, h, pol = build_workload(cfg, dev)
+    layer = pmpe.MoeLayer(s, w, device=dev)
+    out = torch.empty_like(h)
+    audit = torch.zeros(pmpe.audit_words(s.T, s.E), dtype=torch.int32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+
+    def step():
+        layer.forward(h, pol, out=out)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize(dev)
+
+    # ---- timed region: K steps, L2 flushed before each, CUDA events per step
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clk:
+        t_wall0 = time.perf_counter()
+        for e0, e1 in evs:
+            flush.zero_()
+            e0.record(stream)
+            step()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        t_wall = time.perf_counter() - t_wall0
+        barrier()
+    step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
+    total_ms = torch.tensor([sum(step_ms)], dtype=torch.float64, device=dev)
+    if ws > 1:
+        torch.distributed.all_reduce(total_ms, op=torch.distributed.ReduceOp.MAX)
+    total_ms = float(total_ms.item())
+    value = ws * s.T * args.steps / (total_ms / 1e3)
+
+    # ---- per-stage breakdown (same launches, events between the stages)
+    stages = [("route", pmpe.STAGE_ROUTE), ("permute", pmpe.STAGE_PERMUTE), ("gateup", pmpe.STAGE_GATEUP),
+              ("down", pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE)]
+    stage_ms = {n: [] for n, _ in stages}
+    for _ in range(args.steps):
+        flush.zero_()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)]
+        ev[0].record(stream)
+        for i, (n, bit) in enumerate(stages):
+            layer.forward(h, pol, out=out, stages=bit)
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize(dev)
+        for i, (n, _) in enumerate(stages):
+            stage_ms[n].append(ev[i].elapsed_time(ev[i + 1]))
+    stage_avg = {n: float(np.mean(v)) for n, v in stage_ms.items()}
+
+    # ---- audit of one forward (exactness of the counters is a test; here: sanity + expert loads)
+    pmpe.audit_reset(audit, s.T, s.E)
+    layer.forward(h, pol, out=out, audit=audit)
+    a = pmpe.audit_read(audit, s.T, s.E)
+    counts = a["route_count"]
+    work = algorithmic_work(s, counts)
+
+    # ---- end to end through the public API with host buffers
+    h_host = h.cpu().pin_memory()
+    pol_host = pol.cpu().pin_memory()
+    out_host = torch.empty(h.shape, dtype=h.dtype).pin_memory()
+    h_dev = torch.empty_like(h)
+    pol_dev = torch.empty_like(pol)
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(max(args.warmup, 3) + args.steps):
+        if i >= max(args.warmup, 3):
+            flush.zero_()
+            e2e_ev[i - max(args.warmup, 3)][0].record(stream)
+        h_dev.copy_(h_host, non_blocking=True)
+        pol_dev.copy_(pol_host, non_blocking=True)
+        layer.forward(h_dev, pol_dev, out=out)
+        out_host.copy_(out, non_blocking=True)
+        if i >= max(args.warmup, 3):
+            e2e_ev[i - max(args.warmup, 3)][1].record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = sum(e0.elapsed_time(e1) for e0, e1 in e2e_ev)
+    e2e_t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+    if ws > 1:
+        torch.distributed.all_reduce(e2e_t, op=torch.distributed.ReduceOp.MAX)
+    e2e_value = ws * s.T * args.steps / (float(e2e_t.item()) / 1e3)
+
+    if rank != 0:
+        if ws > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    hbm, tf_burst, tf_sus, peak_src = _peaks()
+    dominant = max(stage_avg, key=stage_avg.get)
+    if dominant in ("gateup", "down"):
+        achieved = work[f"flops_{dominant}"] / (stage_avg[dominant] / 1e3) / 1e12
+        roof = {"kernel": dominant, "bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
+                "frac": achieved / tf_burst, "peak_source": f"{peak_src} bf16 burst",
+                "hbm_gbs": work[f"bytes_{dominant}"] / (stage_avg[dominant] / 1e3) / 1e9,
+                "hbm_frac": work[f"bytes_{dominant}"] / (stage_avg[dominant] / 1e3) / 1e9 / hbm}
+    else:
+        achieved = work[f"bytes_{dominant}"] / (stage_avg[dominant] / 1e3) / 1e9
+        roof = {"kernel": dominant, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "peak_source": f"{peak_src} HBM copy"}
+    roof["traffic"] = args.traffic
+    stage_report = {}
+    for n, ms in stage_avg.items():
+        d = {"ms": ms}
+        if n in ("gateup", "down"):
+            d["tflops"] = work[f"flops_{n}"] / (ms / 1e3) / 1e12
+        d["gbs"] = work[f"bytes_{n}"] / (ms / 1e3) / 1e9
+        stage_report[n] = d
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name, "T": s.T, "H": s.H, "I": s.I, "E_pub": s.E_pub, "E_priv": s.E_priv,
+                   "E_shared": s.E_sh, "k": s.k, "renormalize": s.renormalize, "requests": cfg.n_requests,
+                   "allow_tokens": int((pol == 1).sum().item()), "l2": "flushed (512 MB write) before every step",
+                   "parallelism": f"replicas x{ws}"},
+        "roofline": roof,
+        "stages": stage_report,
+        "expert_load": {"touched": work["touched_experts"], "max_rows": int(counts.max()),
+                        "mean_rows_public": float(counts[:s.E_pub].mean()),
+                        "mean_rows_private": float(counts[s.E_pub:].mean())},
+        "gpu_launches": pmpe.KERNELS_PER_FORWARD * args.steps,
+        "clocks": clk.summary(),
+        "wall_s_timed_region": t_wall,
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h.numel() * 2 + pol.numel(),
+                "d2h_bytes_per_step": out.numel() * 2},
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(cfg, w, h, pol, budget_s=args.cpu_budget)
+    print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="qwen3_prefill", choices=sorted(CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--ref-tokens", type=int, default=96)
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="DRAM bytes per launch of the dominant kernel from an ncu capture of this build")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

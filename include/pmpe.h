@@ -1,0 +1,185 @@
+/*
+ * pmpe.h -- C ABI of libpmpe: the GB300 (sm_103a) forward pass of one
+ * policy-masked sparse-MoE layer, the method of "Policy-Masked Private
+ * Experts" (arXiv 2608.06690).
+ *
+ * The layer (Sec. 3.1 and App. B.1 of the paper):
+ *   1. a trusted per-token policy byte is resolved fail-closed: only 0x01 is
+ *      ALLOW (tau = 1), every other byte and a missing (NULL) policy is DENY
+ *      (Sec. 2.1, App. B.1 "Policy resolution and masked routing");
+ *   2. tau selects one of two mutually exclusive expert pools -- the private
+ *      pool for ALLOW, the original public pool for DENY -- and the router
+ *      logits are computed over that pool only, so an ineligible expert never
+ *      enters the candidate set (Sec. 3.1, Eq. 4 and the sentence after it);
+ *   3. top-k inside the pool with softmax weights (renormalised over the top-k,
+ *      or the pool softmax without renormalisation);
+ *   4. token rows are grouped by expert, each expert runs its SwiGLU MLP
+ *      (gate/up projection, silu(gate) * up, down projection; private experts
+ *      copy the public expert architecture, Sec. 3.1), and the outputs are
+ *      combined with the routing weights, plus always-on shared experts;
+ *   5. the expert kernels themselves count the rows they execute, an audit
+ *      trail independent of the route log (Sec. 5.2 and App. F.1: the
+ *      independent hooks that counted physical private rows).
+ *
+ * Global expert ids: public 0 .. E_pub-1, private E_pub .. E_pub+E_priv-1
+ * (the concatenated public/private pool of Sec. 4.2).
+ *
+ * Conventions for every entry point:
+ *   - All tensor pointers are DEVICE pointers unless stated otherwise; the
+ *     caller allocates and owns every buffer.  The library keeps no mutable
+ *     global state between calls and never allocates device memory.
+ *   - BF16 tensors are passed as raw 16-bit words (void *), row-major, with
+ *     the [out, in] layout of a linear layer.  Every pointer must be 16-byte
+ *     aligned.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Calls
+ *     are asynchronous on it unless stated otherwise.
+ *   - Return value: PMPE_OK or a negative PMPE_ERR_* code.  When a call
+ *     returns an error before launching, nothing has been enqueued and no
+ *     output has been touched.
+ *   - A malformed policy byte is never an error: it resolves to DENY.
+ */
+#ifndef PMPE_H
+#define PMPE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define PMPE_API __attribute__((visibility("default")))
+#else
+#define PMPE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ----------------------------------------------------------- status codes */
+#define PMPE_OK 0
+#define PMPE_ERR_INVALID_ARG (-1)       /* NULL required pointer, k < 1, k > a pool size, T < 0, ... */
+#define PMPE_ERR_UNSUPPORTED_SHAPE (-2) /* H or I not a multiple of 128, a pool above 256, k above 32,
+                                           or a pointer not 16-byte aligned */
+#define PMPE_ERR_WORKSPACE (-3)         /* workspace NULL or smaller than pmpe_moe_workspace_size() */
+#define PMPE_ERR_CUDA (-4)              /* a CUDA runtime call failed */
+#define PMPE_ERR_TIMEOUT (-5)           /* a bounded host wait ran out */
+#define PMPE_ERR_DEVICE_STATUS (-6)     /* a kernel recorded an error in the audit status word */
+
+/* Bits a kernel may OR into the device status word (audit word 0). */
+#define PMPE_STATUS_DISPATCH_MISMATCH 0x1u /* dispatch count differs from the router's count */
+#define PMPE_STATUS_PIPELINE_TIMEOUT 0x2u  /* a bounded wait inside an expert kernel gave up */
+#define PMPE_STATUS_BAD_EXPERT_ID 0x4u     /* a routed id outside [0, E) reached the dispatcher */
+
+/* Stage bits for pmpe_moe_forward_stages(). */
+#define PMPE_STAGE_ROUTE 0x01u   /* resolve + masked router + top-k + route log */
+#define PMPE_STAGE_PERMUTE 0x02u /* per-expert dispatch order + row gather */
+#define PMPE_STAGE_GATEUP 0x04u  /* grouped gate/up GEMM with fused silu(g)*u, execution audit */
+#define PMPE_STAGE_DOWN 0x08u    /* grouped down GEMM, scaled by the routing weight */
+#define PMPE_STAGE_COMBINE 0x10u /* weighted unpermute-combine (+ shared experts) */
+#define PMPE_STAGE_ALL 0x1Fu
+
+/* ------------------------------------------------------------ layer desc */
+typedef struct pmpe_moe_desc {
+    int T;            /* tokens, >= 0 (0 is a no-op) */
+    int H;            /* hidden size, multiple of 128 */
+    int I;            /* expert intermediate size, multiple of 128 */
+    int E_pub;        /* public routed experts, k <= E_pub <= 256 */
+    int E_priv;       /* private routed experts, k <= E_priv <= 256 */
+    int E_shared;     /* always-on shared experts (0 = none), weight 1, run for every token */
+    int k;            /* experts per token inside the selected pool, 1 <= k <= 32 */
+    int renormalize;  /* 1: w = softmax over the k selected logits; 0: w = pool-softmax probabilities */
+
+    const void *hidden;          /* [T, H] BF16 */
+    const uint8_t *policy;       /* [T] trusted policy bytes; NULL = metadata missing = all DENY */
+
+    const void *w_router_pub;    /* [E_pub, H] BF16 */
+    const void *w_router_priv;   /* [E_priv, H] BF16 */
+    const void *w_gate_pub;      /* [E_pub, I, H] BF16 */
+    const void *w_up_pub;        /* [E_pub, I, H] BF16 */
+    const void *w_down_pub;      /* [E_pub, H, I] BF16 */
+    const void *w_gate_priv;     /* [E_priv, I, H] BF16 */
+    const void *w_up_priv;       /* [E_priv, I, H] BF16 */
+    const void *w_down_priv;     /* [E_priv, H, I] BF16 */
+    const void *w_gate_sh;       /* [E_shared, I, H] BF16, or NULL when E_shared == 0 */
+    const void *w_up_sh;         /* [E_shared, I, H] BF16 */
+    const void *w_down_sh;       /* [E_shared, H, I] BF16 */
+
+    void *out;                   /* [T, H] BF16 output */
+    int32_t *topk_idx;           /* optional [T, k] route log: global expert ids, descending score */
+    float *topk_w;               /* optional [T, k] routing weights */
+    uint32_t *audit;             /* optional pmpe_audit_words(T, E_pub+E_priv) counters; accumulate
+                                    across calls until pmpe_audit_reset() */
+    void *workspace;             /* device scratch, >= pmpe_moe_workspace_size() bytes, 256-byte aligned */
+    size_t workspace_bytes;
+} pmpe_moe_desc;
+
+/* Bytes of device workspace pmpe_moe_forward() needs for this shape.
+ * Returns 0 for an invalid shape. */
+PMPE_API size_t pmpe_moe_workspace_size(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k);
+
+/* Byte offsets of the named regions inside the workspace (for tests that
+ * inspect intermediate results, and for the stage-by-stage entry point).
+ * Returns PMPE_ERR_INVALID_ARG for an invalid shape. */
+typedef struct pmpe_workspace_layout {
+    size_t total;
+    size_t tau;          /* uint8  [T]      resolved policy bits */
+    size_t counts;       /* uint32 [E]      rows routed to each expert (router's count) */
+    size_t offsets;      /* uint32 [E+1]    exclusive prefix sum of counts */
+    size_t topk_idx;     /* int32  [T, k]   used when desc.topk_idx is NULL */
+    size_t topk_w;       /* float  [T, k]   used when desc.topk_w is NULL */
+    size_t slot_of;      /* int32  [T, k]   dispatch row of (t, j) */
+    size_t tok_of_slot;  /* int32  [T*k]    token of each dispatch row */
+    size_t w_of_slot;    /* float  [T*k]    routing weight of each dispatch row */
+    size_t a_perm;       /* BF16   [T*k, H] token rows in dispatch order */
+    size_t act;          /* BF16   [T*k, I] silu(g)*u of each dispatch row */
+    size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row */
+    size_t act_sh;       /* BF16   [T, E_shared*I] shared-expert activations (0 if none) */
+    size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs (0 if none) */
+} pmpe_workspace_layout;
+PMPE_API int pmpe_moe_workspace_layout(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k,
+                              pmpe_workspace_layout *out);
+
+/* Number of uint32 words of the audit buffer for T tokens and E routed
+ * experts.  Layout (word offsets):
+ *   [0]                  status   OR of PMPE_STATUS_* bits
+ *   [1]                  shared_rows      (token, shared expert) pairs executed
+ *   [2, 2+E)             route_count[e]   rows the router sent to expert e
+ *   [2+E, 2+2E)          exec_rows[e]     rows the expert kernels executed for e
+ *   [2+2E, 2+3E)         exec_tiles[e]    row tiles the expert kernels ran for e
+ *   [2+3E, 2+3E+T)       route_priv_rows[t]  private experts in token t's route
+ *   [2+3E+T, 2+3E+2T)    exec_priv_rows[t]   private expert rows executed for token t
+ * The route words come from the router; the exec words are written from inside
+ * the grouped expert GEMM tiles, from the rows each tile processed. */
+PMPE_API size_t pmpe_audit_words(int T, int E);
+
+/* Resolve T trusted policy bytes to tau (0/1 bytes): tau[t] = (policy[t] == 0x01).
+ * policy == NULL means missing metadata: every tau is 0.  tau: [T] device.
+ * App. B.1, step 2 of the fail-closed procedure. */
+PMPE_API int pmpe_policy_resolve(const uint8_t *policy, int T, uint8_t *tau, void *stream);
+
+/* The whole layer forward (all stages) on `stream`.  No host synchronisation;
+ * expert row counts stay on the device. */
+PMPE_API int pmpe_moe_forward(const pmpe_moe_desc *d, void *stream);
+
+/* Run a subset of the stages (PMPE_STAGE_* bits), in pipeline order.  Each
+ * stage reads what the previous stages left in the same workspace, so a
+ * stage may only be run after its predecessors have run on that workspace
+ * with the same inputs.  pmpe_moe_forward() == stages PMPE_STAGE_ALL. */
+PMPE_API int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *stream);
+
+/* Zero the audit buffer (pmpe_audit_words(T, E) words). */
+PMPE_API int pmpe_audit_reset(uint32_t *audit, int T, int E, void *stream);
+
+/* Copy the audit buffer to caller host memory `host_out` (same word count)
+ * and wait for the copy with a bounded poll.  Returns PMPE_ERR_TIMEOUT if it
+ * has not completed after timeout_ms milliseconds (the copy stays enqueued),
+ * PMPE_ERR_DEVICE_STATUS if the status word is nonzero, PMPE_OK otherwise. */
+PMPE_API int pmpe_audit_read(const uint32_t *audit, int T, int E, uint32_t *host_out, void *stream, int timeout_ms);
+
+/* Human-readable text of a status code (static storage). */
+PMPE_API const char *pmpe_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PMPE_H */

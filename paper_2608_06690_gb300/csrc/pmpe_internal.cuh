@@ -1,0 +1,111 @@
+// Internal declarations shared by the libpmpe translation units: the launch
+// context, the workspace carve-up and small device helpers.  Nothing here is
+// part of the C ABI (include/pmpe.h is).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/pmpe.h"
+
+namespace pmpe {
+
+typedef __nv_bfloat16 bf16;
+
+// Limits checked on the host before any launch.
+constexpr int kMaxPool = 256;   // experts per pool (router smem tiles)
+constexpr int kMaxTopK = 32;    // one warp lane per selected expert
+constexpr int kDimAlign = 128;  // H and I granularity
+
+struct Shape {
+    int T, H, I, E_pub, E_priv, E_sh, k, renorm;
+    int E() const { return E_pub + E_priv; }
+};
+
+// Pointers into the audit buffer (all NULL when the caller passed none).
+struct Audit {
+    uint32_t *status, *shared_rows, *route_count, *exec_rows, *exec_tiles, *route_priv_rows, *exec_priv_rows;
+};
+
+Audit audit_ptrs(uint32_t *base, int T, int E);
+
+// Everything one forward call needs, resolved from the descriptor.
+struct Ctx {
+    Shape s;
+    const bf16 *hidden;
+    const uint8_t *policy;
+    const bf16 *router_pub, *router_priv;
+    // [0] public, [1] private, [2] shared
+    const bf16 *gate[3], *up[3], *down[3];
+    bf16 *out;
+    int32_t *idx;
+    float *w;
+    Audit audit;
+    // workspace regions
+    uint8_t *tau;
+    uint32_t *counts, *offsets;
+    int32_t *slot_of, *tok_of_slot;
+    float *w_of_slot;
+    bf16 *a_perm, *act, *y, *act_sh, *y_sh;
+    cudaStream_t stream;
+    int num_sms;
+};
+
+int compute_layout(const Shape &s, pmpe_workspace_layout *L);
+
+// Launchers (one per stage); each returns the launch's cudaError_t.
+cudaError_t launch_route(const Ctx &c);
+cudaError_t launch_permute(const Ctx &c);
+cudaError_t launch_gateup(const Ctx &c);
+cudaError_t launch_down(const Ctx &c);
+cudaError_t launch_combine(const Ctx &c);
+cudaError_t launch_resolve(const uint8_t *policy, int T, uint8_t *tau, cudaStream_t stream);
+
+// ------------------------------------------------------------ device helpers
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// 16-byte async copy global -> shared; src_bytes = 0 zero-fills the 16 bytes.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3, uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+// D += A * B for one m16n8k16 BF16 tile, FP32 accumulate.
+__device__ __forceinline__ void mma_bf16_16816(float *d, const uint32_t *a, uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Byte offset of 16-byte chunk `c` of row `r` in a tile whose rows are 128
+// bytes (64 BF16): chunks are XOR-swizzled by the row's low 3 bits so that
+// ldmatrix reads of 8 consecutive rows hit 8 distinct bank groups.
+__device__ __forceinline__ uint32_t swz128(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&v);
+}
+
+__device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + __expf(-g)) * u; }
+
+}  // namespace pmpe

@@ -1,0 +1,220 @@
+"""ctypes binding over libpmpe.so (the C ABI of include/pmpe.h).
+
+Argument marshalling only: every step of the layer runs in the library's
+CUDA kernels.  PyTorch supplies device memory and streams.  If the library
+has not been built this module raises on import -- there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+import torch
+
+from .inputs import LayerShape
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libpmpe.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+OK = 0
+ERR_INVALID_ARG = -1
+ERR_UNSUPPORTED_SHAPE = -2
+ERR_WORKSPACE = -3
+ERR_CUDA = -4
+ERR_TIMEOUT = -5
+ERR_DEVICE_STATUS = -6
+
+STATUS_DISPATCH_MISMATCH = 0x1
+STATUS_PIPELINE_TIMEOUT = 0x2
+STATUS_BAD_EXPERT_ID = 0x4
+
+STAGE_ROUTE = 0x01
+STAGE_PERMUTE = 0x02
+STAGE_GATEUP = 0x04
+STAGE_DOWN = 0x08
+STAGE_COMBINE = 0x10
+STAGE_ALL = 0x1F
+
+# Kernels one full forward launches: router/top-k, dispatch order, row
+# gather, gate/up GEMM, down GEMM, combine (plus one memset of the per-expert
+# counters, which is not a kernel of this library).
+KERNELS_PER_FORWARD = 6
+
+EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
+            "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
+            "pmpe_status_string")
+
+_vp = ctypes.c_void_p
+
+
+class MoeDesc(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int), ("H", ctypes.c_int), ("I", ctypes.c_int), ("E_pub", ctypes.c_int),
+                ("E_priv", ctypes.c_int), ("E_shared", ctypes.c_int), ("k", ctypes.c_int),
+                ("renormalize", ctypes.c_int),
+                ("hidden", _vp), ("policy", _vp),
+                ("w_router_pub", _vp), ("w_router_priv", _vp),
+                ("w_gate_pub", _vp), ("w_up_pub", _vp), ("w_down_pub", _vp),
+                ("w_gate_priv", _vp), ("w_up_priv", _vp), ("w_down_priv", _vp),
+                ("w_gate_sh", _vp), ("w_up_sh", _vp), ("w_down_sh", _vp),
+                ("out", _vp), ("topk_idx", _vp), ("topk_w", _vp), ("audit", _vp),
+                ("workspace", _vp), ("workspace_bytes", ctypes.c_size_t)]
+
+
+class WorkspaceLayout(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_size_t) for n in ("total", "tau", "counts", "offsets", "topk_idx", "topk_w", "slot_of",
+                                                "tok_of_slot", "w_of_slot", "a_perm", "act", "y", "act_sh", "y_sh")]
+
+
+_lib.pmpe_moe_workspace_size.restype = ctypes.c_size_t
+_lib.pmpe_moe_workspace_size.argtypes = [ctypes.c_int] * 7
+_lib.pmpe_moe_workspace_layout.restype = ctypes.c_int
+_lib.pmpe_moe_workspace_layout.argtypes = [ctypes.c_int] * 7 + [ctypes.POINTER(WorkspaceLayout)]
+_lib.pmpe_audit_words.restype = ctypes.c_size_t
+_lib.pmpe_audit_words.argtypes = [ctypes.c_int, ctypes.c_int]
+_lib.pmpe_policy_resolve.restype = ctypes.c_int
+_lib.pmpe_policy_resolve.argtypes = [_vp, ctypes.c_int, _vp, _vp]
+_lib.pmpe_moe_forward.restype = ctypes.c_int
+_lib.pmpe_moe_forward.argtypes = [ctypes.POINTER(MoeDesc), _vp]
+_lib.pmpe_moe_forward_stages.restype = ctypes.c_int
+_lib.pmpe_moe_forward_stages.argtypes = [ctypes.POINTER(MoeDesc), ctypes.c_uint, _vp]
+_lib.pmpe_audit_reset.restype = ctypes.c_int
+_lib.pmpe_audit_reset.argtypes = [_vp, ctypes.c_int, ctypes.c_int, _vp]
+_lib.pmpe_audit_read.restype = ctypes.c_int
+_lib.pmpe_audit_read.argtypes = [_vp, ctypes.c_int, ctypes.c_int, _vp, _vp, ctypes.c_int]
+_lib.pmpe_status_string.restype = ctypes.c_char_p
+_lib.pmpe_status_string.argtypes = [ctypes.c_int]
+
+
+class PmpeError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__(f"{what}: {status_string(code)} ({code})")
+        self.code = code
+
+
+def status_string(code: int) -> str:
+    return _lib.pmpe_status_string(code).decode()
+
+
+def _check(code: int, what: str):
+    if code != OK:
+        raise PmpeError(code, what)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def workspace_size(s: LayerShape) -> int:
+    return int(_lib.pmpe_moe_workspace_size(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k))
+
+
+def workspace_layout(s: LayerShape) -> dict:
+    L = WorkspaceLayout()
+    _check(_lib.pmpe_moe_workspace_layout(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, ctypes.byref(L)),
+           "pmpe_moe_workspace_layout")
+    return {n: int(getattr(L, n)) for n, _ in WorkspaceLayout._fields_}
+
+
+def audit_words(T: int, E: int) -> int:
+    return int(_lib.pmpe_audit_words(T, E))
+
+
+def audit_fields(words: np.ndarray, T: int, E: int) -> dict:
+    """Split an audit buffer read back to the host into its named counters."""
+    a = np.asarray(words, dtype=np.uint32)
+    return dict(status=int(a[0]), shared_rows=int(a[1]), route_count=a[2:2 + E], exec_rows=a[2 + E:2 + 2 * E],
+                exec_tiles=a[2 + 2 * E:2 + 3 * E], route_priv_rows=a[2 + 3 * E:2 + 3 * E + T],
+                exec_priv_rows=a[2 + 3 * E + T:2 + 3 * E + 2 * T])
+
+
+def policy_resolve(policy, T: int, tau=None, stream=None):
+    """tau[t] = (policy[t] == 0x01) on the device; policy None = all DENY."""
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.uint8, device="cuda")
+    _check(_lib.pmpe_policy_resolve(_ptr(policy), T, _ptr(tau), _stream(stream)), "pmpe_policy_resolve")
+    return tau
+
+
+def audit_reset(audit, T: int, E: int, stream=None):
+    _check(_lib.pmpe_audit_reset(_ptr(audit), T, E, _stream(stream)), "pmpe_audit_reset")
+
+
+def audit_read(audit, T: int, E: int, stream=None, timeout_ms: int = 10000, check_status: bool = True) -> dict:
+    host = torch.empty(audit_words(T, E), dtype=torch.int32).pin_memory()
+    rc = _lib.pmpe_audit_read(_ptr(audit), T, E, ctypes.c_void_p(host.data_ptr()), _stream(stream), timeout_ms)
+    if rc == ERR_DEVICE_STATUS and not check_status:
+        rc = OK
+    _check(rc, "pmpe_audit_read")
+    return audit_fields(host.numpy().view(np.uint32).copy(), T, E)
+
+
+def make_desc(s: LayerShape, weights: dict, hidden, policy, out, workspace, topk_idx=None, topk_w=None,
+              audit=None) -> MoeDesc:
+    """Fill the C descriptor from torch tensors (device pointers only)."""
+    W = weights
+    return MoeDesc(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, int(bool(s.renormalize)),
+                   _ptr(hidden), _ptr(policy),
+                   _ptr(W["router_pub"]), _ptr(W["router_priv"]),
+                   _ptr(W["gate_pub"]), _ptr(W["up_pub"]), _ptr(W["down_pub"]),
+                   _ptr(W["gate_priv"]), _ptr(W["up_priv"]), _ptr(W["down_priv"]),
+                   _ptr(W.get("gate_sh")), _ptr(W.get("up_sh")), _ptr(W.get("down_sh")),
+                   _ptr(out), _ptr(topk_idx), _ptr(topk_w), _ptr(audit),
+                   _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size())
+
+
+def forward_desc(desc: MoeDesc, stages: int = STAGE_ALL, stream=None):
+    """Enqueue the layer (or a subset of its stages) for a prepared descriptor."""
+    if stages == STAGE_ALL:
+        rc = _lib.pmpe_moe_forward(ctypes.byref(desc), _stream(stream))
+    else:
+        rc = _lib.pmpe_moe_forward_stages(ctypes.byref(desc), stages, _stream(stream))
+    _check(rc, "pmpe_moe_forward")
+
+
+class MoeLayer:
+    """One policy-masked MoE layer with its weights resident on the GPU and
+    a reusable workspace.  ``forward`` enqueues the C-ABI call on the
+    current stream and returns the output tensor."""
+
+    def __init__(self, shape: LayerShape, weights: dict, device="cuda"):
+        self.shape = shape
+        self.weights = weights
+        self.device = torch.device(device)
+        self._ws = None
+        self._ws_T = -1
+
+    def workspace(self, T: int) -> torch.Tensor:
+        if self._ws is None or self._ws_T < T:
+            s = self._shape_T(T)
+            self._ws = torch.empty(max(workspace_size(s), 1), dtype=torch.uint8, device=self.device)
+            self._ws_T = T
+        return self._ws
+
+    def _shape_T(self, T: int) -> LayerShape:
+        s = self.shape
+        return LayerShape(T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, s.renormalize)
+
+    def forward(self, hidden, policy, out=None, topk_idx=None, topk_w=None, audit=None, stages=STAGE_ALL,
+                stream=None):
+        T = hidden.shape[0]
+        s = self._shape_T(T)
+        assert hidden.is_contiguous() and hidden.dtype == torch.bfloat16 and hidden.shape == (T, s.H)
+        if policy is not None:
+            assert policy.dtype == torch.uint8 and policy.numel() == T and policy.is_contiguous()
+        if out is None:
+            out = torch.empty_like(hidden)
+        desc = make_desc(s, self.weights, hidden, policy, out, self.workspace(T), topk_idx, topk_w, audit)
+        forward_desc(desc, stages, stream)
+        return out

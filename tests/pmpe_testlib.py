@@ -60,3 +60,104 @@ MEAN_REL = 5e-3
 # Router gap rule: a token whose k-th and (k+1)-th fp32 logits (oracle) are
 # closer than this may legitimately pick a different k-th expert.
 GAP_EPS = 1e-4
+
+
+# ------------------------------------------------------------ GPU helpers
+
+def to_device(w: dict, h, pol, device="cuda"):
+    wd = {k: (None if v is None else v.to(device).contiguous()) for k, v in w.items()}
+    return wd, h.to(device).contiguous(), (None if pol is None else pol.to(device).contiguous())
+
+
+def run_gpu_layer(shape: LayerShape, w: dict, h, pol, audit_reset=True, stages=None):
+    """Run the layer through the C ABI; return outputs, the route log, the
+    audit counters and the dispatch intermediates, all on the host."""
+    from paper_2608_06690_gb300 import pmpe
+    layer = pmpe.MoeLayer(shape, w)
+    T, k, E = shape.T, shape.k, shape.E
+    idx = torch.full((T, k), -1, dtype=torch.int32, device="cuda")
+    wt = torch.full((T, k), float("nan"), dtype=torch.float32, device="cuda")
+    audit = torch.zeros(pmpe.audit_words(T, E), dtype=torch.int32, device="cuda")
+    out = torch.full((T, shape.H), float("nan"), dtype=torch.bfloat16, device="cuda")
+    layer.forward(h, pol, out=out, topk_idx=idx, topk_w=wt, audit=audit,
+                  stages=pmpe.STAGE_ALL if stages is None else stages)
+    torch.cuda.synchronize()
+    a = pmpe.audit_read(audit, T, E, check_status=False)
+    ws = layer.workspace(T)
+    L = pmpe.workspace_layout(shape)
+    R = T * k
+
+    def region(name, dtype, n):
+        nbytes = n * torch.tensor([], dtype=dtype).element_size()
+        return ws[L[name]:L[name] + nbytes].view(dtype).cpu()
+
+    return dict(out=bf16_bits(out), idx=idx.cpu().numpy(), w=wt.cpu().numpy(), audit=a,
+                tau=region("tau", torch.uint8, T).numpy(),
+                counts=region("counts", torch.int32, E).numpy().view(np.uint32),
+                offsets=region("offsets", torch.int32, E + 1).numpy().view(np.uint32),
+                slot_of=region("slot_of", torch.int32, R).numpy().reshape(T, k),
+                tok_of_slot=region("tok_of_slot", torch.int32, R).numpy(),
+                a_perm=(region("a_perm", torch.bfloat16, R * shape.H).view(torch.int16).numpy().view(np.uint16)
+                        .reshape(R, shape.H) if R * shape.H <= (1 << 24) else None),
+                layer=layer)
+
+
+def check_against_oracle(shape: LayerShape, w_cpu: dict, h_cpu, pol_cpu, gpu: dict, tokens=None):
+    """Compare a GPU run with the oracle on the same inputs, on all tokens
+    or on the sampled ``tokens``.  Returns a report dict; asserts the rules:
+      * tau bit-exact; every routed id inside the pool tau selects;
+      * top-k ids bit-exact except tokens whose oracle gap z_(k) - z_(k+1) is
+        below GAP_EPS (counted, and only checked for pool membership);
+      * routing weights within 2e-5 (absolute);
+      * outputs within MAX_ABS_REL * max|ref| and MEAN_REL mean relative error.
+    """
+    import oracle
+    L = oracle_layer(shape, w_cpu, h_cpu, pol_cpu)
+    r = oracle.forward(L, tokens=tokens)
+    toks = np.arange(shape.T) if tokens is None else np.asarray(tokens)
+    tau = oracle.resolve(None if pol_cpu is None else pol_cpu.numpy(), shape.T)
+    assert np.array_equal(gpu["tau"], tau), "resolved policy differs"
+    gi = gpu["idx"]
+    in_priv = gi >= shape.E_pub
+    assert np.all((gi >= 0) & (gi < shape.E)), "routed id out of range"
+    assert np.all(in_priv == (tau[:, None] == 1)), "a routed id lies outside the pool tau selects"
+    excused = r["gap"] < GAP_EPS
+    ok = ~excused
+    assert np.array_equal(gi[toks][ok], r["idx"][ok]), "top-k ids differ on tokens outside the gap rule"
+    np.testing.assert_allclose(gpu["w"][toks][ok], r["w"][ok], rtol=0, atol=2e-5)
+    mx, mean = output_errors(gpu["out"][toks][ok], r["out"][ok])
+    assert mx <= MAX_ABS_REL and mean <= MEAN_REL, (mx, mean)
+    return dict(excused=int(excused.sum()), max_abs_rel=mx, mean_rel=mean, oracle=r)
+
+
+def check_audit(shape: LayerShape, pol_cpu, gpu: dict):
+    """Audit invariants that hold at any size (G1 of Sec. 2.2 Eq. 1 and the
+    hook audit of Sec. 5.2): route log == histogram of the routed ids,
+    execution counts == route counts, no private row for a DENY token."""
+    import oracle
+    a = gpu["audit"]
+    tau = oracle.resolve(None if pol_cpu is None else pol_cpu.numpy(), shape.T)
+    hist = np.bincount(gpu["idx"].reshape(-1), minlength=shape.E).astype(np.uint32)
+    assert a["status"] == 0, a["status"]
+    assert np.array_equal(a["route_count"], hist)
+    assert np.array_equal(gpu["counts"], hist)
+    assert a["route_count"].sum() == shape.T * shape.k
+    assert a["route_count"][shape.E_pub:].sum() == shape.k * tau.sum()
+    assert np.array_equal(a["exec_rows"], a["route_count"]), "execution audit differs from the route log"
+    assert np.array_equal(a["exec_tiles"] > 0, hist > 0), "an expert ran tiles without rows, or rows without tiles"
+    assert np.array_equal(a["route_priv_rows"], shape.k * tau.astype(np.uint32))
+    assert np.array_equal(a["exec_priv_rows"], a["route_priv_rows"])
+    assert np.all(a["exec_priv_rows"][tau == 0] == 0), "a DENY token executed a private expert row"
+    assert a["shared_rows"] == shape.T * shape.E_sh
+
+
+def check_dispatch(shape: LayerShape, h_cpu, gpu: dict):
+    """The dispatch order equals the oracle's definition applied to the GPU's
+    own route log, bit for bit, and each gathered row is its token's row."""
+    import oracle
+    counts, offsets, slot_of, tok_of_slot = oracle.permute(gpu["idx"], shape.E)
+    assert np.array_equal(gpu["offsets"], offsets)
+    assert np.array_equal(gpu["slot_of"], slot_of)
+    assert np.array_equal(gpu["tok_of_slot"], tok_of_slot)
+    if gpu.get("a_perm") is not None:
+        assert np.array_equal(gpu["a_perm"], bf16_bits(h_cpu)[tok_of_slot])

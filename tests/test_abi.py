@@ -1,0 +1,132 @@
+"""The C ABI without a GPU: the library builds for sm_103a, loads, exports
+every function include/pmpe.h declares, and its host-only entry points
+(sizes, layout, status text, argument validation) behave as documented.
+No call here reaches a CUDA kernel."""
+import ctypes
+import os
+import re
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "pmpe.h")
+
+pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"),
+                                reason="no CUDA toolkit to build the library")
+
+
+@pytest.fixture(scope="module")
+def pmpe():
+    from paper_2608_06690_gb300 import build
+    build.build()
+    from paper_2608_06690_gb300 import pmpe as m
+    return m
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^PMPE_API\s+[\w\s\*]*?\b(pmpe_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_documented_entry_points():
+    names = declared_functions()
+    for must in ("pmpe_moe_forward", "pmpe_policy_resolve", "pmpe_audit_read"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(pmpe):
+    lib = ctypes.CDLL(pmpe.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(declared_functions()) == set(pmpe.EXPORTED)
+    out = subprocess.run(["nm", "-D", "--defined-only", pmpe.LIB_PATH], capture_output=True, text=True).stdout
+    exported = sorted(l.split()[-1] for l in out.splitlines() if " T " in l)
+    assert exported == declared_functions()
+
+
+def test_audit_words_and_fields(pmpe):
+    import numpy as np
+    T, E = 5, 7
+    n = pmpe.audit_words(T, E)
+    assert n == 2 + 3 * E + 2 * T
+    f = pmpe.audit_fields(np.arange(n, dtype=np.uint32), T, E)
+    assert f["status"] == 0 and f["shared_rows"] == 1
+    assert f["route_count"][0] == 2 and f["exec_priv_rows"][-1] == n - 1
+
+
+def test_workspace_size_and_layout(pmpe):
+    from paper_2608_06690_gb300.inputs import LayerShape
+    s = LayerShape(T=4096, H=2048, I=768, E_pub=128, E_priv=32, E_sh=0, k=8, renormalize=True)
+    L = pmpe.workspace_layout(s)
+    assert pmpe.workspace_size(s) == L["total"]
+    R = s.T * s.k
+    assert L["a_perm"] % 1024 == 0 and L["act"] % 1024 == 0 and L["y"] % 1024 == 0
+    assert L["act"] >= L["a_perm"] + 2 * R * s.H and L["y"] >= L["act"] + 2 * R * s.I
+    assert L["total"] >= L["y"] + 2 * R * s.H
+    assert L["act_sh"] == 0 and L["y_sh"] == 0
+    s2 = LayerShape(T=100, H=256, I=128, E_pub=8, E_priv=4, E_sh=2, k=2, renormalize=False)
+    L2 = pmpe.workspace_layout(s2)
+    assert L2["y_sh"] >= L2["act_sh"] + 2 * s2.T * s2.E_sh * s2.I
+    assert pmpe.workspace_size(LayerShape(64, 200, 128, 8, 4, 0, 2, True)) == 0    # H % 128
+    assert pmpe.workspace_size(LayerShape(64, 256, 128, 8, 4, 0, 9, True)) == 0    # k > pool
+
+
+def test_status_strings(pmpe):
+    assert pmpe.status_string(0) == "ok"
+    for c in (-1, -2, -3, -4, -5, -6):
+        assert pmpe.status_string(c) not in ("ok", "unknown status")
+    assert pmpe.status_string(-99) == "unknown status"
+
+
+def test_validation_rejects_before_any_cuda_call(pmpe):
+    """Invalid descriptors are rejected on the host; with fake (never
+    dereferenced) device pointers nothing is launched."""
+    from paper_2608_06690_gb300.inputs import LayerShape
+    lib = pmpe._lib
+    assert lib.pmpe_moe_forward(None, None) == pmpe.ERR_INVALID_ARG
+
+    class Fake:
+        def __init__(self, addr):
+            self.addr = addr
+
+        def data_ptr(self):
+            return self.addr
+
+        def numel(self):
+            return 1 << 40
+
+        def element_size(self):
+            return 1
+
+    p = Fake(0x10000000)
+    W = {n: p for n in ("router_pub", "router_priv", "gate_pub", "up_pub", "down_pub", "gate_priv", "up_priv",
+                        "down_priv")}
+
+    def rc(shape, **over):
+        args = dict(weights=W, hidden=p, policy=None, out=p, workspace=p)
+        args.update(over)
+        d = pmpe.make_desc(shape, args["weights"], args["hidden"], args["policy"], args["out"], args["workspace"])
+        return lib.pmpe_moe_forward(ctypes.byref(d), None)
+
+    ok = LayerShape(64, 256, 128, 8, 4, 0, 2, True)
+    assert rc(LayerShape(64, 256, 128, 8, 4, 0, 5, True)) == pmpe.ERR_INVALID_ARG      # k > E_priv
+    assert rc(LayerShape(64, 256, 128, 8, 4, 0, 0, True)) == pmpe.ERR_INVALID_ARG      # k < 1
+    assert rc(LayerShape(-1, 256, 128, 8, 4, 0, 2, True)) == pmpe.ERR_INVALID_ARG     # T < 0
+    assert rc(LayerShape(64, 192, 128, 8, 4, 0, 2, True)) == pmpe.ERR_UNSUPPORTED_SHAPE  # H % 128
+    assert rc(LayerShape(64, 256, 64, 8, 4, 0, 2, True)) == pmpe.ERR_UNSUPPORTED_SHAPE   # I % 128
+    assert rc(LayerShape(64, 256, 128, 300, 4, 0, 2, True)) == pmpe.ERR_UNSUPPORTED_SHAPE  # pool > 256
+    assert rc(LayerShape(64, 256, 128, 40, 40, 0, 33, True)) == pmpe.ERR_UNSUPPORTED_SHAPE  # k > 32
+    assert rc(ok, hidden=None) == pmpe.ERR_INVALID_ARG
+    assert rc(ok, out=None) == pmpe.ERR_INVALID_ARG
+    assert rc(ok, weights=dict(W, down_priv=None)) == pmpe.ERR_INVALID_ARG
+    assert rc(LayerShape(64, 256, 128, 8, 4, 1, 2, True)) == pmpe.ERR_INVALID_ARG      # shared weights missing
+    assert rc(ok, hidden=Fake(0x10000008)) == pmpe.ERR_UNSUPPORTED_SHAPE               # not 16-byte aligned
+    assert rc(ok, workspace=None) == pmpe.ERR_WORKSPACE
+    assert rc(ok, workspace=Fake(0x10000010)) == pmpe.ERR_WORKSPACE                   # not 256-byte aligned
+    assert rc(LayerShape(0, 256, 128, 8, 4, 0, 2, True), hidden=None, out=None, workspace=None) == pmpe.OK
+    assert lib.pmpe_policy_resolve(None, -1, None, None) == pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_policy_resolve(None, 0, None, None) == pmpe.OK
+    assert lib.pmpe_audit_reset(None, 4, 4, None) == pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_audit_read(None, 4, 4, None, None, 10) == pmpe.ERR_INVALID_ARG
