@@ -166,6 +166,32 @@ PMPE_API int pmpe_moe_forward(const pmpe_moe_desc *d, void *stream);
  * with the same inputs.  pmpe_moe_forward() == stages PMPE_STAGE_ALL. */
 PMPE_API int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *stream);
 
+/* Size of the device scratch array that pmpe_moe_forward_noalloc() uses in
+ * place of a caller workspace: 32 MiB, reserved on every GPU that loads the
+ * library until the process exits.  (A 64-token decode step of a layer with
+ * H = 2048, I = 768, top-8 needs about 5 MB of it.) */
+#define PMPE_STATIC_SCRATCH_BYTES (32u << 20)
+
+/* The layer forward for callers that cannot allocate device memory where
+ * they run it -- a plugin whose host owns all device memory and offers it no
+ * allocator, or a serving loop that must not pay cudaMalloc's device-wide
+ * synchronisation or risk running out of memory mid-request.  The paper has
+ * no counterpart to this entry point; it is a deployment convenience.
+ *   - Same arguments and results as pmpe_moe_forward(), except that
+ *     d->workspace and d->workspace_bytes are ignored: the scratch is the
+ *     library's own static device array of PMPE_STATIC_SCRATCH_BYTES.
+ *   - Returns PMPE_ERR_WORKSPACE, launching nothing, when the shape's
+ *     pmpe_moe_workspace_size() exceeds PMPE_STATIC_SCRATCH_BYTES.
+ *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current) and caches it; make
+ *     that first call before any stream capture.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents (the forward clears what must start at zero).  Calls whose
+ *     kernels overlap on the GPU race on it: order them on one stream or with
+ *     events. */
+PMPE_API int pmpe_moe_forward_noalloc(const pmpe_moe_desc *d, void *stream);
+
 /* Zero the audit buffer (pmpe_audit_words(T, E) words). */
 PMPE_API int pmpe_audit_reset(uint32_t *audit, int T, int E, void *stream);
 

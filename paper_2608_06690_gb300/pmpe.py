@@ -48,7 +48,10 @@ KERNELS_PER_FORWARD = 6
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
-            "pmpe_status_string")
+            "pmpe_status_string", "pmpe_moe_forward_noalloc")
+
+# Bytes of the library's static scratch array used by pmpe_moe_forward_noalloc.
+STATIC_SCRATCH_BYTES = 32 << 20
 
 _vp = ctypes.c_void_p
 
@@ -83,6 +86,8 @@ _lib.pmpe_moe_forward.restype = ctypes.c_int
 _lib.pmpe_moe_forward.argtypes = [ctypes.POINTER(MoeDesc), _vp]
 _lib.pmpe_moe_forward_stages.restype = ctypes.c_int
 _lib.pmpe_moe_forward_stages.argtypes = [ctypes.POINTER(MoeDesc), ctypes.c_uint, _vp]
+_lib.pmpe_moe_forward_noalloc.restype = ctypes.c_int
+_lib.pmpe_moe_forward_noalloc.argtypes = [ctypes.POINTER(MoeDesc), _vp]
 _lib.pmpe_audit_reset.restype = ctypes.c_int
 _lib.pmpe_audit_reset.argtypes = [_vp, ctypes.c_int, ctypes.c_int, _vp]
 _lib.pmpe_audit_read.restype = ctypes.c_int
