@@ -1,0 +1,551 @@
+// Stages 3 and 4 of the layer on the 5th-generation tensor cores: grouped
+// BF16 expert GEMMs with tcgen05.mma accumulating in tensor memory (TMEM),
+// operands staged by TMA into 128-byte-swizzled shared memory.
+//
+//   gate/up:  act = bf16(silu(A_e W_gate,e^T) * (A_e W_up,e^T))    (SwiGLU fused)
+//   down:     y   = bf16(w_row * (act_e W_down,e^T))
+//
+// Groups are the routed experts (rows of the dispatch order) plus, with
+// shared experts, one dense group over all T tokens (gate/up weights of the
+// E_sh experts side by side; the down projection sums the E_sh experts in
+// one accumulator).  A persistent grid (one CTA per SM) walks a tile list
+// built on the device from the dispatch offsets: no host sync, and empty
+// experts contribute no tile.
+//
+// CTA roles (192 threads):
+//   warp 0       one thread issues the TMA loads of a 4-stage ring (A: 128
+//                rows x 64 K; B: 256 rows x 64 K, i.e. 128 gate + 128 up rows,
+//                or 256 / 128 output columns of the down projection)
+//   warp 1       allocates 512 TMEM columns (two 128 x 256 FP32
+//                accumulators, so the epilogue of one tile overlaps the MMAs
+//                of the next) and one thread issues tcgen05.mma M=128 N=256
+//                K=16, committing stage releases and accumulator-full events
+//   warps 2..5   epilogue: tcgen05.ld of the warp's 32 TMEM lanes (= 32 tile
+//                rows), SwiGLU or weight scaling, BF16 stores; in gate/up mode
+//                the tiles of N-tile 0 also write the execution audit
+// Every mbarrier wait is bounded in time: on expiry the CTA records
+// PMPE_STATUS_PIPELINE_TIMEOUT, stops issuing work, waits (bounded) for its
+// own copies and MMAs in flight, frees its TMEM and exits.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+#include <mutex>
+
+#include "pmpe_internal.cuh"
+
+namespace pmpe {
+namespace {
+
+constexpr int BM = 128;                       // rows per tile (MMA M)
+constexpr int BK = 64;                        // K per stage: one 128-byte swizzle row
+constexpr int kStages = 4;
+constexpr int kABytes = BM * BK * 2;          // 16 KB
+constexpr int kBBytes = 256 * BK * 2;         // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kAccCols = 256;                 // FP32 TMEM columns per accumulator
+constexpr int kTmemCols = 2 * kAccCols;
+constexpr int kThreads = 192;
+constexpr int kMaxGroups = 2 * kMaxPool + 1;
+constexpr int kDynSmem = kStages * kStageBytes + 1024 /* alignment slack */;
+constexpr unsigned long long kWaitLimitNs = 4000000000ull;  // 4 s: far beyond any legitimate wait
+
+enum { kGateUp = 0, kDown = 1 };
+
+struct TcParams {
+    int mode;
+    int E, E_pub, E_sh, T, H, I, R;
+    int bn;           // output columns per tile (gate/up: 128 activation columns; down: 256 or 128)
+    uint32_t idesc;   // tcgen05 instruction descriptor (BF16 x BF16 -> FP32, M = 128, N = MMA width)
+    uint32_t tx_bytes;
+    const uint32_t *offsets;
+    bf16 *C_routed, *C_shared;
+    const float *w_of_slot;
+    const int32_t *tok_of_slot;
+    uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
+};
+
+struct TcMaps {
+    CUtensorMap a_routed, a_shared;
+    CUtensorMap b0[3];  // per pool [pub, priv, shared]: gate (gate/up mode) or down
+    CUtensorMap b1[3];  // up (gate/up mode)
+};
+
+// ------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ unsigned long long globaltimer_ns()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Wait for the phase of `bar` with parity `parity`, for at most kWaitLimitNs
+// or until another role raised the abort flag.  Returns false on give-up.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, uint32_t *status)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    for (;;) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            *abort_flag = 1;
+            if (status) atomicOr(status, PMPE_STATUS_PIPELINE_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];\n" ::
+            "r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row groups 1024 bytes apart (SBO); LBO is unused for this
+// layout; bits 46..48 hold the fixed value 0b001; swizzle mode 2 = 128 B.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
+{
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate)
+{
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
+                 : "memory");
+}
+
+// 32 consecutive FP32 columns of this warp's 32 TMEM lanes: thread i gets
+// lane (base lane + i), columns col .. col+31.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v)
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
+
+// ------------------------------------------------------------- tile list
+
+struct Tile {
+    int g, m0, n0, rows, row_base, nkb;
+    bool shared;
+};
+
+struct TileTable {
+    int prefix[kMaxGroups + 1];
+    int rows[kMaxGroups];
+    int base[kMaxGroups];
+};
+
+__device__ __forceinline__ int group_n(const TcParams &p, bool shared)
+{
+    return p.mode == kGateUp ? (shared ? p.E_sh * p.I : p.I) : p.H;
+}
+__device__ __forceinline__ int group_k(const TcParams &p, bool shared)
+{
+    return p.mode == kGateUp ? p.H : (shared ? p.E_sh * p.I : p.I);
+}
+
+__device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &tt, int G, int tile)
+{
+    int lo = 0, hi = G - 1;  // last group with prefix <= tile
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (tt.prefix[mid] <= tile) lo = mid; else hi = mid - 1;
+    }
+    Tile t;
+    t.g = lo;
+    t.shared = lo >= p.E;
+    const int rows = tt.rows[lo];
+    const int mt = (rows + BM - 1) / BM;
+    const int local = tile - tt.prefix[lo];
+    const int n_tile = local / mt, m_tile = local - n_tile * mt;
+    t.m0 = m_tile * BM;
+    t.n0 = n_tile * p.bn;
+    t.rows = min(BM, rows - t.m0);
+    t.row_base = tt.base[lo];
+    t.nkb = group_k(p, t.shared) / BK;
+    return t;
+}
+
+// ---------------------------------------------------------------- kernel
+
+__global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcParams p, const __grid_constant__ TcMaps maps)
+{
+    extern __shared__ uint8_t dsmem[];
+    __shared__ TileTable tt;
+    __shared__ __align__(8) uint64_t bars[2 * kStages + 5];
+    __shared__ uint32_t s_tmem;
+    __shared__ volatile int s_abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
+    const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
+
+    const int G = p.E + (p.E_sh > 0 ? 1 : 0);
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
+        for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
+        mbar_init(done_bar, 1);
+        s_abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(&s_tmem)),
+                     "r"(kTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
+    }
+    // tile list: rows and tiles per group, prefix over groups
+    for (int g = tid; g < G; g += kThreads) {
+        const bool shared = g >= p.E;
+        int rows, base;
+        if (shared) {
+            rows = p.T;
+            base = 0;
+        } else {  // clamped to [0, R): only a corrupt workspace could make this matter
+            const int b = min((int)p.offsets[g], p.R), e = min(max((int)p.offsets[g + 1], b), p.R);
+            rows = e - b;
+            base = b;
+        }
+        tt.rows[g] = rows;
+        tt.base[g] = base;
+        tt.prefix[g + 1] = ((rows + BM - 1) / BM) * (group_n(p, shared) / p.bn);
+    }
+    __syncthreads();
+    if (warp == 0) {
+        int carry = 0;
+        for (int b = 0; b < G; b += 32) {
+            int v = b + lane < G ? tt.prefix[b + lane + 1] : 0;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(~0u, v, off);
+                if (lane >= off) v += y;
+            }
+            __syncwarp();
+            if (b + lane < G) tt.prefix[b + lane + 1] = carry + v;
+            carry += __shfl_sync(~0u, v, 31);
+        }
+        if (lane == 0) tt.prefix[0] = 0;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = s_tmem;
+    const int total = tt.prefix[G];
+
+    if (warp == 0 && lane == 0) {
+        // ------------------------------------------------ TMA producer
+        int stage = 0;
+        uint32_t phase = 0;
+        uint32_t filled = 0, last_parity = 0;  // per-stage bits, for the drain below
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
+            const Tile t = decode_tile(p, tt, G, tile);
+            const int q = t.shared ? 2 : (t.g < p.E_pub ? 0 : 1);
+            const int ei = t.shared ? 0 : (q == 0 ? t.g : t.g - p.E_pub);
+            const CUtensorMap *amap = t.shared ? &maps.a_shared : &maps.a_routed;
+            const int arow = t.row_base + t.m0;
+            bool ok = true;
+            for (int kb = 0; kb < t.nkb; ++kb) {
+                if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
+                const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
+                mbar_expect_tx(full_bar(stage), p.tx_bytes);
+                const int kx = kb * BK;
+                tma_load_2d(sA, amap, full_bar(stage), kx, arow);
+                if (p.mode == kGateUp) {
+                    const int brow = ei * p.I + t.n0;  // shared: n0 spans E_sh * I rows
+                    tma_load_2d(sB, &maps.b0[q], full_bar(stage), kx, brow);
+                    tma_load_2d(sB + BM * 128, &maps.b1[q], full_bar(stage), kx, brow);
+                } else if (t.shared) {
+                    const int s = kx / p.I;
+                    tma_load_2d(sB, &maps.b0[2], full_bar(stage), kx - s * p.I, s * p.H + t.n0);
+                } else {
+                    tma_load_2d(sB, &maps.b0[q], full_bar(stage), kx, ei * p.H + t.n0);
+                }
+                filled |= 1u << stage;
+                last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+        }
+        // drain: every copy this thread issued has landed before the CTA exits
+        for (int s = 0; s < kStages; ++s)
+            if ((filled >> s) & 1u) {
+                const unsigned long long t0 = globaltimer_ns();
+                while (!mbar_try_wait(full_bar(s), (last_parity >> s) & 1u))
+                    if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+            }
+    } else if (warp == 1 && lane == 0) {
+        // ------------------------------------------------ MMA issuer
+        int stage = 0, it = 0;
+        uint32_t phase = 0;
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x, ++it) {
+            const Tile t = decode_tile(p, tt, G, tile);
+            const int buf = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            if (!mbar_wait(tempty_bar(buf), use ^ 1u, &s_abort, p.status)) break;
+            tc_fence_after();
+            const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kAccCols);
+            bool ok = true;
+            for (int kb = 0; kb < t.nkb; ++kb) {
+                if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
+                const uint64_t ad = sw128_desc(sA), bd = sw128_desc(sB);
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)  // +32 bytes of K per step inside the swizzle row
+                    tc_mma(d_tmem, ad + 2 * k, bd + 2 * k, p.idesc, (kb | k) != 0);
+                tc_commit(empty_bar(stage));
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+            tc_commit(tfull_bar(buf));
+        }
+        // every MMA this thread issued has completed before TMEM is freed
+        tc_commit(done_bar);
+        {
+            const unsigned long long t0 = globaltimer_ns();
+            while (!mbar_try_wait(done_bar, 0))
+                if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+        }
+    } else if (warp >= 2) {
+        // ------------------------------------------------ epilogue
+        const int quarter = warp & 3;  // TMEM lanes this warp may access
+        int it = 0;
+        for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+            const Tile t = decode_tile(p, tt, G, tile);
+            const int buf = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            // one lane waits, the warp follows: tcgen05.ld below is warp-collective
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(tfull_bar(buf), use, &s_abort, p.status) ? 1 : 0;
+            ok = __shfl_sync(~0u, ok, 0);
+            if (!ok) break;
+            __syncwarp();
+            tc_fence_after();
+            const int r = quarter * 32 + lane;  // tile row of this thread
+            const bool valid = r < t.rows;
+            const int grow = t.row_base + t.m0 + r;
+            const uint32_t taddr = tmem_base + (uint32_t)(buf * kAccCols) + ((uint32_t)(quarter * 32) << 16);
+            if (p.mode == kGateUp) {
+                const int ldc = t.shared ? p.E_sh * p.I : p.I;
+                bf16 *crow = (t.shared ? p.C_shared : p.C_routed) + (size_t)grow * ldc + t.n0;
+#pragma unroll 1
+                for (int c = 0; c < BM / 32; ++c) {
+                    float gv[32], uv[32];
+                    tmem_ld32(taddr + c * 32, gv);
+                    tmem_ld32(taddr + 128 + c * 32, uv);
+                    tmem_ld_wait();
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        pk[i] = pack_bf16x2(silu_mul(gv[2 * i], uv[2 * i]), silu_mul(gv[2 * i + 1], uv[2 * i + 1]));
+                    if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    }
+                }
+            } else {
+                bf16 *crow = (t.shared ? p.C_shared : p.C_routed) + (size_t)grow * p.H + t.n0;
+                const float sc = t.shared ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
+#pragma unroll 1
+                for (int c = 0; c < p.bn / 32; ++c) {
+                    float v[32];
+                    tmem_ld32(taddr + c * 32, v);
+                    tmem_ld_wait();
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(v[2 * i] * sc, v[2 * i + 1] * sc);
+                    if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty_bar(buf));
+            // execution audit: rows this tile processed, counted where they ran
+            if (p.mode == kGateUp) {
+                const unsigned vm = __ballot_sync(~0u, valid);
+                if (!t.shared && t.n0 == 0) {
+                    if (lane == 0 && p.exec_rows && vm) atomicAdd(&p.exec_rows[t.g], (unsigned)__popc(vm));
+                    if (lane == 0 && quarter == 0 && p.exec_tiles) atomicAdd(&p.exec_tiles[t.g], 1u);
+                    if (valid && t.g >= p.E_pub && p.exec_priv_rows) atomicAdd(&p.exec_priv_rows[p.tok_of_slot[grow]], 1u);
+                }
+                if (t.shared && p.shared_rows && lane == 0 && vm && (t.n0 % p.I) == 0)
+                    atomicAdd(p.shared_rows, (unsigned)__popc(vm));
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(kTmemCols));
+    }
+}
+
+// ------------------------------------------------------------ host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    });
+    return fn;
+}
+
+// 2-D BF16 tensor map over a row-major [rows, cols] matrix, box = 64 x box_rows,
+// 128-byte swizzle, zero fill out of bounds.
+bool encode_2d(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_rows)
+{
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+uint32_t make_idesc(int M, int N)
+{
+    return (1u << 4)                    // D: FP32
+           | (1u << 7)                  // A: BF16
+           | (1u << 10)                 // B: BF16
+           | ((uint32_t)(N >> 3) << 17) // N / 8
+           | ((uint32_t)(M >> 4) << 24);// M / 16   (A and B K-major: transpose bits 15, 16 = 0)
+}
+
+cudaError_t launch_tc(const Ctx &c, int mode)
+{
+    const Shape &s = c.s;
+    TcParams p;
+    TcMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    p.mode = mode;
+    p.E = s.E(); p.E_pub = s.E_pub; p.E_sh = s.E_sh; p.T = s.T; p.H = s.H; p.I = s.I; p.R = s.T * s.k;
+    p.offsets = c.offsets;
+    p.w_of_slot = c.w_of_slot;
+    p.tok_of_slot = c.tok_of_slot;
+    p.exec_rows = c.audit.exec_rows;
+    p.exec_tiles = c.audit.exec_tiles;
+    p.exec_priv_rows = c.audit.exec_priv_rows;
+    p.shared_rows = c.audit.shared_rows;
+    p.status = c.audit.status;
+    const uint64_t R = (uint64_t)p.R, T = (uint64_t)s.T;
+    bool ok = true;
+    if (mode == kGateUp) {
+        p.bn = 128;
+        p.idesc = make_idesc(BM, 256);
+        p.tx_bytes = kABytes + 2 * 128 * BK * 2;
+        p.C_routed = c.act;
+        p.C_shared = c.act_sh;
+        ok &= encode_2d(&maps.a_routed, c.a_perm, s.H, R, BM);
+        for (int q = 0; q < 2; ++q) {
+            const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.I;
+            ok &= encode_2d(&maps.b0[q], c.gate[q], s.H, n, 128);
+            ok &= encode_2d(&maps.b1[q], c.up[q], s.H, n, 128);
+        }
+        if (s.E_sh > 0) {
+            ok &= encode_2d(&maps.a_shared, c.hidden, s.H, T, BM);
+            ok &= encode_2d(&maps.b0[2], c.gate[2], s.H, (uint64_t)s.E_sh * s.I, 128);
+            ok &= encode_2d(&maps.b1[2], c.up[2], s.H, (uint64_t)s.E_sh * s.I, 128);
+        }
+    } else {
+        p.bn = (s.H % 256 == 0) ? 256 : 128;
+        p.idesc = make_idesc(BM, p.bn);
+        p.tx_bytes = kABytes + p.bn * BK * 2;
+        p.C_routed = c.y;
+        p.C_shared = c.y_sh;
+        ok &= encode_2d(&maps.a_routed, c.act, s.I, R, BM);
+        for (int q = 0; q < 2; ++q) {
+            const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
+            ok &= encode_2d(&maps.b0[q], c.down[q], s.I, n, p.bn);
+        }
+        if (s.E_sh > 0) {
+            ok &= encode_2d(&maps.a_shared, c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
+            ok &= encode_2d(&maps.b0[2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, p.bn);
+        }
+    }
+    if (!ok) return cudaErrorInvalidValue;
+    cudaError_t err = cudaFuncSetAttribute(expert_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem);
+    if (err != cudaSuccess) return err;
+    expert_gemm_tc_kernel<<<c.num_sms, kThreads, kDynSmem, c.stream>>>(p, maps);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, kGateUp); }
+cudaError_t launch_down(const Ctx &c) { return launch_tc(c, kDown); }
+
+}  // namespace pmpe
