@@ -64,7 +64,7 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
@@ -216,6 +216,7 @@ def run_ours(args):
     def step():
         layer.forward(h, pol, out=out)
 
+    clk = ClockSampler(local).__enter__()   # samples through warm-up, timed region and breakdowns
     for _ in range(max(args.warmup, 3)):
         step()
     torch.cuda.synchronize(dev)
@@ -224,16 +225,15 @@ def run_ours(args):
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     barrier()
     torch.cuda.synchronize(dev)
-    with ClockSampler(local) as clk:
-        t_wall0 = time.perf_counter()
-        for e0, e1 in evs:
-            flush.zero_()
-            e0.record(stream)
-            step()
-            e1.record(stream)
-        torch.cuda.synchronize(dev)
-        t_wall = time.perf_counter() - t_wall0
-        barrier()
+    t_wall0 = time.perf_counter()
+    for e0, e1 in evs:
+        flush.zero_()
+        e0.record(stream)
+        step()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall = time.perf_counter() - t_wall0
+    barrier()
     step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
     total_ms = torch.tensor([sum(step_ms)], dtype=torch.float64, device=dev)
     if ws > 1:
@@ -241,20 +241,25 @@ def run_ours(args):
     total_ms = float(total_ms.item())
     value = ws * s.T * args.steps / (total_ms / 1e3)
 
-    # ---- per-stage breakdown (same launches, events between the stages)
+    # ---- per-stage breakdown: each stage after its own L2 flush, so the GPU
+    # is still busy flushing while the host enqueues the stage (no host gap
+    # inside the measured interval); stages run in pipeline order on the
+    # workspace the previous stage filled
     stages = [("route", pmpe.STAGE_ROUTE), ("permute", pmpe.STAGE_PERMUTE), ("gateup", pmpe.STAGE_GATEUP),
               ("down", pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE)]
     stage_ms = {n: [] for n, _ in stages}
     for _ in range(args.steps):
-        flush.zero_()
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)]
-        ev[0].record(stream)
-        for i, (n, bit) in enumerate(stages):
+        evs_s = []
+        for n, bit in stages:
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
             layer.forward(h, pol, out=out, stages=bit)
-            ev[i + 1].record(stream)
+            b.record(stream)
+            evs_s.append((n, a, b))
         torch.cuda.synchronize(dev)
-        for i, (n, _) in enumerate(stages):
-            stage_ms[n].append(ev[i].elapsed_time(ev[i + 1]))
+        for n, a, b in evs_s:
+            stage_ms[n].append(a.elapsed_time(b))
     stage_avg = {n: float(np.mean(v)) for n, v in stage_ms.items()}
 
     # ---- audit of one forward (exactness of the counters is a test; here: sanity + expert loads)
@@ -287,6 +292,7 @@ def run_ours(args):
     if ws > 1:
         torch.distributed.all_reduce(e2e_t, op=torch.distributed.ReduceOp.MAX)
     e2e_value = ws * s.T * args.steps / (float(e2e_t.item()) / 1e3)
+    clk.__exit__(None, None, None)
 
     if rank != 0:
         if ws > 1:

@@ -122,13 +122,14 @@ PMPE_API size_t pmpe_moe_workspace_size(int T, int H, int I, int E_pub, int E_pr
 typedef struct pmpe_workspace_layout {
     size_t total;
     size_t tau;          /* uint8  [T]      resolved policy bits */
-    size_t counts;       /* uint32 [E]      rows routed to each expert (router's count) */
+    size_t counts;       /* uint32 [E]      rows routed to each expert (counted by the dispatch stage) */
     size_t offsets;      /* uint32 [E+1]    exclusive prefix sum of counts */
     size_t topk_idx;     /* int32  [T, k]   used when desc.topk_idx is NULL */
     size_t topk_w;       /* float  [T, k]   used when desc.topk_w is NULL */
     size_t slot_of;      /* int32  [T, k]   dispatch row of (t, j) */
     size_t tok_of_slot;  /* int32  [T*k]    token of each dispatch row */
     size_t w_of_slot;    /* float  [T*k]    routing weight of each dispatch row */
+    size_t router_rows;  /* BF16   [(ceil(T/128)+1)*128, H] token rows of each router tile, pool order */
     size_t a_perm;       /* BF16   [T*k, H] token rows in dispatch order */
     size_t act;          /* BF16   [T*k, I] silu(g)*u of each dispatch row */
     size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row */

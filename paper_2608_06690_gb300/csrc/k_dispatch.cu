@@ -4,10 +4,10 @@
 // Dispatch order (the grouping any grouped expert execution needs): rows are
 // grouped by expert id and, inside an expert, ordered by token then rank, so
 // the order is a pure function of the route log.  One CTA per expert scans
-// the [T, k] id list with block-wide ballots and writes that expert's rows;
-// its row count is cross-checked against the router's atomic count and a
-// mismatch is recorded in the status word.  The gather then copies each
-// token row into its dispatch row with 16-byte vector loads, one warp per row.
+// the [T, k] id list twice: first to count the routed rows of lower ids (its
+// offset) and its own, then to write its rows with block-wide scans.  An id
+// outside [0, E) is recorded in the status word.  The gather then copies each
+// token row into its dispatch row with 16-byte vector loads.
 //
 // Combine: out_t = bf16( sum_{j < k} y[slot(t, j)] + y_shared[t] ), summed in
 // FP32 in a fixed order (j ascending, then shared), so the result of a token
@@ -51,9 +51,8 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int *warp_tot, int &t
 struct DispatchParams {
     const int32_t *idx;
     const float *w;
-    const uint32_t *counts;
     int R, k, E;
-    uint32_t *offsets;
+    uint32_t *counts, *offsets;
     int32_t *slot_of, *tok_of_slot;
     float *w_of_slot;
     uint32_t *status;
@@ -62,46 +61,45 @@ struct DispatchParams {
 __global__ void __launch_bounds__(kScanThreads) dispatch_order_kernel(const DispatchParams p)
 {
     __shared__ int warp_tot[32];
-    __shared__ unsigned s_off;
     const int e = blockIdx.x, tid = threadIdx.x;
 
-    // offset of expert e = sum of the router's counts of the experts before it
-    unsigned part = 0;
-    for (int i = tid; i < e; i += kScanThreads) part += p.counts[i];
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(~0u, part, off);
-    if (tid == 0) s_off = 0;
-    __syncthreads();
-    if ((tid & 31) == 0 && part) atomicAdd(&s_off, part);
-    __syncthreads();
-    const unsigned off = s_off;
-    const unsigned n_e = p.counts[e];
-    if (tid == 0) {
-        p.offsets[e] = off;
-        if (e == p.E - 1) p.offsets[p.E] = off + n_e;
-    }
-
-    int running = 0;
+    // pass 1: this expert's offset = routed rows of lower expert ids; its count
+    int less = 0, mine = 0;
     bool bad = false;
+    for (int r = tid; r < p.R; r += kScanThreads) {
+        const int id = p.idx[r];
+        less += id < e;
+        mine += id == e;
+        bad |= id < 0 || id >= p.E;
+    }
+    int off, n_e;
+    block_exclusive_scan(less, warp_tot, off);
+    block_exclusive_scan(mine, warp_tot, n_e);
+    if (tid == 0) {
+        p.offsets[e] = (uint32_t)off;
+        p.counts[e] = (uint32_t)n_e;
+        if (e == p.E - 1) p.offsets[p.E] = (uint32_t)(off + n_e);
+    }
+    if (e == 0 && p.status && __syncthreads_or(bad) && tid == 0) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+
+    // pass 2: this expert's rows in (token, rank) order
+    int running = 0;
     for (int base = 0; base < p.R; base += kScanThreads * kPerThread) {
         const int r0 = base + tid * kPerThread;
         int ids[kPerThread];
 #pragma unroll
         for (int q = 0; q < kPerThread; ++q) ids[q] = (r0 + q < p.R) ? p.idx[r0 + q] : -1;
-        int mine = 0;
+        int cnt = 0;
 #pragma unroll
-        for (int q = 0; q < kPerThread; ++q) {
-            mine += ids[q] == e;
-            bad |= (r0 + q < p.R) && (ids[q] < 0 || ids[q] >= p.E);
-        }
+        for (int q = 0; q < kPerThread; ++q) cnt += ids[q] == e;
         int total;
-        int rank = block_exclusive_scan(mine, warp_tot, total);
+        int rank = block_exclusive_scan(cnt, warp_tot, total);
 #pragma unroll
         for (int q = 0; q < kPerThread; ++q) {
             if (ids[q] == e) {
                 const int r = r0 + q;
-                const int slot = (int)off + running + rank;
-                if (slot < p.R) {  // always true when the router's counts match its ids
+                const int slot = off + running + rank;
+                if (slot < p.R) {  // always true: off + n_e <= R
                     p.slot_of[r] = slot;
                     p.tok_of_slot[slot] = r / p.k;
                     p.w_of_slot[slot] = p.w[r];
@@ -111,61 +109,70 @@ __global__ void __launch_bounds__(kScanThreads) dispatch_order_kernel(const Disp
         }
         running += total;
     }
-    if (p.status) {
-        if (tid == 0 && (unsigned)running != n_e) atomicOr(p.status, PMPE_STATUS_DISPATCH_MISMATCH);
-        if (e == 0 && __syncthreads_or(bad) && tid == 0) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
-    }
 }
 
-// One warp copies one H-wide BF16 row with 16-byte vectors.
+// Row gather: one thread per 16-byte chunk of a dispatch row, so a row is
+// copied by H/8 consecutive threads with fully coalesced loads and stores.
 __global__ void __launch_bounds__(256) gather_rows_kernel(const bf16 *__restrict__ hidden,
                                                           const int32_t *__restrict__ tok_of_slot, int R, int T,
                                                           int H, bf16 *__restrict__ a_perm)
 {
-    const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-    if (row >= R) return;
-    int t = tok_of_slot[row];
-    if ((unsigned)t >= (unsigned)T) t = 0;  // only reachable after a dispatch mismatch (status word set)
-    const uint4 *src = reinterpret_cast<const uint4 *>(hidden + (size_t)t * H);
-    uint4 *dst = reinterpret_cast<uint4 *>(a_perm + (size_t)row * H);
     const int nv = H / 8;
-    for (int c = lane; c < nv; c += 32) dst[c] = __ldg(src + c);
+    const long long total = (long long)R * nv;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int row = (int)(i / nv), c = (int)(i - (long long)row * nv);
+        int t = tok_of_slot[row];
+        if ((unsigned)t >= (unsigned)T) t = 0;  // only reachable after a dispatch mismatch (status word set)
+        reinterpret_cast<uint4 *>(a_perm + (size_t)row * H)[c] =
+            __ldg(reinterpret_cast<const uint4 *>(hidden + (size_t)t * H) + c);
+    }
 }
 
+__device__ __forceinline__ void add_bf16x8(float *acc, const uint4 &v)
+{
+    const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(b[i]);
+        acc[2 * i] += f.x;
+        acc[2 * i + 1] += f.y;
+    }
+}
+
+// Combine: one thread per (token, 16-byte chunk of the output row).  The k
+// routed rows are loaded in batches of 8 independent 16-byte loads before
+// they are summed (in j order), so the loads overlap instead of forming a
+// chain of dependent memory round trips.
 __global__ void __launch_bounds__(256) combine_kernel(const bf16 *__restrict__ y, const bf16 *__restrict__ y_sh,
                                                       const int32_t *__restrict__ slot_of, int T, int H, int k,
                                                       bf16 *__restrict__ out)
 {
-    const int t = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-    if (t >= T) return;
-    int my_slot = lane < k ? slot_of[(size_t)t * k + lane] : 0;
-    if ((unsigned)my_slot >= (unsigned)(T * k)) my_slot = 0;  // only after a dispatch mismatch (status word set)
     const int nv = H / 8;
-    for (int c = lane; c < nv; c += 32) {
+    const int R = T * k;
+    const long long total = (long long)T * nv;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int t = (int)(i / nv), c = (int)(i - (long long)t * nv);
+        const int32_t *slots = slot_of + (size_t)t * k;
         float acc[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-        for (int j = 0; j < k; ++j) {
-            const int slot = __shfl_sync(~0u, my_slot, j);
-            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(y + (size_t)slot * H) + c);
-            const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+        for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+        for (int j0 = 0; j0 < k; j0 += 8) {
+            uint4 v[8];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float2 f = __bfloat1622float2(b[i]);
-                acc[2 * i] += f.x;
-                acc[2 * i + 1] += f.y;
+            for (int u = 0; u < 8; ++u) {
+                if (j0 + u < k) {
+                    int slot = __ldg(slots + j0 + u);
+                    if ((unsigned)slot >= (unsigned)R) slot = 0;  // only after a dispatch mismatch (status set)
+                    v[u] = __ldg(reinterpret_cast<const uint4 *>(y + (size_t)slot * H) + c);
+                }
             }
-        }
-        if (y_sh) {
-            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(y_sh + (size_t)t * H) + c);
-            const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float2 f = __bfloat1622float2(b[i]);
-                acc[2 * i] += f.x;
-                acc[2 * i + 1] += f.y;
-            }
+            for (int u = 0; u < 8; ++u)
+                if (j0 + u < k) add_bf16x8(acc, v[u]);
         }
+        if (y_sh) add_bf16x8(acc, __ldg(reinterpret_cast<const uint4 *>(y_sh + (size_t)t * H) + c));
         uint4 o;
         o.x = pack_bf16x2(acc[0], acc[1]);
         o.y = pack_bf16x2(acc[2], acc[3]);
@@ -173,6 +180,15 @@ __global__ void __launch_bounds__(256) combine_kernel(const bf16 *__restrict__ y
         o.w = pack_bf16x2(acc[6], acc[7]);
         reinterpret_cast<uint4 *>(out + (size_t)t * H)[c] = o;
     }
+}
+
+// Grid for a grid-stride loop over `work` items of 256-thread blocks: enough
+// blocks to cover the work once, capped at 8 resident blocks per SM.
+int grid_for(long long work, int num_sms)
+{
+    const long long blocks = (work + 255) / 256;
+    const long long cap = 8LL * num_sms;
+    return (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
 }
 
 }  // namespace
@@ -189,15 +205,16 @@ cudaError_t launch_permute(const Ctx &c)
     dispatch_order_kernel<<<s.E(), kScanThreads, 0, c.stream>>>(p);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    gather_rows_kernel<<<(R + 7) / 8, 256, 0, c.stream>>>(c.hidden, c.tok_of_slot, R, s.T, s.H, c.a_perm);
+    gather_rows_kernel<<<grid_for((long long)R * (s.H / 8), c.num_sms), 256, 0, c.stream>>>(c.hidden, c.tok_of_slot, R,
+                                                                                      s.T, s.H, c.a_perm);
     return cudaGetLastError();
 }
 
 cudaError_t launch_combine(const Ctx &c)
 {
     const Shape &s = c.s;
-    combine_kernel<<<(s.T + 7) / 8, 256, 0, c.stream>>>(c.y, s.E_sh > 0 ? c.y_sh : nullptr, c.slot_of, s.T, s.H,
-                                                         s.k, c.out);
+    combine_kernel<<<grid_for((long long)s.T * (s.H / 8), c.num_sms), 256, 0, c.stream>>>(
+        c.y, s.E_sh > 0 ? c.y_sh : nullptr, c.slot_of, s.T, s.H, s.k, c.out);
     return cudaGetLastError();
 }
 

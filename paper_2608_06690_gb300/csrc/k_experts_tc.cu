@@ -33,6 +33,7 @@
 #include <mutex>
 
 #include "pmpe_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace pmpe {
 namespace {
@@ -47,8 +48,10 @@ constexpr int kAccCols = 256;                 // FP32 TMEM columns per accumulat
 constexpr int kTmemCols = 2 * kAccCols;
 constexpr int kThreads = 192;
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
-constexpr int kDynSmem = kStages * kStageBytes + 1024 /* alignment slack */;
-constexpr unsigned long long kWaitLimitNs = 4000000000ull;  // 4 s: far beyond any legitimate wait
+constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
+constexpr int kOutBufBytes = kOutBox * kOutBox * 2;
+constexpr int kOutBytes = 4 * 2 * kOutBufBytes;  // 4 epilogue warps x 2 buffers
+constexpr int kDynSmem = kStages * kStageBytes + kOutBytes + 1024 /* alignment slack */;
 
 enum { kGateUp = 0, kDown = 1 };
 
@@ -66,112 +69,11 @@ struct TcParams {
 };
 
 struct TcMaps {
+    CUtensorMap c_routed, c_shared;  // outputs, 32 x 32 boxes, 64-byte swizzle
     CUtensorMap a_routed, a_shared;
     CUtensorMap b0[3];  // per pool [pub, priv, shared]: gate (gate/up mode) or down
     CUtensorMap b1[3];  // up (gate/up mode)
 };
-
-// ------------------------------------------------------------ PTX wrappers
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count));
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-__device__ __forceinline__ unsigned long long globaltimer_ns()
-{
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-// Wait for the phase of `bar` with parity `parity`, for at most kWaitLimitNs
-// or until another role raised the abort flag.  Returns false on give-up.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, uint32_t *status)
-{
-    if (mbar_try_wait(bar, parity)) return true;
-    const unsigned long long t0 = globaltimer_ns();
-    for (;;) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-            *abort_flag = 1;
-            if (status) atomicOr(status, PMPE_STATUS_PIPELINE_TIMEOUT);
-            return false;
-        }
-    }
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];\n" ::
-            "r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y)
-        : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
-
-// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
-// 128 bytes, 8-row groups 1024 bytes apart (SBO); LBO is unused for this
-// layout; bits 46..48 hold the fixed value 0b001; swizzle mode 2 = 128 B.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
-{
-    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                       uint32_t accumulate)
-{
-    asm volatile(
-        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-__device__ __forceinline__ void tc_commit(uint32_t bar)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(bar)
-                 : "memory");
-}
-
-// 32 consecutive FP32 columns of this warp's 32 TMEM lanes: thread i gets
-// lane (base lane + i), columns col .. col+31.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v)
-{
-    uint32_t r[32];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 
 // ------------------------------------------------------------- tile list
 
@@ -282,6 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         }
         if (lane == 0) tt.prefix[0] = 0;
     }
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -365,6 +268,8 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     } else if (warp >= 2) {
         // ------------------------------------------------ epilogue
         const int quarter = warp & 3;  // TMEM lanes this warp may access
+        const uint32_t out_base = sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * 2 * kOutBufBytes);
+        int out_parity = 0;
         int it = 0;
         for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
             const Tile t = decode_tile(p, tt, G, tile);
@@ -381,41 +286,57 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             const bool valid = r < t.rows;
             const int grow = t.row_base + t.m0 + r;
             const uint32_t taddr = tmem_base + (uint32_t)(buf * kAccCols) + ((uint32_t)(quarter * 32) << 16);
-            if (p.mode == kGateUp) {
-                const int ldc = t.shared ? p.E_sh * p.I : p.I;
-                bf16 *crow = (t.shared ? p.C_shared : p.C_routed) + (size_t)grow * ldc + t.n0;
+            // Whole 32-row blocks go out through shared memory and TMA stores;
+            // the block holding a tile's last rows is written row by row so that
+            // it never touches the next expert's rows.
+            const bool full_block = (t.rows - quarter * 32) >= 32;
+            const int ldc = p.mode == kGateUp ? (t.shared ? p.E_sh * p.I : p.I) : p.H;
+            bf16 *crow = (t.shared ? p.C_shared : p.C_routed) + (size_t)grow * ldc + t.n0;
+            const CUtensorMap *cmap = t.shared ? &maps.c_shared : &maps.c_routed;
+            const int nchunks = p.mode == kGateUp ? BM / 32 : p.bn / 32;
+            const float sc = (p.mode == kGateUp || t.shared) ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
 #pragma unroll 1
-                for (int c = 0; c < BM / 32; ++c) {
+            for (int c = 0; c < nchunks; ++c) {
+                uint32_t pk[16];
+                if (p.mode == kGateUp) {
                     float gv[32], uv[32];
                     tmem_ld32(taddr + c * 32, gv);
                     tmem_ld32(taddr + 128 + c * 32, uv);
                     tmem_ld_wait();
-                    uint32_t pk[16];
 #pragma unroll
                     for (int i = 0; i < 16; ++i)
                         pk[i] = pack_bf16x2(silu_mul(gv[2 * i], uv[2 * i]), silu_mul(gv[2 * i + 1], uv[2 * i + 1]));
-                    if (valid) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-                    }
-                }
-            } else {
-                bf16 *crow = (t.shared ? p.C_shared : p.C_routed) + (size_t)grow * p.H + t.n0;
-                const float sc = t.shared ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
-#pragma unroll 1
-                for (int c = 0; c < p.bn / 32; ++c) {
+                } else {
                     float v[32];
                     tmem_ld32(taddr + c * 32, v);
                     tmem_ld_wait();
-                    uint32_t pk[16];
 #pragma unroll
                     for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(v[2 * i] * sc, v[2 * i + 1] * sc);
-                    if (valid) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
+                }
+                if (full_block) {
+                    const uint32_t sbuf = out_base + (uint32_t)(out_parity * kOutBufBytes);
+                    if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+                    __syncwarp();
+                    // 64-byte rows, 16-byte chunk j of row r at chunk j ^ ((r >> 1) & 3): the
+                    // TMA 64-byte swizzle, and conflict-free for these 16-byte writes
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    for (int j = 0; j < 4; ++j) {
+                        const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[4 * j]),
+                                     "r"(pk[4 * j + 1]), "r"(pk[4 * j + 2]), "r"(pk[4 * j + 3])
+                                     : "memory");
                     }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(cmap, sbuf, t.n0 + c * 32, t.row_base + t.m0 + quarter * 32);
+                        bulk_commit();
+                    }
+                    out_parity ^= 1;
+                } else if (valid) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
                 }
             }
             tc_fence_before();
@@ -433,57 +354,22 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                     atomicAdd(p.shared_rows, (unsigned)__popc(vm));
             }
         }
+        if (lane == 0) bulk_wait_all();  // this warp's TMA stores are complete before the CTA exits
     }
 
+    // every warp reconverges before the block barrier: __syncthreads is a
+    // warp-aligned barrier, and the single-thread roles above diverge from
+    // their warps; TMEM is freed only after all epilogue reads completed
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
-        __syncwarp();
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(kTmemCols));
     }
 }
 
 // ------------------------------------------------------------ host side
-
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
-{
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    });
-    return fn;
-}
-
-// 2-D BF16 tensor map over a row-major [rows, cols] matrix, box = 64 x box_rows,
-// 128-byte swizzle, zero fill out of bounds.
-bool encode_2d(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_rows)
-{
-    auto fn = encode_fn();
-    if (!fn) return false;
-    const cuuint64_t dims[2] = {cols, rows};
-    const cuuint64_t strides[1] = {cols * 2};
-    const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
-    const cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-uint32_t make_idesc(int M, int N)
-{
-    return (1u << 4)                    // D: FP32
-           | (1u << 7)                  // A: BF16
-           | (1u << 10)                 // B: BF16
-           | ((uint32_t)(N >> 3) << 17) // N / 8
-           | ((uint32_t)(M >> 4) << 24);// M / 16   (A and B K-major: transpose bits 15, 16 = 0)
-}
 
 cudaError_t launch_tc(const Ctx &c, int mode)
 {
@@ -509,6 +395,10 @@ cudaError_t launch_tc(const Ctx &c, int mode)
         p.tx_bytes = kABytes + 2 * 128 * BK * 2;
         p.C_routed = c.act;
         p.C_shared = c.act_sh;
+        ok &= encode_2d_box(&maps.c_routed, c.act, s.I, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        if (s.E_sh > 0)
+            ok &= encode_2d_box(&maps.c_shared, c.act_sh, (uint64_t)s.E_sh * s.I, T, kOutBox, kOutBox,
+                                CU_TENSOR_MAP_SWIZZLE_64B);
         ok &= encode_2d(&maps.a_routed, c.a_perm, s.H, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.I;
@@ -526,6 +416,9 @@ cudaError_t launch_tc(const Ctx &c, int mode)
         p.tx_bytes = kABytes + p.bn * BK * 2;
         p.C_routed = c.y;
         p.C_shared = c.y_sh;
+        ok &= encode_2d_box(&maps.c_routed, c.y, s.H, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        if (s.E_sh > 0)
+            ok &= encode_2d_box(&maps.c_shared, c.y_sh, s.H, T, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
         ok &= encode_2d(&maps.a_routed, c.act, s.I, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
@@ -544,6 +437,51 @@ cudaError_t launch_tc(const Ctx &c, int mode)
 }
 
 }  // namespace
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    });
+    return fn;
+}
+
+// 2-D BF16 tensor map over a row-major [rows, cols] matrix, box = 64 x box_rows,
+// 128-byte swizzle, zero fill out of bounds.
+bool encode_2d_box(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
+                   uint32_t box_rows, CUtensorMapSwizzle swizzle)
+{
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * 2};
+    const cuuint32_t box[2] = {box_cols, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_2d(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_rows)
+{
+    return encode_2d_box(m, ptr, cols, rows, 64u, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+uint32_t make_idesc(int M, int N)
+{
+    return (1u << 4)                    // D: FP32
+           | (1u << 7)                  // A: BF16
+           | (1u << 10)                 // B: BF16
+           | ((uint32_t)(N >> 3) << 17) // N / 8
+           | ((uint32_t)(M >> 4) << 24);// M / 16   (A and B K-major: transpose bits 15, 16 = 0)
+}
 
 cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, kGateUp); }
 cudaError_t launch_down(const Ctx &c) { return launch_tc(c, kDown); }

@@ -1,223 +1,380 @@
 // Stage 1 of the layer: fail-closed policy resolve, masked router, top-k and
 // the route log (Sec. 3.1 Eq. 4; App. B.1 steps 2, 4, 5).
 //
-// One CTA owns 32 consecutive tokens.  It resolves their policy bytes, then
-// packs the rows pool by pool: DENY rows first, padded to a multiple of 16,
-// then ALLOW rows.  Every 16-row MMA group therefore belongs to one pool and
-// multiplies only that pool's router rows -- the other pool's router weights
-// are never read for it, so an ineligible expert never becomes a candidate.
-// Logits are BF16 x BF16 -> FP32 on mma.sync tensor-core tiles (this GEMM is
-// about 0.4 % of the layer's FLOPs), staged through shared memory, and each
-// warp then selects the top-k of one token with warp shuffles.
+// router_tc_kernel: each CTA owns one 128-token tile of ONE pool.  It first
+// resolves the policy bytes itself (only the trusted byte 0x01 is ALLOW) and
+// ranks the tokens inside their pool, so that the DENY tokens form tiles
+// 0 .. ceil(n_deny/128)-1 and the ALLOW tokens the tiles after them, each in
+// ascending token order.  A TMA ring streams the tile's token rows and the
+// pool's router rows as 128-byte-swizzled tiles into shared memory: straight
+// from `hidden` when the tile's tokens are consecutive, otherwise from a
+// contiguous workspace block the CTA first fills by token index (row gathers
+// through TMA gather4 or cp.async ran 2.5-5x slower than copy + tile loads).
+// tcgen05.mma computes the 128 x E_pool logits in tensor memory.  A DENY row
+// is therefore only ever multiplied by public router rows and an ALLOW row
+// only by private ones: an ineligible expert never becomes a candidate.
+// Sixteen epilogue warps read the logits: four threads per token (one TMEM
+// lane, four column slices) each select the top-k of their slice (descending
+// score, ties to the lower expert id) by ordered passes with four independent
+// selection chains, and one thread per token merges the four sorted lists and
+// writes the softmax weights and the route log.
+#include <cuda.h>
+
 #include "pmpe_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace pmpe {
 namespace {
 
-constexpr int kTok = 32;               // tokens per CTA
-constexpr int kRows = 48;              // DENY rows padded to 16 + ALLOW rows <= 32 + 15
-constexpr int kWarps = 6;              // 3 row groups x 2 expert halves
-constexpr int kThreads = kWarps * 32;
-constexpr int kBK = 64;                // K elements per pipeline stage (128 bytes per row)
-constexpr int kStages = 3;
-constexpr int kMaxTiles = kMaxPool / 8 / 2;  // n8 tiles per warp
-constexpr int kLdl = kMaxPool + 1;           // logits row stride (floats)
+constexpr int kEpiWarps = 16;    // 4 per TMEM lane quarter, each on a quarter of the logit columns
+constexpr int kRThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2..17 epilogue
+constexpr int kRMaxStages = 8;
+constexpr int kTileRows = 128;
+constexpr int kABytes = kTileRows * 128;  // 128 rows x 64 BF16
 
-struct RouteParams {
-    const bf16 *hidden;
-    const uint8_t *policy;
-    const bf16 *wr[2];  // [0] public router [E_pub, H], [1] private router [E_priv, H]
+struct RouterParams {
     int T, H, E_pub, E_priv, k, renorm;
-    int pad[2];         // pool sizes rounded up to 16
+    int n_pad[2];        // MMA N of each pool: pool size rounded up to 16 (>= 16)
+    uint32_t idesc[2];
+    uint32_t tmem_cols;  // power of two >= max n_pad
+    int stages;
+    uint32_t stage_bytes;
+    const uint8_t *policy;
+    const bf16 *hidden;
+    bf16 *rows_ws;       // [grid * 128, H] tile rows in pool order (workspace)
     uint8_t *tau;
     int32_t *idx;
     float *w;
-    uint32_t *counts;
-    uint32_t *route_count, *route_priv_rows;  // audit words, may be NULL
+    uint32_t *route_count, *route_priv_rows, *status;
 };
 
-__device__ __forceinline__ void ldmatrix_x2(uint32_t &r0, uint32_t &r1, uint32_t addr)
+struct RouterMaps {
+    CUtensorMap hidden;     // [T, H], box 64 x 128 (tiles of consecutive tokens)
+    CUtensorMap rows;       // rows_ws, box 64 x 128 (copied tiles)
+    CUtensorMap router[2];  // [E_pool, H], box 64 x n_pad
+};
+
+// Exclusive scan over the block of one int per thread (kRThreads threads).
+__device__ __forceinline__ int block_scan(int v, int *warp_tot, int &total)
 {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];\n" : "=r"(r0), "=r"(r1) : "r"(addr));
-}
-
-__global__ void __launch_bounds__(kThreads) router_topk_kernel(const RouteParams p)
-{
-    extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ int row_tok[kRows];  // token of each packed row, -1 = padding
-    __shared__ int s_pd, s_na, s_nd;
-
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int t0 = blockIdx.x * kTok;
-    const int ntok = min(kTok, p.T - t0);
-
-    // ---- resolve (only the trusted byte 0x01 is ALLOW) and pack rows by pool
-    if (warp == 0) {
-        const int t = t0 + lane;
-        const bool valid = lane < ntok;
-        const bool allow = valid && p.policy != nullptr && p.policy[t] == 0x01;
-        const unsigned am = __ballot_sync(~0u, allow);
-        const unsigned dm = __ballot_sync(~0u, valid && !allow);
-        const int nd = __popc(dm), na = __popc(am);
-        const int pd = (nd + 15) & ~15;
-        const unsigned below = (1u << lane) - 1u;
-        for (int r = lane; r < kRows; r += 32) row_tok[r] = -1;
-        __syncwarp();
-        if (valid) {
-            row_tok[allow ? pd + __popc(am & below) : __popc(dm & below)] = t;
-            p.tau[t] = allow ? 1 : 0;
-        }
-        if (lane == 0) { s_pd = pd; s_na = na; s_nd = nd; }
+    constexpr int kW = kRThreads / 32;  // 18
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(~0u, x, off);
+        if (lane >= off) x += y;
+    }
+    if (lane == 31) warp_tot[warp] = x;
+    __syncthreads();
+    int before = 0;
+    total = 0;
+#pragma unroll
+    for (int i = 0; i < kW; ++i) {
+        const int t = warp_tot[i];
+        before += i < warp ? t : 0;
+        total += t;
     }
     __syncthreads();
-    const int pd = s_pd, na = s_na;
-    const bool need[2] = {s_nd > 0, na > 0};
-    const int stage_bytes = (kRows + p.pad[0] + p.pad[1]) * 128;
+    return before + x - v;
+}
 
-    // ---- warp role: row group g (16 rows, one pool), expert half
-    const int g = warp >> 1, half = warp & 1;
-    const int pool = (16 * g < pd) ? 0 : 1;
-    const bool active = 16 * g < pd + na;
-    const int P = pool ? p.E_priv : p.E_pub;
-    const int ntp = (P + 7) >> 3;
-    const int h0 = (ntp + 1) >> 1;
-    const int tile0 = half ? h0 : 0;
-    const int mt = half ? ntp - h0 : h0;
+__device__ __forceinline__ bool is_allow(const uint8_t *policy, int t)
+{
+    return policy != nullptr && policy[t] == 0x01;
+}
 
-    auto load_stage = [&](int st, int kb) {
-        const uint32_t sA = smem_u32(smem + st * stage_bytes);
-        const int kofs = kb * kBK;
-        for (int i = tid; i < kRows * 8; i += kThreads) {
-            const int r = i >> 3, c = i & 7, t = row_tok[r];
-            const bf16 *src = p.hidden + (size_t)(t < 0 ? 0 : t) * p.H + kofs + c * 8;
-            cp_async16(sA + swz128(r, c), src, t < 0 ? 0 : 16);
+// (x, e) ranks above (bx, be): larger logit, or equal logit and lower id.
+__device__ __forceinline__ bool ranks_above(float x, int e, float bx, int be)
+{
+    return x > bx || (x == bx && e < be);
+}
+
+__global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterParams p,
+                                                                  const __grid_constant__ RouterMaps maps)
+{
+    extern __shared__ uint8_t dsmem[];
+    __shared__ int s_tok[kTileRows];
+    __shared__ int warp_tot[kRThreads / 32];
+    __shared__ __align__(8) uint64_t bars[2 * kRMaxStages + 2];
+    __shared__ uint32_t s_tmem;
+    __shared__ volatile int s_abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    // ---- resolve and rank: pass 1 counts the ALLOW tokens
+    int my_allow = 0;
+    for (int t = tid; t < p.T; t += kRThreads) my_allow += is_allow(p.policy, t);
+    int na_total;
+    block_scan(my_allow, warp_tot, na_total);
+    const int na = na_total, nd = p.T - na;
+    const int tiles_d = (nd + kTileRows - 1) / kTileRows;
+    int pool, m0;
+    if ((int)blockIdx.x < tiles_d) {
+        pool = 0;
+        m0 = blockIdx.x * kTileRows;
+    } else {
+        pool = 1;
+        m0 = (blockIdx.x - tiles_d) * kTileRows;
+        if (m0 >= na) return;  // uniform: no tile for this CTA
+    }
+    const int rows = min(kTileRows, (pool ? na : nd) - m0);
+    // pass 2: each thread takes a contiguous run of tokens, ranks them in
+    // their pool, and keeps the ones that fall into this CTA's tile
+    {
+        const int per = (p.T + kRThreads - 1) / kRThreads;
+        const int t0 = tid * per, t1 = min(p.T, t0 + per);
+        int a = 0;
+        for (int t = t0; t < t1; ++t) a += is_allow(p.policy, t);
+        int dummy;
+        const int a_before = block_scan(a, warp_tot, dummy);
+        int ra = a_before, rd = t0 - a_before;  // ranks inside the ALLOW / DENY pools
+        for (int t = t0; t < t1; ++t) {
+            const bool al = is_allow(p.policy, t);
+            const int rank = al ? ra++ : rd++;
+            if ((al ? 1 : 0) == pool && rank >= m0 && rank < m0 + rows) {
+                s_tok[rank - m0] = t;
+                p.tau[t] = al ? 1 : 0;  // every token is written by exactly one CTA
+            }
         }
-        uint32_t sB = sA + kRows * 128;
-        for (int q = 0; q < 2; ++q) {
-            const int E = q ? p.E_priv : p.E_pub;
-            if (need[q]) {
-                for (int i = tid; i < p.pad[q] * 8; i += kThreads) {
-                    const int r = i >> 3, c = i & 7;
-                    const bf16 *src = p.wr[q] + (size_t)min(r, E - 1) * p.H + kofs + c * 8;
-                    cp_async16(sB + swz128(r, c), src, r < E ? 16 : 0);
+    }
+    __syncthreads();
+    for (int r = rows + tid; r < kTileRows; r += kRThreads) s_tok[r] = s_tok[0];  // padding rows name a real token
+    // The TMA ring reads the tile's rows as one 128-row tile.  When the tile's
+    // tokens are consecutive (a request with one policy) that tile is read
+    // from `hidden` directly; otherwise the CTA first copies its token rows
+    // into a contiguous block (padding rows are not copied: their logits are
+    // never read) and makes the generic-proxy writes visible to the async
+    // proxy of the TMA reads.
+    const int contiguous = __syncthreads_and(tid >= rows || s_tok[tid < kTileRows ? tid : 0] == s_tok[0] + tid);
+    if (!contiguous) {
+        constexpr int kBatch = 16;  // independent 16-byte loads in flight per thread
+        const int nv = p.H / 8;
+        const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden);
+        uint4 *dst = reinterpret_cast<uint4 *>(p.rows_ws) + (size_t)blockIdx.x * kTileRows * nv;
+        const int total = rows * nv;
+        for (int i0 = tid; i0 < total; i0 += kBatch * kRThreads) {
+            uint4 v[kBatch];
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                const int q = i0 + u * kRThreads;
+                if (q < total) {
+                    const int r = q / nv;
+                    v[u] = __ldg(src + (size_t)s_tok[r] * nv + (q - r * nv));
                 }
             }
-            sB += p.pad[q] * 128;
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u)
+                if (i0 + u * kRThreads < total) dst[i0 + u * kRThreads] = v[u];
         }
-    };
-
-    float acc[kMaxTiles][4];
-#pragma unroll
-    for (int i = 0; i < kMaxTiles; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-
-    const int nkb = p.H / kBK;
-#pragma unroll
-    for (int s = 0; s < kStages - 1; ++s) {
-        if (s < nkb) load_stage(s, s);
-        cp_async_commit();
+        asm volatile("fence.proxy.async.global;\n" ::: "memory");
     }
-    for (int kb = 0; kb < nkb; ++kb) {
-        cp_async_wait<kStages - 2>();
-        __syncthreads();
-        const int nk = kb + kStages - 1;
-        if (nk < nkb) load_stage(nk % kStages, nk);
-        cp_async_commit();
-        if (active && mt > 0) {
-            const uint32_t sA = smem_u32(smem + (kb % kStages) * stage_bytes);
-            const uint32_t sB = sA + kRows * 128 + (pool ? p.pad[0] * 128 : 0);
+    const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (kRMaxStages + s); };
+    const uint32_t tfull_bar = bar0 + 8u * (2 * kRMaxStages);
+    const uint32_t done_bar = bar0 + 8u * (2 * kRMaxStages + 1);
+    if (tid == 0) {
+        for (int s = 0; s < p.stages; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
+        mbar_init(tfull_bar, 1);
+        mbar_init(done_bar, 1);
+        s_abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == 1) tmem_alloc(smem_u32(&s_tmem), p.tmem_cols);
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    const int N = p.n_pad[pool];
+    const int nkb = p.H / 64;
+
+    if (warp == 0 && lane == 0) {
+        // ---- TMA producer: 128 tile rows + the pool's router rows per stage
+        int stage = 0;
+        uint32_t phase = 0, filled = 0, last_parity = 0;
+        const uint32_t tx = (uint32_t)kABytes + (uint32_t)N * 128u;
+        for (int kb = 0; kb < nkb; ++kb) {
+            if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) break;
+            const uint32_t sA = sbase + stage * p.stage_bytes, sB = sA + kABytes;
+            mbar_expect_tx(full_bar(stage), tx);
+            if (contiguous)
+                tma_load_2d(sA, &maps.hidden, full_bar(stage), kb * 64, s_tok[0]);
+            else
+                tma_load_2d(sA, &maps.rows, full_bar(stage), kb * 64, blockIdx.x * kTileRows);
+            tma_load_2d(sB, &maps.router[pool], full_bar(stage), kb * 64, 0);
+            filled |= 1u << stage;
+            last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+            if (++stage == p.stages) { stage = 0; phase ^= 1u; }
+        }
+        // every copy this thread issued has landed before the CTA exits
+        for (int s = 0; s < p.stages; ++s)
+            if ((filled >> s) & 1u) {
+                const unsigned long long t0 = globaltimer_ns();
+                while (!mbar_try_wait(full_bar(s), (last_parity >> s) & 1u))
+                    if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+            }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer: logits[128, N] += rows[128, 64] x router[N, 64]^T per stage
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb) {
+            if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t sA = sbase + stage * p.stage_bytes, sB = sA + kABytes;
+            const uint64_t ad = sw128_desc(sA), bd = sw128_desc(sB);
 #pragma unroll
-            for (int ks = 0; ks < kBK / 16; ++ks) {
-                uint32_t a[4];
-                ldmatrix_x4(a[0], a[1], a[2], a[3], sA + swz128(16 * g + (lane & 15), ks * 2 + (lane >> 4)));
+            for (int k = 0; k < 4; ++k) tc_mma(tmem, ad + 2 * k, bd + 2 * k, p.idesc[pool], (kb | k) != 0);
+            tc_commit(empty_bar(stage));
+            if (++stage == p.stages) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) tc_commit(tfull_bar);
+        tc_commit(done_bar);
+        const unsigned long long t0 = globaltimer_ns();
+        while (!mbar_try_wait(done_bar, 0))
+            if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    } else if (warp >= 2) {
+        // ---- epilogue.  Thread (quarter q, slice sl) owns TMEM lane 32q + lane
+        // (one token) and the logit columns of chunks sl, sl+4, ... (32 each);
+        // it selects the top-k of its columns, then one thread per token merges
+        // the four sorted slice lists.
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait(tfull_bar, 0, &s_abort, p.status) ? 1 : 0;
+        ok = __shfl_sync(~0u, ok, 0);
+        const int q = warp & 3, sl = (warp - 2) >> 2;
+        const int r = q * 32 + lane;
+        const int P = pool ? p.E_priv : p.E_pub;
+        const int base = pool ? p.E_pub : 0;
+        float *lv = reinterpret_cast<float *>(dsmem + (sbase - smem_u32(dsmem)));  // [128][4][k] values
+        int *li = reinterpret_cast<int *>(lv + kTileRows * 4 * p.k);               // [128][4][k] ids
+        float *lmax = reinterpret_cast<float *>(li + kTileRows * 4 * p.k);          // [128][4]
+        float *lsum = lmax + kTileRows * 4;                                          // [128][4]
+        int *lcnt = reinterpret_cast<int *>(lsum + kTileRows * 4);                   // [128][4]
+        if (ok) {
+            __syncwarp();
+            tc_fence_after();
+            const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16);
+            const int nch = (N + 31) / 32;
+            const int my_cols = (sl < nch) ? min(P, N) : 0;  // any columns at all in this slice?
+            int cnt = 0;
+            float pv = 0.f, mx = -INFINITY;
+            int pe = -1;
+            const int slot = (r * 4 + sl) * p.k;
+            for (int j = 0; j < p.k; ++j) {
+                float bv = -INFINITY;
+                int be = 0x7fffffff;
+                for (int ch = sl; ch < nch; ch += 4) {
+                    const int c0 = ch * 32;
+                    float v[32];
+                    tmem_ld32(taddr + c0, v);
+                    tmem_ld_wait();
+                    float cb[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    int ce[4] = {0x7fffffff, 0x7fffffff, 0x7fffffff, 0x7fffffff};
 #pragma unroll
-                for (int nt = 0; nt < kMaxTiles; ++nt) {
-                    if (nt < mt) {
-                        uint32_t b0, b1;
-                        ldmatrix_x2(b0, b1, sB + swz128((tile0 + nt) * 8 + (lane & 7), ks * 2 + ((lane >> 3) & 1)));
-                        mma_bf16_16816(acc[nt], a, b0, b1);
+                    for (int i = 0; i < 32; ++i) {
+                        const int e = c0 + i, u = i & 3;
+                        float x = v[i];
+                        if (x != x) x = -INFINITY;  // NaN never outranks a number
+                        const bool after = (j == 0) || (x < pv) || (x == pv && e > pe);
+                        if (e < P && after && (ce[u] == 0x7fffffff || x > cb[u])) { cb[u] = x; ce[u] = e; }
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (ce[u] != 0x7fffffff && (be == 0x7fffffff || ranks_above(cb[u], ce[u], bv, be))) {
+                            bv = cb[u];
+                            be = ce[u];
+                        }
+                }
+                if (be == 0x7fffffff) break;  // this slice has no further column
+                lv[slot + j] = bv;
+                li[slot + j] = be;
+                pv = bv;
+                pe = be;
+                if (cnt == 0) mx = bv;
+                ++cnt;
+            }
+            // pool-softmax partial of this slice: sum of exp(x - slice max)
+            float ssum = 0.f;
+            if (!p.renorm && cnt > 0) {
+                for (int ch = sl; ch < nch; ch += 4) {
+                    const int c0 = ch * 32;
+                    float v[32];
+                    tmem_ld32(taddr + c0, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        float x = v[i];
+                        if (x != x) x = -INFINITY;
+                        if (c0 + i < P) ssum += expf(x - mx);
                     }
                 }
             }
+            (void)my_cols;
+            lcnt[r * 4 + sl] = cnt;
+            lmax[r * 4 + sl] = mx;
+            lsum[r * 4 + sl] = ssum;
         }
-    }
-    cp_async_wait<0>();
-    __syncthreads();
-
-    // ---- logits to shared memory (reusing the pipeline buffers)
-    float *lg = reinterpret_cast<float *>(smem);
-    if (active) {
+        // all 16 epilogue warps: slice lists complete before the merge
+        asm volatile("bar.sync 1, %0;\n" ::"r"(32 * kEpiWarps) : "memory");
+        if (ok && sl == 0) {
+            const bool valid = r < rows;
+            const int t = s_tok[r];
+            int head[4], n[4];
 #pragma unroll
-        for (int nt = 0; nt < kMaxTiles; ++nt) {
-            if (nt < mt) {
-                const int e = (tile0 + nt) * 8 + 2 * (lane & 3);
-                const int r = 16 * g + (lane >> 2);
-                if (e < P) { lg[r * kLdl + e] = acc[nt][0]; lg[(r + 8) * kLdl + e] = acc[nt][2]; }
-                if (e + 1 < P) { lg[r * kLdl + e + 1] = acc[nt][1]; lg[(r + 8) * kLdl + e + 1] = acc[nt][3]; }
-            }
-        }
-    }
-    __syncthreads();
-
-    // ---- top-k per token: one warp per packed row
-    for (int r = warp; r < kRows; r += kWarps) {
-        const int t = row_tok[r];
-        if (t < 0) continue;
-        const int q = r < pd ? 0 : 1;
-        const int Pq = q ? p.E_priv : p.E_pub;
-        const int base = q ? p.E_pub : 0;
-        float v[kMaxPool / 32];
-        unsigned avail = 0;
+            for (int u = 0; u < 4; ++u) { head[u] = 0; n[u] = lcnt[r * 4 + u]; }
+            float sel_v[kMaxTopK];
+            float top = 0.f;
+            int npriv = 0;
+            for (int j = 0; j < p.k; ++j) {
+                int bu = -1;
+                float bv = 0.f;
+                int be = 0;
 #pragma unroll
-        for (int i = 0; i < kMaxPool / 32; ++i) {
-            const int e = lane + 32 * i;
-            float x = -INFINITY;
-            if (e < Pq) {
-                x = lg[r * kLdl + e];
-                if (x != x) x = -INFINITY;  // NaN never outranks a number
-                avail |= 1u << i;
-            }
-            v[i] = x;
-        }
-        float my_v = -INFINITY, top = -INFINITY;
-        int my_e = 0;
-        for (int j = 0; j < p.k; ++j) {
-            float bv = -INFINITY;
-            int be = 0x7fffffff;
-#pragma unroll
-            for (int i = 0; i < kMaxPool / 32; ++i)
-                if ((avail >> i) & 1u) {
-                    if (be == 0x7fffffff || v[i] > bv) { bv = v[i]; be = lane + 32 * i; }
+                for (int u = 0; u < 4; ++u) {
+                    if (head[u] < n[u]) {
+                        const float x = lv[(r * 4 + u) * p.k + head[u]];
+                        const int e = li[(r * 4 + u) * p.k + head[u]];
+                        if (bu < 0 || ranks_above(x, e, bv, be)) { bu = u; bv = x; be = e; }
+                    }
                 }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-                const float ov = __shfl_xor_sync(~0u, bv, off);
-                const int oe = __shfl_xor_sync(~0u, be, off);
-                if (ov > bv || (ov == bv && oe < be)) { bv = ov; be = oe; }
+                if (bu < 0) break;  // unreachable for k <= pool size
+                head[bu] += 1;
+                sel_v[j] = bv;
+                if (j == 0) top = bv;
+                const int gid = base + be;
+                npriv += gid >= p.E_pub;
+                if (valid) {
+                    p.idx[(size_t)t * p.k + j] = gid;
+                    if (p.route_count) atomicAdd(&p.route_count[gid], 1u);
+                }
             }
-            if ((be & 31) == lane) avail &= ~(1u << (be >> 5));
-            if (lane == j) { my_v = bv; my_e = be; }
-            if (j == 0) top = bv;
-        }
-        // softmax weights
-        float denom = 0.f;
-        if (p.renorm) {
-            denom = lane < p.k ? expf(my_v - top) : 0.f;
-        } else {
+            float S = 0.f;
+            if (p.renorm) {
+                for (int j = 0; j < p.k; ++j) S += expf(sel_v[j] - top);
+            } else {
 #pragma unroll
-            for (int i = 0; i < kMaxPool / 32; ++i)
-                if (lane + 32 * i < Pq) denom += expf(v[i] - top);
+                for (int u = 0; u < 4; ++u)  // fixed order: deterministic
+                    if (n[u] > 0) S += lsum[r * 4 + u] * expf(lmax[r * 4 + u] - top);
+            }
+            if (valid) {
+                for (int j = 0; j < p.k; ++j) p.w[(size_t)t * p.k + j] = expf(sel_v[j] - top) / S;
+                if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], (unsigned)npriv);
+            }
         }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) denom += __shfl_xor_sync(~0u, denom, off);
-        const int gid = base + my_e;
-        const unsigned privm = __ballot_sync(~0u, lane < p.k && gid >= p.E_pub);
-        if (lane < p.k) {
-            p.idx[(size_t)t * p.k + lane] = gid;
-            p.w[(size_t)t * p.k + lane] = expf(my_v - top) / denom;
-            atomicAdd(&p.counts[gid], 1u);
-            if (p.route_count) atomicAdd(&p.route_count[gid], 1u);
-        }
-        if (lane == 0 && p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], (unsigned)__popc(privm));
+    }
+
+    // every warp reconverges before the block barrier: __syncthreads is a
+    // warp-aligned barrier, and the single-thread roles above diverge from
+    // their warps; TMEM is freed only after all epilogue reads completed
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, p.tmem_cols);
     }
 }
 
@@ -232,26 +389,46 @@ __global__ void resolve_kernel(const uint8_t *policy, int T, uint8_t *tau)
 cudaError_t launch_route(const Ctx &c)
 {
     const Shape &s = c.s;
-    cudaError_t err = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
-    if (err != cudaSuccess) return err;
-    RouteParams p;
-    p.hidden = c.hidden;
-    p.policy = c.policy;
-    p.wr[0] = c.router_pub;
-    p.wr[1] = c.router_priv;
+    RouterParams p;
+    RouterMaps maps;
+    memset(&maps, 0, sizeof(maps));
     p.T = s.T; p.H = s.H; p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.k = s.k; p.renorm = s.renorm;
-    p.pad[0] = (s.E_pub + 15) & ~15;
-    p.pad[1] = (s.E_priv + 15) & ~15;
-    p.tau = c.tau; p.idx = c.idx; p.w = c.w; p.counts = c.counts;
+    int nmax = 0;
+    for (int q = 0; q < 2; ++q) {
+        const int P = q ? s.E_priv : s.E_pub;
+        p.n_pad[q] = ((P < 16 ? 16 : P) + 15) & ~15;
+        p.idesc[q] = make_idesc(kTileRows, p.n_pad[q]);
+        nmax = p.n_pad[q] > nmax ? p.n_pad[q] : nmax;
+    }
+    p.tmem_cols = 32;
+    while ((int)p.tmem_cols < nmax) p.tmem_cols <<= 1;
+    p.stage_bytes = (uint32_t)(kABytes + nmax * 128);
+    p.stages = (int)((200u * 1024u) / p.stage_bytes);
+    if (p.stages > kRMaxStages) p.stages = kRMaxStages;
+    p.policy = c.policy;
+    p.hidden = c.hidden;
+    p.rows_ws = c.router_rows;
+    p.tau = c.tau;
+    p.idx = c.idx;
+    p.w = c.w;
     p.route_count = c.audit.route_count;
     p.route_priv_rows = c.audit.route_priv_rows;
-    const int pipe = kStages * (kRows + p.pad[0] + p.pad[1]) * 128;
-    const int logits = kRows * kLdl * (int)sizeof(float);
-    const int smem = pipe > logits ? pipe : logits;
-    err = cudaFuncSetAttribute(router_topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    p.status = c.audit.status;
+    const int grid = (s.T + kTileRows - 1) / kTileRows + 1;
+    bool ok = encode_2d(&maps.rows, c.router_rows, s.H, (uint64_t)grid * kTileRows, kTileRows);
+    ok &= encode_2d(&maps.hidden, c.hidden, s.H, s.T, kTileRows);
+    ok &= encode_2d(&maps.router[0], c.router_pub, s.H, s.E_pub, p.n_pad[0]);
+    ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, p.n_pad[1]);
+    if (!ok) return cudaErrorInvalidValue;
+    // at least 116 KB of shared memory keeps one router CTA per SM, so the
+    // TMEM allocation never waits for another CTA
+    int smem = p.stages * (int)p.stage_bytes + 1024;
+    if (smem < 116 * 1024) smem = 116 * 1024;
+    const int lists = kTileRows * 4 * (s.k * 8 + 12) + 1024;  // top-k slice lists, reused after the MMAs
+    if (smem < lists) smem = lists;
+    cudaError_t err = cudaFuncSetAttribute(router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (err != cudaSuccess) return err;
-    const int grid = (s.T + kTok - 1) / kTok;
-    router_topk_kernel<<<grid, kThreads, smem, c.stream>>>(p);
+    router_tc_kernel<<<grid, kRThreads, smem, c.stream>>>(p, maps);
     return cudaGetLastError();
 }
 

@@ -35,6 +35,7 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     L->slot_of = take(4 * R, 256);
     L->tok_of_slot = take(4 * R, 256);
     L->w_of_slot = take(4 * R, 256);
+    L->router_rows = take(2 * ((T + 127) / 128 + 1) * 128 * (size_t)s.H, 1024);
     L->a_perm = take(2 * R * s.H, 1024);
     L->act = take(2 * R * s.I, 1024);
     L->y = take(2 * R * s.H, 1024);
@@ -113,6 +114,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->slot_of = (int32_t *)(ws + L.slot_of);
     c->tok_of_slot = (int32_t *)(ws + L.tok_of_slot);
     c->w_of_slot = (float *)(ws + L.w_of_slot);
+    c->router_rows = (bf16 *)(ws + L.router_rows);
     c->a_perm = (bf16 *)(ws + L.a_perm);
     c->act = (bf16 *)(ws + L.act);
     c->y = (bf16 *)(ws + L.y);

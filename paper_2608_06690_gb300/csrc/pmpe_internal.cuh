@@ -47,6 +47,7 @@ struct Ctx {
     uint32_t *counts, *offsets;
     int32_t *slot_of, *tok_of_slot;
     float *w_of_slot;
+    bf16 *router_rows;  // [(ceil(T/128)+1)*128, H] router tiles' token rows
     bf16 *a_perm, *act, *y, *act_sh, *y_sh;
     cudaStream_t stream;
     int num_sms;
@@ -106,6 +107,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
     return *reinterpret_cast<uint32_t *>(&v);
 }
 
-__device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + __expf(-g)) * u; }
+// silu(g) * u with the fast reciprocal-based division (for g -> -inf the
+// denominator overflows to +inf and the quotient is 0, the correct limit).
+__device__ __forceinline__ float silu_mul(float g, float u) { return __fdividef(g, 1.0f + __expf(-g)) * u; }
 
 }  // namespace pmpe
