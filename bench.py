@@ -33,12 +33,34 @@ from paper_2608_06690_gb300.configs import CONFIGS  # noqa: E402
 METRIC = "MoE-layer tokens/s (mixed allow/deny)"
 L2_FLUSH_BYTES = 512 << 20   # > 129 MB L2
 
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
+# grouped GEMM kernels, from one ncu capture of the current kernels on the
+# named workload; None where no capture of the current kernels exists.
+NCU_TRAFFIC = {
+    "qwen3_prefill": {"gateup": 1.146401e9 + 44.646912e6, "down": 0.553858e9 + 103.074048e6},
+}
+
 
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return ws, rank, local
+
+
+def max_over_ranks(x: float, device) -> float:
+    """Maximum of a per-rank float over all ranks (identity without a process
+    group); `device` is where the reduction tensor lives (cuda for NCCL, cpu
+    for gloo)."""
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    if torch.distributed.is_available() and torch.distributed.is_initialized():
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, n_ranks: int, slowest_s: float) -> float:
+    """Units processed by all ranks divided by the slowest rank's time."""
+    return n_ranks * units_per_rank / slowest_s
 
 
 def _peaks():
@@ -235,11 +257,8 @@ def run_ours(args):
     t_wall = time.perf_counter() - t_wall0
     barrier()
     step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
-    total_ms = torch.tensor([sum(step_ms)], dtype=torch.float64, device=dev)
-    if ws > 1:
-        torch.distributed.all_reduce(total_ms, op=torch.distributed.ReduceOp.MAX)
-    total_ms = float(total_ms.item())
-    value = ws * s.T * args.steps / (total_ms / 1e3)
+    total_ms = max_over_ranks(sum(step_ms), dev)
+    value = whole_job_rate(s.T * args.steps, ws, total_ms / 1e3)
 
     # ---- per-stage breakdown: each stage after its own L2 flush, so the GPU
     # is still busy flushing while the host enqueues the stage (no host gap
@@ -287,11 +306,8 @@ def run_ours(args):
         if i >= max(args.warmup, 3):
             e2e_ev[i - max(args.warmup, 3)][1].record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = sum(e0.elapsed_time(e1) for e0, e1 in e2e_ev)
-    e2e_t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-    if ws > 1:
-        torch.distributed.all_reduce(e2e_t, op=torch.distributed.ReduceOp.MAX)
-    e2e_value = ws * s.T * args.steps / (float(e2e_t.item()) / 1e3)
+    e2e_ms = max_over_ranks(sum(e0.elapsed_time(e1) for e0, e1 in e2e_ev), dev)
+    e2e_value = whole_job_rate(s.T * args.steps, ws, e2e_ms / 1e3)
     clk.__exit__(None, None, None)
 
     if rank != 0:
@@ -311,7 +327,7 @@ def run_ours(args):
         achieved = work[f"bytes_{dominant}"] / (stage_avg[dominant] / 1e3) / 1e9
         roof = {"kernel": dominant, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": achieved / hbm, "peak_source": f"{peak_src} HBM copy"}
-    roof["traffic"] = args.traffic
+    roof["traffic"] = args.traffic if args.traffic is not None else NCU_TRAFFIC.get(cfg.name, {}).get(dominant)
     stage_report = {}
     for n, ms in stage_avg.items():
         d = {"ms": ms}

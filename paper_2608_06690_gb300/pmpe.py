@@ -187,24 +187,33 @@ def forward_desc(desc: MoeDesc, stages: int = STAGE_ALL, stream=None):
     _check(rc, "pmpe_moe_forward")
 
 
+class Workspace:
+    """A device scratch buffer that grows on demand; layers that run one after
+    another on the same stream can share one."""
+
+    def __init__(self, device="cuda"):
+        self.device = torch.device(device)
+        self._buf = None
+
+    def get(self, nbytes: int) -> torch.Tensor:
+        if self._buf is None or self._buf.numel() < nbytes:
+            self._buf = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=self.device)
+        return self._buf
+
+
 class MoeLayer:
     """One policy-masked MoE layer with its weights resident on the GPU and
     a reusable workspace.  ``forward`` enqueues the C-ABI call on the
     current stream and returns the output tensor."""
 
-    def __init__(self, shape: LayerShape, weights: dict, device="cuda"):
+    def __init__(self, shape: LayerShape, weights: dict, device="cuda", workspace: "Workspace | None" = None):
         self.shape = shape
         self.weights = weights
         self.device = torch.device(device)
-        self._ws = None
-        self._ws_T = -1
+        self._ws = workspace if workspace is not None else Workspace(self.device)
 
     def workspace(self, T: int) -> torch.Tensor:
-        if self._ws is None or self._ws_T < T:
-            s = self._shape_T(T)
-            self._ws = torch.empty(max(workspace_size(s), 1), dtype=torch.uint8, device=self.device)
-            self._ws_T = T
-        return self._ws
+        return self._ws.get(workspace_size(self._shape_T(T)))
 
     def _shape_T(self, T: int) -> LayerShape:
         s = self.shape
