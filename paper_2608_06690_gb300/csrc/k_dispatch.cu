@@ -62,6 +62,8 @@ __global__ void __launch_bounds__(kScanThreads) dispatch_order_kernel(const Disp
 {
     __shared__ int warp_tot[32];
     const int e = blockIdx.x, tid = threadIdx.x;
+    pdl_trigger();
+    pdl_wait();
 
     // pass 1: this expert's offset = routed rows of lower expert ids; its count
     int less = 0, mine = 0;
@@ -117,6 +119,8 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const bf16 *__restrict
                                                           const int32_t *__restrict__ tok_of_slot, int R, int T,
                                                           int H, bf16 *__restrict__ a_perm)
 {
+    pdl_trigger();
+    pdl_wait();
     const int nv = H / 8;
     const long long total = (long long)R * nv;
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
@@ -148,6 +152,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const bf16 *__restrict__ y
                                                       const int32_t *__restrict__ slot_of, int T, int H, int k,
                                                       bf16 *__restrict__ out)
 {
+    pdl_trigger();
+    pdl_wait();
     const int nv = H / 8;
     const int R = T * k;
     const long long total = (long long)T * nv;
@@ -202,20 +208,18 @@ cudaError_t launch_permute(const Ctx &c)
     p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.status = c.audit.status;
-    dispatch_order_kernel<<<s.E(), kScanThreads, 0, c.stream>>>(p);
-    cudaError_t err = cudaGetLastError();
+    cudaError_t err = launch_pdl(dispatch_order_kernel, dim3(s.E()), dim3(kScanThreads), 0, c.stream, p);
     if (err != cudaSuccess) return err;
-    gather_rows_kernel<<<grid_for((long long)R * (s.H / 8), c.num_sms), 256, 0, c.stream>>>(c.hidden, c.tok_of_slot, R,
-                                                                                      s.T, s.H, c.a_perm);
-    return cudaGetLastError();
+    return launch_pdl(gather_rows_kernel, dim3(grid_for((long long)R * (s.H / 8), c.num_sms)), dim3(256), 0, c.stream,
+                      (const bf16 *)c.hidden, (const int32_t *)c.tok_of_slot, R, s.T, s.H, c.a_perm);
 }
 
 cudaError_t launch_combine(const Ctx &c)
 {
     const Shape &s = c.s;
-    combine_kernel<<<grid_for((long long)s.T * (s.H / 8), c.num_sms), 256, 0, c.stream>>>(
-        c.y, s.E_sh > 0 ? c.y_sh : nullptr, c.slot_of, s.T, s.H, s.k, c.out);
-    return cudaGetLastError();
+    return launch_pdl(combine_kernel, dim3(grid_for((long long)s.T * (s.H / 8), c.num_sms)), dim3(256), 0, c.stream,
+                      (const bf16 *)c.y, (const bf16 *)(s.E_sh > 0 ? c.y_sh : nullptr), (const int32_t *)c.slot_of, s.T,
+                      s.H, s.k, c.out);
 }
 
 }  // namespace pmpe

@@ -13,9 +13,10 @@
 // experts contribute no tile.
 //
 // CTA roles (192 threads):
-//   warp 0       one thread issues the TMA loads of a 4-stage ring (A: 128
-//                rows x 64 K; B: 256 rows x 64 K, i.e. 128 gate + 128 up rows,
-//                or 256 / 128 output columns of the down projection)
+//   warp 0       three lanes issue the TMA loads of a 4-stage ring, one
+//                operand box each (A: 128 rows x 64 K; B: 256 rows x 64 K,
+//                i.e. 128 gate + 128 up rows, or 256 / 128 output columns of
+//                the down projection in two halves)
 //   warp 1       allocates 512 TMEM columns (two 128 x 256 FP32
 //                accumulators, so the epilogue of one tile overlaps the MMAs
 //                of the next) and one thread issues tcgen05.mma M=128 N=256
@@ -47,6 +48,7 @@ constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kAccCols = 256;                 // FP32 TMEM columns per accumulator
 constexpr int kTmemCols = 2 * kAccCols;
 constexpr int kThreads = 192;
+constexpr int kLoaders = 3;                   // TMA-issuing lanes of warp 0
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
 constexpr int kOutBufBytes = kOutBox * kOutBox * 2;
@@ -139,9 +141,10 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
 
     const int G = p.E + (p.E_sh > 0 ? 1 : 0);
+    pdl_trigger();
 
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
+        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
         for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
         mbar_init(done_bar, 1);
         s_abort = 0;
@@ -152,6 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                      "r"(kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
     }
+    pdl_wait();  // the dispatch offsets and the A operand come from the previous kernels
     // tile list: rows and tiles per group, prefix over groups
     for (int g = tid; g < G; g += kThreads) {
         const bool shared = g >= p.E;
@@ -191,11 +195,19 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     const uint32_t tmem_base = s_tmem;
     const int total = tt.prefix[G];
 
-    if (warp == 0 && lane == 0) {
-        // ------------------------------------------------ TMA producer
+    if (warp == 0 && lane < kLoaders) {
+        // ------------------------------------------------ TMA producers
+        // Three lanes, one operand box each: a single thread's TMA boxes are
+        // processed one after another, so spreading a stage's boxes over
+        // three issuing threads triples the ring's fill rate.
+        //   lane 0: A tile (128 rows x 64 K)
+        //   lane 1: gate rows (gate/up) or B rows [0, bn/2) (down)
+        //   lane 2: up rows (gate/up)   or B rows [bn/2, bn) (down)
         int stage = 0;
         uint32_t phase = 0;
         uint32_t filled = 0, last_parity = 0;  // per-stage bits, for the drain below
+        const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes
+                                         : (p.mode == kGateUp ? (uint32_t)(BM * 128) : (uint32_t)(p.bn / 2 * 128));
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
             const int q = t.shared ? 2 : (t.g < p.E_pub ? 0 : 1);
@@ -206,18 +218,23 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             for (int kb = 0; kb < t.nkb; ++kb) {
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
                 const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
-                mbar_expect_tx(full_bar(stage), p.tx_bytes);
+                mbar_expect_tx(full_bar(stage), my_tx);
                 const int kx = kb * BK;
-                tma_load_2d(sA, amap, full_bar(stage), kx, arow);
-                if (p.mode == kGateUp) {
+                if (lane == 0) {
+                    tma_load_2d(sA, amap, full_bar(stage), kx, arow);
+                } else if (p.mode == kGateUp) {
                     const int brow = ei * p.I + t.n0;  // shared: n0 spans E_sh * I rows
-                    tma_load_2d(sB, &maps.b0[q], full_bar(stage), kx, brow);
-                    tma_load_2d(sB + BM * 128, &maps.b1[q], full_bar(stage), kx, brow);
-                } else if (t.shared) {
-                    const int s = kx / p.I;
-                    tma_load_2d(sB, &maps.b0[2], full_bar(stage), kx - s * p.I, s * p.H + t.n0);
+                    tma_load_2d(sB + (lane - 1) * BM * 128, lane == 1 ? &maps.b0[q] : &maps.b1[q], full_bar(stage), kx,
+                                brow);
                 } else {
-                    tma_load_2d(sB, &maps.b0[q], full_bar(stage), kx, ei * p.H + t.n0);
+                    const int half = (lane - 1) * (p.bn / 2);
+                    if (t.shared) {
+                        const int sidx = kx / p.I;
+                        tma_load_2d(sB + half * 128, &maps.b0[2], full_bar(stage), kx - sidx * p.I,
+                                    sidx * p.H + t.n0 + half);
+                    } else {
+                        tma_load_2d(sB + half * 128, &maps.b0[q], full_bar(stage), kx, ei * p.H + t.n0 + half);
+                    }
                 }
                 filled |= 1u << stage;
                 last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
@@ -422,18 +439,17 @@ cudaError_t launch_tc(const Ctx &c, int mode)
         ok &= encode_2d(&maps.a_routed, c.act, s.I, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
-            ok &= encode_2d(&maps.b0[q], c.down[q], s.I, n, p.bn);
+            ok &= encode_2d(&maps.b0[q], c.down[q], s.I, n, p.bn / 2);
         }
         if (s.E_sh > 0) {
             ok &= encode_2d(&maps.a_shared, c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
-            ok &= encode_2d(&maps.b0[2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, p.bn);
+            ok &= encode_2d(&maps.b0[2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, p.bn / 2);
         }
     }
     if (!ok) return cudaErrorInvalidValue;
     cudaError_t err = cudaFuncSetAttribute(expert_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem);
     if (err != cudaSuccess) return err;
-    expert_gemm_tc_kernel<<<c.num_sms, kThreads, kDynSmem, c.stream>>>(p, maps);
-    return cudaGetLastError();
+    return launch_pdl(expert_gemm_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
 }
 
 }  // namespace

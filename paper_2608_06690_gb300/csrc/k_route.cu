@@ -101,6 +101,8 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     __shared__ volatile int s_abort;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    pdl_trigger();
+    pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
 
     // ---- resolve and rank: pass 1 counts the ALLOW tokens
     int my_allow = 0;
@@ -176,7 +178,7 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     const uint32_t tfull_bar = bar0 + 8u * (2 * kRMaxStages);
     const uint32_t done_bar = bar0 + 8u * (2 * kRMaxStages + 1);
     if (tid == 0) {
-        for (int s = 0; s < p.stages; ++s) { mbar_init(full_bar(s), 1); mbar_init(empty_bar(s), 1); }
+        for (int s = 0; s < p.stages; ++s) { mbar_init(full_bar(s), 2); mbar_init(empty_bar(s), 1); }
         mbar_init(tfull_bar, 1);
         mbar_init(done_bar, 1);
         s_abort = 0;
@@ -191,20 +193,22 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     const int N = p.n_pad[pool];
     const int nkb = p.H / 64;
 
-    if (warp == 0 && lane == 0) {
-        // ---- TMA producer: 128 tile rows + the pool's router rows per stage
+    if (warp == 0 && lane < 2) {
+        // ---- TMA producers: lane 0 the 128 tile rows, lane 1 the pool's router
+        // rows (one box each: boxes of one issuing thread are serialised)
         int stage = 0;
         uint32_t phase = 0, filled = 0, last_parity = 0;
-        const uint32_t tx = (uint32_t)kABytes + (uint32_t)N * 128u;
+        const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes : (uint32_t)N * 128u;
         for (int kb = 0; kb < nkb; ++kb) {
             if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) break;
             const uint32_t sA = sbase + stage * p.stage_bytes, sB = sA + kABytes;
-            mbar_expect_tx(full_bar(stage), tx);
-            if (contiguous)
+            mbar_expect_tx(full_bar(stage), my_tx);
+            if (lane == 1)
+                tma_load_2d(sB, &maps.router[pool], full_bar(stage), kb * 64, 0);
+            else if (contiguous)
                 tma_load_2d(sA, &maps.hidden, full_bar(stage), kb * 64, s_tok[0]);
             else
                 tma_load_2d(sA, &maps.rows, full_bar(stage), kb * 64, blockIdx.x * kTileRows);
-            tma_load_2d(sB, &maps.router[pool], full_bar(stage), kb * 64, 0);
             filled |= 1u << stage;
             last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
             if (++stage == p.stages) { stage = 0; phase ^= 1u; }
@@ -428,8 +432,7 @@ cudaError_t launch_route(const Ctx &c)
     if (smem < lists) smem = lists;
     cudaError_t err = cudaFuncSetAttribute(router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (err != cudaSuccess) return err;
-    router_tc_kernel<<<grid, kRThreads, smem, c.stream>>>(p, maps);
-    return cudaGetLastError();
+    return launch_pdl(router_tc_kernel, dim3(grid), dim3(kRThreads), smem, c.stream, p, maps);
 }
 
 cudaError_t launch_resolve(const uint8_t *policy, int T, uint8_t *tau, cudaStream_t stream)

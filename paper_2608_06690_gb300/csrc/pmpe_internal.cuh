@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/pmpe.h"
 
 namespace pmpe {
@@ -63,7 +65,35 @@ cudaError_t launch_down(const Ctx &c);
 cudaError_t launch_combine(const Ctx &c);
 cudaError_t launch_resolve(const uint8_t *policy, int T, uint8_t *tau, cudaStream_t stream);
 
+// Launch with programmatic dependent launch: the kernel may start (and run
+// its prologue) while the previous kernel in the stream finishes; it must
+// execute pdl_wait() before touching anything that kernel wrote, or writing
+// anything a previous kernel might still read.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // ------------------------------------------------------------ device helpers
+
+// Wait until the previous kernel in the stream has completed and its memory
+// operations are visible (programmatic dependent launch).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+// Allow the next kernel in the stream to launch now (it still waits for this
+// one to complete before touching its results).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
