@@ -65,7 +65,7 @@ extern "C" {
 #define PMPE_ERR_DEVICE_STATUS (-6)     /* a kernel recorded an error in the audit status word */
 
 /* Bits a kernel may OR into the device status word (audit word 0). */
-#define PMPE_STATUS_DISPATCH_MISMATCH 0x1u /* dispatch count differs from the router's count */
+#define PMPE_STATUS_DISPATCH_MISMATCH 0x1u /* reserved */
 #define PMPE_STATUS_PIPELINE_TIMEOUT 0x2u  /* a bounded wait inside an expert kernel gave up */
 #define PMPE_STATUS_BAD_EXPERT_ID 0x4u     /* a routed id outside [0, E) reached the dispatcher */
 
@@ -122,11 +122,12 @@ PMPE_API size_t pmpe_moe_workspace_size(int T, int H, int I, int E_pub, int E_pr
 typedef struct pmpe_workspace_layout {
     size_t total;
     size_t tau;          /* uint8  [T]      resolved policy bits */
-    size_t counts;       /* uint32 [E]      rows routed to each expert (counted by the dispatch stage) */
+    size_t counts;       /* uint32 [E]      rows routed to each expert (router's integer atomics) */
     size_t offsets;      /* uint32 [E+1]    exclusive prefix sum of counts */
     size_t topk_idx;     /* int32  [T, k]   used when desc.topk_idx is NULL */
     size_t topk_w;       /* float  [T, k]   used when desc.topk_w is NULL */
     size_t slot_of;      /* int32  [T, k]   dispatch row of (t, j) */
+    size_t ticket;       /* int32  [T, k]   position of (t, j) among its expert's rows */
     size_t tok_of_slot;  /* int32  [T*k]    token of each dispatch row */
     size_t w_of_slot;    /* float  [T*k]    routing weight of each dispatch row */
     size_t router_rows;  /* BF16   [(ceil(T/128)+1)*128, H] token rows of each router tile, pool order */

@@ -1,13 +1,14 @@
 // Stages 2 and 5 of the layer: the dispatch order of the routed rows with
 // the row gather, and the weighted unpermute-combine.
 //
-// Dispatch order (the grouping any grouped expert execution needs): rows are
-// grouped by expert id and, inside an expert, ordered by token then rank, so
-// the order is a pure function of the route log.  One CTA per expert scans
-// the [T, k] id list twice: first to count the routed rows of lower ids (its
-// offset) and its own, then to write its rows with block-wide scans.  An id
-// outside [0, E) is recorded in the status word.  The gather then copies each
-// token row into its dispatch row with 16-byte vector loads.
+// Dispatch (the grouping any grouped expert execution needs): the routed rows
+// are grouped by expert id -- expert e owns slots [offset[e], offset[e+1]) --
+// and, inside an expert, placed by the ticket the router took with an integer
+// atomic, so the order inside an expert depends on timing.  The layer's output
+// does not: every expert GEMM row depends only on its own input row, and the
+// combine sums each token's rows in rank order.  The same pass copies each
+// token row into its slot with 16-byte vector loads.  An id outside [0, E) is
+// recorded in the status word.
 //
 // Combine: out_t = bf16( sum_{j < k} y[slot(t, j)] + y_shared[t] ), summed in
 // FP32 in a fixed order (j ascending, then shared), so the result of a token
@@ -17,119 +18,84 @@
 namespace pmpe {
 namespace {
 
-constexpr int kScanThreads = 1024;
-constexpr int kPerThread = 4;
-
-// Exclusive block scan of one value per thread (blockDim.x == kScanThreads).
-__device__ __forceinline__ int block_exclusive_scan(int v, int *warp_tot, int &total)
-{
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    int x = v;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const int y = __shfl_up_sync(~0u, x, off);
-        if (lane >= off) x += y;
-    }
-    if (lane == 31) warp_tot[warp] = x;
-    __syncthreads();
-    if (warp == 0) {
-        int w = warp_tot[lane];
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const int y = __shfl_up_sync(~0u, w, off);
-            if (lane >= off) w += y;
-        }
-        warp_tot[lane] = w;  // inclusive
-    }
-    __syncthreads();
-    total = warp_tot[31];
-    const int before = warp == 0 ? 0 : warp_tot[warp - 1];
-    __syncthreads();  // warp_tot is reused by the next call
-    return before + x - v;
-}
+constexpr int kDispThreads = 256;
 
 struct DispatchParams {
     const int32_t *idx;
+    const int32_t *ticket;
     const float *w;
-    int R, k, E;
-    uint32_t *counts, *offsets;
+    const uint32_t *counts;
+    const bf16 *hidden;
+    int T, H, R, k, E;
+    uint32_t *offsets;
     int32_t *slot_of, *tok_of_slot;
     float *w_of_slot;
+    bf16 *a_perm;
     uint32_t *status;
 };
 
-__global__ void __launch_bounds__(kScanThreads) dispatch_order_kernel(const DispatchParams p)
+// Dispatch and gather in one pass.  Every CTA forms the experts' offsets
+// (exclusive prefix sum of the router's per-expert counts) in shared memory;
+// routed row r = (t, j) of expert e goes to slot offset[e] + ticket[r], and its
+// token row is copied there by one warp with 16-byte vectors.
+__global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const DispatchParams p)
 {
-    __shared__ int warp_tot[32];
-    const int e = blockIdx.x, tid = threadIdx.x;
+    __shared__ uint32_t s_off[2 * kMaxPool + 1];
     pdl_trigger();
     pdl_wait();
-
-    // pass 1: this expert's offset = routed rows of lower expert ids; its count
-    int less = 0, mine = 0;
-    bool bad = false;
-    for (int r = tid; r < p.R; r += kScanThreads) {
-        const int id = p.idx[r];
-        less += id < e;
-        mine += id == e;
-        bad |= id < 0 || id >= p.E;
+    if (threadIdx.x < 32) {
+        uint32_t carry = 0;
+        const int lane = threadIdx.x;
+        for (int b = 0; b < p.E; b += 32) {
+            uint32_t v = b + lane < p.E ? p.counts[b + lane] : 0u;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const uint32_t y = __shfl_up_sync(~0u, v, off);
+                if (lane >= off) v += y;
+            }
+            if (b + lane < p.E) s_off[b + lane + 1] = carry + v;
+            carry += __shfl_sync(~0u, v, 31);
+        }
+        if (lane == 0) s_off[0] = 0;
     }
-    int off, n_e;
-    block_exclusive_scan(less, warp_tot, off);
-    block_exclusive_scan(mine, warp_tot, n_e);
-    if (tid == 0) {
-        p.offsets[e] = (uint32_t)off;
-        p.counts[e] = (uint32_t)n_e;
-        if (e == p.E - 1) p.offsets[p.E] = (uint32_t)(off + n_e);
-    }
-    if (e == 0 && p.status && __syncthreads_or(bad) && tid == 0) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+    __syncthreads();
+    if (blockIdx.x == 0)
+        for (int e = threadIdx.x; e <= p.E; e += kDispThreads) p.offsets[e] = s_off[e];
 
-    // pass 2: this expert's rows in (token, rank) order
-    int running = 0;
-    for (int base = 0; base < p.R; base += kScanThreads * kPerThread) {
-        const int r0 = base + tid * kPerThread;
-        int ids[kPerThread];
+    // one warp per routed row: the slot is resolved once, then every lane
+    // issues a batch of independent 16-byte loads before its stores
+    const int lane = threadIdx.x & 31;
+    const int nv = p.H / 8;
+    const int warps = gridDim.x * (kDispThreads / 32);
+    for (int r = blockIdx.x * (kDispThreads / 32) + (threadIdx.x >> 5); r < p.R; r += warps) {
+        const int e = p.idx[r];
+        if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
+            if (lane == 0 && p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+            continue;
+        }
+        const int slot = (int)s_off[e] + p.ticket[r];
+        if ((unsigned)slot >= (unsigned)p.R) continue;  // only a corrupt ticket could get here
+        const int t = r / p.k;
+        const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
+        uint4 *dst = reinterpret_cast<uint4 *>(p.a_perm + (size_t)slot * p.H);
+        for (int c0 = 0; c0 < nv; c0 += 32 * 8) {
+            uint4 v[8];
 #pragma unroll
-        for (int q = 0; q < kPerThread; ++q) ids[q] = (r0 + q < p.R) ? p.idx[r0 + q] : -1;
-        int cnt = 0;
+            for (int u = 0; u < 8; ++u) {
+                const int c = c0 + u * 32 + lane;
+                if (c < nv) v[u] = __ldg(src + c);
+            }
 #pragma unroll
-        for (int q = 0; q < kPerThread; ++q) cnt += ids[q] == e;
-        int total;
-        int rank = block_exclusive_scan(cnt, warp_tot, total);
-#pragma unroll
-        for (int q = 0; q < kPerThread; ++q) {
-            if (ids[q] == e) {
-                const int r = r0 + q;
-                const int slot = off + running + rank;
-                if (slot < p.R) {  // always true: off + n_e <= R
-                    p.slot_of[r] = slot;
-                    p.tok_of_slot[slot] = r / p.k;
-                    p.w_of_slot[slot] = p.w[r];
-                }
-                ++rank;
+            for (int u = 0; u < 8; ++u) {
+                const int c = c0 + u * 32 + lane;
+                if (c < nv) dst[c] = v[u];
             }
         }
-        running += total;
-    }
-}
-
-// Row gather: one thread per 16-byte chunk of a dispatch row, so a row is
-// copied by H/8 consecutive threads with fully coalesced loads and stores.
-__global__ void __launch_bounds__(256) gather_rows_kernel(const bf16 *__restrict__ hidden,
-                                                          const int32_t *__restrict__ tok_of_slot, int R, int T,
-                                                          int H, bf16 *__restrict__ a_perm)
-{
-    pdl_trigger();
-    pdl_wait();
-    const int nv = H / 8;
-    const long long total = (long long)R * nv;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int row = (int)(i / nv), c = (int)(i - (long long)row * nv);
-        int t = tok_of_slot[row];
-        if ((unsigned)t >= (unsigned)T) t = 0;  // only reachable after a dispatch mismatch (status word set)
-        reinterpret_cast<uint4 *>(a_perm + (size_t)row * H)[c] =
-            __ldg(reinterpret_cast<const uint4 *>(hidden + (size_t)t * H) + c);
+        if (lane == 0) {
+            p.slot_of[r] = slot;
+            p.tok_of_slot[slot] = t;
+            p.w_of_slot[slot] = p.w[r];
+        }
     }
 }
 
@@ -204,14 +170,13 @@ cudaError_t launch_permute(const Ctx &c)
     const Shape &s = c.s;
     const int R = s.T * s.k;
     DispatchParams p;
-    p.idx = c.idx; p.w = c.w; p.counts = c.counts;
-    p.R = R; p.k = s.k; p.E = s.E();
+    p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts; p.hidden = c.hidden;
+    p.T = s.T; p.H = s.H; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
+    p.a_perm = c.a_perm;
     p.status = c.audit.status;
-    cudaError_t err = launch_pdl(dispatch_order_kernel, dim3(s.E()), dim3(kScanThreads), 0, c.stream, p);
-    if (err != cudaSuccess) return err;
-    return launch_pdl(gather_rows_kernel, dim3(grid_for((long long)R * (s.H / 8), c.num_sms)), dim3(256), 0, c.stream,
-                      (const bf16 *)c.hidden, (const int32_t *)c.tok_of_slot, R, s.T, s.H, c.a_perm);
+    return launch_pdl(dispatch_gather_kernel, dim3(grid_for((long long)R * 32, c.num_sms)), dim3(kDispThreads), 0,
+                      c.stream, p);
 }
 
 cudaError_t launch_combine(const Ctx &c)

@@ -17,7 +17,8 @@
 // lane, four column slices) each select the top-k of their slice (descending
 // score, ties to the lower expert id) by ordered passes with four independent
 // selection chains, and one thread per token merges the four sorted lists and
-// writes the softmax weights and the route log.
+// writes the softmax weights and the route log, and takes the row's position
+// inside its expert (an integer atomic ticket) for the dispatch stage.
 #include <cuda.h>
 
 #include "pmpe_internal.cuh"
@@ -45,6 +46,8 @@ struct RouterParams {
     uint8_t *tau;
     int32_t *idx;
     float *w;
+    uint32_t *counts;  // per-expert row counters (zeroed before the launch)
+    int32_t *ticket;   // [T, k] row position inside its expert
     uint32_t *route_count, *route_priv_rows, *status;
 };
 
@@ -352,6 +355,9 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
                 npriv += gid >= p.E_pub;
                 if (valid) {
                     p.idx[(size_t)t * p.k + j] = gid;
+                    // this row's position among the expert's rows (the dispatch
+                    // stage adds the expert's offset)
+                    p.ticket[(size_t)t * p.k + j] = (int32_t)atomicAdd(&p.counts[gid], 1u);
                     if (p.route_count) atomicAdd(&p.route_count[gid], 1u);
                 }
             }
@@ -393,6 +399,8 @@ __global__ void resolve_kernel(const uint8_t *policy, int T, uint8_t *tau)
 cudaError_t launch_route(const Ctx &c)
 {
     const Shape &s = c.s;
+    cudaError_t merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
+    if (merr != cudaSuccess) return merr;
     RouterParams p;
     RouterMaps maps;
     memset(&maps, 0, sizeof(maps));
@@ -415,6 +423,8 @@ cudaError_t launch_route(const Ctx &c)
     p.tau = c.tau;
     p.idx = c.idx;
     p.w = c.w;
+    p.counts = c.counts;
+    p.ticket = c.ticket;
     p.route_count = c.audit.route_count;
     p.route_priv_rows = c.audit.route_priv_rows;
     p.status = c.audit.status;

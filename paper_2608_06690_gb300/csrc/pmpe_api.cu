@@ -33,6 +33,7 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     L->topk_idx = take(4 * R, 256);
     L->topk_w = take(4 * R, 256);
     L->slot_of = take(4 * R, 256);
+    L->ticket = take(4 * R, 256);
     L->tok_of_slot = take(4 * R, 256);
     L->w_of_slot = take(4 * R, 256);
     L->router_rows = take(2 * ((T + 127) / 128 + 1) * 128 * (size_t)s.H, 1024);
@@ -112,6 +113,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->counts = (uint32_t *)(ws + L.counts);
     c->offsets = (uint32_t *)(ws + L.offsets);
     c->slot_of = (int32_t *)(ws + L.slot_of);
+    c->ticket = (int32_t *)(ws + L.ticket);
     c->tok_of_slot = (int32_t *)(ws + L.tok_of_slot);
     c->w_of_slot = (float *)(ws + L.w_of_slot);
     c->router_rows = (bf16 *)(ws + L.router_rows);

@@ -48,6 +48,7 @@ struct Ctx {
     uint8_t *tau;
     uint32_t *counts, *offsets;
     int32_t *slot_of, *tok_of_slot;
+    int32_t *ticket;    // [T, k] position of each routed row inside its expert
     float *w_of_slot;
     bf16 *router_rows;  // [(ceil(T/128)+1)*128, H] router tiles' token rows
     bf16 *a_perm, *act, *y, *act_sh, *y_sh;
