@@ -16,9 +16,11 @@ from __future__ import annotations
 import argparse
 import json
 import os
+import shutil
 import statistics
 import subprocess
 import sys
+import threading
 import time
 
 import numpy as np
@@ -37,7 +39,7 @@ L2_FLUSH_BYTES = 512 << 20   # > 129 MB L2
 # grouped GEMM kernels, from one ncu capture of the current kernels on the
 # named workload; None where no capture of the current kernels exists.
 NCU_TRAFFIC = {
-    "qwen3_prefill": {"gateup": 1.146401e9 + 44.646912e6, "down": 0.553858e9 + 103.074048e6},
+    "qwen3_prefill": {"gateup": 1.145576e9 + 44.352512e6, "down": 0.553868e9 + 103.251456e6},
 }
 
 
@@ -73,7 +75,9 @@ def _peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle-reason samples during the timed region."""
+    """nvidia-smi clock / throttle-reason samples, taken every 50 ms from
+    before the warm-up until after the end-to-end leg; each sample is stamped
+    on arrival so the ones inside the timed region can be counted."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -82,31 +86,44 @@ class ClockSampler:
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
+        self.lines = []
+        self._first = threading.Event()
+
+    def _read(self):
+        for l in self.proc.stdout:
+            if l.strip():
+                self.lines.append((time.perf_counter(), l))
+                self._first.set()
 
     def __enter__(self):
+        cmd = ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+               "-lms", "50"]
+        if shutil.which("stdbuf"):
+            cmd = ["stdbuf", "-oL"] + cmd   # one line per sample, as it is taken
         try:
-            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "50"],
-                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
+            return self
+        self._thread = threading.Thread(target=self._read, daemon=True)
+        self._thread.start()
+        self._first.wait(3.0)          # the sampler is running before the GPU work starts
         return self
 
     def __exit__(self, *a):
-        self.lines = []
         if self.proc is not None:
             self.proc.terminate()
             try:
-                out, _ = self.proc.communicate(timeout=5)
+                self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
-                out, _ = self.proc.communicate()
-            self.lines = [l for l in out.splitlines() if l.strip()]
+                self.proc.wait()
+            self._thread.join(timeout=5)
 
-    def summary(self):
-        sm, mx, reasons = [], None, set()
+    def summary(self, window=None):
+        sm, mx, reasons, inside = [], None, set(), 0
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for l in getattr(self, "lines", []):
+        for t, l in list(self.lines):
             f = [x.strip() for x in l.split(",")]
             if len(f) < 9:
                 continue
@@ -115,11 +132,16 @@ class ClockSampler:
                 mx = float(f[2])
             except ValueError:
                 continue
+            if window is not None and window[0] <= t <= window[1]:
+                inside += 1
             for n, v in zip(names, f[5:9]):
                 if v.lower() == "active":
                     reasons.add(n)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        out = {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+               "samples": len(sm)}
+        if window is not None:
+            out["samples_in_timed_region"] = inside
+        return out
 
 
 def build_workload(cfg, device, seed_offset=0):
@@ -350,7 +372,7 @@ def run_ours(args):
                         "mean_rows_public": float(counts[:s.E_pub].mean()),
                         "mean_rows_private": float(counts[s.E_pub:].mean())},
         "gpu_launches": pmpe.KERNELS_PER_FORWARD * args.steps,
-        "clocks": clk.summary(),
+        "clocks": clk.summary(window=(t_wall0, t_wall0 + t_wall)),
         "wall_s_timed_region": t_wall,
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h.numel() * 2 + pol.numel(),
                 "d2h_bytes_per_step": out.numel() * 2},
@@ -365,8 +387,8 @@ def run_ours(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--config", default="qwen3_prefill", choices=sorted(CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--ref-tokens", type=int, default=96)

@@ -168,6 +168,17 @@ PMPE_API int pmpe_moe_forward(const pmpe_moe_desc *d, void *stream);
  * with the same inputs.  pmpe_moe_forward() == stages PMPE_STAGE_ALL. */
 PMPE_API int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *stream);
 
+/* Self-test of the failure path of the layer's pipelined kernels: launches one
+ * kernel whose shared-memory barrier wait can never complete (nothing
+ * arrives), through the same bounded wait the layer's tensor-core kernels use
+ * at every pipeline stage, with a limit of limit_us microseconds (1 ..
+ * 1,000,000).  The wait expires, ORs PMPE_STATUS_PIPELINE_TIMEOUT into
+ * *status (a device word, e.g. audit word 0) and the kernel returns; the CUDA
+ * context stays usable.  Asynchronous on `stream`.  Not part of the paper's
+ * method: it tests the library's failure detection (device waits are bounded,
+ * expiry is reported, never a hang or a trap). */
+PMPE_API int pmpe_selftest_wait_timeout(uint32_t *status, int limit_us, void *stream);
+
 /* Size of the device scratch array that pmpe_moe_forward_noalloc() uses in
  * place of a caller workspace: 32 MiB, reserved on every GPU that loads the
  * library until the process exits.  (A 64-token decode step of a layer with

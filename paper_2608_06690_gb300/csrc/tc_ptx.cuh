@@ -43,21 +43,29 @@ __device__ __forceinline__ unsigned long long globaltimer_ns()
     return t;
 }
 
-// Wait for the phase of `bar` with parity `parity`, for at most kWaitLimitNs
-// or until another role raised the abort flag.  Returns false on give-up.
-__device__ __noinline__ static bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, uint32_t *status)
+// Wait for the phase of `bar` with parity `parity`, for at most limit_ns
+// (kWaitLimitNs for the layer's kernels) or until another role raised the
+// abort flag.  On expiry it raises the abort flag, records
+// PMPE_STATUS_PIPELINE_TIMEOUT and returns false.
+__device__ __noinline__ static bool mbar_wait_for(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                                  uint32_t *status, unsigned long long limit_ns)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer_ns();
     for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             *abort_flag = 1;
             if (status) atomicOr(status, PMPE_STATUS_PIPELINE_TIMEOUT);
             return false;
         }
     }
+}
+__device__ __forceinline__ static bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                                 uint32_t *status)
+{
+    return mbar_wait_for(bar, parity, abort_flag, status, kWaitLimitNs);
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y)

@@ -48,7 +48,7 @@ KERNELS_PER_FORWARD = 5
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
-            "pmpe_status_string", "pmpe_moe_forward_noalloc")
+            "pmpe_status_string", "pmpe_moe_forward_noalloc", "pmpe_selftest_wait_timeout")
 
 # Bytes of the library's static scratch array used by pmpe_moe_forward_noalloc.
 STATIC_SCRATCH_BYTES = 32 << 20
@@ -88,6 +88,8 @@ _lib.pmpe_moe_forward_stages.restype = ctypes.c_int
 _lib.pmpe_moe_forward_stages.argtypes = [ctypes.POINTER(MoeDesc), ctypes.c_uint, _vp]
 _lib.pmpe_moe_forward_noalloc.restype = ctypes.c_int
 _lib.pmpe_moe_forward_noalloc.argtypes = [ctypes.POINTER(MoeDesc), _vp]
+_lib.pmpe_selftest_wait_timeout.restype = ctypes.c_int
+_lib.pmpe_selftest_wait_timeout.argtypes = [_vp, ctypes.c_int, _vp]
 _lib.pmpe_audit_reset.restype = ctypes.c_int
 _lib.pmpe_audit_reset.argtypes = [_vp, ctypes.c_int, ctypes.c_int, _vp]
 _lib.pmpe_audit_read.restype = ctypes.c_int
@@ -163,6 +165,14 @@ def audit_read(audit, T: int, E: int, stream=None, timeout_ms: int = 10000, chec
         rc = OK
     _check(rc, "pmpe_audit_read")
     return audit_fields(host.numpy().view(np.uint32).copy(), T, E)
+
+
+def selftest_wait_timeout(status, limit_us: int, stream=None):
+    """Enqueue the bounded-wait self-test: a barrier wait that can never
+    complete expires after ``limit_us`` microseconds and ORs
+    STATUS_PIPELINE_TIMEOUT into the device word ``status[0]``."""
+    _check(_lib.pmpe_selftest_wait_timeout(_ptr(status), int(limit_us), _stream(stream)),
+           "pmpe_selftest_wait_timeout")
 
 
 def make_desc(s: LayerShape, weights: dict, hidden, policy, out, workspace, topk_idx=None, topk_w=None,

@@ -130,3 +130,6 @@ def test_validation_rejects_before_any_cuda_call(pmpe):
     assert lib.pmpe_policy_resolve(None, 0, None, None) == pmpe.OK
     assert lib.pmpe_audit_reset(None, 4, 4, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_audit_read(None, 4, 4, None, None, 10) == pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_selftest_wait_timeout(None, 1000, None) == pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 0, None) == pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 1000001, None) == pmpe.ERR_INVALID_ARG
