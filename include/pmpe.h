@@ -118,7 +118,10 @@ PMPE_API size_t pmpe_moe_workspace_size(int T, int H, int I, int E_pub, int E_pr
 
 /* Byte offsets of the named regions inside the workspace (for tests that
  * inspect intermediate results, and for the stage-by-stage entry point).
- * Returns PMPE_ERR_INVALID_ARG for an invalid shape. */
+ * Router geometry used below: S = ceil(T/128) + 1 token-tile slots and
+ * C = S * max(ceil(E_pub/32), ceil(E_priv/32)) router CTAs (one per tile and
+ * 32-expert chunk of its pool).  Returns PMPE_ERR_INVALID_ARG for an invalid
+ * shape. */
 typedef struct pmpe_workspace_layout {
     size_t total;
     size_t tau;          /* uint8  [T]      resolved policy bits */
@@ -130,12 +133,15 @@ typedef struct pmpe_workspace_layout {
     size_t ticket;       /* int32  [T, k]   position of (t, j) among its expert's rows */
     size_t tok_of_slot;  /* int32  [T*k]    token of each dispatch row */
     size_t w_of_slot;    /* float  [T*k]    routing weight of each dispatch row */
-    size_t router_rows;  /* BF16   [(ceil(T/128)+1)*128, H] token rows of each router tile, pool order */
+    size_t router_rows;  /* BF16   [C*128, H]  token rows of each router CTA whose tile is not consecutive */
     size_t a_perm;       /* BF16   [T*k, H] token rows in dispatch order */
     size_t act;          /* BF16   [T*k, I] silu(g)*u of each dispatch row */
     size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row */
     size_t act_sh;       /* BF16   [T, E_shared*I] shared-expert activations (0 if none) */
     size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs (0 if none) */
+    size_t tile_done;    /* uint32 [S]      router CTAs finished per 128-token tile */
+    size_t router_lists; /* float2 [C*128, k] per 32-expert chunk: each token's best k (score, id) */
+    size_t router_meta;  /* float4 [C*128]  per chunk: max score, sum exp(score - max), entries */
 } pmpe_workspace_layout;
 PMPE_API int pmpe_moe_workspace_layout(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k,
                               pmpe_workspace_layout *out);

@@ -1,24 +1,26 @@
 // Stage 1 of the layer: fail-closed policy resolve, masked router, top-k and
 // the route log (Sec. 3.1 Eq. 4; App. B.1 steps 2, 4, 5).
 //
-// router_tc_kernel: each CTA owns one 128-token tile of ONE pool.  It first
-// resolves the policy bytes itself (only the trusted byte 0x01 is ALLOW) and
-// ranks the tokens inside their pool, so that the DENY tokens form tiles
-// 0 .. ceil(n_deny/128)-1 and the ALLOW tokens the tiles after them, each in
-// ascending token order.  A TMA ring streams the tile's token rows and the
-// pool's router rows as 128-byte-swizzled tiles into shared memory: straight
-// from `hidden` when the tile's tokens are consecutive, otherwise from a
-// contiguous workspace block the CTA first fills by token index (row gathers
-// through TMA gather4 or cp.async ran 2.5-5x slower than copy + tile loads).
-// tcgen05.mma computes the 128 x E_pool logits in tensor memory.  A DENY row
-// is therefore only ever multiplied by public router rows and an ALLOW row
-// only by private ones: an ineligible expert never becomes a candidate.
-// Sixteen epilogue warps read the logits: four threads per token (one TMEM
-// lane, four column slices) each select the top-k of their slice (descending
-// score, ties to the lower expert id) by ordered passes with four independent
-// selection chains, and one thread per token merges the four sorted lists and
-// writes the softmax weights and the route log, and takes the row's position
-// inside its expert (an integer atomic ticket) for the dispatch stage.
+// router_tc_kernel: the tokens of each pool form 128-token tiles (DENY tiles
+// first, then ALLOW tiles, each in ascending token order), and each tile is
+// split by 32-expert chunks of its pool's router: one CTA per (tile, chunk).
+// Every CTA resolves the policy bytes itself (only the trusted byte 0x01 is
+// ALLOW) and ranks the tokens inside their pool, which gives it its tile.  A
+// TMA ring streams the tile's token rows and the chunk's 32 router rows as
+// 128-byte-swizzled tiles into shared memory: straight from `hidden` when
+// the tile's tokens are consecutive, otherwise from a contiguous workspace
+// block the CTA first fills by token index.  tcgen05.mma computes the
+// 128 x 32 logits of the chunk in tensor memory.  A DENY row is only ever
+// multiplied by public router rows and an ALLOW row only by private ones: an
+// ineligible expert never becomes a candidate.
+//
+// One epilogue thread per token sorts its 32 logits (descending score, ties
+// to the lower expert id; a bitonic network in registers) and publishes the
+// first k with the chunk's softmax partial to the workspace.  The CTA that
+// completes a tile last (an integer atomic per tile, after a memory fence)
+// merges the chunk lists in chunk order, writes the softmax weights and the
+// route log, and hands out the rows' positions inside their experts: one
+// shared-memory atomic per row and one global atomic per expert and tile.
 #include <cuda.h>
 
 #include "pmpe_internal.cuh"
@@ -27,40 +29,46 @@
 namespace pmpe {
 namespace {
 
-constexpr int kEpiWarps = 16;    // 4 per TMEM lane quarter, each on a quarter of the logit columns
-constexpr int kRThreads = 64 + 32 * kEpiWarps;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2..17 epilogue
-constexpr int kRMaxStages = 8;
+constexpr int kRThreads = 192;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2..5 epilogue (one thread per token)
+constexpr int kRMaxStages = 10;
 constexpr int kTileRows = 128;
-constexpr int kABytes = kTileRows * 128;  // 128 rows x 64 BF16
+constexpr int kChunk = 32;                  // experts per CTA (MMA N)
+constexpr int kMaxChunks = kMaxPool / kChunk;
+constexpr int kABytes = kTileRows * 128;    // 128 rows x 64 BF16
+constexpr int kBBytes = kChunk * 128;       // 32 router rows x 64 BF16
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kEpi = 128;                   // epilogue threads
 
 struct RouterParams {
     int T, H, E_pub, E_priv, k, renorm;
-    int n_pad[2];        // MMA N of each pool: pool size rounded up to 16 (>= 16)
-    uint32_t idesc[2];
-    uint32_t tmem_cols;  // power of two >= max n_pad
+    int nch[2];          // 32-expert chunks of each pool
+    int nch_max;         // CTAs per tile slot
+    uint32_t idesc;      // M = 128, N = 32
     int stages;
-    uint32_t stage_bytes;
     const uint8_t *policy;
     const bf16 *hidden;
-    bf16 *rows_ws;       // [grid * 128, H] tile rows in pool order (workspace)
+    bf16 *rows_ws;       // [slots * nch_max * 128, H] copied tile rows, one block per CTA
+    float2 *lists;       // [slots * nch_max][128][k] (score, id) sorted per chunk
+    float4 *meta;        // [slots * nch_max][128] (chunk max, sum exp(x - max), entries, -)
+    uint32_t *tile_done; // [slots] chunk CTAs finished (zeroed before the launch)
     uint8_t *tau;
     int32_t *idx;
     float *w;
-    uint32_t *counts;  // per-expert row counters (zeroed before the launch)
-    int32_t *ticket;   // [T, k] row position inside its expert
+    uint32_t *counts;    // per-expert row counters (zeroed before the launch)
+    int32_t *ticket;     // [T, k] row position inside its expert
     uint32_t *route_count, *route_priv_rows, *status;
 };
 
 struct RouterMaps {
     CUtensorMap hidden;     // [T, H], box 64 x 128 (tiles of consecutive tokens)
     CUtensorMap rows;       // rows_ws, box 64 x 128 (copied tiles)
-    CUtensorMap router[2];  // [E_pool, H], box 64 x n_pad
+    CUtensorMap router[2];  // [E_pool, H], box 64 x 32
 };
 
 // Exclusive scan over the block of one int per thread (kRThreads threads).
 __device__ __forceinline__ int block_scan(int v, int *warp_tot, int &total)
 {
-    constexpr int kW = kRThreads / 32;  // 18
+    constexpr int kW = kRThreads / 32;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     int x = v;
 #pragma unroll
@@ -88,10 +96,57 @@ __device__ __forceinline__ bool is_allow(const uint8_t *policy, int t)
 }
 
 // (x, e) ranks above (bx, be): larger logit, or equal logit and lower id.
+// Evaluated without short-circuit branches (it sits inside sorting networks).
 __device__ __forceinline__ bool ranks_above(float x, int e, float bx, int be)
 {
-    return x > bx || (x == bx && e < be);
+    return (x > bx) | ((x == bx) & (e < be));
 }
+
+// One compare-exchange of the bitonic network on positions I < J: after it,
+// position I holds the pair that ranks higher when `best_first`, else lower.
+template <int I, int J, bool kBestFirst>
+__device__ __forceinline__ void cex(float (&v)[32], int (&e)[32])
+{
+    const bool sw = kBestFirst ? ranks_above(v[J], e[J], v[I], e[I]) : ranks_above(v[I], e[I], v[J], e[J]);
+    const float tv = v[I];
+    const int te = e[I];
+    v[I] = sw ? v[J] : v[I];
+    e[I] = sw ? e[J] : e[I];
+    v[J] = sw ? tv : v[J];
+    e[J] = sw ? te : e[J];
+}
+
+// All compare-exchanges of one (SIZE, STRIDE) step for positions I .. 31.
+template <int SIZE, int STRIDE, int I>
+__device__ __forceinline__ void bitonic_step(float (&v)[32], int (&e)[32])
+{
+    if constexpr (I < 32) {
+        if constexpr ((I ^ STRIDE) > I) cex<I, (I ^ STRIDE), (I & SIZE) == 0>(v, e);
+        bitonic_step<SIZE, STRIDE, I + 1>(v, e);
+    }
+}
+
+template <int SIZE, int STRIDE>
+__device__ __forceinline__ void bitonic_merge(float (&v)[32], int (&e)[32])
+{
+    if constexpr (STRIDE > 0) {
+        bitonic_step<SIZE, STRIDE, 0>(v, e);
+        bitonic_merge<SIZE, STRIDE / 2>(v, e);
+    }
+}
+
+template <int SIZE>
+__device__ __forceinline__ void bitonic_sort(float (&v)[32], int (&e)[32])
+{
+    if constexpr (SIZE <= 32) {
+        bitonic_merge<SIZE, SIZE / 2>(v, e);
+        bitonic_sort<SIZE * 2>(v, e);
+    }
+}
+
+// Sort 32 (score, id) pairs held in registers into rank order (best first)
+// with a bitonic network whose every index is a compile-time constant.
+__device__ __forceinline__ void sort32(float (&v)[32], int (&e)[32]) { bitonic_sort<2>(v, e); }
 
 __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterParams p,
                                                                   const __grid_constant__ RouterMaps maps)
@@ -102,44 +157,42 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     __shared__ __align__(8) uint64_t bars[2 * kRMaxStages + 2];
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
+    __shared__ int s_last;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int slot = blockIdx.x / p.nch_max, chunk = blockIdx.x - slot * p.nch_max;
     pdl_trigger();
     pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
 
-    // ---- resolve and rank: pass 1 counts the ALLOW tokens
-    int my_allow = 0;
-    for (int t = tid; t < p.T; t += kRThreads) my_allow += is_allow(p.policy, t);
-    int na_total;
-    block_scan(my_allow, warp_tot, na_total);
-    const int na = na_total, nd = p.T - na;
+    // ---- resolve and rank in one pass: each thread takes a contiguous run of
+    // tokens; the scan of its ALLOW count gives the pool sizes and its ranks
+    const int per = (p.T + kRThreads - 1) / kRThreads;
+    const int t0 = min(p.T, tid * per), t1 = min(p.T, t0 + per);
+    int a = 0;
+    for (int t = t0; t < t1; ++t) a += is_allow(p.policy, t);
+    int na;
+    const int a_before = block_scan(a, warp_tot, na);
+    const int nd = p.T - na;
     const int tiles_d = (nd + kTileRows - 1) / kTileRows;
     int pool, m0;
-    if ((int)blockIdx.x < tiles_d) {
+    if (slot < tiles_d) {
         pool = 0;
-        m0 = blockIdx.x * kTileRows;
+        m0 = slot * kTileRows;
     } else {
         pool = 1;
-        m0 = (blockIdx.x - tiles_d) * kTileRows;
-        if (m0 >= na) return;  // uniform: no tile for this CTA
+        m0 = (slot - tiles_d) * kTileRows;
+        if (m0 >= na) return;  // uniform: no tile for this slot
     }
+    if (chunk >= p.nch[pool]) return;  // uniform: the pool has fewer chunks
     const int rows = min(kTileRows, (pool ? na : nd) - m0);
-    // pass 2: each thread takes a contiguous run of tokens, ranks them in
-    // their pool, and keeps the ones that fall into this CTA's tile
     {
-        const int per = (p.T + kRThreads - 1) / kRThreads;
-        const int t0 = tid * per, t1 = min(p.T, t0 + per);
-        int a = 0;
-        for (int t = t0; t < t1; ++t) a += is_allow(p.policy, t);
-        int dummy;
-        const int a_before = block_scan(a, warp_tot, dummy);
         int ra = a_before, rd = t0 - a_before;  // ranks inside the ALLOW / DENY pools
         for (int t = t0; t < t1; ++t) {
             const bool al = is_allow(p.policy, t);
             const int rank = al ? ra++ : rd++;
             if ((al ? 1 : 0) == pool && rank >= m0 && rank < m0 + rows) {
                 s_tok[rank - m0] = t;
-                p.tau[t] = al ? 1 : 0;  // every token is written by exactly one CTA
+                if (chunk == 0) p.tau[t] = al ? 1 : 0;  // every token is written by exactly one CTA
             }
         }
     }
@@ -148,8 +201,8 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     // The TMA ring reads the tile's rows as one 128-row tile.  When the tile's
     // tokens are consecutive (a request with one policy) that tile is read
     // from `hidden` directly; otherwise the CTA first copies its token rows
-    // into a contiguous block (padding rows are not copied: their logits are
-    // never read) and makes the generic-proxy writes visible to the async
+    // into its own contiguous block (padding rows are not copied: their logits
+    // are never read) and makes the generic-proxy writes visible to the async
     // proxy of the TMA reads.
     const int contiguous = __syncthreads_and(tid >= rows || s_tok[tid < kTileRows ? tid : 0] == s_tok[0] + tid);
     if (!contiguous) {
@@ -187,27 +240,28 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         s_abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
-    if (warp == 1) tmem_alloc(smem_u32(&s_tmem), p.tmem_cols);
+    if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kChunk);
     __syncwarp();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = s_tmem;
-    const int N = p.n_pad[pool];
     const int nkb = p.H / 64;
+    const int P = pool ? p.E_priv : p.E_pub;
+    const int base = pool ? p.E_pub : 0;
 
     if (warp == 0 && lane < 2) {
-        // ---- TMA producers: lane 0 the 128 tile rows, lane 1 the pool's router
-        // rows (one box each: boxes of one issuing thread are serialised)
+        // ---- TMA producers: lane 0 the 128 tile rows, lane 1 the chunk's 32
+        // router rows (one box each; router rows past the pool read as zeros)
         int stage = 0;
         uint32_t phase = 0, filled = 0, last_parity = 0;
-        const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes : (uint32_t)N * 128u;
+        const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes : (uint32_t)kBBytes;
         for (int kb = 0; kb < nkb; ++kb) {
             if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) break;
-            const uint32_t sA = sbase + stage * p.stage_bytes, sB = sA + kABytes;
+            const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
             mbar_expect_tx(full_bar(stage), my_tx);
             if (lane == 1)
-                tma_load_2d(sB, &maps.router[pool], full_bar(stage), kb * 64, 0);
+                tma_load_2d(sB, &maps.router[pool], full_bar(stage), kb * 64, chunk * kChunk);
             else if (contiguous)
                 tma_load_2d(sA, &maps.hidden, full_bar(stage), kb * 64, s_tok[0]);
             else
@@ -219,158 +273,176 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         // every copy this thread issued has landed before the CTA exits
         for (int s = 0; s < p.stages; ++s)
             if ((filled >> s) & 1u) {
-                const unsigned long long t0 = globaltimer_ns();
+                const unsigned long long w0 = globaltimer_ns();
                 while (!mbar_try_wait(full_bar(s), (last_parity >> s) & 1u))
-                    if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+                    if (globaltimer_ns() - w0 > kWaitLimitNs) break;
             }
     } else if (warp == 1 && lane == 0) {
-        // ---- MMA issuer: logits[128, N] += rows[128, 64] x router[N, 64]^T per stage
+        // ---- MMA issuer: logits[128, 32] += rows[128, 64] x router[32, 64]^T per stage
         int stage = 0;
         uint32_t phase = 0;
         bool ok = true;
         for (int kb = 0; kb < nkb; ++kb) {
             if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
             tc_fence_after();
-            const uint32_t sA = sbase + stage * p.stage_bytes, sB = sA + kABytes;
+            const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
             const uint64_t ad = sw128_desc(sA), bd = sw128_desc(sB);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) tc_mma(tmem, ad + 2 * k, bd + 2 * k, p.idesc[pool], (kb | k) != 0);
+            for (int k = 0; k < 4; ++k) tc_mma(tmem, ad + 2 * k, bd + 2 * k, p.idesc, (kb | k) != 0);
             tc_commit(empty_bar(stage));
             if (++stage == p.stages) { stage = 0; phase ^= 1u; }
         }
         if (ok) tc_commit(tfull_bar);
         tc_commit(done_bar);
-        const unsigned long long t0 = globaltimer_ns();
+        const unsigned long long w0 = globaltimer_ns();
         while (!mbar_try_wait(done_bar, 0))
-            if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+            if (globaltimer_ns() - w0 > kWaitLimitNs) break;
     } else if (warp >= 2) {
-        // ---- epilogue.  Thread (quarter q, slice sl) owns TMEM lane 32q + lane
-        // (one token) and the logit columns of chunks sl, sl+4, ... (32 each);
-        // it selects the top-k of its columns, then one thread per token merges
-        // the four sorted slice lists.
+        // ---- epilogue: thread r owns TMEM lane r (one token) and the chunk's 32 columns
+        const int q = warp & 3;
+        const int r = q * 32 + lane;
+        const int et = (warp - 2) * 32 + lane;  // 0 .. 127 over the epilogue threads
         int ok = 1;
         if (lane == 0) ok = mbar_wait(tfull_bar, 0, &s_abort, p.status) ? 1 : 0;
         ok = __shfl_sync(~0u, ok, 0);
-        const int q = warp & 3, sl = (warp - 2) >> 2;
-        const int r = q * 32 + lane;
-        const int P = pool ? p.E_priv : p.E_pub;
-        const int base = pool ? p.E_pub : 0;
-        float *lv = reinterpret_cast<float *>(dsmem + (sbase - smem_u32(dsmem)));  // [128][4][k] values
-        int *li = reinterpret_cast<int *>(lv + kTileRows * 4 * p.k);               // [128][4][k] ids
-        float *lmax = reinterpret_cast<float *>(li + kTileRows * 4 * p.k);          // [128][4]
-        float *lsum = lmax + kTileRows * 4;                                          // [128][4]
-        int *lcnt = reinterpret_cast<int *>(lsum + kTileRows * 4);                   // [128][4]
+        const size_t list_base = (size_t)blockIdx.x * kTileRows;  // this CTA's lists
         if (ok) {
             __syncwarp();
             tc_fence_after();
-            const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16);
-            const int nch = (N + 31) / 32;
-            const int my_cols = (sl < nch) ? min(P, N) : 0;  // any columns at all in this slice?
-            int cnt = 0;
-            float pv = 0.f, mx = -INFINITY;
-            int pe = -1;
-            const int slot = (r * 4 + sl) * p.k;
-            for (int j = 0; j < p.k; ++j) {
-                float bv = -INFINITY;
-                int be = 0x7fffffff;
-                for (int ch = sl; ch < nch; ch += 4) {
-                    const int c0 = ch * 32;
-                    float v[32];
-                    tmem_ld32(taddr + c0, v);
-                    tmem_ld_wait();
-                    float cb[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                    int ce[4] = {0x7fffffff, 0x7fffffff, 0x7fffffff, 0x7fffffff};
+            float v[32];
+            int e[32];
+            tmem_ld32(tmem + ((uint32_t)(q * 32) << 16), v);
+            tmem_ld_wait();
+            const int c0 = chunk * kChunk;
+            const int nvalid = min(kChunk, P - c0);
+            float mx = -INFINITY;
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        const int e = c0 + i, u = i & 3;
-                        float x = v[i];
-                        if (x != x) x = -INFINITY;  // NaN never outranks a number
-                        const bool after = (j == 0) || (x < pv) || (x == pv && e > pe);
-                        if (e < P && after && (ce[u] == 0x7fffffff || x > cb[u])) { cb[u] = x; ce[u] = e; }
-                    }
+            for (int i = 0; i < 32; ++i) {
+                float x = v[i];
+                if (x != x) x = -INFINITY;  // NaN never outranks a number
+                const bool in_pool = i < nvalid;
+                v[i] = in_pool ? x : -INFINITY;
+                e[i] = in_pool ? c0 + i : 0x7fffffff;  // columns past the pool rank below every expert
+                mx = in_pool ? fmaxf(mx, x) : mx;
+            }
+            float ssum = 0.f;
+            if (!p.renorm) {
 #pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        if (ce[u] != 0x7fffffff && (be == 0x7fffffff || ranks_above(cb[u], ce[u], bv, be))) {
-                            bv = cb[u];
-                            be = ce[u];
+                for (int i = 0; i < 32; ++i)
+                    if (i < nvalid) ssum += expf(v[i] - mx);
+            }
+            sort32(v, e);
+            const int cnt = min(p.k, nvalid);
+            float2 *lst = p.lists + (list_base + r) * p.k;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)  // constant indices keep v, e in registers
+                if (j < p.k) lst[j] = make_float2(v[j], __int_as_float(e[j]));
+            p.meta[list_base + r] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
+        }
+        // publish, then count this chunk done for the tile; the CTA that
+        // completes the tile merges (the fence orders the lists before the count)
+        __threadfence();
+        asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
+        if (et == 0) s_last = ok && (atomicAdd(&p.tile_done[slot], 1u) == (unsigned)(p.nch[pool] - 1));
+        asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
+        if (s_last) {
+            __threadfence();
+            const int nl = p.nch[pool];
+            const int K = p.k;
+            // shared scratch (the ring is idle: all loads were consumed by the MMAs)
+            float *sv = reinterpret_cast<float *>(dsmem + (sbase - smem_u32(dsmem)));  // [nl][128][K] scores
+            uint16_t *se = reinterpret_cast<uint16_t *>(sv + nl * kTileRows * K);      // [nl][128][K] ids
+            uint16_t *sloc = se + nl * kTileRows * K;                                   // [128][K] rank in expert
+            uint32_t *scnt = reinterpret_cast<uint32_t *>(sloc + ((kTileRows * K + 1) & ~1));  // [P]
+            uint32_t *sbas = scnt + kMaxPool;                                           // [P]
+            float4 *smeta = reinterpret_cast<float4 *>(sbas + kMaxPool);               // [nl][128]
+            const size_t tile_lists = (size_t)slot * p.nch_max * kTileRows;
+            {
+                constexpr int kB = 8;  // loads in flight per thread
+                const int n_ent = nl * kTileRows * K;
+                for (int i0 = et; i0 < n_ent; i0 += kB * kEpi) {
+                    float2 x[kB];
+#pragma unroll
+                    for (int u = 0; u < kB; ++u)
+                        if (i0 + u * kEpi < n_ent) x[u] = __ldcg(p.lists + tile_lists * K + i0 + u * kEpi);
+#pragma unroll
+                    for (int u = 0; u < kB; ++u)
+                        if (i0 + u * kEpi < n_ent) {
+                            sv[i0 + u * kEpi] = x[u].x;
+                            se[i0 + u * kEpi] = (uint16_t)min(__float_as_int(x[u].y), 0xffff);
                         }
                 }
-                if (be == 0x7fffffff) break;  // this slice has no further column
-                lv[slot + j] = bv;
-                li[slot + j] = be;
-                pv = bv;
-                pe = be;
-                if (cnt == 0) mx = bv;
-                ++cnt;
-            }
-            // pool-softmax partial of this slice: sum of exp(x - slice max)
-            float ssum = 0.f;
-            if (!p.renorm && cnt > 0) {
-                for (int ch = sl; ch < nch; ch += 4) {
-                    const int c0 = ch * 32;
-                    float v[32];
-                    tmem_ld32(taddr + c0, v);
-                    tmem_ld_wait();
+                float4 m[kMaxChunks];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        float x = v[i];
-                        if (x != x) x = -INFINITY;
-                        if (c0 + i < P) ssum += expf(x - mx);
-                    }
-                }
-            }
-            (void)my_cols;
-            lcnt[r * 4 + sl] = cnt;
-            lmax[r * 4 + sl] = mx;
-            lsum[r * 4 + sl] = ssum;
-        }
-        // all 16 epilogue warps: slice lists complete before the merge
-        asm volatile("bar.sync 1, %0;\n" ::"r"(32 * kEpiWarps) : "memory");
-        if (ok && sl == 0) {
-            const bool valid = r < rows;
-            const int t = s_tok[r];
-            int head[4], n[4];
+                for (int u = 0; u < kMaxChunks; ++u)
+                    if (u < nl) m[u] = __ldcg(p.meta + tile_lists + u * kTileRows + et);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) { head[u] = 0; n[u] = lcnt[r * 4 + u]; }
+                for (int u = 0; u < kMaxChunks; ++u)
+                    if (u < nl) smeta[u * kTileRows + et] = m[u];
+            }
+            for (int i = et; i < P; i += kEpi) scnt[i] = 0u;
+            asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
+            // merge the chunk lists of token r in chunk order
+            const bool valid = et < rows;
             float sel_v[kMaxTopK];
-            float top = 0.f;
+            int sel_e[kMaxTopK];
+            float top = 0.f, S = 0.f;
             int npriv = 0;
-            for (int j = 0; j < p.k; ++j) {
-                int bu = -1;
-                float bv = 0.f;
-                int be = 0;
+            if (valid) {
+                int head[kMaxChunks], n[kMaxChunks];
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    if (head[u] < n[u]) {
-                        const float x = lv[(r * 4 + u) * p.k + head[u]];
-                        const int e = li[(r * 4 + u) * p.k + head[u]];
-                        if (bu < 0 || ranks_above(x, e, bv, be)) { bu = u; bv = x; be = e; }
+                for (int u = 0; u < kMaxChunks; ++u) {
+                    head[u] = 0;
+                    n[u] = u < nl ? __float_as_int(smeta[u * kTileRows + et].z) : 0;
+                }
+                for (int j = 0; j < K; ++j) {
+                    int bu = -1, be = 0;
+                    float bv = 0.f;
+#pragma unroll
+                    for (int u = 0; u < kMaxChunks; ++u) {
+                        if (head[u] < n[u]) {
+                            const int o = (u * kTileRows + et) * K + head[u];
+                            const float x = sv[o];
+                            const int ee = se[o];
+                            if (bu < 0 || ranks_above(x, ee, bv, be)) { bu = u; bv = x; be = ee; }
+                        }
+                    }
+                    if (bu < 0) break;  // unreachable for k <= pool size
+#pragma unroll
+                    for (int u = 0; u < kMaxChunks; ++u) head[u] += (u == bu) ? 1 : 0;
+                    sel_v[j] = bv;
+                    sel_e[j] = be;
+                    if (j == 0) top = bv;
+                    npriv += base + be >= p.E_pub;
+                    sloc[et * K + j] = (uint16_t)atomicAdd(&scnt[be], 1u);
+                }
+                if (p.renorm) {
+                    for (int j = 0; j < K; ++j) S += expf(sel_v[j] - top);
+                } else {
+                    for (int u = 0; u < nl; ++u) {  // fixed order: deterministic
+                        const float4 m = smeta[u * kTileRows + et];
+                        if (__float_as_int(m.z) > 0) S += m.y * expf(m.x - top);
                     }
                 }
-                if (bu < 0) break;  // unreachable for k <= pool size
-                head[bu] += 1;
-                sel_v[j] = bv;
-                if (j == 0) top = bv;
-                const int gid = base + be;
-                npriv += gid >= p.E_pub;
-                if (valid) {
-                    p.idx[(size_t)t * p.k + j] = gid;
-                    // this row's position among the expert's rows (the dispatch
-                    // stage adds the expert's offset)
-                    p.ticket[(size_t)t * p.k + j] = (int32_t)atomicAdd(&p.counts[gid], 1u);
-                    if (p.route_count) atomicAdd(&p.route_count[gid], 1u);
+            }
+            asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
+            // one global atomic per expert of the tile: the tile's block of rows
+            for (int i = et; i < P; i += kEpi) {
+                const uint32_t c = scnt[i];
+                if (c) {
+                    sbas[i] = atomicAdd(&p.counts[base + i], c);
+                    if (p.route_count) atomicAdd(&p.route_count[base + i], c);
                 }
             }
-            float S = 0.f;
-            if (p.renorm) {
-                for (int j = 0; j < p.k; ++j) S += expf(sel_v[j] - top);
-            } else {
-#pragma unroll
-                for (int u = 0; u < 4; ++u)  // fixed order: deterministic
-                    if (n[u] > 0) S += lsum[r * 4 + u] * expf(lmax[r * 4 + u] - top);
-            }
+            asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
             if (valid) {
-                for (int j = 0; j < p.k; ++j) p.w[(size_t)t * p.k + j] = expf(sel_v[j] - top) / S;
+                const int t = s_tok[et];
+                for (int j = 0; j < K; ++j) {
+                    const int be = sel_e[j];
+                    p.idx[(size_t)t * K + j] = base + be;
+                    p.ticket[(size_t)t * K + j] = (int32_t)(sbas[be] + sloc[et * K + j]);
+                    p.w[(size_t)t * K + j] = expf(sel_v[j] - top) / S;
+                }
                 if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], (unsigned)npriv);
             }
         }
@@ -384,7 +456,7 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem, p.tmem_cols);
+        tmem_dealloc(tmem, kChunk);
     }
 }
 
@@ -396,30 +468,39 @@ __global__ void resolve_kernel(const uint8_t *policy, int T, uint8_t *tau)
 
 }  // namespace
 
+// Chunks of a pool (32 experts each) and the router's per-tile sizes.
+int router_chunks(int pool_size) { return (pool_size + kChunk - 1) / kChunk; }
+int router_slots(int T) { return (T + kTileRows - 1) / kTileRows + 1; }
+
 cudaError_t launch_route(const Ctx &c)
 {
     const Shape &s = c.s;
-    cudaError_t merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
-    if (merr != cudaSuccess) return merr;
     RouterParams p;
     RouterMaps maps;
     memset(&maps, 0, sizeof(maps));
     p.T = s.T; p.H = s.H; p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.k = s.k; p.renorm = s.renorm;
-    int nmax = 0;
-    for (int q = 0; q < 2; ++q) {
-        const int P = q ? s.E_priv : s.E_pub;
-        p.n_pad[q] = ((P < 16 ? 16 : P) + 15) & ~15;
-        p.idesc[q] = make_idesc(kTileRows, p.n_pad[q]);
-        nmax = p.n_pad[q] > nmax ? p.n_pad[q] : nmax;
+    p.nch[0] = router_chunks(s.E_pub);
+    p.nch[1] = router_chunks(s.E_priv);
+    p.nch_max = p.nch[0] > p.nch[1] ? p.nch[0] : p.nch[1];
+    const int slots = router_slots(s.T);
+    // per-expert counters and per-tile completion counts start at zero (the
+    // workspace places them side by side: one memset clears both)
+    cudaError_t merr;
+    if (c.tile_done == c.counts + s.E()) {
+        merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * (s.E() + slots), c.stream);
+    } else {
+        merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
+        if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_done, 0, sizeof(uint32_t) * slots, c.stream);
     }
-    p.tmem_cols = 32;
-    while ((int)p.tmem_cols < nmax) p.tmem_cols <<= 1;
-    p.stage_bytes = (uint32_t)(kABytes + nmax * 128);
-    p.stages = (int)((200u * 1024u) / p.stage_bytes);
-    if (p.stages > kRMaxStages) p.stages = kRMaxStages;
+    if (merr != cudaSuccess) return merr;
+    p.idesc = make_idesc(kTileRows, kChunk);
+    p.stages = kRMaxStages;
     p.policy = c.policy;
     p.hidden = c.hidden;
     p.rows_ws = c.router_rows;
+    p.lists = c.router_lists;
+    p.meta = c.router_meta;
+    p.tile_done = c.tile_done;
     p.tau = c.tau;
     p.idx = c.idx;
     p.w = c.w;
@@ -428,18 +509,16 @@ cudaError_t launch_route(const Ctx &c)
     p.route_count = c.audit.route_count;
     p.route_priv_rows = c.audit.route_priv_rows;
     p.status = c.audit.status;
-    const int grid = (s.T + kTileRows - 1) / kTileRows + 1;
+    const int grid = slots * p.nch_max;
     bool ok = encode_2d(&maps.rows, c.router_rows, s.H, (uint64_t)grid * kTileRows, kTileRows);
     ok &= encode_2d(&maps.hidden, c.hidden, s.H, s.T, kTileRows);
-    ok &= encode_2d(&maps.router[0], c.router_pub, s.H, s.E_pub, p.n_pad[0]);
-    ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, p.n_pad[1]);
+    ok &= encode_2d(&maps.router[0], c.router_pub, s.H, s.E_pub, kChunk);
+    ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, kChunk);
     if (!ok) return cudaErrorInvalidValue;
-    // at least 116 KB of shared memory keeps one router CTA per SM, so the
-    // TMEM allocation never waits for another CTA
-    int smem = p.stages * (int)p.stage_bytes + 1024;
-    if (smem < 116 * 1024) smem = 116 * 1024;
-    const int lists = kTileRows * 4 * (s.k * 8 + 12) + 1024;  // top-k slice lists, reused after the MMAs
-    if (smem < lists) smem = lists;
+    const int ring = p.stages * kStageBytes + 1024;
+    const int merge = p.nch_max * kTileRows * s.k * 6 + kTileRows * s.k * 2 + 4 + 2 * kMaxPool * 4 +
+                      p.nch_max * kTileRows * 16 + 1024 + 16;
+    const int smem = ring > merge ? ring : merge;
     cudaError_t err = cudaFuncSetAttribute(router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (err != cudaSuccess) return err;
     return launch_pdl(router_tc_kernel, dim3(grid), dim3(kRThreads), smem, c.stream, p, maps);

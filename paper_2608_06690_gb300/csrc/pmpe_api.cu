@@ -1,5 +1,6 @@
 // Host side of the C ABI declared in include/pmpe.h: argument validation,
 // the workspace carve-up, stage dispatch and the bounded audit read.
+#include <algorithm>
 #include <chrono>
 #include <thread>
 
@@ -29,6 +30,9 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     };
     L->tau = take(T, 256);
     L->counts = take(4 * E, 256);
+    const size_t slots = (size_t)router_slots(s.T);
+    const size_t rctas = slots * (size_t)std::max(router_chunks(s.E_pub), router_chunks(s.E_priv));
+    L->tile_done = take(4 * slots, 4);
     L->offsets = take(4 * (E + 1), 256);
     L->topk_idx = take(4 * R, 256);
     L->topk_w = take(4 * R, 256);
@@ -36,7 +40,9 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     L->ticket = take(4 * R, 256);
     L->tok_of_slot = take(4 * R, 256);
     L->w_of_slot = take(4 * R, 256);
-    L->router_rows = take(2 * ((T + 127) / 128 + 1) * 128 * (size_t)s.H, 1024);
+    L->router_lists = take(8 * rctas * 128 * (size_t)s.k, 256);
+    L->router_meta = take(16 * rctas * 128, 256);
+    L->router_rows = take(2 * rctas * 128 * (size_t)s.H, 1024);
     L->a_perm = take(2 * R * s.H, 1024);
     L->act = take(2 * R * s.I, 1024);
     L->y = take(2 * R * s.H, 1024);
@@ -116,6 +122,9 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->ticket = (int32_t *)(ws + L.ticket);
     c->tok_of_slot = (int32_t *)(ws + L.tok_of_slot);
     c->w_of_slot = (float *)(ws + L.w_of_slot);
+    c->tile_done = (uint32_t *)(ws + L.tile_done);
+    c->router_lists = (float2 *)(ws + L.router_lists);
+    c->router_meta = (float4 *)(ws + L.router_meta);
     c->router_rows = (bf16 *)(ws + L.router_rows);
     c->a_perm = (bf16 *)(ws + L.a_perm);
     c->act = (bf16 *)(ws + L.act);

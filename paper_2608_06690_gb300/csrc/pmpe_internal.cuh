@@ -50,13 +50,19 @@ struct Ctx {
     int32_t *slot_of, *tok_of_slot;
     int32_t *ticket;    // [T, k] position of each routed row inside its expert
     float *w_of_slot;
-    bf16 *router_rows;  // [(ceil(T/128)+1)*128, H] router tiles' token rows
+    uint32_t *tile_done;  // [router slots] chunk CTAs finished per router tile
+    float2 *router_lists; // [router CTAs * 128, k] per-chunk sorted (score, id)
+    float4 *router_meta;  // [router CTAs * 128] per-chunk softmax partials
+    bf16 *router_rows;  // [router CTAs * 128, H] copied token rows of non-contiguous router tiles
     bf16 *a_perm, *act, *y, *act_sh, *y_sh;
     cudaStream_t stream;
     int num_sms;
 };
 
 int compute_layout(const Shape &s, pmpe_workspace_layout *L);
+// Router geometry: 32-expert chunks of a pool, 128-token tile slots for T tokens.
+int router_chunks(int pool_size);
+int router_slots(int T);
 
 // Launchers (one per stage); each returns the launch's cudaError_t.
 cudaError_t launch_route(const Ctx &c);

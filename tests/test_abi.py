@@ -69,6 +69,22 @@ def test_workspace_size_and_layout(pmpe):
     s2 = LayerShape(T=100, H=256, I=128, E_pub=8, E_priv=4, E_sh=2, k=2, renormalize=False)
     L2 = pmpe.workspace_layout(s2)
     assert L2["y_sh"] >= L2["act_sh"] + 2 * s2.T * s2.E_sh * s2.I
+    # every region lies inside the workspace and no two overlap
+    for sh, LL in ((s, L), (s2, L2)):
+        T, E, R = sh.T, sh.E_pub + sh.E_priv, sh.T * sh.k
+        slots = (T + 127) // 128 + 1
+        ctas = slots * max((sh.E_pub + 31) // 32, (sh.E_priv + 31) // 32)
+        size = dict(tau=T, counts=4 * E, offsets=4 * (E + 1), topk_idx=4 * R, topk_w=4 * R, slot_of=4 * R,
+                    ticket=4 * R, tok_of_slot=4 * R, w_of_slot=4 * R, tile_done=4 * slots,
+                    router_lists=8 * ctas * 128 * sh.k, router_meta=16 * ctas * 128,
+                    router_rows=2 * ctas * 128 * sh.H, a_perm=2 * R * sh.H, act=2 * R * sh.I, y=2 * R * sh.H,
+                    act_sh=2 * T * sh.E_sh * sh.I, y_sh=2 * T * sh.H if sh.E_sh else 0)
+        spans = sorted((LL[n], LL[n] + b, n) for n, b in size.items() if b)
+        for (a0, a1, na), (b0, b1, nb) in zip(spans, spans[1:]):
+            assert a1 <= b0, (na, nb)
+        assert spans[-1][1] <= LL["total"]
+        assert LL["router_meta"] % 16 == 0 and LL["router_lists"] % 8 == 0 and LL["router_rows"] % 1024 == 0
+        assert LL["tile_done"] == LL["counts"] + 4 * E  # one memset clears both
     assert pmpe.workspace_size(LayerShape(64, 200, 128, 8, 4, 0, 2, True)) == 0    # H % 128
     assert pmpe.workspace_size(LayerShape(64, 256, 128, 8, 4, 0, 9, True)) == 0    # k > pool
 
