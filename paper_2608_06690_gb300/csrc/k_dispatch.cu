@@ -13,6 +13,8 @@
 // Combine: out_t = bf16( sum_{j < k} y[slot(t, j)] + y_shared[t] ), summed in
 // FP32 in a fixed order (j ascending, then shared), so the result of a token
 // never depends on the other tokens of the batch.
+#include <algorithm>
+
 #include "pmpe_internal.cuh"
 
 namespace pmpe {
@@ -27,6 +29,7 @@ struct DispatchParams {
     const uint32_t *counts;
     const bf16 *hidden;
     int T, H, R, k, E;
+    int groups;  // warps per token: each stores the row to a share of its k slots
     uint32_t *offsets;
     int32_t *slot_of, *tok_of_slot;
     float *w_of_slot;
@@ -36,8 +39,8 @@ struct DispatchParams {
 
 // Dispatch and gather in one pass.  Every CTA forms the experts' offsets
 // (exclusive prefix sum of the router's per-expert counts) in shared memory;
-// routed row r = (t, j) of expert e goes to slot offset[e] + ticket[r], and its
-// token row is copied there by one warp with 16-byte vectors.
+// routed row r = (t, j) of expert e goes to slot offset[e] + ticket[r].  One
+// warp per token loads the token's row once and stores it to its k slots.
 __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const DispatchParams p)
 {
     __shared__ uint32_t s_off[2 * kMaxPool + 1];
@@ -62,22 +65,33 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
     if (blockIdx.x == 0)
         for (int e = threadIdx.x; e <= p.E; e += kDispThreads) p.offsets[e] = s_off[e];
 
-    // one warp per routed row: the slot is resolved once, then every lane
-    // issues a batch of independent 16-byte loads before its stores
+    // one warp per (token, group of its routed rows): the token's row is
+    // loaded once (16-byte vectors, all in flight together) and stored to the
+    // group's slots; lane j resolves row (t, j)
     const int lane = threadIdx.x & 31;
     const int nv = p.H / 8;
     const int warps = gridDim.x * (kDispThreads / 32);
-    for (int r = blockIdx.x * (kDispThreads / 32) + (threadIdx.x >> 5); r < p.R; r += warps) {
-        const int e = p.idx[r];
-        if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
-            if (lane == 0 && p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
-            continue;
+    const int per = (p.k + p.groups - 1) / p.groups;
+    for (int wi = blockIdx.x * (kDispThreads / 32) + (threadIdx.x >> 5); wi < p.T * p.groups; wi += warps) {
+        const int t = wi / p.groups, gj = wi - t * p.groups;
+        const int j0 = gj * per, j1 = min(p.k, j0 + per);
+        int my_slot = -1;
+        if (lane >= j0 && lane < j1) {
+            const int r = t * p.k + lane;
+            const int e = p.idx[r];
+            if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
+                if (p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+            } else {
+                const int slot = (int)s_off[e] + p.ticket[r];
+                if ((unsigned)slot < (unsigned)p.R) {  // only a corrupt ticket could fail this
+                    my_slot = slot;
+                    p.slot_of[r] = slot;
+                    p.tok_of_slot[slot] = t;
+                    p.w_of_slot[slot] = p.w[r];
+                }
+            }
         }
-        const int slot = (int)s_off[e] + p.ticket[r];
-        if ((unsigned)slot >= (unsigned)p.R) continue;  // only a corrupt ticket could get here
-        const int t = r / p.k;
         const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
-        uint4 *dst = reinterpret_cast<uint4 *>(p.a_perm + (size_t)slot * p.H);
         for (int c0 = 0; c0 < nv; c0 += 32 * 8) {
             uint4 v[8];
 #pragma unroll
@@ -85,16 +99,16 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
                 const int c = c0 + u * 32 + lane;
                 if (c < nv) v[u] = __ldg(src + c);
             }
+            for (int j = j0; j < j1; ++j) {
+                const int slot = __shfl_sync(~0u, my_slot, j);
+                if (slot < 0) continue;
+                uint4 *dst = reinterpret_cast<uint4 *>(p.a_perm + (size_t)slot * p.H);
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const int c = c0 + u * 32 + lane;
-                if (c < nv) dst[c] = v[u];
+                for (int u = 0; u < 8; ++u) {
+                    const int c = c0 + u * 32 + lane;
+                    if (c < nv) dst[c] = v[u];
+                }
             }
-        }
-        if (lane == 0) {
-            p.slot_of[r] = slot;
-            p.tok_of_slot[slot] = t;
-            p.w_of_slot[slot] = p.w[r];
         }
     }
 }
@@ -175,8 +189,12 @@ cudaError_t launch_permute(const Ctx &c)
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.a_perm = c.a_perm;
     p.status = c.audit.status;
-    return launch_pdl(dispatch_gather_kernel, dim3(grid_for((long long)R * 32, c.num_sms)), dim3(kDispThreads), 0,
-                      c.stream, p);
+    // enough warps for about one full wave (32 per SM); a token's row is
+    // loaded once per group
+    const long long want = 32LL * c.num_sms;
+    p.groups = (int)std::min<long long>(s.k, std::max<long long>(1, (want + s.T - 1) / s.T));
+    return launch_pdl(dispatch_gather_kernel, dim3(grid_for((long long)s.T * p.groups * 32, c.num_sms)),
+                      dim3(kDispThreads), 0, c.stream, p);
 }
 
 cudaError_t launch_combine(const Ctx &c)
