@@ -127,8 +127,9 @@ __device__ __forceinline__ void add_bf16x8(float *acc, const uint4 &v)
 // Combine: one thread per (token, 16-byte chunk of the output row).  The k
 // routed rows are loaded in batches of 8 independent 16-byte loads before
 // they are summed (in j order), so the loads overlap instead of forming a
-// chain of dependent memory round trips.
-__global__ void __launch_bounds__(256) combine_kernel(const bf16 *__restrict__ y, const bf16 *__restrict__ y_sh,
+// chain of dependent memory round trips.  Four resident CTAs per SM (at most
+// 64 registers a thread) keep more of those loads in flight.
+__global__ void __launch_bounds__(256, 4) combine_kernel(const bf16 *__restrict__ y, const bf16 *__restrict__ y_sh,
                                                       const int32_t *__restrict__ slot_of, int T, int H, int k,
                                                       bf16 *__restrict__ out)
 {
