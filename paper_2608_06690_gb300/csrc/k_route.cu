@@ -148,6 +148,27 @@ __device__ __forceinline__ void bitonic_sort(float (&v)[32], int (&e)[32])
 // with a bitonic network whose every index is a compile-time constant.
 __device__ __forceinline__ void sort32(float (&v)[32], int (&e)[32]) { bitonic_sort<2>(v, e); }
 
+// The best pair among positions not yet taken (bit i of `taken`), by two
+// interleaved chains of a branch-free scan; returns its position (-1: none).
+__device__ __forceinline__ int best_untaken(const float (&v)[32], const int (&e)[32], uint32_t taken, float &bv,
+                                            int &be)
+{
+    float cv[2] = {-INFINITY, -INFINITY};
+    int ce[2] = {0x7fffffff, 0x7fffffff}, ci[2] = {-1, -1};
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        const int c = i & 1;
+        const bool better = !((taken >> i) & 1u) & ((ci[c] < 0) | ranks_above(v[i], e[i], cv[c], ce[c]));
+        cv[c] = better ? v[i] : cv[c];
+        ce[c] = better ? e[i] : ce[c];
+        ci[c] = better ? i : ci[c];
+    }
+    const bool second = ci[1] >= 0 && (ci[0] < 0 || ranks_above(cv[1], ce[1], cv[0], ce[0]));
+    bv = second ? cv[1] : cv[0];
+    be = second ? ce[1] : ce[0];
+    return second ? ci[1] : ci[0];
+}
+
 __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterParams p,
                                                                   const __grid_constant__ RouterMaps maps)
 {
@@ -306,6 +327,17 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         if (lane == 0) ok = mbar_wait(tfull_bar, 0, &s_abort, p.status) ? 1 : 0;
         ok = __shfl_sync(~0u, ok, 0);
         const size_t list_base = (size_t)blockIdx.x * kTileRows;  // this CTA's lists
+        const int nl = p.nch[pool];
+        const int K = p.k;
+        // A pool of one chunk needs no cross-CTA merge: the CTA keeps its lists
+        // in shared memory and merges at once.  Shared scratch of the merge
+        // (the ring is idle: all loads were consumed by the MMAs):
+        float *sv = reinterpret_cast<float *>(dsmem + (sbase - smem_u32(dsmem)));  // [nl][128][K] scores
+        uint16_t *se = reinterpret_cast<uint16_t *>(sv + nl * kTileRows * K);      // [nl][128][K] ids
+        uint16_t *sloc = se + nl * kTileRows * K;                                   // [128][K] rank in expert
+        uint32_t *scnt = reinterpret_cast<uint32_t *>(sloc + ((kTileRows * K + 1) & ~1));  // [P]
+        uint32_t *sbas = scnt + kMaxPool;                                           // [P]
+        float4 *smeta = reinterpret_cast<float4 *>(sbas + kMaxPool);               // [nl][128]
         if (ok) {
             __syncwarp();
             tc_fence_after();
@@ -331,33 +363,51 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
                 for (int i = 0; i < 32; ++i)
                     if (i < nvalid) ssum += expf(v[i] - mx);
             }
-            sort32(v, e);
-            const int cnt = min(p.k, nvalid);
-            float2 *lst = p.lists + (list_base + r) * p.k;
+            const int cnt = min(K, nvalid);
+            // the chunk's best K pairs in rank order: k selection passes for
+            // small K, the sorting network otherwise
+            float2 *lst = p.lists + (list_base + r) * K;
+            if (K <= 8) {
+                uint32_t taken = nvalid >= 32 ? 0u : ~((1u << nvalid) - 1u);  // columns past the pool
+                for (int j = 0; j < cnt; ++j) {
+                    float bv;
+                    int be;
+                    const int bi = best_untaken(v, e, taken, bv, be);
+                    taken |= 1u << bi;
+                    if (nl == 1) {
+                        sv[r * K + j] = bv;
+                        se[r * K + j] = (uint16_t)be;
+                    } else {
+                        lst[j] = make_float2(bv, __int_as_float(be));
+                    }
+                }
+            } else {
+                sort32(v, e);
 #pragma unroll
-            for (int j = 0; j < 32; ++j)  // constant indices keep v, e in registers
-                if (j < p.k) lst[j] = make_float2(v[j], __int_as_float(e[j]));
-            p.meta[list_base + r] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
+                for (int j = 0; j < 32; ++j)  // constant indices keep v, e in registers
+                    if (j < K) {
+                        if (nl == 1) {
+                            sv[r * K + j] = v[j];
+                            se[r * K + j] = (uint16_t)min(e[j], 0xffff);
+                        } else {
+                            lst[j] = make_float2(v[j], __int_as_float(e[j]));
+                        }
+                    }
+            }
+            if (nl == 1) smeta[r] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
+            else p.meta[list_base + r] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
         }
         // publish, then count this chunk done for the tile; the CTA that
         // completes the tile merges (the fence orders the lists before the count)
-        __threadfence();
+        if (nl > 1) __threadfence();
         asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
-        if (et == 0) s_last = ok && (atomicAdd(&p.tile_done[slot], 1u) == (unsigned)(p.nch[pool] - 1));
+        if (et == 0)
+            s_last = ok && (nl == 1 || atomicAdd(&p.tile_done[slot], 1u) == (unsigned)(nl - 1));
         asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
         if (s_last) {
-            __threadfence();
-            const int nl = p.nch[pool];
-            const int K = p.k;
-            // shared scratch (the ring is idle: all loads were consumed by the MMAs)
-            float *sv = reinterpret_cast<float *>(dsmem + (sbase - smem_u32(dsmem)));  // [nl][128][K] scores
-            uint16_t *se = reinterpret_cast<uint16_t *>(sv + nl * kTileRows * K);      // [nl][128][K] ids
-            uint16_t *sloc = se + nl * kTileRows * K;                                   // [128][K] rank in expert
-            uint32_t *scnt = reinterpret_cast<uint32_t *>(sloc + ((kTileRows * K + 1) & ~1));  // [P]
-            uint32_t *sbas = scnt + kMaxPool;                                           // [P]
-            float4 *smeta = reinterpret_cast<float4 *>(sbas + kMaxPool);               // [nl][128]
-            const size_t tile_lists = (size_t)slot * p.nch_max * kTileRows;
-            {
+            if (nl > 1) {
+                __threadfence();
+                const size_t tile_lists = (size_t)slot * p.nch_max * kTileRows;
                 constexpr int kB = 8;  // loads in flight per thread
                 const int n_ent = nl * kTileRows * K;
                 for (int i0 = et; i0 < n_ent; i0 += kB * kEpi) {
