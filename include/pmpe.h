@@ -142,6 +142,8 @@ typedef struct pmpe_workspace_layout {
     size_t tile_done;    /* uint32 [S]      router CTAs finished per 128-token tile */
     size_t router_lists; /* float2 [C*128, k] per 32-expert chunk: each token's best k (score, id) */
     size_t router_meta;  /* float4 [C*128]  per chunk: max score, sum exp(score - max), entries */
+    size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1]  gate/up epilogue warps done per
+                          * (expert group, 128-row block), read by the down tiles of the same launch */
 } pmpe_workspace_layout;
 PMPE_API int pmpe_moe_workspace_layout(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k,
                               pmpe_workspace_layout *out);

@@ -57,68 +57,92 @@ constexpr int kDynSmem = kStages * kStageBytes + kOutBytes + 1024 /* alignment s
 
 enum { kGateUp = 0, kDown = 1 };
 
-struct TcParams {
+// One GEMM of the layer: gate/up (SwiGLU fused) or down (routing weight fused).
+struct TcPhase {
     int mode;
-    int E, E_pub, E_sh, T, H, I, R;
     int bn;           // output columns per tile (gate/up: 128 activation columns; down: 256 or 128)
     uint32_t idesc;   // tcgen05 instruction descriptor (BF16 x BF16 -> FP32, M = 128, N = MMA width)
-    uint32_t tx_bytes;
-    const uint32_t *offsets;
     bf16 *C_routed, *C_shared;
+};
+
+struct TcParams {
+    int nph;          // 1: the GEMM of ph[0]; 2: gate/up (ph[0]) then down (ph[1]) in one persistent grid
+    TcPhase ph[2];
+    int E, E_pub, E_sh, T, H, I, R;
+    const uint32_t *offsets;
     const float *w_of_slot;
     const int32_t *tok_of_slot;
+    // nph == 2: per (group, 128-row block), the gate/up epilogue warps whose
+    // activations are stored (zeroed before the launch)
+    uint32_t *ready;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
 };
 
-struct TcMaps {
-    CUtensorMap c_routed, c_shared;  // outputs, 32 x 32 boxes, 64-byte swizzle
-    CUtensorMap a_routed, a_shared;
-    CUtensorMap b0[3];  // per pool [pub, priv, shared]: gate (gate/up mode) or down
-    CUtensorMap b1[3];  // up (gate/up mode)
+struct TcMaps {  // [phase]
+    CUtensorMap c_routed[2], c_shared[2];  // outputs, 32 x 32 boxes, 64-byte swizzle
+    CUtensorMap a_routed[2], a_shared[2];
+    CUtensorMap b0[2][3];  // per pool [pub, priv, shared]: gate (gate/up) or down
+    CUtensorMap b1[2][3];  // up (gate/up)
 };
 
 // ------------------------------------------------------------- tile list
 
 struct Tile {
-    int g, m0, n0, rows, row_base, nkb;
+    int ph, mode, bn, g, m_tile, m0, n0, rows, row_base, nkb;
     bool shared;
 };
 
 struct TileTable {
-    int prefix[kMaxGroups + 1];
+    int prefix[2][kMaxGroups + 1];  // tiles of the groups before g, per phase
+    int mpre[kMaxGroups + 1];       // 128-row blocks of the groups before g
     int rows[kMaxGroups];
     int base[kMaxGroups];
 };
 
-__device__ __forceinline__ int group_n(const TcParams &p, bool shared)
+__device__ __forceinline__ int group_n(const TcParams &p, int mode, bool shared)
 {
-    return p.mode == kGateUp ? (shared ? p.E_sh * p.I : p.I) : p.H;
+    return mode == kGateUp ? (shared ? p.E_sh * p.I : p.I) : p.H;
 }
-__device__ __forceinline__ int group_k(const TcParams &p, bool shared)
+__device__ __forceinline__ int group_k(const TcParams &p, int mode, bool shared)
 {
-    return p.mode == kGateUp ? p.H : (shared ? p.E_sh * p.I : p.I);
+    return mode == kGateUp ? p.H : (shared ? p.E_sh * p.I : p.I);
 }
 
+// Tile `tile` of the list: the tiles of phase 0 (all groups), then those of
+// phase 1; inside a phase, group by group, n-tile major.
 __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &tt, int G, int tile)
 {
-    int lo = 0, hi = G - 1;  // last group with prefix <= tile
+    Tile t;
+    t.ph = (p.nph == 2 && tile >= tt.prefix[0][G]) ? 1 : 0;
+    const int local_all = tile - (t.ph ? tt.prefix[0][G] : 0);
+    const int *pre = tt.prefix[t.ph];
+    int lo = 0, hi = G - 1;  // last group with prefix <= local_all
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
-        if (tt.prefix[mid] <= tile) lo = mid; else hi = mid - 1;
+        if (pre[mid] <= local_all) lo = mid; else hi = mid - 1;
     }
-    Tile t;
+    t.mode = p.ph[t.ph].mode;
+    t.bn = p.ph[t.ph].bn;
     t.g = lo;
     t.shared = lo >= p.E;
     const int rows = tt.rows[lo];
     const int mt = (rows + BM - 1) / BM;
-    const int local = tile - tt.prefix[lo];
-    const int n_tile = local / mt, m_tile = local - n_tile * mt;
-    t.m0 = m_tile * BM;
-    t.n0 = n_tile * p.bn;
+    const int local = local_all - pre[lo];
+    const int n_tile = local / mt;
+    t.m_tile = local - n_tile * mt;
+    t.m0 = t.m_tile * BM;
+    t.n0 = n_tile * t.bn;
     t.rows = min(BM, rows - t.m0);
     t.row_base = tt.base[lo];
-    t.nkb = group_k(p, t.shared) / BK;
+    t.nkb = group_k(p, t.mode, t.shared) / BK;
     return t;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *ptr)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];\n" : "=r"(v) : "l"(ptr) : "memory");
+    return v;
 }
 
 // ---------------------------------------------------------------- kernel
@@ -156,7 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
     }
     pdl_wait();  // the dispatch offsets and the A operand come from the previous kernels
-    // tile list: rows and tiles per group, prefix over groups
+    // tile list: rows and tiles per group, prefixes over groups
     for (int g = tid; g < G; g += kThreads) {
         const bool shared = g >= p.E;
         int rows, base;
@@ -168,32 +192,36 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             rows = e - b;
             base = b;
         }
+        const int mt = (rows + BM - 1) / BM;
         tt.rows[g] = rows;
         tt.base[g] = base;
-        tt.prefix[g + 1] = ((rows + BM - 1) / BM) * (group_n(p, shared) / p.bn);
+        tt.mpre[g + 1] = mt;
+        for (int ph = 0; ph < 2; ++ph)
+            tt.prefix[ph][g + 1] = ph < p.nph ? mt * (group_n(p, p.ph[ph].mode, shared) / p.ph[ph].bn) : 0;
     }
     __syncthreads();
-    if (warp == 0) {
+    if (warp < 3) {  // three inclusive scans, one per warp: tiles of phase 0, of phase 1, row blocks
+        int *arr = warp == 2 ? tt.mpre : tt.prefix[warp];
         int carry = 0;
         for (int b = 0; b < G; b += 32) {
-            int v = b + lane < G ? tt.prefix[b + lane + 1] : 0;
+            int v = b + lane < G ? arr[b + lane + 1] : 0;
 #pragma unroll
             for (int off = 1; off < 32; off <<= 1) {
                 const int y = __shfl_up_sync(~0u, v, off);
                 if (lane >= off) v += y;
             }
             __syncwarp();
-            if (b + lane < G) tt.prefix[b + lane + 1] = carry + v;
+            if (b + lane < G) arr[b + lane + 1] = carry + v;
             carry += __shfl_sync(~0u, v, 31);
         }
-        if (lane == 0) tt.prefix[0] = 0;
+        if (lane == 0) arr[0] = 0;
     }
     __syncwarp();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
-    const int total = tt.prefix[G];
+    const int total = tt.prefix[0][G] + (p.nph == 2 ? tt.prefix[1][G] : 0);
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
@@ -206,34 +234,54 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         int stage = 0;
         uint32_t phase = 0;
         uint32_t filled = 0, last_parity = 0;  // per-stage bits, for the drain below
-        const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes
-                                         : (p.mode == kGateUp ? (uint32_t)(BM * 128) : (uint32_t)(p.bn / 2 * 128));
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
             const int q = t.shared ? 2 : (t.g < p.E_pub ? 0 : 1);
             const int ei = t.shared ? 0 : (q == 0 ? t.g : t.g - p.E_pub);
-            const CUtensorMap *amap = t.shared ? &maps.a_shared : &maps.a_routed;
+            const CUtensorMap *amap = t.shared ? &maps.a_shared[t.ph] : &maps.a_routed[t.ph];
             const int arow = t.row_base + t.m0;
+            const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes
+                                             : (t.mode == kGateUp ? (uint32_t)(BM * 128) : (uint32_t)(t.bn / 2 * 128));
             bool ok = true;
-            for (int kb = 0; kb < t.nkb; ++kb) {
+            if (t.ph == 1 && lane == 0) {
+                // a down tile of the persistent pair: its activation rows are
+                // complete once every gate/up epilogue warp of their row block
+                // has stored its part (bounded wait; the weights are loaded meanwhile)
+                const uint32_t need = 4u * (uint32_t)(group_n(p, kGateUp, t.shared) / p.ph[0].bn);
+                const uint32_t *rp = p.ready + tt.mpre[t.g] + t.m_tile;
+                const unsigned long long t0 = globaltimer_ns();
+                while (ld_acquire_gpu(rp) < need) {
+                    if (s_abort) { ok = false; break; }
+                    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                        s_abort = 1;
+                        if (p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
+                    __nanosleep(128);
+                }
+                // the async proxy (TMA) reads what the generic acquire observed
+                asm volatile("fence.proxy.async.global;\n" ::: "memory");
+            }
+            for (int kb = 0; kb < t.nkb && ok; ++kb) {
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
                 const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
                 mbar_expect_tx(full_bar(stage), my_tx);
                 const int kx = kb * BK;
                 if (lane == 0) {
                     tma_load_2d(sA, amap, full_bar(stage), kx, arow);
-                } else if (p.mode == kGateUp) {
+                } else if (t.mode == kGateUp) {
                     const int brow = ei * p.I + t.n0;  // shared: n0 spans E_sh * I rows
-                    tma_load_2d(sB + (lane - 1) * BM * 128, lane == 1 ? &maps.b0[q] : &maps.b1[q], full_bar(stage), kx,
-                                brow);
+                    tma_load_2d(sB + (lane - 1) * BM * 128, lane == 1 ? &maps.b0[t.ph][q] : &maps.b1[t.ph][q],
+                                full_bar(stage), kx, brow);
                 } else {
-                    const int half = (lane - 1) * (p.bn / 2);
+                    const int half = (lane - 1) * (t.bn / 2);
                     if (t.shared) {
                         const int sidx = kx / p.I;
-                        tma_load_2d(sB + half * 128, &maps.b0[2], full_bar(stage), kx - sidx * p.I,
+                        tma_load_2d(sB + half * 128, &maps.b0[t.ph][2], full_bar(stage), kx - sidx * p.I,
                                     sidx * p.H + t.n0 + half);
                     } else {
-                        tma_load_2d(sB + half * 128, &maps.b0[q], full_bar(stage), kx, ei * p.H + t.n0 + half);
+                        tma_load_2d(sB + half * 128, &maps.b0[t.ph][q], full_bar(stage), kx, ei * p.H + t.n0 + half);
                     }
                 }
                 filled |= 1u << stage;
@@ -255,6 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         uint32_t phase = 0;
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x, ++it) {
             const Tile t = decode_tile(p, tt, G, tile);
+            const uint32_t idesc = p.ph[t.ph].idesc;
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
             if (!mbar_wait(tempty_bar(buf), use ^ 1u, &s_abort, p.status)) break;
@@ -268,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 const uint64_t ad = sw128_desc(sA), bd = sw128_desc(sB);
 #pragma unroll
                 for (int k = 0; k < BK / 16; ++k)  // +32 bytes of K per step inside the swizzle row
-                    tc_mma(d_tmem, ad + 2 * k, bd + 2 * k, p.idesc, (kb | k) != 0);
+                    tc_mma(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
                 tc_commit(empty_bar(stage));
                 if (++stage == kStages) { stage = 0; phase ^= 1u; }
             }
@@ -299,6 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             if (!ok) break;
             __syncwarp();
             tc_fence_after();
+            const TcPhase &ph = p.ph[t.ph];
             const int r = quarter * 32 + lane;  // tile row of this thread
             const bool valid = r < t.rows;
             const int grow = t.row_base + t.m0 + r;
@@ -307,15 +357,15 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             // the block holding a tile's last rows is written row by row so that
             // it never touches the next expert's rows.
             const bool full_block = (t.rows - quarter * 32) >= 32;
-            const int ldc = p.mode == kGateUp ? (t.shared ? p.E_sh * p.I : p.I) : p.H;
-            bf16 *crow = (t.shared ? p.C_shared : p.C_routed) + (size_t)grow * ldc + t.n0;
-            const CUtensorMap *cmap = t.shared ? &maps.c_shared : &maps.c_routed;
-            const int nchunks = p.mode == kGateUp ? BM / 32 : p.bn / 32;
-            const float sc = (p.mode == kGateUp || t.shared) ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
+            const int ldc = t.mode == kGateUp ? (t.shared ? p.E_sh * p.I : p.I) : p.H;
+            bf16 *crow = (t.shared ? ph.C_shared : ph.C_routed) + (size_t)grow * ldc + t.n0;
+            const CUtensorMap *cmap = t.shared ? &maps.c_shared[t.ph] : &maps.c_routed[t.ph];
+            const int nchunks = t.mode == kGateUp ? BM / 32 : t.bn / 32;
+            const float sc = (t.mode == kGateUp || t.shared) ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
 #pragma unroll 1
             for (int c = 0; c < nchunks; ++c) {
                 uint32_t pk[16];
-                if (p.mode == kGateUp) {
+                if (t.mode == kGateUp) {
                     float gv[32], uv[32];
                     tmem_ld32(taddr + c * 32, gv);
                     tmem_ld32(taddr + 128 + c * 32, uv);
@@ -360,7 +410,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty_bar(buf));
             // execution audit: rows this tile processed, counted where they ran
-            if (p.mode == kGateUp) {
+            if (t.mode == kGateUp) {
                 const unsigned vm = __ballot_sync(~0u, valid);
                 if (!t.shared && t.n0 == 0) {
                     if (lane == 0 && p.exec_rows && vm) atomicAdd(&p.exec_rows[t.g], (unsigned)__popc(vm));
@@ -369,6 +419,20 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 }
                 if (t.shared && p.shared_rows && lane == 0 && vm && (t.n0 % p.I) == 0)
                     atomicAdd(p.shared_rows, (unsigned)__popc(vm));
+            }
+            if (p.nph == 2 && t.ph == 0) {
+                // release this warp's activation rows to the down tiles that read
+                // them: the row stores (generic) and the TMA stores (async proxy,
+                // complete after wait_group 0) are ordered before the count
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) {
+                    bulk_wait_all();
+                    asm volatile("fence.proxy.async.global;\n" ::: "memory");
+                    __threadfence();
+                    atomicAdd(p.ready + tt.mpre[t.g] + t.m_tile, 1u);
+                }
+                __syncwarp();
             }
         }
         if (lane == 0) bulk_wait_all();  // this warp's TMA stores are complete before the CTA exits
@@ -388,64 +452,76 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
 
 // ------------------------------------------------------------ host side
 
-cudaError_t launch_tc(const Ctx &c, int mode)
+// Parameters and tensor maps of one GEMM (`mode`) as phase `ph` of a launch.
+bool fill_phase(const Ctx &c, int mode, int ph, TcParams &p, TcMaps &maps)
+{
+    const Shape &s = c.s;
+    const uint64_t R = (uint64_t)s.T * s.k, T = (uint64_t)s.T;
+    TcPhase &f = p.ph[ph];
+    f.mode = mode;
+    bool ok = true;
+    if (mode == kGateUp) {
+        f.bn = 128;
+        f.idesc = make_idesc(BM, 256);
+        f.C_routed = c.act;
+        f.C_shared = c.act_sh;
+        ok &= encode_2d_box(&maps.c_routed[ph], c.act, s.I, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        if (s.E_sh > 0)
+            ok &= encode_2d_box(&maps.c_shared[ph], c.act_sh, (uint64_t)s.E_sh * s.I, T, kOutBox, kOutBox,
+                                CU_TENSOR_MAP_SWIZZLE_64B);
+        ok &= encode_2d(&maps.a_routed[ph], c.a_perm, s.H, R, BM);
+        for (int q = 0; q < 2; ++q) {
+            const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.I;
+            ok &= encode_2d(&maps.b0[ph][q], c.gate[q], s.H, n, 128);
+            ok &= encode_2d(&maps.b1[ph][q], c.up[q], s.H, n, 128);
+        }
+        if (s.E_sh > 0) {
+            ok &= encode_2d(&maps.a_shared[ph], c.hidden, s.H, T, BM);
+            ok &= encode_2d(&maps.b0[ph][2], c.gate[2], s.H, (uint64_t)s.E_sh * s.I, 128);
+            ok &= encode_2d(&maps.b1[ph][2], c.up[2], s.H, (uint64_t)s.E_sh * s.I, 128);
+        }
+    } else {
+        f.bn = (s.H % 256 == 0) ? 256 : 128;
+        f.idesc = make_idesc(BM, f.bn);
+        f.C_routed = c.y;
+        f.C_shared = c.y_sh;
+        ok &= encode_2d_box(&maps.c_routed[ph], c.y, s.H, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        if (s.E_sh > 0)
+            ok &= encode_2d_box(&maps.c_shared[ph], c.y_sh, s.H, T, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        ok &= encode_2d(&maps.a_routed[ph], c.act, s.I, R, BM);
+        for (int q = 0; q < 2; ++q) {
+            const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
+            ok &= encode_2d(&maps.b0[ph][q], c.down[q], s.I, n, f.bn / 2);
+        }
+        if (s.E_sh > 0) {
+            ok &= encode_2d(&maps.a_shared[ph], c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
+            ok &= encode_2d(&maps.b0[ph][2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, f.bn / 2);
+        }
+    }
+    return ok;
+}
+
+// One persistent launch running the GEMMs of `modes` in order (one or two).
+cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
 {
     const Shape &s = c.s;
     TcParams p;
     TcMaps maps;
+    memset(&p, 0, sizeof(p));
     memset(&maps, 0, sizeof(maps));
-    p.mode = mode;
+    p.nph = nph;
     p.E = s.E(); p.E_pub = s.E_pub; p.E_sh = s.E_sh; p.T = s.T; p.H = s.H; p.I = s.I; p.R = s.T * s.k;
     p.offsets = c.offsets;
     p.w_of_slot = c.w_of_slot;
     p.tok_of_slot = c.tok_of_slot;
+    p.ready = c.gemm_ready;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
     p.exec_priv_rows = c.audit.exec_priv_rows;
     p.shared_rows = c.audit.shared_rows;
     p.status = c.audit.status;
-    const uint64_t R = (uint64_t)p.R, T = (uint64_t)s.T;
     bool ok = true;
-    if (mode == kGateUp) {
-        p.bn = 128;
-        p.idesc = make_idesc(BM, 256);
-        p.tx_bytes = kABytes + 2 * 128 * BK * 2;
-        p.C_routed = c.act;
-        p.C_shared = c.act_sh;
-        ok &= encode_2d_box(&maps.c_routed, c.act, s.I, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
-        if (s.E_sh > 0)
-            ok &= encode_2d_box(&maps.c_shared, c.act_sh, (uint64_t)s.E_sh * s.I, T, kOutBox, kOutBox,
-                                CU_TENSOR_MAP_SWIZZLE_64B);
-        ok &= encode_2d(&maps.a_routed, c.a_perm, s.H, R, BM);
-        for (int q = 0; q < 2; ++q) {
-            const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.I;
-            ok &= encode_2d(&maps.b0[q], c.gate[q], s.H, n, 128);
-            ok &= encode_2d(&maps.b1[q], c.up[q], s.H, n, 128);
-        }
-        if (s.E_sh > 0) {
-            ok &= encode_2d(&maps.a_shared, c.hidden, s.H, T, BM);
-            ok &= encode_2d(&maps.b0[2], c.gate[2], s.H, (uint64_t)s.E_sh * s.I, 128);
-            ok &= encode_2d(&maps.b1[2], c.up[2], s.H, (uint64_t)s.E_sh * s.I, 128);
-        }
-    } else {
-        p.bn = (s.H % 256 == 0) ? 256 : 128;
-        p.idesc = make_idesc(BM, p.bn);
-        p.tx_bytes = kABytes + p.bn * BK * 2;
-        p.C_routed = c.y;
-        p.C_shared = c.y_sh;
-        ok &= encode_2d_box(&maps.c_routed, c.y, s.H, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
-        if (s.E_sh > 0)
-            ok &= encode_2d_box(&maps.c_shared, c.y_sh, s.H, T, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
-        ok &= encode_2d(&maps.a_routed, c.act, s.I, R, BM);
-        for (int q = 0; q < 2; ++q) {
-            const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
-            ok &= encode_2d(&maps.b0[q], c.down[q], s.I, n, p.bn / 2);
-        }
-        if (s.E_sh > 0) {
-            ok &= encode_2d(&maps.a_shared, c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
-            ok &= encode_2d(&maps.b0[2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, p.bn / 2);
-        }
-    }
+    for (int ph = 0; ph < nph; ++ph) ok &= fill_phase(c, modes[ph], ph, p, maps);
     if (!ok) return cudaErrorInvalidValue;
     cudaError_t err = cudaFuncSetAttribute(expert_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem);
     if (err != cudaSuccess) return err;
@@ -453,6 +529,26 @@ cudaError_t launch_tc(const Ctx &c, int mode)
 }
 
 }  // namespace
+
+cudaError_t launch_gateup(const Ctx &c)
+{
+    const int m[1] = {kGateUp};
+    return launch_tc(c, 1, m);
+}
+cudaError_t launch_down(const Ctx &c)
+{
+    const int m[1] = {kDown};
+    return launch_tc(c, 1, m);
+}
+cudaError_t launch_experts(const Ctx &c, bool zero_ready)
+{
+    if (zero_ready) {
+        const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
+        if (err != cudaSuccess) return err;
+    }
+    const int m[2] = {kGateUp, kDown};
+    return launch_tc(c, 2, m);
+}
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 {
@@ -499,7 +595,5 @@ uint32_t make_idesc(int M, int N)
            | ((uint32_t)(M >> 4) << 24);// M / 16   (A and B K-major: transpose bits 15, 16 = 0)
 }
 
-cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, kGateUp); }
-cudaError_t launch_down(const Ctx &c) { return launch_tc(c, kDown); }
 
 }  // namespace pmpe

@@ -533,14 +533,17 @@ cudaError_t launch_route(const Ctx &c)
     p.nch[1] = router_chunks(s.E_priv);
     p.nch_max = p.nch[0] > p.nch[1] ? p.nch[0] : p.nch[1];
     const int slots = router_slots(s.T);
-    // per-expert counters and per-tile completion counts start at zero (the
-    // workspace places them side by side: one memset clears both)
+    // per-expert counters, per-tile completion counts and the expert GEMMs'
+    // readiness counters start at zero (the workspace places them side by
+    // side: one memset clears all three)
     cudaError_t merr;
-    if (c.tile_done == c.counts + s.E()) {
-        merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * (s.E() + slots), c.stream);
+    const size_t nready = gemm_ready_words(s);
+    if (c.tile_done == c.counts + s.E() && c.gemm_ready == c.tile_done + slots) {
+        merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * (s.E() + slots + nready), c.stream);
     } else {
         merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
         if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_done, 0, sizeof(uint32_t) * slots, c.stream);
+        if (merr == cudaSuccess) merr = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * nready, c.stream);
     }
     if (merr != cudaSuccess) return merr;
     p.idesc = make_idesc(kTileRows, kChunk);

@@ -10,6 +10,14 @@ namespace pmpe {
 
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Each routed group adds at most one partial 128-row block beyond R/128; the
+// shared-expert group covers the T tokens.
+size_t gemm_ready_words(const Shape &s)
+{
+    const size_t R = (size_t)s.T * (size_t)s.k;
+    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 1;
+}
+
 static bool shape_ok(const Shape &s)
 {
     return s.T >= 0 && s.H > 0 && s.I > 0 && s.k >= 1 && s.k <= kMaxTopK && s.E_pub >= s.k && s.E_priv >= s.k &&
@@ -33,6 +41,7 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     const size_t slots = (size_t)router_slots(s.T);
     const size_t rctas = slots * (size_t)std::max(router_chunks(s.E_pub), router_chunks(s.E_priv));
     L->tile_done = take(4 * slots, 4);
+    L->gemm_ready = take(4 * gemm_ready_words(s), 4);
     L->offsets = take(4 * (E + 1), 256);
     L->topk_idx = take(4 * R, 256);
     L->topk_w = take(4 * R, 256);
@@ -123,6 +132,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->tok_of_slot = (int32_t *)(ws + L.tok_of_slot);
     c->w_of_slot = (float *)(ws + L.w_of_slot);
     c->tile_done = (uint32_t *)(ws + L.tile_done);
+    c->gemm_ready = (uint32_t *)(ws + L.gemm_ready);
     c->router_lists = (float2 *)(ws + L.router_lists);
     c->router_meta = (float4 *)(ws + L.router_meta);
     c->router_rows = (bf16 *)(ws + L.router_rows);
@@ -183,8 +193,14 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     cudaError_t err = cudaSuccess;
     if (err == cudaSuccess && (stages & PMPE_STAGE_ROUTE)) err = launch_route(c);
     if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE)) err = launch_permute(c);
-    if (err == cudaSuccess && (stages & PMPE_STAGE_GATEUP)) err = launch_gateup(c);
-    if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c);
+    if ((stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN)) {
+        // one persistent launch; its readiness counters are cleared by the
+        // router's memset when the router runs in this call
+        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_ROUTE));
+    } else {
+        if (err == cudaSuccess && (stages & PMPE_STAGE_GATEUP)) err = launch_gateup(c);
+        if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c);
+    }
     if (err == cudaSuccess && (stages & PMPE_STAGE_COMBINE)) err = launch_combine(c);
     return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
 }

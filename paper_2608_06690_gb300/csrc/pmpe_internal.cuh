@@ -51,6 +51,7 @@ struct Ctx {
     int32_t *ticket;    // [T, k] position of each routed row inside its expert
     float *w_of_slot;
     uint32_t *tile_done;  // [router slots] chunk CTAs finished per router tile
+    uint32_t *gemm_ready; // [gemm_ready_words] gate/up warps done per (group, 128-row block)
     float2 *router_lists; // [router CTAs * 128, k] per-chunk sorted (score, id)
     float4 *router_meta;  // [router CTAs * 128] per-chunk softmax partials
     bf16 *router_rows;  // [router CTAs * 128, H] copied token rows of non-contiguous router tiles
@@ -63,12 +64,18 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L);
 // Router geometry: 32-expert chunks of a pool, 128-token tile slots for T tokens.
 int router_chunks(int pool_size);
 int router_slots(int T);
+// Readiness counters of the persistent expert GEMMs: one per (group, 128-row
+// block), an upper bound over all routings.
+size_t gemm_ready_words(const Shape &s);
 
 // Launchers (one per stage); each returns the launch's cudaError_t.
 cudaError_t launch_route(const Ctx &c);
 cudaError_t launch_permute(const Ctx &c);
 cudaError_t launch_gateup(const Ctx &c);
 cudaError_t launch_down(const Ctx &c);
+// Gate/up and down in one persistent launch (down tiles wait for their
+// activation rows); zero_ready clears the readiness counters first.
+cudaError_t launch_experts(const Ctx &c, bool zero_ready);
 cudaError_t launch_combine(const Ctx &c);
 cudaError_t launch_resolve(const uint8_t *policy, int T, uint8_t *tau, cudaStream_t stream);
 

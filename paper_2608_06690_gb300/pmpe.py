@@ -44,7 +44,7 @@ STAGE_ALL = 0x1F
 # Kernels one full forward launches: router/top-k (with the policy resolve),
 # dispatch + row gather, gate/up GEMM, down GEMM, combine (plus one memset of
 # the per-expert counters, which is not a kernel of this library).
-KERNELS_PER_FORWARD = 5
+KERNELS_PER_FORWARD = 4
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
@@ -72,7 +72,7 @@ class MoeDesc(ctypes.Structure):
 class WorkspaceLayout(ctypes.Structure):
     _fields_ = [(n, ctypes.c_size_t) for n in ("total", "tau", "counts", "offsets", "topk_idx", "topk_w", "slot_of", "ticket",
                                                 "tok_of_slot", "w_of_slot", "router_rows", "a_perm", "act", "y", "act_sh", "y_sh",
-                                                "tile_done", "router_lists", "router_meta")]
+                                                "tile_done", "router_lists", "router_meta", "gemm_ready")]
 
 
 _lib.pmpe_moe_workspace_size.restype = ctypes.c_size_t
