@@ -227,3 +227,28 @@ def test_audit_read_reports_status_and_accumulates():
     audit[0] = 1   # a status bit set by a kernel is reported as an error
     with pytest.raises(pmpe.PmpeError):
         pmpe.audit_read(audit, shape.T, shape.E)
+
+
+def test_persistent_gemm_pair_matches_separate_launches():
+    """The forward runs gate/up and down in one persistent launch, down tiles
+    waiting for their activation rows; launching the two GEMMs one after the
+    other computes every tile the same way, so the outputs are bitwise equal.
+    Shared experts and ragged tiles are included."""
+    from paper_2608_06690_gb300 import pmpe
+    shape = LayerShape(T=700, H=256, I=256, E_pub=16, E_priv=8, E_sh=2, k=3, renormalize=False)
+    w, h, pol = make_layer(shape, 45)
+    wd, hd, pd = to_device(w, h, pol)
+    layer = pmpe.MoeLayer(shape, wd)
+    fused = layer.forward(hd, pd).clone()
+    split = torch.full_like(fused, float("nan"))
+    for st in (pmpe.STAGE_ROUTE | pmpe.STAGE_PERMUTE, pmpe.STAGE_GATEUP, pmpe.STAGE_DOWN, pmpe.STAGE_COMBINE):
+        layer.forward(hd, pd, out=split, stages=st)
+    torch.cuda.synchronize()
+    assert torch.equal(fused.view(torch.int16), split.view(torch.int16))
+    # and the pair alone, with its counters cleared by its own launch
+    again = torch.full_like(fused, float("nan"))
+    layer.forward(hd, pd, out=again, stages=pmpe.STAGE_ROUTE | pmpe.STAGE_PERMUTE)
+    layer.forward(hd, pd, out=again, stages=pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN)
+    layer.forward(hd, pd, out=again, stages=pmpe.STAGE_COMBINE)
+    torch.cuda.synchronize()
+    assert torch.equal(fused.view(torch.int16), again.view(torch.int16))
