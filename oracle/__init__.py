@@ -44,6 +44,7 @@ class _Layer(ctypes.Structure):
         ("gate_pub", _u16p), ("up_pub", _u16p), ("down_pub", _u16p),
         ("gate_priv", _u16p), ("up_priv", _u16p), ("down_priv", _u16p),
         ("gate_sh", _u16p), ("up_sh", _u16p), ("down_sh", _u16p),
+        ("unmasked", ctypes.c_int),
     ]
 
 
@@ -106,10 +107,12 @@ class Layer:
     ``tensors`` maps names (hidden, router_pub, router_priv, gate_pub, up_pub,
     down_pub, gate_priv, up_priv, down_priv, and optionally gate_sh, up_sh,
     down_sh) to BF16 tensors or uint16 arrays; ``policy`` is a uint8 array of
-    T bytes or None (missing metadata).
+    T bytes or None (missing metadata).  ``unmasked`` selects the paper's
+    soft-router control: routing over the concatenated pool without the hard
+    mask (a negative control, not the method).
     """
 
-    def __init__(self, shape, tensors: dict, policy):
+    def __init__(self, shape, tensors: dict, policy, unmasked: bool = False):
         self.shape = shape
         self._keep = {}
         for name in ("hidden", "router_pub", "router_priv", "gate_pub", "up_pub", "down_pub",
@@ -128,7 +131,8 @@ class Layer:
                         _ptr(k["router_pub"], _u16p), _ptr(k["router_priv"], _u16p),
                         _ptr(k["gate_pub"], _u16p), _ptr(k["up_pub"], _u16p), _ptr(k["down_pub"], _u16p),
                         _ptr(k["gate_priv"], _u16p), _ptr(k["up_priv"], _u16p), _ptr(k["down_priv"], _u16p),
-                        _ptr(k["gate_sh"], _u16p), _ptr(k["up_sh"], _u16p), _ptr(k["down_sh"], _u16p))
+                        _ptr(k["gate_sh"], _u16p), _ptr(k["up_sh"], _u16p), _ptr(k["down_sh"], _u16p),
+                        int(bool(unmasked)))
 
 
 def bf16_round(x: float) -> int:

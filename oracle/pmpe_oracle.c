@@ -39,6 +39,10 @@
  *     architecture (gate, up, down projections: a SwiGLU MLP).
  *   - Sec. 5.2 / App. F.1: independent execution counts observed at the
  *     expert modules themselves, separate from the route log.
+ *   - Sec. 4.3 control matrix, row 3, and the Qwen control matrix appendix
+ *     ("soft-router-only"): routing over the concatenated public/private pool
+ *     without the hard mask.  With `unmasked` set, m(tau) = 0 for every
+ *     expert; this is a negative control, not the method (G1 does not hold).
  */
 #include <math.h>
 #include <stdint.h>
@@ -58,6 +62,7 @@ typedef struct {
     const uint16_t *gate_pub, *up_pub, *down_pub;     /* [E_pub][I][H], [E_pub][I][H], [E_pub][H][I] */
     const uint16_t *gate_priv, *up_priv, *down_priv;  /* [E_priv][I][H], ..., [E_priv][H][I] */
     const uint16_t *gate_sh, *up_sh, *down_sh;        /* [E_sh][I][H], ..., [E_sh][H][I]; NULL if E_sh == 0 */
+    int unmasked;                    /* 1: the soft-router control, no hard mask (all E experts eligible) */
 } oracle_layer;
 
 /* ---------------------------------------------------------------- BF16 -- */
@@ -113,7 +118,8 @@ static const uint16_t *router_row(const oracle_layer *L, int e)
 }
 
 /* Route one token: z_e over the concatenated pool, s = z + m(tau), top-k of s
- * (descending, ties to the lower id), weights from the softmax of s.
+ * (descending, ties to the lower id), weights from the softmax of s.  In the
+ * unmasked control m = 0, so the top-k and the softmax run over all E.
  * Writes idx[k], w[k], and the gap s_(k) - s_(k+1) inside the visible pool
  * (+inf when k equals the pool size). */
 static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, double *gap,
@@ -127,7 +133,7 @@ static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, d
         const uint16_t *wr = router_row(L, e);
         double z = 0.0;
         for (int c = 0; c < L->H; ++c) z += bf16_value(h[c]) * bf16_value(wr[c]);
-        const int eligible = tau ? (e >= L->E_pub) : (e < L->E_pub);
+        const int eligible = L->unmasked ? 1 : (tau ? (e >= L->E_pub) : (e < L->E_pub));
         s[e] = eligible ? (double)(float)z : -INFINITY;   /* z + m(tau), z rounded to fp32 */
         taken[e] = 0;
     }

@@ -29,11 +29,11 @@ def make_layer(shape: LayerShape, seed: int, device="cpu", policy="iid", skew=No
     return w, h, pol
 
 
-def oracle_layer(shape, w, h, pol):
+def oracle_layer(shape, w, h, pol, unmasked=False):
     import oracle
     t = dict(w)
     t["hidden"] = h
-    return oracle.Layer(shape, t, None if pol is None else pol.cpu().numpy())
+    return oracle.Layer(shape, t, None if pol is None else pol.cpu().numpy(), unmasked=unmasked)
 
 
 def bf16_bits(t: torch.Tensor) -> np.ndarray:

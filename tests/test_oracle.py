@@ -132,6 +132,69 @@ def test_route_k_equals_pool_selects_whole_pool():
     assert np.all(np.isinf(gap))
 
 
+def test_unmasked_control_routes_over_the_whole_pool_brute_force():
+    """The soft-router control (Sec. 4.3 control matrix, row 3): without the
+    hard mask every expert of the concatenated pool is eligible.  Logits from
+    numpy's float64 matmul rounded to fp32, a full sort over all E, and the
+    softmax over all E (pool softmax) or over the top-k (renormalised)."""
+    for renorm in (True, False):
+        s = LayerShape(T=120, H=64, I=16, E_pub=12, E_priv=6, E_sh=0, k=3, renormalize=renorm)
+        w, h, pol = make_layer(s, seed=21)
+        idx, wt, gap = oracle.route(oracle_layer(s, w, h, pol, unmasked=True))
+        R = torch.cat([w["router_pub"], w["router_priv"]]).double().numpy()
+        Z = (h.double().numpy() @ R.T).astype(np.float32).astype(np.float64)
+        for t in range(s.T):
+            srow = list(Z[t])
+            top, order = _expected_topk(srow, s.k)
+            assert list(idx[t]) == top
+            m = srow[top[0]]
+            ex = {e: math.exp(srow[e] - m) for e in order}
+            denom = sum(ex[e] for e in (top if renorm else order))
+            np.testing.assert_allclose(wt[t], [ex[e] / denom for e in top], rtol=1e-12)
+            assert gap[t] == srow[top[-1]] - srow[order[s.k]]
+
+
+def test_unmasked_control_top1_is_the_better_masked_top1():
+    """Without the mask, the best expert is the better of the best public
+    expert (the masked DENY route) and the best private expert (the masked
+    ALLOW route); and when the whole unmasked top-k lies in one pool, the
+    renormalised weights equal that pool's masked ones."""
+    s = LayerShape(T=300, H=128, I=16, E_pub=16, E_priv=8, E_sh=0, k=4, renormalize=True)
+    w, h, _ = make_layer(s, seed=22)
+    deny = torch.zeros(s.T, dtype=torch.uint8)
+    allow = torch.ones(s.T, dtype=torch.uint8)
+    i_d, w_d, _ = oracle.route(oracle_layer(s, w, h, deny))
+    i_a, w_a, _ = oracle.route(oracle_layer(s, w, h, allow))
+    i_u, w_u, _ = oracle.route(oracle_layer(s, w, h, deny, unmasked=True))
+    R = torch.cat([w["router_pub"], w["router_priv"]]).double().numpy()
+    Z = (h.double().numpy() @ R.T).astype(np.float32)
+    one_pool = 0
+    for t in range(s.T):
+        a, b = i_d[t, 0], i_a[t, 0]
+        best = a if (Z[t, a] > Z[t, b] or (Z[t, a] == Z[t, b] and a < b)) else b
+        assert i_u[t, 0] == best
+        if np.all(i_u[t] < s.E_pub):
+            assert list(i_u[t]) == list(i_d[t]); np.testing.assert_allclose(w_u[t], w_d[t], rtol=1e-12); one_pool += 1
+        elif np.all(i_u[t] >= s.E_pub):
+            assert list(i_u[t]) == list(i_a[t]); np.testing.assert_allclose(w_u[t], w_a[t], rtol=1e-12); one_pool += 1
+    assert one_pool > 0
+
+
+def test_unmasked_control_executes_private_rows_for_deny_tokens():
+    """The negative control: without the hard mask, DENY tokens reach private
+    experts (the route log and the independent execution count both show it),
+    which the masked layer never does (Sec. 2.2, G1)."""
+    s = LayerShape(T=64, H=64, I=16, E_pub=8, E_priv=8, E_sh=0, k=2, renormalize=True)
+    w, h, _ = make_layer(s, seed=23)
+    deny = torch.zeros(s.T, dtype=torch.uint8)
+    r_m = oracle.forward(oracle_layer(s, w, h, deny))
+    r_u = oracle.forward(oracle_layer(s, w, h, deny, unmasked=True))
+    assert r_m["exec_priv_rows"].sum() == 0 and r_m["route_priv_rows"].sum() == 0
+    assert r_u["exec_priv_rows"].sum() > 0
+    assert np.array_equal(r_u["exec_priv_rows"], r_u["route_priv_rows"])
+    assert np.array_equal(r_u["route_priv_rows"], (r_u["idx"] >= s.E_pub).sum(1))
+
+
 def test_route_k1_argmax_weight_one():
     s = LayerShape(T=50, H=64, I=8, E_pub=8, E_priv=3, E_sh=0, k=1, renormalize=True)
     w, h, pol = make_layer(s, seed=6)
