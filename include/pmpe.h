@@ -110,6 +110,15 @@ typedef struct pmpe_moe_desc {
                                     across calls until pmpe_audit_reset() */
     void *workspace;             /* device scratch, >= pmpe_moe_workspace_size() bytes, 256-byte aligned */
     size_t workspace_bytes;
+
+    /* 0: the method.  1: the paper's soft-router control (Sec. 4.3 control
+     * matrix, row 3): every token routes over the concatenated public/private
+     * pool without the hard mask, whatever its policy byte.  A negative
+     * control for audits: private rows then execute for DENY tokens, which
+     * the audit counters record.  Requires the merge of the router's chunk
+     * lists to fit in shared memory: ceil(E_pub/32) + ceil(E_priv/32) <= 16
+     * and that count * k <= 96; PMPE_ERR_UNSUPPORTED_SHAPE otherwise. */
+    int unmasked_control;
 } pmpe_moe_desc;
 
 /* Bytes of device workspace pmpe_moe_forward() needs for this shape.
@@ -118,9 +127,10 @@ PMPE_API size_t pmpe_moe_workspace_size(int T, int H, int I, int E_pub, int E_pr
 
 /* Byte offsets of the named regions inside the workspace (for tests that
  * inspect intermediate results, and for the stage-by-stage entry point).
- * Router geometry used below: S = ceil(T/128) + 1 token-tile slots and
+ * Router geometry used below: S = ceil(T/128) + 1 token-tile slots,
  * C = S * max(ceil(E_pub/32), ceil(E_priv/32)) router CTAs (one per tile and
- * 32-expert chunk of its pool).  Returns PMPE_ERR_INVALID_ARG for an invalid
+ * 32-expert chunk of its pool) and C2 = S * (ceil(E_pub/32) + ceil(E_priv/32))
+ * (the unmasked control's chunks of the concatenated pool).  Returns PMPE_ERR_INVALID_ARG for an invalid
  * shape. */
 typedef struct pmpe_workspace_layout {
     size_t total;
@@ -140,8 +150,8 @@ typedef struct pmpe_workspace_layout {
     size_t act_sh;       /* BF16   [T, E_shared*I] shared-expert activations (0 if none) */
     size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs (0 if none) */
     size_t tile_done;    /* uint32 [S]      router CTAs finished per 128-token tile */
-    size_t router_lists; /* float2 [C*128, k] per 32-expert chunk: each token's best k (score, id) */
-    size_t router_meta;  /* float4 [C*128]  per chunk: max score, sum exp(score - max), entries */
+    size_t router_lists; /* float2 [C2*128, k] per 32-expert chunk: each token's best k (score, id) */
+    size_t router_meta;  /* float4 [C2*128] per chunk: max score, sum exp(score - max), entries */
     size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1]  gate/up epilogue warps done per
                           * (expert group, 128-row block), read by the down tiles of the same launch */
 } pmpe_workspace_layout;

@@ -33,7 +33,7 @@ constexpr int kRThreads = 192;  // warp 0 TMA, warp 1 TMEM + MMA, warps 2..5 epi
 constexpr int kRMaxStages = 10;
 constexpr int kTileRows = 128;
 constexpr int kChunk = 32;                  // experts per CTA (MMA N)
-constexpr int kMaxChunks = kMaxPool / kChunk;
+constexpr int kMaxChunks = 2 * kMaxPool / kChunk;  // chunks of one tile: 8 per pool, 16 unmasked
 constexpr int kABytes = kTileRows * 128;    // 128 rows x 64 BF16
 constexpr int kBBytes = kChunk * 128;       // 32 router rows x 64 BF16
 constexpr int kStageBytes = kABytes + kBBytes;
@@ -41,8 +41,9 @@ constexpr int kEpi = 128;                   // epilogue threads
 
 struct RouterParams {
     int T, H, E_pub, E_priv, k, renorm;
-    int nch[2];          // 32-expert chunks of each pool
+    int nch[3];          // 32-expert chunks of the public pool, the private pool, and both (unmasked)
     int nch_max;         // CTAs per tile slot
+    int unmasked;        // the soft-router control: one pool of all experts, no hard mask
     uint32_t idesc;      // M = 128, N = 32
     int stages;
     const uint8_t *policy;
@@ -189,8 +190,10 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     // tokens; the scan of its ALLOW count gives the pool sizes and its ranks
     const int per = (p.T + kRThreads - 1) / kRThreads;
     const int t0 = min(p.T, tid * per), t1 = min(p.T, t0 + per);
+    // the unmasked control tiles all tokens as one pool, in token order
     int a = 0;
-    for (int t = t0; t < t1; ++t) a += is_allow(p.policy, t);
+    if (!p.unmasked)
+        for (int t = t0; t < t1; ++t) a += is_allow(p.policy, t);
     int na;
     const int a_before = block_scan(a, warp_tot, na);
     const int nd = p.T - na;
@@ -204,19 +207,21 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         m0 = (slot - tiles_d) * kTileRows;
         if (m0 >= na) return;  // uniform: no tile for this slot
     }
-    if (chunk >= p.nch[pool]) return;  // uniform: the pool has fewer chunks
     const int rows = min(kTileRows, (pool ? na : nd) - m0);
     {
         int ra = a_before, rd = t0 - a_before;  // ranks inside the ALLOW / DENY pools
         for (int t = t0; t < t1; ++t) {
-            const bool al = is_allow(p.policy, t);
+            const bool al_byte = is_allow(p.policy, t);
+            const bool al = al_byte && !p.unmasked;
             const int rank = al ? ra++ : rd++;
             if ((al ? 1 : 0) == pool && rank >= m0 && rank < m0 + rows) {
                 s_tok[rank - m0] = t;
-                if (chunk == 0) p.tau[t] = al ? 1 : 0;  // every token is written by exactly one CTA
+                if (chunk == 0) p.tau[t] = al_byte ? 1 : 0;  // every token is written by exactly one CTA
             }
         }
     }
+    if (p.unmasked) pool = 2;
+    if (chunk >= p.nch[pool]) return;  // uniform: the pool has fewer chunks
     __syncthreads();
     for (int r = rows + tid; r < kTileRows; r += kRThreads) s_tok[r] = s_tok[0];  // padding rows name a real token
     // The TMA ring reads the tile's rows as one 128-row tile.  When the tile's
@@ -268,8 +273,15 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     tc_fence_after();
     const uint32_t tmem = s_tmem;
     const int nkb = p.H / 64;
-    const int P = pool ? p.E_priv : p.E_pub;
-    const int base = pool ? p.E_pub : 0;
+    // This CTA's chunk: router tensor q (0 public, 1 private) and chunk lc in
+    // it.  Pool ids run 0 .. P-1 (the concatenated ids in the unmasked pool);
+    // base is the global id of pool id 0; c0 the pool id of column 0.
+    const int q = pool == 2 ? (chunk < p.nch[0] ? 0 : 1) : pool;
+    const int lc = (pool == 2 && q == 1) ? chunk - p.nch[0] : chunk;
+    const int P = pool == 2 ? p.E_pub + p.E_priv : (pool ? p.E_priv : p.E_pub);
+    const int base = pool == 1 ? p.E_pub : 0;
+    const int c0 = (pool == 2 && q == 1 ? p.E_pub : 0) + lc * kChunk;
+    const int nvalid = min(kChunk, (q ? p.E_priv : p.E_pub) - lc * kChunk);
 
     if (warp == 0 && lane < 2) {
         // ---- TMA producers: lane 0 the 128 tile rows, lane 1 the chunk's 32
@@ -282,7 +294,7 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
             const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
             mbar_expect_tx(full_bar(stage), my_tx);
             if (lane == 1)
-                tma_load_2d(sB, &maps.router[pool], full_bar(stage), kb * 64, chunk * kChunk);
+                tma_load_2d(sB, &maps.router[q], full_bar(stage), kb * 64, lc * kChunk);
             else if (contiguous)
                 tma_load_2d(sA, &maps.hidden, full_bar(stage), kb * 64, s_tok[0]);
             else
@@ -336,8 +348,8 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         uint16_t *se = reinterpret_cast<uint16_t *>(sv + nl * kTileRows * K);      // [nl][128][K] ids
         uint16_t *sloc = se + nl * kTileRows * K;                                   // [128][K] rank in expert
         uint32_t *scnt = reinterpret_cast<uint32_t *>(sloc + ((kTileRows * K + 1) & ~1));  // [P]
-        uint32_t *sbas = scnt + kMaxPool;                                           // [P]
-        float4 *smeta = reinterpret_cast<float4 *>(sbas + kMaxPool);               // [nl][128]
+        uint32_t *sbas = scnt + 2 * kMaxPool;                                       // [P]
+        float4 *smeta = reinterpret_cast<float4 *>(sbas + 2 * kMaxPool);           // [nl][128]
         if (ok) {
             __syncwarp();
             tc_fence_after();
@@ -345,8 +357,6 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
             int e[32];
             tmem_ld32(tmem + ((uint32_t)(q * 32) << 16), v);
             tmem_ld_wait();
-            const int c0 = chunk * kChunk;
-            const int nvalid = min(kChunk, P - c0);
             float mx = -INFINITY;
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
@@ -531,7 +541,9 @@ cudaError_t launch_route(const Ctx &c)
     p.T = s.T; p.H = s.H; p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.k = s.k; p.renorm = s.renorm;
     p.nch[0] = router_chunks(s.E_pub);
     p.nch[1] = router_chunks(s.E_priv);
-    p.nch_max = p.nch[0] > p.nch[1] ? p.nch[0] : p.nch[1];
+    p.nch[2] = p.nch[0] + p.nch[1];
+    p.unmasked = c.unmasked;
+    p.nch_max = p.unmasked ? p.nch[2] : (p.nch[0] > p.nch[1] ? p.nch[0] : p.nch[1]);
     const int slots = router_slots(s.T);
     // per-expert counters, per-tile completion counts and the expert GEMMs'
     // readiness counters start at zero (the workspace places them side by
@@ -569,7 +581,7 @@ cudaError_t launch_route(const Ctx &c)
     ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, kChunk);
     if (!ok) return cudaErrorInvalidValue;
     const int ring = p.stages * kStageBytes + 1024;
-    const int merge = p.nch_max * kTileRows * s.k * 6 + kTileRows * s.k * 2 + 4 + 2 * kMaxPool * 4 +
+    const int merge = p.nch_max * kTileRows * s.k * 6 + kTileRows * s.k * 2 + 4 + 4 * kMaxPool * 4 +
                       p.nch_max * kTileRows * 16 + 1024 + 16;
     const int smem = ring > merge ? ring : merge;
     cudaError_t err = cudaFuncSetAttribute(router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);

@@ -40,6 +40,7 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     L->counts = take(4 * E, 256);
     const size_t slots = (size_t)router_slots(s.T);
     const size_t rctas = slots * (size_t)std::max(router_chunks(s.E_pub), router_chunks(s.E_priv));
+    const size_t rctas_all = slots * (size_t)(router_chunks(s.E_pub) + router_chunks(s.E_priv));
     L->tile_done = take(4 * slots, 4);
     L->gemm_ready = take(4 * gemm_ready_words(s), 4);
     L->offsets = take(4 * (E + 1), 256);
@@ -49,8 +50,8 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     L->ticket = take(4 * R, 256);
     L->tok_of_slot = take(4 * R, 256);
     L->w_of_slot = take(4 * R, 256);
-    L->router_lists = take(8 * rctas * 128 * (size_t)s.k, 256);
-    L->router_meta = take(16 * rctas * 128, 256);
+    L->router_lists = take(8 * rctas_all * 128 * (size_t)s.k, 256);
+    L->router_meta = take(16 * rctas_all * 128, 256);
     L->router_rows = take(2 * rctas * 128 * (size_t)s.H, 1024);
     L->a_perm = take(2 * R * s.H, 1024);
     L->act = take(2 * R * s.I, 1024);
@@ -101,6 +102,11 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     for (const void *q : required)
         if (!q && s.T > 0) return PMPE_ERR_INVALID_ARG;
     if (s.E_sh > 0 && (!d->w_gate_sh || !d->w_up_sh || !d->w_down_sh)) return PMPE_ERR_INVALID_ARG;
+    if (d->unmasked_control != 0 && d->unmasked_control != 1) return PMPE_ERR_INVALID_ARG;
+    if (d->unmasked_control) {
+        const int nall = router_chunks(s.E_pub) + router_chunks(s.E_priv);
+        if (nall > 16 || nall * s.k > 96) return PMPE_ERR_UNSUPPORTED_SHAPE;
+    }
     const void *all[] = {d->hidden, d->w_router_pub, d->w_router_priv, d->w_gate_pub, d->w_up_pub, d->w_down_pub,
                          d->w_gate_priv, d->w_up_priv, d->w_down_priv, d->w_gate_sh, d->w_up_sh, d->w_down_sh,
                          d->out, d->topk_idx, d->topk_w, d->audit, d->workspace};
@@ -142,6 +148,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->act_sh = s.E_sh > 0 ? (bf16 *)(ws + L.act_sh) : nullptr;
     c->y_sh = s.E_sh > 0 ? (bf16 *)(ws + L.y_sh) : nullptr;
     c->stream = (cudaStream_t)stream;
+    c->unmasked = d->unmasked_control;
     if (s.T == 0) return PMPE_OK;  // a no-op: no device query, no launch
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PMPE_ERR_CUDA;

@@ -58,6 +58,7 @@ struct Ctx {
     bf16 *a_perm, *act, *y, *act_sh, *y_sh;
     cudaStream_t stream;
     int num_sms;
+    int unmasked;  // the soft-router control: no hard mask (a negative control, not the method)
 };
 
 int compute_layout(const Shape &s, pmpe_workspace_layout *L);

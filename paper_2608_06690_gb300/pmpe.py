@@ -66,7 +66,7 @@ class MoeDesc(ctypes.Structure):
                 ("w_gate_priv", _vp), ("w_up_priv", _vp), ("w_down_priv", _vp),
                 ("w_gate_sh", _vp), ("w_up_sh", _vp), ("w_down_sh", _vp),
                 ("out", _vp), ("topk_idx", _vp), ("topk_w", _vp), ("audit", _vp),
-                ("workspace", _vp), ("workspace_bytes", ctypes.c_size_t)]
+                ("workspace", _vp), ("workspace_bytes", ctypes.c_size_t), ("unmasked_control", ctypes.c_int)]
 
 
 class WorkspaceLayout(ctypes.Structure):
@@ -177,7 +177,7 @@ def selftest_wait_timeout(status, limit_us: int, stream=None):
 
 
 def make_desc(s: LayerShape, weights: dict, hidden, policy, out, workspace, topk_idx=None, topk_w=None,
-              audit=None) -> MoeDesc:
+              audit=None, unmasked_control: bool = False) -> MoeDesc:
     """Fill the C descriptor from torch tensors (device pointers only)."""
     W = weights
     return MoeDesc(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, int(bool(s.renormalize)),
@@ -187,7 +187,8 @@ def make_desc(s: LayerShape, weights: dict, hidden, policy, out, workspace, topk
                    _ptr(W["gate_priv"]), _ptr(W["up_priv"]), _ptr(W["down_priv"]),
                    _ptr(W.get("gate_sh")), _ptr(W.get("up_sh")), _ptr(W.get("down_sh")),
                    _ptr(out), _ptr(topk_idx), _ptr(topk_w), _ptr(audit),
-                   _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size())
+                   _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
+                   int(bool(unmasked_control)))
 
 
 def forward_desc(desc: MoeDesc, stages: int = STAGE_ALL, stream=None):
@@ -232,7 +233,10 @@ class MoeLayer:
         return LayerShape(T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, s.renormalize)
 
     def forward(self, hidden, policy, out=None, topk_idx=None, topk_w=None, audit=None, stages=STAGE_ALL,
-                stream=None):
+                stream=None, unmasked_control: bool = False):
+        """Enqueue the layer on ``stream`` (default: the current stream).
+        ``unmasked_control`` runs the paper's soft-router control instead of
+        the method: routing over the concatenated pool without the hard mask."""
         T = hidden.shape[0]
         s = self._shape_T(T)
         assert hidden.is_contiguous() and hidden.dtype == torch.bfloat16 and hidden.shape == (T, s.H)
@@ -240,6 +244,7 @@ class MoeLayer:
             assert policy.dtype == torch.uint8 and policy.numel() == T and policy.is_contiguous()
         if out is None:
             out = torch.empty_like(hidden)
-        desc = make_desc(s, self.weights, hidden, policy, out, self.workspace(T), topk_idx, topk_w, audit)
+        desc = make_desc(s, self.weights, hidden, policy, out, self.workspace(T), topk_idx, topk_w, audit,
+                         unmasked_control)
         forward_desc(desc, stages, stream)
         return out

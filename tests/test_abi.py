@@ -74,9 +74,10 @@ def test_workspace_size_and_layout(pmpe):
         T, E, R = sh.T, sh.E_pub + sh.E_priv, sh.T * sh.k
         slots = (T + 127) // 128 + 1
         ctas = slots * max((sh.E_pub + 31) // 32, (sh.E_priv + 31) // 32)
+        ctas_all = slots * ((sh.E_pub + 31) // 32 + (sh.E_priv + 31) // 32)
         size = dict(tau=T, counts=4 * E, offsets=4 * (E + 1), topk_idx=4 * R, topk_w=4 * R, slot_of=4 * R,
                     ticket=4 * R, tok_of_slot=4 * R, w_of_slot=4 * R, tile_done=4 * slots,
-                    router_lists=8 * ctas * 128 * sh.k, router_meta=16 * ctas * 128,
+                    router_lists=8 * ctas_all * 128 * sh.k, router_meta=16 * ctas_all * 128,
                     gemm_ready=4 * ((R + 127) // 128 + E + (T + 127) // 128 + 1),
                     router_rows=2 * ctas * 128 * sh.H, a_perm=2 * R * sh.H, act=2 * R * sh.I, y=2 * R * sh.H,
                     act_sh=2 * T * sh.E_sh * sh.I, y_sh=2 * T * sh.H if sh.E_sh else 0)
@@ -148,6 +149,11 @@ def test_validation_rejects_before_any_cuda_call(pmpe):
     assert lib.pmpe_policy_resolve(None, 0, None, None) == pmpe.OK
     assert lib.pmpe_audit_reset(None, 4, 4, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_audit_read(None, 4, 4, None, None, 10) == pmpe.ERR_INVALID_ARG
+    d = pmpe.make_desc(ok, W, p, None, p, p)
+    d.unmasked_control = 2
+    assert lib.pmpe_moe_forward(ctypes.byref(d), None) == pmpe.ERR_INVALID_ARG          # flag is 0 or 1
+    d = pmpe.make_desc(LayerShape(64, 256, 128, 256, 256, 0, 8, True), W, p, None, p, p, unmasked_control=True)
+    assert lib.pmpe_moe_forward(ctypes.byref(d), None) == pmpe.ERR_UNSUPPORTED_SHAPE     # merge too large
     assert lib.pmpe_selftest_wait_timeout(None, 1000, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 0, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 1000001, None) == pmpe.ERR_INVALID_ARG
