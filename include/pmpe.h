@@ -176,6 +176,20 @@ PMPE_API size_t pmpe_audit_words(int T, int E);
  * App. B.1, step 2 of the fail-closed procedure. */
 PMPE_API int pmpe_policy_resolve(const uint8_t *policy, int T, uint8_t *tau, void *stream);
 
+/* Per-token policy bytes from per-request ones, for callers that carry one
+ * trusted authorisation byte per request and the requests' cumulative token
+ * offsets (cu_seqlens[0..n_req], device int32) instead of a byte per token.
+ * policy_out[t] = req_policy[r] for cu_seqlens[r] <= t < cu_seqlens[r+1];
+ * tokens after cu_seqlens[n_req] get 0x00 (DENY).  Malformed offsets
+ * (cu_seqlens[0] != 0, a decreasing step, or cu_seqlens[n_req] > T) are
+ * malformed metadata: every token gets 0x00 (Sec. 2.1, App. B.1 fail
+ * closed).  The result feeds pmpe_moe_desc.policy.  All pointers device;
+ * asynchronous on `stream`; PMPE_ERR_INVALID_ARG for negative sizes or a
+ * NULL pointer that is needed.  (The request-offset ABI of the serving path;
+ * the paper specifies the authorisation per request, Sec. 2.1.) */
+PMPE_API int pmpe_policy_from_requests(const uint8_t *req_policy, const int32_t *cu_seqlens, int n_req, int T,
+                                       uint8_t *policy_out, void *stream);
+
 /* The whole layer forward (all stages) on `stream`.  No host synchronisation;
  * expert row counts stay on the device. */
 PMPE_API int pmpe_moe_forward(const pmpe_moe_desc *d, void *stream);

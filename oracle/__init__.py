@@ -155,6 +155,16 @@ def resolve(policy, T: int) -> np.ndarray:
     return tau
 
 
+def policy_from_requests(req_policy, cu_seqlens, T: int) -> np.ndarray:
+    """Per-token policy bytes from one byte per request and the cumulative
+    token offsets of the requests (fail-closed on malformed offsets)."""
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    rp = np.ascontiguousarray(req_policy, dtype=np.uint8)
+    out = np.zeros(T, dtype=np.uint8)
+    _load().oracle_policy_from_requests(_ptr(rp, _u8p), _ptr(cu, _i32p), len(cu) - 1, T, out.ctypes.data_as(_u8p))
+    return out
+
+
 def _token_list(layer: Layer, tokens):
     if tokens is None:
         return None, layer.shape.T

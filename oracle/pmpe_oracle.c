@@ -108,6 +108,23 @@ void oracle_resolve(const uint8_t *policy, int T, uint8_t *tau)
         tau[t] = (policy != NULL && policy[t] == 0x01) ? 1 : 0;
 }
 
+/* Per-request policy (one trusted byte per request, requests given by the
+ * cumulative token offsets cu[0..n]) expanded to one byte per token.  Any
+ * malformed offset list (cu[0] != 0, a decreasing step, or cu[n] > T) is
+ * malformed metadata: every token becomes DENY (0x00).  Tokens after cu[n]
+ * belong to no request and are DENY.  Sec. 2.1 / App. B.1: missing or
+ * malformed authorisation resolves to DENY. */
+void oracle_policy_from_requests(const uint8_t *req_policy, const int32_t *cu, int n, int T, uint8_t *out)
+{
+    int valid = (n >= 0 && cu != NULL && (n == 0 || req_policy != NULL) && cu[0] == 0 && cu[n] <= T);
+    for (int r = 0; valid && r < n; ++r)
+        if (cu[r + 1] < cu[r]) valid = 0;
+    for (int t = 0; t < T; ++t) out[t] = 0x00;
+    if (!valid) return;
+    for (int r = 0; r < n; ++r)
+        for (int t = cu[r]; t < cu[r + 1]; ++t) out[t] = req_policy[r];
+}
+
 /* ------------------------------------------------------------- routing -- */
 
 /* The row of the concatenated router for global expert id e. */

@@ -523,7 +523,8 @@ cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
     bool ok = true;
     for (int ph = 0; ph < nph; ++ph) ok &= fill_phase(c, modes[ph], ph, p, maps);
     if (!ok) return cudaErrorInvalidValue;
-    cudaError_t err = cudaFuncSetAttribute(expert_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem);
+    static std::atomic<int> smem_limit[64];
+    cudaError_t err = ensure_dynamic_smem(expert_gemm_tc_kernel, kDynSmem, smem_limit);
     if (err != cudaSuccess) return err;
     return launch_pdl(expert_gemm_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
 }

@@ -520,6 +520,33 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     }
 }
 
+// Per-request policy bytes to per-token bytes, in one CTA: the offsets are
+// checked first (cu[0] == 0, non-decreasing, cu[n] <= T); any violation is
+// malformed metadata and every token becomes DENY.  Otherwise token t takes
+// the byte of the request whose range holds it (the last request starting at
+// or before t; empty requests hold no token), and tokens after cu[n] are DENY.
+__global__ void __launch_bounds__(1024) policy_from_requests_kernel(const uint8_t *rp, const int32_t *cu, int n, int T,
+                                                                    uint8_t *out)
+{
+    int bad = 0;
+    if (threadIdx.x == 0) bad = (cu[0] != 0) | (cu[n] > T) | (n > 0 && rp == nullptr);
+    for (int r = threadIdx.x; r < n; r += blockDim.x) bad |= cu[r + 1] < cu[r];
+    const int any_bad = __syncthreads_or(bad);
+    const int end = any_bad ? 0 : cu[n];
+    for (int t = threadIdx.x; t < T; t += blockDim.x) {
+        uint8_t v = 0x00;
+        if (t < end) {
+            int lo = 0, hi = n - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (cu[mid] <= t) lo = mid; else hi = mid - 1;
+            }
+            v = rp[lo];
+        }
+        out[t] = v;
+    }
+}
+
 __global__ void resolve_kernel(const uint8_t *policy, int T, uint8_t *tau)
 {
     for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < T; t += gridDim.x * blockDim.x)
@@ -584,9 +611,17 @@ cudaError_t launch_route(const Ctx &c)
     const int merge = p.nch_max * kTileRows * s.k * 6 + kTileRows * s.k * 2 + 4 + 4 * kMaxPool * 4 +
                       p.nch_max * kTileRows * 16 + 1024 + 16;
     const int smem = ring > merge ? ring : merge;
-    cudaError_t err = cudaFuncSetAttribute(router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    static std::atomic<int> smem_limit[64];
+    cudaError_t err = ensure_dynamic_smem(router_tc_kernel, smem, smem_limit);
     if (err != cudaSuccess) return err;
     return launch_pdl(router_tc_kernel, dim3(grid), dim3(kRThreads), smem, c.stream, p, maps);
+}
+
+cudaError_t launch_policy_from_requests(const uint8_t *req_policy, const int32_t *cu_seqlens, int n_req, int T,
+                                        uint8_t *policy_out, cudaStream_t stream)
+{
+    policy_from_requests_kernel<<<1, 1024, 0, stream>>>(req_policy, cu_seqlens, n_req, T, policy_out);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_resolve(const uint8_t *policy, int T, uint8_t *tau, cudaStream_t stream)

@@ -190,6 +190,18 @@ int pmpe_policy_resolve(const uint8_t *policy, int T, uint8_t *tau, void *stream
     return launch_resolve(policy, T, tau, (cudaStream_t)stream) == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
 }
 
+int pmpe_policy_from_requests(const uint8_t *req_policy, const int32_t *cu_seqlens, int n_req, int T,
+                              uint8_t *policy_out, void *stream)
+{
+    if (n_req < 0 || T < 0 || !cu_seqlens || (T > 0 && !policy_out) || (n_req > 0 && !req_policy))
+        return PMPE_ERR_INVALID_ARG;
+    if (T == 0) return PMPE_OK;
+    return launch_policy_from_requests(req_policy, cu_seqlens, n_req, T, policy_out, (cudaStream_t)stream) ==
+                   cudaSuccess
+               ? PMPE_OK
+               : PMPE_ERR_CUDA;
+}
+
 int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *stream)
 {
     Ctx c;

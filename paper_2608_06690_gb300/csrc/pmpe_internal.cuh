@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <utility>
 
 #include "../../include/pmpe.h"
@@ -79,6 +80,28 @@ cudaError_t launch_down(const Ctx &c);
 cudaError_t launch_experts(const Ctx &c, bool zero_ready);
 cudaError_t launch_combine(const Ctx &c);
 cudaError_t launch_resolve(const uint8_t *policy, int T, uint8_t *tau, cudaStream_t stream);
+cudaError_t launch_policy_from_requests(const uint8_t *req_policy, const int32_t *cu_seqlens, int n_req, int T,
+                                        uint8_t *policy_out, cudaStream_t stream);
+
+// Raise `kernel`'s dynamic shared-memory limit on the current device to at
+// least `bytes`, calling the runtime only when the limit must grow (the
+// setting persists for the process; `limit` caches it per device, 64 devices).
+template <typename Kernel>
+cudaError_t ensure_dynamic_smem(Kernel kernel, int bytes, std::atomic<int> *limit)
+{
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    if (dev < 0 || dev >= 64) return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (limit[dev].load() >= bytes) return cudaSuccess;
+    err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (err == cudaSuccess) {
+        int cur = limit[dev].load();
+        while (cur < bytes && !limit[dev].compare_exchange_weak(cur, bytes)) {
+        }
+    }
+    return err;
+}
 
 // Launch with programmatic dependent launch: the kernel may start (and run
 // its prologue) while the previous kernel in the stream finishes; it must

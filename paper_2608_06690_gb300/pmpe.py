@@ -48,7 +48,8 @@ KERNELS_PER_FORWARD = 4
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
-            "pmpe_status_string", "pmpe_moe_forward_noalloc", "pmpe_selftest_wait_timeout")
+            "pmpe_status_string", "pmpe_moe_forward_noalloc", "pmpe_selftest_wait_timeout",
+            "pmpe_policy_from_requests")
 
 # Bytes of the library's static scratch array used by pmpe_moe_forward_noalloc.
 STATIC_SCRATCH_BYTES = 32 << 20
@@ -89,6 +90,8 @@ _lib.pmpe_moe_forward_stages.restype = ctypes.c_int
 _lib.pmpe_moe_forward_stages.argtypes = [ctypes.POINTER(MoeDesc), ctypes.c_uint, _vp]
 _lib.pmpe_moe_forward_noalloc.restype = ctypes.c_int
 _lib.pmpe_moe_forward_noalloc.argtypes = [ctypes.POINTER(MoeDesc), _vp]
+_lib.pmpe_policy_from_requests.restype = ctypes.c_int
+_lib.pmpe_policy_from_requests.argtypes = [_vp, _vp, ctypes.c_int, ctypes.c_int, _vp, _vp]
 _lib.pmpe_selftest_wait_timeout.restype = ctypes.c_int
 _lib.pmpe_selftest_wait_timeout.argtypes = [_vp, ctypes.c_int, _vp]
 _lib.pmpe_audit_reset.restype = ctypes.c_int
@@ -145,6 +148,18 @@ def audit_fields(words: np.ndarray, T: int, E: int) -> dict:
     return dict(status=int(a[0]), shared_rows=int(a[1]), route_count=a[2:2 + E], exec_rows=a[2 + E:2 + 2 * E],
                 exec_tiles=a[2 + 2 * E:2 + 3 * E], route_priv_rows=a[2 + 3 * E:2 + 3 * E + T],
                 exec_priv_rows=a[2 + 3 * E + T:2 + 3 * E + 2 * T])
+
+
+def policy_from_requests(req_policy, cu_seqlens, T: int, out=None, stream=None):
+    """Per-token policy bytes (uint8 [T], device) from one byte per request
+    and the requests' cumulative token offsets (int32 [n+1], device);
+    fail-closed on malformed offsets."""
+    if out is None:
+        out = torch.empty(T, dtype=torch.uint8, device="cuda")
+    n = cu_seqlens.numel() - 1
+    _check(_lib.pmpe_policy_from_requests(_ptr(req_policy), _ptr(cu_seqlens), n, T, _ptr(out), _stream(stream)),
+           "pmpe_policy_from_requests")
+    return out
 
 
 def policy_resolve(policy, T: int, tau=None, stream=None):

@@ -154,6 +154,10 @@ def test_validation_rejects_before_any_cuda_call(pmpe):
     assert lib.pmpe_moe_forward(ctypes.byref(d), None) == pmpe.ERR_INVALID_ARG          # flag is 0 or 1
     d = pmpe.make_desc(LayerShape(64, 256, 128, 256, 256, 0, 8, True), W, p, None, p, p, unmasked_control=True)
     assert lib.pmpe_moe_forward(ctypes.byref(d), None) == pmpe.ERR_UNSUPPORTED_SHAPE     # merge too large
+    assert lib.pmpe_policy_from_requests(None, None, 1, 4, None, None) == pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_policy_from_requests(p_ptr := ctypes.c_void_p(0x10000000), p_ptr, -1, 4, p_ptr, None) == \
+        pmpe.ERR_INVALID_ARG
+    assert lib.pmpe_policy_from_requests(None, ctypes.c_void_p(0x10000000), 0, 0, None, None) == pmpe.OK  # T = 0
     assert lib.pmpe_selftest_wait_timeout(None, 1000, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 0, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 1000001, None) == pmpe.ERR_INVALID_ARG

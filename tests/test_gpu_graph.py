@@ -1,0 +1,65 @@
+"""A 48-layer decode-shaped stack (64 requests of one token, alternating
+ALLOW / DENY, residual add between layers) captured into one CUDA graph:
+replaying the graph gives bit for bit the result of running the layers one
+call at a time, twice in a row, and the audit counters accumulated inside
+the graph satisfy the per-token closed form 48 * k * tau (Sec. 2.2, G1)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_06690_gb300 import inputs as inp
+from paper_2608_06690_gb300 import pmpe
+from paper_2608_06690_gb300.inputs import LayerShape
+
+pytestmark = pytest.mark.gpu
+
+N_LAYERS = 48
+SHAPE = LayerShape(T=64, H=1024, I=256, E_pub=64, E_priv=16, E_sh=0, k=8, renormalize=True)
+
+
+def _stack(layers, x_in, pol, x_out, audit):
+    x = x_in
+    out = torch.empty_like(x_in)
+    for layer in layers:
+        layer.forward(x, pol, out=out, audit=audit)
+        x = (x.float() + out.float()).to(torch.bfloat16)
+    x_out.copy_(x)
+
+
+def test_48_layer_stack_replays_bitwise_from_a_cuda_graph():
+    s = SHAPE
+    ws = pmpe.Workspace("cuda")
+    layers = [pmpe.MoeLayer(s, inp.make_weights(s, 7000 + l, device="cuda"), workspace=ws) for l in range(N_LAYERS)]
+    x0 = inp.make_hidden(s, 7, device="cuda")
+    pol = torch.tensor([1 if t % 2 == 0 else 0 for t in range(s.T)], dtype=torch.uint8, device="cuda")
+    E = s.E
+    audit_e = torch.zeros(pmpe.audit_words(s.T, E), dtype=torch.int32, device="cuda")
+    eager = torch.empty_like(x0)
+    _stack(layers, x0, pol, eager, audit_e)   # also sizes the shared workspace before capture
+    torch.cuda.synchronize()
+
+    x_in = x0.clone()
+    x_out = torch.empty_like(x0)
+    audit_g = torch.zeros_like(audit_e)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):                 # warm-up on the capture stream
+        _stack(layers, x_in, pol, x_out, audit_g)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        _stack(layers, x_in, pol, x_out, audit_g)
+    audit_g.zero_()
+    for rep in range(2):
+        x_out.fill_(0)
+        graph.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(x_out.view(torch.int16), eager.view(torch.int16)), rep
+    a = pmpe.audit_read(audit_g, s.T, E)
+    tau = oracle.resolve(pol.cpu().numpy(), s.T)
+    assert np.array_equal(a["route_priv_rows"], 2 * N_LAYERS * s.k * tau.astype(np.uint32))
+    assert np.array_equal(a["exec_priv_rows"], a["route_priv_rows"])
+    assert np.array_equal(a["exec_rows"], a["route_count"])
+    assert a["route_count"].sum() == 2 * N_LAYERS * s.T * s.k

@@ -252,3 +252,38 @@ def test_persistent_gemm_pair_matches_separate_launches():
     layer.forward(hd, pd, out=again, stages=pmpe.STAGE_COMBINE)
     torch.cuda.synchronize()
     assert torch.equal(fused.view(torch.int16), again.view(torch.int16))
+
+
+def test_policy_from_requests_matches_oracle_and_feeds_the_layer():
+    """Per-request policy bytes expanded on the device equal the oracle's
+    expansion bit for bit (random partitions with empty requests and trailing
+    tokens, malformed offsets failing closed), and the layer run on them
+    equals the layer run on the per-token bytes."""
+    from paper_2608_06690_gb300 import pmpe
+    g = np.random.default_rng(9)
+    for trial in range(40):
+        n = int(g.integers(0, 30))
+        lens = g.integers(0, 60, size=n)
+        T = int(lens.sum() + g.integers(0, 8))
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        rp = g.integers(0, 256, size=n).astype(np.uint8)
+        rp[g.random(n) < 0.5] = 1
+        if trial % 5 == 4 and n >= 2:   # malformed offsets
+            cu[int(g.integers(1, n + 1))] = -1 if trial % 10 == 4 else T + 1
+        want = oracle.policy_from_requests(rp, cu, T)
+        got = pmpe.policy_from_requests(torch.from_numpy(rp).cuda(), torch.from_numpy(cu).cuda(), T)
+        torch.cuda.synchronize()
+        assert np.array_equal(got.cpu().numpy(), want), (trial, cu, rp)
+    shape = LayerShape(T=300, H=256, I=128, E_pub=16, E_priv=8, E_sh=0, k=2, renormalize=True)
+    w, h, _ = make_layer(shape, 46)
+    lens = np.array([70, 0, 100, 30, 100])
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    rp = np.array([1, 1, 0, 1, 9], np.uint8)
+    wd, hd, _ = to_device(w, h, None)
+    layer = pmpe.MoeLayer(shape, wd)
+    pol_dev = pmpe.policy_from_requests(torch.from_numpy(rp).cuda(), torch.from_numpy(cu).cuda(), shape.T)
+    pol_tok = torch.from_numpy(oracle.policy_from_requests(rp, cu, shape.T)).cuda()
+    a = layer.forward(hd, pol_dev).clone()
+    b = layer.forward(hd, pol_tok).clone()
+    torch.cuda.synchronize()
+    assert torch.equal(a.view(torch.int16), b.view(torch.int16))

@@ -53,6 +53,26 @@ def test_resolve_missing_metadata_is_deny():
     assert oracle.resolve(None, 37).sum() == 0
 
 
+def test_policy_from_requests_closed_forms():
+    """Per-request bytes expand to their requests' tokens; tokens after the
+    last request are DENY; malformed offsets make the whole batch DENY."""
+    g = np.random.default_rng(3)
+    for _ in range(50):
+        n = int(g.integers(1, 20))
+        lens = g.integers(0, 40, size=n)
+        T = int(lens.sum() + g.integers(0, 5))
+        cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        rp = g.integers(0, 256, size=n).astype(np.uint8)
+        rp[g.random(n) < 0.5] = 1
+        got = oracle.policy_from_requests(rp, cu, T)
+        want = np.concatenate([np.full(l, b, np.uint8) for l, b in zip(lens, rp)] + [np.zeros(T - lens.sum(), np.uint8)])
+        assert np.array_equal(got, want)
+    rp = np.array([1, 1, 1], np.uint8)
+    for bad in ([1, 3, 5, 7], [0, 5, 3, 7], [0, 3, 5, 99]):   # cu[0] != 0, a decreasing step, past T
+        assert oracle.policy_from_requests(rp, np.array(bad), 10).sum() == 0
+    assert oracle.policy_from_requests(np.zeros(0, np.uint8), np.array([0]), 6).sum() == 0
+
+
 # ---------------------------------------------------------------- routing
 
 def _expected_topk(s_row, k):
