@@ -44,7 +44,7 @@ class _Layer(ctypes.Structure):
         ("gate_pub", _u16p), ("up_pub", _u16p), ("down_pub", _u16p),
         ("gate_priv", _u16p), ("up_priv", _u16p), ("down_priv", _u16p),
         ("gate_sh", _u16p), ("up_sh", _u16p), ("down_sh", _u16p),
-        ("unmasked", ctypes.c_int),
+        ("unmasked", ctypes.c_int), ("exact", ctypes.c_int),
     ]
 
 
@@ -109,10 +109,12 @@ class Layer:
     down_sh) to BF16 tensors or uint16 arrays; ``policy`` is a uint8 array of
     T bytes or None (missing metadata).  ``unmasked`` selects the paper's
     soft-router control: routing over the concatenated pool without the hard
-    mask (a negative control, not the method).
+    mask (a negative control, not the method).  ``exact`` removes the
+    rounding of logits (fp32) and activations (BF16): the smooth function the
+    finite-difference pins of the backward differentiate.
     """
 
-    def __init__(self, shape, tensors: dict, policy, unmasked: bool = False):
+    def __init__(self, shape, tensors: dict, policy, unmasked: bool = False, exact: bool = False):
         self.shape = shape
         self._keep = {}
         for name in ("hidden", "router_pub", "router_priv", "gate_pub", "up_pub", "down_pub",
@@ -132,7 +134,7 @@ class Layer:
                         _ptr(k["gate_pub"], _u16p), _ptr(k["up_pub"], _u16p), _ptr(k["down_pub"], _u16p),
                         _ptr(k["gate_priv"], _u16p), _ptr(k["up_priv"], _u16p), _ptr(k["down_priv"], _u16p),
                         _ptr(k["gate_sh"], _u16p), _ptr(k["up_sh"], _u16p), _ptr(k["down_sh"], _u16p),
-                        int(bool(unmasked)))
+                        int(bool(unmasked)), int(bool(exact)))
 
 
 def bf16_round(x: float) -> int:
@@ -163,6 +165,21 @@ def policy_from_requests(req_policy, cu_seqlens, T: int) -> np.ndarray:
     out = np.zeros(T, dtype=np.uint8)
     _load().oracle_policy_from_requests(_ptr(rp, _u8p), _ptr(cu, _i32p), len(cu) - 1, T, out.ctypes.data_as(_u8p))
     return out
+
+
+def backward_private(layer: Layer, dout) -> dict:
+    """Gradients of sum(dout * out) with respect to the private parameters
+    (d_router [E_priv,H], d_gate / d_up [E_priv,I,H], d_down [E_priv,H,I],
+    float64), for the routing the forward takes; public parameters get none."""
+    s = layer.shape
+    d = np.ascontiguousarray(dout, dtype=np.float64).reshape(s.T, s.H)
+    r = dict(d_router=np.zeros((s.E_priv, s.H)), d_gate=np.zeros((s.E_priv, s.I, s.H)),
+             d_up=np.zeros((s.E_priv, s.I, s.H)), d_down=np.zeros((s.E_priv, s.H, s.I)))
+    rc = _load().oracle_backward_private(ctypes.byref(layer.c), d.ctypes.data_as(_f64p),
+                                         *(r[n].ctypes.data_as(_f64p) for n in ("d_router", "d_gate", "d_up", "d_down")))
+    if rc != 0:
+        raise ValueError("oracle_backward_private rejected the layer description")
+    return r
 
 
 def _token_list(layer: Layer, tokens):

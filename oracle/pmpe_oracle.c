@@ -63,6 +63,8 @@ typedef struct {
     const uint16_t *gate_priv, *up_priv, *down_priv;  /* [E_priv][I][H], ..., [E_priv][H][I] */
     const uint16_t *gate_sh, *up_sh, *down_sh;        /* [E_sh][I][H], ..., [E_sh][H][I]; NULL if E_sh == 0 */
     int unmasked;                    /* 1: the soft-router control, no hard mask (all E experts eligible) */
+    int exact;                       /* 1: no rounding of logits (fp32) or activations (BF16): the smooth
+                                        function that finite-difference pins of the backward differentiate */
 } oracle_layer;
 
 /* ---------------------------------------------------------------- BF16 -- */
@@ -151,7 +153,7 @@ static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, d
         double z = 0.0;
         for (int c = 0; c < L->H; ++c) z += bf16_value(h[c]) * bf16_value(wr[c]);
         const int eligible = L->unmasked ? 1 : (tau ? (e >= L->E_pub) : (e < L->E_pub));
-        s[e] = eligible ? (double)(float)z : -INFINITY;   /* z + m(tau), z rounded to fp32 */
+        s[e] = eligible ? (L->exact ? z : (double)(float)z) : -INFINITY;   /* z + m(tau), z rounded to fp32 */
         taken[e] = 0;
     }
     /* top-k by repeated selection: largest s, lower id on ties */
@@ -192,7 +194,7 @@ static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, d
  * *exec_counter: the execution count is observed here, where the expert
  * runs, not copied from the route log. */
 static void swiglu_expert(const uint16_t *Wg, const uint16_t *Wu, const uint16_t *Wd, int H, int I,
-                          const double *h, double *y, double *a, uint32_t *exec_counter)
+                          const double *h, double *y, double *a, uint32_t *exec_counter, int exact)
 {
     for (int i = 0; i < I; ++i) {
         const uint16_t *rg = Wg + (size_t)i * H, *ru = Wu + (size_t)i * H;
@@ -202,7 +204,7 @@ static void swiglu_expert(const uint16_t *Wg, const uint16_t *Wu, const uint16_t
             u += h[c] * bf16_value(ru[c]);
         }
         const double silu = g / (1.0 + exp(-g));
-        a[i] = bf16_value(oracle_bf16_round(silu * u));
+        a[i] = exact ? silu * u : bf16_value(oracle_bf16_round(silu * u));
     }
     for (int o = 0; o < H; ++o) {
         const uint16_t *rd = Wd + (size_t)o * I;
@@ -282,7 +284,7 @@ int oracle_expert(const oracle_layer *L, int e, int shared, const uint16_t *h_ro
     double *a = (double *)malloc(sizeof(double) * L->I);
     for (int c = 0; c < L->H; ++c) h[c] = bf16_value(h_row[c]);
     uint32_t dummy = 0;
-    swiglu_expert(g, u, d, L->H, L->I, h, y, a, &dummy);
+    swiglu_expert(g, u, d, L->H, L->I, h, y, a, &dummy, L->exact);
     free(h);
     free(a);
     return 0;
@@ -341,14 +343,14 @@ int oracle_forward(const oracle_layer *L, const int32_t *tokens, int n, uint16_t
                 const uint16_t *g, *u, *d;
                 routed_expert_weights(L, e, &g, &u, &d);
                 uint32_t before = my_exec[e];
-                swiglu_expert(g, u, d, H, I, h, y, a, &my_exec[e]);
+                swiglu_expert(g, u, d, H, I, h, y, a, &my_exec[e], L->exact);
                 if (e >= L->E_pub) exec_priv_local[p] += my_exec[e] - before;
                 for (int c = 0; c < H; ++c) acc[c] += tw[j] * y[c];
             }
             const size_t ih = (size_t)I * H;
             for (int sidx = 0; sidx < L->E_sh; ++sidx) {
                 swiglu_expert(L->gate_sh + sidx * ih, L->up_sh + sidx * ih, L->down_sh + sidx * ih, H, I, h, y, a,
-                              &my_exec[E]);
+                              &my_exec[E], L->exact);
                 for (int c = 0; c < H; ++c) acc[c] += y[c];
             }
             for (int c = 0; c < H; ++c) {
@@ -387,6 +389,119 @@ int oracle_forward(const oracle_layer *L, const int32_t *tokens, int n, uint16_t
  * token then rank.  counts[e] = #{(t,j): idx[t][j] = e}; offsets = exclusive
  * prefix sum of counts (E+1 entries); slot_of[t][j] = the row's position;
  * tok_of_slot[slot] = t.  Returns -1 on an id outside [0, E). */
+/* ------------------------------------------------------------ backward -- */
+
+/* Gradients of  L = sum_t dout_t . out_t  with respect to the PRIVATE
+ * parameters only -- the private router rows and the private experts' gate,
+ * up and down projections -- for the routing the forward takes (the top-k
+ * choice is piecewise constant).  The public parameters are frozen and get no
+ * gradient (G2, Sec. 2.2 and Sec. 3.2: only the private branch is trained).
+ * Chain rule through the forward as computed, with its rounding points
+ * (fp32 logits, BF16 activation) taken as the identity:
+ *   y'_j = W_down a_j,  a = silu(g) u,  out_t = sum_j w_j y'_j (+ shared)
+ *   dL/dw_j = dout_t . y'_j
+ *   private e = idx[j]:  dW_down[e] += (w_j dout_t) a_j^T,  da = W_down^T (w_j dout_t),
+ *     dg = da u silu'(g),  du = da silu(g),  dW_gate[e] += dg h^T,  dW_up[e] += du h^T
+ *   router (softmax over the eligible pool p, or renormalised over the top-k w):
+ *     renorm:     dz_j = w_j (dL/dw_j - sum_i w_i dL/dw_i) on the selected ids
+ *     pool:       dz_e = p_e (dL/dp_e - sum_e' p_e' dL/dp_e') on the pool, dL/dp_e = dL/dw_j if selected
+ *     dW_router[e] += dz_e h^T for private e
+ * dout [T][H]; outputs (overwritten): d_router [E_priv][H], d_gate / d_up
+ * [E_priv][I][H], d_down [E_priv][H][I].  Serial (test sizes). */
+int oracle_backward_private(const oracle_layer *L, const double *dout, double *d_router, double *d_gate,
+                            double *d_up, double *d_down)
+{
+    if (check_layer(L)) return -1;
+    const int E = L->E_pub + L->E_priv, H = L->H, I = L->I, k = L->k, Ep = L->E_pub;
+    memset(d_router, 0, sizeof(double) * L->E_priv * H);
+    memset(d_gate, 0, sizeof(double) * L->E_priv * I * H);
+    memset(d_up, 0, sizeof(double) * L->E_priv * I * H);
+    memset(d_down, 0, sizeof(double) * L->E_priv * H * I);
+    double *s = (double *)malloc(sizeof(double) * E), *h = (double *)malloc(sizeof(double) * H);
+    double *a = (double *)malloc(sizeof(double) * I), *g = (double *)malloc(sizeof(double) * I);
+    double *u = (double *)malloc(sizeof(double) * I), *dy = (double *)malloc(sizeof(double) * H);
+    double *da = (double *)malloc(sizeof(double) * I), *dz = (double *)malloc(sizeof(double) * E);
+    double *gw = (double *)malloc(sizeof(double) * k), *w = (double *)malloc(sizeof(double) * k);
+    char *taken = (char *)malloc(E);
+    int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * k);
+    for (int t = 0; t < L->T; ++t) {
+        double gap;
+        route_token(L, t, idx, w, &gap, s, taken);
+        const uint16_t *hr = L->hidden + (size_t)t * H;
+        const double *dt = dout + (size_t)t * H;
+        for (int c = 0; c < H; ++c) h[c] = bf16_value(hr[c]);
+        for (int j = 0; j < k; ++j) {
+            const int e = idx[j];
+            const uint16_t *Wg, *Wu, *Wd;
+            routed_expert_weights(L, e, &Wg, &Wu, &Wd);
+            for (int i = 0; i < I; ++i) {
+                double gi = 0.0, ui = 0.0;
+                for (int c = 0; c < H; ++c) {
+                    gi += h[c] * bf16_value(Wg[(size_t)i * H + c]);
+                    ui += h[c] * bf16_value(Wu[(size_t)i * H + c]);
+                }
+                g[i] = gi;
+                u[i] = ui;
+                const double silu = gi / (1.0 + exp(-gi));
+                a[i] = L->exact ? silu * ui : bf16_value(oracle_bf16_round(silu * ui));
+            }
+            double gwj = 0.0;  /* dout_t . y'_j */
+            for (int o = 0; o < H; ++o) {
+                double yo = 0.0;
+                for (int i = 0; i < I; ++i) yo += a[i] * bf16_value(Wd[(size_t)o * I + i]);
+                gwj += dt[o] * yo;
+            }
+            gw[j] = gwj;
+            if (e < Ep) continue;  /* public expert: frozen */
+            const int q = e - Ep;
+            for (int o = 0; o < H; ++o) dy[o] = w[j] * dt[o];
+            double *Dd = d_down + (size_t)q * H * I, *Dg = d_gate + (size_t)q * I * H, *Du = d_up + (size_t)q * I * H;
+            for (int o = 0; o < H; ++o)
+                for (int i = 0; i < I; ++i) Dd[(size_t)o * I + i] += dy[o] * a[i];
+            for (int i = 0; i < I; ++i) {
+                double acc = 0.0;
+                for (int o = 0; o < H; ++o) acc += bf16_value(Wd[(size_t)o * I + i]) * dy[o];
+                da[i] = acc;
+            }
+            for (int i = 0; i < I; ++i) {
+                const double sg = 1.0 / (1.0 + exp(-g[i]));
+                const double dg = da[i] * u[i] * sg * (1.0 + g[i] * (1.0 - sg));
+                const double du = da[i] * g[i] * sg;
+                for (int c = 0; c < H; ++c) {
+                    Dg[(size_t)i * H + c] += dg * h[c];
+                    Du[(size_t)i * H + c] += du * h[c];
+                }
+            }
+        }
+        /* router: dz over the eligible pool */
+        for (int e = 0; e < E; ++e) dz[e] = 0.0;
+        if (L->renormalize) {
+            double sum = 0.0;
+            for (int j = 0; j < k; ++j) sum += w[j] * gw[j];
+            for (int j = 0; j < k; ++j) dz[idx[j]] = w[j] * (gw[j] - sum);
+        } else {
+            const double smax = s[idx[0]];
+            double denom = 0.0;
+            for (int e = 0; e < E; ++e) denom += exp(s[e] - smax);
+            double sum = 0.0;
+            for (int j = 0; j < k; ++j) sum += w[j] * gw[j];  /* w_j = p_{idx[j]} */
+            for (int e = 0; e < E; ++e) {
+                if (s[e] == -INFINITY) continue;
+                const double pe = exp(s[e] - smax) / denom;
+                double dpe = 0.0;
+                for (int j = 0; j < k; ++j)
+                    if (idx[j] == e) dpe = gw[j];
+                dz[e] = pe * (dpe - sum);
+            }
+        }
+        for (int e = Ep; e < E; ++e)
+            if (dz[e] != 0.0)
+                for (int c = 0; c < H; ++c) d_router[(size_t)(e - Ep) * H + c] += dz[e] * h[c];
+    }
+    free(s); free(h); free(a); free(g); free(u); free(dy); free(da); free(dz); free(gw); free(w); free(taken); free(idx);
+    return 0;
+}
+
 int oracle_permute(const int32_t *idx, int T, int k, int E, uint32_t *counts, uint32_t *offsets, int32_t *slot_of,
                    int32_t *tok_of_slot)
 {

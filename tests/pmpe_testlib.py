@@ -29,11 +29,11 @@ def make_layer(shape: LayerShape, seed: int, device="cpu", policy="iid", skew=No
     return w, h, pol
 
 
-def oracle_layer(shape, w, h, pol, unmasked=False):
+def oracle_layer(shape, w, h, pol, unmasked=False, exact=False):
     import oracle
     t = dict(w)
     t["hidden"] = h
-    return oracle.Layer(shape, t, None if pol is None else pol.cpu().numpy(), unmasked=unmasked)
+    return oracle.Layer(shape, t, None if pol is None else pol.cpu().numpy(), unmasked=unmasked, exact=exact)
 
 
 def bf16_bits(t: torch.Tensor) -> np.ndarray:

@@ -384,3 +384,104 @@ def test_golden_hand_worked(case):
     assert r["idx"].tolist() == case["expected_idx"]
     np.testing.assert_allclose(r["w"], case["expected_w"], rtol=1e-15)
     assert bits_to_f64(r["out"]).tolist() == case["expected_out"]
+
+
+# ---------------------------------------------------- private-branch backward
+
+def _bf16_step(t: torch.Tensor, index, up: bool) -> torch.Tensor:
+    """A copy of BF16 tensor t with one element moved to the next BF16 value
+    up or down (one unit in the last place)."""
+    bits = t.view(torch.int16).clone()
+    flat = bits.view(-1)
+    i = int(np.ravel_multi_index(index, t.shape))
+    v = int(flat[i]) & 0xFFFF
+    mag, neg = v & 0x7FFF, v >> 15
+    if (not neg) == up:
+        mag += 1
+    else:
+        mag -= 1
+    flat[i] = np.int16(np.uint16(mag | (neg << 15)).astype(np.int16))
+    return bits.view(torch.bfloat16)
+
+
+def _loss(s, w, h, pol, dout, unmasked=False):
+    r = oracle.forward(oracle_layer(s, w, h, pol, unmasked=unmasked, exact=True))
+    return float((r["out_f64"] * dout).sum()), r["idx"]
+
+
+@pytest.mark.parametrize("renorm", [True, False])
+def test_backward_matches_central_differences(renorm):
+    """Central differences of sum(dout * out) over one-ULP BF16 steps of single
+    private weights, on the forward without rounding (exact mode), routing
+    unchanged under every step: router, gate, up and down gradients."""
+    s = LayerShape(T=40, H=32, I=16, E_pub=6, E_priv=5, E_sh=0, k=2, renormalize=renorm)
+    w, h, pol = make_layer(s, seed=31)
+    w = {n: (v * 8).to(torch.bfloat16) if v is not None and n.endswith("priv") else v for n, v in w.items()}
+    g = np.random.default_rng(5)
+    dout = g.standard_normal((s.T, s.H))
+    grads = oracle.backward_private(oracle_layer(s, w, h, pol, exact=True), dout)
+    _, idx0 = _loss(s, w, h, pol, dout)
+    checked = 0
+    for name, gname in (("router_priv", "d_router"), ("gate_priv", "d_gate"), ("up_priv", "d_up"),
+                        ("down_priv", "d_down")):
+        G = grads[gname]
+        picks = [np.unravel_index(int(i), G.shape) for i in np.argsort(-np.abs(G).ravel())[:4]]
+        for index in picks:
+            t0 = w[name]
+            x = float(t0[index])
+            wp, wm = dict(w), dict(w)
+            wp[name] = _bf16_step(t0, index, True)
+            wm[name] = _bf16_step(t0, index, False)
+            lp, ip = _loss(s, wp, h, pol, dout)
+            lm, im = _loss(s, wm, h, pol, dout)
+            if not (np.array_equal(ip, idx0) and np.array_equal(im, idx0)):
+                continue  # the step crossed a routing decision
+            fd = (lp - lm) / (float(wp[name][index]) - float(wm[name][index]))
+            assert fd == pytest.approx(G[index], rel=2e-3, abs=1e-9 * np.abs(G).max()), (gname, index, x)
+            checked += 1
+    assert checked >= 12
+
+
+def test_backward_single_private_expert_is_the_dense_mlp_gradient():
+    """E_priv = k = 1: every ALLOW token runs the one private expert with
+    weight 1, so its gradients are torch.autograd's for the dense SwiGLU MLP
+    (fp64, no rounding) summed over the ALLOW tokens, and the router gradient
+    is exactly zero."""
+    s = LayerShape(T=30, H=32, I=16, E_pub=3, E_priv=1, E_sh=0, k=1, renormalize=True)
+    w, h, pol = make_layer(s, seed=32)
+    dout = np.random.default_rng(6).standard_normal((s.T, s.H))
+    r = oracle.backward_private(oracle_layer(s, w, h, pol, exact=True), dout)
+    allow = oracle.resolve(pol.numpy(), s.T) == 1
+    Wg = w["gate_priv"][0].double().requires_grad_()
+    Wu = w["up_priv"][0].double().requires_grad_()
+    Wd = w["down_priv"][0].double().requires_grad_()
+    x = h.double()[torch.from_numpy(allow)]
+    y = (F.silu(x @ Wg.T) * (x @ Wu.T)) @ Wd.T
+    (y * torch.from_numpy(dout[allow])).sum().backward()
+    np.testing.assert_allclose(r["d_gate"][0], Wg.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(r["d_up"][0], Wu.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(r["d_down"][0], Wd.grad.numpy(), rtol=1e-10, atol=1e-12)
+    assert np.all(r["d_router"] == 0.0)
+
+
+@pytest.mark.parametrize("renorm", [True, False])
+def test_backward_g2_invariants(renorm):
+    """G2: the upstream gradient of DENY tokens never reaches the private
+    parameters (bitwise), and the router gradient sums to zero over the pool
+    (softmax gradients are orthogonal to the constant vector).  Under the
+    unmasked control, DENY tokens do reach them (the negative control)."""
+    s = LayerShape(T=60, H=32, I=16, E_pub=6, E_priv=4, E_sh=0, k=2, renormalize=renorm)
+    w, h, pol = make_layer(s, seed=33)
+    tau = oracle.resolve(pol.numpy(), s.T)
+    g = np.random.default_rng(7)
+    d1 = g.standard_normal((s.T, s.H))
+    d2 = d1.copy()
+    d2[tau == 0] = g.standard_normal(((tau == 0).sum(), s.H))
+    L = oracle_layer(s, w, h, pol)
+    r1, r2 = oracle.backward_private(L, d1), oracle.backward_private(L, d2)
+    for n in r1:
+        assert np.array_equal(r1[n], r2[n]), n
+    np.testing.assert_allclose(r1["d_router"].sum(0), 0.0, atol=1e-12 * np.abs(r1["d_router"]).max())
+    Lu = oracle_layer(s, w, h, pol, unmasked=True)
+    u1, u2 = oracle.backward_private(Lu, d1), oracle.backward_private(Lu, d2)
+    assert any(not np.array_equal(u1[n], u2[n]) for n in u1)
