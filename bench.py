@@ -176,6 +176,19 @@ def algorithmic_work(s, counts: np.ndarray):
                 touched_experts=touched, gemm_weight_bytes=gemm_weight_bytes)
 
 
+def backward_flops(s, counts: np.ndarray, allow_tokens: int) -> float:
+    """Algorithmic FLOPs of the private-branch backward: per private row,
+    dL/da = W_down^T dout, the recomputed gate and up projections, and the
+    three weight gradients (2 H I each: 12 H I); the router weight gradient
+    over every token (2 T E_priv H), plus the private logits the pool softmax
+    recomputes (2 E_priv H per ALLOW token)."""
+    rows = float(counts[s.E_pub:].sum())
+    f = 12.0 * rows * s.H * s.I + 2.0 * s.T * s.E_priv * s.H
+    if not s.renormalize:
+        f += 2.0 * allow_tokens * s.E_priv * s.H
+    return f
+
+
 def cpu_baseline(cfg, w, h, pol, budget_s=12.0, max_tokens=4096):
     """The CPU oracle, as it stands, on a bounded sample of the workload's
     tokens (the first n tokens of each request, spread evenly)."""
@@ -317,6 +330,24 @@ def run_ours(args):
     counts = a["route_count"]
     work = algorithmic_work(s, counts)
 
+    # ---- the private-branch backward after that forward (outside the step;
+    # each pass after its own L2 flush)
+    g_dout = torch.Generator(device=dev)
+    g_dout.manual_seed(7)
+    dout = torch.randn(h.shape, generator=g_dout, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    for _ in range(2):
+        layer.backward_private(h, pol, dout)
+    bwd_ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_ev.record(stream)
+        layer.backward_private(h, pol, dout)
+        b_ev.record(stream)
+        bwd_ms.append((a_ev, b_ev))
+    torch.cuda.synchronize(dev)
+    bwd_ms = [x.elapsed_time(y) for x, y in bwd_ms]
+
     # ---- end to end through the public API with host buffers, pipelined as a
     # serving loop would run it: step i+1's inputs are copied in (copy-in
     # stream) while step i computes, and step i's result is copied out
@@ -403,6 +434,13 @@ def run_ours(args):
         d["gbs"] = work[f"bytes_{n}"] / (ms / 1e3) / 1e9
         stage_report[n] = d
 
+    bwd_avg = float(np.mean(bwd_ms))
+    f_bwd = backward_flops(s, counts, int((pol == 1).sum().item()))
+    backward = {"ms": bwd_avg, "flops": f_bwd, "tflops": f_bwd / (bwd_avg / 1e3) / 1e12,
+                "tensor_frac": f_bwd / (bwd_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
+                "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.KERNELS_PER_BACKWARD,
+                "l2": "flushed before every pass"}
+
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -413,6 +451,7 @@ def run_ours(args):
                    "parallelism": f"replicas x{ws}"},
         "roofline": roof,
         "stages": stage_report,
+        "backward_private": backward,
         "expert_load": {"touched": work["touched_experts"], "max_rows": int(counts.max()),
                         "mean_rows_public": float(counts[:s.E_pub].mean()),
                         "mean_rows_private": float(counts[s.E_pub:].mean())},

@@ -176,6 +176,32 @@ PMPE_API size_t pmpe_audit_words(int T, int E);
  * App. B.1, step 2 of the fail-closed procedure. */
 PMPE_API int pmpe_policy_resolve(const uint8_t *policy, int T, uint8_t *tau, void *stream);
 
+/* ------------------------------------------------- private-branch backward */
+
+/* Bytes of device scratch pmpe_moe_backward_private() needs; 0 for an invalid
+ * shape. */
+PMPE_API size_t pmpe_moe_backward_workspace_size(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k);
+
+/* Gradients of L = sum_t dout_t . out_t with respect to the PRIVATE
+ * parameters only, for the routing of the forward just run with the same
+ * descriptor (G2, Sec. 2.2; Sec. 3.2: only the private branch is trained, the
+ * public parameters are frozen and get no gradient, and DENY tokens reach no
+ * private parameter).  The descriptor's workspace must still hold that
+ * forward's state (route log, dispatch order, dispatched rows, activations):
+ * run the forward, then this, on the same stream, with nothing in between
+ * that reuses the workspace, passing that forward's descriptor (its route
+ * outputs topk_idx / topk_w included; its `out` is not written).
+ * dout: [T, H] BF16 upstream gradient.  Outputs
+ * (FP32, overwritten, 16-byte aligned): d_router_priv [E_priv, H],
+ * d_gate_priv and d_up_priv [E_priv, I, H], d_down_priv [E_priv, H, I].  The
+ * rounding points of the forward (FP32 logits, BF16 activations) are taken as
+ * the identity.  Not defined for the unmasked control
+ * (PMPE_ERR_UNSUPPORTED_SHAPE).  bwd_workspace: >= the size above, 256-byte
+ * aligned (PMPE_ERR_WORKSPACE otherwise).  Asynchronous on `stream`. */
+PMPE_API int pmpe_moe_backward_private(const pmpe_moe_desc *d, const void *dout, float *d_router_priv,
+                                       float *d_gate_priv, float *d_up_priv, float *d_down_priv,
+                                       void *bwd_workspace, size_t bwd_workspace_bytes, void *stream);
+
 /* Per-token policy bytes from per-request ones, for callers that carry one
  * trusted authorisation byte per request and the requests' cumulative token
  * offsets (cu_seqlens[0..n_req], device int32) instead of a byte per token.

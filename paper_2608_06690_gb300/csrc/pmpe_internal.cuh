@@ -75,6 +75,10 @@ cudaError_t launch_route(const Ctx &c);
 cudaError_t launch_permute(const Ctx &c);
 cudaError_t launch_gateup(const Ctx &c);
 cudaError_t launch_down(const Ctx &c);
+// Backward of the private branch (k_backward.cu): scratch bytes and launch.
+size_t backward_workspace_bytes(const Shape &s);
+cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_router, float *d_gate, float *d_up,
+                                    float *d_down, uint8_t *bws);
 // Gate/up and down in one persistent launch (down tiles wait for their
 // activation rows); zero_ready clears the readiness counters first.
 cudaError_t launch_experts(const Ctx &c, bool zero_ready);

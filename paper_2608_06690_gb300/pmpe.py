@@ -45,11 +45,15 @@ STAGE_ALL = 0x1F
 # dispatch + row gather, gate/up GEMM, down GEMM, combine (plus one memset of
 # the per-expert counters, which is not a kernel of this library).
 KERNELS_PER_FORWARD = 4
+# kernels one private-branch backward launches: gather, dL/da, gate and up
+# recompute, SwiGLU backward, three weight gradients, router, router weight
+# gradient partials and their reduction
+KERNELS_PER_BACKWARD = 11
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
             "pmpe_status_string", "pmpe_moe_forward_noalloc", "pmpe_selftest_wait_timeout",
-            "pmpe_policy_from_requests")
+            "pmpe_policy_from_requests", "pmpe_moe_backward_workspace_size", "pmpe_moe_backward_private")
 
 # Bytes of the library's static scratch array used by pmpe_moe_forward_noalloc.
 STATIC_SCRATCH_BYTES = 32 << 20
@@ -90,6 +94,10 @@ _lib.pmpe_moe_forward_stages.restype = ctypes.c_int
 _lib.pmpe_moe_forward_stages.argtypes = [ctypes.POINTER(MoeDesc), ctypes.c_uint, _vp]
 _lib.pmpe_moe_forward_noalloc.restype = ctypes.c_int
 _lib.pmpe_moe_forward_noalloc.argtypes = [ctypes.POINTER(MoeDesc), _vp]
+_lib.pmpe_moe_backward_workspace_size.restype = ctypes.c_size_t
+_lib.pmpe_moe_backward_workspace_size.argtypes = [ctypes.c_int] * 7
+_lib.pmpe_moe_backward_private.restype = ctypes.c_int
+_lib.pmpe_moe_backward_private.argtypes = [ctypes.POINTER(MoeDesc), _vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, _vp]
 _lib.pmpe_policy_from_requests.restype = ctypes.c_int
 _lib.pmpe_policy_from_requests.argtypes = [_vp, _vp, ctypes.c_int, ctypes.c_int, _vp, _vp]
 _lib.pmpe_selftest_wait_timeout.restype = ctypes.c_int
@@ -148,6 +156,14 @@ def audit_fields(words: np.ndarray, T: int, E: int) -> dict:
     return dict(status=int(a[0]), shared_rows=int(a[1]), route_count=a[2:2 + E], exec_rows=a[2 + E:2 + 2 * E],
                 exec_tiles=a[2 + 2 * E:2 + 3 * E], route_priv_rows=a[2 + 3 * E:2 + 3 * E + T],
                 exec_priv_rows=a[2 + 3 * E + T:2 + 3 * E + 2 * T])
+
+
+def private_gradient_shapes(s: LayerShape) -> dict:
+    """Shapes of the gradients the private-branch backward writes: the
+    private router and the private experts' gate, up and down weights, the
+    only parameters trained (G2, Sec. 2.2).  No public parameter has one."""
+    return {"d_router": (s.E_priv, s.H), "d_gate": (s.E_priv, s.I, s.H), "d_up": (s.E_priv, s.I, s.H),
+            "d_down": (s.E_priv, s.H, s.I)}
 
 
 def policy_from_requests(req_policy, cu_seqlens, T: int, out=None, stream=None):
@@ -239,6 +255,8 @@ class MoeLayer:
         self.weights = weights
         self.device = torch.device(device)
         self._ws = workspace if workspace is not None else Workspace(self.device)
+        self._bws = None
+        self._route_out = (None, None)  # the last forward's caller-owned route outputs
 
     def workspace(self, T: int) -> torch.Tensor:
         return self._ws.get(workspace_size(self._shape_T(T)))
@@ -262,4 +280,31 @@ class MoeLayer:
         desc = make_desc(s, self.weights, hidden, policy, out, self.workspace(T), topk_idx, topk_w, audit,
                          unmasked_control)
         forward_desc(desc, stages, stream)
+        self._route_out = (topk_idx, topk_w)
         return out
+
+    def backward_private(self, hidden, policy, dout, topk_idx=None, topk_w=None, stream=None) -> dict:
+        """Gradients of sum(dout * out) with respect to the private parameters
+        (router, gate, up, down; FP32) for the forward just run with the same
+        hidden states and policy on the same stream (its workspace holds the
+        route and the activations; the route outputs default to those that
+        forward wrote).  The public parameters get none."""
+        T = hidden.shape[0]
+        s = self._shape_T(T)
+        assert dout.is_contiguous() and dout.dtype == torch.bfloat16 and dout.shape == (T, s.H)
+        dev = hidden.device
+        g = {n: torch.empty(shp, dtype=torch.float32, device=dev) for n, shp in private_gradient_shapes(s).items()}
+        nb = _lib.pmpe_moe_backward_workspace_size(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k)
+        if nb == 0:
+            raise PmpeError(ERR_UNSUPPORTED_SHAPE, "pmpe_moe_backward_workspace_size")
+        if self._bws is None or self._bws.numel() < nb:
+            self._bws = torch.empty(nb, dtype=torch.uint8, device=dev)
+        bws = self._bws
+        if topk_idx is None and topk_w is None:
+            topk_idx, topk_w = self._route_out
+        # the descriptor's output pointer is never written by the backward
+        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w)
+        _check(_lib.pmpe_moe_backward_private(ctypes.byref(desc), _ptr(dout), _ptr(g["d_router"]), _ptr(g["d_gate"]),
+                                              _ptr(g["d_up"]), _ptr(g["d_down"]), _ptr(bws), bws.numel(),
+                                              _stream(stream)), "pmpe_moe_backward_private")
+        return g

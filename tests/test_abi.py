@@ -8,6 +8,7 @@ import re
 import shutil
 import subprocess
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -161,3 +162,68 @@ def test_validation_rejects_before_any_cuda_call(pmpe):
     assert lib.pmpe_selftest_wait_timeout(None, 1000, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 0, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_selftest_wait_timeout(ctypes.c_void_p(0x10000000), 1000001, None) == pmpe.ERR_INVALID_ARG
+
+
+def test_backward_validation_rejects_before_any_cuda_call(pmpe):
+    """The private-branch backward checks its gradient buffers, dout, the
+    control flag and its scratch size on the host; fake device pointers are
+    never dereferenced."""
+    from paper_2608_06690_gb300.inputs import LayerShape
+    lib = pmpe._lib
+    shape = LayerShape(64, 256, 128, 8, 4, 0, 2, True)
+    need = lib.pmpe_moe_backward_workspace_size(64, 256, 128, 8, 4, 0, 2)
+    assert need >= 256 and need % 256 == 0
+    assert lib.pmpe_moe_backward_workspace_size(64, 192, 128, 8, 4, 0, 2) == 0   # H % 128
+    assert lib.pmpe_moe_backward_workspace_size(0, 256, 128, 8, 4, 0, 2) == 256  # empty batch: the floor
+    # scratch grows with the routed rows
+    assert lib.pmpe_moe_backward_workspace_size(128, 256, 128, 8, 4, 0, 2) > need
+
+    class Fake:
+        def __init__(self, addr):
+            self.addr = addr
+
+        def data_ptr(self):
+            return self.addr
+
+        def numel(self):
+            return 1 << 40
+
+        def element_size(self):
+            return 1
+
+    p = Fake(0x10000000)
+    W = {n: p for n in ("router_pub", "router_priv", "gate_pub", "up_pub", "down_pub", "gate_priv", "up_priv",
+                        "down_priv")}
+    v = ctypes.c_void_p(p.addr)
+
+    def rc(desc_ok=True, dout=v, grads=(v, v, v, v), bws=v, nbytes=need, unmasked=False):
+        d = pmpe.make_desc(shape, W, p, None, p, p, unmasked_control=unmasked)
+        return lib.pmpe_moe_backward_private(ctypes.byref(d) if desc_ok else None, dout, *grads, bws, nbytes, None)
+
+    assert rc(desc_ok=False) == pmpe.ERR_INVALID_ARG
+    assert rc(dout=None) == pmpe.ERR_INVALID_ARG
+    assert rc(dout=ctypes.c_void_p(p.addr + 2)) == pmpe.ERR_INVALID_ARG
+    assert rc(grads=(v, None, v, v)) == pmpe.ERR_INVALID_ARG
+    assert rc(grads=(v, v, v, ctypes.c_void_p(p.addr + 4))) == pmpe.ERR_INVALID_ARG
+    assert rc(unmasked=True) == pmpe.ERR_UNSUPPORTED_SHAPE
+    assert rc(bws=None) == pmpe.ERR_WORKSPACE
+    assert rc(nbytes=need - 256) == pmpe.ERR_WORKSPACE
+    assert rc(bws=ctypes.c_void_p(p.addr + 16)) == pmpe.ERR_WORKSPACE
+
+
+def test_optimizer_partition_matches_the_papers_trainable_parameter_counts(pmpe):
+    """G2 optimizer partition (Sec. 2.2): the backward produces gradients for
+    the private router and private experts only, and over the paper's two
+    wrapped layers of 16 private experts their sizes add up to the trainable
+    parameter counts the paper's model table prints."""
+    import json
+    from paper_2608_06690_gb300.inputs import LayerShape
+    gold = json.load(open(os.path.join(ROOT, "tests", "golden", "trainable_parameters.json")))
+    for c in gold["cases"]:
+        s = LayerShape(T=1, H=c["H"], I=c["I"], E_pub=64, E_priv=c["E_priv"], E_sh=0, k=6, renormalize=True)
+        shapes = pmpe.private_gradient_shapes(s)
+        assert set(shapes) == {"d_router", "d_gate", "d_up", "d_down"}
+        per_layer = sum(int(np.prod(v)) for v in shapes.values())
+        assert c["wrapped_layers"] * per_layer == c["trainable_parameters"], c["model"]
+    # the binding has no entry point that could write a public parameter's gradient
+    assert not [n for n in pmpe.EXPORTED if "backward" in n and "pub" in n]
