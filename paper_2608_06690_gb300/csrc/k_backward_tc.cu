@@ -1,0 +1,657 @@
+// Backward of the private branch on the 5th-generation tensor cores (G2,
+// Sec. 2.2; Sec. 3.2 trains the private experts and the private router only).
+// Two persistent grouped GEMM launches over the private experts, each in the
+// TMA -> shared memory -> tcgen05.mma -> TMEM -> epilogue pipeline of the
+// forward's expert GEMMs:
+//
+//   bwd_dzgu_tc_kernel    rows of an expert as M, K = H:
+//     G = A W_gate^T, U = A W_up^T  (A: the expert's dispatched rows; recomputed)
+//     Z = D W_down                  (D: the rows' upstream gradients; W_down read MN-major)
+//   and in the epilogue, per row and column:
+//     act = bf16(silu(G) U) (the forward's activation), dL/dw partial = sum Z act,
+//     dG = w Z U silu'(G), dU = w Z silu(G)  -> BF16 [dG | dU];  w act -> BF16
+//   written in a padded row layout: expert q's rows start at a multiple of 128
+//   and the rows past its count are written as zeros.
+//
+//   bwd_wgrad_tc_kernel   rows of an expert as the contracted K:
+//     [dW_gate; dW_up]_q = [dG | dU]^T A     (M = 2I, N = H)
+//     dW_down_q          = D^T (w act)        (M = H,  N = I)
+//   both operands MN-major, read as stored (no transpose in memory); the zero
+//   rows of the padded operand cancel what the other operand holds past the
+//   expert's rows.  FP32 outputs.
+//
+// CTA roles (192 threads), as in the forward: warp 0 lanes 0-2 issue TMA
+// loads into a ring of stages, warp 1 allocates TMEM and one thread issues the
+// MMAs, warps 2-5 drain TMEM (one tile row per thread).  Every wait is bounded
+// in time; on expiry the CTA records PMPE_STATUS_PIPELINE_TIMEOUT, stops,
+// waits (bounded) for its copies and MMAs in flight, frees TMEM and exits.
+#include <cuda.h>
+
+#include <algorithm>
+#include <cstring>
+
+#include "pmpe_internal.cuh"
+#include "tc_ptx.cuh"
+
+namespace pmpe {
+namespace {
+
+constexpr int BM = 128;                        // MMA M (rows of a tile)
+constexpr int BK = 64;                         // K per stage
+constexpr int kABytes = BM * BK * 2;           // 16 KB
+constexpr int kBBytes = 256 * BK * 2;          // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kMnBlockBytes = 64 * BK * 2;     // one 64-element MN block of an MN-major operand: 8 KB
+constexpr int kThreads = 192;
+constexpr int kLoaders = 3;
+constexpr int kPad = 128;                      // padded row layout: each expert starts at a multiple of 128
+
+// dzgu: 4 stages, BF16 output boxes of 32 x 32 (64-byte rows), two per warp
+constexpr int kDzguStages = 4;
+constexpr int kOutBf16Bytes = 32 * 32 * 2;
+constexpr int kDzguOutBufs = 2;
+constexpr int kDzguDynSmem = kDzguStages * kStageBytes + 4 * kDzguOutBufs * kOutBf16Bytes + 1024;
+// wgrad: 3 stages, FP32 output boxes of 32 x 32 (128-byte rows), two per warp
+constexpr int kWgStages = 3;
+constexpr int kOutF32Bytes = 32 * 32 * 4;
+constexpr int kWgOutBufs = 2;
+constexpr int kWgDynSmem = kWgStages * kStageBytes + 4 * kWgOutBufs * kOutF32Bytes + 1024;
+constexpr int kTmemCols = 512;
+
+// Per private expert q: its rows, first row relative to the first private
+// slot, first row of the padded layout; and the tiles of the experts before q.
+struct GroupTable {
+    int tiles[kMaxPool + 1];
+    int rows[kMaxPool];
+    int off[kMaxPool];
+    int pad[kMaxPool];
+};
+
+// All threads: fill the table from the forward's dispatch offsets.
+// tiles_per_row_block: tiles of an expert per 128-row block (0: every expert
+// has `fixed_tiles` tiles whatever its rows).
+__device__ void build_groups(GroupTable &gt, const uint32_t *offsets, int E_pub, int E_priv, int R,
+                             int tiles_per_row_block, int fixed_tiles)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int p0 = (int)min(offsets[E_pub], (uint32_t)R);
+    for (int q = tid; q < E_priv; q += blockDim.x) {
+        const int b = min(max((int)offsets[E_pub + q], p0), R), e = min(max((int)offsets[E_pub + q + 1], b), R);
+        const int rows = e - b;
+        gt.rows[q] = rows;
+        gt.off[q] = b - p0;
+        gt.tiles[q + 1] = tiles_per_row_block ? ((rows + BM - 1) / BM) * tiles_per_row_block : fixed_tiles;
+        gt.pad[q] = (rows + kPad - 1) / kPad * kPad;  // made exclusive prefix below
+    }
+    __syncthreads();
+    if (warp < 2) {  // warp 0: inclusive scan of tiles; warp 1: exclusive scan of padded rows
+        int carry = 0;
+        for (int b = 0; b < E_priv; b += 32) {
+            const int q = b + lane;
+            const int v = q < E_priv ? (warp == 0 ? gt.tiles[q + 1] : gt.pad[q]) : 0;
+            int x = v;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(~0u, x, off);
+                if (lane >= off) x += y;
+            }
+            if (q < E_priv) {
+                if (warp == 0) gt.tiles[q + 1] = carry + x;
+                else gt.pad[q] = carry + x - v;
+            }
+            carry += __shfl_sync(~0u, x, 31);
+        }
+        if (warp == 0 && lane == 0) gt.tiles[0] = 0;
+    }
+    __syncthreads();
+}
+
+__device__ __forceinline__ void store_bf16_block(uint32_t sbuf, int lane, const uint32_t *pk)
+{
+    // 64-byte rows, 16-byte chunk j of row r at chunk j ^ ((r >> 1) & 3): the
+    // TMA 64-byte swizzle, conflict-free for these 16-byte writes
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[4 * j]), "r"(pk[4 * j + 1]),
+                     "r"(pk[4 * j + 2]), "r"(pk[4 * j + 3])
+                     : "memory");
+    }
+}
+
+__device__ __forceinline__ void store_f32_block(uint32_t sbuf, int lane, const float *v)
+{
+    // 128-byte rows, 16-byte chunk j of row r at chunk j ^ (r & 7): the TMA
+    // 128-byte swizzle
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const uint32_t addr = sbuf + lane * 128 + ((j ^ (lane & 7)) << 4);
+        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "f"(v[4 * j]), "f"(v[4 * j + 1]),
+                     "f"(v[4 * j + 2]), "f"(v[4 * j + 3])
+                     : "memory");
+    }
+}
+
+// Bounded wait for the drain at exit: every copy a loader issued has landed.
+__device__ __forceinline__ void drain_stages(uint32_t bar0, int stages, uint32_t filled, uint32_t last_parity)
+{
+    for (int s = 0; s < stages; ++s)
+        if ((filled >> s) & 1u) {
+            const unsigned long long t0 = globaltimer_ns();
+            while (!mbar_try_wait(bar0 + 8u * s, (last_parity >> s) & 1u))
+                if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+        }
+}
+
+// ------------------------------------------------------------- dzgu
+
+struct DzguParams {
+    int E_pub, E_priv, H, I, R;
+    const uint32_t *offsets;
+    const float *w_of_slot;
+    float *gw_part;  // [R][I / 128]: dL/dw partial of each private row per 128-column tile
+    uint32_t *status;
+    uint32_t idesc_gu, idesc_z;
+};
+
+struct DzguMaps {
+    CUtensorMap a_perm;     // [R][H], 64 x 128 box (K-major)
+    CUtensorMap dout_rows;  // [R + 64][H], 64 x 128 box (K-major)
+    CUtensorMap gate, up;   // [E_priv I][H], 64 x 128 box (K-major)
+    CUtensorMap down;       // [E_priv H][I], 64 x 64 box (MN-major B)
+    CUtensorMap dgu;        // [padded rows][2I], 32 x 32 box, 64-byte swizzle (store)
+    CUtensorMap wact;       // [padded rows][I], 32 x 32 box, 64-byte swizzle (store)
+};
+
+struct DzguTile {
+    int q, m0, n0, n_tile, rows;
+};
+
+__device__ __forceinline__ DzguTile decode_dzgu(const GroupTable &gt, int E_priv, int nt, int tile)
+{
+    int lo = 0, hi = E_priv - 1;  // last expert whose tile prefix is <= tile (skips empty experts)
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (gt.tiles[mid] <= tile) lo = mid; else hi = mid - 1;
+    }
+    DzguTile t;
+    t.q = lo;
+    const int mt = (gt.rows[lo] + BM - 1) / BM;
+    const int local = tile - gt.tiles[lo];
+    t.n_tile = local / mt;
+    const int m_tile = local - t.n_tile * mt;
+    t.m0 = m_tile * BM;
+    t.n0 = t.n_tile * 128;
+    t.rows = min(BM, gt.rows[lo] - t.m0);
+    return t;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) bwd_dzgu_tc_kernel(const DzguParams p, const __grid_constant__ DzguMaps maps)
+{
+    extern __shared__ uint8_t dsmem[];
+    __shared__ GroupTable gt;
+    __shared__ __align__(8) uint64_t bars[2 * kDzguStages + 3];
+    __shared__ uint32_t s_tmem;
+    __shared__ volatile int s_abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (kDzguStages + s); };
+    const uint32_t tfull_bar = bar0 + 8u * (2 * kDzguStages);
+    const uint32_t tempty_bar = tfull_bar + 8u;
+    const uint32_t done_bar = tfull_bar + 16u;
+
+    if (tid == 0) {
+        for (int s = 0; s < kDzguStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
+        mbar_init(tfull_bar, 1);
+        mbar_init(tempty_bar, 4);
+        mbar_init(done_bar, 1);
+        s_abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
+    pdl_wait();
+    const int nt = p.I / 128;
+    build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, nt, 0);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = s_tmem;
+    const int total = gt.tiles[p.E_priv];
+    const int nkh = p.H / BK;
+    const int p0 = (int)min(p.offsets[p.E_pub], (uint32_t)p.R);
+
+    if (warp == 0 && lane < kLoaders) {
+        // ------------------------------------------------ TMA producers
+        //   K blocks [0, nkh): lane 0 A rows, lane 1 gate rows, lane 2 up rows (16 KB each)
+        //   K blocks [nkh, 2 nkh): lane 0 dout rows (16 KB), lanes 1-2 one
+        //   64-column MN block of W_down each (8 KB)
+        int stage = 0;
+        uint32_t phase = 0, filled = 0, last_parity = 0;
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
+            const DzguTile t = decode_dzgu(gt, p.E_priv, nt, tile);
+            const int off = gt.off[t.q];
+            bool ok = true;
+            for (int kb = 0; kb < 2 * nkh; ++kb) {
+                if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
+                const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
+                const bool gu = kb < nkh;
+                const int kx = (gu ? kb : kb - nkh) * BK;
+                mbar_expect_tx(full_bar(stage), (gu || lane == 0) ? (uint32_t)kABytes : (uint32_t)kMnBlockBytes);
+                if (gu) {
+                    if (lane == 0)
+                        tma_load_2d(sA, &maps.a_perm, full_bar(stage), kx, p0 + off + t.m0);
+                    else
+                        tma_load_2d(sB + (lane - 1) * kABytes, lane == 1 ? &maps.gate : &maps.up, full_bar(stage), kx,
+                                    t.q * p.I + t.n0);
+                } else {
+                    if (lane == 0)
+                        tma_load_2d(sA, &maps.dout_rows, full_bar(stage), kx, off + t.m0);
+                    else
+                        tma_load_2d(sB + (lane - 1) * kMnBlockBytes, &maps.down, full_bar(stage), t.n0 + (lane - 1) * 64,
+                                    t.q * p.H + kx);
+                }
+                filled |= 1u << stage;
+                last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+                if (++stage == kDzguStages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+        }
+        drain_stages(bar0, kDzguStages, filled, last_parity);
+    } else if (warp == 1 && lane == 0) {
+        // ------------------------------------------------ MMA issuer
+        // TMEM columns: G [0, 128), U [128, 256) (one N = 256 MMA over gate and
+        // up rows), Z [256, 384); one accumulator set
+        int stage = 0, it = 0;
+        uint32_t phase = 0;
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x, ++it) {
+            if (!mbar_wait(tempty_bar, ((uint32_t)it & 1u) ^ 1u, &s_abort, p.status)) break;
+            tc_fence_after();
+            bool ok = true;
+            for (int kb = 0; kb < 2 * nkh; ++kb) {
+                if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
+                const uint64_t ad = sw128_desc(sA);
+                if (kb < nkh) {
+                    const uint64_t bd = sw128_desc(sB);
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k) tc_mma(tmem_base, ad + 2 * k, bd + 2 * k, p.idesc_gu, (kb | k) != 0);
+                } else {
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)  // 16 K rows of the MN-major operand: 2048 bytes
+                        tc_mma(tmem_base + 256, ad + 2 * k, mn_sw128_desc(sB + k * 2048, kMnBlockBytes), p.idesc_z,
+                               ((kb - nkh) | k) != 0);
+                }
+                tc_commit(empty_bar(stage));
+                if (++stage == kDzguStages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+            tc_commit(tfull_bar);
+        }
+        tc_commit(done_bar);
+        const unsigned long long t0 = globaltimer_ns();
+        while (!mbar_try_wait(done_bar, 0))
+            if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    } else if (warp >= 2) {
+        // ------------------------------------------------ epilogue
+        const int quarter = warp & 3;
+        const uint32_t out_base =
+            sbase + kDzguStages * kStageBytes + (uint32_t)((warp - 2) * kDzguOutBufs * kOutBf16Bytes);
+        int ob = 0, it = 0;
+        auto put = [&](const uint32_t *pk, const CUtensorMap *map, int x, int y) {
+            const uint32_t sbuf = out_base + (uint32_t)(ob * kOutBf16Bytes);
+            if (lane == 0) bulk_wait_read<kDzguOutBufs - 1>();  // the store that used this buffer has read it
+            __syncwarp();
+            store_bf16_block(sbuf, lane, pk);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tma_store_2d(map, sbuf, x, y);
+                bulk_commit();
+            }
+            ob = (ob + 1) % kDzguOutBufs;
+        };
+        for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+            const DzguTile t = decode_dzgu(gt, p.E_priv, nt, tile);
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(tfull_bar, (uint32_t)it & 1u, &s_abort, p.status) ? 1 : 0;
+            ok = __shfl_sync(~0u, ok, 0);
+            if (!ok) break;
+            __syncwarp();
+            tc_fence_after();
+            const int r = quarter * 32 + lane;
+            const bool valid = r < t.rows;
+            const int prow = gt.off[t.q] + t.m0 + r;  // private row (relative to the first private slot)
+            const float w = valid ? p.w_of_slot[p0 + prow] : 0.f;
+            const int orow = gt.pad[t.q] + t.m0 + quarter * 32;
+            const uint32_t tb = tmem_base + ((uint32_t)(quarter * 32) << 16);
+            float gw = 0.f;
+#pragma unroll 1
+            for (int c = 0; c < 4; ++c) {
+                float g[32], u[32], z[32];
+                tmem_ld32(tb + c * 32, g);
+                tmem_ld32(tb + 128 + c * 32, u);
+                tmem_ld32(tb + 256 + c * 32, z);
+                tmem_ld_wait();
+                uint32_t pg[16], pu[16], pa[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    float dg[2], du[2], wa[2];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int j = 2 * i + h;
+                        const float a = __bfloat162float(__float2bfloat16_rn(silu_mul(g[j], u[j])));
+                        gw += z[j] * a;
+                        const float sg = 1.f / (1.f + __expf(-g[j]));
+                        const float wz = w * z[j];
+                        dg[h] = valid ? wz * u[j] * sg * (1.f + g[j] * (1.f - sg)) : 0.f;
+                        du[h] = valid ? wz * g[j] * sg : 0.f;
+                        wa[h] = valid ? w * a : 0.f;
+                    }
+                    pg[i] = pack_bf16x2(dg[0], dg[1]);
+                    pu[i] = pack_bf16x2(du[0], du[1]);
+                    pa[i] = pack_bf16x2(wa[0], wa[1]);
+                }
+                put(pg, &maps.dgu, t.n0 + c * 32, orow);
+                put(pu, &maps.dgu, p.I + t.n0 + c * 32, orow);
+                put(pa, &maps.wact, t.n0 + c * 32, orow);
+            }
+            if (valid) p.gw_part[(size_t)prow * nt + t.n_tile] = gw;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty_bar);
+        }
+        if (lane == 0) bulk_wait_all();
+    }
+
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+// ------------------------------------------------------------- wgrad
+
+struct WgParams {
+    int E_pub, E_priv, H, I, R;
+    int bn_a, bn_b;  // output columns per tile: [dW_gate; dW_up] (N = H), dW_down (N = I)
+    const uint32_t *offsets;
+    uint32_t *status;
+    uint32_t idesc_a, idesc_b;
+};
+
+struct WgMaps {
+    CUtensorMap dgu;        // [padded rows][2I], 64 x 64 box (MN-major A)
+    CUtensorMap a_perm;     // [R][H], 64 x 64 box (MN-major B)
+    CUtensorMap dout_rows;  // [R + 64][H], 64 x 64 box (MN-major A)
+    CUtensorMap wact;       // [padded rows][I], 64 x 64 box (MN-major B)
+    CUtensorMap d_gate, d_up, d_down;  // FP32 outputs, 32 x 32 boxes, 128-byte swizzle
+};
+
+struct WgTile {
+    int prob, q, m0, n0, bn, nkb;
+};
+
+__device__ __forceinline__ WgTile decode_wg(const WgParams &p, const GroupTable &gt, int tile)
+{
+    WgTile t;
+    const int na = p.H / p.bn_a, nta = (2 * p.I / BM) * na;
+    const int nb = p.I / p.bn_b, ntb = (p.H / BM) * nb;
+    int local;
+    if (tile < p.E_priv * nta) {
+        t.prob = 0;
+        t.q = tile / nta;
+        local = tile - t.q * nta;
+        t.m0 = (local / na) * BM;
+        t.n0 = (local % na) * p.bn_a;
+        t.bn = p.bn_a;
+    } else {
+        tile -= p.E_priv * nta;
+        t.prob = 1;
+        t.q = tile / ntb;
+        local = tile - t.q * ntb;
+        t.m0 = (local / nb) * BM;
+        t.n0 = (local % nb) * p.bn_b;
+        t.bn = p.bn_b;
+    }
+    t.nkb = (gt.rows[t.q] + BK - 1) / BK;
+    return t;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParams p, const __grid_constant__ WgMaps maps)
+{
+    extern __shared__ uint8_t dsmem[];
+    __shared__ GroupTable gt;
+    __shared__ __align__(8) uint64_t bars[2 * kWgStages + 5];
+    __shared__ uint32_t s_tmem;
+    __shared__ volatile int s_abort;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (kWgStages + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kWgStages + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kWgStages + 2 + b); };
+    const uint32_t done_bar = bar0 + 8u * (2 * kWgStages + 4);
+
+    if (tid == 0) {
+        for (int s = 0; s < kWgStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
+        for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
+        mbar_init(done_bar, 1);
+        s_abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
+    pdl_wait();
+    build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, 0, 0);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = s_tmem;
+    const int total = p.E_priv * ((2 * p.I / BM) * (p.H / p.bn_a) + (p.H / BM) * (p.I / p.bn_b));
+    const int p0 = (int)min(p.offsets[p.E_pub], (uint32_t)p.R);
+
+    if (warp == 0 && lane < kLoaders) {
+        // ------------------------------------------------ TMA producers
+        // lane 0: the two 64-element MN blocks of A; lanes 1-2: half of B's
+        // bn / 64 blocks each.  Boxes are 64 MN elements x 64 rows (K).
+        int stage = 0;
+        uint32_t phase = 0, filled = 0, last_parity = 0;
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
+            const WgTile t = decode_wg(p, gt, tile);
+            const int nbox = t.bn / 64, half = nbox / 2;
+            const int rowA = t.prob == 0 ? gt.pad[t.q] : gt.off[t.q];
+            const int rowB = t.prob == 0 ? p0 + gt.off[t.q] : gt.pad[t.q];
+            const CUtensorMap *amap = t.prob == 0 ? &maps.dgu : &maps.dout_rows;
+            const CUtensorMap *bmap = t.prob == 0 ? &maps.a_perm : &maps.wact;
+            bool ok = true;
+            for (int kb = 0; kb < t.nkb; ++kb) {
+                if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
+                const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
+                const int ky = kb * BK;
+                mbar_expect_tx(full_bar(stage), lane == 0 ? (uint32_t)kABytes : (uint32_t)(half * kMnBlockBytes));
+                if (lane == 0) {
+                    tma_load_2d(sA, amap, full_bar(stage), t.m0, rowA + ky);
+                    tma_load_2d(sA + kMnBlockBytes, amap, full_bar(stage), t.m0 + 64, rowA + ky);
+                } else {
+                    for (int b = (lane - 1) * half; b < lane * half; ++b)
+                        tma_load_2d(sB + b * kMnBlockBytes, bmap, full_bar(stage), t.n0 + b * 64, rowB + ky);
+                }
+                filled |= 1u << stage;
+                last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+                if (++stage == kWgStages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+        }
+        drain_stages(bar0, kWgStages, filled, last_parity);
+    } else if (warp == 1 && lane == 0) {
+        // ------------------------------------------------ MMA issuer
+        // two 128 x 256 FP32 accumulators: the epilogue of one tile overlaps the
+        // MMAs of the next.  A tile of an expert without rows issues no MMA;
+        // its epilogue writes zeros.
+        int stage = 0, it = 0;
+        uint32_t phase = 0;
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x, ++it) {
+            const WgTile t = decode_wg(p, gt, tile);
+            const uint32_t idesc = t.prob == 0 ? p.idesc_a : p.idesc_b;
+            const int buf = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            if (!mbar_wait(tempty_bar(buf), use ^ 1u, &s_abort, p.status)) break;
+            tc_fence_after();
+            const uint32_t d_tmem = tmem_base + (uint32_t)(buf * 256);
+            bool ok = true;
+            for (int kb = 0; kb < t.nkb; ++kb) {
+                if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                    tc_mma(d_tmem, mn_sw128_desc(sA + k * 2048, kMnBlockBytes), mn_sw128_desc(sB + k * 2048, kMnBlockBytes),
+                           idesc, (kb | k) != 0);
+                tc_commit(empty_bar(stage));
+                if (++stage == kWgStages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+            tc_commit(tfull_bar(buf));
+        }
+        tc_commit(done_bar);
+        const unsigned long long t0 = globaltimer_ns();
+        while (!mbar_try_wait(done_bar, 0))
+            if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    } else if (warp >= 2) {
+        // ------------------------------------------------ epilogue
+        const int quarter = warp & 3;
+        const uint32_t out_base = sbase + kWgStages * kStageBytes + (uint32_t)((warp - 2) * kWgOutBufs * kOutF32Bytes);
+        int ob = 0, it = 0;
+        for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+            const WgTile t = decode_wg(p, gt, tile);
+            const int buf = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(tfull_bar(buf), use, &s_abort, p.status) ? 1 : 0;
+            ok = __shfl_sync(~0u, ok, 0);
+            if (!ok) break;
+            __syncwarp();
+            tc_fence_after();
+            const CUtensorMap *omap;
+            int orow;
+            if (t.prob == 0) {
+                omap = t.m0 < p.I ? &maps.d_gate : &maps.d_up;
+                orow = t.q * p.I + (t.m0 < p.I ? t.m0 : t.m0 - p.I);
+            } else {
+                omap = &maps.d_down;
+                orow = t.q * p.H + t.m0;
+            }
+            orow += quarter * 32;
+            const uint32_t tb = tmem_base + (uint32_t)(buf * 256) + ((uint32_t)(quarter * 32) << 16);
+#pragma unroll 1
+            for (int c = 0; c < t.bn / 32; ++c) {
+                float v[32];
+                if (t.nkb > 0) {
+                    tmem_ld32(tb + c * 32, v);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = 0.f;
+                }
+                const uint32_t sbuf = out_base + (uint32_t)(ob * kOutF32Bytes);
+                if (lane == 0) bulk_wait_read<kWgOutBufs - 1>();
+                __syncwarp();
+                store_f32_block(sbuf, lane, v);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(omap, sbuf, t.n0 + c * 32, orow);
+                    bulk_commit();
+                }
+                ob = (ob + 1) % kWgOutBufs;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty_bar(buf));
+        }
+        if (lane == 0) bulk_wait_all();
+    }
+
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+}  // namespace
+
+// Rows of the padded layout (an upper bound over all routings).
+size_t backward_padded_rows(const Shape &s) { return (size_t)s.T * s.k + (size_t)kPad * s.E_priv; }
+
+cudaError_t launch_backward_dzgu(const Ctx &c, const bf16 *dout_rows, bf16 *dgu, bf16 *wact, float *gw_part)
+{
+    const Shape &s = c.s;
+    const uint64_t R = (uint64_t)s.T * s.k, RP = backward_padded_rows(s);
+    DzguParams p;
+    DzguMaps maps;
+    memset(&p, 0, sizeof(p));
+    memset(&maps, 0, sizeof(maps));
+    p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.H = s.H; p.I = s.I; p.R = (int)R;
+    p.offsets = c.offsets;
+    p.w_of_slot = c.w_of_slot;
+    p.gw_part = gw_part;
+    p.status = c.audit.status;
+    p.idesc_gu = make_idesc(BM, 256);
+    p.idesc_z = make_idesc_major(BM, 128, false, true);
+    bool ok = encode_2d(&maps.a_perm, c.a_perm, s.H, R, BM);
+    ok &= encode_2d(&maps.dout_rows, dout_rows, s.H, R + 64, BM);
+    ok &= encode_2d(&maps.gate, c.gate[1], s.H, (uint64_t)s.E_priv * s.I, 128);
+    ok &= encode_2d(&maps.up, c.up[1], s.H, (uint64_t)s.E_priv * s.I, 128);
+    ok &= encode_2d_box(&maps.down, c.down[1], s.I, (uint64_t)s.E_priv * s.H, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
+    ok &= encode_2d_box(&maps.dgu, dgu, 2 * (uint64_t)s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+    ok &= encode_2d_box(&maps.wact, wact, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+    if (!ok) return cudaErrorInvalidValue;
+    static std::atomic<int> smem_limit[64];
+    cudaError_t err = ensure_dynamic_smem(bwd_dzgu_tc_kernel, kDzguDynSmem, smem_limit);
+    if (err != cudaSuccess) return err;
+    return launch_pdl(bwd_dzgu_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDzguDynSmem, c.stream, p, maps);
+}
+
+cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
+                                  float *d_gate, float *d_up, float *d_down)
+{
+    const Shape &s = c.s;
+    const uint64_t R = (uint64_t)s.T * s.k, RP = backward_padded_rows(s);
+    WgParams p;
+    WgMaps maps;
+    memset(&p, 0, sizeof(p));
+    memset(&maps, 0, sizeof(maps));
+    p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.H = s.H; p.I = s.I; p.R = (int)R;
+    p.bn_a = s.H % 256 == 0 ? 256 : 128;
+    p.bn_b = s.I % 256 == 0 ? 256 : 128;
+    p.offsets = c.offsets;
+    p.status = c.audit.status;
+    p.idesc_a = make_idesc_major(BM, p.bn_a, true, true);
+    p.idesc_b = make_idesc_major(BM, p.bn_b, true, true);
+    const CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_128B;
+    bool ok = encode_2d_box(&maps.dgu, dgu, 2 * (uint64_t)s.I, RP, 64, 64, sw);
+    ok &= encode_2d_box(&maps.a_perm, c.a_perm, s.H, R, 64, 64, sw);
+    ok &= encode_2d_box(&maps.dout_rows, dout_rows, s.H, R + 64, 64, 64, sw);
+    ok &= encode_2d_box(&maps.wact, wact, s.I, RP, 64, 64, sw);
+    ok &= encode_2d_f32(&maps.d_gate, d_gate, s.H, (uint64_t)s.E_priv * s.I, 32, 32, sw);
+    ok &= encode_2d_f32(&maps.d_up, d_up, s.H, (uint64_t)s.E_priv * s.I, 32, 32, sw);
+    ok &= encode_2d_f32(&maps.d_down, d_down, s.I, (uint64_t)s.E_priv * s.H, 32, 32, sw);
+    if (!ok) return cudaErrorInvalidValue;
+    static std::atomic<int> smem_limit[64];
+    cudaError_t err = ensure_dynamic_smem(bwd_wgrad_tc_kernel, kWgDynSmem, smem_limit);
+    if (err != cudaSuccess) return err;
+    return launch_pdl(bwd_wgrad_tc_kernel, dim3(c.num_sms), dim3(kThreads), kWgDynSmem, c.stream, p, maps);
+}
+
+}  // namespace pmpe

@@ -566,20 +566,32 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// 2-D BF16 tensor map over a row-major [rows, cols] matrix, box = 64 x box_rows,
-// 128-byte swizzle, zero fill out of bounds.
-bool encode_2d_box(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
-                   uint32_t box_rows, CUtensorMapSwizzle swizzle)
+// 2-D tensor map over a row-major [rows, cols] matrix of `type` elements of
+// `elem_bytes` bytes, box = box_cols x box_rows, zero fill out of bounds.
+static bool encode_2d_typed(CUtensorMap *m, CUtensorMapDataType type, uint32_t elem_bytes, const void *ptr,
+                            uint64_t cols, uint64_t rows, uint32_t box_cols, uint32_t box_rows,
+                            CUtensorMapSwizzle swizzle)
 {
     auto fn = encode_fn();
     if (!fn) return false;
     const cuuint64_t dims[2] = {cols, rows};
-    const cuuint64_t strides[1] = {cols * 2};
+    const cuuint64_t strides[1] = {cols * elem_bytes};
     const cuuint32_t box[2] = {box_cols, box_rows};
     const cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return fn(m, type, 2, const_cast<void *>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_2d_box(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
+                   uint32_t box_rows, CUtensorMapSwizzle swizzle)
+{
+    return encode_2d_typed(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, cols, rows, box_cols, box_rows, swizzle);
+}
+
+bool encode_2d_f32(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
+                   uint32_t box_rows, CUtensorMapSwizzle swizzle)
+{
+    return encode_2d_typed(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, ptr, cols, rows, box_cols, box_rows, swizzle);
 }
 
 bool encode_2d(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_rows)
@@ -594,6 +606,11 @@ uint32_t make_idesc(int M, int N)
            | (1u << 10)                 // B: BF16
            | ((uint32_t)(N >> 3) << 17) // N / 8
            | ((uint32_t)(M >> 4) << 24);// M / 16   (A and B K-major: transpose bits 15, 16 = 0)
+}
+
+uint32_t make_idesc_major(int M, int N, bool a_mn_major, bool b_mn_major)
+{
+    return make_idesc(M, N) | ((a_mn_major ? 1u : 0u) << 15) | ((b_mn_major ? 1u : 0u) << 16);
 }
 
 

@@ -89,6 +89,16 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
            ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
+// Shared-memory matrix descriptor: MN-major operand, 128-byte swizzle.  The
+// operand is stored as blocks of 64 MN-contiguous elements (one 128-byte row
+// per K index, 8-row / 1024-byte swizzle atoms along K, SBO = 1024); LBO is the
+// byte distance between consecutive 64-element MN blocks.
+__device__ __forceinline__ uint64_t mn_sw128_desc(uint32_t saddr, uint32_t lbo_bytes)
+{
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo_bytes >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
 __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                        uint32_t accumulate)
 {
@@ -173,7 +183,12 @@ bool encode_2d(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, ui
 // 2-D BF16 tensor map with a box_cols x box_rows box and the given swizzle.
 bool encode_2d_box(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
                    uint32_t box_rows, CUtensorMapSwizzle swizzle);
+// 2-D FP32 tensor map with a box_cols x box_rows box and the given swizzle.
+bool encode_2d_f32(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
+                   uint32_t box_rows, CUtensorMapSwizzle swizzle);
 // tcgen05 instruction descriptor: BF16 x BF16 -> FP32, both operands K-major.
 uint32_t make_idesc(int M, int N);
+// The same with either operand MN-major (transpose bits 15 for A, 16 for B).
+uint32_t make_idesc_major(int M, int N, bool a_mn_major, bool b_mn_major);
 
 }  // namespace pmpe

@@ -16,9 +16,9 @@ pytestmark = pytest.mark.gpu
 
 # Gradient tolerance: per tensor, max-abs error <= 2e-2 * max|ref| and
 # sum|err| / sum|ref| <= 1e-2.  The GPU contracts BF16 operands with FP32
-# accumulation and rounds three intermediates to BF16 (w * dout, and the
-# SwiGLU input gradients dG, dU: 2^-9 relative each), which the weight
-# gradients then sum over an expert's rows.
+# accumulation and rounds three intermediates to BF16 (the SwiGLU input
+# gradients dG, dU and the weighted activation w * act: 2^-9 relative each),
+# which the weight gradients then sum over an expert's rows.
 MAX_ABS_REL = 2e-2
 MEAN_REL = 1e-2
 
