@@ -210,12 +210,12 @@ int router_splits(const Shape &s, int num_sms, int *tok_per_split)
 
 }  // namespace
 
-// Scratch of the backward, in order: dout rows [R + 64][H], [dG | dU] and
-// w act in the padded row layout ([RP][2I], [RP][I], BF16), the dL/dw
+// Scratch of the backward, in order: dout rows [R + 64][H], Z, [dG | dU] and
+// w act in the padded row layout ([RP][I], [RP][2I], [RP][I], BF16), the dL/dw
 // partials [R][I / 128], dz [T][E_priv] and the router weight-gradient
 // partials [splits][E_priv][H] (FP32).
 struct BwdScratch {
-    bf16 *dout_rows, *dgu, *wact;
+    bf16 *dout_rows, *zpad, *dgu, *wact;
     float *gw_part, *dz, *part;
     size_t bytes;
 };
@@ -228,6 +228,7 @@ static BwdScratch backward_scratch(const Shape &s, uint8_t *base)
     BwdScratch b;
     size_t o = 0;
     b.dout_rows = (bf16 *)(base + o); o += al((R + 64) * H * 2);
+    b.zpad = (bf16 *)(base + o);      o += al(RP * I * 2);
     b.dgu = (bf16 *)(base + o);       o += al(RP * 2 * I * 2);
     b.wact = (bf16 *)(base + o);      o += al(RP * I * 2);
     b.gw_part = (float *)(base + o);  o += al(R * (I / 128) * 4);
@@ -255,7 +256,7 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
     bwd_gather_kernel<<<c.num_sms * 8, 256, 0, st>>>(dout, c.tok_of_slot, c.offsets, s.E_pub, E, R, H, b.dout_rows);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    if ((err = launch_backward_dzgu(c, b.dout_rows, b.dgu, b.wact, b.gw_part)) != cudaSuccess) return err;
+    if ((err = launch_backward_rows(c, b.dout_rows, b.zpad, b.dgu, b.wact, b.gw_part)) != cudaSuccess) return err;
 
     bwd_router_kernel<<<c.num_sms * 4, 256, 0, st>>>(c.hidden, c.router_priv, c.tau, c.idx, c.w, c.slot_of, b.gw_part,
                                                      s.I / 128, c.offsets, s.T, H, s.E_pub, s.E_priv, s.k, s.renorm, R,

@@ -1,17 +1,19 @@
 // Backward of the private branch on the 5th-generation tensor cores (G2,
 // Sec. 2.2; Sec. 3.2 trains the private experts and the private router only).
-// Two persistent grouped GEMM launches over the private experts, each in the
+// Three persistent grouped GEMM launches over the private experts, each in the
 // TMA -> shared memory -> tcgen05.mma -> TMEM -> epilogue pipeline of the
 // forward's expert GEMMs:
 //
-//   bwd_dzgu_tc_kernel    rows of an expert as M, K = H:
+//   bwd_rows_tc_kernel<kRowsZ>    rows of an expert as M, K = H:
+//     Z = D W_down                  (D: the rows' upstream gradients; W_down read
+//                                    MN-major; so dL/da = w Z) -> BF16
+//   bwd_rows_tc_kernel<kRowsGU>   rows of an expert as M, K = H:
 //     G = A W_gate^T, U = A W_up^T  (A: the expert's dispatched rows; recomputed)
-//     Z = D W_down                  (D: the rows' upstream gradients; W_down read MN-major)
-//   and in the epilogue, per row and column:
+//   and in the epilogue, with Z read back, per row and column:
 //     act = bf16(silu(G) U) (the forward's activation), dL/dw partial = sum Z act,
 //     dG = w Z U silu'(G), dU = w Z silu(G)  -> BF16 [dG | dU];  w act -> BF16
-//   written in a padded row layout: expert q's rows start at a multiple of 128
-//   and the rows past its count are written as zeros.
+//   Z, [dG | dU] and w act use a padded row layout: expert q's rows start at a
+//   multiple of 128, and the rows past its count of the last two are zeros.
 //
 //   bwd_wgrad_tc_kernel   rows of an expert as the contracted K:
 //     [dW_gate; dW_up]_q = [dG | dU]^T A     (M = 2I, N = H)
@@ -20,11 +22,13 @@
 //   rows of the padded operand cancel what the other operand holds past the
 //   expert's rows.  FP32 outputs.
 //
-// CTA roles (192 threads), as in the forward: warp 0 lanes 0-2 issue TMA
-// loads into a ring of stages, warp 1 allocates TMEM and one thread issues the
-// MMAs, warps 2-5 drain TMEM (one tile row per thread).  Every wait is bounded
-// in time; on expiry the CTA records PMPE_STATUS_PIPELINE_TIMEOUT, stops,
-// waits (bounded) for its copies and MMAs in flight, frees TMEM and exits.
+// Every launch keeps four 48 KB operand stages in flight (a 128 x 256 x 64 MMA
+// block each) and two 128 x 256 FP32 accumulators, so the epilogue of one tile
+// overlaps the MMAs of the next.  CTA roles (192 threads), as in the forward:
+// warp 0 lanes 0-2 issue TMA loads, warp 1 allocates TMEM and one thread
+// issues the MMAs, warps 2-5 drain TMEM (one tile row per thread).  Every wait
+// is bounded in time; on expiry the CTA records PMPE_STATUS_PIPELINE_TIMEOUT,
+// stops, waits (bounded) for its copies and MMAs in flight, frees TMEM and exits.
 #include <cuda.h>
 
 #include <algorithm>
@@ -46,17 +50,14 @@ constexpr int kThreads = 192;
 constexpr int kLoaders = 3;
 constexpr int kPad = 128;                      // padded row layout: each expert starts at a multiple of 128
 
-// dzgu: 4 stages, BF16 output boxes of 32 x 32 (64-byte rows), two per warp
-constexpr int kDzguStages = 4;
-constexpr int kOutBf16Bytes = 32 * 32 * 2;
-constexpr int kDzguOutBufs = 2;
-constexpr int kDzguDynSmem = kDzguStages * kStageBytes + 4 * kDzguOutBufs * kOutBf16Bytes + 1024;
-// wgrad: 3 stages, FP32 output boxes of 32 x 32 (128-byte rows), two per warp
-constexpr int kWgStages = 3;
-constexpr int kOutF32Bytes = 32 * 32 * 4;
-constexpr int kWgOutBufs = 2;
-constexpr int kWgDynSmem = kWgStages * kStageBytes + 4 * kWgOutBufs * kOutF32Bytes + 1024;
-constexpr int kTmemCols = 512;
+// Four operand stages; outputs staged per epilogue warp in two 2 KB boxes of
+// 32 rows x 64 bytes (32 BF16 or 16 FP32 columns, 64-byte swizzle).
+constexpr int kStages = 4;
+constexpr int kOutBoxBytes = 32 * 64;
+constexpr int kOutBufs = 2;
+constexpr int kDynSmem = kStages * kStageBytes + 4 * kOutBufs * kOutBoxBytes + 1024;
+constexpr int kAccCols = 256;
+constexpr int kTmemCols = 2 * kAccCols;
 
 // Per private expert q: its rows, first row relative to the first private
 // slot, first row of the padded layout; and the tiles of the experts before q.
@@ -106,31 +107,40 @@ __device__ void build_groups(GroupTable &gt, const uint32_t *offsets, int E_pub,
     __syncthreads();
 }
 
-__device__ __forceinline__ void store_bf16_block(uint32_t sbuf, int lane, const uint32_t *pk)
+// This lane's 64-byte row of a staged output box: 16-byte chunk j of row r at
+// chunk j ^ ((r >> 1) & 3), the TMA 64-byte swizzle (conflict-free for these
+// 16-byte writes).
+__device__ __forceinline__ void store_box_row(uint32_t sbuf, int lane, const uint32_t *w16)
 {
-    // 64-byte rows, 16-byte chunk j of row r at chunk j ^ ((r >> 1) & 3): the
-    // TMA 64-byte swizzle, conflict-free for these 16-byte writes
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
         const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[4 * j]), "r"(pk[4 * j + 1]),
-                     "r"(pk[4 * j + 2]), "r"(pk[4 * j + 3])
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(w16[4 * j]), "r"(w16[4 * j + 1]),
+                     "r"(w16[4 * j + 2]), "r"(w16[4 * j + 3])
                      : "memory");
     }
 }
 
-__device__ __forceinline__ void store_f32_block(uint32_t sbuf, int lane, const float *v)
-{
-    // 128-byte rows, 16-byte chunk j of row r at chunk j ^ (r & 7): the TMA
-    // 128-byte swizzle
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const uint32_t addr = sbuf + lane * 128 + ((j ^ (lane & 7)) << 4);
-        asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "f"(v[4 * j]), "f"(v[4 * j + 1]),
-                     "f"(v[4 * j + 2]), "f"(v[4 * j + 3])
-                     : "memory");
+// One epilogue warp's output path: stage a 32 x 64-byte box in one of two
+// shared buffers and store it with TMA.
+struct OutStager {
+    uint32_t base;
+    int ob;
+    __device__ __forceinline__ void put(int lane, const uint32_t *w16, const CUtensorMap *map, int x, int y)
+    {
+        const uint32_t sbuf = base + (uint32_t)(ob * kOutBoxBytes);
+        if (lane == 0) bulk_wait_read<kOutBufs - 1>();  // the store that used this buffer has read it
+        __syncwarp();
+        store_box_row(sbuf, lane, w16);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+            tma_store_2d(map, sbuf, x, y);
+            bulk_commit();
+        }
+        ob ^= 1;
     }
-}
+};
 
 // Bounded wait for the drain at exit: every copy a loader issued has landed.
 __device__ __forceinline__ void drain_stages(uint32_t bar0, int stages, uint32_t filled, uint32_t last_parity)
@@ -143,54 +153,57 @@ __device__ __forceinline__ void drain_stages(uint32_t bar0, int stages, uint32_t
         }
 }
 
-// ------------------------------------------------------------- dzgu
+// ------------------------------------------------------------- rows
 
-struct DzguParams {
+enum { kRowsZ = 0, kRowsGU = 1 };
+
+struct RowsParams {
     int E_pub, E_priv, H, I, R;
+    int bn;           // output columns per tile (Z: of I, 256 or 128; gate/up: 128 activation columns)
     const uint32_t *offsets;
     const float *w_of_slot;
-    float *gw_part;  // [R][I / 128]: dL/dw partial of each private row per 128-column tile
+    const bf16 *zpad;  // gate/up: Z in the padded row layout [RP][I]
+    float *gw_part;    // gate/up: [R][I / 128] dL/dw partial of each private row per 128-column tile
     uint32_t *status;
-    uint32_t idesc_gu, idesc_z;
+    uint32_t idesc;
 };
 
-struct DzguMaps {
-    CUtensorMap a_perm;     // [R][H], 64 x 128 box (K-major)
-    CUtensorMap dout_rows;  // [R + 64][H], 64 x 128 box (K-major)
-    CUtensorMap gate, up;   // [E_priv I][H], 64 x 128 box (K-major)
-    CUtensorMap down;       // [E_priv H][I], 64 x 64 box (MN-major B)
-    CUtensorMap dgu;        // [padded rows][2I], 32 x 32 box, 64-byte swizzle (store)
-    CUtensorMap wact;       // [padded rows][I], 32 x 32 box, 64-byte swizzle (store)
+struct RowsMaps {
+    CUtensorMap a;       // Z: dout rows [R + 64][H]; gate/up: A rows [R][H]; 64 x 128 box (K-major)
+    CUtensorMap b0, b1;  // Z: W_down [E_priv H][I], 64 x 64 box (MN-major); gate/up: gate, up [E_priv I][H], 64 x 128
+    CUtensorMap out0;    // Z: Z [RP][I]; gate/up: [dG | dU] [RP][2I]  (32 x 32 BF16 boxes, 64-byte swizzle)
+    CUtensorMap out1;    // gate/up: w act [RP][I]
 };
 
-struct DzguTile {
+struct RowsTile {
     int q, m0, n0, n_tile, rows;
 };
 
-__device__ __forceinline__ DzguTile decode_dzgu(const GroupTable &gt, int E_priv, int nt, int tile)
+__device__ __forceinline__ RowsTile decode_rows(const GroupTable &gt, int E_priv, int nt, int bn, int tile)
 {
     int lo = 0, hi = E_priv - 1;  // last expert whose tile prefix is <= tile (skips empty experts)
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
         if (gt.tiles[mid] <= tile) lo = mid; else hi = mid - 1;
     }
-    DzguTile t;
+    RowsTile t;
     t.q = lo;
     const int mt = (gt.rows[lo] + BM - 1) / BM;
     const int local = tile - gt.tiles[lo];
-    t.n_tile = local / mt;
+    t.n_tile = local / mt;  // n-tile major inside an expert: its m tiles share the weight slice
     const int m_tile = local - t.n_tile * mt;
     t.m0 = m_tile * BM;
-    t.n0 = t.n_tile * 128;
+    t.n0 = t.n_tile * bn;
     t.rows = min(BM, gt.rows[lo] - t.m0);
     return t;
 }
 
-__global__ void __launch_bounds__(kThreads, 1) bwd_dzgu_tc_kernel(const DzguParams p, const __grid_constant__ DzguMaps maps)
+template <int kMode>
+__global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsParams p, const __grid_constant__ RowsMaps maps)
 {
     extern __shared__ uint8_t dsmem[];
     __shared__ GroupTable gt;
-    __shared__ __align__(8) uint64_t bars[2 * kDzguStages + 3];
+    __shared__ __align__(8) uint64_t bars[2 * kStages + 5];
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
 
@@ -198,98 +211,96 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_dzgu_tc_kernel(const DzguPara
     const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
-    auto empty_bar = [&](int s) { return bar0 + 8u * (kDzguStages + s); };
-    const uint32_t tfull_bar = bar0 + 8u * (2 * kDzguStages);
-    const uint32_t tempty_bar = tfull_bar + 8u;
-    const uint32_t done_bar = tfull_bar + 16u;
+    auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
+    const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
 
     if (tid == 0) {
-        for (int s = 0; s < kDzguStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
-        mbar_init(tfull_bar, 1);
-        mbar_init(tempty_bar, 4);
+        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
+        for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
         mbar_init(done_bar, 1);
         s_abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
     pdl_wait();
-    const int nt = p.I / 128;
+    const int nt = p.I / p.bn;
     build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, nt, 0);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
     const int total = gt.tiles[p.E_priv];
-    const int nkh = p.H / BK;
+    const int nkb = p.H / BK;
     const int p0 = (int)min(p.offsets[p.E_pub], (uint32_t)p.R);
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
-        //   K blocks [0, nkh): lane 0 A rows, lane 1 gate rows, lane 2 up rows (16 KB each)
-        //   K blocks [nkh, 2 nkh): lane 0 dout rows (16 KB), lanes 1-2 one
-        //   64-column MN block of W_down each (8 KB)
+        // lane 0: the tile's 128 rows x 64 K of A (16 KB).  Gate/up: lane 1 the
+        // 128 gate rows, lane 2 the 128 up rows (16 KB each).  Z: lanes 1-2 half
+        // of the bn / 64 MN blocks of W_down each (8 KB per block).
         int stage = 0;
         uint32_t phase = 0, filled = 0, last_parity = 0;
+        const int half = p.bn / 128;  // Z: MN blocks per loader lane
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
-            const DzguTile t = decode_dzgu(gt, p.E_priv, nt, tile);
-            const int off = gt.off[t.q];
+            const RowsTile t = decode_rows(gt, p.E_priv, nt, p.bn, tile);
+            const int arow = (kMode == kRowsGU ? p0 : 0) + gt.off[t.q] + t.m0;
             bool ok = true;
-            for (int kb = 0; kb < 2 * nkh; ++kb) {
+            for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
                 const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
-                const bool gu = kb < nkh;
-                const int kx = (gu ? kb : kb - nkh) * BK;
-                mbar_expect_tx(full_bar(stage), (gu || lane == 0) ? (uint32_t)kABytes : (uint32_t)kMnBlockBytes);
-                if (gu) {
-                    if (lane == 0)
-                        tma_load_2d(sA, &maps.a_perm, full_bar(stage), kx, p0 + off + t.m0);
-                    else
-                        tma_load_2d(sB + (lane - 1) * kABytes, lane == 1 ? &maps.gate : &maps.up, full_bar(stage), kx,
-                                    t.q * p.I + t.n0);
+                const int kx = kb * BK;
+                if (lane == 0) {
+                    mbar_expect_tx(full_bar(stage), kABytes);
+                    tma_load_2d(sA, &maps.a, full_bar(stage), kx, arow);
+                } else if (kMode == kRowsGU) {
+                    mbar_expect_tx(full_bar(stage), kABytes);
+                    tma_load_2d(sB + (lane - 1) * kABytes, lane == 1 ? &maps.b0 : &maps.b1, full_bar(stage), kx,
+                                t.q * p.I + t.n0);
                 } else {
-                    if (lane == 0)
-                        tma_load_2d(sA, &maps.dout_rows, full_bar(stage), kx, off + t.m0);
-                    else
-                        tma_load_2d(sB + (lane - 1) * kMnBlockBytes, &maps.down, full_bar(stage), t.n0 + (lane - 1) * 64,
-                                    t.q * p.H + kx);
+                    mbar_expect_tx(full_bar(stage), (uint32_t)(half * kMnBlockBytes));
+                    for (int b = (lane - 1) * half; b < lane * half; ++b)
+                        tma_load_2d(sB + b * kMnBlockBytes, &maps.b0, full_bar(stage), t.n0 + b * 64, t.q * p.H + kx);
                 }
                 filled |= 1u << stage;
                 last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
-                if (++stage == kDzguStages) { stage = 0; phase ^= 1u; }
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
             }
             if (!ok) break;
         }
-        drain_stages(bar0, kDzguStages, filled, last_parity);
+        drain_stages(bar0, kStages, filled, last_parity);
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------ MMA issuer
-        // TMEM columns: G [0, 128), U [128, 256) (one N = 256 MMA over gate and
-        // up rows), Z [256, 384); one accumulator set
+        // gate/up: one N = 256 MMA over the gate and up rows, G in accumulator
+        // columns [0, 128) and U in [128, 256); Z: N = bn, W_down MN-major.
         int stage = 0, it = 0;
         uint32_t phase = 0;
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x, ++it) {
-            if (!mbar_wait(tempty_bar, ((uint32_t)it & 1u) ^ 1u, &s_abort, p.status)) break;
+            const int buf = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            if (!mbar_wait(tempty_bar(buf), use ^ 1u, &s_abort, p.status)) break;
             tc_fence_after();
+            const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kAccCols);
             bool ok = true;
-            for (int kb = 0; kb < 2 * nkh; ++kb) {
+            for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
                 const uint64_t ad = sw128_desc(sA);
-                if (kb < nkh) {
-                    const uint64_t bd = sw128_desc(sB);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) tc_mma(tmem_base, ad + 2 * k, bd + 2 * k, p.idesc_gu, (kb | k) != 0);
-                } else {
-#pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)  // 16 K rows of the MN-major operand: 2048 bytes
-                        tc_mma(tmem_base + 256, ad + 2 * k, mn_sw128_desc(sB + k * 2048, kMnBlockBytes), p.idesc_z,
-                               ((kb - nkh) | k) != 0);
+                for (int k = 0; k < BK / 16; ++k) {
+                    // K-major: +32 bytes of K per step inside the swizzle row;
+                    // MN-major: 16 K rows = 2048 bytes per step
+                    const uint64_t bd = kMode == kRowsGU ? sw128_desc(sB) + 2 * k
+                                                         : mn_sw128_desc(sB + k * 2048, kMnBlockBytes);
+                    tc_mma(d_tmem, ad + 2 * k, bd, p.idesc, (kb | k) != 0);
                 }
                 tc_commit(empty_bar(stage));
-                if (++stage == kDzguStages) { stage = 0; phase ^= 1u; }
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
             }
             if (!ok) break;
-            tc_commit(tfull_bar);
+            tc_commit(tfull_bar(buf));
         }
         tc_commit(done_bar);
         const unsigned long long t0 = globaltimer_ns();
@@ -298,71 +309,80 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_dzgu_tc_kernel(const DzguPara
     } else if (warp >= 2) {
         // ------------------------------------------------ epilogue
         const int quarter = warp & 3;
-        const uint32_t out_base =
-            sbase + kDzguStages * kStageBytes + (uint32_t)((warp - 2) * kDzguOutBufs * kOutBf16Bytes);
-        int ob = 0, it = 0;
-        auto put = [&](const uint32_t *pk, const CUtensorMap *map, int x, int y) {
-            const uint32_t sbuf = out_base + (uint32_t)(ob * kOutBf16Bytes);
-            if (lane == 0) bulk_wait_read<kDzguOutBufs - 1>();  // the store that used this buffer has read it
-            __syncwarp();
-            store_bf16_block(sbuf, lane, pk);
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                tma_store_2d(map, sbuf, x, y);
-                bulk_commit();
-            }
-            ob = (ob + 1) % kDzguOutBufs;
-        };
+        OutStager out{sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * kOutBufs * kOutBoxBytes), 0};
+        int it = 0;
         for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
-            const DzguTile t = decode_dzgu(gt, p.E_priv, nt, tile);
+            const RowsTile t = decode_rows(gt, p.E_priv, nt, p.bn, tile);
+            const int buf = it & 1;
+            const uint32_t use = (uint32_t)(it >> 1) & 1u;
             int ok = 1;
-            if (lane == 0) ok = mbar_wait(tfull_bar, (uint32_t)it & 1u, &s_abort, p.status) ? 1 : 0;
+            if (lane == 0) ok = mbar_wait(tfull_bar(buf), use, &s_abort, p.status) ? 1 : 0;
             ok = __shfl_sync(~0u, ok, 0);
             if (!ok) break;
             __syncwarp();
             tc_fence_after();
             const int r = quarter * 32 + lane;
             const bool valid = r < t.rows;
-            const int prow = gt.off[t.q] + t.m0 + r;  // private row (relative to the first private slot)
-            const float w = valid ? p.w_of_slot[p0 + prow] : 0.f;
-            const int orow = gt.pad[t.q] + t.m0 + quarter * 32;
-            const uint32_t tb = tmem_base + ((uint32_t)(quarter * 32) << 16);
-            float gw = 0.f;
+            const int orow = gt.pad[t.q] + t.m0 + quarter * 32;  // this warp's 32 rows in the padded layout
+            const uint32_t tb = tmem_base + (uint32_t)(buf * kAccCols) + ((uint32_t)(quarter * 32) << 16);
+            if (kMode == kRowsZ) {
 #pragma unroll 1
-            for (int c = 0; c < 4; ++c) {
-                float g[32], u[32], z[32];
-                tmem_ld32(tb + c * 32, g);
-                tmem_ld32(tb + 128 + c * 32, u);
-                tmem_ld32(tb + 256 + c * 32, z);
-                tmem_ld_wait();
-                uint32_t pg[16], pu[16], pa[16];
+                for (int c = 0; c < p.bn / 32; ++c) {
+                    float v[32];
+                    tmem_ld32(tb + c * 32, v);
+                    tmem_ld_wait();
+                    uint32_t pk[16];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    float dg[2], du[2], wa[2];
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const int j = 2 * i + h;
-                        const float a = __bfloat162float(__float2bfloat16_rn(silu_mul(g[j], u[j])));
-                        gw += z[j] * a;
-                        const float sg = 1.f / (1.f + __expf(-g[j]));
-                        const float wz = w * z[j];
-                        dg[h] = valid ? wz * u[j] * sg * (1.f + g[j] * (1.f - sg)) : 0.f;
-                        du[h] = valid ? wz * g[j] * sg : 0.f;
-                        wa[h] = valid ? w * a : 0.f;
-                    }
-                    pg[i] = pack_bf16x2(dg[0], dg[1]);
-                    pu[i] = pack_bf16x2(du[0], du[1]);
-                    pa[i] = pack_bf16x2(wa[0], wa[1]);
+                    for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+                    out.put(lane, pk, &maps.out0, t.n0 + c * 32, orow);
                 }
-                put(pg, &maps.dgu, t.n0 + c * 32, orow);
-                put(pu, &maps.dgu, p.I + t.n0 + c * 32, orow);
-                put(pa, &maps.wact, t.n0 + c * 32, orow);
+            } else {
+                const int prow = gt.off[t.q] + t.m0 + r;  // private row (relative to the first private slot)
+                const float w = valid ? p.w_of_slot[p0 + prow] : 0.f;
+                const uint4 *zrow = reinterpret_cast<const uint4 *>(p.zpad + (size_t)(orow + lane) * p.I + t.n0);
+                float gw = 0.f;
+#pragma unroll 1
+                for (int c = 0; c < 4; ++c) {
+                    uint4 zq[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) zq[i] = valid ? zrow[c * 4 + i] : make_uint4(0u, 0u, 0u, 0u);
+                    float g[32], u[32];
+                    tmem_ld32(tb + c * 32, g);
+                    tmem_ld32(tb + 128 + c * 32, u);
+                    tmem_ld_wait();
+                    const __nv_bfloat162 *zb = reinterpret_cast<const __nv_bfloat162 *>(zq);
+                    uint32_t pg[16], pu[16], pa[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const float2 z2 = __bfloat1622float2(zb[i]);
+                        float dg[2], du[2], wa[2];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const int j = 2 * i + h;
+                            const float z = h ? z2.y : z2.x;
+                            const float den = 1.f + __expf(-g[j]);
+                            const float silu = __fdividef(g[j], den);  // the forward's silu(g) u, same arithmetic
+                            const float a = __bfloat162float(__float2bfloat16_rn(silu * u[j]));
+                            const float sg = __fdividef(1.f, den);
+                            gw += z * a;
+                            const float wz = w * z;
+                            dg[h] = valid ? wz * u[j] * sg * (1.f + g[j] * (1.f - sg)) : 0.f;
+                            du[h] = valid ? wz * silu : 0.f;
+                            wa[h] = valid ? w * a : 0.f;
+                        }
+                        pg[i] = pack_bf16x2(dg[0], dg[1]);
+                        pu[i] = pack_bf16x2(du[0], du[1]);
+                        pa[i] = pack_bf16x2(wa[0], wa[1]);
+                    }
+                    out.put(lane, pg, &maps.out0, t.n0 + c * 32, orow);
+                    out.put(lane, pu, &maps.out0, p.I + t.n0 + c * 32, orow);
+                    out.put(lane, pa, &maps.out1, t.n0 + c * 32, orow);
+                }
+                if (valid) p.gw_part[(size_t)prow * nt + t.n_tile] = gw;
             }
-            if (valid) p.gw_part[(size_t)prow * nt + t.n_tile] = gw;
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(tempty_bar);
+            if (lane == 0) mbar_arrive(tempty_bar(buf));
         }
         if (lane == 0) bulk_wait_all();
     }
@@ -391,7 +411,7 @@ struct WgMaps {
     CUtensorMap a_perm;     // [R][H], 64 x 64 box (MN-major B)
     CUtensorMap dout_rows;  // [R + 64][H], 64 x 64 box (MN-major A)
     CUtensorMap wact;       // [padded rows][I], 64 x 64 box (MN-major B)
-    CUtensorMap d_gate, d_up, d_down;  // FP32 outputs, 32 x 32 boxes, 128-byte swizzle
+    CUtensorMap d_gate, d_up, d_down;  // FP32 outputs, 16 x 32 boxes, 64-byte swizzle
 };
 
 struct WgTile {
@@ -428,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
 {
     extern __shared__ uint8_t dsmem[];
     __shared__ GroupTable gt;
-    __shared__ __align__(8) uint64_t bars[2 * kWgStages + 5];
+    __shared__ __align__(8) uint64_t bars[2 * kStages + 5];
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
 
@@ -436,13 +456,13 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
     const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
-    auto empty_bar = [&](int s) { return bar0 + 8u * (kWgStages + s); };
-    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kWgStages + b); };
-    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kWgStages + 2 + b); };
-    const uint32_t done_bar = bar0 + 8u * (2 * kWgStages + 4);
+    auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+    auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
+    auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
+    const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
 
     if (tid == 0) {
-        for (int s = 0; s < kWgStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
+        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
         for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
         mbar_init(done_bar, 1);
         s_abort = 0;
@@ -486,11 +506,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
                 }
                 filled |= 1u << stage;
                 last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
-                if (++stage == kWgStages) { stage = 0; phase ^= 1u; }
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
             }
             if (!ok) break;
         }
-        drain_stages(bar0, kWgStages, filled, last_parity);
+        drain_stages(bar0, kStages, filled, last_parity);
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------ MMA issuer
         // two 128 x 256 FP32 accumulators: the epilogue of one tile overlaps the
@@ -516,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
                     tc_mma(d_tmem, mn_sw128_desc(sA + k * 2048, kMnBlockBytes), mn_sw128_desc(sB + k * 2048, kMnBlockBytes),
                            idesc, (kb | k) != 0);
                 tc_commit(empty_bar(stage));
-                if (++stage == kWgStages) { stage = 0; phase ^= 1u; }
+                if (++stage == kStages) { stage = 0; phase ^= 1u; }
             }
             if (!ok) break;
             tc_commit(tfull_bar(buf));
@@ -528,8 +548,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
     } else if (warp >= 2) {
         // ------------------------------------------------ epilogue
         const int quarter = warp & 3;
-        const uint32_t out_base = sbase + kWgStages * kStageBytes + (uint32_t)((warp - 2) * kWgOutBufs * kOutF32Bytes);
-        int ob = 0, it = 0;
+        OutStager out{sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * kOutBufs * kOutBoxBytes), 0};
+        int it = 0;
         for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
             const WgTile t = decode_wg(p, gt, tile);
             const int buf = it & 1;
@@ -561,17 +581,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = 0.f;
                 }
-                const uint32_t sbuf = out_base + (uint32_t)(ob * kOutF32Bytes);
-                if (lane == 0) bulk_wait_read<kWgOutBufs - 1>();
-                __syncwarp();
-                store_f32_block(sbuf, lane, v);
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    tma_store_2d(omap, sbuf, t.n0 + c * 32, orow);
-                    bulk_commit();
-                }
-                ob = (ob + 1) % kWgOutBufs;
+                out.put(lane, reinterpret_cast<const uint32_t *>(v), omap, t.n0 + c * 32, orow);
+                out.put(lane, reinterpret_cast<const uint32_t *>(v + 16), omap, t.n0 + c * 32 + 16, orow);
             }
             tc_fence_before();
             __syncwarp();
@@ -594,33 +605,48 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
 // Rows of the padded layout (an upper bound over all routings).
 size_t backward_padded_rows(const Shape &s) { return (size_t)s.T * s.k + (size_t)kPad * s.E_priv; }
 
-cudaError_t launch_backward_dzgu(const Ctx &c, const bf16 *dout_rows, bf16 *dgu, bf16 *wact, float *gw_part)
+cudaError_t launch_backward_rows(const Ctx &c, const bf16 *dout_rows, bf16 *zpad, bf16 *dgu, bf16 *wact,
+                                 float *gw_part)
 {
     const Shape &s = c.s;
     const uint64_t R = (uint64_t)s.T * s.k, RP = backward_padded_rows(s);
-    DzguParams p;
-    DzguMaps maps;
-    memset(&p, 0, sizeof(p));
-    memset(&maps, 0, sizeof(maps));
-    p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.H = s.H; p.I = s.I; p.R = (int)R;
-    p.offsets = c.offsets;
-    p.w_of_slot = c.w_of_slot;
-    p.gw_part = gw_part;
-    p.status = c.audit.status;
-    p.idesc_gu = make_idesc(BM, 256);
-    p.idesc_z = make_idesc_major(BM, 128, false, true);
-    bool ok = encode_2d(&maps.a_perm, c.a_perm, s.H, R, BM);
-    ok &= encode_2d(&maps.dout_rows, dout_rows, s.H, R + 64, BM);
-    ok &= encode_2d(&maps.gate, c.gate[1], s.H, (uint64_t)s.E_priv * s.I, 128);
-    ok &= encode_2d(&maps.up, c.up[1], s.H, (uint64_t)s.E_priv * s.I, 128);
-    ok &= encode_2d_box(&maps.down, c.down[1], s.I, (uint64_t)s.E_priv * s.H, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
-    ok &= encode_2d_box(&maps.dgu, dgu, 2 * (uint64_t)s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
-    ok &= encode_2d_box(&maps.wact, wact, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
-    if (!ok) return cudaErrorInvalidValue;
-    static std::atomic<int> smem_limit[64];
-    cudaError_t err = ensure_dynamic_smem(bwd_dzgu_tc_kernel, kDzguDynSmem, smem_limit);
-    if (err != cudaSuccess) return err;
-    return launch_pdl(bwd_dzgu_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDzguDynSmem, c.stream, p, maps);
+    static std::atomic<int> smem_limit[2][64];
+    cudaError_t err;
+    for (int mode = 0; mode < 2; ++mode) {
+        RowsParams p;
+        RowsMaps maps;
+        memset(&p, 0, sizeof(p));
+        memset(&maps, 0, sizeof(maps));
+        p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.H = s.H; p.I = s.I; p.R = (int)R;
+        p.offsets = c.offsets;
+        p.w_of_slot = c.w_of_slot;
+        p.zpad = zpad;
+        p.gw_part = gw_part;
+        p.status = c.audit.status;
+        bool ok;
+        if (mode == kRowsZ) {
+            p.bn = s.I % 256 == 0 ? 256 : 128;
+            p.idesc = make_idesc_major(BM, p.bn, false, true);
+            ok = encode_2d(&maps.a, dout_rows, s.H, R + 64, BM);
+            ok &= encode_2d_box(&maps.b0, c.down[1], s.I, (uint64_t)s.E_priv * s.H, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
+            ok &= encode_2d_box(&maps.out0, zpad, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+        } else {
+            p.bn = 128;
+            p.idesc = make_idesc(BM, 256);
+            ok = encode_2d(&maps.a, c.a_perm, s.H, R, BM);
+            ok &= encode_2d(&maps.b0, c.gate[1], s.H, (uint64_t)s.E_priv * s.I, 128);
+            ok &= encode_2d(&maps.b1, c.up[1], s.H, (uint64_t)s.E_priv * s.I, 128);
+            ok &= encode_2d_box(&maps.out0, dgu, 2 * (uint64_t)s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+            ok &= encode_2d_box(&maps.out1, wact, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+        }
+        if (!ok) return cudaErrorInvalidValue;
+        auto kernel = mode == kRowsZ ? bwd_rows_tc_kernel<kRowsZ> : bwd_rows_tc_kernel<kRowsGU>;
+        err = ensure_dynamic_smem(kernel, kDynSmem, smem_limit[mode]);
+        if (err != cudaSuccess) return err;
+        err = launch_pdl(kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
+        if (err != cudaSuccess) return err;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
@@ -644,14 +670,15 @@ cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf1
     ok &= encode_2d_box(&maps.a_perm, c.a_perm, s.H, R, 64, 64, sw);
     ok &= encode_2d_box(&maps.dout_rows, dout_rows, s.H, R + 64, 64, 64, sw);
     ok &= encode_2d_box(&maps.wact, wact, s.I, RP, 64, 64, sw);
-    ok &= encode_2d_f32(&maps.d_gate, d_gate, s.H, (uint64_t)s.E_priv * s.I, 32, 32, sw);
-    ok &= encode_2d_f32(&maps.d_up, d_up, s.H, (uint64_t)s.E_priv * s.I, 32, 32, sw);
-    ok &= encode_2d_f32(&maps.d_down, d_down, s.I, (uint64_t)s.E_priv * s.H, 32, 32, sw);
+    const CUtensorMapSwizzle osw = CU_TENSOR_MAP_SWIZZLE_64B;
+    ok &= encode_2d_f32(&maps.d_gate, d_gate, s.H, (uint64_t)s.E_priv * s.I, 16, 32, osw);
+    ok &= encode_2d_f32(&maps.d_up, d_up, s.H, (uint64_t)s.E_priv * s.I, 16, 32, osw);
+    ok &= encode_2d_f32(&maps.d_down, d_down, s.I, (uint64_t)s.E_priv * s.H, 16, 32, osw);
     if (!ok) return cudaErrorInvalidValue;
     static std::atomic<int> smem_limit[64];
-    cudaError_t err = ensure_dynamic_smem(bwd_wgrad_tc_kernel, kWgDynSmem, smem_limit);
+    cudaError_t err = ensure_dynamic_smem(bwd_wgrad_tc_kernel, kDynSmem, smem_limit);
     if (err != cudaSuccess) return err;
-    return launch_pdl(bwd_wgrad_tc_kernel, dim3(c.num_sms), dim3(kThreads), kWgDynSmem, c.stream, p, maps);
+    return launch_pdl(bwd_wgrad_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
 }
 
 }  // namespace pmpe

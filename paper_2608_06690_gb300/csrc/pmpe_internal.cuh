@@ -80,9 +80,10 @@ size_t backward_workspace_bytes(const Shape &s);
 cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_router, float *d_gate, float *d_up,
                                     float *d_down, uint8_t *bws);
 // Its tensor-core GEMMs (k_backward_tc.cu): rows of the padded layout, the
-// recompute + dL/da launch and the weight-gradient launch.
+// dL/da and gate/up recompute launches, and the weight-gradient launch.
 size_t backward_padded_rows(const Shape &s);
-cudaError_t launch_backward_dzgu(const Ctx &c, const bf16 *dout_rows, bf16 *dgu, bf16 *wact, float *gw_part);
+cudaError_t launch_backward_rows(const Ctx &c, const bf16 *dout_rows, bf16 *zpad, bf16 *dgu, bf16 *wact,
+                                 float *gw_part);
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
                                   float *d_gate, float *d_up, float *d_down);
 // Gate/up and down in one persistent launch (down tiles wait for their

@@ -45,10 +45,11 @@ STAGE_ALL = 0x1F
 # dispatch + row gather, gate/up GEMM, down GEMM, combine (plus one memset of
 # the per-expert counters, which is not a kernel of this library).
 KERNELS_PER_FORWARD = 4
-# kernels one private-branch backward launches: dout row gather, the fused
-# dL/da + gate/up recompute GEMM, router gradient, router weight-gradient
-# partials and their reduction, the expert weight-gradient GEMM
-KERNELS_PER_BACKWARD = 6
+# kernels one private-branch backward launches: dout row gather, the dL/da
+# GEMM, the gate/up recompute GEMM with the SwiGLU backward, router gradient,
+# router weight-gradient partials and their reduction, the expert
+# weight-gradient GEMM
+KERNELS_PER_BACKWARD = 7
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
