@@ -140,7 +140,8 @@ typedef struct pmpe_workspace_layout {
     size_t topk_idx;     /* int32  [T, k]   used when desc.topk_idx is NULL */
     size_t topk_w;       /* float  [T, k]   used when desc.topk_w is NULL */
     size_t slot_of;      /* int32  [T, k]   dispatch row of (t, j) */
-    size_t ticket;       /* int32  [T, k]   position of (t, j) among its expert's rows */
+    size_t ticket;       /* int32  [T, k]   128 * (router tile of t) + position of (t, j) among the
+                          * tile's rows of its expert (the tile's tokens in ascending order) */
     size_t tok_of_slot;  /* int32  [T*k]    token of each dispatch row */
     size_t w_of_slot;    /* float  [T*k]    routing weight of each dispatch row */
     size_t router_rows;  /* BF16   [C*128, H]  token rows of each router CTA whose tile is not consecutive */
@@ -154,6 +155,10 @@ typedef struct pmpe_workspace_layout {
     size_t router_meta;  /* float4 [C2*128] per chunk: max score, sum exp(score - max), entries */
     size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1]  gate/up epilogue warps done per
                           * (expert group, 128-row block), read by the down tiles of the same launch */
+    size_t tile_counts;  /* uint32 [E, S4]  rows of expert e in router tile s (S4 = S rounded up to 4).
+                          * With the tiles of a pool in ascending token order, slot
+                          * offsets[e] + sum_{s' < s} tile_counts[e, s'] + position gives every expert
+                          * its rows in ascending (t, j) order: the dispatch order is deterministic */
 } pmpe_workspace_layout;
 PMPE_API int pmpe_moe_workspace_layout(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k,
                               pmpe_workspace_layout *out);

@@ -425,10 +425,14 @@ int oracle_backward_private(const oracle_layer *L, const double *dout, double *d
     char *taken = (char *)malloc(E);
     int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * k);
     for (int t = 0; t < L->T; ++t) {
+        const double *dt = dout + (size_t)t * H;
+        /* every gradient term is linear in dout_t: a zero row contributes exactly zero */
+        int nonzero = 0;
+        for (int o = 0; o < H && !nonzero; ++o) nonzero = dt[o] != 0.0;
+        if (!nonzero) continue;
         double gap;
         route_token(L, t, idx, w, &gap, s, taken);
         const uint16_t *hr = L->hidden + (size_t)t * H;
-        const double *dt = dout + (size_t)t * H;
         for (int c = 0; c < H; ++c) h[c] = bf16_value(hr[c]);
         for (int j = 0; j < k; ++j) {
             const int e = idx[j];

@@ -3,12 +3,13 @@
 //
 // Dispatch (the grouping any grouped expert execution needs): the routed rows
 // are grouped by expert id -- expert e owns slots [offset[e], offset[e+1]) --
-// and, inside an expert, placed by the ticket the router took with an integer
-// atomic, so the order inside an expert depends on timing.  The layer's output
-// does not: every expert GEMM row depends only on its own input row, and the
-// combine sums each token's rows in rank order.  The same pass copies each
-// token row into its slot with 16-byte vector loads.  An id outside [0, E) is
-// recorded in the status word.
+// and, inside an expert, ordered by token: the router's ticket names the
+// row's 128-token tile and its position among that tile's rows of the expert,
+// and the rows of the earlier tiles (tile_counts) come first.  The tiles of a
+// pool run in ascending token order, so every run gives the same order: the
+// stable (t, j) order.  The same pass copies each token row into its slot
+// with 16-byte vector loads.  An id outside [0, E) is recorded in the status
+// word.
 //
 // Combine: out_t = bf16( sum_{j < k} y[slot(t, j)] + y_shared[t] ), summed in
 // FP32 in a fixed order (j ascending, then shared), so the result of a token
@@ -27,6 +28,8 @@ struct DispatchParams {
     const int32_t *ticket;
     const float *w;
     const uint32_t *counts;
+    const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
+    int slots4;
     const bf16 *hidden;
     int T, H, R, k, E;
     int groups;  // warps per token: each stores the row to a share of its k slots
@@ -37,10 +40,48 @@ struct DispatchParams {
     uint32_t *status;
 };
 
+// Slot of routed row (t, j): offset[e] + the rows of expert e in the router
+// tiles before the row's tile + its position in that tile (ticket = 128 *
+// tile + position).  The tile counts are read 4 x 16 bytes at a time, all in
+// flight together.  Records the row in slot_of, tok_of_slot and w_of_slot and
+// returns the slot (-1 for an id outside [0, E) or a slot outside [0, R)).
+__device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, int t, int j)
+{
+    const int r = t * p.k + j;
+    const int e = p.idx[r];
+    if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
+        if (p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+        return -1;
+    }
+    const int tk = p.ticket[r];
+    const int ts = min(tk >> 7, p.slots4);
+    const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
+    const uint4 *tc4 = reinterpret_cast<const uint4 *>(tc);
+    uint32_t before = 0;
+    const int full = ts >> 2;
+    for (int g0 = 0; g0 < full; g0 += 4) {
+        uint4 x[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (g0 + u < full) x[u] = __ldg(tc4 + g0 + u);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (g0 + u < full) before += x[u].x + x[u].y + x[u].z + x[u].w;
+    }
+    for (int s2 = full << 2; s2 < ts; ++s2) before += __ldg(tc + s2);
+    const int slot = (int)(s_off[e] + before) + (tk & 127);
+    if ((unsigned)slot >= (unsigned)p.R) return -1;  // only a corrupt ticket could fail this
+    p.slot_of[r] = slot;
+    p.tok_of_slot[slot] = t;
+    p.w_of_slot[slot] = p.w[r];
+    return slot;
+}
+
 // Dispatch and gather in one pass.  Every CTA forms the experts' offsets
 // (exclusive prefix sum of the router's per-expert counts) in shared memory;
-// routed row r = (t, j) of expert e goes to slot offset[e] + ticket[r].  One
-// warp per token loads the token's row once and stores it to its k slots.
+// routed row r = (t, j) of expert e, in tile s at position q of the tile's
+// rows of e, goes to slot offset[e] + sum_{s' < s} tile_counts[e][s'] + q.
+// One warp per token loads the token's row once and stores it to its k slots.
 __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const DispatchParams p)
 {
     __shared__ uint32_t s_off[2 * kMaxPool + 1];
@@ -75,23 +116,8 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
     for (int wi = blockIdx.x * (kDispThreads / 32) + (threadIdx.x >> 5); wi < p.T * p.groups; wi += warps) {
         const int t = wi / p.groups, gj = wi - t * p.groups;
         const int j0 = gj * per, j1 = min(p.k, j0 + per);
-        int my_slot = -1;
-        if (lane >= j0 && lane < j1) {
-            const int r = t * p.k + lane;
-            const int e = p.idx[r];
-            if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
-                if (p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
-            } else {
-                const int slot = (int)s_off[e] + p.ticket[r];
-                if ((unsigned)slot < (unsigned)p.R) {  // only a corrupt ticket could fail this
-                    my_slot = slot;
-                    p.slot_of[r] = slot;
-                    p.tok_of_slot[slot] = t;
-                    p.w_of_slot[slot] = p.w[r];
-                }
-            }
-        }
         const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
+        int my_slot = -1;
         for (int c0 = 0; c0 < nv; c0 += 32 * 8) {
             uint4 v[8];
 #pragma unroll
@@ -99,6 +125,8 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
                 const int c = c0 + u * 32 + lane;
                 if (c < nv) v[u] = __ldg(src + c);
             }
+            // the slots are resolved while the row's loads are in flight
+            if (c0 == 0 && lane >= j0 && lane < j1) my_slot = resolve_slot(p, s_off, t, lane);
             for (int j = j0; j < j1; ++j) {
                 const int slot = __shfl_sync(~0u, my_slot, j);
                 if (slot < 0) continue;
@@ -186,6 +214,8 @@ cudaError_t launch_permute(const Ctx &c)
     const int R = s.T * s.k;
     DispatchParams p;
     p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts; p.hidden = c.hidden;
+    p.tile_counts = c.tile_counts;
+    p.slots4 = router_slots4(c.s.T);
     p.T = s.T; p.H = s.H; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.a_perm = c.a_perm;

@@ -19,8 +19,10 @@
 // first k with the chunk's softmax partial to the workspace.  The CTA that
 // completes a tile last (an integer atomic per tile, after a memory fence)
 // merges the chunk lists in chunk order, writes the softmax weights and the
-// route log, and hands out the rows' positions inside their experts: one
-// shared-memory atomic per row and one global atomic per expert and tile.
+// route log, and ranks each row among the tile's rows of its expert by token
+// order (a 128-bit token mask per expert: the rank is a popcount), so that
+// the dispatch order is deterministic; it records the tile's per-expert
+// counts in its column of tile_counts.
 #include <cuda.h>
 
 #include "pmpe_internal.cuh"
@@ -56,7 +58,9 @@ struct RouterParams {
     int32_t *idx;
     float *w;
     uint32_t *counts;    // per-expert row counters (zeroed before the launch)
-    int32_t *ticket;     // [T, k] row position inside its expert
+    uint32_t *tile_counts;  // [E][slots4] rows of each expert per tile (a column per tile slot)
+    int slots4;
+    int32_t *ticket;     // [T, k] 128 * tile slot + position among the tile's rows of its expert
     uint32_t *route_count, *route_priv_rows, *status;
 };
 
@@ -94,6 +98,37 @@ __device__ __forceinline__ int block_scan(int v, int *warp_tot, int &total)
 __device__ __forceinline__ bool is_allow(const uint8_t *policy, int t)
 {
     return policy != nullptr && policy[t] == 0x01;
+}
+
+// Bytes of policy[t0, t1) equal to the trusted ALLOW value 0x01.  Whole
+// 16-byte groups inside the range are read with vector loads when the
+// pointer allows it (the caller's runs start at multiples of 16); any other
+// byte is read on its own.  Nothing outside [t0, t1) is read.
+__device__ __forceinline__ int count_allow(const uint8_t *policy, int t0, int t1)
+{
+    if (policy == nullptr || t0 >= t1) return 0;
+    int n = 0, t = t0;
+    if ((((uintptr_t)(policy + t0)) & 15u) == 0) {
+        const uint4 *v = reinterpret_cast<const uint4 *>(policy + t0);
+        const int groups = (t1 - t0) >> 4;
+        constexpr int kBatch = 4;  // independent 16-byte loads in flight
+        for (int g0 = 0; g0 < groups; g0 += kBatch) {
+            uint4 x[kBatch];
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u)
+                if (g0 + u < groups) x[u] = __ldg(v + g0 + u);
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u)
+                if (g0 + u < groups) {
+                    // __vcmpeq4 sets each equal byte to 0xff: eight set bits per ALLOW byte
+                    n += (__popc(__vcmpeq4(x[u].x, 0x01010101u)) + __popc(__vcmpeq4(x[u].y, 0x01010101u)) +
+                          __popc(__vcmpeq4(x[u].z, 0x01010101u)) + __popc(__vcmpeq4(x[u].w, 0x01010101u))) >> 3;
+                }
+        }
+        t = t0 + (groups << 4);
+    }
+    for (; t < t1; ++t) n += policy[t] == 0x01;
+    return n;
 }
 
 // (x, e) ranks above (bx, be): larger logit, or equal logit and lower id.
@@ -187,13 +222,12 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
 
     // ---- resolve and rank in one pass: each thread takes a contiguous run of
-    // tokens; the scan of its ALLOW count gives the pool sizes and its ranks
-    const int per = (p.T + kRThreads - 1) / kRThreads;
+    // tokens (a multiple of 16 long, so that runs start 16-byte aligned); the
+    // scan of its ALLOW count gives the pool sizes and its ranks
+    const int per = ((p.T + kRThreads - 1) / kRThreads + 15) & ~15;
     const int t0 = min(p.T, tid * per), t1 = min(p.T, t0 + per);
     // the unmasked control tiles all tokens as one pool, in token order
-    int a = 0;
-    if (!p.unmasked)
-        for (int t = t0; t < t1; ++t) a += is_allow(p.policy, t);
+    const int a = p.unmasked ? 0 : count_allow(p.policy, t0, t1);
     int na;
     const int a_before = block_scan(a, warp_tot, na);
     const int nd = p.T - na;
@@ -208,7 +242,9 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         if (m0 >= na) return;  // uniform: no tile for this slot
     }
     const int rows = min(kTileRows, (pool ? na : nd) - m0);
-    {
+    // only a thread whose ranks in the tile's pool overlap the tile walks its run
+    if ((pool ? a_before : t0 - a_before) < m0 + rows &&
+        (pool ? a_before + a : t1 - a_before - a) > m0) {
         int ra = a_before, rd = t0 - a_before;  // ranks inside the ALLOW / DENY pools
         for (int t = t0; t < t1; ++t) {
             const bool al_byte = is_allow(p.policy, t);
@@ -346,10 +382,9 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
         // (the ring is idle: all loads were consumed by the MMAs):
         float *sv = reinterpret_cast<float *>(dsmem + (sbase - smem_u32(dsmem)));  // [nl][128][K] scores
         uint16_t *se = reinterpret_cast<uint16_t *>(sv + nl * kTileRows * K);      // [nl][128][K] ids
-        uint16_t *sloc = se + nl * kTileRows * K;                                   // [128][K] rank in expert
-        uint32_t *scnt = reinterpret_cast<uint32_t *>(sloc + ((kTileRows * K + 1) & ~1));  // [P]
-        uint32_t *sbas = scnt + 2 * kMaxPool;                                       // [P]
-        float4 *smeta = reinterpret_cast<float4 *>(sbas + 2 * kMaxPool);           // [nl][128]
+        uint32_t *smask = reinterpret_cast<uint32_t *>(se + ((nl * kTileRows * K + 1) & ~1));  // [P][4] token bits
+        uint32_t *scum = smask + 4 * 2 * kMaxPool;                                  // [P] tokens before words 1-3
+        float4 *smeta = reinterpret_cast<float4 *>(scum + 2 * kMaxPool);           // [nl][128]
         if (ok) {
             __syncwarp();
             tc_fence_after();
@@ -440,7 +475,7 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
                 for (int u = 0; u < kMaxChunks; ++u)
                     if (u < nl) smeta[u * kTileRows + et] = m[u];
             }
-            for (int i = et; i < P; i += kEpi) scnt[i] = 0u;
+            for (int i = et; i < 4 * P; i += kEpi) smask[i] = 0u;
             asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
             // merge the chunk lists of token r in chunk order
             const bool valid = et < rows;
@@ -474,7 +509,7 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
                     sel_e[j] = be;
                     if (j == 0) top = bv;
                     npriv += base + be >= p.E_pub;
-                    sloc[et * K + j] = (uint16_t)atomicAdd(&scnt[be], 1u);
+                    atomicOr(&smask[be * 4 + (et >> 5)], 1u << (et & 31));
                 }
                 if (p.renorm) {
                     for (int j = 0; j < K; ++j) S += expf(sel_v[j] - top);
@@ -486,21 +521,32 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
                 }
             }
             asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
-            // one global atomic per expert of the tile: the tile's block of rows
+            // the tile's rows per expert of the pool: its entries of tile_counts
+            // (zeroed before the launch) and one global atomic per expert for the
+            // totals; scum packs the tokens of mask words < 1, < 2, < 3 (8 bits each)
             for (int i = et; i < P; i += kEpi) {
-                const uint32_t c = scnt[i];
+                const uint32_t c0 = __popc(smask[i * 4]), c1 = __popc(smask[i * 4 + 1]);
+                const uint32_t c2 = __popc(smask[i * 4 + 2]), c3 = __popc(smask[i * 4 + 3]);
+                scum[i] = c0 | ((c0 + c1) << 8) | ((c0 + c1 + c2) << 16);
+                const uint32_t c = c0 + c1 + c2 + c3;
                 if (c) {
-                    sbas[i] = atomicAdd(&p.counts[base + i], c);
+                    p.tile_counts[(size_t)(base + i) * p.slots4 + slot] = c;
+                    atomicAdd(&p.counts[base + i], c);
                     if (p.route_count) atomicAdd(&p.route_count[base + i], c);
                 }
             }
             asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
             if (valid) {
                 const int t = s_tok[et];
+                const int wd = et >> 5;
+                const uint32_t below = (1u << (et & 31)) - 1u;
                 for (int j = 0; j < K; ++j) {
                     const int be = sel_e[j];
+                    // rank among the tile's rows of expert be: its tokens before t
+                    const int rank = (int)__popc(smask[be * 4 + wd] & below) +
+                                     (wd ? (int)((scum[be] >> (8 * (wd - 1))) & 0xffu) : 0);
                     p.idx[(size_t)t * K + j] = base + be;
-                    p.ticket[(size_t)t * K + j] = (int32_t)(sbas[be] + sloc[et * K + j]);
+                    p.ticket[(size_t)t * K + j] = (int32_t)(slot * kTileRows + rank);
                     p.w[(size_t)t * K + j] = expf(sel_v[j] - top) / S;
                 }
                 if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], (unsigned)npriv);
@@ -558,6 +604,7 @@ __global__ void resolve_kernel(const uint8_t *policy, int T, uint8_t *tau)
 // Chunks of a pool (32 experts each) and the router's per-tile sizes.
 int router_chunks(int pool_size) { return (pool_size + kChunk - 1) / kChunk; }
 int router_slots(int T) { return (T + kTileRows - 1) / kTileRows + 1; }
+int router_slots4(int T) { return (router_slots(T) + 3) & ~3; }
 
 cudaError_t launch_route(const Ctx &c)
 {
@@ -572,17 +619,21 @@ cudaError_t launch_route(const Ctx &c)
     p.unmasked = c.unmasked;
     p.nch_max = p.unmasked ? p.nch[2] : (p.nch[0] > p.nch[1] ? p.nch[0] : p.nch[1]);
     const int slots = router_slots(s.T);
-    // per-expert counters, per-tile completion counts and the expert GEMMs'
-    // readiness counters start at zero (the workspace places them side by
-    // side: one memset clears all three)
+    // per-expert counters, per-tile completion counts, the expert GEMMs'
+    // readiness counters and the per-tile expert counts start at zero (the
+    // workspace places them side by side: one memset clears all four)
     cudaError_t merr;
     const size_t nready = gemm_ready_words(s);
-    if (c.tile_done == c.counts + s.E() && c.gemm_ready == c.tile_done + slots) {
-        merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * (s.E() + slots + nready), c.stream);
+    const size_t ntc = (size_t)s.E() * router_slots4(s.T);
+    // tile_counts starts 16-byte aligned right after gemm_ready (at most 3 words between)
+    if (c.tile_done == c.counts + s.E() && c.gemm_ready == c.tile_done + slots &&
+        c.tile_counts >= c.gemm_ready + nready && c.tile_counts <= c.gemm_ready + nready + 3) {
+        merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * (size_t)(c.tile_counts + ntc - c.counts), c.stream);
     } else {
         merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
         if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_done, 0, sizeof(uint32_t) * slots, c.stream);
         if (merr == cudaSuccess) merr = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * nready, c.stream);
+        if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_counts, 0, sizeof(uint32_t) * ntc, c.stream);
     }
     if (merr != cudaSuccess) return merr;
     p.idesc = make_idesc(kTileRows, kChunk);
@@ -597,6 +648,8 @@ cudaError_t launch_route(const Ctx &c)
     p.idx = c.idx;
     p.w = c.w;
     p.counts = c.counts;
+    p.tile_counts = c.tile_counts;
+    p.slots4 = router_slots4(s.T);
     p.ticket = c.ticket;
     p.route_count = c.audit.route_count;
     p.route_priv_rows = c.audit.route_priv_rows;
@@ -608,8 +661,8 @@ cudaError_t launch_route(const Ctx &c)
     ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, kChunk);
     if (!ok) return cudaErrorInvalidValue;
     const int ring = p.stages * kStageBytes + 1024;
-    const int merge = p.nch_max * kTileRows * s.k * 6 + kTileRows * s.k * 2 + 4 + 4 * kMaxPool * 4 +
-                      p.nch_max * kTileRows * 16 + 1024 + 16;
+    const int merge = p.nch_max * kTileRows * s.k * 6 + 4 + 5 * 2 * kMaxPool * 4 + p.nch_max * kTileRows * 16 +
+                      1024 + 16;
     const int smem = ring > merge ? ring : merge;
     static std::atomic<int> smem_limit[64];
     cudaError_t err = ensure_dynamic_smem(router_tc_kernel, smem, smem_limit);

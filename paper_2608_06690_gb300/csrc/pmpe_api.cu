@@ -43,6 +43,7 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     const size_t rctas_all = slots * (size_t)(router_chunks(s.E_pub) + router_chunks(s.E_priv));
     L->tile_done = take(4 * slots, 4);
     L->gemm_ready = take(4 * gemm_ready_words(s), 4);
+    L->tile_counts = take(4 * E * (size_t)router_slots4(s.T), 16);  // read as 16-byte vectors
     L->offsets = take(4 * (E + 1), 256);
     L->topk_idx = take(4 * R, 256);
     L->topk_w = take(4 * R, 256);
@@ -138,6 +139,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->tok_of_slot = (int32_t *)(ws + L.tok_of_slot);
     c->w_of_slot = (float *)(ws + L.w_of_slot);
     c->tile_done = (uint32_t *)(ws + L.tile_done);
+    c->tile_counts = (uint32_t *)(ws + L.tile_counts);
     c->gemm_ready = (uint32_t *)(ws + L.gemm_ready);
     c->router_lists = (float2 *)(ws + L.router_lists);
     c->router_meta = (float4 *)(ws + L.router_meta);

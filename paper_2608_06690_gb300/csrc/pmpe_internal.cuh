@@ -49,9 +49,10 @@ struct Ctx {
     uint8_t *tau;
     uint32_t *counts, *offsets;
     int32_t *slot_of, *tok_of_slot;
-    int32_t *ticket;    // [T, k] position of each routed row inside its expert
+    int32_t *ticket;    // [T, k] 128 * router tile + position among the tile's rows of its expert
     float *w_of_slot;
     uint32_t *tile_done;  // [router slots] chunk CTAs finished per router tile
+    uint32_t *tile_counts; // [E][router_slots4] rows of each expert per router tile
     uint32_t *gemm_ready; // [gemm_ready_words] gate/up warps done per (group, 128-row block)
     float2 *router_lists; // [router CTAs * 128, k] per-chunk sorted (score, id)
     float4 *router_meta;  // [router CTAs * 128] per-chunk softmax partials
@@ -66,6 +67,8 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L);
 // Router geometry: 32-expert chunks of a pool, 128-token tile slots for T tokens.
 int router_chunks(int pool_size);
 int router_slots(int T);
+// router_slots rounded up to a multiple of 4 (the row pitch of tile_counts).
+int router_slots4(int T);
 // Readiness counters of the persistent expert GEMMs: one per (group, 128-row
 // block), an upper bound over all routings.
 size_t gemm_ready_words(const Shape &s);

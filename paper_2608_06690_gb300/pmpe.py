@@ -78,7 +78,8 @@ class MoeDesc(ctypes.Structure):
 class WorkspaceLayout(ctypes.Structure):
     _fields_ = [(n, ctypes.c_size_t) for n in ("total", "tau", "counts", "offsets", "topk_idx", "topk_w", "slot_of", "ticket",
                                                 "tok_of_slot", "w_of_slot", "router_rows", "a_perm", "act", "y", "act_sh", "y_sh",
-                                                "tile_done", "router_lists", "router_meta", "gemm_ready")]
+                                                "tile_done", "router_lists", "router_meta", "gemm_ready",
+                                                "tile_counts")]
 
 
 _lib.pmpe_moe_workspace_size.restype = ctypes.c_size_t

@@ -153,15 +153,15 @@ def check_audit(shape: LayerShape, pol_cpu, gpu: dict):
 
 def check_dispatch(shape: LayerShape, h_cpu, gpu: dict):
     """The dispatch grouping against the oracle's definition applied to the
-    GPU's own route log.  The expert offsets are unique and compared bit for
-    bit; the order of rows inside an expert is not (the router hands out
-    positions with atomics), so the rest is checked for validity: each expert's
-    slots hold exactly its routed (token, rank) pairs, slot_of is a bijection
-    onto [0, T*k) that tok_of_slot inverts, and each gathered row is its
-    token's row."""
+    GPU's own route log, bit for bit: the expert offsets, and the stable slot
+    order (expert-major, then token, then rank) in slot_of and tok_of_slot;
+    plus the structure (slot_of a bijection onto [0, T*k) that tok_of_slot
+    inverts) and every gathered row equal to its token's row."""
     import oracle
     counts, offsets, slot_of_ref, tok_of_slot_ref = oracle.permute(gpu["idx"], shape.E)
     assert np.array_equal(gpu["offsets"], offsets)
+    assert np.array_equal(gpu["slot_of"], slot_of_ref), "slot_of differs from the stable dispatch order"
+    assert np.array_equal(gpu["tok_of_slot"], tok_of_slot_ref), "tok_of_slot differs from the stable dispatch order"
     T, k = gpu["idx"].shape
     so = gpu["slot_of"]
     assert np.array_equal(np.sort(so.reshape(-1)), np.arange(T * k)), "slot_of is not a bijection"

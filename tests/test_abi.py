@@ -81,7 +81,8 @@ def test_workspace_size_and_layout(pmpe):
                     router_lists=8 * ctas_all * 128 * sh.k, router_meta=16 * ctas_all * 128,
                     gemm_ready=4 * ((R + 127) // 128 + E + (T + 127) // 128 + 1),
                     router_rows=2 * ctas * 128 * sh.H, a_perm=2 * R * sh.H, act=2 * R * sh.I, y=2 * R * sh.H,
-                    act_sh=2 * T * sh.E_sh * sh.I, y_sh=2 * T * sh.H if sh.E_sh else 0)
+                    act_sh=2 * T * sh.E_sh * sh.I, y_sh=2 * T * sh.H if sh.E_sh else 0,
+                    tile_counts=4 * E * ((slots + 3) // 4 * 4))
         spans = sorted((LL[n], LL[n] + b, n) for n, b in size.items() if b)
         for (a0, a1, na), (b0, b1, nb) in zip(spans, spans[1:]):
             assert a1 <= b0, (na, nb)
@@ -89,6 +90,8 @@ def test_workspace_size_and_layout(pmpe):
         assert LL["router_meta"] % 16 == 0 and LL["router_lists"] % 8 == 0 and LL["router_rows"] % 1024 == 0
         assert LL["tile_done"] == LL["counts"] + 4 * E  # one memset clears these three
         assert LL["gemm_ready"] == LL["tile_done"] + 4 * slots
+        gr_end = LL["gemm_ready"] + 4 * ((R + 127) // 128 + E + (T + 127) // 128 + 1)
+        assert LL["tile_counts"] % 16 == 0 and gr_end <= LL["tile_counts"] <= gr_end + 12
     assert pmpe.workspace_size(LayerShape(64, 200, 128, 8, 4, 0, 2, True)) == 0    # H % 128
     assert pmpe.workspace_size(LayerShape(64, 256, 128, 8, 4, 0, 9, True)) == 0    # k > pool
 

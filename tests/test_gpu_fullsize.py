@@ -62,3 +62,51 @@ def _check_sampled(s, w_cpu, h_cpu, pol, gpu, toks):
     mx, mean = output_errors(gpu["out"][toks][ok], r["out"][ok])
     assert mx <= MAX_ABS_REL and mean <= MEAN_REL, (mx, mean)
     return dict(excused=int((~ok).sum()), max_abs_rel=mx, mean_rel=mean)
+
+
+@pytest.mark.parametrize("name", ["qwen3_prefill", "deepseek_v2_lite"])
+def test_full_size_backward_on_sampled_tokens(name):
+    """The private-branch backward at full size, launched as the benchmark
+    launches it.  dout is nonzero on sampled ALLOW and DENY tokens only, so
+    the oracle computes every gradient element exactly from those tokens
+    (every gradient term is linear in a token's dout row); all four gradients
+    are compared element by element.  G2 on all tokens: random upstream
+    gradients on every DENY token change no gradient bit."""
+    from paper_2608_06690_gb300 import pmpe
+    from pmpe_testlib import GAP_EPS, oracle_layer
+    cfg = CONFIGS[name]
+    s = cfg.shape
+    w = inp.make_weights(s, cfg.seed, device="cuda", skew=cfg.skew)
+    h = inp.make_hidden(s, cfg.seed, device="cuda", skew=cfg.skew)
+    pol = cfg.policy(s.T)
+    w_cpu = {k: (None if v is None else v.cpu()) for k, v in w.items()}
+    L = oracle_layer(s, w_cpu, h.cpu(), pol)
+    toks = _sample_tokens(cfg, per_pool=12, seed=1)
+    _, _, gap = oracle.route(L, tokens=toks)
+    keep = toks[gap >= GAP_EPS]  # a token at a routing near-tie may pick another k-th expert
+    gen = torch.Generator().manual_seed(11)
+    dout = torch.zeros((s.T, s.H), dtype=torch.bfloat16)
+    dout[torch.from_numpy(keep).long()] = torch.randn((len(keep), s.H), generator=gen).to(torch.bfloat16)
+    layer = pmpe.MoeLayer(s, w)
+    pd = pol.cuda()
+    layer.forward(h, pd)
+    g = {n: v.cpu().numpy().astype(np.float64) for n, v in layer.backward_private(h, pd, dout.cuda()).items()}
+    ref = oracle.backward_private(L, dout.double().numpy())
+    tau = oracle.resolve(pol.numpy(), s.T)
+    assert tau[keep].sum() >= 8 and (tau[keep] == 0).sum() >= 8
+    for n in ("d_router", "d_gate", "d_up", "d_down"):
+        err = np.abs(g[n] - ref[n])
+        mx = err.max() / np.abs(ref[n]).max()
+        mean = err.sum() / np.abs(ref[n]).sum()
+        assert mx <= 2e-2 and mean <= 1e-2, (n, mx, mean)
+        # the same experts receive gradients (an expert no sampled row reached gets exact zeros)
+        assert np.array_equal(np.abs(g[n]).reshape(s.E_priv, -1).max(1) == 0,
+                              np.abs(ref[n]).reshape(s.E_priv, -1).max(1) == 0), n
+    # G2 at full size: DENY rows of dout reach no private gradient
+    d2 = dout.clone()
+    deny = torch.from_numpy(tau == 0)
+    d2[deny] = torch.randn((int(deny.sum()), s.H), generator=gen).to(torch.bfloat16)
+    layer.forward(h, pd)
+    g2 = layer.backward_private(h, pd, d2.cuda())
+    for n in g:
+        assert np.array_equal(g[n], g2[n].cpu().numpy().astype(np.float64)), n
