@@ -30,6 +30,7 @@ struct DispatchParams {
     const uint32_t *counts;
     const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
     int slots4;
+    int pre_in_smem;              // 1: each CTA keeps the table's prefix in shared memory
     const bf16 *hidden;
     int T, H, R, k, E;
     int groups;  // warps per token: each stores the row to a share of its k slots
@@ -41,11 +42,13 @@ struct DispatchParams {
 };
 
 // Slot of routed row (t, j): offset[e] + the rows of expert e in the router
-// tiles before the row's tile + its position in that tile (ticket = 128 *
-// tile + position).  The tile counts are read 4 x 16 bytes at a time, all in
-// flight together.  Records the row in slot_of, tok_of_slot and w_of_slot and
-// returns the slot (-1 for an id outside [0, E) or a slot outside [0, R)).
-__device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, int t, int j)
+// tiles before the row's tile (s_pre: the exclusive prefix over tiles, or
+// null to sum tile_counts from global memory) + its position in that tile
+// (ticket = 128 * tile + position).  Records the row in slot_of, tok_of_slot
+// and w_of_slot and returns the slot (-1 for an id outside [0, E) or a slot
+// outside [0, R)).
+__device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, const uint32_t *s_pre, int t,
+                                            int j)
 {
     const int r = t * p.k + j;
     const int e = p.idx[r];
@@ -54,21 +57,14 @@ __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint3
         return -1;
     }
     const int tk = p.ticket[r];
-    const int ts = min(tk >> 7, p.slots4);
-    const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
-    const uint4 *tc4 = reinterpret_cast<const uint4 *>(tc);
+    const int ts = min(tk >> 7, p.slots4 - 1);
     uint32_t before = 0;
-    const int full = ts >> 2;
-    for (int g0 = 0; g0 < full; g0 += 4) {
-        uint4 x[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-            if (g0 + u < full) x[u] = __ldg(tc4 + g0 + u);
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-            if (g0 + u < full) before += x[u].x + x[u].y + x[u].z + x[u].w;
+    if (s_pre) {
+        before = s_pre[e * p.slots4 + ts];
+    } else {  // a table too large for shared memory: sum the earlier tiles' counts
+        const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
+        for (int s2 = 0; s2 < ts; ++s2) before += __ldg(tc + s2);
     }
-    for (int s2 = full << 2; s2 < ts; ++s2) before += __ldg(tc + s2);
     const int slot = (int)(s_off[e] + before) + (tk & 127);
     if ((unsigned)slot >= (unsigned)p.R) return -1;  // only a corrupt ticket could fail this
     p.slot_of[r] = slot;
@@ -85,8 +81,16 @@ __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint3
 __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const DispatchParams p)
 {
     __shared__ uint32_t s_off[2 * kMaxPool + 1];
+    extern __shared__ __align__(16) uint32_t s_pre[];  // [E][slots4] when it fits (dynamic size > 0)
     pdl_trigger();
     pdl_wait();
+    // the per-expert exclusive prefix of the router's tile counts, once per CTA
+    const bool pre = p.pre_in_smem != 0;
+    if (pre) {
+        const int n4 = p.E * p.slots4 / 4;
+        for (int i = threadIdx.x; i < n4; i += kDispThreads)
+            reinterpret_cast<uint4 *>(s_pre)[i] = __ldg(reinterpret_cast<const uint4 *>(p.tile_counts) + i);
+    }
     if (threadIdx.x < 32) {
         uint32_t carry = 0;
         const int lane = threadIdx.x;
@@ -103,6 +107,17 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
         if (lane == 0) s_off[0] = 0;
     }
     __syncthreads();
+    if (pre) {
+        for (int e = threadIdx.x; e < p.E; e += kDispThreads) {
+            uint32_t acc = 0;
+            for (int s2 = 0; s2 < p.slots4; ++s2) {
+                const uint32_t v = s_pre[e * p.slots4 + s2];
+                s_pre[e * p.slots4 + s2] = acc;
+                acc += v;
+            }
+        }
+        __syncthreads();
+    }
     if (blockIdx.x == 0)
         for (int e = threadIdx.x; e <= p.E; e += kDispThreads) p.offsets[e] = s_off[e];
 
@@ -118,6 +133,7 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
         const int j0 = gj * per, j1 = min(p.k, j0 + per);
         const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
         int my_slot = -1;
+        if (lane >= j0 && lane < j1) my_slot = resolve_slot(p, s_off, pre ? s_pre : nullptr, t, lane);
         for (int c0 = 0; c0 < nv; c0 += 32 * 8) {
             uint4 v[8];
 #pragma unroll
@@ -125,8 +141,6 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
                 const int c = c0 + u * 32 + lane;
                 if (c < nv) v[u] = __ldg(src + c);
             }
-            // the slots are resolved while the row's loads are in flight
-            if (c0 == 0 && lane >= j0 && lane < j1) my_slot = resolve_slot(p, s_off, t, lane);
             for (int j = j0; j < j1; ++j) {
                 const int slot = __shfl_sync(~0u, my_slot, j);
                 if (slot < 0) continue;
@@ -216,6 +230,10 @@ cudaError_t launch_permute(const Ctx &c)
     p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts; p.hidden = c.hidden;
     p.tile_counts = c.tile_counts;
     p.slots4 = router_slots4(c.s.T);
+    // the table's prefix per CTA in shared memory when it is small (no opt-in
+    // above the default 48 KB); otherwise each row sums it from global memory
+    const size_t pre_bytes = sizeof(uint32_t) * (size_t)s.E() * p.slots4;
+    p.pre_in_smem = pre_bytes <= 40 * 1024 ? 1 : 0;
     p.T = s.T; p.H = s.H; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.a_perm = c.a_perm;
@@ -225,7 +243,7 @@ cudaError_t launch_permute(const Ctx &c)
     const long long want = 32LL * c.num_sms;
     p.groups = (int)std::min<long long>(s.k, std::max<long long>(1, (want + s.T - 1) / s.T));
     return launch_pdl(dispatch_gather_kernel, dim3(grid_for((long long)s.T * p.groups * 32, c.num_sms)),
-                      dim3(kDispThreads), 0, c.stream, p);
+                      dim3(kDispThreads), p.pre_in_smem ? pre_bytes : 0, c.stream, p);
 }
 
 cudaError_t launch_combine(const Ctx &c)
