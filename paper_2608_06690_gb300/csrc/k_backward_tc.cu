@@ -170,7 +170,7 @@ struct RowsParams {
 
 struct RowsMaps {
     CUtensorMap a;       // Z: dout rows [R + 64][H]; gate/up: A rows [R][H]; 64 x 128 box (K-major)
-    CUtensorMap b0, b1;  // Z: W_down [E_priv H][I], 64 x 64 box (MN-major); gate/up: gate, up [E_priv I][H], 64 x 128
+    CUtensorMap b0, b1;  // Z: W_down [E_priv H][I], 64 x 64 x bn/128 3-D box (MN-major); gate/up: gate, up, 64 x 128
     CUtensorMap out0;    // Z: Z [RP][I]; gate/up: [dG | dU] [RP][2I]  (32 x 32 BF16 boxes, 64-byte swizzle)
     CUtensorMap out1;    // gate/up: w act [RP][I]
 };
@@ -239,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
         // ------------------------------------------------ TMA producers
         // lane 0: the tile's 128 rows x 64 K of A (16 KB).  Gate/up: lane 1 the
         // 128 gate rows, lane 2 the 128 up rows (16 KB each).  Z: lanes 1-2 half
-        // of the bn / 64 MN blocks of W_down each (8 KB per block).
+        // of the bn / 64 MN blocks of W_down each, as one 3-D box (8 KB per block).
         int stage = 0;
         uint32_t phase = 0, filled = 0, last_parity = 0;
         const int half = p.bn / 128;  // Z: MN blocks per loader lane
@@ -259,9 +259,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
                     tma_load_2d(sB + (lane - 1) * kABytes, lane == 1 ? &maps.b0 : &maps.b1, full_bar(stage), kx,
                                 t.q * p.I + t.n0);
                 } else {
+                    const int b0 = (lane - 1) * half;
                     mbar_expect_tx(full_bar(stage), (uint32_t)(half * kMnBlockBytes));
-                    for (int b = (lane - 1) * half; b < lane * half; ++b)
-                        tma_load_2d(sB + b * kMnBlockBytes, &maps.b0, full_bar(stage), t.n0 + b * 64, t.q * p.H + kx);
+                    tma_load_3d(sB + b0 * kMnBlockBytes, &maps.b0, full_bar(stage), 0, t.q * p.H + kx, t.n0 / 64 + b0);
                 }
                 filled |= 1u << stage;
                 last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
@@ -407,10 +407,11 @@ struct WgParams {
 };
 
 struct WgMaps {
-    CUtensorMap dgu;        // [padded rows][2I], 64 x 64 box (MN-major A)
-    CUtensorMap a_perm;     // [R][H], 64 x 64 box (MN-major B)
-    CUtensorMap dout_rows;  // [R + 64][H], 64 x 64 box (MN-major A)
-    CUtensorMap wact;       // [padded rows][I], 64 x 64 box (MN-major B)
+    // 3-D maps, boxes of 64 rows (K) x 64-element MN blocks (encode_3d_blocks)
+    CUtensorMap dgu;        // [padded rows][2I], 2 blocks per box (MN-major A)
+    CUtensorMap a_perm;     // [R][H], bn_a / 128 blocks per box (MN-major B)
+    CUtensorMap dout_rows;  // [R + 64][H], 2 blocks per box (MN-major A)
+    CUtensorMap wact;       // [padded rows][I], bn_b / 128 blocks per box (MN-major B)
     CUtensorMap d_gate, d_up, d_down;  // FP32 outputs, 16 x 32 boxes, 64-byte swizzle
 };
 
@@ -481,7 +482,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
         // lane 0: the two 64-element MN blocks of A; lanes 1-2: half of B's
-        // bn / 64 blocks each.  Boxes are 64 MN elements x 64 rows (K).
+        // bn / 64 blocks each; one 3-D box per lane (64 MN elements x 64 rows of
+        // K per block).
         int stage = 0;
         uint32_t phase = 0, filled = 0, last_parity = 0;
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
@@ -498,11 +500,10 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
                 const int ky = kb * BK;
                 mbar_expect_tx(full_bar(stage), lane == 0 ? (uint32_t)kABytes : (uint32_t)(half * kMnBlockBytes));
                 if (lane == 0) {
-                    tma_load_2d(sA, amap, full_bar(stage), t.m0, rowA + ky);
-                    tma_load_2d(sA + kMnBlockBytes, amap, full_bar(stage), t.m0 + 64, rowA + ky);
+                    tma_load_3d(sA, amap, full_bar(stage), 0, rowA + ky, t.m0 / 64);
                 } else {
-                    for (int b = (lane - 1) * half; b < lane * half; ++b)
-                        tma_load_2d(sB + b * kMnBlockBytes, bmap, full_bar(stage), t.n0 + b * 64, rowB + ky);
+                    const int b0 = (lane - 1) * half;
+                    tma_load_3d(sB + b0 * kMnBlockBytes, bmap, full_bar(stage), 0, rowB + ky, t.n0 / 64 + b0);
                 }
                 filled |= 1u << stage;
                 last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
@@ -628,7 +629,7 @@ cudaError_t launch_backward_rows(const Ctx &c, const bf16 *dout_rows, bf16 *zpad
             p.bn = s.I % 256 == 0 ? 256 : 128;
             p.idesc = make_idesc_major(BM, p.bn, false, true);
             ok = encode_2d(&maps.a, dout_rows, s.H, R + 64, BM);
-            ok &= encode_2d_box(&maps.b0, c.down[1], s.I, (uint64_t)s.E_priv * s.H, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
+            ok &= encode_3d_blocks(&maps.b0, c.down[1], s.I, (uint64_t)s.E_priv * s.H, 64, p.bn / 128);
             ok &= encode_2d_box(&maps.out0, zpad, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
         } else {
             p.bn = 128;
@@ -665,11 +666,11 @@ cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf1
     p.status = c.audit.status;
     p.idesc_a = make_idesc_major(BM, p.bn_a, true, true);
     p.idesc_b = make_idesc_major(BM, p.bn_b, true, true);
-    const CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_128B;
-    bool ok = encode_2d_box(&maps.dgu, dgu, 2 * (uint64_t)s.I, RP, 64, 64, sw);
-    ok &= encode_2d_box(&maps.a_perm, c.a_perm, s.H, R, 64, 64, sw);
-    ok &= encode_2d_box(&maps.dout_rows, dout_rows, s.H, R + 64, 64, 64, sw);
-    ok &= encode_2d_box(&maps.wact, wact, s.I, RP, 64, 64, sw);
+    // A: both 64-element MN blocks in one box; B: half of its blocks per box
+    bool ok = encode_3d_blocks(&maps.dgu, dgu, 2 * (uint64_t)s.I, RP, 64, 2);
+    ok &= encode_3d_blocks(&maps.a_perm, c.a_perm, s.H, R, 64, p.bn_a / 128);
+    ok &= encode_3d_blocks(&maps.dout_rows, dout_rows, s.H, R + 64, 64, 2);
+    ok &= encode_3d_blocks(&maps.wact, wact, s.I, RP, 64, p.bn_b / 128);
     const CUtensorMapSwizzle osw = CU_TENSOR_MAP_SWIZZLE_64B;
     ok &= encode_2d_f32(&maps.d_gate, d_gate, s.H, (uint64_t)s.E_priv * s.I, 16, 32, osw);
     ok &= encode_2d_f32(&maps.d_up, d_up, s.H, (uint64_t)s.E_priv * s.I, 16, 32, osw);

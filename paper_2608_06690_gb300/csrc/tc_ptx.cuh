@@ -77,6 +77,15 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// 3-D tile load: box coordinates (x, y, z) of a map made by encode_3d_blocks.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y, int z)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], [%2];\n" ::
+            "r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(x), "r"(y), "r"(z)
+        : "memory");
+}
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
 
@@ -186,6 +195,12 @@ bool encode_2d_box(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows
 // 2-D FP32 tensor map with a box_cols x box_rows box and the given swizzle.
 bool encode_2d_f32(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_cols,
                    uint32_t box_rows, CUtensorMapSwizzle swizzle);
+// 3-D BF16 tensor map over a row-major [rows, cols] matrix seen as
+// [cols / 64 blocks][rows][64]: a box of box_rows rows x nblocks consecutive
+// 64-column blocks lands in shared memory as nblocks 128-byte-swizzled
+// [box_rows][64] tiles one after another (the layout of an MN-major operand
+// whose MN blocks are box_rows * 128 bytes apart).
+bool encode_3d_blocks(CUtensorMap *m, const void *ptr, uint64_t cols, uint64_t rows, uint32_t box_rows, uint32_t nblocks);
 // tcgen05 instruction descriptor: BF16 x BF16 -> FP32, both operands K-major.
 uint32_t make_idesc(int M, int N);
 // The same with either operand MN-major (transpose bits 15 for A, 16 for B).
