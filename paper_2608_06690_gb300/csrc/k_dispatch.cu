@@ -28,9 +28,9 @@ struct DispatchParams {
     const int32_t *ticket;
     const float *w;
     const uint32_t *counts;
-    const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
+    const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile, or their prefix sums
     int slots4;
-    int pre_in_smem;              // 1: each CTA keeps the table's prefix in shared memory
+    int tile_prefix;              // 1: the router replaced each row by its exclusive prefix sum
     const bf16 *hidden;
     int T, H, R, k, E;
     int groups;  // warps per token: each stores the row to a share of its k slots
@@ -42,13 +42,12 @@ struct DispatchParams {
 };
 
 // Slot of routed row (t, j): offset[e] + the rows of expert e in the router
-// tiles before the row's tile (s_pre: the exclusive prefix over tiles, or
-// null to sum tile_counts from global memory) + its position in that tile
+// tiles before the row's tile (the router's prefix sums, or a sum of the
+// per-tile counts for tables too large for it) + its position in that tile
 // (ticket = 128 * tile + position).  Records the row in slot_of, tok_of_slot
 // and w_of_slot and returns the slot (-1 for an id outside [0, E) or a slot
 // outside [0, R)).
-__device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, const uint32_t *s_pre, int t,
-                                            int j)
+__device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, int t, int j)
 {
     const int r = t * p.k + j;
     const int e = p.idx[r];
@@ -58,11 +57,11 @@ __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint3
     }
     const int tk = p.ticket[r];
     const int ts = min(tk >> 7, p.slots4 - 1);
+    const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
     uint32_t before = 0;
-    if (s_pre) {
-        before = s_pre[e * p.slots4 + ts];
-    } else {  // a table too large for shared memory: sum the earlier tiles' counts
-        const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
+    if (p.tile_prefix) {
+        before = __ldg(tc + ts);
+    } else {  // a table too large for the router's shared memory: sum the earlier tiles' counts
         for (int s2 = 0; s2 < ts; ++s2) before += __ldg(tc + s2);
     }
     const int slot = (int)(s_off[e] + before) + (tk & 127);
@@ -81,16 +80,8 @@ __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint3
 __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const DispatchParams p)
 {
     __shared__ uint32_t s_off[2 * kMaxPool + 1];
-    extern __shared__ __align__(16) uint32_t s_pre[];  // [E][slots4] when it fits (dynamic size > 0)
     pdl_trigger();
     pdl_wait();
-    // the per-expert exclusive prefix of the router's tile counts, once per CTA
-    const bool pre = p.pre_in_smem != 0;
-    if (pre) {
-        const int n4 = p.E * p.slots4 / 4;
-        for (int i = threadIdx.x; i < n4; i += kDispThreads)
-            reinterpret_cast<uint4 *>(s_pre)[i] = __ldg(reinterpret_cast<const uint4 *>(p.tile_counts) + i);
-    }
     if (threadIdx.x < 32) {
         uint32_t carry = 0;
         const int lane = threadIdx.x;
@@ -107,17 +98,6 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
         if (lane == 0) s_off[0] = 0;
     }
     __syncthreads();
-    if (pre) {
-        for (int e = threadIdx.x; e < p.E; e += kDispThreads) {
-            uint32_t acc = 0;
-            for (int s2 = 0; s2 < p.slots4; ++s2) {
-                const uint32_t v = s_pre[e * p.slots4 + s2];
-                s_pre[e * p.slots4 + s2] = acc;
-                acc += v;
-            }
-        }
-        __syncthreads();
-    }
     if (blockIdx.x == 0)
         for (int e = threadIdx.x; e <= p.E; e += kDispThreads) p.offsets[e] = s_off[e];
 
@@ -133,7 +113,7 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
         const int j0 = gj * per, j1 = min(p.k, j0 + per);
         const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
         int my_slot = -1;
-        if (lane >= j0 && lane < j1) my_slot = resolve_slot(p, s_off, pre ? s_pre : nullptr, t, lane);
+        if (lane >= j0 && lane < j1) my_slot = resolve_slot(p, s_off, t, lane);
         for (int c0 = 0; c0 < nv; c0 += 32 * 8) {
             uint4 v[8];
 #pragma unroll
@@ -230,10 +210,7 @@ cudaError_t launch_permute(const Ctx &c)
     p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts; p.hidden = c.hidden;
     p.tile_counts = c.tile_counts;
     p.slots4 = router_slots4(c.s.T);
-    // the table's prefix per CTA in shared memory when it is small (no opt-in
-    // above the default 48 KB); otherwise each row sums it from global memory
-    const size_t pre_bytes = sizeof(uint32_t) * (size_t)s.E() * p.slots4;
-    p.pre_in_smem = pre_bytes <= 40 * 1024 ? 1 : 0;
+    p.tile_prefix = router_tile_prefix(s) ? 1 : 0;
     p.T = s.T; p.H = s.H; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.a_perm = c.a_perm;
@@ -243,7 +220,7 @@ cudaError_t launch_permute(const Ctx &c)
     const long long want = 32LL * c.num_sms;
     p.groups = (int)std::min<long long>(s.k, std::max<long long>(1, (want + s.T - 1) / s.T));
     return launch_pdl(dispatch_gather_kernel, dim3(grid_for((long long)s.T * p.groups * 32, c.num_sms)),
-                      dim3(kDispThreads), p.pre_in_smem ? pre_bytes : 0, c.stream, p);
+                      dim3(kDispThreads), 0, c.stream, p);
 }
 
 cudaError_t launch_combine(const Ctx &c)
