@@ -150,17 +150,15 @@ typedef struct pmpe_workspace_layout {
     size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row */
     size_t act_sh;       /* BF16   [T, E_shared*I] shared-expert activations (0 if none) */
     size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs (0 if none) */
-    size_t tile_done;    /* uint32 [S + 1]  router CTAs finished per 128-token tile; [S]: tiles merged */
+    size_t tile_done;    /* uint32 [S]      router CTAs finished per 128-token tile */
     size_t router_lists; /* float2 [C2*128, k] per 32-expert chunk: each token's best k (score, id) */
     size_t router_meta;  /* float4 [C2*128] per chunk: max score, sum exp(score - max), entries */
     size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1]  gate/up epilogue warps done per
                           * (expert group, 128-row block), read by the down tiles of the same launch */
-    size_t tile_counts;  /* uint32 [E, S4]  rows of expert e in router tile s (S4 = S rounded up to 4);
-                          * when E * S4 * 4 <= 192 KB the router's last merging CTA replaces each row
-                          * by its exclusive prefix sum.  With the tiles of a pool in ascending token
-                          * order, slot offsets[e] + sum_{s' < s} tile_counts[e, s'] + position gives
-                          * every expert its rows in ascending (t, j) order: the dispatch order is
-                          * deterministic */
+    size_t tile_counts;  /* uint32 [E, S4]  rows of expert e in router tile s (S4 = S rounded up to 4).
+                          * With the tiles of a pool in ascending token order, slot
+                          * offsets[e] + sum_{s' < s} tile_counts[e, s'] + position gives every expert
+                          * its rows in ascending (t, j) order: the dispatch order is deterministic */
 } pmpe_workspace_layout;
 PMPE_API int pmpe_moe_workspace_layout(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k,
                               pmpe_workspace_layout *out);

@@ -28,9 +28,8 @@ struct DispatchParams {
     const int32_t *ticket;
     const float *w;
     const uint32_t *counts;
-    const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile, or their prefix sums
+    const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
     int slots4;
-    int tile_prefix;              // 1: the router replaced each row by its exclusive prefix sum
     const bf16 *hidden;
     int T, H, R, k, E;
     int groups;  // warps per token: each stores the row to a share of its k slots
@@ -42,9 +41,10 @@ struct DispatchParams {
 };
 
 // Slot of routed row (t, j): offset[e] + the rows of expert e in the router
-// tiles before the row's tile (the router's prefix sums, or a sum of the
-// per-tile counts for tables too large for it) + its position in that tile
-// (ticket = 128 * tile + position).  Records the row in slot_of, tok_of_slot
+// tiles before the row's tile + its position in that tile (ticket = 128 *
+// tile + position).  Summing the earlier tiles' counts per row measured
+// faster than building their prefix once, in the router's last CTA or in
+// every dispatch CTA's shared memory.  Records the row in slot_of, tok_of_slot
 // and w_of_slot and returns the slot (-1 for an id outside [0, E) or a slot
 // outside [0, R)).
 __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, int t, int j)
@@ -59,11 +59,7 @@ __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint3
     const int ts = min(tk >> 7, p.slots4 - 1);
     const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
     uint32_t before = 0;
-    if (p.tile_prefix) {
-        before = __ldg(tc + ts);
-    } else {  // a table too large for the router's shared memory: sum the earlier tiles' counts
-        for (int s2 = 0; s2 < ts; ++s2) before += __ldg(tc + s2);
-    }
+    for (int s2 = 0; s2 < ts; ++s2) before += __ldg(tc + s2);
     const int slot = (int)(s_off[e] + before) + (tk & 127);
     if ((unsigned)slot >= (unsigned)p.R) return -1;  // only a corrupt ticket could fail this
     p.slot_of[r] = slot;
@@ -210,7 +206,6 @@ cudaError_t launch_permute(const Ctx &c)
     p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts; p.hidden = c.hidden;
     p.tile_counts = c.tile_counts;
     p.slots4 = router_slots4(c.s.T);
-    p.tile_prefix = router_tile_prefix(s) ? 1 : 0;
     p.T = s.T; p.H = s.H; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.a_perm = c.a_perm;

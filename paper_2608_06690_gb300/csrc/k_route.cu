@@ -53,9 +53,7 @@ struct RouterParams {
     bf16 *rows_ws;       // [slots * nch_max * 128, H] copied tile rows, one block per CTA
     float2 *lists;       // [slots * nch_max][128][k] (score, id) sorted per chunk
     float4 *meta;        // [slots * nch_max][128] (chunk max, sum exp(x - max), entries, -)
-    uint32_t *tile_done; // [slots + 1] chunk CTAs finished per tile; [slots]: tiles merged (zeroed before the launch)
-    int slots;           // tile slots
-    int tile_prefix;     // 1: the last merging CTA turns tile_counts into per-expert prefix sums
+    uint32_t *tile_done; // [slots] chunk CTAs finished (zeroed before the launch)
     uint8_t *tau;
     int32_t *idx;
     float *w;
@@ -216,7 +214,7 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     __shared__ __align__(8) uint64_t bars[2 * kRMaxStages + 2];
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
-    __shared__ int s_last, s_last_tile;
+    __shared__ int s_last;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int slot = blockIdx.x / p.nch_max, chunk = blockIdx.x - slot * p.nch_max;
@@ -553,35 +551,6 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
                 }
                 if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], (unsigned)npriv);
             }
-            if (p.tile_prefix) {
-                // the CTA that merges the last tile turns each expert's row of
-                // tile_counts into its exclusive prefix over the tiles (the
-                // fence orders this tile's counts before the count of merged tiles)
-                __threadfence();
-                asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
-                const int n_tiles = tiles_d + (na + kTileRows - 1) / kTileRows;
-                if (et == 0) s_last_tile = atomicAdd(&p.tile_done[p.slots], 1u) == (unsigned)(n_tiles - 1);
-                asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
-                if (s_last_tile) {
-                    __threadfence();
-                    const int E = p.E_pub + p.E_priv;
-                    const int n4 = E * p.slots4 / 4;
-                    uint32_t *tab = reinterpret_cast<uint32_t *>(sv);  // the merge scratch is free again
-                    uint4 *g4 = reinterpret_cast<uint4 *>(p.tile_counts);
-                    for (int i = et; i < n4; i += kEpi) reinterpret_cast<uint4 *>(tab)[i] = __ldcg(g4 + i);
-                    asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
-                    for (int e = et; e < E; e += kEpi) {
-                        uint32_t acc = 0;
-                        for (int s2 = 0; s2 < p.slots4; ++s2) {
-                            const uint32_t v = tab[e * p.slots4 + s2];
-                            tab[e * p.slots4 + s2] = acc;
-                            acc += v;
-                        }
-                    }
-                    asm volatile("bar.sync 1, %0;\n" ::"r"(kEpi) : "memory");
-                    for (int i = et; i < n4; i += kEpi) g4[i] = reinterpret_cast<uint4 *>(tab)[i];
-                }
-            }
         }
     }
 
@@ -636,7 +605,6 @@ __global__ void resolve_kernel(const uint8_t *policy, int T, uint8_t *tau)
 int router_chunks(int pool_size) { return (pool_size + kChunk - 1) / kChunk; }
 int router_slots(int T) { return (T + kTileRows - 1) / kTileRows + 1; }
 int router_slots4(int T) { return (router_slots(T) + 3) & ~3; }
-bool router_tile_prefix(const Shape &s) { return (size_t)s.E() * router_slots4(s.T) * 4 <= 192 * 1024; }
 
 cudaError_t launch_route(const Ctx &c)
 {
@@ -658,12 +626,12 @@ cudaError_t launch_route(const Ctx &c)
     const size_t nready = gemm_ready_words(s);
     const size_t ntc = (size_t)s.E() * router_slots4(s.T);
     // tile_counts starts 16-byte aligned right after gemm_ready (at most 3 words between)
-    if (c.tile_done == c.counts + s.E() && c.gemm_ready == c.tile_done + slots + 1 &&
+    if (c.tile_done == c.counts + s.E() && c.gemm_ready == c.tile_done + slots &&
         c.tile_counts >= c.gemm_ready + nready && c.tile_counts <= c.gemm_ready + nready + 3) {
         merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * (size_t)(c.tile_counts + ntc - c.counts), c.stream);
     } else {
         merr = cudaMemsetAsync(c.counts, 0, sizeof(uint32_t) * s.E(), c.stream);
-        if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_done, 0, sizeof(uint32_t) * (slots + 1), c.stream);
+        if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_done, 0, sizeof(uint32_t) * slots, c.stream);
         if (merr == cudaSuccess) merr = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * nready, c.stream);
         if (merr == cudaSuccess) merr = cudaMemsetAsync(c.tile_counts, 0, sizeof(uint32_t) * ntc, c.stream);
     }
@@ -676,8 +644,6 @@ cudaError_t launch_route(const Ctx &c)
     p.lists = c.router_lists;
     p.meta = c.router_meta;
     p.tile_done = c.tile_done;
-    p.slots = slots;
-    p.tile_prefix = router_tile_prefix(s) ? 1 : 0;
     p.tau = c.tau;
     p.idx = c.idx;
     p.w = c.w;

@@ -41,7 +41,7 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     const size_t slots = (size_t)router_slots(s.T);
     const size_t rctas = slots * (size_t)std::max(router_chunks(s.E_pub), router_chunks(s.E_priv));
     const size_t rctas_all = slots * (size_t)(router_chunks(s.E_pub) + router_chunks(s.E_priv));
-    L->tile_done = take(4 * (slots + 1), 4);  // + the count of merged tiles
+    L->tile_done = take(4 * slots, 4);
     L->gemm_ready = take(4 * gemm_ready_words(s), 4);
     L->tile_counts = take(4 * E * (size_t)router_slots4(s.T), 16);  // read as 16-byte vectors
     L->offsets = take(4 * (E + 1), 256);

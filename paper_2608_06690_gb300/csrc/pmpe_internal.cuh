@@ -51,7 +51,7 @@ struct Ctx {
     int32_t *slot_of, *tok_of_slot;
     int32_t *ticket;    // [T, k] 128 * router tile + position among the tile's rows of its expert
     float *w_of_slot;
-    uint32_t *tile_done;  // [router slots + 1] chunk CTAs finished per router tile; the last: tiles merged
+    uint32_t *tile_done;  // [router slots] chunk CTAs finished per router tile
     uint32_t *tile_counts; // [E][router_slots4] rows of each expert per router tile
     uint32_t *gemm_ready; // [gemm_ready_words] gate/up warps done per (group, 128-row block)
     float2 *router_lists; // [router CTAs * 128, k] per-chunk sorted (score, id)
@@ -69,9 +69,6 @@ int router_chunks(int pool_size);
 int router_slots(int T);
 // router_slots rounded up to a multiple of 4 (the row pitch of tile_counts).
 int router_slots4(int T);
-// Whether the router turns tile_counts into per-expert prefix sums (the table
-// fits in its shared memory); otherwise the dispatch sums the counts per row.
-bool router_tile_prefix(const Shape &s);
 // Readiness counters of the persistent expert GEMMs: one per (group, 128-row
 // block), an upper bound over all routings.
 size_t gemm_ready_words(const Shape &s);

@@ -77,7 +77,7 @@ def test_workspace_size_and_layout(pmpe):
         ctas = slots * max((sh.E_pub + 31) // 32, (sh.E_priv + 31) // 32)
         ctas_all = slots * ((sh.E_pub + 31) // 32 + (sh.E_priv + 31) // 32)
         size = dict(tau=T, counts=4 * E, offsets=4 * (E + 1), topk_idx=4 * R, topk_w=4 * R, slot_of=4 * R,
-                    ticket=4 * R, tok_of_slot=4 * R, w_of_slot=4 * R, tile_done=4 * (slots + 1),
+                    ticket=4 * R, tok_of_slot=4 * R, w_of_slot=4 * R, tile_done=4 * slots,
                     router_lists=8 * ctas_all * 128 * sh.k, router_meta=16 * ctas_all * 128,
                     gemm_ready=4 * ((R + 127) // 128 + E + (T + 127) // 128 + 1),
                     router_rows=2 * ctas * 128 * sh.H, a_perm=2 * R * sh.H, act=2 * R * sh.I, y=2 * R * sh.H,
@@ -89,7 +89,7 @@ def test_workspace_size_and_layout(pmpe):
         assert spans[-1][1] <= LL["total"]
         assert LL["router_meta"] % 16 == 0 and LL["router_lists"] % 8 == 0 and LL["router_rows"] % 1024 == 0
         assert LL["tile_done"] == LL["counts"] + 4 * E  # one memset clears these three
-        assert LL["gemm_ready"] == LL["tile_done"] + 4 * (slots + 1)
+        assert LL["gemm_ready"] == LL["tile_done"] + 4 * slots
         gr_end = LL["gemm_ready"] + 4 * ((R + 127) // 128 + E + (T + 127) // 128 + 1)
         assert LL["tile_counts"] % 16 == 0 and gr_end <= LL["tile_counts"] <= gr_end + 12
     assert pmpe.workspace_size(LayerShape(64, 200, 128, 8, 4, 0, 2, True)) == 0    # H % 128

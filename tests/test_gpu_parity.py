@@ -34,10 +34,9 @@ CASES = {
     "large_pools_256": (LayerShape(T=96, H=128, I=128, E_pub=256, E_priv=256, E_sh=0, k=6, renormalize=True), 39,
                         "iid"),
     "single_token": (LayerShape(T=1, H=256, I=128, E_pub=8, E_priv=4, E_sh=1, k=2, renormalize=True), 40, "allow"),
-    # 512 experts x 104 router tiles: the per-tile count table (208 KB) exceeds
-    # the router's shared memory, so every dispatched row sums it from global memory
-    "dispatch_table_in_global_memory": (LayerShape(T=13000, H=128, I=128, E_pub=256, E_priv=256, E_sh=0, k=2,
-                                                   renormalize=True), 45, "iid"),
+    # 512 experts x 104 router tiles: the stable dispatch order across many tiles
+    "many_router_tiles_512_experts": (LayerShape(T=13000, H=128, I=128, E_pub=256, E_priv=256, E_sh=0, k=2,
+                                                 renormalize=True), 45, "iid"),
     # k > 8 takes the router's sorting-network path; 40 public experts span two chunks
     "k12_two_chunks_pool_softmax": (LayerShape(T=150, H=256, I=128, E_pub=40, E_priv=16, E_sh=0, k=12,
                                                renormalize=False), 44, "iid"),
