@@ -63,3 +63,51 @@ def test_48_layer_stack_replays_bitwise_from_a_cuda_graph():
     assert np.array_equal(a["exec_priv_rows"], a["route_priv_rows"])
     assert np.array_equal(a["exec_rows"], a["route_count"])
     assert a["route_count"].sum() == 2 * N_LAYERS * s.T * s.k
+
+
+def test_training_step_with_private_backward_replays_bitwise_from_a_cuda_graph():
+    """One training step of a two-layer stack captured into one CUDA graph:
+    the layers' forwards (the second fed the first one's output), then the
+    private-branch backward of each layer for its upstream gradient.  Each
+    layer keeps its own workspace, which holds that layer's forward state for
+    its backward.  Replaying the graph twice gives bit for bit the outputs and
+    the four private gradients of each layer computed one call at a time."""
+    s = LayerShape(T=512, H=512, I=256, E_pub=32, E_priv=8, E_sh=0, k=4, renormalize=True)
+    layers = [pmpe.MoeLayer(s, inp.make_weights(s, 8000 + l, device="cuda")) for l in range(2)]
+    x0 = inp.make_hidden(s, 8, device="cuda")
+    pol = inp.policy_iid_mixed(s.T, 8).cuda()
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(9)
+    douts = [torch.randn((s.T, s.H), generator=gen, device="cuda").to(torch.bfloat16) for _ in layers]
+
+    def step(x_in, outs):
+        ins = [x_in, outs[0]]
+        for l, layer in enumerate(layers):
+            layer.forward(ins[l], pol, out=outs[l])
+        return [layers[l].backward_private(ins[l], pol, douts[l]) for l in range(len(layers))]
+
+    outs_e = [torch.empty_like(x0) for _ in layers]
+    grads_e = step(x0, outs_e)   # also sizes every workspace before capture
+    torch.cuda.synchronize()
+    grads_e = [{n: v.clone() for n, v in g.items()} for g in grads_e]
+
+    x_in = x0.clone()
+    outs_g = [torch.empty_like(x0) for _ in layers]
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):                 # warm-up on the capture stream
+        step(x_in, outs_g)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        grads_g = step(x_in, outs_g)
+    for rep in range(2):
+        for o in outs_g:
+            o.fill_(0)
+        graph.replay()
+        torch.cuda.synchronize()
+        for l in range(len(layers)):
+            assert torch.equal(outs_g[l].view(torch.int16), outs_e[l].view(torch.int16)), (rep, l)
+            for n in grads_e[l]:
+                assert torch.equal(grads_g[l][n], grads_e[l][n]), (rep, l, n)
