@@ -182,6 +182,20 @@ def backward_private(layer: Layer, dout) -> dict:
     return r
 
 
+def backward_input(layer: Layer, dout) -> np.ndarray:
+    """Gradient of sum(dout * out) with respect to the layer's input hidden
+    states [T, H] (float64), through the frozen public, private and shared
+    weights and the router of each token's pool, for the routing the forward
+    takes.  No parameter gets a gradient here."""
+    s = layer.shape
+    d = np.ascontiguousarray(dout, dtype=np.float64).reshape(s.T, s.H)
+    dh = np.zeros((s.T, s.H))
+    rc = _load().oracle_backward_input(ctypes.byref(layer.c), d.ctypes.data_as(_f64p), dh.ctypes.data_as(_f64p))
+    if rc != 0:
+        raise ValueError("oracle_backward_input rejected the layer description")
+    return dh
+
+
 def _token_list(layer: Layer, tokens):
     if tokens is None:
         return None, layer.shape.T

@@ -43,6 +43,11 @@
  *     ("soft-router-only"): routing over the concatenated public/private pool
  *     without the hard mask.  With `unmasked` set, m(tau) = 0 for every
  *     expert; this is a negative control, not the method (G1 does not hold).
+ *   - Sec. 2.2 (G2) and Sec. 3.2 (training of the private branch): the two
+ *     backward functions -- the gradients of the private parameters, and the
+ *     gradient of the layer's input that the layer below needs -- by the chain
+ *     rule through the forward as computed (rounding points as the identity;
+ *     `exact` drops them so that finite differences can pin the functions).
  */
 #include <math.h>
 #include <stdint.h>
@@ -503,6 +508,116 @@ int oracle_backward_private(const oracle_layer *L, const double *dout, double *d
                 for (int c = 0; c < H; ++c) d_router[(size_t)(e - Ep) * H + c] += dz[e] * h[c];
     }
     free(s); free(h); free(a); free(g); free(u); free(dy); free(da); free(dz); free(gw); free(w); free(taken); free(idx);
+    return 0;
+}
+
+/* Gradient of L = sum_t dout_t . out_t with respect to the layer's input h
+ * (the hidden states), for the routing the forward takes: what the layer
+ * below needs when its own private branch is trained (Sec. 3.2 trains the
+ * private experts of two wrapped layers).  Every parameter is held fixed
+ * here -- public, private and shared alike -- and none gets a gradient; the
+ * input gradient still flows through the frozen ones (Sec. 2.2: G2 is a
+ * claim about the optimizer state, not about the derivative).  Chain rule
+ * through the forward as computed, rounding points as the identity:
+ *   per pick j (expert e, weight w_j):  da = W_down,e^T (w_j dout_t),
+ *     dg = da u silu'(g),  du = da silu(g),  dh += W_gate,e^T dg + W_up,e^T du
+ *   per shared expert (weight 1): the same with da = W_down,s^T dout_t
+ *   router, over the token's eligible pool (the unmasked control: all E):
+ *     dz as in oracle_backward_private,  dh += sum_e dz_e W_router,e
+ * A token whose dout row is zero contributes nothing and is skipped.
+ * dout [T][H]; d_hidden [T][H] (overwritten).  Serial (test sizes). */
+int oracle_backward_input(const oracle_layer *L, const double *dout, double *d_hidden)
+{
+    if (check_layer(L)) return -1;
+    const int E = L->E_pub + L->E_priv, H = L->H, I = L->I, k = L->k;
+    memset(d_hidden, 0, sizeof(double) * (size_t)L->T * H);
+    double *s = (double *)malloc(sizeof(double) * E), *h = (double *)malloc(sizeof(double) * H);
+    double *a = (double *)malloc(sizeof(double) * I), *g = (double *)malloc(sizeof(double) * I);
+    double *u = (double *)malloc(sizeof(double) * I), *da = (double *)malloc(sizeof(double) * I);
+    double *dz = (double *)malloc(sizeof(double) * E);
+    double *gw = (double *)malloc(sizeof(double) * k), *w = (double *)malloc(sizeof(double) * k);
+    char *taken = (char *)malloc(E);
+    int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * k);
+    for (int t = 0; t < L->T; ++t) {
+        const double *dt = dout + (size_t)t * H;
+        int nonzero = 0;
+        for (int o = 0; o < H && !nonzero; ++o) nonzero = dt[o] != 0.0;
+        if (!nonzero) continue;
+        double gap;
+        route_token(L, t, idx, w, &gap, s, taken);
+        const uint16_t *hr = L->hidden + (size_t)t * H;
+        for (int c = 0; c < H; ++c) h[c] = bf16_value(hr[c]);
+        double *dh = d_hidden + (size_t)t * H;
+        /* routed experts (j < k) and shared experts (j >= k, weight 1) */
+        for (int j = 0; j < k + L->E_sh; ++j) {
+            const uint16_t *Wg, *Wu, *Wd;
+            double wj = 1.0;
+            if (j < k) {
+                routed_expert_weights(L, idx[j], &Wg, &Wu, &Wd);
+                wj = w[j];
+            } else {
+                const size_t ih = (size_t)I * H;
+                Wg = L->gate_sh + (j - k) * ih; Wu = L->up_sh + (j - k) * ih; Wd = L->down_sh + (j - k) * ih;
+            }
+            for (int i = 0; i < I; ++i) {
+                double gi = 0.0, ui = 0.0;
+                for (int c = 0; c < H; ++c) {
+                    gi += h[c] * bf16_value(Wg[(size_t)i * H + c]);
+                    ui += h[c] * bf16_value(Wu[(size_t)i * H + c]);
+                }
+                g[i] = gi;
+                u[i] = ui;
+                const double silu = gi / (1.0 + exp(-gi));
+                a[i] = L->exact ? silu * ui : bf16_value(oracle_bf16_round(silu * ui));
+            }
+            if (j < k) {  /* dL/dw_j = dout_t . y'_j */
+                double gwj = 0.0;
+                for (int o = 0; o < H; ++o) {
+                    double yo = 0.0;
+                    for (int i = 0; i < I; ++i) yo += a[i] * bf16_value(Wd[(size_t)o * I + i]);
+                    gwj += dt[o] * yo;
+                }
+                gw[j] = gwj;
+            }
+            for (int i = 0; i < I; ++i) {
+                double acc = 0.0;
+                for (int o = 0; o < H; ++o) acc += bf16_value(Wd[(size_t)o * I + i]) * dt[o];
+                da[i] = wj * acc;
+            }
+            for (int i = 0; i < I; ++i) {
+                const double sg = 1.0 / (1.0 + exp(-g[i]));
+                const double dg = da[i] * u[i] * sg * (1.0 + g[i] * (1.0 - sg));
+                const double du = da[i] * g[i] * sg;
+                for (int c = 0; c < H; ++c)
+                    dh[c] += dg * bf16_value(Wg[(size_t)i * H + c]) + du * bf16_value(Wu[(size_t)i * H + c]);
+            }
+        }
+        /* router: dz over the eligible pool, dh += sum_e dz_e W_router,e */
+        for (int e = 0; e < E; ++e) dz[e] = 0.0;
+        double sum = 0.0;
+        for (int j = 0; j < k; ++j) sum += w[j] * gw[j];
+        if (L->renormalize) {
+            for (int j = 0; j < k; ++j) dz[idx[j]] = w[j] * (gw[j] - sum);
+        } else {
+            const double smax = s[idx[0]];
+            double denom = 0.0;
+            for (int e = 0; e < E; ++e) denom += exp(s[e] - smax);
+            for (int e = 0; e < E; ++e) {
+                if (s[e] == -INFINITY) continue;
+                const double pe = exp(s[e] - smax) / denom;
+                double dpe = 0.0;
+                for (int j = 0; j < k; ++j)
+                    if (idx[j] == e) dpe = gw[j];
+                dz[e] = pe * (dpe - sum);
+            }
+        }
+        for (int e = 0; e < E; ++e)
+            if (dz[e] != 0.0) {
+                const uint16_t *wr = router_row(L, e);
+                for (int c = 0; c < H; ++c) dh[c] += dz[e] * bf16_value(wr[c]);
+            }
+    }
+    free(s); free(h); free(a); free(g); free(u); free(da); free(dz); free(gw); free(w); free(taken); free(idx);
     return 0;
 }
 

@@ -485,3 +485,79 @@ def test_backward_g2_invariants(renorm):
     Lu = oracle_layer(s, w, h, pol, unmasked=True)
     u1, u2 = oracle.backward_private(Lu, d1), oracle.backward_private(Lu, d2)
     assert any(not np.array_equal(u1[n], u2[n]) for n in u1)
+
+
+# ------------------------------------------------- input gradient (backward)
+
+@pytest.mark.parametrize("renorm", [True, False])
+def test_input_gradient_matches_central_differences(renorm):
+    """Central differences of sum(dout * out) over one-ULP BF16 steps of single
+    hidden-state elements, on the forward without rounding (exact mode),
+    routing unchanged under every step: the path through the routed experts
+    (public for DENY, private for ALLOW tokens), the shared expert and the
+    router of the token's pool."""
+    s = LayerShape(T=24, H=32, I=16, E_pub=6, E_priv=5, E_sh=1, k=2, renormalize=renorm)
+    w, h, pol = make_layer(s, seed=41)
+    w = {n: (v * 8).to(torch.bfloat16) if v is not None else v for n, v in w.items()}
+    g = np.random.default_rng(11)
+    dout = g.standard_normal((s.T, s.H))
+    dh = oracle.backward_input(oracle_layer(s, w, h, pol, exact=True), dout)
+    _, idx0 = _loss(s, w, h, pol, dout)
+    tau = oracle.resolve(pol.numpy(), s.T)
+    checked = {0: 0, 1: 0}
+    for pool in (0, 1):
+        rows = np.flatnonzero(tau == pool)
+        sub = np.abs(dh[rows])
+        for flat in np.argsort(-sub.ravel())[:8]:
+            r, c = np.unravel_index(int(flat), sub.shape)
+            index = (int(rows[r]), int(c))
+            hp, hm = _bf16_step(h, index, True), _bf16_step(h, index, False)
+            lp, ip = _loss(s, w, hp, pol, dout)
+            lm, im = _loss(s, w, hm, pol, dout)
+            if not (np.array_equal(ip, idx0) and np.array_equal(im, idx0)):
+                continue  # the step crossed a routing decision
+            fd = (lp - lm) / (float(hp[index]) - float(hm[index]))
+            assert fd == pytest.approx(dh[index], rel=2e-3, abs=1e-9 * np.abs(dh).max()), (index, pool)
+            checked[pool] += 1
+    assert checked[0] >= 4 and checked[1] >= 4, checked
+
+
+def test_input_gradient_single_expert_pools_is_the_dense_mlp_gradient():
+    """One expert per pool and k = 1: every token runs its pool's expert with
+    weight 1 (the router contributes no gradient), plus the shared expert, so
+    the input gradient is torch.autograd's for those dense SwiGLU MLPs (fp64,
+    no rounding)."""
+    s = LayerShape(T=20, H=32, I=16, E_pub=1, E_priv=1, E_sh=1, k=1, renormalize=True)
+    w, h, pol = make_layer(s, seed=42)
+    dout = np.random.default_rng(12).standard_normal((s.T, s.H))
+    dh = oracle.backward_input(oracle_layer(s, w, h, pol, exact=True), dout)
+    tau = oracle.resolve(pol.numpy(), s.T)
+
+    def mlp(x, pre):
+        Wg, Wu, Wd = (w[f"{n}_{pre}"][0].double() for n in ("gate", "up", "down"))
+        return (F.silu(x @ Wg.T) * (x @ Wu.T)) @ Wd.T
+
+    x = h.double().clone().requires_grad_()
+    y = torch.where(torch.from_numpy(tau == 1)[:, None], mlp(x, "priv"), mlp(x, "pub")) + mlp(x, "sh")
+    (y * torch.from_numpy(dout)).sum().backward()
+    np.testing.assert_allclose(dh, x.grad.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_input_gradient_pool_separation_and_linearity():
+    """A DENY token's input gradient does not depend on the private weights
+    and an ALLOW token's not on the public ones (bitwise): the mask of Sec. 3.1
+    separates the backward paths as it separates the forward ones.  And the
+    gradient is linear in dout."""
+    s = LayerShape(T=40, H=32, I=16, E_pub=6, E_priv=4, E_sh=0, k=2, renormalize=False)
+    w, h, pol = make_layer(s, seed=43)
+    tau = oracle.resolve(pol.numpy(), s.T)
+    dout = np.random.default_rng(13).standard_normal((s.T, s.H))
+    base = oracle.backward_input(oracle_layer(s, w, h, pol), dout)
+    for side, rows in (("priv", tau == 0), ("pub", tau == 1)):
+        w2 = {n: ((v.float() * 1.5).to(torch.bfloat16) if v is not None and n.endswith(side) else v)
+              for n, v in w.items()}
+        other = oracle.backward_input(oracle_layer(s, w2, h, pol), dout)
+        assert np.array_equal(base[rows], other[rows]), side
+        assert not np.array_equal(base[~rows], other[~rows]), side
+    np.testing.assert_allclose(oracle.backward_input(oracle_layer(s, w, h, pol), 2.5 * dout), 2.5 * base,
+                               rtol=1e-12, atol=1e-14 * np.abs(base).max())
