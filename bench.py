@@ -189,6 +189,22 @@ def backward_flops(s, counts: np.ndarray, allow_tokens: int) -> float:
     return f
 
 
+def backward_input_flops(s, counts: np.ndarray, allow_tokens: int) -> float:
+    """Algorithmic FLOPs of the input gradient: per routed row and per token
+    of each shared expert, Z = W_down^T dout, the recomputed gate and up
+    projections and dA = W_gate^T dG + W_up^T dU (10 H I); the router term
+    W_router^T dz over the token's k picks (renormalised) or its whole pool,
+    whose logits the pool softmax also recomputes."""
+    rows = float(counts.sum()) + float(s.T * s.E_sh)
+    f = 10.0 * rows * s.H * s.I
+    if s.renormalize:
+        f += 2.0 * s.T * s.k * s.H
+    else:
+        pool = allow_tokens * s.E_priv + (s.T - allow_tokens) * s.E_pub
+        f += 4.0 * pool * s.H
+    return f
+
+
 def cpu_baseline(cfg, w, h, pol, budget_s=12.0, max_tokens=4096):
     """The CPU oracle, as it stands, on a bounded sample of the workload's
     tokens (the first n tokens of each request, spread evenly)."""
@@ -347,6 +363,19 @@ def run_ours(args):
         bwd_ms.append((a_ev, b_ev))
     torch.cuda.synchronize(dev)
     bwd_ms = [x.elapsed_time(y) for x, y in bwd_ms]
+    # ---- the gradient of the layer's input after the same forward
+    for _ in range(2):
+        layer.backward_input(h, pol, dout)
+    bin_ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_ev.record(stream)
+        layer.backward_input(h, pol, dout)
+        b_ev.record(stream)
+        bin_ms.append((a_ev, b_ev))
+    torch.cuda.synchronize(dev)
+    bin_ms = [x.elapsed_time(y) for x, y in bin_ms]
 
     # ---- end to end through the public API with host buffers, pipelined as a
     # serving loop would run it: step i+1's inputs are copied in (copy-in
@@ -441,6 +470,13 @@ def run_ours(args):
                 "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.KERNELS_PER_BACKWARD,
                 "l2": "flushed before every pass"}
 
+    bin_avg = float(np.mean(bin_ms))
+    f_bin = backward_input_flops(s, counts, int((pol == 1).sum().item()))
+    backward_in = {"ms": bin_avg, "flops": f_bin, "tflops": f_bin / (bin_avg / 1e3) / 1e12,
+                   "tensor_frac": f_bin / (bin_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
+                   "routed_rows": int(counts.sum()), "launches": pmpe.kernels_per_backward_input(s),
+                   "l2": "flushed before every pass"}
+
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
         "warmup": max(args.warmup, 3), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -452,6 +488,7 @@ def run_ours(args):
         "roofline": roof,
         "stages": stage_report,
         "backward_private": backward,
+        "backward_input": backward_in,
         "expert_load": {"touched": work["touched_experts"], "max_rows": int(counts.max()),
                         "mean_rows_public": float(counts[:s.E_pub].mean()),
                         "mean_rows_private": float(counts[s.E_pub:].mean())},

@@ -207,6 +207,31 @@ PMPE_API int pmpe_moe_backward_private(const pmpe_moe_desc *d, const void *dout,
                                        float *d_gate_priv, float *d_up_priv, float *d_down_priv,
                                        void *bwd_workspace, size_t bwd_workspace_bytes, void *stream);
 
+/* ------------------------------------------------- input gradient */
+
+/* Bytes of device scratch pmpe_moe_backward_input() needs; 0 for an invalid
+ * shape. */
+PMPE_API size_t pmpe_moe_backward_input_workspace_size(int T, int H, int I, int E_pub, int E_priv, int E_shared,
+                                                       int k);
+
+/* Gradient of L = sum_t dout_t . out_t with respect to the layer's input
+ * hidden [T, H], through the frozen layer, for the routing of the forward just
+ * run with the same descriptor: what the layer below needs when its own private
+ * branch is trained (Sec. 3.2).  Every term of the forward contributes: each
+ * token's k routed experts of its own pool (Eq. 1: public for DENY, private
+ * for ALLOW) through their routing weights, the shared experts with weight 1,
+ * and the router of that pool through the softmax of Eq. 2 (renormalised over
+ * the top-k, or over the pool).  The routing itself (which experts, the hard
+ * mask) is piecewise constant and contributes no gradient.  The descriptor's
+ * workspace must still hold that forward's state, as for
+ * pmpe_moe_backward_private().  dout: [T, H] BF16.  d_hidden: [T, H] FP32,
+ * overwritten, 16-byte aligned.  The per-pick input gradients are rounded to
+ * BF16 before the FP32 sum.  Not defined for the unmasked control
+ * (PMPE_ERR_UNSUPPORTED_SHAPE).  bwd_workspace: >= the size above, 256-byte
+ * aligned (PMPE_ERR_WORKSPACE otherwise).  Asynchronous on `stream`. */
+PMPE_API int pmpe_moe_backward_input(const pmpe_moe_desc *d, const void *dout, float *d_hidden, void *bwd_workspace,
+                                     size_t bwd_workspace_bytes, void *stream);
+
 /* Per-token policy bytes from per-request ones, for callers that carry one
  * trusted authorisation byte per request and the requests' cumulative token
  * offsets (cu_seqlens[0..n_req], device int32) instead of a byte per token.

@@ -41,32 +41,37 @@ __global__ void bwd_gather_kernel(const bf16 *dout, const int32_t *tok_of_slot, 
     }
 }
 
-// Router gradient per ALLOW token (one warp): the softmax gradient dz over the
-// private pool from dL/dw of its k rows (summed from the expert GEMM's per-tile
-// partials) -- renormalised over the top-k, or the
-// pool softmax, whose probabilities need every private logit, recomputed here
-// in FP32 from the BF16 operands.  dz [T][E_priv] (zero for DENY tokens).
-__global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_priv, const uint8_t *tau,
-                                  const int32_t *idx, const float *wts, const int32_t *slot_of, const float *gw_part,
-                                  int n_part, const uint32_t *offsets, int T, int H, int E_pub, int E_priv, int k,
-                                  int renorm, int R, float *dz)
+// Router gradient per token (one warp): the softmax gradient dz over the
+// token's pool from dL/dw of its k rows (summed from the expert GEMM's per-tile
+// partials, indexed by dispatch slot) -- renormalised over the top-k, or the
+// pool softmax, whose probabilities need every logit of the pool, recomputed
+// here in FP32 from the BF16 operands.  both_pools = 0: the private pool only,
+// dz [T][ld = E_priv], zero for DENY tokens; both_pools = 1: each token's own
+// pool (tau selects it), dz [T][ld] holding that pool's E_pub or E_priv entries.
+__global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_pub, const bf16 *router_priv,
+                                  const uint8_t *tau, const int32_t *idx, const float *wts, const int32_t *slot_of,
+                                  const float *gw_part, int n_part, int T, int H, int E_pub, int E_priv, int k,
+                                  int renorm, int both_pools, int ld, float *dz)
 {
-    const uint32_t p0 = min(offsets[E_pub], (uint32_t)R);
     const int lane = threadIdx.x & 31;
     const int warps = gridDim.x * (blockDim.x >> 5);
     for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < T; t += warps) {
-        float *dzt = dz + (size_t)t * E_priv;
-        if (!tau[t]) {
+        float *dzt = dz + (size_t)t * ld;
+        const int priv = tau[t] ? 1 : 0;
+        if (!priv && !both_pools) {
             for (int e = lane; e < E_priv; e += 32) dzt[e] = 0.f;
             continue;
         }
+        const int E_pool = priv ? E_priv : E_pub;
+        const int e_base = priv ? E_pub : 0;
+        const bf16 *router = priv ? router_priv : router_pub;
         // lane j < k holds pick j: its pool id and dL/dw
         int pe = -1;
         float g = 0.f, wj = 0.f;
         if (lane < k) {
-            pe = idx[(size_t)t * k + lane] - E_pub;
+            pe = idx[(size_t)t * k + lane] - e_base;
             const int slot = slot_of[(size_t)t * k + lane];
-            const float *gp = gw_part + (size_t)(slot - (int)p0) * n_part;
+            const float *gp = gw_part + (size_t)slot * n_part;
             for (int j = 0; j < n_part; ++j) g += gp[j];  // the per-tile partials of dL/dw, in order
             wj = wts[(size_t)t * k + lane];
         }
@@ -74,17 +79,17 @@ __global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_priv, c
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(~0u, sum, off);
         if (renorm) {
-            for (int e = lane; e < E_priv; e += 32) dzt[e] = 0.f;
+            for (int e = lane; e < E_pool; e += 32) dzt[e] = 0.f;
             __syncwarp();
-            if (lane < k && pe >= 0 && pe < E_priv) dzt[pe] = wj * (g - sum);
+            if (lane < k && pe >= 0 && pe < E_pool) dzt[pe] = wj * (g - sum);
         } else {
             // pool softmax over the private experts: logits of this token
             const bf16 *h = hidden + (size_t)t * H;
-            for (int e0 = 0; e0 < E_priv; e0 += 32) {
+            for (int e0 = 0; e0 < E_pool; e0 += 32) {
                 const int e = e0 + lane;
                 float z = -INFINITY;
-                if (e < E_priv) {
-                    const bf16 *wr = router_priv + (size_t)e * H;
+                if (e < E_pool) {
+                    const bf16 *wr = router + (size_t)e * H;
                     float a = 0.f;
                     for (int c = 0; c < H; c += 8) {
                         const uint4 hv = *reinterpret_cast<const uint4 *>(h + c);
@@ -99,25 +104,25 @@ __global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_priv, c
                     }
                     z = a;
                 }
-                if (e < E_priv) dzt[e] = z;  // logits parked in dz, finished below
+                if (e < E_pool) dzt[e] = z;  // logits parked in dz, finished below
             }
             __syncwarp();
             float mx = -INFINITY;
-            for (int e = lane; e < E_priv; e += 32) mx = fmaxf(mx, dzt[e]);
+            for (int e = lane; e < E_pool; e += 32) mx = fmaxf(mx, dzt[e]);
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(~0u, mx, off));
             float den = 0.f;
-            for (int e = lane; e < E_priv; e += 32) den += expf(dzt[e] - mx);
+            for (int e = lane; e < E_pool; e += 32) den += expf(dzt[e] - mx);
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(~0u, den, off);
             __syncwarp();
             // dz_e = p_e (dL/dp_e - sum): -p_e sum everywhere, plus p_e dL/dw_j at the k picks
             float pj = 0.f;
-            if (lane < k && pe >= 0 && pe < E_priv) pj = expf(dzt[pe] - mx) / den;
+            if (lane < k && pe >= 0 && pe < E_pool) pj = expf(dzt[pe] - mx) / den;
             __syncwarp();
-            for (int e = lane; e < E_priv; e += 32) dzt[e] = -(expf(dzt[e] - mx) / den) * sum;
+            for (int e = lane; e < E_pool; e += 32) dzt[e] = -(expf(dzt[e] - mx) / den) * sum;
             __syncwarp();
-            if (lane < k && pe >= 0 && pe < E_priv) dzt[pe] += pj * g;
+            if (lane < k && pe >= 0 && pe < E_pool) dzt[pe] += pj * g;
         }
         __syncwarp();
     }
@@ -214,6 +219,21 @@ int router_splits(const Shape &s, int num_sms, int *tok_per_split)
 // w act in the padded row layout ([RP][I], [RP][2I], [RP][I], BF16), the dL/dw
 // partials [R][I / 128], dz [T][E_priv] and the router weight-gradient
 // partials [splits][E_priv][H] (FP32).
+void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint32_t *offsets, int g0, int g1, int R,
+                        int H, bf16 *rows, int num_sms, cudaStream_t st)
+{
+    bwd_gather_kernel<<<num_sms * 8, 256, 0, st>>>(dout, tok_of_slot, offsets, g0, g1, R, H, rows);
+}
+
+cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz)
+{
+    const Shape &s = c.s;
+    bwd_router_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(c.hidden, c.router_pub, c.router_priv, c.tau, c.idx, c.w,
+                                                           c.slot_of, gw_part, s.I / 128, s.T, s.H, s.E_pub, s.E_priv,
+                                                           s.k, s.renorm, both_pools, ld, dz);
+    return cudaGetLastError();
+}
+
 struct BwdScratch {
     bf16 *dout_rows, *zpad, *dgu, *wact;
     float *gw_part, *dz, *part;
@@ -253,15 +273,11 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
     const int E = s.E();
     cudaStream_t st = c.stream;
 
-    bwd_gather_kernel<<<c.num_sms * 8, 256, 0, st>>>(dout, c.tok_of_slot, c.offsets, s.E_pub, E, R, H, b.dout_rows);
+    launch_gather_rows(dout, c.tok_of_slot, c.offsets, s.E_pub, E, R, H, b.dout_rows, c.num_sms, st);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     if ((err = launch_backward_rows(c, b.dout_rows, b.zpad, b.dgu, b.wact, b.gw_part)) != cudaSuccess) return err;
-
-    bwd_router_kernel<<<c.num_sms * 4, 256, 0, st>>>(c.hidden, c.router_priv, c.tau, c.idx, c.w, c.slot_of, b.gw_part,
-                                                     s.I / 128, c.offsets, s.T, H, s.E_pub, s.E_priv, s.k, s.renorm, R,
-                                                     b.dz);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 0, s.E_priv, b.dz)) != cudaSuccess) return err;
     int per = 32;
     const int nsplit = router_splits(s, c.num_sms, &per);
     dim3 grid((H + 127) / 128, (s.E_priv + 31) / 32, nsplit);

@@ -1,0 +1,187 @@
+// Gradient of the layer's input through the frozen layer (what the layer
+// below needs when its own private branch is trained, Sec. 3.2).  For
+// L = sum_t dout_t . out_t and the routing the forward took:
+//
+//   every pick (t, j) of expert e with weight w, its dispatch row r:
+//     Z_r = W_down,e^T dout_t,  g, u = W_gate,e h_t, W_up,e h_t (recomputed)
+//     dG_r = w Z_r u silu'(g),  dU_r = w Z_r silu(g)
+//     dA_r = W_gate,e^T dG_r + W_up,e^T dU_r
+//   every shared expert s (weight 1): the same with the token's own row
+//   the router of the token's pool (Eq. 1: public for DENY, private for
+//   ALLOW): dz = softmax gradient of dL/dw, dh += W_router^T dz
+//
+//   d_hidden_t = sum_j dA_{r(t, j)} + sum_s dA_{s, t} + sum_e dz_{t, e} W_router,e
+//
+// Z, [dG | dU] and dA run on the tensor cores (the row launches of
+// k_backward_tc.cu over all routed experts, then over the shared experts);
+// this file holds the final per-token sum and the launch sequence.
+#include <algorithm>
+#include <cstring>
+
+#include "pmpe_internal.cuh"
+
+namespace pmpe {
+namespace {
+
+constexpr int kPadRows = 128;  // the padded row layout of the row launches
+
+// d_hidden_t in FP32, one CTA per token at a time, each thread 8 columns.
+// The sum runs in a fixed order (picks in top-k order, shared experts, the
+// pool's router rows), so the result does not depend on scheduling.  The
+// padded start of every routed expert's rows is rebuilt per CTA from the
+// dispatch offsets.
+__global__ void __launch_bounds__(256) bwd_input_reduce_kernel(
+    const bf16 *da, const bf16 *da_sh, const float *dz, int ld, const bf16 *router_pub, const bf16 *router_priv,
+    const uint8_t *tau, const int32_t *idx, const int32_t *slot_of, const uint32_t *offsets, int T, int H, int E_pub,
+    int E_priv, int E_sh, int k, int R, int renorm, int Tp, float *d_hidden)
+{
+    __shared__ int pad_start[2 * kMaxPool];
+    __shared__ int s_carry;
+    const int E = E_pub + E_priv;
+    const int tid = threadIdx.x, lane = tid & 31;
+    pdl_wait();
+    // exclusive scan of the padded row counts, 256 experts per pass
+    if (tid == 0) s_carry = 0;
+    __syncthreads();
+    __shared__ int s_warp[8];
+    for (int b = 0; b < E; b += blockDim.x) {
+        const int e = b + tid;
+        int v = 0;
+        if (e < E) {
+            const int lo = (int)min(offsets[e], (uint32_t)R), hi = (int)min(max(offsets[e + 1], (uint32_t)lo), (uint32_t)R);
+            v = (hi - lo + kPadRows - 1) / kPadRows * kPadRows;
+        }
+        int x = v;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(~0u, x, off);
+            if (lane >= off) x += y;
+        }
+        if (lane == 31) s_warp[tid >> 5] = x;
+        __syncthreads();
+        int before = s_carry;
+        for (int w = 0; w < (tid >> 5); ++w) before += s_warp[w];
+        if (e < E) pad_start[e] = before + x - v;
+        __syncthreads();
+        if (tid == blockDim.x - 1) s_carry = before + x;
+        __syncthreads();
+    }
+
+    const int nv = H / 8;
+    for (int t = blockIdx.x; t < T; t += gridDim.x) {
+        const int priv = tau[t] ? 1 : 0;
+        const int e_base = priv ? E_pub : 0, E_pool = priv ? E_priv : E_pub;
+        const bf16 *router = priv ? router_priv : router_pub;
+        const float *dzt = dz + (size_t)t * ld;
+        for (int c = tid; c < nv; c += blockDim.x) {
+            float acc[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+            auto add_row = [&](const bf16 *row, float scale) {
+                const uint4 v = reinterpret_cast<const uint4 *>(row)[c];
+                const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float2 f = __bfloat1622float2(b[i]);
+                    acc[2 * i] += scale * f.x;
+                    acc[2 * i + 1] += scale * f.y;
+                }
+            };
+            for (int j = 0; j < k; ++j) {
+                const int e = idx[(size_t)t * k + j];
+                const int slot = slot_of[(size_t)t * k + j];
+                if (e < 0 || e >= E || slot < 0 || slot >= R) continue;
+                const int prow = pad_start[e] + slot - (int)offsets[e];
+                add_row(da + (size_t)prow * H, 1.f);
+            }
+            for (int s = 0; s < E_sh; ++s) add_row(da_sh + ((size_t)s * Tp + t) * H, 1.f);
+            if (renorm) {  // dz is zero outside the token's k picks
+                for (int j = 0; j < k; ++j) {
+                    const int pe = idx[(size_t)t * k + j] - e_base;
+                    if (pe >= 0 && pe < E_pool) add_row(router + (size_t)pe * H, dzt[pe]);
+                }
+            } else {
+                for (int e = 0; e < E_pool; ++e) add_row(router + (size_t)e * H, dzt[e]);
+            }
+            float4 *o = reinterpret_cast<float4 *>(d_hidden + (size_t)t * H) + 2 * c;
+            o[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+            o[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+        }
+    }
+}
+
+}  // namespace
+
+struct InScratch {
+    bf16 *dout_rows, *zpad, *dgu, *da, *zpad_sh, *dgu_sh, *da_sh;
+    float *gw_part, *dz;
+    uint64_t rp, rp_sh;  // padded rows: routed, shared
+    int tp;              // tokens rounded up to the padded layout (rows of one shared expert)
+    size_t bytes;
+};
+
+static InScratch input_scratch(const Shape &s, uint8_t *base)
+{
+    const size_t R = (size_t)s.T * s.k, H = s.H, I = s.I;
+    auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+    InScratch b;
+    b.rp = R + (uint64_t)kPadRows * s.E();
+    b.tp = (s.T + kPadRows - 1) / kPadRows * kPadRows;
+    b.rp_sh = (uint64_t)s.E_sh * b.tp;
+    size_t o = 0;
+    b.dout_rows = (bf16 *)(base + o); o += al((R + 64) * H * 2);
+    b.zpad = (bf16 *)(base + o);      o += al(b.rp * I * 2);
+    b.dgu = (bf16 *)(base + o);       o += al(b.rp * 2 * I * 2);
+    b.da = (bf16 *)(base + o);        o += al(b.rp * H * 2);
+    b.zpad_sh = (bf16 *)(base + o);   o += al(b.rp_sh * I * 2);
+    b.dgu_sh = (bf16 *)(base + o);    o += al(b.rp_sh * 2 * I * 2);
+    b.da_sh = (bf16 *)(base + o);     o += al(b.rp_sh * H * 2);
+    b.gw_part = (float *)(base + o);  o += al(R * (I / 128) * 4);
+    b.dz = (float *)(base + o);       o += al((size_t)s.T * std::max(s.E_pub, s.E_priv) * 4);
+    b.bytes = o;
+    return b;
+}
+
+size_t backward_input_workspace_bytes(const Shape &s)
+{
+    if (s.T == 0) return 256;
+    return input_scratch(s, nullptr).bytes;
+}
+
+cudaError_t launch_backward_input(const Ctx &c, const bf16 *dout, float *d_hidden, uint8_t *bws)
+{
+    const Shape &s = c.s;
+    const int R = s.T * s.k, H = s.H, E = s.E();
+    const InScratch b = input_scratch(s, bws);
+    cudaStream_t st = c.stream;
+
+    // routed experts: the upstream gradient of every dispatch row, then Z,
+    // [dG | dU] (and dL/dw partials) and dA over all E experts
+    launch_gather_rows(dout, c.tok_of_slot, c.offsets, 0, E, R, H, b.dout_rows, c.num_sms, st);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    const RowsGroups g{0, E, 0, b.rp};
+    if ((err = launch_rows_z(c, g, b.dout_rows, (uint64_t)R + 64, 1, b.zpad)) != cudaSuccess) return err;
+    if ((err = launch_rows_gu(c, g, c.a_perm, (uint64_t)R, b.zpad, b.dgu, nullptr, b.gw_part)) != cudaSuccess)
+        return err;
+    if ((err = launch_rows_da(c, g, b.dgu, b.da)) != cudaSuccess) return err;
+    // shared experts: every token's own row, weight 1
+    if (s.E_sh > 0) {
+        const RowsGroups gs{0, s.E_sh, s.T, b.rp_sh};
+        if ((err = launch_rows_z(c, gs, dout, (uint64_t)s.T, 0, b.zpad_sh)) != cudaSuccess) return err;
+        if ((err = launch_rows_gu(c, gs, c.hidden, (uint64_t)s.T, b.zpad_sh, b.dgu_sh, nullptr, nullptr)) !=
+            cudaSuccess)
+            return err;
+        if ((err = launch_rows_da(c, gs, b.dgu_sh, b.da_sh)) != cudaSuccess) return err;
+    }
+    // the router of each token's pool
+    const int ld = std::max(s.E_pub, s.E_priv);
+    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz)) != cudaSuccess) return err;
+    return launch_pdl(bwd_input_reduce_kernel, dim3(std::min(s.T, c.num_sms * 8)), dim3(256), 0, st,
+                      (const bf16 *)b.da, (const bf16 *)b.da_sh, (const float *)b.dz, ld, c.router_pub,
+                      c.router_priv, (const uint8_t *)c.tau, (const int32_t *)c.idx, (const int32_t *)c.slot_of,
+                      (const uint32_t *)c.offsets, s.T, H, s.E_pub, s.E_priv, s.E_sh, s.k, R, s.renorm, b.tp,
+                      d_hidden);
+}
+
+}  // namespace pmpe

@@ -4,7 +4,7 @@
 // TMA -> shared memory -> tcgen05.mma -> TMEM -> epilogue pipeline of the
 // forward's expert GEMMs:
 //
-//   bwd_rows_tc_kernel<kRowsZ>    rows of an expert as M, K = H:
+//   bwd_rows_tc_kernel<kRowsMN>   rows of an expert as M, K = H:
 //     Z = D W_down                  (D: the rows' upstream gradients; W_down read
 //                                    MN-major; so dL/da = w Z) -> BF16
 //   bwd_rows_tc_kernel<kRowsGU>   rows of an expert as M, K = H:
@@ -21,6 +21,10 @@
 //   both operands MN-major, read as stored (no transpose in memory); the zero
 //   rows of the padded operand cancel what the other operand holds past the
 //   expert's rows.  FP32 outputs.
+//
+// The same two row kernels, over all routed experts and the shared experts,
+// and an MN-mode launch dA = [dG | dU] [W_gate; W_up] give the gradient of
+// the layer's input (launch_backward_input_gemms).
 //
 // Every launch keeps four 48 KB operand stages in flight (a 128 x 256 x 64 MMA
 // block each) and two 128 x 256 FP32 accumulators, so the epilogue of one tile
@@ -59,25 +63,33 @@ constexpr int kDynSmem = kStages * kStageBytes + 4 * kOutBufs * kOutBoxBytes + 1
 constexpr int kAccCols = 256;
 constexpr int kTmemCols = 2 * kAccCols;
 
-// Per private expert q: its rows, first row relative to the first private
-// slot, first row of the padded layout; and the tiles of the experts before q.
+// Groups of a launch: the routed experts g0 .. g0 + G - 1 (rows = their
+// dispatch slots), or G shared experts that each run every one of shared_T
+// tokens.  Per group q: its rows, its first row relative to the first slot of
+// expert g0 (0 for shared groups), its first row of the padded layout; and the
+// tiles of the groups before q.
+constexpr int kMaxGroups = 2 * kMaxPool;
 struct GroupTable {
-    int tiles[kMaxPool + 1];
-    int rows[kMaxPool];
-    int off[kMaxPool];
-    int pad[kMaxPool];
+    int tiles[kMaxGroups + 1];
+    int rows[kMaxGroups];
+    int off[kMaxGroups];
+    int pad[kMaxGroups];
 };
 
-// All threads: fill the table from the forward's dispatch offsets.
-// tiles_per_row_block: tiles of an expert per 128-row block (0: every expert
-// has `fixed_tiles` tiles whatever its rows).
-__device__ void build_groups(GroupTable &gt, const uint32_t *offsets, int E_pub, int E_priv, int R,
+// All threads: fill the table (routed groups from the forward's dispatch
+// offsets).  tiles_per_row_block: tiles of a group per 128-row block (0:
+// every group has `fixed_tiles` tiles whatever its rows).
+__device__ void build_groups(GroupTable &gt, const uint32_t *offsets, int g0, int G, int R, int shared_T,
                              int tiles_per_row_block, int fixed_tiles)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int p0 = (int)min(offsets[E_pub], (uint32_t)R);
-    for (int q = tid; q < E_priv; q += blockDim.x) {
-        const int b = min(max((int)offsets[E_pub + q], p0), R), e = min(max((int)offsets[E_pub + q + 1], b), R);
+    const int p0 = shared_T ? 0 : (int)min(offsets[g0], (uint32_t)R);
+    for (int q = tid; q < G; q += blockDim.x) {
+        int b = 0, e = shared_T;
+        if (!shared_T) {
+            b = min(max((int)offsets[g0 + q], p0), R);
+            e = min(max((int)offsets[g0 + q + 1], b), R);
+        }
         const int rows = e - b;
         gt.rows[q] = rows;
         gt.off[q] = b - p0;
@@ -87,16 +99,16 @@ __device__ void build_groups(GroupTable &gt, const uint32_t *offsets, int E_pub,
     __syncthreads();
     if (warp < 2) {  // warp 0: inclusive scan of tiles; warp 1: exclusive scan of padded rows
         int carry = 0;
-        for (int b = 0; b < E_priv; b += 32) {
+        for (int b = 0; b < G; b += 32) {
             const int q = b + lane;
-            const int v = q < E_priv ? (warp == 0 ? gt.tiles[q + 1] : gt.pad[q]) : 0;
+            const int v = q < G ? (warp == 0 ? gt.tiles[q + 1] : gt.pad[q]) : 0;
             int x = v;
 #pragma unroll
             for (int off = 1; off < 32; off <<= 1) {
                 const int y = __shfl_up_sync(~0u, x, off);
                 if (lane >= off) x += y;
             }
-            if (q < E_priv) {
+            if (q < G) {
                 if (warp == 0) gt.tiles[q + 1] = carry + x;
                 else gt.pad[q] = carry + x - v;
             }
@@ -155,33 +167,45 @@ __device__ __forceinline__ void drain_stages(uint32_t bar0, int stages, uint32_t
 
 // ------------------------------------------------------------- rows
 
-enum { kRowsZ = 0, kRowsGU = 1 };
+enum { kRowsMN = 0, kRowsGU = 1 };
+enum { kArowsTight = 0, kArowsSlot = 1, kArowsPad = 2 };
 
+// One launch of the row GEMMs.  Mode kRowsMN: C = A B with A K-major rows
+// (K = K) and B read MN-major from a weight tensor of the group's expert
+// (K blocks below k_split from b0, the rest from b1; kb_rows rows of K per
+// expert in those tensors), C -> BF16 [padded rows][N].  Mode kRowsGU: the
+// gate/up recompute (K = H) and the SwiGLU backward epilogue.
 struct RowsParams {
-    int E_pub, E_priv, H, I, R;
-    int bn;           // output columns per tile (Z: of I, 256 or 128; gate/up: 128 activation columns)
+    int E_pub, H, I, R;
+    int g0, G, shared_T;  // the groups (see build_groups)
+    int K, N, bn;         // contracted size, output columns, output columns per tile
+    int kb_rows, k_split; // MN mode: K rows of B per expert; first K block taken from b1
+    int a_rows;           // A row of a tile row: kArowsTight (relative to expert g0's first slot),
+                          // kArowsSlot (the dispatch slot; the token for shared groups), kArowsPad
     const uint32_t *offsets;
-    const float *w_of_slot;
-    const bf16 *zpad;  // gate/up: Z in the padded row layout [RP][I]
-    float *gw_part;    // gate/up: [R][I / 128] dL/dw partial of each private row per 128-column tile
+    const float *w_of_slot;  // gate/up: routing weights per slot (shared groups: weight 1)
+    const bf16 *zpad;     // gate/up: Z in the padded row layout [RP][I]
+    float *gw_part;       // gate/up (routed, may be null): [R][I / 128] dL/dw partial per 128-column tile
+    int wact;             // gate/up: 1 to write w act to out1
     uint32_t *status;
     uint32_t idesc;
 };
 
 struct RowsMaps {
-    CUtensorMap a;       // Z: dout rows [R + 64][H]; gate/up: A rows [R][H]; 64 x 128 box (K-major)
-    CUtensorMap b0, b1;  // Z: W_down [E_priv H][I], 64 x 64 x bn/128 3-D box (MN-major); gate/up: gate, up, 64 x 128
-    CUtensorMap out0;    // Z: Z [RP][I]; gate/up: [dG | dU] [RP][2I]  (32 x 32 BF16 boxes, 64-byte swizzle)
-    CUtensorMap out1;    // gate/up: w act [RP][I]
+    CUtensorMap a;           // A rows, 64 x 128 box (K-major)
+    CUtensorMap b0[2], b1[2];  // per weight pool (public, private; shared groups use [0]): MN mode:
+                             // 64 x 64 x bn/128 3-D boxes (MN-major); gate/up: gate, up, 64 x 128 (K-major)
+    CUtensorMap out0;        // MN: C [RP][N]; gate/up: [dG | dU] [RP][2I]  (32 x 32 BF16 boxes, 64-byte swizzle)
+    CUtensorMap out1;        // gate/up: w act [RP][I]
 };
 
 struct RowsTile {
     int q, m0, n0, n_tile, rows;
 };
 
-__device__ __forceinline__ RowsTile decode_rows(const GroupTable &gt, int E_priv, int nt, int bn, int tile)
+__device__ __forceinline__ RowsTile decode_rows(const GroupTable &gt, int G, int nt, int bn, int tile)
 {
-    int lo = 0, hi = E_priv - 1;  // last expert whose tile prefix is <= tile (skips empty experts)
+    int lo = 0, hi = G - 1;  // last group whose tile prefix is <= tile (skips empty groups)
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
         if (gt.tiles[mid] <= tile) lo = mid; else hi = mid - 1;
@@ -190,12 +214,20 @@ __device__ __forceinline__ RowsTile decode_rows(const GroupTable &gt, int E_priv
     t.q = lo;
     const int mt = (gt.rows[lo] + BM - 1) / BM;
     const int local = tile - gt.tiles[lo];
-    t.n_tile = local / mt;  // n-tile major inside an expert: its m tiles share the weight slice
+    t.n_tile = local / mt;  // n-tile major inside a group: its m tiles share the weight slice
     const int m_tile = local - t.n_tile * mt;
     t.m0 = m_tile * BM;
     t.n0 = t.n_tile * bn;
     t.rows = min(BM, gt.rows[lo] - t.m0);
     return t;
+}
+
+// Weight pool (0 public or shared, 1 private) and index inside it of group q.
+__device__ __forceinline__ int2 group_weights(const RowsParams &p, int q)
+{
+    if (p.shared_T) return make_int2(0, q);
+    const int e = p.g0 + q;
+    return e >= p.E_pub ? make_int2(1, e - p.E_pub) : make_int2(0, e);
 }
 
 template <int kMode>
@@ -225,27 +257,28 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
     }
     if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
     pdl_wait();
-    const int nt = p.I / p.bn;
-    build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, nt, 0);
+    const int nt = p.N / p.bn;
+    build_groups(gt, p.offsets, p.g0, p.G, p.R, p.shared_T, nt, 0);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
-    const int total = gt.tiles[p.E_priv];
-    const int nkb = p.H / BK;
-    const int p0 = (int)min(p.offsets[p.E_pub], (uint32_t)p.R);
+    const int total = gt.tiles[p.G];
+    const int nkb = p.K / BK;
+    const int p0 = p.shared_T ? 0 : (int)min(p.offsets[p.g0], (uint32_t)p.R);
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
         // lane 0: the tile's 128 rows x 64 K of A (16 KB).  Gate/up: lane 1 the
-        // 128 gate rows, lane 2 the 128 up rows (16 KB each).  Z: lanes 1-2 half
-        // of the bn / 64 MN blocks of W_down each, as one 3-D box (8 KB per block).
+        // 128 gate rows, lane 2 the 128 up rows (16 KB each).  MN mode: lanes 1-2
+        // half of the bn / 64 MN blocks of B each, as one 3-D box (8 KB per block).
         int stage = 0;
         uint32_t phase = 0, filled = 0, last_parity = 0;
-        const int half = p.bn / 128;  // Z: MN blocks per loader lane
+        const int half = p.bn / 128;  // MN mode: MN blocks per loader lane
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
-            const RowsTile t = decode_rows(gt, p.E_priv, nt, p.bn, tile);
-            const int arow = (kMode == kRowsGU ? p0 : 0) + gt.off[t.q] + t.m0;
+            const RowsTile t = decode_rows(gt, p.G, nt, p.bn, tile);
+            const int2 wq = group_weights(p, t.q);
+            const int arow = (p.a_rows == kArowsPad ? gt.pad[t.q] : (p.a_rows == kArowsSlot ? p0 : 0) + gt.off[t.q]) + t.m0;
             bool ok = true;
             for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status)) { ok = false; break; }
@@ -256,12 +289,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
                     tma_load_2d(sA, &maps.a, full_bar(stage), kx, arow);
                 } else if (kMode == kRowsGU) {
                     mbar_expect_tx(full_bar(stage), kABytes);
-                    tma_load_2d(sB + (lane - 1) * kABytes, lane == 1 ? &maps.b0 : &maps.b1, full_bar(stage), kx,
-                                t.q * p.I + t.n0);
+                    tma_load_2d(sB + (lane - 1) * kABytes, lane == 1 ? &maps.b0[wq.x] : &maps.b1[wq.x], full_bar(stage),
+                                kx, wq.y * p.I + t.n0);
                 } else {
                     const int b0 = (lane - 1) * half;
+                    const bool second = kb >= p.k_split;
+                    const int krow = wq.y * p.kb_rows + (second ? kx - p.k_split * BK : kx);
                     mbar_expect_tx(full_bar(stage), (uint32_t)(half * kMnBlockBytes));
-                    tma_load_3d(sB + b0 * kMnBlockBytes, &maps.b0, full_bar(stage), 0, t.q * p.H + kx, t.n0 / 64 + b0);
+                    tma_load_3d(sB + b0 * kMnBlockBytes, second ? &maps.b1[wq.x] : &maps.b0[wq.x], full_bar(stage), 0,
+                                krow, t.n0 / 64 + b0);
                 }
                 filled |= 1u << stage;
                 last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
@@ -312,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
         OutStager out{sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * kOutBufs * kOutBoxBytes), 0};
         int it = 0;
         for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
-            const RowsTile t = decode_rows(gt, p.E_priv, nt, p.bn, tile);
+            const RowsTile t = decode_rows(gt, p.G, nt, p.bn, tile);
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
             int ok = 1;
@@ -325,7 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
             const bool valid = r < t.rows;
             const int orow = gt.pad[t.q] + t.m0 + quarter * 32;  // this warp's 32 rows in the padded layout
             const uint32_t tb = tmem_base + (uint32_t)(buf * kAccCols) + ((uint32_t)(quarter * 32) << 16);
-            if (kMode == kRowsZ) {
+            if (kMode == kRowsMN) {
 #pragma unroll 1
                 for (int c = 0; c < p.bn / 32; ++c) {
                     float v[32];
@@ -337,8 +373,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
                     out.put(lane, pk, &maps.out0, t.n0 + c * 32, orow);
                 }
             } else {
-                const int prow = gt.off[t.q] + t.m0 + r;  // private row (relative to the first private slot)
-                const float w = valid ? p.w_of_slot[p0 + prow] : 0.f;
+                const int prow = gt.off[t.q] + t.m0 + r;  // row relative to expert g0's first slot (shared: token)
+                const float w = valid ? (p.shared_T ? 1.f : p.w_of_slot[p0 + prow]) : 0.f;
                 const uint4 *zrow = reinterpret_cast<const uint4 *>(p.zpad + (size_t)(orow + lane) * p.I + t.n0);
                 float gw = 0.f;
 #pragma unroll 1
@@ -376,9 +412,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
                     }
                     out.put(lane, pg, &maps.out0, t.n0 + c * 32, orow);
                     out.put(lane, pu, &maps.out0, p.I + t.n0 + c * 32, orow);
-                    out.put(lane, pa, &maps.out1, t.n0 + c * 32, orow);
+                    if (p.wact) out.put(lane, pa, &maps.out1, t.n0 + c * 32, orow);
                 }
-                if (valid) p.gw_part[(size_t)prow * nt + t.n_tile] = gw;
+                if (valid && p.gw_part) p.gw_part[(size_t)(p0 + prow) * nt + t.n_tile] = gw;
             }
             tc_fence_before();
             __syncwarp();
@@ -471,7 +507,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
     }
     if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
     pdl_wait();
-    build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, 0, 0);
+    build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, 0, 0, 0);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -606,48 +642,123 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
 // Rows of the padded layout (an upper bound over all routings).
 size_t backward_padded_rows(const Shape &s) { return (size_t)s.T * s.k + (size_t)kPad * s.E_priv; }
 
+namespace {
+
+// Fields shared by every row launch over the groups `g`.
+RowsParams rows_params(const Ctx &c, const RowsGroups &g)
+{
+    const Shape &s = c.s;
+    RowsParams p;
+    memset(&p, 0, sizeof(p));
+    p.E_pub = s.E_pub; p.H = s.H; p.I = s.I; p.R = s.T * s.k;
+    p.g0 = g.g0; p.G = g.G; p.shared_T = g.shared_T;
+    p.offsets = c.offsets;
+    p.w_of_slot = c.w_of_slot;
+    p.status = c.audit.status;
+    return p;
+}
+
+// The weight tensor of pool q (0 public, 1 private) for routed groups, or the
+// shared one, with its rows: experts x rows_per_expert.
+const bf16 *pool_tensor(const Ctx &c, const RowsGroups &g, const bf16 *const *w, int q, int rows_per_expert,
+                        uint64_t *rows)
+{
+    const Shape &s = c.s;
+    const int n = g.shared_T ? s.E_sh : (q ? s.E_priv : s.E_pub);
+    *rows = (uint64_t)n * rows_per_expert;
+    return g.shared_T ? w[2] : w[q];
+}
+
+cudaError_t run_rows(int mode, const Ctx &c, const RowsParams &p, const RowsMaps &maps)
+{
+    static std::atomic<int> smem_limit[2][64];
+    auto kernel = mode == kRowsMN ? bwd_rows_tc_kernel<kRowsMN> : bwd_rows_tc_kernel<kRowsGU>;
+    cudaError_t err = ensure_dynamic_smem(kernel, kDynSmem, smem_limit[mode]);
+    if (err != cudaSuccess) return err;
+    return launch_pdl(kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
+}
+
+}  // namespace
+
+cudaError_t launch_rows_z(const Ctx &c, const RowsGroups &g, const bf16 *d, uint64_t d_rows, int tight, bf16 *zpad)
+{
+    const Shape &s = c.s;
+    RowsParams p = rows_params(c, g);
+    RowsMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    p.K = s.H; p.N = s.I; p.bn = s.I % 256 == 0 ? 256 : 128;
+    p.kb_rows = s.H; p.k_split = s.H / BK;
+    p.a_rows = tight ? kArowsTight : kArowsSlot;
+    p.idesc = make_idesc_major(BM, p.bn, false, true);
+    bool ok = encode_2d(&maps.a, d, s.H, d_rows, BM);
+    for (int q = 0; q < (g.shared_T ? 1 : 2); ++q) {
+        uint64_t rows;
+        const bf16 *w = pool_tensor(c, g, c.down, q, s.H, &rows);
+        ok &= encode_3d_blocks(&maps.b0[q], w, s.I, rows, 64, p.bn / 128);
+    }
+    ok &= encode_2d_box(&maps.out0, zpad, s.I, g.padded_rows, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+    if (!ok) return cudaErrorInvalidValue;
+    return run_rows(kRowsMN, c, p, maps);
+}
+
+cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uint64_t a_rows, const bf16 *zpad,
+                           bf16 *dgu, bf16 *wact, float *gw_part)
+{
+    const Shape &s = c.s;
+    RowsParams p = rows_params(c, g);
+    RowsMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    p.K = s.H; p.N = s.I; p.bn = 128;
+    p.a_rows = kArowsSlot;
+    p.zpad = zpad;
+    p.gw_part = gw_part;
+    p.wact = wact ? 1 : 0;
+    p.idesc = make_idesc(BM, 256);
+    bool ok = encode_2d(&maps.a, a, s.H, a_rows, BM);
+    for (int q = 0; q < (g.shared_T ? 1 : 2); ++q) {
+        uint64_t rows;
+        const bf16 *wg = pool_tensor(c, g, c.gate, q, s.I, &rows);
+        const bf16 *wu = pool_tensor(c, g, c.up, q, s.I, &rows);
+        ok &= encode_2d(&maps.b0[q], wg, s.H, rows, 128);
+        ok &= encode_2d(&maps.b1[q], wu, s.H, rows, 128);
+    }
+    ok &= encode_2d_box(&maps.out0, dgu, 2 * (uint64_t)s.I, g.padded_rows, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+    if (wact) ok &= encode_2d_box(&maps.out1, wact, s.I, g.padded_rows, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+    if (!ok) return cudaErrorInvalidValue;
+    return run_rows(kRowsGU, c, p, maps);
+}
+
+cudaError_t launch_rows_da(const Ctx &c, const RowsGroups &g, const bf16 *dgu, bf16 *da)
+{
+    const Shape &s = c.s;
+    RowsParams p = rows_params(c, g);
+    RowsMaps maps;
+    memset(&maps, 0, sizeof(maps));
+    p.K = 2 * s.I; p.N = s.H; p.bn = s.H % 256 == 0 ? 256 : 128;
+    p.kb_rows = s.I; p.k_split = s.I / BK;  // K blocks of dG take W_gate, those of dU take W_up
+    p.a_rows = kArowsPad;
+    p.idesc = make_idesc_major(BM, p.bn, false, true);
+    bool ok = encode_2d(&maps.a, dgu, 2 * (uint64_t)s.I, g.padded_rows, BM);
+    for (int q = 0; q < (g.shared_T ? 1 : 2); ++q) {
+        uint64_t rows;
+        const bf16 *wg = pool_tensor(c, g, c.gate, q, s.I, &rows);
+        const bf16 *wu = pool_tensor(c, g, c.up, q, s.I, &rows);
+        ok &= encode_3d_blocks(&maps.b0[q], wg, s.H, rows, 64, p.bn / 128);
+        ok &= encode_3d_blocks(&maps.b1[q], wu, s.H, rows, 64, p.bn / 128);
+    }
+    ok &= encode_2d_box(&maps.out0, da, s.H, g.padded_rows, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+    if (!ok) return cudaErrorInvalidValue;
+    return run_rows(kRowsMN, c, p, maps);
+}
+
 cudaError_t launch_backward_rows(const Ctx &c, const bf16 *dout_rows, bf16 *zpad, bf16 *dgu, bf16 *wact,
                                  float *gw_part)
 {
     const Shape &s = c.s;
-    const uint64_t R = (uint64_t)s.T * s.k, RP = backward_padded_rows(s);
-    static std::atomic<int> smem_limit[2][64];
-    cudaError_t err;
-    for (int mode = 0; mode < 2; ++mode) {
-        RowsParams p;
-        RowsMaps maps;
-        memset(&p, 0, sizeof(p));
-        memset(&maps, 0, sizeof(maps));
-        p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.H = s.H; p.I = s.I; p.R = (int)R;
-        p.offsets = c.offsets;
-        p.w_of_slot = c.w_of_slot;
-        p.zpad = zpad;
-        p.gw_part = gw_part;
-        p.status = c.audit.status;
-        bool ok;
-        if (mode == kRowsZ) {
-            p.bn = s.I % 256 == 0 ? 256 : 128;
-            p.idesc = make_idesc_major(BM, p.bn, false, true);
-            ok = encode_2d(&maps.a, dout_rows, s.H, R + 64, BM);
-            ok &= encode_3d_blocks(&maps.b0, c.down[1], s.I, (uint64_t)s.E_priv * s.H, 64, p.bn / 128);
-            ok &= encode_2d_box(&maps.out0, zpad, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
-        } else {
-            p.bn = 128;
-            p.idesc = make_idesc(BM, 256);
-            ok = encode_2d(&maps.a, c.a_perm, s.H, R, BM);
-            ok &= encode_2d(&maps.b0, c.gate[1], s.H, (uint64_t)s.E_priv * s.I, 128);
-            ok &= encode_2d(&maps.b1, c.up[1], s.H, (uint64_t)s.E_priv * s.I, 128);
-            ok &= encode_2d_box(&maps.out0, dgu, 2 * (uint64_t)s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
-            ok &= encode_2d_box(&maps.out1, wact, s.I, RP, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
-        }
-        if (!ok) return cudaErrorInvalidValue;
-        auto kernel = mode == kRowsZ ? bwd_rows_tc_kernel<kRowsZ> : bwd_rows_tc_kernel<kRowsGU>;
-        err = ensure_dynamic_smem(kernel, kDynSmem, smem_limit[mode]);
-        if (err != cudaSuccess) return err;
-        err = launch_pdl(kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
-        if (err != cudaSuccess) return err;
-    }
-    return cudaSuccess;
+    const RowsGroups g{s.E_pub, s.E_priv, 0, backward_padded_rows(s)};
+    cudaError_t err = launch_rows_z(c, g, dout_rows, (uint64_t)s.T * s.k + 64, 1, zpad);
+    if (err != cudaSuccess) return err;
+    return launch_rows_gu(c, g, c.a_perm, (uint64_t)s.T * s.k, zpad, dgu, wact, gw_part);
 }
 
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,

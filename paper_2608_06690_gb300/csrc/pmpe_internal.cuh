@@ -82,11 +82,35 @@ cudaError_t launch_down(const Ctx &c);
 size_t backward_workspace_bytes(const Shape &s);
 cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_router, float *d_gate, float *d_up,
                                     float *d_down, uint8_t *bws);
+// Its pieces shared with the input gradient: the upstream gradients of the
+// dispatch rows of experts g0 .. g1 - 1 (and 64 zero rows after them); the
+// router's softmax gradient from the dL/dw partials per slot (both_pools = 0:
+// the private pool, zero for DENY tokens; 1: each token's own pool), dz [T][ld].
+void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint32_t *offsets, int g0, int g1, int R,
+                        int H, bf16 *rows, int num_sms, cudaStream_t st);
+cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz);
+// Gradient of the layer's input (k_backward_input.cu): scratch bytes and launch.
+size_t backward_input_workspace_bytes(const Shape &s);
+cudaError_t launch_backward_input(const Ctx &c, const bf16 *dout, float *d_hidden, uint8_t *bws);
 // Its tensor-core GEMMs (k_backward_tc.cu): rows of the padded layout, the
 // dL/da and gate/up recompute launches, and the weight-gradient launch.
 size_t backward_padded_rows(const Shape &s);
 cudaError_t launch_backward_rows(const Ctx &c, const bf16 *dout_rows, bf16 *zpad, bf16 *dgu, bf16 *wact,
                                  float *gw_part);
+// The groups of one row launch: routed experts g0 .. g0 + G - 1 (shared_T = 0)
+// or the G = E_sh shared experts over shared_T tokens; padded_rows bounds the
+// padded row layout of their outputs (each group's rows rounded up to 128).
+struct RowsGroups {
+    int g0, G, shared_T;
+    uint64_t padded_rows;
+};
+// Z = D W_down (D rows: tight = relative to expert g0's first slot, else the
+// slot or token) -> zpad; the gate/up recompute with the SwiGLU backward ->
+// [dG | dU] (and w act, dL/dw partials when non-null); dA = [dG | dU] [W_gate; W_up].
+cudaError_t launch_rows_z(const Ctx &c, const RowsGroups &g, const bf16 *d, uint64_t d_rows, int tight, bf16 *zpad);
+cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uint64_t a_rows, const bf16 *zpad,
+                           bf16 *dgu, bf16 *wact, float *gw_part);
+cudaError_t launch_rows_da(const Ctx &c, const RowsGroups &g, const bf16 *dgu, bf16 *da);
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
                                   float *d_gate, float *d_up, float *d_down);
 // Gate/up and down in one persistent launch (down tiles wait for their

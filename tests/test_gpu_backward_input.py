@@ -1,0 +1,137 @@
+"""GPU parity of the gradient of the layer's input (through the frozen layer,
+Sec. 3.2: what the layer below needs when its private branch is trained)
+against the oracle's backward_input, through the C ABI, on seeded inputs:
+both pools (Eq. 1), renormalised top-k and pool softmax (Eq. 2), shared
+experts, ragged expert row counts over several 128-row tiles, experts without
+rows, H and I that take the 128- and the 256-column tiles, the largest pools,
+the all-DENY, all-ALLOW and empty batches."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_06690_gb300 import pmpe
+from paper_2608_06690_gb300.inputs import LayerShape
+from pmpe_testlib import GAP_EPS, make_layer, oracle_layer, to_device
+
+pytestmark = pytest.mark.gpu
+
+# Tolerance on d_hidden: max-abs error <= 2e-2 * max|ref| and
+# sum|err| / sum|ref| <= 1e-2.  The GPU contracts BF16 operands with FP32
+# accumulation, rounds dG, dU (2^-9 relative each) and every pick's input
+# gradient dA to BF16, and sums the picks in FP32.
+MAX_ABS_REL = 2e-2
+MEAN_REL = 1e-2
+
+CASES = {
+    "renorm_ragged": (LayerShape(T=300, H=384, I=256, E_pub=24, E_priv=8, E_sh=0, k=4, renormalize=True), 61,
+                      "iid"),
+    "pool_softmax_with_shared": (LayerShape(T=200, H=256, I=256, E_pub=16, E_priv=8, E_sh=2, k=3,
+                                            renormalize=False), 62, "iid"),
+    "all_allow_multi_tile": (LayerShape(T=500, H=256, I=128, E_pub=8, E_priv=4, E_sh=0, k=2, renormalize=True),
+                             63, "allow"),
+    "all_deny_shared": (LayerShape(T=260, H=256, I=128, E_pub=8, E_priv=4, E_sh=1, k=2, renormalize=True), 64,
+                        "deny"),
+    "sparse_pool_empty_experts": (LayerShape(T=90, H=128, I=128, E_pub=8, E_priv=64, E_sh=0, k=2,
+                                             renormalize=True), 65, "iid"),
+    "k12_pool_softmax": (LayerShape(T=150, H=256, I=128, E_pub=40, E_priv=16, E_sh=0, k=12, renormalize=False), 66,
+                         "iid"),
+    "k1": (LayerShape(T=100, H=128, I=128, E_pub=12, E_priv=5, E_sh=0, k=1, renormalize=True), 67, "iid"),
+    "single_token": (LayerShape(T=1, H=256, I=128, E_pub=8, E_priv=4, E_sh=1, k=2, renormalize=False), 68, "allow"),
+    # 256 + 256 experts: the largest group table of one launch
+    "largest_pools": (LayerShape(T=700, H=128, I=128, E_pub=256, E_priv=256, E_sh=1, k=4, renormalize=False), 69,
+                      "iid"),
+}
+
+
+def _dout(shape: LayerShape, seed: int) -> torch.Tensor:
+    g = torch.Generator().manual_seed(seed)
+    return torch.randn((shape.T, shape.H), generator=g).to(torch.bfloat16)
+
+
+def _gpu_input_grad(shape, w, h, pol, dout):
+    wd, hd, pd = to_device(w, h, pol)
+    layer = pmpe.MoeLayer(shape, wd)
+    idx = torch.empty((shape.T, shape.k), dtype=torch.int32, device="cuda")
+    wt = torch.empty((shape.T, shape.k), dtype=torch.float32, device="cuda")
+    layer.forward(hd, pd, topk_idx=idx, topk_w=wt)
+    dh = layer.backward_input(hd, pd, dout.cuda().contiguous(), topk_idx=idx, topk_w=wt)
+    torch.cuda.synchronize()
+    return dh.cpu().numpy().astype(np.float64), idx.cpu().numpy(), layer, (wd, hd, pd)
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_backward_input_parity_with_oracle(name):
+    shape, seed, policy = CASES[name]
+    w, h, pol = make_layer(shape, seed, policy=policy)
+    L = oracle_layer(shape, w, h, pol)
+    oidx, _, gap = oracle.route(L)
+    dout = _dout(shape, seed)
+    # a token at a routing near-tie may take another k-th expert on the GPU;
+    # its input gradient is linear in its own dout row, so that row is zeroed
+    # on both sides (and its gradient is then exactly zero)
+    near = gap < GAP_EPS
+    dout[torch.from_numpy(near)] = 0
+    got, gidx, _, _ = _gpu_input_grad(shape, w, h, pol, dout)
+    ok = ~near
+    assert np.array_equal(gidx[ok], oidx[ok])
+    ref = oracle.backward_input(L, dout.double().numpy())
+    assert got.shape == (shape.T, shape.H) and np.all(np.isfinite(got))
+    assert np.all(got[near] == 0.0)
+    err = np.abs(got - ref)
+    mx = float(err.max() / np.abs(ref).max())
+    mean = float(err.sum() / np.abs(ref).sum())
+    assert mx <= MAX_ABS_REL and mean <= MEAN_REL, (mx, mean)
+    # every token with a nonzero upstream gradient gets a nonzero input gradient
+    assert np.all(np.abs(got[ok]).max(1) > 0)
+
+
+def test_backward_input_empty_batch():
+    shape = LayerShape(T=0, H=256, I=128, E_pub=16, E_priv=8, E_sh=1, k=2, renormalize=True)
+    w, h, pol = make_layer(shape, 70, policy="iid")
+    got, _, _, _ = _gpu_input_grad(shape, w, h, pol, _dout(shape, 70))
+    assert got.shape == (0, 256)
+
+
+def test_backward_input_deny_tokens_never_see_private_weights_and_is_deterministic():
+    """G2 through the input gradient: a DENY token's gradient passes through
+    the public router and experts and the shared experts only, so replacing
+    every private weight leaves the DENY rows of d_hidden bitwise unchanged;
+    a second run is bitwise identical (no atomics)."""
+    shape, seed, _ = CASES["pool_softmax_with_shared"]
+    w, h, pol = make_layer(shape, seed, policy="iid")
+    tau = oracle.resolve(pol.numpy(), shape.T)
+    assert 0 < tau.sum() < shape.T
+    dout = _dout(shape, 3)
+    g1, _, layer, (wd, hd, pd) = _gpu_input_grad(shape, w, h, pol, dout)
+    layer.forward(hd, pd)
+    g2 = layer.backward_input(hd, pd, dout.cuda()).cpu().numpy().astype(np.float64)
+    assert np.array_equal(g1, g2)
+    w_other, _, _ = make_layer(shape, seed + 1000, policy="iid")
+    w_mixed = dict(w)
+    for n in ("router_priv", "gate_priv", "up_priv", "down_priv"):
+        w_mixed[n] = w_other[n]
+    g3, _, _, _ = _gpu_input_grad(shape, w_mixed, h, pol, dout)
+    deny = tau == 0
+    assert np.array_equal(g1[deny], g3[deny])
+    assert not np.array_equal(g1[~deny], g3[~deny])
+
+
+def test_backward_input_leaves_the_private_backward_unchanged():
+    """The input gradient and the private-parameter backward share the row
+    GEMM launches' scratch layout; running one between a forward and the
+    other gives the other's result bitwise."""
+    shape, seed, _ = CASES["renorm_ragged"]
+    w, h, pol = make_layer(shape, seed, policy="iid")
+    wd, hd, pd = to_device(w, h, pol)
+    layer = pmpe.MoeLayer(shape, wd)
+    dout = _dout(shape, 5).cuda()
+    layer.forward(hd, pd)
+    a = {n: v.clone() for n, v in layer.backward_private(hd, pd, dout).items()}
+    dh1 = layer.backward_input(hd, pd, dout).clone()
+    b = layer.backward_private(hd, pd, dout)
+    dh2 = layer.backward_input(hd, pd, dout)
+    torch.cuda.synchronize()
+    for n in a:
+        assert torch.equal(a[n], b[n]), n
+    assert torch.equal(dh1, dh2)
