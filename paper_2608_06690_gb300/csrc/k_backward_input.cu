@@ -68,17 +68,31 @@ __global__ void __launch_bounds__(256) bwd_input_reduce_kernel(
     }
 
     const int nv = H / 8;
+    __shared__ int s_row[kMaxTopK];      // padded dA row of each pick (-1: none)
+    __shared__ int s_pe[kMaxTopK];       // router row of each pick in the token's pool (-1: none)
+    __shared__ float s_dz[kMaxTopK];
     for (int t = blockIdx.x; t < T; t += gridDim.x) {
         const int priv = tau[t] ? 1 : 0;
         const int e_base = priv ? E_pub : 0, E_pool = priv ? E_priv : E_pub;
         const bf16 *router = priv ? router_priv : router_pub;
         const float *dzt = dz + (size_t)t * ld;
+        __syncthreads();  // the previous token's picks are consumed
+        if (tid < k) {
+            const int e = idx[(size_t)t * k + tid];
+            const int slot = slot_of[(size_t)t * k + tid];
+            const bool ok = e >= 0 && e < E && slot >= 0 && slot < R;
+            s_row[tid] = ok ? pad_start[e] + slot - (int)offsets[e] : -1;
+            const int pe = e - e_base;
+            const bool in_pool = pe >= 0 && pe < E_pool;
+            s_pe[tid] = in_pool ? pe : -1;
+            s_dz[tid] = in_pool ? dzt[pe] : 0.f;
+        }
+        __syncthreads();
         for (int c = tid; c < nv; c += blockDim.x) {
             float acc[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-            auto add_row = [&](const bf16 *row, float scale) {
-                const uint4 v = reinterpret_cast<const uint4 *>(row)[c];
+            auto add = [&](const uint4 &v, float scale) {
                 const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
@@ -87,25 +101,40 @@ __global__ void __launch_bounds__(256) bwd_input_reduce_kernel(
                     acc[2 * i + 1] += scale * f.y;
                 }
             };
-            for (int j = 0; j < k; ++j) {
-                const int e = idx[(size_t)t * k + j];
-                const int slot = slot_of[(size_t)t * k + j];
-                if (e < 0 || e >= E || slot < 0 || slot >= R) continue;
-                const int prow = pad_start[e] + slot - (int)offsets[e];
-                add_row(da + (size_t)prow * H, 1.f);
+            // the picks' rows are requested 8 at a time before they are summed
+            constexpr int kBatch = 8;
+            uint4 v[kBatch];
+            for (int j0 = 0; j0 < k; j0 += kBatch) {
+#pragma unroll
+                for (int j = 0; j < kBatch; ++j) {
+                    const int r = j0 + j < k ? s_row[j0 + j] : -1;
+                    v[j] = r >= 0 ? __ldcs(reinterpret_cast<const uint4 *>(da + (size_t)r * H) + c)
+                                  : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int j = 0; j < kBatch; ++j)
+                    if (j0 + j < k && s_row[j0 + j] >= 0) add(v[j], 1.f);
             }
-            for (int s = 0; s < E_sh; ++s) add_row(da_sh + ((size_t)s * Tp + t) * H, 1.f);
+            for (int s = 0; s < E_sh; ++s)
+                add(__ldcs(reinterpret_cast<const uint4 *>(da_sh + ((size_t)s * Tp + t) * H) + c), 1.f);
             if (renorm) {  // dz is zero outside the token's k picks
-                for (int j = 0; j < k; ++j) {
-                    const int pe = idx[(size_t)t * k + j] - e_base;
-                    if (pe >= 0 && pe < E_pool) add_row(router + (size_t)pe * H, dzt[pe]);
+                for (int j0 = 0; j0 < k; j0 += kBatch) {
+#pragma unroll
+                    for (int j = 0; j < kBatch; ++j) {
+                        const int pe = j0 + j < k ? s_pe[j0 + j] : -1;
+                        v[j] = pe >= 0 ? reinterpret_cast<const uint4 *>(router + (size_t)pe * H)[c]
+                                       : make_uint4(0u, 0u, 0u, 0u);
+                    }
+#pragma unroll
+                    for (int j = 0; j < kBatch; ++j)
+                        if (j0 + j < k && s_pe[j0 + j] >= 0) add(v[j], s_dz[j0 + j]);
                 }
             } else {
-                for (int e = 0; e < E_pool; ++e) add_row(router + (size_t)e * H, dzt[e]);
+                for (int e = 0; e < E_pool; ++e) add(reinterpret_cast<const uint4 *>(router + (size_t)e * H)[c], dzt[e]);
             }
             float4 *o = reinterpret_cast<float4 *>(d_hidden + (size_t)t * H) + 2 * c;
-            o[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-            o[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+            __stcs(o, make_float4(acc[0], acc[1], acc[2], acc[3]));
+            __stcs(o + 1, make_float4(acc[4], acc[5], acc[6], acc[7]));
         }
     }
 }

@@ -187,6 +187,7 @@ struct RowsParams {
     const bf16 *zpad;     // gate/up: Z in the padded row layout [RP][I]
     float *gw_part;       // gate/up (routed, may be null): [R][I / 128] dL/dw partial per 128-column tile
     int wact;             // gate/up: 1 to write w act to out1
+    int reverse;          // 1: walk the tiles from the last group to the first
     uint32_t *status;
     uint32_t idesc;
 };
@@ -203,8 +204,9 @@ struct RowsTile {
     int q, m0, n0, n_tile, rows;
 };
 
-__device__ __forceinline__ RowsTile decode_rows(const GroupTable &gt, int G, int nt, int bn, int tile)
+__device__ __forceinline__ RowsTile decode_rows(const GroupTable &gt, int G, int nt, int bn, int tile, int reverse)
 {
+    if (reverse) tile = gt.tiles[G] - 1 - tile;
     int lo = 0, hi = G - 1;  // last group whose tile prefix is <= tile (skips empty groups)
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
@@ -276,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
         uint32_t phase = 0, filled = 0, last_parity = 0;
         const int half = p.bn / 128;  // MN mode: MN blocks per loader lane
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
-            const RowsTile t = decode_rows(gt, p.G, nt, p.bn, tile);
+            const RowsTile t = decode_rows(gt, p.G, nt, p.bn, tile, p.reverse);
             const int2 wq = group_weights(p, t.q);
             const int arow = (p.a_rows == kArowsPad ? gt.pad[t.q] : (p.a_rows == kArowsSlot ? p0 : 0) + gt.off[t.q]) + t.m0;
             bool ok = true;
@@ -348,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
         OutStager out{sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * kOutBufs * kOutBoxBytes), 0};
         int it = 0;
         for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
-            const RowsTile t = decode_rows(gt, p.G, nt, p.bn, tile);
+            const RowsTile t = decode_rows(gt, p.G, nt, p.bn, tile, p.reverse);
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
             int ok = 1;
@@ -710,6 +712,10 @@ cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uin
     memset(&maps, 0, sizeof(maps));
     p.K = s.H; p.N = s.I; p.bn = 128;
     p.a_rows = kArowsSlot;
+    // last group first: the Z launch before ended on the last groups, whose
+    // rows are still in L2, and the launch after starts on the first groups,
+    // whose operands this one read last
+    p.reverse = 1;
     p.zpad = zpad;
     p.gw_part = gw_part;
     p.wact = wact ? 1 : 0;

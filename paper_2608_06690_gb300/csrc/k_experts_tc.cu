@@ -138,13 +138,6 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
     return t;
 }
 
-__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *ptr)
-{
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];\n" : "=r"(v) : "l"(ptr) : "memory");
-    return v;
-}
-
 // ---------------------------------------------------------------- kernel
 
 __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcParams p, const __grid_constant__ TcMaps maps)

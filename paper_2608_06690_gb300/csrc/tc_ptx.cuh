@@ -184,6 +184,14 @@ __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.w
 // Wait until all committed bulk groups have completed.
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
 
+// A counter another CTA releases (ld.acquire at GPU scope).
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *ptr)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];\n" : "=r"(v) : "l"(ptr) : "memory");
+    return v;
+}
+
 // ---------------------------------------------------------------- host side
 
 // 2-D BF16 tensor map over a row-major [rows, cols] matrix with a 64-column x

@@ -110,3 +110,42 @@ def test_full_size_backward_on_sampled_tokens(name):
     g2 = layer.backward_private(h, pd, d2.cuda())
     for n in g:
         assert np.array_equal(g[n], g2[n].cpu().numpy().astype(np.float64)), n
+
+
+@pytest.mark.parametrize("name", ["qwen3_prefill", "deepseek_v2_lite"])
+def test_full_size_input_gradient_on_sampled_tokens(name):
+    """The gradient of the layer's input at full size, launched as the
+    benchmark launches it.  dout is nonzero on sampled ALLOW and DENY tokens
+    only: the oracle computes their rows, which are compared element by
+    element; every other row is exactly zero (each term is linear in the
+    token's own dout row).  A second run is bitwise identical."""
+    from paper_2608_06690_gb300 import pmpe
+    from pmpe_testlib import GAP_EPS, oracle_layer
+    cfg = CONFIGS[name]
+    s = cfg.shape
+    w = inp.make_weights(s, cfg.seed, device="cuda", skew=cfg.skew)
+    h = inp.make_hidden(s, cfg.seed, device="cuda", skew=cfg.skew)
+    pol = cfg.policy(s.T)
+    w_cpu = {k: (None if v is None else v.cpu()) for k, v in w.items()}
+    L = oracle_layer(s, w_cpu, h.cpu(), pol)
+    toks = _sample_tokens(cfg, per_pool=12, seed=2)
+    _, _, gap = oracle.route(L, tokens=toks)
+    keep = toks[gap >= GAP_EPS]
+    gen = torch.Generator().manual_seed(12)
+    dout = torch.zeros((s.T, s.H), dtype=torch.bfloat16)
+    dout[torch.from_numpy(keep).long()] = torch.randn((len(keep), s.H), generator=gen).to(torch.bfloat16)
+    layer = pmpe.MoeLayer(s, w)
+    pd = pol.cuda()
+    layer.forward(h, pd)
+    dh = layer.backward_input(h, pd, dout.cuda())
+    got = dh.cpu().numpy().astype(np.float64)
+    ref = oracle.backward_input(L, dout.double().numpy())
+    tau = oracle.resolve(pol.numpy(), s.T)
+    assert tau[keep].sum() >= 8 and (tau[keep] == 0).sum() >= 8
+    err = np.abs(got[keep] - ref[keep])
+    assert err.max() / np.abs(ref[keep]).max() <= 2e-2 and err.sum() / np.abs(ref[keep]).sum() <= 1e-2
+    rest = np.ones(s.T, bool)
+    rest[keep] = False
+    assert np.all(got[rest] == 0.0)
+    layer.forward(h, pd)
+    assert torch.equal(dh, layer.backward_input(h, pd, dout.cuda()))
