@@ -68,28 +68,35 @@ def test_48_layer_stack_replays_bitwise_from_a_cuda_graph():
 def test_training_step_with_private_backward_replays_bitwise_from_a_cuda_graph():
     """One training step of a two-layer stack captured into one CUDA graph:
     the layers' forwards (the second fed the first one's output), then the
-    private-branch backward of each layer for its upstream gradient.  Each
-    layer keeps its own workspace, which holds that layer's forward state for
-    its backward.  Replaying the graph twice gives bit for bit the outputs and
-    the four private gradients of each layer computed one call at a time."""
-    s = LayerShape(T=512, H=512, I=256, E_pub=32, E_priv=8, E_sh=0, k=4, renormalize=True)
+    top layer's private-branch backward and its input gradient, which in BF16
+    is the upstream gradient of the lower layer's private-branch backward.
+    Each layer keeps its own workspace, which holds that layer's forward state
+    for its backward.  Replaying the graph twice gives bit for bit the outputs,
+    the four private gradients of each layer and the top layer's input
+    gradient computed one call at a time."""
+    s = LayerShape(T=512, H=512, I=256, E_pub=32, E_priv=8, E_sh=1, k=4, renormalize=True)
     layers = [pmpe.MoeLayer(s, inp.make_weights(s, 8000 + l, device="cuda")) for l in range(2)]
     x0 = inp.make_hidden(s, 8, device="cuda")
     pol = inp.policy_iid_mixed(s.T, 8).cuda()
     gen = torch.Generator(device="cuda")
     gen.manual_seed(9)
-    douts = [torch.randn((s.T, s.H), generator=gen, device="cuda").to(torch.bfloat16) for _ in layers]
+    dtop = torch.randn((s.T, s.H), generator=gen, device="cuda").to(torch.bfloat16)
 
     def step(x_in, outs):
         ins = [x_in, outs[0]]
         for l, layer in enumerate(layers):
             layer.forward(ins[l], pol, out=outs[l])
-        return [layers[l].backward_private(ins[l], pol, douts[l]) for l in range(len(layers))]
+        g1 = layers[1].backward_private(ins[1], pol, dtop)
+        dh1 = layers[1].backward_input(ins[1], pol, dtop)
+        g0 = layers[0].backward_private(ins[0], pol, dh1.to(torch.bfloat16))
+        return [g0, g1, {"d_hidden": dh1}]
 
     outs_e = [torch.empty_like(x0) for _ in layers]
-    grads_e = step(x0, outs_e)   # also sizes every workspace before capture
+    res_e = step(x0, outs_e)   # also sizes every workspace before capture
     torch.cuda.synchronize()
-    grads_e = [{n: v.clone() for n, v in g.items()} for g in grads_e]
+    res_e = [{n: v.clone() for n, v in g.items()} for g in res_e]
+    assert torch.all(torch.isfinite(res_e[2]["d_hidden"])) and res_e[2]["d_hidden"].abs().max() > 0
+    assert res_e[0]["d_gate"].abs().max() > 0
 
     x_in = x0.clone()
     outs_g = [torch.empty_like(x0) for _ in layers]
@@ -101,7 +108,7 @@ def test_training_step_with_private_backward_replays_bitwise_from_a_cuda_graph()
     torch.cuda.synchronize()
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
-        grads_g = step(x_in, outs_g)
+        res_g = step(x_in, outs_g)
     for rep in range(2):
         for o in outs_g:
             o.fill_(0)
@@ -109,5 +116,6 @@ def test_training_step_with_private_backward_replays_bitwise_from_a_cuda_graph()
         torch.cuda.synchronize()
         for l in range(len(layers)):
             assert torch.equal(outs_g[l].view(torch.int16), outs_e[l].view(torch.int16)), (rep, l)
-            for n in grads_e[l]:
-                assert torch.equal(grads_g[l][n], grads_e[l][n]), (rep, l, n)
+        for i in range(len(res_e)):
+            for n in res_e[i]:
+                assert torch.equal(res_g[i][n], res_e[i][n]), (rep, i, n)
