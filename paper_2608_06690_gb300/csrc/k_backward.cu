@@ -128,13 +128,19 @@ __global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_pub, co
     }
 }
 
+constexpr int kMaxRouterSplits = 64;  // token ranges of the router weight gradient
+
 // dW_router[e][c] = sum_t dz[t][e] h[t][c] in FP32, split over the tokens:
 // CTA (x, y, z) owns a 32 x 128 output tile and the z-th token range, staged
 // through shared memory 32 tokens at a time, and writes its partial sum to
 // part[z]; bwd_router_reduce_kernel adds the partials in split order, so the
-// result does not depend on scheduling.
-__global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, const bf16 *hidden, int T, int H,
-                                                               int E_priv, int tok_per_split, float *part)
+// result does not depend on scheduling.  A block of 32 DENY tokens (dz
+// exactly zero) is skipped: its products would add exact zeros.  A range of
+// DENY tokens only writes no partial and clears active[z], so the reduction
+// skips it; otherwise active[z] = 1.
+__global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, const bf16 *hidden,
+                                                               const uint8_t *tau, int T, int H, int E_priv,
+                                                               int tok_per_split, float *part, int *active)
 {
     __shared__ float s_dz[32][33];
     __shared__ __align__(16) float s_h[32][128];
@@ -146,7 +152,10 @@ __global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, 
     for (int a = 0; a < 4; ++a)
 #pragma unroll
         for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
+    bool any = false;
     for (int t0 = t_begin; t0 < t_end; t0 += 32) {
+        if (!__syncthreads_or(threadIdx.x < 32 && t0 + (int)threadIdx.x < t_end && tau[t0 + threadIdx.x])) continue;
+        any = true;
         for (int i = threadIdx.x; i < 32 * 32; i += 256) {
             const int tt = i >> 5, ee = i & 31;
             s_dz[tt][ee] = (t0 + tt < t_end && e0 + ee < E_priv) ? dz[(size_t)(t0 + tt) * E_priv + e0 + ee] : 0.f;
@@ -180,6 +189,8 @@ __global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, 
         }
         __syncthreads();
     }
+    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) active[blockIdx.z] = any ? 1 : 0;
+    if (!any) return;  // uniform over the CTA
     float *out = part + (size_t)blockIdx.z * E_priv * H;
 #pragma unroll
     for (int a = 0; a < 4; ++a)
@@ -190,23 +201,41 @@ __global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, 
         }
 }
 
-__global__ void bwd_router_reduce_kernel(const float *part, int nsplit, int n, float *d_router)
+// d_router = the active partials summed in split order (a skipped range
+// contributes exact zeros).
+__global__ void bwd_router_reduce_kernel(const float *part, const int *active, int nsplit, int n, float *d_router)
 {
+    __shared__ int s_list[kMaxRouterSplits];
+    __shared__ int s_n;
+    if (threadIdx.x == 0) {
+        int m = 0;
+        for (int z = 0; z < nsplit; ++z)
+            if (active[z]) s_list[m++] = z;
+        s_n = m;
+    }
+    __syncthreads();
+    const int m = s_n;
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
         float a = 0.f;
-        for (int z = 0; z < nsplit; ++z) a += part[(size_t)z * n + i];
+        int j = 0;
+        for (; j + 4 <= m; j += 4) {  // four loads in flight, summed in order
+            const float v0 = part[(size_t)s_list[j] * n + i], v1 = part[(size_t)s_list[j + 1] * n + i];
+            const float v2 = part[(size_t)s_list[j + 2] * n + i], v3 = part[(size_t)s_list[j + 3] * n + i];
+            a += v0; a += v1; a += v2; a += v3;
+        }
+        for (; j < m; ++j) a += part[(size_t)s_list[j] * n + i];
         d_router[i] = a;
     }
 }
 
-// Token splits of the router weight gradient: enough CTAs for two per SM,
+// Token splits of the router weight gradient: enough CTAs for eight per SM
+// (ranges of DENY tokens end at once, so short ranges keep the SMs busy),
 // each range a multiple of 32 tokens, at most kMaxRouterSplits ranges.
-constexpr int kMaxRouterSplits = 64;
 int router_splits(const Shape &s, int num_sms, int *tok_per_split)
 {
     const int tiles = ((s.H + 127) / 128) * ((s.E_priv + 31) / 32);
     const int chunks = std::max(1, (s.T + 31) / 32);
-    int n = std::min(std::min(kMaxRouterSplits, chunks), std::max(1, (2 * num_sms + tiles - 1) / tiles));
+    int n = std::min(std::min(kMaxRouterSplits, chunks), std::max(1, (8 * num_sms + tiles - 1) / tiles));
     const int per = ((chunks + n - 1) / n) * 32;
     n = std::max(1, (s.T + per - 1) / per);
     *tok_per_split = per;
@@ -237,6 +266,7 @@ cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools,
 struct BwdScratch {
     bf16 *dout_rows, *zpad, *dgu, *wact;
     float *gw_part, *dz, *part;
+    int *active;  // per token range of the router weight gradient: 1 if it holds an ALLOW token
     size_t bytes;
 };
 
@@ -254,6 +284,7 @@ static BwdScratch backward_scratch(const Shape &s, uint8_t *base)
     b.gw_part = (float *)(base + o);  o += al(R * (I / 128) * 4);
     b.dz = (float *)(base + o);       o += al((size_t)s.T * s.E_priv * 4);
     b.part = (float *)(base + o);     o += al(splits * s.E_priv * H * 4);
+    b.active = (int *)(base + o);     o += al(kMaxRouterSplits * 4);
     b.bytes = o;
     return b;
 }
@@ -281,10 +312,12 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
     int per = 32;
     const int nsplit = router_splits(s, c.num_sms, &per);
     dim3 grid((H + 127) / 128, (s.E_priv + 31) / 32, nsplit);
-    bwd_router_wgrad_kernel<<<grid, 256, 0, st>>>(b.dz, c.hidden, s.T, H, s.E_priv, per, b.part);
+    bwd_router_wgrad_kernel<<<grid, 256, 0, st>>>(b.dz, c.hidden, c.tau, s.T, H, s.E_priv, per, b.part,
+                                                  b.active);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     const int n = s.E_priv * H;
-    bwd_router_reduce_kernel<<<std::min((n + 255) / 256, c.num_sms * 4), 256, 0, st>>>(b.part, nsplit, n, d_router);
+    bwd_router_reduce_kernel<<<std::min((n + 255) / 256, c.num_sms * 4), 256, 0, st>>>(b.part, b.active, nsplit, n,
+                                                                                              d_router);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
 
     return launch_backward_wgrad(c, b.dout_rows, b.dgu, b.wact, d_gate, d_up, d_down);
