@@ -21,23 +21,37 @@
 namespace pmpe {
 namespace {
 
-// Upstream gradients of the private dispatch rows, in dispatch order, and 64
-// zero rows after the last one (the weight-gradient GEMM reads up to 63 rows
-// past an expert's rows, multiplied by zeros there, which must be finite).
-__global__ void bwd_gather_kernel(const bf16 *dout, const int32_t *tok_of_slot, const uint32_t *offsets, int E_pub,
-                                  int E, int R, int H, bf16 *dout_rows)
+// Upstream gradients of the dispatch rows of experts g0 .. g1 - 1, in
+// dispatch order, and 64 zero rows after the last one (the weight-gradient
+// GEMM reads up to 63 rows past an expert's rows, multiplied by zeros there,
+// which must be finite).  One warp per row, eight 16-byte loads in flight per
+// lane.
+__global__ void __launch_bounds__(256) bwd_gather_kernel(const bf16 *dout, const int32_t *tok_of_slot,
+                                                         const uint32_t *offsets, int g0, int g1, int R, int H,
+                                                         bf16 *dout_rows)
 {
-    const uint32_t p0 = min(offsets[E_pub], (uint32_t)R), p1 = min(max(offsets[E], p0), (uint32_t)R);
+    const uint32_t p0 = min(offsets[g0], (uint32_t)R), p1 = min(max(offsets[g1], p0), (uint32_t)R);
     const int nv = H / 8;
-    const long long rows = (long long)(p1 - p0);
-    const long long total = (rows + 64) * nv;
-    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const long long r = i / nv;
-        const int c = (int)(i - r * nv);
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (r < rows) v = reinterpret_cast<const uint4 *>(dout + (size_t)tok_of_slot[p0 + r] * H)[c];
-        reinterpret_cast<uint4 *>(dout_rows + (size_t)r * H)[c] = v;
+    const int rows = (int)(p1 - p0);
+    const int lane = threadIdx.x & 31;
+    const int warps = gridDim.x * (blockDim.x >> 5);
+    constexpr int kU = 8;
+    for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows + 64; r += warps) {
+        const uint4 *src = r < rows ? reinterpret_cast<const uint4 *>(dout + (size_t)tok_of_slot[p0 + r] * H) : nullptr;
+        uint4 *dst = reinterpret_cast<uint4 *>(dout_rows + (size_t)r * H);
+        for (int c0 = 0; c0 < nv; c0 += 32 * kU) {
+            uint4 v[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + u * 32 + lane;
+                v[u] = (src != nullptr && c < nv) ? src[c] : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + u * 32 + lane;
+                if (c < nv) dst[c] = v[u];
+            }
+        }
     }
 }
 
