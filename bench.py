@@ -205,6 +205,20 @@ def backward_input_flops(s, counts: np.ndarray, allow_tokens: int) -> float:
     return f
 
 
+def backward_min_bytes(s, counts: np.ndarray, allow_tokens: int, which: str) -> float:
+    """Lower bound of a backward pass's DRAM bytes: every input read once and
+    every output written once (the weights of the experts with rows, the
+    hidden and dout rows of the tokens that reach them, the routers, and the
+    FP32 outputs); intermediates and the recompute are not counted."""
+    per_expert = 3.0 * s.I * s.H * 2
+    if which == "private":
+        touched = float((counts[s.E_pub:] > 0).sum())
+        return (touched * per_expert + 2.0 * allow_tokens * s.H * 2 + s.E_priv * s.H * 2
+                + 3.0 * s.E_priv * s.I * s.H * 4 + s.E_priv * s.H * 4)
+    touched = float((counts > 0).sum()) + s.E_sh
+    return touched * per_expert + 2.0 * s.T * s.H * 2 + s.E * s.H * 2 + s.T * s.H * 4
+
+
 def cpu_baseline(cfg, w, h, pol, budget_s=12.0, max_tokens=4096):
     """The CPU oracle, as it stands, on a bounded sample of the workload's
     tokens (the first n tokens of each request, spread evenly)."""
@@ -469,6 +483,9 @@ def run_ours(args):
                 "tensor_frac": f_bwd / (bwd_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
                 "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.KERNELS_PER_BACKWARD,
                 "l2": "flushed before every pass"}
+    mb = backward_min_bytes(s, counts, int((pol == 1).sum().item()), "private")
+    backward.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9,
+                     "hbm_frac_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9 / hbm})
 
     bin_avg = float(np.mean(bin_ms))
     f_bin = backward_input_flops(s, counts, int((pol == 1).sum().item()))
@@ -476,6 +493,9 @@ def run_ours(args):
                    "tensor_frac": f_bin / (bin_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
                    "routed_rows": int(counts.sum()), "launches": pmpe.kernels_per_backward_input(s),
                    "l2": "flushed before every pass"}
+    mb = backward_min_bytes(s, counts, int((pol == 1).sum().item()), "input")
+    backward_in.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bin_avg / 1e3) / 1e9,
+                        "hbm_frac_of_min_bytes": mb / (bin_avg / 1e3) / 1e9 / hbm})
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
