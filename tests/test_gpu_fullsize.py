@@ -149,3 +149,32 @@ def test_full_size_input_gradient_on_sampled_tokens(name):
     assert np.all(got[rest] == 0.0)
     layer.forward(h, pd)
     assert torch.equal(dh, layer.backward_input(h, pd, dout.cuda()))
+
+
+@pytest.mark.parametrize("name", ["qwen3_prefill", "deepseek_v2_lite"])
+def test_full_size_input_gradient_of_deny_tokens_ignores_private_weights(name):
+    """G2 through the input gradient at full size: every private weight
+    (router, gate, up, down) replaced by other random values leaves the DENY
+    tokens' rows of d_hidden bitwise unchanged, while the ALLOW rows change."""
+    from paper_2608_06690_gb300 import pmpe
+    cfg = CONFIGS[name]
+    s = cfg.shape
+    w = inp.make_weights(s, cfg.seed, device="cuda", skew=cfg.skew)
+    h = inp.make_hidden(s, cfg.seed, device="cuda", skew=cfg.skew)
+    pd = cfg.policy(s.T).cuda()
+    tau = torch.from_numpy(oracle.resolve(cfg.policy(s.T).numpy(), s.T).astype(bool)).cuda()
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(13)
+    dout = torch.randn((s.T, s.H), generator=gen, device="cuda").to(torch.bfloat16)
+    layer = pmpe.MoeLayer(s, w)
+    layer.forward(h, pd)
+    dh1 = layer.backward_input(h, pd, dout).clone()
+    w2 = dict(w)
+    for n in ("router_priv", "gate_priv", "up_priv", "down_priv"):
+        w2[n] = (torch.randn(w[n].shape, generator=gen, device="cuda") * 0.02).to(torch.bfloat16)
+    layer2 = pmpe.MoeLayer(s, w2)
+    layer2.forward(h, pd)
+    dh2 = layer2.backward_input(h, pd, dout)
+    torch.cuda.synchronize()
+    assert torch.equal(dh1[~tau], dh2[~tau])
+    assert not torch.equal(dh1[tau], dh2[tau])
