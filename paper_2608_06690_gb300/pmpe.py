@@ -42,8 +42,9 @@ STAGE_COMBINE = 0x10
 STAGE_ALL = 0x1F
 
 # Kernels one full forward launches: router/top-k (with the policy resolve),
-# dispatch + row gather, gate/up GEMM, down GEMM, combine (plus one memset of
-# the per-expert counters, which is not a kernel of this library).
+# dispatch + row gather, the gate/up and down GEMMs (one persistent launch),
+# combine (plus one memset of the per-expert counters, which is not a kernel
+# of this library).
 KERNELS_PER_FORWARD = 4
 # kernels one private-branch backward launches: dout row gather, the dL/da
 # GEMM, the gate/up recompute GEMM with the SwiGLU backward, router gradient,
