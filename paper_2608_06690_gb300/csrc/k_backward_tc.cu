@@ -24,7 +24,7 @@
 //
 // The same two row kernels, over all routed experts and the shared experts,
 // and an MN-mode launch dA = [dG | dU] [W_gate; W_up] give the gradient of
-// the layer's input (launch_backward_input_gemms).
+// the layer's input (launch_rows_z, launch_rows_gu, launch_rows_da).
 //
 // Every launch keeps four 48 KB operand stages in flight (a 128 x 256 x 64 MMA
 // block each) and two 128 x 256 FP32 accumulators, so the epilogue of one tile
