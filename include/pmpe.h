@@ -232,6 +232,28 @@ PMPE_API size_t pmpe_moe_backward_input_workspace_size(int T, int H, int I, int 
 PMPE_API int pmpe_moe_backward_input(const pmpe_moe_desc *d, const void *dout, float *d_hidden, void *bwd_workspace,
                                      size_t bwd_workspace_bytes, void *stream);
 
+/* ------------------------------------------------- both, in one pass */
+
+/* Bytes of device scratch pmpe_moe_backward_step() needs; 0 for an invalid
+ * shape. */
+PMPE_API size_t pmpe_moe_backward_step_workspace_size(int T, int H, int I, int E_pub, int E_priv, int E_shared,
+                                                      int k);
+
+/* The private-parameter gradients of pmpe_moe_backward_private() and the
+ * input gradient of pmpe_moe_backward_input() in one pass, for a training
+ * step that needs both (Sec. 3.2: the private branch of every wrapped layer
+ * is trained, so each layer also passes dL/dh to the layer below).  The
+ * private experts' rows are recomputed once for both.  Every output is
+ * bitwise the one the two separate calls give.  Arguments, preconditions and
+ * errors are those of the two calls: the forward's descriptor and workspace,
+ * dout [T, H] BF16, d_router_priv [E_priv, H], d_gate_priv and d_up_priv
+ * [E_priv, I, H], d_down_priv [E_priv, H, I] and d_hidden [T, H], all FP32,
+ * overwritten and 16-byte aligned; bwd_workspace of at least the size above,
+ * 256-byte aligned.  Asynchronous on `stream`. */
+PMPE_API int pmpe_moe_backward_step(const pmpe_moe_desc *d, const void *dout, float *d_router_priv,
+                                    float *d_gate_priv, float *d_up_priv, float *d_down_priv, float *d_hidden,
+                                    void *bwd_workspace, size_t bwd_workspace_bytes, void *stream);
+
 /* Per-token policy bytes from per-request ones, for callers that carry one
  * trusted authorisation byte per request and the requests' cumulative token
  * offsets (cu_seqlens[0..n_req], device int32) instead of a byte per token.

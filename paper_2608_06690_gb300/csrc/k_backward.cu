@@ -142,8 +142,6 @@ __global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_pub, co
     }
 }
 
-constexpr int kMaxRouterSplits = 64;  // token ranges of the router weight gradient
-
 // dW_router[e][c] = sum_t dz[t][e] h[t][c] in FP32, split over the tokens:
 // CTA (x, y, z) owns a 32 x 128 output tile and the z-th token range, staged
 // through shared memory 32 tokens at a time, and writes its partial sum to
@@ -151,8 +149,9 @@ constexpr int kMaxRouterSplits = 64;  // token ranges of the router weight gradi
 // result does not depend on scheduling.  A block of 32 DENY tokens (dz
 // exactly zero) is skipped: its products would add exact zeros.  A range of
 // DENY tokens only writes no partial and clears active[z], so the reduction
-// skips it; otherwise active[z] = 1.
-__global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, const bf16 *hidden,
+// skips it; otherwise active[z] = 1.  dz rows are ld apart; a DENY token's
+// row is read as zeros (it may hold its public pool's gradient).
+__global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, int ld, const bf16 *hidden,
                                                                const uint8_t *tau, int T, int H, int E_priv,
                                                                int tok_per_split, float *part, int *active)
 {
@@ -172,7 +171,8 @@ __global__ void __launch_bounds__(256) bwd_router_wgrad_kernel(const float *dz, 
         any = true;
         for (int i = threadIdx.x; i < 32 * 32; i += 256) {
             const int tt = i >> 5, ee = i & 31;
-            s_dz[tt][ee] = (t0 + tt < t_end && e0 + ee < E_priv) ? dz[(size_t)(t0 + tt) * E_priv + e0 + ee] : 0.f;
+            s_dz[tt][ee] = (t0 + tt < t_end && e0 + ee < E_priv && tau[t0 + tt]) ? dz[(size_t)(t0 + tt) * ld + e0 + ee]
+                                                                                  : 0.f;
         }
         for (int i = threadIdx.x; i < 32 * 16; i += 256) {
             const int tt = i >> 4, cc = (i & 15) * 8;
@@ -288,7 +288,6 @@ static BwdScratch backward_scratch(const Shape &s, uint8_t *base)
 {
     const size_t R = (size_t)s.T * s.k, H = s.H, I = s.I, RP = backward_padded_rows(s);
     auto al = [](size_t x) { return (x + 255) / 256 * 256; };
-    const size_t splits = (size_t)std::min(kMaxRouterSplits, (s.T + 31) / 32);
     BwdScratch b;
     size_t o = 0;
     b.dout_rows = (bf16 *)(base + o); o += al((R + 64) * H * 2);
@@ -297,7 +296,7 @@ static BwdScratch backward_scratch(const Shape &s, uint8_t *base)
     b.wact = (bf16 *)(base + o);      o += al(RP * I * 2);
     b.gw_part = (float *)(base + o);  o += al(R * (I / 128) * 4);
     b.dz = (float *)(base + o);       o += al((size_t)s.T * s.E_priv * 4);
-    b.part = (float *)(base + o);     o += al(splits * s.E_priv * H * 4);
+    b.part = (float *)(base + o);     o += al(router_wgrad_part_bytes(s));
     b.active = (int *)(base + o);     o += al(kMaxRouterSplits * 4);
     b.bytes = o;
     return b;
@@ -323,18 +322,30 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
     if (err != cudaSuccess) return err;
     if ((err = launch_backward_rows(c, b.dout_rows, b.zpad, b.dgu, b.wact, b.gw_part)) != cudaSuccess) return err;
     if ((err = launch_router_dz(c, b.gw_part, 0, s.E_priv, b.dz)) != cudaSuccess) return err;
+    if ((err = launch_router_wgrad(c, b.dz, s.E_priv, b.part, b.active, d_router)) != cudaSuccess) return err;
+    return launch_backward_wgrad(c, b.dout_rows, b.dgu, b.wact, d_gate, d_up, d_down);
+}
+
+size_t router_wgrad_part_bytes(const Shape &s)
+{
+    const size_t splits = (size_t)std::min(kMaxRouterSplits, (s.T + 31) / 32);
+    return splits * s.E_priv * s.H * 4;
+}
+
+cudaError_t launch_router_wgrad(const Ctx &c, const float *dz, int ld, float *part, int *active, float *d_router)
+{
+    const Shape &s = c.s;
     int per = 32;
     const int nsplit = router_splits(s, c.num_sms, &per);
-    dim3 grid((H + 127) / 128, (s.E_priv + 31) / 32, nsplit);
-    bwd_router_wgrad_kernel<<<grid, 256, 0, st>>>(b.dz, c.hidden, c.tau, s.T, H, s.E_priv, per, b.part,
-                                                  b.active);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    const int n = s.E_priv * H;
-    bwd_router_reduce_kernel<<<std::min((n + 255) / 256, c.num_sms * 4), 256, 0, st>>>(b.part, b.active, nsplit, n,
-                                                                                              d_router);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-
-    return launch_backward_wgrad(c, b.dout_rows, b.dgu, b.wact, d_gate, d_up, d_down);
+    dim3 grid((s.H + 127) / 128, (s.E_priv + 31) / 32, nsplit);
+    bwd_router_wgrad_kernel<<<grid, 256, 0, c.stream>>>(dz, ld, c.hidden, c.tau, s.T, s.H, s.E_priv, per, part,
+                                                        active);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    const int n = s.E_priv * s.H;
+    bwd_router_reduce_kernel<<<std::min((n + 255) / 256, c.num_sms * 4), 256, 0, c.stream>>>(part, active, nsplit,
+                                                                                              n, d_router);
+    return cudaGetLastError();
 }
 
 }  // namespace pmpe

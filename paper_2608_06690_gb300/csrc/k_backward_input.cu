@@ -171,6 +171,19 @@ static InScratch input_scratch(const Shape &s, uint8_t *base)
     return b;
 }
 
+// The per-token sum of the picks' dA, the shared experts' dA and the router
+// term (dz rows max(E_pub, E_priv) apart).
+static cudaError_t launch_input_reduce(const Ctx &c, const InScratch &b, float *d_hidden)
+{
+    const Shape &s = c.s;
+    const int ld = std::max(s.E_pub, s.E_priv);
+    return launch_pdl(bwd_input_reduce_kernel, dim3(std::min(s.T, c.num_sms * 8)), dim3(256), 0, c.stream,
+                      (const bf16 *)b.da, (const bf16 *)b.da_sh, (const float *)b.dz, ld, c.router_pub,
+                      c.router_priv, (const uint8_t *)c.tau, (const int32_t *)c.idx, (const int32_t *)c.slot_of,
+                      (const uint32_t *)c.offsets, s.T, s.H, s.E_pub, s.E_priv, s.E_sh, s.k, s.T * s.k, s.renorm,
+                      b.tp, d_hidden);
+}
+
 size_t backward_input_workspace_bytes(const Shape &s)
 {
     if (s.T == 0) return 256;
@@ -206,11 +219,77 @@ cudaError_t launch_backward_input(const Ctx &c, const bf16 *dout, float *d_hidde
     // the router of each token's pool
     const int ld = std::max(s.E_pub, s.E_priv);
     if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz)) != cudaSuccess) return err;
-    return launch_pdl(bwd_input_reduce_kernel, dim3(std::min(s.T, c.num_sms * 8)), dim3(256), 0, st,
-                      (const bf16 *)b.da, (const bf16 *)b.da_sh, (const float *)b.dz, ld, c.router_pub,
-                      c.router_priv, (const uint8_t *)c.tau, (const int32_t *)c.idx, (const int32_t *)c.slot_of,
-                      (const uint32_t *)c.offsets, s.T, H, s.E_pub, s.E_priv, s.E_sh, s.k, R, s.renorm, b.tp,
-                      d_hidden);
+    return launch_input_reduce(c, b, d_hidden);
+}
+
+// ------------------------------------------------------------- both
+
+// The private-parameter gradients and the input gradient of one backward from
+// a single set of row launches over all routed experts: Z and [dG | dU] of
+// the private experts are the same rows either way, so they are computed
+// once.  The weight gradients read the private experts' rows in the padded
+// layout of all experts; w act is written for the private experts only; the
+// router's dz of both pools serves the input gradient and, read as zeros on
+// DENY rows, the private router's weight gradient.  Every result is bitwise
+// the one the two separate passes give.
+struct StepScratch {
+    InScratch in;
+    bf16 *wact;
+    float *part;
+    int *active;
+    size_t bytes;
+};
+
+static StepScratch step_scratch(const Shape &s, uint8_t *base)
+{
+    auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+    StepScratch b;
+    b.in = input_scratch(s, base);
+    size_t o = b.in.bytes;
+    b.wact = (bf16 *)(base + o);   o += al(b.in.rp * s.I * 2);
+    b.part = (float *)(base + o);  o += al(router_wgrad_part_bytes(s));
+    b.active = (int *)(base + o);  o += al(kMaxRouterSplits * 4);
+    b.bytes = o;
+    return b;
+}
+
+size_t backward_step_workspace_bytes(const Shape &s)
+{
+    if (s.T == 0) return 256;
+    return step_scratch(s, nullptr).bytes;
+}
+
+cudaError_t launch_backward_step(const Ctx &c, const bf16 *dout, float *d_router, float *d_gate, float *d_up,
+                                 float *d_down, float *d_hidden, uint8_t *bws)
+{
+    const Shape &s = c.s;
+    const int R = s.T * s.k, H = s.H, E = s.E();
+    const StepScratch st = step_scratch(s, bws);
+    const InScratch &b = st.in;
+    cudaStream_t stream = c.stream;
+
+    launch_gather_rows(dout, c.tok_of_slot, c.offsets, 0, E, R, H, b.dout_rows, c.num_sms, stream);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    const RowsGroups g{0, E, 0, b.rp};
+    if ((err = launch_rows_z(c, g, b.dout_rows, (uint64_t)R + 64, 1, b.zpad)) != cudaSuccess) return err;
+    if ((err = launch_rows_gu(c, g, c.a_perm, (uint64_t)R, b.zpad, b.dgu, st.wact, b.gw_part)) != cudaSuccess)
+        return err;
+    if ((err = launch_rows_da(c, g, b.dgu, b.da)) != cudaSuccess) return err;
+    if (s.E_sh > 0) {
+        const RowsGroups gs{0, s.E_sh, s.T, b.rp_sh};
+        if ((err = launch_rows_z(c, gs, dout, (uint64_t)s.T, 0, b.zpad_sh)) != cudaSuccess) return err;
+        if ((err = launch_rows_gu(c, gs, c.hidden, (uint64_t)s.T, b.zpad_sh, b.dgu_sh, nullptr, nullptr)) !=
+            cudaSuccess)
+            return err;
+        if ((err = launch_rows_da(c, gs, b.dgu_sh, b.da_sh)) != cudaSuccess) return err;
+    }
+    const int ld = std::max(s.E_pub, s.E_priv);
+    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz)) != cudaSuccess) return err;
+    if ((err = launch_router_wgrad(c, b.dz, ld, st.part, st.active, d_router)) != cudaSuccess) return err;
+    if ((err = launch_backward_wgrad(c, b.dout_rows, b.dgu, st.wact, d_gate, d_up, d_down, &g)) != cudaSuccess)
+        return err;
+    return launch_input_reduce(c, b, d_hidden);
 }
 
 }  // namespace pmpe

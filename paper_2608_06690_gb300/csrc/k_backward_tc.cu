@@ -186,7 +186,7 @@ struct RowsParams {
     const float *w_of_slot;  // gate/up: routing weights per slot (shared groups: weight 1)
     const bf16 *zpad;     // gate/up: Z in the padded row layout [RP][I]
     float *gw_part;       // gate/up (routed, may be null): [R][I / 128] dL/dw partial per 128-column tile
-    int wact;             // gate/up: 1 to write w act to out1
+    int wact;             // gate/up: 1 to write w act to out1 for the private experts' rows
     int reverse;          // 1: walk the tiles from the last group to the first
     uint32_t *status;
     uint32_t idesc;
@@ -414,7 +414,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
                     }
                     out.put(lane, pg, &maps.out0, t.n0 + c * 32, orow);
                     out.put(lane, pu, &maps.out0, p.I + t.n0 + c * 32, orow);
-                    if (p.wact) out.put(lane, pa, &maps.out1, t.n0 + c * 32, orow);
+                    if (p.wact && !p.shared_T && p.g0 + t.q >= p.E_pub)
+                        out.put(lane, pa, &maps.out1, t.n0 + c * 32, orow);
                 }
                 if (valid && p.gw_part) p.gw_part[(size_t)(p0 + prow) * nt + t.n_tile] = gw;
             }
@@ -438,6 +439,10 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
 
 struct WgParams {
     int E_pub, E_priv, H, I, R;
+    // the group table's groups (the private experts alone, g0 = E_pub, or all
+    // routed experts, g0 = 0, whose padded layout the operands then use) and
+    // the table index of private expert 0
+    int g0, G, q_off;
     int bn_a, bn_b;  // output columns per tile: [dW_gate; dW_up] (N = H), dW_down (N = I)
     const uint32_t *offsets;
     uint32_t *status;
@@ -479,7 +484,7 @@ __device__ __forceinline__ WgTile decode_wg(const WgParams &p, const GroupTable 
         t.n0 = (local % nb) * p.bn_b;
         t.bn = p.bn_b;
     }
-    t.nkb = (gt.rows[t.q] + BK - 1) / BK;
+    t.nkb = (gt.rows[t.q + p.q_off] + BK - 1) / BK;
     return t;
 }
 
@@ -509,13 +514,13 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
     }
     if (warp == 1) tmem_alloc(smem_u32(&s_tmem), kTmemCols);
     pdl_wait();
-    build_groups(gt, p.offsets, p.E_pub, p.E_priv, p.R, 0, 0, 0);
+    build_groups(gt, p.offsets, p.g0, p.G, p.R, 0, 0, 0);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
     const int total = p.E_priv * ((2 * p.I / BM) * (p.H / p.bn_a) + (p.H / BM) * (p.I / p.bn_b));
-    const int p0 = (int)min(p.offsets[p.E_pub], (uint32_t)p.R);
+    const int p0 = (int)min(p.offsets[p.g0], (uint32_t)p.R);
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
@@ -527,8 +532,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_wgrad_tc_kernel(const WgParam
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const WgTile t = decode_wg(p, gt, tile);
             const int nbox = t.bn / 64, half = nbox / 2;
-            const int rowA = t.prob == 0 ? gt.pad[t.q] : gt.off[t.q];
-            const int rowB = t.prob == 0 ? p0 + gt.off[t.q] : gt.pad[t.q];
+            const int gq = t.q + p.q_off;  // the expert's entry in the group table
+            const int rowA = t.prob == 0 ? gt.pad[gq] : gt.off[gq];
+            const int rowB = t.prob == 0 ? p0 + gt.off[gq] : gt.pad[gq];
             const CUtensorMap *amap = t.prob == 0 ? &maps.dgu : &maps.dout_rows;
             const CUtensorMap *bmap = t.prob == 0 ? &maps.a_perm : &maps.wact;
             bool ok = true;
@@ -768,15 +774,18 @@ cudaError_t launch_backward_rows(const Ctx &c, const bf16 *dout_rows, bf16 *zpad
 }
 
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
-                                  float *d_gate, float *d_up, float *d_down)
+                                  float *d_gate, float *d_up, float *d_down, const RowsGroups *all)
 {
     const Shape &s = c.s;
-    const uint64_t R = (uint64_t)s.T * s.k, RP = backward_padded_rows(s);
+    const uint64_t R = (uint64_t)s.T * s.k, RP = all ? all->padded_rows : backward_padded_rows(s);
     WgParams p;
     WgMaps maps;
     memset(&p, 0, sizeof(p));
     memset(&maps, 0, sizeof(maps));
     p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.H = s.H; p.I = s.I; p.R = (int)R;
+    p.g0 = all ? 0 : s.E_pub;
+    p.G = all ? s.E() : s.E_priv;
+    p.q_off = all ? s.E_pub : 0;
     p.bn_a = s.H % 256 == 0 ? 256 : 128;
     p.bn_b = s.I % 256 == 0 ? 256 : 128;
     p.offsets = c.offsets;

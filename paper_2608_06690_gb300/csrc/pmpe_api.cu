@@ -296,6 +296,48 @@ int pmpe_moe_backward_input(const pmpe_moe_desc *d, const void *dout, float *d_h
                : PMPE_ERR_CUDA;
 }
 
+size_t pmpe_moe_backward_step_workspace_size(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k)
+{
+    Shape s;
+    s.T = T; s.H = H; s.I = I; s.E_pub = E_pub; s.E_priv = E_priv; s.E_sh = E_shared; s.k = k; s.renorm = 1;
+    if (!shape_ok(s)) return 0;
+    return backward_step_workspace_bytes(s);
+}
+
+int pmpe_moe_backward_step(const pmpe_moe_desc *d, const void *dout, float *d_router_priv, float *d_gate_priv,
+                           float *d_up_priv, float *d_down_priv, float *d_hidden, void *bwd_workspace,
+                           size_t bwd_workspace_bytes, void *stream)
+{
+    // every argument is checked before the first CUDA call
+    if (!d) return PMPE_ERR_INVALID_ARG;
+    const Shape s = shape_of(d);
+    const void *need[] = {d_router_priv, d_gate_priv, d_up_priv, d_down_priv};
+    for (const void *q : need)
+        if (!q || !aligned16(q)) return PMPE_ERR_INVALID_ARG;
+    if (s.T > 0 && (!dout || !aligned16(dout) || !d_hidden || !aligned16(d_hidden))) return PMPE_ERR_INVALID_ARG;
+    if (d->unmasked_control == 1) return PMPE_ERR_UNSUPPORTED_SHAPE;
+    if (shape_ok(s) && s.T > 0 &&
+        (!bwd_workspace || bwd_workspace_bytes < backward_step_workspace_bytes(s) ||
+         ((uintptr_t)bwd_workspace & 255u)))
+        return PMPE_ERR_WORKSPACE;
+    Ctx c;
+    const int rc = make_ctx(d, stream, &c);
+    if (rc != PMPE_OK) return rc;
+    if (s.T == 0) {  // nothing routed: every parameter gradient is zero, d_hidden is empty
+        cudaStream_t st = (cudaStream_t)stream;
+        const size_t ih = (size_t)s.E_priv * s.I * s.H * sizeof(float);
+        cudaError_t err = cudaMemsetAsync(d_router_priv, 0, (size_t)s.E_priv * s.H * sizeof(float), st);
+        if (err == cudaSuccess) err = cudaMemsetAsync(d_gate_priv, 0, ih, st);
+        if (err == cudaSuccess) err = cudaMemsetAsync(d_up_priv, 0, ih, st);
+        if (err == cudaSuccess) err = cudaMemsetAsync(d_down_priv, 0, ih, st);
+        return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
+    }
+    return launch_backward_step(c, (const bf16 *)dout, d_router_priv, d_gate_priv, d_up_priv, d_down_priv, d_hidden,
+                                (uint8_t *)bwd_workspace) == cudaSuccess
+               ? PMPE_OK
+               : PMPE_ERR_CUDA;
+}
+
 int pmpe_moe_forward(const pmpe_moe_desc *d, void *stream)
 {
     return pmpe_moe_forward_stages(d, PMPE_STAGE_ALL, stream);

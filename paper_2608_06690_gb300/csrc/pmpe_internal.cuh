@@ -89,9 +89,20 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
 void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint32_t *offsets, int g0, int g1, int R,
                         int H, bf16 *rows, int num_sms, cudaStream_t st);
 cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz);
+constexpr int kMaxRouterSplits = 64;  // token ranges of the router weight gradient
+// The private router's weight gradient from dz (rows ld apart; DENY rows read
+// as zeros): token-range partials (part, router_wgrad_part_bytes) and their
+// fixed-order sum into d_router [E_priv, H]; active: kMaxRouterSplits words.
+size_t router_wgrad_part_bytes(const Shape &s);
+cudaError_t launch_router_wgrad(const Ctx &c, const float *dz, int ld, float *part, int *active, float *d_router);
 // Gradient of the layer's input (k_backward_input.cu): scratch bytes and launch.
 size_t backward_input_workspace_bytes(const Shape &s);
 cudaError_t launch_backward_input(const Ctx &c, const bf16 *dout, float *d_hidden, uint8_t *bws);
+// Both in one pass (k_backward_input.cu): the private gradients and the input
+// gradient from one set of row launches over all routed experts.
+size_t backward_step_workspace_bytes(const Shape &s);
+cudaError_t launch_backward_step(const Ctx &c, const bf16 *dout, float *d_router, float *d_gate, float *d_up,
+                                 float *d_down, float *d_hidden, uint8_t *bws);
 // Its tensor-core GEMMs (k_backward_tc.cu): rows of the padded layout, the
 // dL/da and gate/up recompute launches, and the weight-gradient launch.
 size_t backward_padded_rows(const Shape &s);
@@ -111,8 +122,11 @@ cudaError_t launch_rows_z(const Ctx &c, const RowsGroups &g, const bf16 *d, uint
 cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uint64_t a_rows, const bf16 *zpad,
                            bf16 *dgu, bf16 *wact, float *gw_part);
 cudaError_t launch_rows_da(const Ctx &c, const RowsGroups &g, const bf16 *dgu, bf16 *da);
+// all == null: the operands use the private experts' own padded layout and
+// dout_rows starts at the first private slot; otherwise the padded layout of
+// all routed experts (`all`) and dout_rows indexed by dispatch slot.
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
-                                  float *d_gate, float *d_up, float *d_down);
+                                  float *d_gate, float *d_up, float *d_down, const RowsGroups *all = nullptr);
 // Gate/up and down in one persistent launch (down tiles wait for their
 // activation rows); zero_ready clears the readiness counters first.
 cudaError_t launch_experts(const Ctx &c, bool zero_ready);

@@ -60,11 +60,20 @@ def kernels_per_backward_input(shape) -> int:
     router's softmax gradient and the per-token sum."""
     return 6 + (3 if shape.E_sh > 0 else 0)
 
+
+def kernels_per_backward_step(shape) -> int:
+    """Kernels one combined backward launches: the dout row gather, Z, the
+    gate/up recompute and dA over the routed experts (the same three over the
+    shared experts, if any), the router's dz, its weight-gradient partials
+    and their sum, the expert weight-gradient GEMM and the per-token sum."""
+    return 8 + (3 if shape.E_sh > 0 else 0)
+
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
             "pmpe_status_string", "pmpe_moe_forward_noalloc", "pmpe_selftest_wait_timeout",
             "pmpe_policy_from_requests", "pmpe_moe_backward_workspace_size", "pmpe_moe_backward_private",
-            "pmpe_moe_backward_input_workspace_size", "pmpe_moe_backward_input")
+            "pmpe_moe_backward_input_workspace_size", "pmpe_moe_backward_input",
+            "pmpe_moe_backward_step_workspace_size", "pmpe_moe_backward_step")
 
 # Bytes of the library's static scratch array used by pmpe_moe_forward_noalloc.
 STATIC_SCRATCH_BYTES = 32 << 20
@@ -114,6 +123,10 @@ _lib.pmpe_moe_backward_input_workspace_size.restype = ctypes.c_size_t
 _lib.pmpe_moe_backward_input_workspace_size.argtypes = [ctypes.c_int] * 7
 _lib.pmpe_moe_backward_input.restype = ctypes.c_int
 _lib.pmpe_moe_backward_input.argtypes = [ctypes.POINTER(MoeDesc), _vp, _vp, _vp, ctypes.c_size_t, _vp]
+_lib.pmpe_moe_backward_step_workspace_size.restype = ctypes.c_size_t
+_lib.pmpe_moe_backward_step_workspace_size.argtypes = [ctypes.c_int] * 7
+_lib.pmpe_moe_backward_step.restype = ctypes.c_int
+_lib.pmpe_moe_backward_step.argtypes = [ctypes.POINTER(MoeDesc)] + [_vp] * 7 + [ctypes.c_size_t, _vp]
 _lib.pmpe_policy_from_requests.restype = ctypes.c_int
 _lib.pmpe_policy_from_requests.argtypes = [_vp, _vp, ctypes.c_int, ctypes.c_int, _vp, _vp]
 _lib.pmpe_selftest_wait_timeout.restype = ctypes.c_int
@@ -324,6 +337,31 @@ class MoeLayer:
                                               _ptr(g["d_up"]), _ptr(g["d_down"]), _ptr(bws), bws.numel(),
                                               _stream(stream)), "pmpe_moe_backward_private")
         return g
+
+    def backward(self, hidden, policy, dout, topk_idx=None, topk_w=None, stream=None):
+        """Both backward results of the forward just run with the same hidden
+        states and policy on the same stream, in one pass: the private
+        parameters' gradients (as backward_private) and the gradient of the
+        hidden states (as backward_input), each bitwise as those calls give."""
+        T = hidden.shape[0]
+        s = self._shape_T(T)
+        assert dout.is_contiguous() and dout.dtype == torch.bfloat16 and dout.shape == (T, s.H)
+        dev = hidden.device
+        g = {n: torch.empty(shp, dtype=torch.float32, device=dev) for n, shp in private_gradient_shapes(s).items()}
+        d_hidden = torch.empty((T, s.H), dtype=torch.float32, device=dev)
+        nb = _lib.pmpe_moe_backward_step_workspace_size(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k)
+        if nb == 0:
+            raise PmpeError(ERR_UNSUPPORTED_SHAPE, "pmpe_moe_backward_step_workspace_size")
+        if self._bws is None or self._bws.numel() < nb:
+            self._bws = torch.empty(nb, dtype=torch.uint8, device=dev)
+        bws = self._bws
+        if topk_idx is None and topk_w is None:
+            topk_idx, topk_w = self._route_out
+        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w)
+        _check(_lib.pmpe_moe_backward_step(ctypes.byref(desc), _ptr(dout), _ptr(g["d_router"]), _ptr(g["d_gate"]),
+                                           _ptr(g["d_up"]), _ptr(g["d_down"]), _ptr(d_hidden), _ptr(bws),
+                                           bws.numel(), _stream(stream)), "pmpe_moe_backward_step")
+        return g, d_hidden
 
     def backward_input(self, hidden, policy, dout, topk_idx=None, topk_w=None, stream=None) -> torch.Tensor:
         """Gradient of sum(dout * out) with respect to the hidden states [T, H]

@@ -261,6 +261,54 @@ def test_backward_input_validation_rejects_before_any_cuda_call(pmpe):
     assert rc(bws=ctypes.c_void_p(p.addr + 16)) == pmpe.ERR_WORKSPACE
 
 
+def test_backward_step_validation_rejects_before_any_cuda_call(pmpe):
+    """The combined backward checks its gradient buffers, dout, d_hidden, the
+    control flag and its scratch size on the host; fake device pointers are
+    never dereferenced."""
+    from paper_2608_06690_gb300.inputs import LayerShape
+    lib = pmpe._lib
+    shape = LayerShape(64, 256, 128, 8, 4, 1, 2, True)
+    need = lib.pmpe_moe_backward_step_workspace_size(64, 256, 128, 8, 4, 1, 2)
+    assert need >= 256 and need % 256 == 0
+    assert lib.pmpe_moe_backward_step_workspace_size(64, 192, 128, 8, 4, 1, 2) == 0   # H % 128
+    assert lib.pmpe_moe_backward_step_workspace_size(0, 256, 128, 8, 4, 1, 2) == 256  # empty batch: the floor
+    # it holds the input gradient's scratch and more
+    assert need > lib.pmpe_moe_backward_input_workspace_size(64, 256, 128, 8, 4, 1, 2)
+
+    class Fake:
+        def __init__(self, addr):
+            self.addr = addr
+
+        def data_ptr(self):
+            return self.addr
+
+        def numel(self):
+            return 1 << 40
+
+        def element_size(self):
+            return 1
+
+    p = Fake(0x10000000)
+    W = {n: p for n in ("router_pub", "router_priv", "gate_pub", "up_pub", "down_pub", "gate_priv", "up_priv",
+                        "down_priv", "gate_sh", "up_sh", "down_sh")}
+    v = ctypes.c_void_p(p.addr)
+
+    def rc(desc_ok=True, dout=v, grads=(v, v, v, v), dh=v, bws=v, nbytes=need, unmasked=False):
+        d = pmpe.make_desc(shape, W, p, None, p, p, unmasked_control=unmasked)
+        return lib.pmpe_moe_backward_step(ctypes.byref(d) if desc_ok else None, dout, *grads, dh, bws, nbytes, None)
+
+    assert rc(desc_ok=False) == pmpe.ERR_INVALID_ARG
+    assert rc(dout=None) == pmpe.ERR_INVALID_ARG
+    assert rc(grads=(v, None, v, v)) == pmpe.ERR_INVALID_ARG
+    assert rc(grads=(v, v, v, ctypes.c_void_p(p.addr + 4))) == pmpe.ERR_INVALID_ARG
+    assert rc(dh=None) == pmpe.ERR_INVALID_ARG
+    assert rc(dh=ctypes.c_void_p(p.addr + 8)) == pmpe.ERR_INVALID_ARG
+    assert rc(unmasked=True) == pmpe.ERR_UNSUPPORTED_SHAPE
+    assert rc(bws=None) == pmpe.ERR_WORKSPACE
+    assert rc(nbytes=need - 256) == pmpe.ERR_WORKSPACE
+    assert rc(bws=ctypes.c_void_p(p.addr + 16)) == pmpe.ERR_WORKSPACE
+
+
 def test_optimizer_partition_matches_the_papers_trainable_parameter_counts(pmpe):
     """G2 optimizer partition (Sec. 2.2): the backward produces gradients for
     the private router and private experts only, and over the paper's two
