@@ -404,6 +404,39 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     bst_ms = [x.elapsed_time(y) for x, y in bst_ms]
 
+    # ---- a training step of the layer: forward, then both backward results;
+    # with the forward saving its gate/up accumulators for the backward, and
+    # without (the backward recomputes them)
+    def timed(fn, n):
+        evs = []
+        for _ in range(n):
+            flush.zero_()
+            a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a_ev.record(stream)
+            fn()
+            b_ev.record(stream)
+            evs.append((a_ev, b_ev))
+        torch.cuda.synchronize(dev)
+        return float(np.mean([x.elapsed_time(y) for x, y in evs]))
+
+    def train_step(save):
+        layer.forward(h, pol, out=out, save_for_backward=save)
+        layer.backward(h, pol, dout)
+
+    def fwd_only(save):
+        layer.forward(h, pol, out=out, save_for_backward=save)
+
+    train = {}
+    for save in (True, False):
+        for _ in range(2):
+            train_step(save)
+        key = "saved_gate_up" if save else "recomputed_gate_up"
+        train[key] = {"step_ms": timed(lambda: train_step(save), args.steps),
+                      "forward_ms": timed(lambda: fwd_only(save), args.steps)}
+        train[key]["backward_ms"] = timed(lambda: layer.backward(h, pol, dout), args.steps)
+    train["saved_bytes"] = s.T * s.k * 2 * s.I * 4
+    train["l2"] = "flushed before every step"
+
     # ---- end to end through the public API with host buffers, pipelined as a
     # serving loop would run it: step i+1's inputs are copied in (copy-in
     # stream) while step i computes, and step i's result is copied out
@@ -530,6 +563,7 @@ def run_ours(args):
         "backward_private": backward,
         "backward_input": backward_in,
         "backward_step": backward_step,
+        "training_step": train,
         "expert_load": {"touched": work["touched_experts"], "max_rows": int(counts.max()),
                         "mean_rows_public": float(counts[:s.E_pub].mean()),
                         "mean_rows_private": float(counts[s.E_pub:].mean())},

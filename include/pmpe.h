@@ -119,6 +119,14 @@ typedef struct pmpe_moe_desc {
      * lists to fit in shared memory: ceil(E_pub/32) + ceil(E_priv/32) <= 16
      * and that count * k <= 96; PMPE_ERR_UNSUPPORTED_SHAPE otherwise. */
     int unmasked_control;
+
+    /* Optional, for training: [T*k, 2I] FP32, 16-byte aligned, or NULL.  When
+     * set, the forward also writes each dispatch row's gate and up
+     * pre-activations G | U (the FP32 accumulators its SwiGLU reads), and the
+     * backward calls given the same descriptor read them instead of
+     * recomputing the gate/up GEMM.  Their results are then bitwise those of
+     * the recomputation. */
+    float *saved_gu;
 } pmpe_moe_desc;
 
 /* Bytes of device workspace pmpe_moe_forward() needs for this shape.

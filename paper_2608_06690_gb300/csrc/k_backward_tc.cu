@@ -232,6 +232,38 @@ __device__ __forceinline__ int2 group_weights(const RowsParams &p, int q)
     return e >= p.E_pub ? make_int2(1, e - p.E_pub) : make_int2(0, e);
 }
 
+// SwiGLU backward of one element, from the gate and up accumulators g, u,
+// the row's Z value z and routing weight w: a = bf16(silu(g) u) with the
+// forward's arithmetic, dG = w z u silu'(g), dU = w z silu(g), and w a.
+__device__ __forceinline__ void swiglu_bwd(float g, float u, float z, float w, float &a, float &dg, float &du,
+                                           float &wa)
+{
+    const float den = 1.f + __expf(-g);
+    const float silu = __fdividef(g, den);
+    a = __bfloat162float(__float2bfloat16_rn(silu * u));
+    const float sg = __fdividef(1.f, den);
+    const float wz = w * z;
+    dg = wz * u * sg * (1.f + g * (1.f - sg));
+    du = wz * silu;
+    wa = w * a;
+}
+
+// dL/dw over 32 columns of a row: the products z a of four consecutive
+// columns summed pairwise, then those eight sums pairwise.  The order is the
+// butterfly of eight lanes holding four columns each, so a thread holding all
+// 32 (the gate/up epilogue) and a warp holding the row's columns four per
+// lane (bwd_swiglu_saved_kernel) get the same bits.
+__device__ __forceinline__ float chunk_tree_sum(const float (&q)[32])
+{
+    float s[8];
+#pragma unroll
+    for (int l = 0; l < 8; ++l)
+        s[l] = __fadd_rn(__fadd_rn(q[4 * l], q[4 * l + 1]), __fadd_rn(q[4 * l + 2], q[4 * l + 3]));
+    const float t0 = __fadd_rn(s[0], s[1]), t1 = __fadd_rn(s[2], s[3]);
+    const float t2 = __fadd_rn(s[4], s[5]), t3 = __fadd_rn(s[6], s[7]);
+    return __fadd_rn(__fadd_rn(t0, t1), __fadd_rn(t2, t3));
+}
+
 template <int kMode>
 __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsParams p, const __grid_constant__ RowsMaps maps)
 {
@@ -390,6 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
                     tmem_ld_wait();
                     const __nv_bfloat162 *zb = reinterpret_cast<const __nv_bfloat162 *>(zq);
                     uint32_t pg[16], pu[16], pa[16];
+                    float zq_a[32];
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
                         const float2 z2 = __bfloat1622float2(zb[i]);
@@ -397,21 +430,17 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
 #pragma unroll
                         for (int h = 0; h < 2; ++h) {
                             const int j = 2 * i + h;
+                            float a;
                             const float z = h ? z2.y : z2.x;
-                            const float den = 1.f + __expf(-g[j]);
-                            const float silu = __fdividef(g[j], den);  // the forward's silu(g) u, same arithmetic
-                            const float a = __bfloat162float(__float2bfloat16_rn(silu * u[j]));
-                            const float sg = __fdividef(1.f, den);
-                            gw += z * a;
-                            const float wz = w * z;
-                            dg[h] = valid ? wz * u[j] * sg * (1.f + g[j] * (1.f - sg)) : 0.f;
-                            du[h] = valid ? wz * silu : 0.f;
-                            wa[h] = valid ? w * a : 0.f;
+                            swiglu_bwd(g[j], u[j], z, w, a, dg[h], du[h], wa[h]);
+                            zq_a[j] = __fmul_rn(z, a);
+                            if (!valid) dg[h] = du[h] = wa[h] = 0.f;
                         }
                         pg[i] = pack_bf16x2(dg[0], dg[1]);
                         pu[i] = pack_bf16x2(du[0], du[1]);
                         pa[i] = pack_bf16x2(wa[0], wa[1]);
                     }
+                    gw = __fadd_rn(gw, chunk_tree_sum(zq_a));
                     out.put(lane, pg, &maps.out0, t.n0 + c * 32, orow);
                     out.put(lane, pu, &maps.out0, p.I + t.n0 + c * 32, orow);
                     if (p.wact && !p.shared_T && p.g0 + t.q >= p.E_pub)
@@ -432,6 +461,82 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_rows_tc_kernel(const RowsPara
     if (warp == 1) {
         tc_fence_after();
         tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+// ------------------------------------------------------------- saved G | U
+
+// The gate/up launch's outputs from the forward's saved accumulators G | U
+// ([R][2I] FP32) instead of a recomputing GEMM: one warp per routed row and
+// 128-column tile, four columns per lane (coalesced rows), with the
+// epilogue's per-element arithmetic and its dL/dw summation order
+// (chunk_tree_sum, then the four 32-column chunks in order), so [dG | dU],
+// w act and the dL/dw partials are bitwise those of kRowsGU.  Tiles and the
+// padded layout come from the same group table; padded tail rows are written
+// as zeros.
+__global__ void __launch_bounds__(256) bwd_swiglu_saved_kernel(const RowsParams p, const float *saved_gu, bf16 *dgu,
+                                                               bf16 *wact)
+{
+    __shared__ GroupTable gt;
+    pdl_wait();
+    const int nt = p.I / 128;
+    build_groups(gt, p.offsets, p.g0, p.G, p.R, 0, nt, 0);
+    const int total = gt.tiles[p.G];
+    const int p0 = (int)min(p.offsets[p.g0], (uint32_t)p.R);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+        const RowsTile t = decode_rows(gt, p.G, nt, 128, tile, 0);
+        const bool wa_out = p.wact && p.g0 + t.q >= p.E_pub;
+        for (int r = warp; r < BM; r += nwarps) {
+            const bool valid = r < t.rows;  // warp-uniform
+            const int prow = gt.off[t.q] + t.m0 + r;
+            const int orow = gt.pad[t.q] + t.m0 + r;
+            const int col = t.n0 + 4 * lane;
+            float g[4] = {0.f, 0.f, 0.f, 0.f}, u[4] = {0.f, 0.f, 0.f, 0.f}, z[4] = {0.f, 0.f, 0.f, 0.f};
+            float w = 0.f;
+            if (valid) {
+                const float *grow = saved_gu + (size_t)(p0 + prow) * 2 * p.I;
+                const float4 gv = *reinterpret_cast<const float4 *>(grow + col);
+                const float4 uv = *reinterpret_cast<const float4 *>(grow + p.I + col);
+                const uint2 zv = *reinterpret_cast<const uint2 *>(p.zpad + (size_t)orow * p.I + col);
+                g[0] = gv.x; g[1] = gv.y; g[2] = gv.z; g[3] = gv.w;
+                u[0] = uv.x; u[1] = uv.y; u[2] = uv.z; u[3] = uv.w;
+                const float2 z01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&zv.x));
+                const float2 z23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&zv.y));
+                z[0] = z01.x; z[1] = z01.y; z[2] = z23.x; z[3] = z23.y;
+                w = p.w_of_slot[p0 + prow];
+            }
+            float dg[4], du[4], wa[4], q[4];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                float a;
+                swiglu_bwd(g[h], u[h], z[h], w, a, dg[h], du[h], wa[h]);
+                q[h] = __fmul_rn(z[h], a);
+                if (!valid) dg[h] = du[h] = wa[h] = 0.f;
+            }
+            bf16 *dst = dgu + (size_t)orow * 2 * p.I + col;
+            *reinterpret_cast<uint2 *>(dst) = make_uint2(pack_bf16x2(dg[0], dg[1]), pack_bf16x2(dg[2], dg[3]));
+            *reinterpret_cast<uint2 *>(dst + p.I) = make_uint2(pack_bf16x2(du[0], du[1]), pack_bf16x2(du[2], du[3]));
+            if (wa_out)
+                *reinterpret_cast<uint2 *>(wact + (size_t)orow * p.I + col) =
+                    make_uint2(pack_bf16x2(wa[0], wa[1]), pack_bf16x2(wa[2], wa[3]));
+            // the 32-column chunk sums in chunk_tree_sum's order: four columns in
+            // the lane, then the butterfly over the chunk's eight lanes
+            float sum = __fadd_rn(__fadd_rn(q[0], q[1]), __fadd_rn(q[2], q[3]));
+            sum = __fadd_rn(sum, __shfl_xor_sync(~0u, sum, 1));
+            sum = __fadd_rn(sum, __shfl_xor_sync(~0u, sum, 2));
+            sum = __fadd_rn(sum, __shfl_xor_sync(~0u, sum, 4));
+            const float c0 = __shfl_sync(~0u, sum, 0), c1 = __shfl_sync(~0u, sum, 8);
+            const float c2 = __shfl_sync(~0u, sum, 16), c3 = __shfl_sync(~0u, sum, 24);
+            if (lane == 0 && valid && p.gw_part) {
+                float gw = 0.f;
+                gw = __fadd_rn(gw, c0);
+                gw = __fadd_rn(gw, c1);
+                gw = __fadd_rn(gw, c2);
+                gw = __fadd_rn(gw, c3);
+                p.gw_part[(size_t)(p0 + prow) * nt + t.n_tile] = gw;
+            }
+        }
     }
 }
 
@@ -714,6 +819,14 @@ cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uin
 {
     const Shape &s = c.s;
     RowsParams p = rows_params(c, g);
+    if (c.saved_gu && !g.shared_T) {  // the forward saved G | U of the routed rows
+        p.K = s.H; p.N = s.I; p.bn = 128;
+        p.zpad = zpad;
+        p.gw_part = gw_part;
+        p.wact = wact ? 1 : 0;
+        return launch_pdl(bwd_swiglu_saved_kernel, dim3(c.num_sms * 4), dim3(256), 0, c.stream, p,
+                          (const float *)c.saved_gu, dgu, wact);
+    }
     RowsMaps maps;
     memset(&maps, 0, sizeof(maps));
     p.K = s.H; p.N = s.I; p.bn = 128;

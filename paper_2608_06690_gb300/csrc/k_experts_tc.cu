@@ -76,6 +76,9 @@ struct TcParams {
     // activations are stored (zeroed before the launch)
     uint32_t *ready;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
+    // optional [R][2I] FP32: the routed rows' gate and up accumulators G | U,
+    // saved for the backward (gu_save map for whole 32-row blocks)
+    float *saved_gu;
 };
 
 struct TcMaps {  // [phase]
@@ -83,6 +86,7 @@ struct TcMaps {  // [phase]
     CUtensorMap a_routed[2], a_shared[2];
     CUtensorMap b0[2][3];  // per pool [pub, priv, shared]: gate (gate/up) or down
     CUtensorMap b1[2][3];  // up (gate/up)
+    CUtensorMap gu_save;   // saved_gu, 16 x 32 FP32 boxes, 64-byte swizzle
 };
 
 // ------------------------------------------------------------- tile list
@@ -366,6 +370,43 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
 #pragma unroll
                     for (int i = 0; i < 16; ++i)
                         pk[i] = pack_bf16x2(silu_mul(gv[2 * i], uv[2 * i]), silu_mul(gv[2 * i + 1], uv[2 * i + 1]));
+                    if (p.saved_gu && !t.shared) {
+                        // G and U of these 32 columns, as FP32, for the backward
+                        const int y0 = t.row_base + t.m0 + quarter * 32;
+                        if (full_block) {
+#pragma unroll
+                            for (int b = 0; b < 4; ++b) {  // G lo, G hi, U lo, U hi: 16 columns each
+                                const float *src = (b < 2 ? gv : uv) + (b & 1) * 16;
+                                const uint32_t sbuf = out_base + (uint32_t)(out_parity * kOutBufBytes);
+                                if (lane == 0) bulk_wait_read<1>();
+                                __syncwarp();
+#pragma unroll
+                                for (int j = 0; j < 4; ++j) {
+                                    const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
+                                    asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr),
+                                                 "f"(src[4 * j]), "f"(src[4 * j + 1]), "f"(src[4 * j + 2]),
+                                                 "f"(src[4 * j + 3])
+                                                 : "memory");
+                                }
+                                fence_proxy_async_smem();
+                                __syncwarp();
+                                if (lane == 0) {
+                                    tma_store_2d(&maps.gu_save, sbuf, (b < 2 ? 0 : p.I) + t.n0 + c * 32 + (b & 1) * 16,
+                                                 y0);
+                                    bulk_commit();
+                                }
+                                out_parity ^= 1;
+                            }
+                        } else if (valid) {
+                            float4 *gd = reinterpret_cast<float4 *>(p.saved_gu + (size_t)grow * 2 * p.I + t.n0 + c * 32);
+                            float4 *ud = gd + p.I / 4;
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                gd[i] = make_float4(gv[4 * i], gv[4 * i + 1], gv[4 * i + 2], gv[4 * i + 3]);
+                                ud[i] = make_float4(uv[4 * i], uv[4 * i + 1], uv[4 * i + 2], uv[4 * i + 3]);
+                            }
+                        }
+                    }
                 } else {
                     float v[32];
                     tmem_ld32(taddr + c * 32, v);
@@ -515,6 +556,11 @@ cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
     p.status = c.audit.status;
     bool ok = true;
     for (int ph = 0; ph < nph; ++ph) ok &= fill_phase(c, modes[ph], ph, p, maps);
+    if (c.saved_gu && modes[0] == kGateUp) {
+        p.saved_gu = c.saved_gu;
+        ok &= encode_2d_f32(&maps.gu_save, c.saved_gu, 2 * (uint64_t)s.I, (uint64_t)s.T * s.k, 16, 32,
+                            CU_TENSOR_MAP_SWIZZLE_64B);
+    }
     if (!ok) return cudaErrorInvalidValue;
     static std::atomic<int> smem_limit[64];
     cudaError_t err = ensure_dynamic_smem(expert_gemm_tc_kernel, kDynSmem, smem_limit);

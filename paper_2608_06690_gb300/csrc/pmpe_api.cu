@@ -110,7 +110,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     }
     const void *all[] = {d->hidden, d->w_router_pub, d->w_router_priv, d->w_gate_pub, d->w_up_pub, d->w_down_pub,
                          d->w_gate_priv, d->w_up_priv, d->w_down_priv, d->w_gate_sh, d->w_up_sh, d->w_down_sh,
-                         d->out, d->topk_idx, d->topk_w, d->audit, d->workspace};
+                         d->out, d->topk_idx, d->topk_w, d->audit, d->workspace, d->saved_gu};
     for (const void *q : all)
         if (!aligned16(q)) return PMPE_ERR_UNSUPPORTED_SHAPE;
     pmpe_workspace_layout L;
@@ -151,6 +151,7 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->y_sh = s.E_sh > 0 ? (bf16 *)(ws + L.y_sh) : nullptr;
     c->stream = (cudaStream_t)stream;
     c->unmasked = d->unmasked_control;
+    c->saved_gu = d->saved_gu;
     if (s.T == 0) return PMPE_OK;  // a no-op: no device query, no launch
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PMPE_ERR_CUDA;

@@ -61,6 +61,7 @@ struct Ctx {
     cudaStream_t stream;
     int num_sms;
     int unmasked;  // the soft-router control: no hard mask (a negative control, not the method)
+    float *saved_gu;  // optional [T*k][2I] FP32 G | U written by the forward, read by the backward
 };
 
 int compute_layout(const Shape &s, pmpe_workspace_layout *L);

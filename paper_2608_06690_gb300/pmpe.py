@@ -91,7 +91,8 @@ class MoeDesc(ctypes.Structure):
                 ("w_gate_priv", _vp), ("w_up_priv", _vp), ("w_down_priv", _vp),
                 ("w_gate_sh", _vp), ("w_up_sh", _vp), ("w_down_sh", _vp),
                 ("out", _vp), ("topk_idx", _vp), ("topk_w", _vp), ("audit", _vp),
-                ("workspace", _vp), ("workspace_bytes", ctypes.c_size_t), ("unmasked_control", ctypes.c_int)]
+                ("workspace", _vp), ("workspace_bytes", ctypes.c_size_t), ("unmasked_control", ctypes.c_int),
+                ("saved_gu", _vp)]
 
 
 class WorkspaceLayout(ctypes.Structure):
@@ -237,7 +238,7 @@ def selftest_wait_timeout(status, limit_us: int, stream=None):
 
 
 def make_desc(s: LayerShape, weights: dict, hidden, policy, out, workspace, topk_idx=None, topk_w=None,
-              audit=None, unmasked_control: bool = False) -> MoeDesc:
+              audit=None, unmasked_control: bool = False, saved_gu=None) -> MoeDesc:
     """Fill the C descriptor from torch tensors (device pointers only)."""
     W = weights
     return MoeDesc(s.T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, int(bool(s.renormalize)),
@@ -248,7 +249,7 @@ def make_desc(s: LayerShape, weights: dict, hidden, policy, out, workspace, topk
                    _ptr(W.get("gate_sh")), _ptr(W.get("up_sh")), _ptr(W.get("down_sh")),
                    _ptr(out), _ptr(topk_idx), _ptr(topk_w), _ptr(audit),
                    _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
-                   int(bool(unmasked_control)))
+                   int(bool(unmasked_control)), _ptr(saved_gu))
 
 
 def forward_desc(desc: MoeDesc, stages: int = STAGE_ALL, stream=None):
@@ -286,6 +287,8 @@ class MoeLayer:
         self._ws = workspace if workspace is not None else Workspace(self.device)
         self._bws = None
         self._route_out = (None, None)  # the last forward's caller-owned route outputs
+        self._saved_gu = None           # the last forward's saved G | U, when it saved them
+        self._saved_buf = None
 
     def workspace(self, T: int) -> torch.Tensor:
         return self._ws.get(workspace_size(self._shape_T(T)))
@@ -295,10 +298,13 @@ class MoeLayer:
         return LayerShape(T, s.H, s.I, s.E_pub, s.E_priv, s.E_sh, s.k, s.renormalize)
 
     def forward(self, hidden, policy, out=None, topk_idx=None, topk_w=None, audit=None, stages=STAGE_ALL,
-                stream=None, unmasked_control: bool = False):
+                stream=None, unmasked_control: bool = False, save_for_backward: bool = False):
         """Enqueue the layer on ``stream`` (default: the current stream).
         ``unmasked_control`` runs the paper's soft-router control instead of
-        the method: routing over the concatenated pool without the hard mask."""
+        the method: routing over the concatenated pool without the hard mask.
+        ``save_for_backward`` also keeps the routed rows' gate and up
+        accumulators ([T k, 2I] FP32, owned by the layer), which the backward
+        calls after this forward then read instead of recomputing them."""
         T = hidden.shape[0]
         s = self._shape_T(T)
         assert hidden.is_contiguous() and hidden.dtype == torch.bfloat16 and hidden.shape == (T, s.H)
@@ -306,10 +312,17 @@ class MoeLayer:
             assert policy.dtype == torch.uint8 and policy.numel() == T and policy.is_contiguous()
         if out is None:
             out = torch.empty_like(hidden)
+        saved = None
+        if save_for_backward:
+            n = T * s.k * 2 * s.I
+            if self._saved_buf is None or self._saved_buf.numel() < n:
+                self._saved_buf = torch.empty(max(n, 4), dtype=torch.float32, device=hidden.device)
+            saved = self._saved_buf
         desc = make_desc(s, self.weights, hidden, policy, out, self.workspace(T), topk_idx, topk_w, audit,
-                         unmasked_control)
+                         unmasked_control, saved)
         forward_desc(desc, stages, stream)
         self._route_out = (topk_idx, topk_w)
+        self._saved_gu = saved
         return out
 
     def backward_private(self, hidden, policy, dout, topk_idx=None, topk_w=None, stream=None) -> dict:
@@ -332,7 +345,8 @@ class MoeLayer:
         if topk_idx is None and topk_w is None:
             topk_idx, topk_w = self._route_out
         # the descriptor's output pointer is never written by the backward
-        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w)
+        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w,
+                         saved_gu=self._saved_gu)
         _check(_lib.pmpe_moe_backward_private(ctypes.byref(desc), _ptr(dout), _ptr(g["d_router"]), _ptr(g["d_gate"]),
                                               _ptr(g["d_up"]), _ptr(g["d_down"]), _ptr(bws), bws.numel(),
                                               _stream(stream)), "pmpe_moe_backward_private")
@@ -357,7 +371,8 @@ class MoeLayer:
         bws = self._bws
         if topk_idx is None and topk_w is None:
             topk_idx, topk_w = self._route_out
-        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w)
+        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w,
+                         saved_gu=self._saved_gu)
         _check(_lib.pmpe_moe_backward_step(ctypes.byref(desc), _ptr(dout), _ptr(g["d_router"]), _ptr(g["d_gate"]),
                                            _ptr(g["d_up"]), _ptr(g["d_down"]), _ptr(d_hidden), _ptr(bws),
                                            bws.numel(), _stream(stream)), "pmpe_moe_backward_step")
@@ -381,7 +396,8 @@ class MoeLayer:
         bws = self._bws
         if topk_idx is None and topk_w is None:
             topk_idx, topk_w = self._route_out
-        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w)
+        desc = make_desc(s, self.weights, hidden, policy, dout, self.workspace(T), topk_idx, topk_w,
+                         saved_gu=self._saved_gu)
         _check(_lib.pmpe_moe_backward_input(ctypes.byref(desc), _ptr(dout), _ptr(d_hidden), _ptr(bws), bws.numel(),
                                             _stream(stream)), "pmpe_moe_backward_input")
         return d_hidden

@@ -88,3 +88,56 @@ def test_full_size_combined_backward_is_bitwise_the_two_separate_passes(name):
     for n in GRADS:
         assert torch.equal(g[n], g_sep[n]), n
     assert torch.equal(dh, dh_sep)
+
+
+def _all_three(layer, h, pol, dout, save):
+    out = layer.forward(h, pol, save_for_backward=save).clone()
+    gp = {n: v.clone() for n, v in layer.backward_private(h, pol, dout).items()}
+    di = layer.backward_input(h, pol, dout).clone()
+    g, dh = layer.backward(h, pol, dout)
+    torch.cuda.synchronize()
+    return out, gp, di, g, dh
+
+
+@pytest.mark.parametrize("name", ["renorm_ragged", "pool_softmax_with_shared", "sparse_pool_empty_experts",
+                                  "single_token"])
+def test_saved_gate_up_accumulators_give_bitwise_the_recomputed_backward(name):
+    """A forward that saves its gate/up accumulators G | U gives the same
+    output, and every backward call that reads them instead of recomputing
+    the gate/up GEMM gives bitwise the recomputation's results."""
+    shape, seed, policy = CASES[name]
+    w, h, pol = make_layer(shape, seed, policy=policy)
+    wd, hd, pd = to_device(w, h, pol)
+    layer = pmpe.MoeLayer(shape, wd)
+    dout = _dout(shape, seed + 1)
+    ref = _all_three(layer, hd, pd, dout, save=False)
+    got = _all_three(layer, hd, pd, dout, save=True)
+    assert torch.equal(got[0].view(torch.int16), ref[0].view(torch.int16))
+    for i in (1, 3):
+        for n in GRADS:
+            assert torch.equal(got[i][n], ref[i][n]), (i, n)
+    assert torch.equal(got[2], ref[2]) and torch.equal(got[4], ref[4])
+    # the buffer holds G | U of every dispatch row (some value written everywhere)
+    R = shape.T * shape.k
+    sg = layer._saved_buf[:R * 2 * shape.I].view(R, 2 * shape.I)
+    assert torch.all(torch.isfinite(sg))
+
+
+@pytest.mark.parametrize("name", ["qwen3_prefill", "deepseek_v2_lite"])
+def test_full_size_saved_gate_up_accumulators_give_bitwise_the_recomputed_backward(name):
+    cfg = CONFIGS[name]
+    s = cfg.shape
+    w = inp.make_weights(s, cfg.seed, device="cuda", skew=cfg.skew)
+    h = inp.make_hidden(s, cfg.seed, device="cuda", skew=cfg.skew)
+    pd = cfg.policy(s.T).cuda()
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(19)
+    dout = torch.randn((s.T, s.H), generator=gen, device="cuda").to(torch.bfloat16)
+    layer = pmpe.MoeLayer(s, w)
+    ref = _all_three(layer, h, pd, dout, save=False)
+    got = _all_three(layer, h, pd, dout, save=True)
+    assert torch.equal(got[0].view(torch.int16), ref[0].view(torch.int16))
+    for i in (1, 3):
+        for n in GRADS:
+            assert torch.equal(got[i][n], ref[i][n]), (i, n)
+    assert torch.equal(got[2], ref[2]) and torch.equal(got[4], ref[4])
