@@ -153,6 +153,8 @@ def test_validation_rejects_before_any_cuda_call(pmpe):
     assert lib.pmpe_policy_resolve(None, 0, None, None) == pmpe.OK
     assert lib.pmpe_audit_reset(None, 4, 4, None) == pmpe.ERR_INVALID_ARG
     assert lib.pmpe_audit_read(None, 4, 4, None, None, 10) == pmpe.ERR_INVALID_ARG
+    d = pmpe.make_desc(ok, W, p, None, p, p, saved_gu=Fake(0x10000004))
+    assert lib.pmpe_moe_forward(ctypes.byref(d), None) == pmpe.ERR_UNSUPPORTED_SHAPE     # saved G | U misaligned
     d = pmpe.make_desc(ok, W, p, None, p, p)
     d.unmasked_control = 2
     assert lib.pmpe_moe_forward(ctypes.byref(d), None) == pmpe.ERR_INVALID_ARG          # flag is 0 or 1
