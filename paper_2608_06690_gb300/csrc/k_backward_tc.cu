@@ -824,7 +824,7 @@ cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uin
         p.zpad = zpad;
         p.gw_part = gw_part;
         p.wact = wact ? 1 : 0;
-        return launch_pdl(bwd_swiglu_saved_kernel, dim3(c.num_sms * 4), dim3(256), 0, c.stream, p,
+        return launch_pdl(bwd_swiglu_saved_kernel, dim3(c.num_sms * 8), dim3(256), 0, c.stream, p,
                           (const float *)c.saved_gu, dgu, wact);
     }
     RowsMaps maps;
