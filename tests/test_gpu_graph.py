@@ -68,7 +68,8 @@ def test_48_layer_stack_replays_bitwise_from_a_cuda_graph():
 def test_training_step_with_private_backward_replays_bitwise_from_a_cuda_graph():
     """One training step of a two-layer stack captured into one CUDA graph:
     the layers' forwards (the second fed the first one's output), then the
-    top layer's private gradients and input gradient in one combined pass;
+    top layer's private gradients and input gradient in one combined pass
+    from the gate/up accumulators its forward saved;
     that input gradient in BF16 is the upstream gradient of the lower layer's
     private-branch backward.
     Each layer keeps its own workspace, which holds that layer's forward state
@@ -86,7 +87,8 @@ def test_training_step_with_private_backward_replays_bitwise_from_a_cuda_graph()
     def step(x_in, outs):
         ins = [x_in, outs[0]]
         for l, layer in enumerate(layers):
-            layer.forward(ins[l], pol, out=outs[l])
+            # the top layer keeps its gate/up accumulators for its backward
+            layer.forward(ins[l], pol, out=outs[l], save_for_backward=(l == 1))
         g1, dh1 = layers[1].backward(ins[1], pol, dtop)  # both results in one pass
         g0 = layers[0].backward_private(ins[0], pol, dh1.to(torch.bfloat16))
         return [g0, g1, {"d_hidden": dh1}]
