@@ -434,7 +434,7 @@ def run_ours(args):
         train[key] = {"step_ms": timed(lambda: train_step(save), args.steps),
                       "forward_ms": timed(lambda: fwd_only(save), args.steps)}
         train[key]["backward_ms"] = timed(lambda: layer.backward(h, pol, dout), args.steps)
-    train["saved_bytes"] = s.T * s.k * 2 * s.I * 4
+    train["saved_bytes"] = int(pmpe._lib.pmpe_saved_gu_floats(s.T, s.I, s.E_sh, s.k)) * 4
     train["l2"] = "flushed before every step"
 
     # ---- end to end through the public API with host buffers, pipelined as a

@@ -120,14 +120,19 @@ typedef struct pmpe_moe_desc {
      * and that count * k <= 96; PMPE_ERR_UNSUPPORTED_SHAPE otherwise. */
     int unmasked_control;
 
-    /* Optional, for training: [T*k, 2I] FP32, 16-byte aligned, or NULL.  When
-     * set, the forward also writes each dispatch row's gate and up
-     * pre-activations G | U (the FP32 accumulators its SwiGLU reads), and the
-     * backward calls given the same descriptor read them instead of
-     * recomputing the gate/up GEMM.  Their results are then bitwise those of
+    /* Optional, for training: pmpe_saved_gu_floats() FP32 values, 16-byte
+     * aligned, or NULL.  When set, the forward also writes the gate and up
+     * pre-activations (the FP32 accumulators its SwiGLU reads): first
+     * [T*k, 2I], G | U of each dispatch row, then, with shared experts,
+     * [T, 2*E_shared*I], the shared experts' G side by side, then their U.
+     * The backward calls given the same descriptor read them instead of
+     * recomputing the gate/up GEMMs; their results are then bitwise those of
      * the recomputation. */
     float *saved_gu;
 } pmpe_moe_desc;
+
+/* FP32 values of the optional saved_gu buffer: T*k*2*I + T*2*E_shared*I. */
+PMPE_API size_t pmpe_saved_gu_floats(int T, int I, int E_shared, int k);
 
 /* Bytes of device workspace pmpe_moe_forward() needs for this shape.
  * Returns 0 for an invalid shape. */

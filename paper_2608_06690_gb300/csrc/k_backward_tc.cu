@@ -480,13 +480,17 @@ __global__ void __launch_bounds__(256) bwd_swiglu_saved_kernel(const RowsParams 
     __shared__ GroupTable gt;
     pdl_wait();
     const int nt = p.I / 128;
-    build_groups(gt, p.offsets, p.g0, p.G, p.R, 0, nt, 0);
+    build_groups(gt, p.offsets, p.g0, p.G, p.R, p.shared_T, nt, 0);
     const int total = gt.tiles[p.G];
-    const int p0 = (int)min(p.offsets[p.g0], (uint32_t)p.R);
+    const int p0 = p.shared_T ? 0 : (int)min(p.offsets[p.g0], (uint32_t)p.R);
+    // saved rows: routed [R][2I] (G | U), then shared [T][2 G I] (all G, then all U)
+    const int ld2 = p.shared_T ? 2 * p.G * p.I : 2 * p.I;
+    const float *sbase = p.shared_T ? saved_gu + (size_t)p.R * 2 * p.I : saved_gu;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
         const RowsTile t = decode_rows(gt, p.G, nt, 128, tile, 0);
-        const bool wa_out = p.wact && p.g0 + t.q >= p.E_pub;
+        const bool wa_out = p.wact && !p.shared_T && p.g0 + t.q >= p.E_pub;
+        const int gcol = p.shared_T ? t.q * p.I : 0;  // the group's G columns in its saved row
         for (int r = warp; r < BM; r += nwarps) {
             const bool valid = r < t.rows;  // warp-uniform
             const int prow = gt.off[t.q] + t.m0 + r;
@@ -495,16 +499,16 @@ __global__ void __launch_bounds__(256) bwd_swiglu_saved_kernel(const RowsParams 
             float g[4] = {0.f, 0.f, 0.f, 0.f}, u[4] = {0.f, 0.f, 0.f, 0.f}, z[4] = {0.f, 0.f, 0.f, 0.f};
             float w = 0.f;
             if (valid) {
-                const float *grow = saved_gu + (size_t)(p0 + prow) * 2 * p.I;
+                const float *grow = sbase + (size_t)(p0 + prow) * ld2 + gcol;
                 const float4 gv = *reinterpret_cast<const float4 *>(grow + col);
-                const float4 uv = *reinterpret_cast<const float4 *>(grow + p.I + col);
+                const float4 uv = *reinterpret_cast<const float4 *>(grow + ld2 / 2 + col);
                 const uint2 zv = *reinterpret_cast<const uint2 *>(p.zpad + (size_t)orow * p.I + col);
                 g[0] = gv.x; g[1] = gv.y; g[2] = gv.z; g[3] = gv.w;
                 u[0] = uv.x; u[1] = uv.y; u[2] = uv.z; u[3] = uv.w;
                 const float2 z01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&zv.x));
                 const float2 z23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&zv.y));
                 z[0] = z01.x; z[1] = z01.y; z[2] = z23.x; z[3] = z23.y;
-                w = p.w_of_slot[p0 + prow];
+                w = p.shared_T ? 1.f : p.w_of_slot[p0 + prow];
             }
             float dg[4], du[4], wa[4], q[4];
 #pragma unroll
@@ -819,7 +823,7 @@ cudaError_t launch_rows_gu(const Ctx &c, const RowsGroups &g, const bf16 *a, uin
 {
     const Shape &s = c.s;
     RowsParams p = rows_params(c, g);
-    if (c.saved_gu && !g.shared_T) {  // the forward saved G | U of the routed rows
+    if (c.saved_gu) {  // the forward saved the G | U accumulators of these rows
         p.K = s.H; p.N = s.I; p.bn = 128;
         p.zpad = zpad;
         p.gw_part = gw_part;

@@ -76,8 +76,9 @@ struct TcParams {
     // activations are stored (zeroed before the launch)
     uint32_t *ready;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
-    // optional [R][2I] FP32: the routed rows' gate and up accumulators G | U,
-    // saved for the backward (gu_save map for whole 32-row blocks)
+    // optional FP32: the gate and up accumulators saved for the backward,
+    // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
+    // experts (gu_save / gu_save_sh maps for whole 32-row blocks)
     float *saved_gu;
 };
 
@@ -86,7 +87,8 @@ struct TcMaps {  // [phase]
     CUtensorMap a_routed[2], a_shared[2];
     CUtensorMap b0[2][3];  // per pool [pub, priv, shared]: gate (gate/up) or down
     CUtensorMap b1[2][3];  // up (gate/up)
-    CUtensorMap gu_save;   // saved_gu, 16 x 32 FP32 boxes, 64-byte swizzle
+    CUtensorMap gu_save;   // saved_gu, routed rows [R][2I], 16 x 32 FP32 boxes, 64-byte swizzle
+    CUtensorMap gu_save_sh;  // saved_gu's shared part [T][2 E_sh I], the same boxes
 };
 
 // ------------------------------------------------------------- tile list
@@ -370,9 +372,12 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
 #pragma unroll
                     for (int i = 0; i < 16; ++i)
                         pk[i] = pack_bf16x2(silu_mul(gv[2 * i], uv[2 * i]), silu_mul(gv[2 * i + 1], uv[2 * i + 1]));
-                    if (p.saved_gu && !t.shared) {
+                    if (p.saved_gu) {
                         // G and U of these 32 columns, as FP32, for the backward
                         const int y0 = t.row_base + t.m0 + quarter * 32;
+                        const int ld2 = t.shared ? 2 * p.E_sh * p.I : 2 * p.I;  // floats per saved row
+                        const int uoff = ld2 / 2;                                // U follows G
+                        const CUtensorMap *smap = t.shared ? &maps.gu_save_sh : &maps.gu_save;
                         if (full_block) {
 #pragma unroll
                             for (int b = 0; b < 4; ++b) {  // G lo, G hi, U lo, U hi: 16 columns each
@@ -391,15 +396,15 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                                 fence_proxy_async_smem();
                                 __syncwarp();
                                 if (lane == 0) {
-                                    tma_store_2d(&maps.gu_save, sbuf, (b < 2 ? 0 : p.I) + t.n0 + c * 32 + (b & 1) * 16,
-                                                 y0);
+                                    tma_store_2d(smap, sbuf, (b < 2 ? 0 : uoff) + t.n0 + c * 32 + (b & 1) * 16, y0);
                                     bulk_commit();
                                 }
                                 out_parity ^= 1;
                             }
                         } else if (valid) {
-                            float4 *gd = reinterpret_cast<float4 *>(p.saved_gu + (size_t)grow * 2 * p.I + t.n0 + c * 32);
-                            float4 *ud = gd + p.I / 4;
+                            float *sbase = t.shared ? p.saved_gu + (size_t)p.R * 2 * p.I : p.saved_gu;
+                            float4 *gd = reinterpret_cast<float4 *>(sbase + (size_t)grow * ld2 + t.n0 + c * 32);
+                            float4 *ud = gd + uoff / 4;
 #pragma unroll
                             for (int i = 0; i < 8; ++i) {
                                 gd[i] = make_float4(gv[4 * i], gv[4 * i + 1], gv[4 * i + 2], gv[4 * i + 3]);
@@ -560,6 +565,9 @@ cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
         p.saved_gu = c.saved_gu;
         ok &= encode_2d_f32(&maps.gu_save, c.saved_gu, 2 * (uint64_t)s.I, (uint64_t)s.T * s.k, 16, 32,
                             CU_TENSOR_MAP_SWIZZLE_64B);
+        if (s.E_sh > 0)
+            ok &= encode_2d_f32(&maps.gu_save_sh, c.saved_gu + (size_t)s.T * s.k * 2 * s.I,
+                                2 * (uint64_t)s.E_sh * s.I, (uint64_t)s.T, 16, 32, CU_TENSOR_MAP_SWIZZLE_64B);
     }
     if (!ok) return cudaErrorInvalidValue;
     static std::atomic<int> smem_limit[64];

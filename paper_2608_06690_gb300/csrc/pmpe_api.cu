@@ -297,6 +297,12 @@ int pmpe_moe_backward_input(const pmpe_moe_desc *d, const void *dout, float *d_h
                : PMPE_ERR_CUDA;
 }
 
+size_t pmpe_saved_gu_floats(int T, int I, int E_shared, int k)
+{
+    if (T < 0 || I < 0 || E_shared < 0 || k < 0) return 0;
+    return (size_t)T * k * 2 * I + (size_t)T * 2 * E_shared * I;
+}
+
 size_t pmpe_moe_backward_step_workspace_size(int T, int H, int I, int E_pub, int E_priv, int E_shared, int k)
 {
     Shape s;

@@ -73,7 +73,7 @@ EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_
             "pmpe_status_string", "pmpe_moe_forward_noalloc", "pmpe_selftest_wait_timeout",
             "pmpe_policy_from_requests", "pmpe_moe_backward_workspace_size", "pmpe_moe_backward_private",
             "pmpe_moe_backward_input_workspace_size", "pmpe_moe_backward_input",
-            "pmpe_moe_backward_step_workspace_size", "pmpe_moe_backward_step")
+            "pmpe_moe_backward_step_workspace_size", "pmpe_moe_backward_step", "pmpe_saved_gu_floats")
 
 # Bytes of the library's static scratch array used by pmpe_moe_forward_noalloc.
 STATIC_SCRATCH_BYTES = 32 << 20
@@ -128,6 +128,8 @@ _lib.pmpe_moe_backward_step_workspace_size.restype = ctypes.c_size_t
 _lib.pmpe_moe_backward_step_workspace_size.argtypes = [ctypes.c_int] * 7
 _lib.pmpe_moe_backward_step.restype = ctypes.c_int
 _lib.pmpe_moe_backward_step.argtypes = [ctypes.POINTER(MoeDesc)] + [_vp] * 7 + [ctypes.c_size_t, _vp]
+_lib.pmpe_saved_gu_floats.restype = ctypes.c_size_t
+_lib.pmpe_saved_gu_floats.argtypes = [ctypes.c_int] * 4
 _lib.pmpe_policy_from_requests.restype = ctypes.c_int
 _lib.pmpe_policy_from_requests.argtypes = [_vp, _vp, ctypes.c_int, ctypes.c_int, _vp, _vp]
 _lib.pmpe_selftest_wait_timeout.restype = ctypes.c_int
@@ -302,9 +304,10 @@ class MoeLayer:
         """Enqueue the layer on ``stream`` (default: the current stream).
         ``unmasked_control`` runs the paper's soft-router control instead of
         the method: routing over the concatenated pool without the hard mask.
-        ``save_for_backward`` also keeps the routed rows' gate and up
-        accumulators ([T k, 2I] FP32, owned by the layer), which the backward
-        calls after this forward then read instead of recomputing them."""
+        ``save_for_backward`` also keeps the gate and up accumulators of the
+        routed rows and the shared experts (FP32, owned by the layer), which
+        the backward calls after this forward then read instead of
+        recomputing them."""
         T = hidden.shape[0]
         s = self._shape_T(T)
         assert hidden.is_contiguous() and hidden.dtype == torch.bfloat16 and hidden.shape == (T, s.H)
@@ -314,7 +317,7 @@ class MoeLayer:
             out = torch.empty_like(hidden)
         saved = None
         if save_for_backward:
-            n = T * s.k * 2 * s.I
+            n = _lib.pmpe_saved_gu_floats(T, s.I, s.E_sh, s.k)
             if self._saved_buf is None or self._saved_buf.numel() < n:
                 self._saved_buf = torch.empty(max(n, 4), dtype=torch.float32, device=hidden.device)
             saved = self._saved_buf
