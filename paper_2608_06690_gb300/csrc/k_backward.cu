@@ -55,17 +55,197 @@ __global__ void __launch_bounds__(256) bwd_gather_kernel(const bf16 *dout, const
     }
 }
 
+// Each pool's tokens in ascending order, the DENY pool's first: pool_tok[0,
+// nd) and pool_tok[nd, T), pool_n = {nd, na}.  One CTA: every thread ranks a
+// contiguous run of tokens.
+__global__ void __launch_bounds__(1024) bwd_pool_tokens_kernel(const uint8_t *tau, int T, int32_t *pool_tok,
+                                                               int *pool_n)
+{
+    __shared__ int s_warp[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    pdl_wait();
+    const int per = (T + blockDim.x - 1) / blockDim.x;
+    const int t0 = min(T, tid * per), t1 = min(T, t0 + per);
+    int a = 0;
+    for (int t = t0; t < t1; ++t) a += tau[t] ? 1 : 0;
+    int x = a;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(~0u, x, off);
+        if (lane >= off) x += y;
+    }
+    if (lane == 31) s_warp[warp] = x;
+    __syncthreads();
+    int before = 0, na = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+        before += w < warp ? s_warp[w] : 0;
+        na += s_warp[w];
+    }
+    int ra = before + x - a, rd = t0 - (before + x - a);  // ranks of this run's first token in its pool
+    const int nd = T - na;
+    for (int t = t0; t < t1; ++t) {
+        if (tau[t]) pool_tok[nd + ra++] = t;
+        else pool_tok[rd++] = t;
+    }
+    if (tid == 0) {
+        pool_n[0] = nd;
+        pool_n[1] = na;
+    }
+}
+
+// Shared-memory tiled FP32 GEMMs over one pool's tokens (blockIdx.z = pool q
+// - pool0; blockIdx.x = the 64-token block of the pool's list): 64 x 64
+// outputs a CTA, K in steps of 32, a 4 x 4 micro-tile a thread.  A DENY
+// token's row only ever meets the public router, an ALLOW token's only the
+// private one.
+constexpr int kPT = 64, kPK = 32, kSkew = 4;  // tile, K step, row skew of the shared tiles
+
+// The pool-softmax logits z[t][e] = sum_h h[t][h] W_q[e][h] of each token
+// of the pool and every expert of it, into the token's dz row (blockIdx.y =
+// 64-expert chunk).
+__global__ void __launch_bounds__(256) bwd_pool_logits_kernel(const bf16 *hidden, const bf16 *router_pub,
+                                                              const bf16 *router_priv, const int32_t *pool_tok,
+                                                              const int *pool_n, int H, int E_pub, int E_priv,
+                                                              int pool0, int ld, float *dz)
+{
+    __shared__ __align__(16) float As[kPK][kPT + kSkew], Bs[kPK][kPT + kSkew];
+    __shared__ int s_tok[kPT];
+    pdl_wait();
+    const int q = pool0 + blockIdx.z;
+    const int n = pool_n[q], i0 = blockIdx.x * kPT, e0 = blockIdx.y * kPT;
+    const int E_q = q ? E_priv : E_pub;
+    if (i0 >= n || e0 >= E_q) return;  // uniform
+    const int32_t *toks = pool_tok + (q ? pool_n[0] : 0);
+    const bf16 *W = q ? router_priv : router_pub;
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    if (tid < kPT) s_tok[tid] = i0 + tid < n ? toks[i0 + tid] : -1;
+    __syncthreads();
+    const int lr = tid >> 2, lk = (tid & 3) * 8;  // this thread's loads: row lr, 8 K values from lk
+    const int tok = s_tok[lr], er = e0 + lr;
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+    for (int k0 = 0; k0 < H; k0 += kPK) {
+        const uint4 av = tok >= 0 ? *reinterpret_cast<const uint4 *>(hidden + (size_t)tok * H + k0 + lk)
+                                  : make_uint4(0u, 0u, 0u, 0u);
+        const uint4 bv = er < E_q ? *reinterpret_cast<const uint4 *>(W + (size_t)er * H + k0 + lk)
+                                  : make_uint4(0u, 0u, 0u, 0u);
+        __syncthreads();  // the previous step's tiles are consumed
+        const __nv_bfloat162 *ab = reinterpret_cast<const __nv_bfloat162 *>(&av);
+        const __nv_bfloat162 *bb = reinterpret_cast<const __nv_bfloat162 *>(&bv);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 fa = __bfloat1622float2(ab[j]), fb = __bfloat1622float2(bb[j]);
+            As[lk + 2 * j][lr] = fa.x; As[lk + 2 * j + 1][lr] = fa.y;
+            Bs[lk + 2 * j][lr] = fb.x; Bs[lk + 2 * j + 1][lr] = fb.y;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int kk = 0; kk < kPK; ++kk) {
+            const float4 a4 = *reinterpret_cast<const float4 *>(&As[kk][ty * 4]);
+            const float4 b4 = *reinterpret_cast<const float4 *>(&Bs[kk][tx * 4]);
+            const float a[4] = {a4.x, a4.y, a4.z, a4.w}, b[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] += a[i] * b[j];
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int t = s_tok[ty * 4 + i];
+        if (t < 0) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int e = e0 + tx * 4 + j;
+            if (e < E_q) dz[(size_t)t * ld + e] = acc[i][j];
+        }
+    }
+}
+
+// The pool-softmax router term of the input gradient, added in place:
+// d_hidden[t][c] += sum_e dz[t][e] W_q[e][c] over the pool's experts in
+// order (blockIdx.y = 64-column block).
+__global__ void __launch_bounds__(256) bwd_pool_router_term_kernel(const float *dz, int ld, const bf16 *router_pub,
+                                                                   const bf16 *router_priv, const int32_t *pool_tok,
+                                                                   const int *pool_n, int H, int E_pub, int E_priv,
+                                                                   float *d_hidden)
+{
+    __shared__ __align__(16) float As[kPK][kPT + kSkew], Bs[kPK][kPT + kSkew];
+    __shared__ int s_tok[kPT];
+    pdl_wait();
+    const int q = blockIdx.z;
+    const int n = pool_n[q], i0 = blockIdx.x * kPT, c0 = blockIdx.y * kPT;
+    if (i0 >= n) return;  // uniform
+    const int E_q = q ? E_priv : E_pub;
+    const int32_t *toks = pool_tok + (q ? pool_n[0] : 0);
+    const bf16 *W = q ? router_priv : router_pub;
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    if (tid < kPT) s_tok[tid] = i0 + tid < n ? toks[i0 + tid] : -1;
+    __syncthreads();
+    const int ar = tid >> 2, ak = (tid & 3) * 8;  // A loads: token row ar, 8 experts from ak
+    const int br = tid >> 3, bc = (tid & 7) * 8;  // B loads: expert row br, 8 columns from bc
+    const int tok = s_tok[ar];
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+    for (int k0 = 0; k0 < E_q; k0 += kPK) {
+        float av[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int e = k0 + ak + j;
+            av[j] = (tok >= 0 && e < E_q) ? dz[(size_t)tok * ld + e] : 0.f;
+        }
+        uint4 bv = make_uint4(0u, 0u, 0u, 0u);
+        if (k0 + br < E_q) bv = *reinterpret_cast<const uint4 *>(W + (size_t)(k0 + br) * H + c0 + bc);
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < 8; ++j) As[ak + j][ar] = av[j];
+        const __nv_bfloat162 *bb = reinterpret_cast<const __nv_bfloat162 *>(&bv);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float2 fb = __bfloat1622float2(bb[j]);
+            Bs[br][bc + 2 * j] = fb.x;
+            Bs[br][bc + 2 * j + 1] = fb.y;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int kk = 0; kk < kPK; ++kk) {
+            const float4 a4 = *reinterpret_cast<const float4 *>(&As[kk][ty * 4]);
+            const float4 b4 = *reinterpret_cast<const float4 *>(&Bs[kk][tx * 4]);
+            const float a[4] = {a4.x, a4.y, a4.z, a4.w}, b[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] += a[i] * b[j];
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int t = s_tok[ty * 4 + i];
+        if (t < 0) continue;
+        float4 *o = reinterpret_cast<float4 *>(d_hidden + (size_t)t * H + c0 + tx * 4);
+        float4 v = *o;
+        v.x += acc[i][0]; v.y += acc[i][1]; v.z += acc[i][2]; v.w += acc[i][3];
+        *o = v;
+    }
+}
+
 // Router gradient per token (one warp): the softmax gradient dz over the
 // token's pool from dL/dw of its k rows (summed from the expert GEMM's per-tile
 // partials, indexed by dispatch slot) -- renormalised over the top-k, or the
-// pool softmax, whose probabilities need every logit of the pool, recomputed
-// here in FP32 from the BF16 operands.  both_pools = 0: the private pool only,
+// pool softmax, whose probabilities need every logit of the pool: those are
+// already in the token's dz row (bwd_pool_logits_kernel).  both_pools = 0:
+// the private pool only,
 // dz [T][ld = E_priv], zero for DENY tokens; both_pools = 1: each token's own
 // pool (tau selects it), dz [T][ld] holding that pool's E_pub or E_priv entries.
-__global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_pub, const bf16 *router_priv,
-                                  const uint8_t *tau, const int32_t *idx, const float *wts, const int32_t *slot_of,
-                                  const float *gw_part, int n_part, int T, int H, int E_pub, int E_priv, int k,
-                                  int renorm, int both_pools, int ld, float *dz)
+__global__ void bwd_router_kernel(const uint8_t *tau, const int32_t *idx, const float *wts, const int32_t *slot_of,
+                                  const float *gw_part, int n_part, int T, int E_pub, int E_priv, int k, int renorm,
+                                  int both_pools, int ld, float *dz)
 {
     const int lane = threadIdx.x & 31;
     const int warps = gridDim.x * (blockDim.x >> 5);
@@ -78,7 +258,6 @@ __global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_pub, co
         }
         const int E_pool = priv ? E_priv : E_pub;
         const int e_base = priv ? E_pub : 0;
-        const bf16 *router = priv ? router_priv : router_pub;
         // lane j < k holds pick j: its pool id and dL/dw
         int pe = -1;
         float g = 0.f, wj = 0.f;
@@ -96,30 +275,7 @@ __global__ void bwd_router_kernel(const bf16 *hidden, const bf16 *router_pub, co
             for (int e = lane; e < E_pool; e += 32) dzt[e] = 0.f;
             __syncwarp();
             if (lane < k && pe >= 0 && pe < E_pool) dzt[pe] = wj * (g - sum);
-        } else {
-            // pool softmax over the private experts: logits of this token
-            const bf16 *h = hidden + (size_t)t * H;
-            for (int e0 = 0; e0 < E_pool; e0 += 32) {
-                const int e = e0 + lane;
-                float z = -INFINITY;
-                if (e < E_pool) {
-                    const bf16 *wr = router + (size_t)e * H;
-                    float a = 0.f;
-                    for (int c = 0; c < H; c += 8) {
-                        const uint4 hv = *reinterpret_cast<const uint4 *>(h + c);
-                        const uint4 rv = *reinterpret_cast<const uint4 *>(wr + c);
-                        const __nv_bfloat162 *hb = reinterpret_cast<const __nv_bfloat162 *>(&hv);
-                        const __nv_bfloat162 *rb = reinterpret_cast<const __nv_bfloat162 *>(&rv);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const float2 x = __bfloat1622float2(hb[q]), y = __bfloat1622float2(rb[q]);
-                            a += x.x * y.x + x.y * y.y;
-                        }
-                    }
-                    z = a;
-                }
-                if (e < E_pool) dzt[e] = z;  // logits parked in dz, finished below
-            }
+        } else {  // the pool's logits are in dz: the softmax gradient replaces them
             __syncwarp();
             float mx = -INFINITY;
             for (int e = lane; e < E_pool; e += 32) mx = fmaxf(mx, dzt[e]);
@@ -268,12 +424,32 @@ void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint
     bwd_gather_kernel<<<num_sms * 8, 256, 0, st>>>(dout, tok_of_slot, offsets, g0, g1, R, H, rows);
 }
 
-cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz)
+cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz, int32_t *pool_tok,
+                             int *pool_n)
 {
     const Shape &s = c.s;
-    bwd_router_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(c.hidden, c.router_pub, c.router_priv, c.tau, c.idx, c.w,
-                                                           c.slot_of, gw_part, s.I / 128, s.T, s.H, s.E_pub, s.E_priv,
-                                                           s.k, s.renorm, both_pools, ld, dz);
+    cudaError_t err;
+    if (!s.renorm) {  // the pool softmax needs every logit of the token's pool: tiled GEMMs per pool
+        bwd_pool_tokens_kernel<<<1, 1024, 0, c.stream>>>(c.tau, s.T, pool_tok, pool_n);
+        if ((err = cudaGetLastError()) != cudaSuccess) return err;
+        const int chunks = (std::max(both_pools ? s.E_pub : 0, s.E_priv) + kPT - 1) / kPT;
+        const dim3 grid((s.T + kPT - 1) / kPT, chunks, both_pools ? 2 : 1);
+        bwd_pool_logits_kernel<<<grid, 256, 0, c.stream>>>(c.hidden, c.router_pub, c.router_priv, pool_tok, pool_n,
+                                                             s.H, s.E_pub, s.E_priv, both_pools ? 0 : 1, ld, dz);
+        if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    }
+    bwd_router_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(c.tau, c.idx, c.w, c.slot_of, gw_part, s.I / 128, s.T,
+                                                           s.E_pub, s.E_priv, s.k, s.renorm, both_pools, ld, dz);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_router_term(const Ctx &c, const float *dz, int ld, const int32_t *pool_tok, const int *pool_n,
+                               float *d_hidden)
+{
+    const Shape &s = c.s;
+    const dim3 grid((s.T + kPT - 1) / kPT, s.H / kPT, 2);
+    bwd_pool_router_term_kernel<<<grid, 256, 0, c.stream>>>(dz, ld, c.router_pub, c.router_priv, pool_tok, pool_n,
+                                                              s.H, s.E_pub, s.E_priv, d_hidden);
     return cudaGetLastError();
 }
 
@@ -281,6 +457,8 @@ struct BwdScratch {
     bf16 *dout_rows, *zpad, *dgu, *wact;
     float *gw_part, *dz, *part;
     int *active;  // per token range of the router weight gradient: 1 if it holds an ALLOW token
+    int32_t *pool_tok;  // [T] each pool's tokens (pool softmax), then pool_n [2]
+    int *pool_n;
     size_t bytes;
 };
 
@@ -298,6 +476,8 @@ static BwdScratch backward_scratch(const Shape &s, uint8_t *base)
     b.dz = (float *)(base + o);       o += al((size_t)s.T * s.E_priv * 4);
     b.part = (float *)(base + o);     o += al(router_wgrad_part_bytes(s));
     b.active = (int *)(base + o);     o += al(kMaxRouterSplits * 4);
+    b.pool_tok = (int32_t *)(base + o); o += al((size_t)s.T * 4);
+    b.pool_n = (int *)(base + o);     o += al(2 * 4);
     b.bytes = o;
     return b;
 }
@@ -321,7 +501,7 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     if ((err = launch_backward_rows(c, b.dout_rows, b.zpad, b.dgu, b.wact, b.gw_part)) != cudaSuccess) return err;
-    if ((err = launch_router_dz(c, b.gw_part, 0, s.E_priv, b.dz)) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 0, s.E_priv, b.dz, b.pool_tok, b.pool_n)) != cudaSuccess) return err;
     if ((err = launch_router_wgrad(c, b.dz, s.E_priv, b.part, b.active, d_router)) != cudaSuccess) return err;
     return launch_backward_wgrad(c, b.dout_rows, b.dgu, b.wact, d_gate, d_up, d_down);
 }

@@ -129,9 +129,7 @@ __global__ void __launch_bounds__(256) bwd_input_reduce_kernel(
                     for (int j = 0; j < kBatch; ++j)
                         if (j0 + j < k && s_pe[j0 + j] >= 0) add(v[j], s_dz[j0 + j]);
                 }
-            } else {
-                for (int e = 0; e < E_pool; ++e) add(reinterpret_cast<const uint4 *>(router + (size_t)e * H)[c], dzt[e]);
-            }
+            }  // the pool softmax's dense router term is added afterwards (launch_router_term)
             float4 *o = reinterpret_cast<float4 *>(d_hidden + (size_t)t * H) + 2 * c;
             __stcs(o, make_float4(acc[0], acc[1], acc[2], acc[3]));
             __stcs(o + 1, make_float4(acc[4], acc[5], acc[6], acc[7]));
@@ -144,6 +142,8 @@ __global__ void __launch_bounds__(256) bwd_input_reduce_kernel(
 struct InScratch {
     bf16 *dout_rows, *zpad, *dgu, *da, *zpad_sh, *dgu_sh, *da_sh;
     float *gw_part, *dz;
+    int32_t *pool_tok;  // [T] each pool's tokens (pool softmax), then pool_n [2]
+    int *pool_n;
     uint64_t rp, rp_sh;  // padded rows: routed, shared
     int tp;              // tokens rounded up to the padded layout (rows of one shared expert)
     size_t bytes;
@@ -167,21 +167,27 @@ static InScratch input_scratch(const Shape &s, uint8_t *base)
     b.da_sh = (bf16 *)(base + o);     o += al(b.rp_sh * H * 2);
     b.gw_part = (float *)(base + o);  o += al(R * (I / 128) * 4);
     b.dz = (float *)(base + o);       o += al((size_t)s.T * std::max(s.E_pub, s.E_priv) * 4);
+    b.pool_tok = (int32_t *)(base + o); o += al((size_t)s.T * 4);
+    b.pool_n = (int *)(base + o);     o += al(2 * 4);
     b.bytes = o;
     return b;
 }
 
 // The per-token sum of the picks' dA, the shared experts' dA and the router
-// term (dz rows max(E_pub, E_priv) apart).
+// term (dz rows max(E_pub, E_priv) apart): renormalised routing adds the k
+// picks' router rows in the same kernel, the pool softmax its dense term in
+// a tiled GEMM afterwards.
 static cudaError_t launch_input_reduce(const Ctx &c, const InScratch &b, float *d_hidden)
 {
     const Shape &s = c.s;
     const int ld = std::max(s.E_pub, s.E_priv);
-    return launch_pdl(bwd_input_reduce_kernel, dim3(std::min(s.T, c.num_sms * 8)), dim3(256), 0, c.stream,
+    const cudaError_t err = launch_pdl(bwd_input_reduce_kernel, dim3(std::min(s.T, c.num_sms * 8)), dim3(256), 0, c.stream,
                       (const bf16 *)b.da, (const bf16 *)b.da_sh, (const float *)b.dz, ld, c.router_pub,
                       c.router_priv, (const uint8_t *)c.tau, (const int32_t *)c.idx, (const int32_t *)c.slot_of,
                       (const uint32_t *)c.offsets, s.T, s.H, s.E_pub, s.E_priv, s.E_sh, s.k, s.T * s.k, s.renorm,
                       b.tp, d_hidden);
+    if (err != cudaSuccess || s.renorm) return err;
+    return launch_router_term(c, b.dz, ld, b.pool_tok, b.pool_n, d_hidden);
 }
 
 size_t backward_input_workspace_bytes(const Shape &s)
@@ -218,7 +224,7 @@ cudaError_t launch_backward_input(const Ctx &c, const bf16 *dout, float *d_hidde
     }
     // the router of each token's pool
     const int ld = std::max(s.E_pub, s.E_priv);
-    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz)) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz, b.pool_tok, b.pool_n)) != cudaSuccess) return err;
     return launch_input_reduce(c, b, d_hidden);
 }
 
@@ -285,7 +291,7 @@ cudaError_t launch_backward_step(const Ctx &c, const bf16 *dout, float *d_router
         if ((err = launch_rows_da(c, gs, b.dgu_sh, b.da_sh)) != cudaSuccess) return err;
     }
     const int ld = std::max(s.E_pub, s.E_priv);
-    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz)) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz, b.pool_tok, b.pool_n)) != cudaSuccess) return err;
     if ((err = launch_router_wgrad(c, b.dz, ld, st.part, st.active, d_router)) != cudaSuccess) return err;
     if ((err = launch_backward_wgrad(c, b.dout_rows, b.dgu, st.wact, d_gate, d_up, d_down, &g)) != cudaSuccess)
         return err;

@@ -86,10 +86,16 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
 // Its pieces shared with the input gradient: the upstream gradients of the
 // dispatch rows of experts g0 .. g1 - 1 (and 64 zero rows after them); the
 // router's softmax gradient from the dL/dw partials per slot (both_pools = 0:
-// the private pool, zero for DENY tokens; 1: each token's own pool), dz [T][ld].
+// the private pool, zero for DENY tokens; 1: each token's own pool), dz [T][ld]
+// (pool softmax: the pools' token lists go to pool_tok [T] and pool_n [2]).
 void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint32_t *offsets, int g0, int g1, int R,
                         int H, bf16 *rows, int num_sms, cudaStream_t st);
-cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz);
+cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz, int32_t *pool_tok,
+                             int *pool_n);
+// The pool-softmax router term of the input gradient, added to d_hidden
+// (pool lists from launch_router_dz).
+cudaError_t launch_router_term(const Ctx &c, const float *dz, int ld, const int32_t *pool_tok, const int *pool_n,
+                               float *d_hidden);
 constexpr int kMaxRouterSplits = 64;  // token ranges of the router weight gradient
 // The private router's weight gradient from dz (rows ld apart; DENY rows read
 // as zeros): token-range partials (part, router_wgrad_part_bytes) and their
