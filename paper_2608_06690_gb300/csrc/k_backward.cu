@@ -101,22 +101,26 @@ __global__ void __launch_bounds__(1024) bwd_pool_tokens_kernel(const uint8_t *ta
 constexpr int kPT = 64, kPK = 32, kSkew = 4;  // tile, K step, row skew of the shared tiles
 
 // The pool-softmax logits z[t][e] = sum_h h[t][h] W_q[e][h] of each token
-// of the pool and every expert of it, into the token's dz row (blockIdx.y =
-// 64-expert chunk).
+// of the pool and every expert of it, as ksplit partial sums over equal
+// ranges of h: blockIdx.y = 64-expert chunk * ksplit + range, partial s into
+// part[s][t][e] (rows ld apart); the dz kernel adds them in range order.
 __global__ void __launch_bounds__(256) bwd_pool_logits_kernel(const bf16 *hidden, const bf16 *router_pub,
                                                               const bf16 *router_priv, const int32_t *pool_tok,
-                                                              const int *pool_n, int H, int E_pub, int E_priv,
-                                                              int pool0, int ld, float *dz)
+                                                              const int *pool_n, int T, int H, int E_pub, int E_priv,
+                                                              int pool0, int ksplit, int ld, float *part)
 {
     __shared__ __align__(16) float As[kPK][kPT + kSkew], Bs[kPK][kPT + kSkew];
     __shared__ int s_tok[kPT];
     pdl_wait();
     const int q = pool0 + blockIdx.z;
-    const int n = pool_n[q], i0 = blockIdx.x * kPT, e0 = blockIdx.y * kPT;
+    const int ks = blockIdx.y % ksplit;
+    const int n = pool_n[q], i0 = blockIdx.x * kPT, e0 = (blockIdx.y / ksplit) * kPT;
     const int E_q = q ? E_priv : E_pub;
     if (i0 >= n || e0 >= E_q) return;  // uniform
     const int32_t *toks = pool_tok + (q ? pool_n[0] : 0);
     const bf16 *W = q ? router_priv : router_pub;
+    const int hs = H / ksplit, h0 = ks * hs;
+    float *dz = part + (size_t)ks * T * ld;
     const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
     if (tid < kPT) s_tok[tid] = i0 + tid < n ? toks[i0 + tid] : -1;
     __syncthreads();
@@ -127,7 +131,7 @@ __global__ void __launch_bounds__(256) bwd_pool_logits_kernel(const bf16 *hidden
     for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-    for (int k0 = 0; k0 < H; k0 += kPK) {
+    for (int k0 = h0; k0 < h0 + hs; k0 += kPK) {
         const uint4 av = tok >= 0 ? *reinterpret_cast<const uint4 *>(hidden + (size_t)tok * H + k0 + lk)
                                   : make_uint4(0u, 0u, 0u, 0u);
         const uint4 bv = er < E_q ? *reinterpret_cast<const uint4 *>(W + (size_t)er * H + k0 + lk)
@@ -238,14 +242,14 @@ __global__ void __launch_bounds__(256) bwd_pool_router_term_kernel(const float *
 // Router gradient per token (one warp): the softmax gradient dz over the
 // token's pool from dL/dw of its k rows (summed from the expert GEMM's per-tile
 // partials, indexed by dispatch slot) -- renormalised over the top-k, or the
-// pool softmax, whose probabilities need every logit of the pool: those are
-// already in the token's dz row (bwd_pool_logits_kernel).  both_pools = 0:
+// pool softmax, whose probabilities need every logit of the pool: those come
+// as partial sums from bwd_pool_logits_kernel.  both_pools = 0:
 // the private pool only,
 // dz [T][ld = E_priv], zero for DENY tokens; both_pools = 1: each token's own
 // pool (tau selects it), dz [T][ld] holding that pool's E_pub or E_priv entries.
 __global__ void bwd_router_kernel(const uint8_t *tau, const int32_t *idx, const float *wts, const int32_t *slot_of,
                                   const float *gw_part, int n_part, int T, int E_pub, int E_priv, int k, int renorm,
-                                  int both_pools, int ld, float *dz)
+                                  int both_pools, int ld, const float *logit_part, int ksplit, float *dz)
 {
     const int lane = threadIdx.x & 31;
     const int warps = gridDim.x * (blockDim.x >> 5);
@@ -275,7 +279,12 @@ __global__ void bwd_router_kernel(const uint8_t *tau, const int32_t *idx, const 
             for (int e = lane; e < E_pool; e += 32) dzt[e] = 0.f;
             __syncwarp();
             if (lane < k && pe >= 0 && pe < E_pool) dzt[pe] = wj * (g - sum);
-        } else {  // the pool's logits are in dz: the softmax gradient replaces them
+        } else {  // the pool's logits: the partial sums in range order, then the softmax gradient
+            for (int e = lane; e < E_pool; e += 32) {
+                float z = 0.f;
+                for (int s2 = 0; s2 < ksplit; ++s2) z += logit_part[((size_t)s2 * T + t) * ld + e];
+                dzt[e] = z;
+            }
             __syncwarp();
             float mx = -INFINITY;
             for (int e = lane; e < E_pool; e += 32) mx = fmaxf(mx, dzt[e]);
@@ -424,22 +433,33 @@ void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint
     bwd_gather_kernel<<<num_sms * 8, 256, 0, st>>>(dout, tok_of_slot, offsets, g0, g1, R, H, rows);
 }
 
+int router_logit_splits(const Shape &s)
+{
+    const int m = s.H / 128;  // ranges of h: a divisor of H / 128, at most 8
+    for (int d = 8; d > 1; --d)
+        if (m % d == 0) return d;
+    return 1;
+}
+
 cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz, int32_t *pool_tok,
-                             int *pool_n)
+                             int *pool_n, float *logit_part)
 {
     const Shape &s = c.s;
     cudaError_t err;
+    const int ksplit = router_logit_splits(s);
     if (!s.renorm) {  // the pool softmax needs every logit of the token's pool: tiled GEMMs per pool
         bwd_pool_tokens_kernel<<<1, 1024, 0, c.stream>>>(c.tau, s.T, pool_tok, pool_n);
         if ((err = cudaGetLastError()) != cudaSuccess) return err;
         const int chunks = (std::max(both_pools ? s.E_pub : 0, s.E_priv) + kPT - 1) / kPT;
-        const dim3 grid((s.T + kPT - 1) / kPT, chunks, both_pools ? 2 : 1);
+        const dim3 grid((s.T + kPT - 1) / kPT, chunks * ksplit, both_pools ? 2 : 1);
         bwd_pool_logits_kernel<<<grid, 256, 0, c.stream>>>(c.hidden, c.router_pub, c.router_priv, pool_tok, pool_n,
-                                                             s.H, s.E_pub, s.E_priv, both_pools ? 0 : 1, ld, dz);
+                                                             s.T, s.H, s.E_pub, s.E_priv, both_pools ? 0 : 1, ksplit, ld,
+                                                             logit_part);
         if ((err = cudaGetLastError()) != cudaSuccess) return err;
     }
     bwd_router_kernel<<<c.num_sms * 4, 256, 0, c.stream>>>(c.tau, c.idx, c.w, c.slot_of, gw_part, s.I / 128, s.T,
-                                                           s.E_pub, s.E_priv, s.k, s.renorm, both_pools, ld, dz);
+                                                           s.E_pub, s.E_priv, s.k, s.renorm, both_pools, ld, logit_part,
+                                                           ksplit, dz);
     return cudaGetLastError();
 }
 
@@ -459,6 +479,7 @@ struct BwdScratch {
     int *active;  // per token range of the router weight gradient: 1 if it holds an ALLOW token
     int32_t *pool_tok;  // [T] each pool's tokens (pool softmax), then pool_n [2]
     int *pool_n;
+    float *logit_part;  // [router_logit_splits][T][E_priv] partial pool logits (pool softmax)
     size_t bytes;
 };
 
@@ -478,6 +499,8 @@ static BwdScratch backward_scratch(const Shape &s, uint8_t *base)
     b.active = (int *)(base + o);     o += al(kMaxRouterSplits * 4);
     b.pool_tok = (int32_t *)(base + o); o += al((size_t)s.T * 4);
     b.pool_n = (int *)(base + o);     o += al(2 * 4);
+    // (sized whatever the routing: the size query does not know it)
+    b.logit_part = (float *)(base + o); o += al((size_t)router_logit_splits(s) * s.T * s.E_priv * 4);
     b.bytes = o;
     return b;
 }
@@ -501,7 +524,7 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     if ((err = launch_backward_rows(c, b.dout_rows, b.zpad, b.dgu, b.wact, b.gw_part)) != cudaSuccess) return err;
-    if ((err = launch_router_dz(c, b.gw_part, 0, s.E_priv, b.dz, b.pool_tok, b.pool_n)) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 0, s.E_priv, b.dz, b.pool_tok, b.pool_n, b.logit_part)) != cudaSuccess) return err;
     if ((err = launch_router_wgrad(c, b.dz, s.E_priv, b.part, b.active, d_router)) != cudaSuccess) return err;
     return launch_backward_wgrad(c, b.dout_rows, b.dgu, b.wact, d_gate, d_up, d_down);
 }

@@ -144,6 +144,7 @@ struct InScratch {
     float *gw_part, *dz;
     int32_t *pool_tok;  // [T] each pool's tokens (pool softmax), then pool_n [2]
     int *pool_n;
+    float *logit_part;  // partial pool logits (pool softmax)
     uint64_t rp, rp_sh;  // padded rows: routed, shared
     int tp;              // tokens rounded up to the padded layout (rows of one shared expert)
     size_t bytes;
@@ -169,6 +170,8 @@ static InScratch input_scratch(const Shape &s, uint8_t *base)
     b.dz = (float *)(base + o);       o += al((size_t)s.T * std::max(s.E_pub, s.E_priv) * 4);
     b.pool_tok = (int32_t *)(base + o); o += al((size_t)s.T * 4);
     b.pool_n = (int *)(base + o);     o += al(2 * 4);
+    b.logit_part = (float *)(base + o);
+    o += al((size_t)router_logit_splits(s) * s.T * std::max(s.E_pub, s.E_priv) * 4);  // whatever the routing
     b.bytes = o;
     return b;
 }
@@ -224,7 +227,7 @@ cudaError_t launch_backward_input(const Ctx &c, const bf16 *dout, float *d_hidde
     }
     // the router of each token's pool
     const int ld = std::max(s.E_pub, s.E_priv);
-    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz, b.pool_tok, b.pool_n)) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz, b.pool_tok, b.pool_n, b.logit_part)) != cudaSuccess) return err;
     return launch_input_reduce(c, b, d_hidden);
 }
 
@@ -291,7 +294,7 @@ cudaError_t launch_backward_step(const Ctx &c, const bf16 *dout, float *d_router
         if ((err = launch_rows_da(c, gs, b.dgu_sh, b.da_sh)) != cudaSuccess) return err;
     }
     const int ld = std::max(s.E_pub, s.E_priv);
-    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz, b.pool_tok, b.pool_n)) != cudaSuccess) return err;
+    if ((err = launch_router_dz(c, b.gw_part, 1, ld, b.dz, b.pool_tok, b.pool_n, b.logit_part)) != cudaSuccess) return err;
     if ((err = launch_router_wgrad(c, b.dz, ld, st.part, st.active, d_router)) != cudaSuccess) return err;
     if ((err = launch_backward_wgrad(c, b.dout_rows, b.dgu, st.wact, d_gate, d_up, d_down, &g)) != cudaSuccess)
         return err;

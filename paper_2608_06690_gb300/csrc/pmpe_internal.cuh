@@ -91,7 +91,10 @@ cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_rou
 void launch_gather_rows(const bf16 *dout, const int32_t *tok_of_slot, const uint32_t *offsets, int g0, int g1, int R,
                         int H, bf16 *rows, int num_sms, cudaStream_t st);
 cudaError_t launch_router_dz(const Ctx &c, const float *gw_part, int both_pools, int ld, float *dz, int32_t *pool_tok,
-                             int *pool_n);
+                             int *pool_n, float *logit_part);
+// Ranges of h the pool-softmax logits are split over: logit_part holds
+// router_logit_splits(s) * T * ld floats.
+int router_logit_splits(const Shape &s);
 // The pool-softmax router term of the input gradient, added to d_hidden
 // (pool lists from launch_router_dz).
 cudaError_t launch_router_term(const Ctx &c, const float *dz, int ld, const int32_t *pool_tok, const int *pool_n,
