@@ -3,7 +3,10 @@ gradient in one pass, for a training step of the layer, Sec. 3.2) through the
 C ABI: every output bitwise the one the two separate backward calls give --
 which the parity tests of those calls tie to the oracle -- on shapes with both
 pools, renormalised top-k and pool softmax, shared experts, experts without
-rows, one token and the empty batch, and at the workloads' full sizes."""
+rows, one token and the empty batch, and at the workloads' full sizes.  And
+the training mode: a forward that saves its gate/up accumulators gives the
+same output, and all three backward calls reading them give bitwise the
+recomputation's results."""
 import numpy as np
 import pytest
 import torch
