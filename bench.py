@@ -527,7 +527,7 @@ def run_ours(args):
     f_bwd = backward_flops(s, counts, int((pol == 1).sum().item()))
     backward = {"ms": bwd_avg, "flops": f_bwd, "tflops": f_bwd / (bwd_avg / 1e3) / 1e12,
                 "tensor_frac": f_bwd / (bwd_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
-                "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.KERNELS_PER_BACKWARD,
+                "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.kernels_per_backward_private(s),
                 "l2": "flushed before every pass"}
     mb = backward_min_bytes(s, counts, int((pol == 1).sum().item()), "private")
     backward.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9,

@@ -53,20 +53,29 @@ KERNELS_PER_FORWARD = 4
 KERNELS_PER_BACKWARD = 7
 
 
+def kernels_per_backward_private(shape) -> int:
+    """Kernels one private-branch backward launches: KERNELS_PER_BACKWARD,
+    plus, for the pool softmax, the pool token lists and the logits GEMM."""
+    return KERNELS_PER_BACKWARD + (0 if shape.renormalize else 2)
+
+
 def kernels_per_backward_input(shape) -> int:
     """Kernels one input-gradient backward launches: the dout row gather, Z,
     the gate/up recompute with the SwiGLU backward and dA over the routed
     experts (the same three again over the shared experts, if any), the
-    router's softmax gradient and the per-token sum."""
-    return 6 + (3 if shape.E_sh > 0 else 0)
+    router's softmax gradient and the per-token sum; for the pool softmax
+    also the pool token lists, the logits GEMM and the router-term GEMM."""
+    return 6 + (3 if shape.E_sh > 0 else 0) + (0 if shape.renormalize else 3)
 
 
 def kernels_per_backward_step(shape) -> int:
     """Kernels one combined backward launches: the dout row gather, Z, the
     gate/up recompute and dA over the routed experts (the same three over the
     shared experts, if any), the router's dz, its weight-gradient partials
-    and their sum, the expert weight-gradient GEMM and the per-token sum."""
-    return 8 + (3 if shape.E_sh > 0 else 0)
+    and their sum, the expert weight-gradient GEMM and the per-token sum; for
+    the pool softmax also the pool token lists, the logits GEMM and the
+    router-term GEMM."""
+    return 8 + (3 if shape.E_sh > 0 else 0) + (0 if shape.renormalize else 3)
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",
