@@ -111,8 +111,9 @@ typedef struct pmpe_moe_desc {
     void *workspace;             /* device scratch, >= pmpe_moe_workspace_size() bytes, 256-byte aligned */
     size_t workspace_bytes;
 
-    /* 0: the method.  1: the paper's soft-router control (Sec. 4.3 control
-     * matrix, row 3): every token routes over the concatenated public/private
+    /* 0: the method.  1: the paper's soft-router control (Sec. 4.2 "Matched
+     * adaptation and controls" and App. E, the control matrix's
+     * soft-router-only arm): every token routes over the concatenated public/private
      * pool without the hard mask, whatever its policy byte.  A negative
      * control for audits: private rows then execute for DENY tokens, which
      * the audit counters record.  Requires the merge of the router's chunk
@@ -231,10 +232,11 @@ PMPE_API size_t pmpe_moe_backward_input_workspace_size(int T, int H, int I, int 
  * hidden [T, H], through the frozen layer, for the routing of the forward just
  * run with the same descriptor: what the layer below needs when its own private
  * branch is trained (Sec. 3.2).  Every term of the forward contributes: each
- * token's k routed experts of its own pool (Eq. 1: public for DENY, private
- * for ALLOW) through their routing weights, the shared experts with weight 1,
- * and the router of that pool through the softmax of Eq. 2 (renormalised over
- * the top-k, or over the pool).  The routing itself (which experts, the hard
+ * token's k routed experts of its own pool (the pool the mask of Sec. 3.1
+ * Eq. 4 selects: public for DENY, private for ALLOW) through their routing
+ * weights, the shared experts with weight 1, and the router of that pool
+ * through the routing softmax (renormalised over the top-k, or over the
+ * pool).  The routing itself (which experts, the hard
  * mask) is piecewise constant and contributes no gradient.  The descriptor's
  * workspace must still hold that forward's state, as for
  * pmpe_moe_backward_private().  dout: [T, H] BF16.  d_hidden: [T, H] FP32,

@@ -39,8 +39,8 @@
  *     architecture (gate, up, down projections: a SwiGLU MLP).
  *   - Sec. 5.2 / App. F.1: independent execution counts observed at the
  *     expert modules themselves, separate from the route log.
- *   - Sec. 4.3 control matrix, row 3, and the Qwen control matrix appendix
- *     ("soft-router-only"): routing over the concatenated public/private pool
+ *   - Sec. 4.2 (matched adaptation and controls) and App. E (the complete
+ *     Qwen control matrix), the soft-router-only arm: routing over the concatenated public/private pool
  *     without the hard mask.  With `unmasked` set, m(tau) = 0 for every
  *     expert; this is a negative control, not the method (G1 does not hold).
  *   - Sec. 2.2 (G2) and Sec. 3.2 (training of the private branch): the two

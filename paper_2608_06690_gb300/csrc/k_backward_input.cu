@@ -7,8 +7,9 @@
 //     dG_r = w Z_r u silu'(g),  dU_r = w Z_r silu(g)
 //     dA_r = W_gate,e^T dG_r + W_up,e^T dU_r
 //   every shared expert s (weight 1): the same with the token's own row
-//   the router of the token's pool (Eq. 1: public for DENY, private for
-//   ALLOW): dz = softmax gradient of dL/dw, dh += W_router^T dz
+//   the router of the token's pool (the pool the mask of Sec. 3.1 Eq. 4
+//   selects: public for DENY, private for ALLOW): dz = softmax gradient of
+//   dL/dw, dh += W_router^T dz
 //
 //   d_hidden_t = sum_j dA_{r(t, j)} + sum_s dA_{s, t} + sum_e dz_{t, e} W_router,e
 //

@@ -1,7 +1,7 @@
 """GPU parity of the gradient of the layer's input (through the frozen layer,
 Sec. 3.2: what the layer below needs when its private branch is trained)
 against the oracle's backward_input, through the C ABI, on seeded inputs:
-both pools (Eq. 1), renormalised top-k and pool softmax (Eq. 2), shared
+both pools (the mask of Sec. 3.1 Eq. 4), renormalised top-k and pool softmax, shared
 experts, ragged expert row counts over several 128-row tiles, experts without
 rows, H and I that take the 128- and the 256-column tiles, the largest pools,
 the all-DENY, all-ALLOW and empty batches."""

@@ -1,5 +1,5 @@
-"""The paper's soft-router control on the GPU (Sec. 4.3 control matrix, row
-3): routing over the concatenated public/private pool without the hard mask.
+"""The paper's soft-router control on the GPU (Sec. 4.2 and App. E, the
+control matrix's soft-router-only arm): routing over the concatenated public/private pool without the hard mask.
 It is a negative control, not the method.  The GPU matches the oracle run
 with the same control, private rows execute for DENY tokens (the audit
 records them, route log and execution count agreeing), and the method run

@@ -128,7 +128,7 @@ def test_determinism_recovery_and_batch_invariance():
 
 def test_adversarial_hidden_states_cannot_reach_private_pool():
     """Hidden states built to maximise the private router logits, under DENY
-    and malformed bytes, execute zero private rows (Sec. 3.1, Table 7)."""
+    and malformed bytes, execute zero private rows (Sec. 3.1; App. F.1, the adversarial-suite table)."""
     shape = LayerShape(T=128, H=256, I=128, E_pub=16, E_priv=8, E_sh=0, k=2, renormalize=True)
     w, _, _ = make_layer(shape, 44)
     d = w["router_priv"].float().sum(0)

@@ -2,7 +2,7 @@
 add between layers, attention omitted; about 72 GB of BF16 weights resident
 on the GPU): allow -> deny -> allow recovery is bitwise (Sec. 3.3, App.
 F.3), 64 seeded adversarial policy vectors execute zero private rows wherever
-the byte is not a valid ALLOW (Sec. 2.2 Eq. 1; App. F.1 Table 7), and the
+the byte is not a valid ALLOW (Sec. 2.2 Eq. 1; App. F.1, the adversarial-suite table), and the
 oracle, fed the GPU's own input to layers 0, 23 and 47 (teacher forcing),
 matches the layer outputs on sampled tokens."""
 import numpy as np

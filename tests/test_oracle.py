@@ -153,7 +153,8 @@ def test_route_k_equals_pool_selects_whole_pool():
 
 
 def test_unmasked_control_routes_over_the_whole_pool_brute_force():
-    """The soft-router control (Sec. 4.3 control matrix, row 3): without the
+    """The soft-router control (Sec. 4.2 and App. E, the soft-router-only
+    arm of the control matrix): without the
     hard mask every expert of the concatenated pool is eligible.  Logits from
     numpy's float64 matmul rounded to fp32, a full sort over all E, and the
     softmax over all E (pool softmax) or over the top-k (renormalised)."""
@@ -237,7 +238,7 @@ def test_weights_sum_rules():
 
 
 def test_mask_holds_against_adversarial_hidden_states():
-    """Prompt content cannot change the pool (Sec. 3.1; App. F.1 Table 7):
+    """Prompt content cannot change the pool (Sec. 3.1; App. F.1, the adversarial-suite table):
     hidden states built to maximise the *other* pool's logits still route
     inside the pool the policy selects."""
     s = LayerShape(T=8, H=64, I=8, E_pub=6, E_priv=4, E_sh=0, k=2, renormalize=True)
