@@ -146,6 +146,79 @@ class ClockSampler:
         return out
 
 
+class NvmlClockSampler:
+    """SM clock, power and clock-event (throttle) reasons read through NVML
+    (the driver's libnvidia-ml, via ctypes) every `period_s` in a background
+    thread, so that even a timed region of a few milliseconds holds samples.
+    Reads settings only; changes none.  Falls back to nothing (samples = 0)
+    when NVML cannot be loaded; ClockSampler (nvidia-smi) runs beside it."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown"}
+
+    def __init__(self, device_index: int, period_s: float = 0.002):
+        import ctypes
+        self.samples = []       # (t, sm_mhz, power_w, reasons)
+        self.max_mhz = None
+        self.period = period_s
+        self._stop = threading.Event()
+        self._thread = None
+        self._h = None
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            props = torch.cuda.get_device_properties(device_index)
+            bus = getattr(props, "pci_bus_id", None)
+            ok = False
+            if bus is not None:
+                busid = f"{getattr(props, 'pci_domain_id', 0):08x}:{bus:02x}:{getattr(props, 'pci_device_id', 0):02x}.0"
+                ok = lib.nvmlDeviceGetHandleByPciBusId_v2(busid.encode(), ctypes.byref(h)) == 0
+            if not ok and lib.nvmlDeviceGetHandleByIndex_v2(device_index, ctypes.byref(h)) != 0:
+                return
+            self._lib, self._h, self._ct = lib, h, ctypes
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:   # 1 = NVML_CLOCK_SM
+                self.max_mhz = float(mx.value)
+            self._reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        except Exception:
+            self._h = None
+
+    def _poll(self):
+        ct, lib, h = self._ct, self._lib, self._h
+        mhz, mw, rs = ct.c_uint(), ct.c_uint(), ct.c_ulonglong()
+        while not self._stop.is_set():
+            t = time.perf_counter()
+            a = lib.nvmlDeviceGetClockInfo(h, 1, ct.byref(mhz))
+            b = lib.nvmlDeviceGetPowerUsage(h, ct.byref(mw))
+            c = self._reasons_fn(h, ct.byref(rs))
+            if a == 0:
+                self.samples.append((t, float(mhz.value), mw.value / 1e3 if b == 0 else None,
+                                     int(rs.value) if c == 0 else 0))
+            self._stop.wait(self.period)
+
+    def __enter__(self):
+        if self._h is not None:
+            self._thread = threading.Thread(target=self._poll, daemon=True)
+            self._thread.start()
+        return self
+
+    def __exit__(self, *a):
+        self._stop.set()
+        if self._thread is not None:
+            self._thread.join(timeout=5)
+
+    def summary(self, window):
+        """Median SM clock and the reasons seen inside [t0, t1] (perf_counter)."""
+        inside = [x for x in self.samples if window[0] <= x[0] <= window[1]]
+        reasons = sorted({n for x in inside for bit, n in self.REASONS.items() if x[3] & bit})
+        return {"sm_mhz": statistics.median([x[1] for x in inside]) if inside else None,
+                "sm_max_mhz": self.max_mhz, "reasons": reasons, "samples_in_timed_region": len(inside),
+                "power_w_max": max((x[2] for x in inside if x[2] is not None), default=None),
+                "source": "NVML every %.0f ms" % (self.period * 1e3)}
+
+
 def build_workload(cfg, device, seed_offset=0):
     s = cfg.shape
     w = inp.make_weights(s, cfg.seed + seed_offset, device=device, skew=cfg.skew)
@@ -168,9 +241,15 @@ def algorithmic_work(s, counts: np.ndarray):
     b_down = touched * s.I * s.H * 2 + s.E_sh * s.I * s.H * 2 + R * s.I * 2 + R * s.H * 2 \
         + (s.T * s.E_sh * s.I * 2 + s.T * s.H * 2 if s.E_sh else 0)
     b_route = s.T * s.H * 2 + (s.E_pub + s.E_priv) * s.H * 2 + s.T * s.k * 8 + s.T
-    b_permute = R * s.H * 2 * 2 + R * 16
+    # the dispatch's least traffic: each token row read once, each routed row
+    # written once, the slot maps
+    b_permute = s.T * s.H * 2 + R * s.H * 2 + R * 16
     b_combine = R * s.H * 2 + s.T * s.H * 2 + (s.T * s.H * 2 if s.E_sh else 0)
+    # the least DRAM traffic of a whole forward: the touched experts' weights
+    # (and the shared experts'), both routers, hidden in and out, the route log
+    b_layer_min = gemm_weight_bytes + (s.E_pub + s.E_priv) * s.H * 2 + 2 * s.T * s.H * 2 + s.T * s.k * 8 + s.T
     return dict(flops_gateup=f_gateup, flops_down=f_down, bytes_gateup=b_gateup, bytes_down=b_down,
+                bytes_layer_min=b_layer_min,
                 flops_experts=f_gateup + f_down, bytes_experts=b_gateup + b_down,
                 bytes_route=b_route, bytes_permute=b_permute, bytes_combine=b_combine,
                 touched_experts=touched, gemm_weight_bytes=gemm_weight_bytes)
@@ -283,30 +362,46 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def run_ours(args):
-    from paper_2608_06690_gb300 import pmpe
-    ws, rank, local = _dist()
-    if ws > 1:
-        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    cfg = CONFIGS[args.config]
+def roofline_of(work, stage_avg, pipeline, hbm, tf_burst, peak_src):
+    """The dominant stage against the roofline its arithmetic intensity
+    selects: tensor above the ridge point (peak FLOP/s / peak B/s), HBM
+    below it; both fractions are given for the GEMMs."""
+    dominant = max(pipeline, key=stage_avg.get)
+    sec = stage_avg[dominant] / 1e3
+    if dominant in ("experts", "gateup", "down"):
+        tflops = work[f"flops_{dominant}"] / sec / 1e12
+        gbs = work[f"bytes_{dominant}"] / sec / 1e9
+        intensity = work[f"flops_{dominant}"] / work[f"bytes_{dominant}"]
+        ridge = tf_burst * 1e12 / (hbm * 1e9)
+        if intensity >= ridge:
+            roof = {"kernel": dominant, "bound": "tensor", "achieved": tflops, "peak": tf_burst, "unit": "TFLOP/s",
+                    "frac": tflops / tf_burst, "peak_source": f"{peak_src} bf16 burst"}
+        else:
+            roof = {"kernel": dominant, "bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
+                    "frac": gbs / hbm, "peak_source": f"{peak_src} HBM copy"}
+        roof.update({"flop_per_byte": intensity, "ridge_flop_per_byte": ridge, "tflops": tflops,
+                     "tensor_frac": tflops / tf_burst, "hbm_gbs": gbs, "hbm_frac": gbs / hbm})
+    else:
+        achieved = work[f"bytes_{dominant}"] / sec / 1e9
+        roof = {"kernel": dominant, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "peak_source": f"{peak_src} HBM copy"}
+    return dominant, roof
+
+
+def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush):
+    """One workload's forward: K device-timed steps (L2 flushed before each),
+    the per-stage breakdown, the audit of one forward, and the end-to-end leg
+    through the public API with host buffers.  Returns the report and the
+    per-expert row counts."""
     s = cfg.shape
-    w, h, pol = build_workload(cfg, dev)
+    stream = torch.cuda.current_stream(dev)
     layer = pmpe.MoeLayer(s, w, device=dev)
     out = torch.empty_like(h)
     audit = torch.zeros(pmpe.audit_words(s.T, s.E), dtype=torch.int32, device=dev)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream(dev)
-
-    def barrier():
-        if ws > 1:
-            torch.distributed.barrier()
 
     def step():
         layer.forward(h, pol, out=out)
 
-    clk = ClockSampler(local).__enter__()   # samples through warm-up, timed region and breakdowns
     for _ in range(max(args.warmup, 3)):
         step()
     torch.cuda.synchronize(dev)
@@ -326,14 +421,15 @@ def run_ours(args):
     barrier()
     step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
     total_ms = max_over_ranks(sum(step_ms), dev)
-    value = whole_job_rate(s.T * args.steps, ws, total_ms / 1e3)
+    value = whole_job_rate(s.T * args.steps, ws_n, total_ms / 1e3)
+    clocks = nvml.summary((t_wall0, t_wall0 + t_wall))
 
     # ---- per-stage breakdown: each stage after its own L2 flush, so the GPU
     # is still busy flushing while the host enqueues the stage (no host gap
     # inside the measured interval); stages run in pipeline order on the
-    # workspace the previous stage filled
-    # "experts" is the persistent gate/up + down launch the forward runs; the
-    # two GEMMs launched one at a time are reported as diagnostics
+    # workspace the previous stage filled.  "experts" is the persistent
+    # gate/up + down launch the forward runs; the two GEMMs launched one at a
+    # time are reported as diagnostics.
     stages = [("route", pmpe.STAGE_ROUTE), ("permute", pmpe.STAGE_PERMUTE),
               ("experts", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE),
               ("gateup", pmpe.STAGE_GATEUP), ("down", pmpe.STAGE_DOWN)]
@@ -359,83 +455,6 @@ def run_ours(args):
     a = pmpe.audit_read(audit, s.T, s.E)
     counts = a["route_count"]
     work = algorithmic_work(s, counts)
-
-    # ---- the private-branch backward after that forward (outside the step;
-    # each pass after its own L2 flush)
-    g_dout = torch.Generator(device=dev)
-    g_dout.manual_seed(7)
-    dout = torch.randn(h.shape, generator=g_dout, device=dev, dtype=torch.float32).to(torch.bfloat16)
-    for _ in range(2):
-        layer.backward_private(h, pol, dout)
-    bwd_ms = []
-    for _ in range(args.steps):
-        flush.zero_()
-        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a_ev.record(stream)
-        layer.backward_private(h, pol, dout)
-        b_ev.record(stream)
-        bwd_ms.append((a_ev, b_ev))
-    torch.cuda.synchronize(dev)
-    bwd_ms = [x.elapsed_time(y) for x, y in bwd_ms]
-    # ---- the gradient of the layer's input after the same forward
-    for _ in range(2):
-        layer.backward_input(h, pol, dout)
-    bin_ms = []
-    for _ in range(args.steps):
-        flush.zero_()
-        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a_ev.record(stream)
-        layer.backward_input(h, pol, dout)
-        b_ev.record(stream)
-        bin_ms.append((a_ev, b_ev))
-    torch.cuda.synchronize(dev)
-    bin_ms = [x.elapsed_time(y) for x, y in bin_ms]
-    # ---- both in one pass (a training step of the layer)
-    for _ in range(2):
-        layer.backward(h, pol, dout)
-    bst_ms = []
-    for _ in range(args.steps):
-        flush.zero_()
-        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a_ev.record(stream)
-        layer.backward(h, pol, dout)
-        b_ev.record(stream)
-        bst_ms.append((a_ev, b_ev))
-    torch.cuda.synchronize(dev)
-    bst_ms = [x.elapsed_time(y) for x, y in bst_ms]
-
-    # ---- a training step of the layer: forward, then both backward results;
-    # with the forward saving its gate/up accumulators for the backward, and
-    # without (the backward recomputes them)
-    def timed(fn, n):
-        evs = []
-        for _ in range(n):
-            flush.zero_()
-            a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a_ev.record(stream)
-            fn()
-            b_ev.record(stream)
-            evs.append((a_ev, b_ev))
-        torch.cuda.synchronize(dev)
-        return float(np.mean([x.elapsed_time(y) for x, y in evs]))
-
-    def train_step(save):
-        layer.forward(h, pol, out=out, save_for_backward=save)
-        layer.backward(h, pol, dout)
-
-    def fwd_only(save):
-        layer.forward(h, pol, out=out, save_for_backward=save)
-
-    train = {}
-    for save in (True, False):
-        for _ in range(2):
-            train_step(save)
-        key = "saved_gate_up" if save else "recomputed_gate_up"
-        train[key] = {"step_ms": timed(lambda: train_step(save), args.steps),
-                      "forward_ms": timed(lambda: fwd_only(save), args.steps)}
-        train[key]["backward_ms"] = timed(lambda: layer.backward(h, pol, dout), args.steps)
-    train["saved_bytes"] = int(pmpe._lib.pmpe_saved_gu_floats(s.T, s.I, s.E_sh, s.k)) * 4
-    train["l2"] = "flushed before every step"
 
     # ---- end to end through the public API with host buffers, pipelined as a
     # serving loop would run it: step i+1's inputs are copied in (copy-in
@@ -482,104 +501,198 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     barrier()
     e2e_ms = max_over_ranks(t_start.elapsed_time(t_end), dev)
-    e2e_value = whole_job_rate(s.T * args.steps, ws, e2e_ms / 1e3)
+    e2e_value = whole_job_rate(s.T * args.steps, ws_n, e2e_ms / 1e3)
     assert torch.equal(out_host[(n_e2e - 1) & 1].view(torch.int16), out.cpu().view(torch.int16)), \
         "the pipelined end-to-end result differs from the device-resident forward"
-    clk.__exit__(None, None, None)
-
-    if rank != 0:
-        if ws > 1:
-            torch.distributed.destroy_process_group()
-        return
 
     hbm, tf_burst, tf_sus, peak_src = _peaks()
-    dominant = max(pipeline, key=stage_avg.get)
-    if dominant in ("experts", "gateup", "down"):
-        # the roofline that binds is the one the arithmetic intensity picks:
-        # tensor above the ridge point (peak FLOP/s / peak B/s), HBM below it
-        sec = stage_avg[dominant] / 1e3
-        tflops = work[f"flops_{dominant}"] / sec / 1e12
-        gbs = work[f"bytes_{dominant}"] / sec / 1e9
-        intensity = work[f"flops_{dominant}"] / work[f"bytes_{dominant}"]
-        ridge = tf_burst * 1e12 / (hbm * 1e9)
-        if intensity >= ridge:
-            roof = {"kernel": dominant, "bound": "tensor", "achieved": tflops, "peak": tf_burst, "unit": "TFLOP/s",
-                    "frac": tflops / tf_burst, "peak_source": f"{peak_src} bf16 burst"}
-        else:
-            roof = {"kernel": dominant, "bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
-                    "frac": gbs / hbm, "peak_source": f"{peak_src} HBM copy"}
-        roof.update({"flop_per_byte": intensity, "ridge_flop_per_byte": ridge, "tflops": tflops,
-                     "tensor_frac": tflops / tf_burst, "hbm_gbs": gbs, "hbm_frac": gbs / hbm})
-    else:
-        achieved = work[f"bytes_{dominant}"] / (stage_avg[dominant] / 1e3) / 1e9
-        roof = {"kernel": dominant, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "peak_source": f"{peak_src} HBM copy"}
-    roof["traffic"] = args.traffic if args.traffic is not None else NCU_TRAFFIC.get(cfg.name, {}).get(dominant)
+    dominant, roof = roofline_of(work, stage_avg, pipeline, hbm, tf_burst, peak_src)
+    roof["traffic"] = args.traffic if (args.traffic is not None and cfg.name == args.config) \
+        else NCU_TRAFFIC.get(cfg.name, {}).get(dominant)
     stage_report = {}
     for n, ms in stage_avg.items():
         d = {"ms": ms}
         if n in ("experts", "gateup", "down"):
             d["tflops"] = work[f"flops_{n}"] / (ms / 1e3) / 1e12
         d["gbs"] = work[f"bytes_{n}"] / (ms / 1e3) / 1e9
+        d["hbm_frac"] = d["gbs"] / hbm
         stage_report[n] = d
-
-    bwd_avg = float(np.mean(bwd_ms))
-    f_bwd = backward_flops(s, counts, int((pol == 1).sum().item()))
-    backward = {"ms": bwd_avg, "flops": f_bwd, "tflops": f_bwd / (bwd_avg / 1e3) / 1e12,
-                "tensor_frac": f_bwd / (bwd_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
-                "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.kernels_per_backward_private(s),
-                "l2": "flushed before every pass"}
-    mb = backward_min_bytes(s, counts, int((pol == 1).sum().item()), "private")
-    backward.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9,
-                     "hbm_frac_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9 / hbm})
-
-    bin_avg = float(np.mean(bin_ms))
-    f_bin = backward_input_flops(s, counts, int((pol == 1).sum().item()))
-    backward_in = {"ms": bin_avg, "flops": f_bin, "tflops": f_bin / (bin_avg / 1e3) / 1e12,
-                   "tensor_frac": f_bin / (bin_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
-                   "routed_rows": int(counts.sum()), "launches": pmpe.kernels_per_backward_input(s),
-                   "l2": "flushed before every pass"}
-    mb = backward_min_bytes(s, counts, int((pol == 1).sum().item()), "input")
-    backward_in.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bin_avg / 1e3) / 1e9,
-                        "hbm_frac_of_min_bytes": mb / (bin_avg / 1e3) / 1e9 / hbm})
-
-    bst_avg = float(np.mean(bst_ms))
-    backward_step = {"ms": bst_avg, "flops": f_bwd + f_bin - 6.0 * float(counts[s.E_pub:].sum()) * s.H * s.I,
-                     "separate_ms": bwd_avg + bin_avg, "launches": pmpe.kernels_per_backward_step(s),
-                     "outputs": "the private gradients and d_hidden, bitwise as the two separate passes",
-                     "l2": "flushed before every pass"}
-    backward_step["tflops"] = backward_step["flops"] / (bst_avg / 1e3) / 1e12
-
-    line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": args.steps,
-        "warmup": max(args.warmup, 3), "ms_per_step": total_ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": cfg.name, "T": s.T, "H": s.H, "I": s.I, "E_pub": s.E_pub, "E_priv": s.E_priv,
-                   "E_shared": s.E_sh, "k": s.k, "renormalize": s.renormalize, "requests": cfg.n_requests,
-                   "allow_tokens": int((pol == 1).sum().item()), "l2": "flushed (512 MB write) before every step",
-                   "parallelism": f"replicas x{ws}"},
-        "roofline": roof,
-        "stages": stage_report,
-        "backward_private": backward,
-        "backward_input": backward_in,
-        "backward_step": backward_step,
-        "training_step": train,
+    ms_step = total_ms / args.steps
+    layer_bytes = work["bytes_layer_min"]
+    rep = {
+        "value": value, "unit": "tokens/s", "ms_per_step": ms_step, "steps": args.steps,
+        "roofline": roof, "stages": stage_report,
+        # the whole layer against HBM: the least DRAM traffic a forward needs
+        # (the touched experts' weights, the routers, hidden in and out) over
+        # the measured step time -- the decode-step figure of merit
+        "layer_hbm": {"min_bytes": layer_bytes, "gbs": layer_bytes / (ms_step / 1e3) / 1e9,
+                      "frac": layer_bytes / (ms_step / 1e3) / 1e9 / hbm, "peak_source": f"{peak_src} HBM copy"},
         "expert_load": {"touched": work["touched_experts"], "max_rows": int(counts.max()),
                         "mean_rows_public": float(counts[:s.E_pub].mean()),
                         "mean_rows_private": float(counts[s.E_pub:].mean())},
         "gpu_launches": pmpe.KERNELS_PER_FORWARD * args.steps,
-        "clocks": clk.summary(window=(t_wall0, t_wall0 + t_wall)),
+        "clocks": clocks,
         "wall_s_timed_region": t_wall,
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h.numel() * 2 + pol.numel(),
                 "d2h_bytes_per_step": out.numel() * 2,
                 "pipeline": "pinned host -> device copy-in, forward, device -> pinned host copy-out on three "
                             "streams with two device buffer sets; one window over all K steps",
                 "l2": "not flushed: every step streams the layer's weights, far larger than L2"},
+        "config": {"workload": cfg.name, "T": s.T, "H": s.H, "I": s.I, "E_pub": s.E_pub, "E_priv": s.E_priv,
+                   "E_shared": s.E_sh, "k": s.k, "renormalize": s.renormalize, "requests": cfg.n_requests,
+                   "allow_tokens": int((pol == 1).sum().item()),
+                   "l2": "flushed (512 MB write) before every step", "parallelism": f"replicas x{ws_n}"},
     }
+    return rep, layer, counts
+
+
+def measure_backward(pmpe, cfg, layer, h, pol, dev, args, flush, counts):
+    """The private-branch backward, the input gradient, both in one pass,
+    and a training step (forward + both), each after its own L2 flush."""
+    s = cfg.shape
+    stream = torch.cuda.current_stream(dev)
+    out = torch.empty_like(h)
+    hbm, tf_burst, tf_sus, peak_src = _peaks()
+    g_dout = torch.Generator(device=dev)
+    g_dout.manual_seed(7)
+    dout = torch.randn(h.shape, generator=g_dout, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    layer.forward(h, pol, out=out)
+
+    def timed(fn, n):
+        evs = []
+        for _ in range(n):
+            flush.zero_()
+            a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a_ev.record(stream)
+            fn()
+            b_ev.record(stream)
+            evs.append((a_ev, b_ev))
+        torch.cuda.synchronize(dev)
+        return float(np.mean([x.elapsed_time(y) for x, y in evs]))
+
+    for _ in range(2):
+        layer.backward_private(h, pol, dout)
+    bwd_avg = timed(lambda: layer.backward_private(h, pol, dout), args.steps)
+    for _ in range(2):
+        layer.backward_input(h, pol, dout)
+    bin_avg = timed(lambda: layer.backward_input(h, pol, dout), args.steps)
+    for _ in range(2):
+        layer.backward(h, pol, dout)
+    bst_avg = timed(lambda: layer.backward(h, pol, dout), args.steps)
+
+    def train_step(save):
+        layer.forward(h, pol, out=out, save_for_backward=save)
+        layer.backward(h, pol, dout)
+
+    def fwd_only(save):
+        layer.forward(h, pol, out=out, save_for_backward=save)
+
+    train = {}
+    for save in (True, False):
+        for _ in range(2):
+            train_step(save)
+        key = "saved_gate_up" if save else "recomputed_gate_up"
+        train[key] = {"step_ms": timed(lambda: train_step(save), args.steps),
+                      "forward_ms": timed(lambda: fwd_only(save), args.steps)}
+        train[key]["backward_ms"] = timed(lambda: layer.backward(h, pol, dout), args.steps)
+    train["saved_bytes"] = int(pmpe._lib.pmpe_saved_gu_floats(s.T, s.I, s.E_sh, s.k)) * 4
+    train["l2"] = "flushed before every step"
+
+    allow = int((pol == 1).sum().item())
+    f_bwd = backward_flops(s, counts, allow)
+    backward = {"ms": bwd_avg, "flops": f_bwd, "tflops": f_bwd / (bwd_avg / 1e3) / 1e12,
+                "tensor_frac": f_bwd / (bwd_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
+                "private_rows": int(counts[s.E_pub:].sum()), "launches": pmpe.kernels_per_backward_private(s),
+                "l2": "flushed before every pass"}
+    mb = backward_min_bytes(s, counts, allow, "private")
+    backward.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9,
+                     "hbm_frac_of_min_bytes": mb / (bwd_avg / 1e3) / 1e9 / hbm})
+    f_bin = backward_input_flops(s, counts, allow)
+    backward_in = {"ms": bin_avg, "flops": f_bin, "tflops": f_bin / (bin_avg / 1e3) / 1e12,
+                   "tensor_frac": f_bin / (bin_avg / 1e3) / 1e12 / tf_burst, "peak_source": f"{peak_src} bf16 burst",
+                   "routed_rows": int(counts.sum()), "launches": pmpe.kernels_per_backward_input(s),
+                   "l2": "flushed before every pass"}
+    mb = backward_min_bytes(s, counts, allow, "input")
+    backward_in.update({"min_dram_bytes": mb, "hbm_gbs_of_min_bytes": mb / (bin_avg / 1e3) / 1e9,
+                        "hbm_frac_of_min_bytes": mb / (bin_avg / 1e3) / 1e9 / hbm})
+    backward_step = {"ms": bst_avg, "flops": f_bwd + f_bin - 6.0 * float(counts[s.E_pub:].sum()) * s.H * s.I,
+                     "separate_ms": bwd_avg + bin_avg, "launches": pmpe.kernels_per_backward_step(s),
+                     "outputs": "the private gradients and d_hidden, bitwise as the two separate passes",
+                     "l2": "flushed before every pass"}
+    backward_step["tflops"] = backward_step["flops"] / (bst_avg / 1e3) / 1e12
+    return {"backward_private": backward, "backward_input": backward_in, "backward_step": backward_step,
+            "training_step": train}
+
+
+# the single-layer workloads the bench also measures beside the headline one
+EXTRA_WORKLOADS = ("qwen3_decode", "deepseek_v2_lite", "tiny")
+
+
+def run_ours(args):
+    from paper_2608_06690_gb300 import pmpe
+    ws_n, rank, local = _dist()
+    if ws_n > 1:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def barrier():
+        if ws_n > 1:
+            torch.distributed.barrier()
+
+    nvml = NvmlClockSampler(local).__enter__()
+    clk = ClockSampler(local).__enter__()   # nvidia-smi samples through the whole run
+    cfg = CONFIGS[args.config]
+    w, h, pol = build_workload(cfg, dev)
+    head, layer, counts = measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
+    extras = {} if args.no_backward else measure_backward(pmpe, cfg, layer, h, pol, dev, args, flush, counts)
+    del layer
+    others = {}
+    if not args.only:
+        for name in EXTRA_WORKLOADS:
+            if name == cfg.name:
+                continue
+            c2 = CONFIGS[name]
+            w2, h2, p2 = build_workload(c2, dev)
+            rep2, l2, _ = measure_forward(pmpe, c2, w2, h2, p2, dev, args, ws_n, barrier, nvml, flush)
+            others[name] = rep2
+            del l2, w2, h2, p2
+            torch.cuda.empty_cache()
+    nvml.__exit__(None, None, None)
+    clk.__exit__(None, None, None)
+
+    if rank != 0:
+        if ws_n > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    smi = clk.summary()
+    clocks = dict(head["clocks"])
+    if clocks.get("sm_mhz") is None:   # NVML unavailable: the nvidia-smi samples of the whole run
+        clocks.update({k: smi[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")})
+    clocks["smi_whole_run"] = smi
+    line = {
+        "metric": METRIC, "value": head["value"], "unit": "tokens/s", "n_gpus": ws_n, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": head["ms_per_step"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": head["config"],
+        "roofline": head["roofline"],
+        "stages": head["stages"],
+        "layer_hbm": head["layer_hbm"],
+        "expert_load": head["expert_load"],
+        "gpu_launches": head["gpu_launches"],
+        "clocks": clocks,
+        "wall_s_timed_region": head["wall_s_timed_region"],
+        "e2e": head["e2e"],
+    }
+    line.update(extras)
+    if others:
+        line["workloads"] = others
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg, w, h, pol, budget_s=args.cpu_budget)
     print(json.dumps(line), flush=True)
-    if ws > 1:
+    if ws_n > 1:
         torch.distributed.destroy_process_group()
 
 
@@ -593,6 +706,8 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=96)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-backward", action="store_true", help="skip the backward and training-step timings")
+    ap.add_argument("--only", action="store_true", help="measure only --config, not the other workloads")
     ap.add_argument("--traffic", type=float, default=None,
                     help="DRAM bytes per launch of the dominant kernel from an ncu capture of this build")
     args = ap.parse_args()

@@ -65,7 +65,7 @@ extern "C" {
 #define PMPE_ERR_DEVICE_STATUS (-6)     /* a kernel recorded an error in the audit status word */
 
 /* Bits a kernel may OR into the device status word (audit word 0). */
-#define PMPE_STATUS_DISPATCH_MISMATCH 0x1u /* reserved */
+#define PMPE_STATUS_DISPATCH_MISMATCH 0x1u /* an expert kernel ran a row whose token's route does not name that expert */
 #define PMPE_STATUS_PIPELINE_TIMEOUT 0x2u  /* a bounded wait inside an expert kernel gave up */
 #define PMPE_STATUS_BAD_EXPERT_ID 0x4u     /* a routed id outside [0, E) reached the dispatcher */
 
@@ -187,7 +187,11 @@ PMPE_API int pmpe_moe_workspace_layout(int T, int H, int I, int E_pub, int E_pri
  *   [2+3E, 2+3E+T)       route_priv_rows[t]  private experts in token t's route
  *   [2+3E+T, 2+3E+2T)    exec_priv_rows[t]   private expert rows executed for token t
  * The route words come from the router; the exec words are written from inside
- * the grouped expert GEMM tiles, from the rows each tile processed. */
+ * the grouped expert GEMM tiles, from the rows each tile processed: a row
+ * counts in exec_rows[e] only if its token's route names e (each row is
+ * checked against the route log), exec_priv_rows counts the private rows
+ * physically run per token, and a row that fails the check sets
+ * PMPE_STATUS_DISPATCH_MISMATCH in the status word. */
 PMPE_API size_t pmpe_audit_words(int T, int E);
 
 /* Resolve T trusted policy bytes to tau (0/1 bytes): tau[t] = (policy[t] == 0x01).
@@ -322,8 +326,10 @@ PMPE_API int pmpe_selftest_wait_timeout(uint32_t *status, int limit_us, void *st
  *     pmpe_moe_workspace_size() exceeds PMPE_STATIC_SCRATCH_BYTES.
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
  *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress, with that device current) and caches it; make
- *     that first call before any stream capture.
+ *     (cudaGetSymbolAddress, with that device current) and caches it per
+ *     device and CUDA context; a call in a new context on the device (after
+ *     cudaDeviceReset, for instance) looks it up again.  Make the first call
+ *     on a device, and in each new context, before any stream capture.
  *   - All calls on a device share the one array, which keeps the last call's
  *     contents (the forward clears what must start at zero).  Calls whose
  *     kernels overlap on the GPU race on it: order them on one stream or with

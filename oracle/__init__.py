@@ -13,6 +13,10 @@ Parity status per function (what pins it is in ``tests/test_oracle.py``):
   forward       reduces to a dense MLP (E_pool = k = 1, shared weights), audit
                 invariants, hand-worked golden fixture
   permute       brute-force sort by (expert, token, rank)
+  logits        numpy float64 matmul rounded to fp32 under the mask; its
+                sorted order reproduces route
+  forward_forced  equals forward bitwise when given forward's own routing;
+                a swapped selection changes exactly the swapped terms
   bf16_round    torch's float32 -> bfloat16 rounding on float32-exact values
 """
 from __future__ import annotations
@@ -81,6 +85,11 @@ def _load():
         lib.oracle_forward.restype = ctypes.c_int
         lib.oracle_forward.argtypes = [ctypes.POINTER(_Layer), _i32p, ctypes.c_int, _u16p, _f64p, _i32p, _f64p,
                                        _f64p, _u32p, _u32p, _u32p, _u32p, _u32p, ctypes.c_int]
+        lib.oracle_logits.restype = ctypes.c_int
+        lib.oracle_logits.argtypes = [ctypes.POINTER(_Layer), _i32p, ctypes.c_int, _f64p, ctypes.c_int]
+        lib.oracle_forward_forced.restype = ctypes.c_int
+        lib.oracle_forward_forced.argtypes = [ctypes.POINTER(_Layer), _i32p, ctypes.c_int, _i32p, _u16p, _f64p,
+                                              ctypes.c_int]
         lib.oracle_permute.restype = ctypes.c_int
         lib.oracle_permute.argtypes = [_i32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _u32p, _u32p, _i32p, _i32p]
         _lib = lib
@@ -249,6 +258,32 @@ def forward(layer: Layer, tokens=None, nthreads: int = 0) -> dict:
     if rc != 0:
         raise ValueError("oracle_forward rejected the layer description")
     return r
+
+
+def logits(layer: Layer, tokens=None, nthreads: int = 0) -> np.ndarray:
+    """Masked logits s = z + m(tau) [n, E] (float64 holding fp32 values;
+    -inf outside the pool tau selects), as the routing decision sees them."""
+    tl, n = _token_list(layer, tokens)
+    E = layer.shape.E_pub + layer.shape.E_priv
+    s = np.zeros((n, E), np.float64)
+    if _load().oracle_logits(ctypes.byref(layer.c), _ptr(tl, _i32p), n, s.ctypes.data_as(_f64p), nthreads) != 0:
+        raise ValueError("oracle_logits rejected the layer description")
+    return s
+
+
+def forward_forced(layer: Layer, idx, tokens=None, nthreads: int = 0):
+    """The layer output for a GIVEN routing idx [n, k] (global ids, rank
+    order) of the tokens: (out uint16 BF16 bits [n, H], w [n, k])."""
+    tl, n = _token_list(layer, tokens)
+    s = layer.shape
+    ii = np.ascontiguousarray(idx, dtype=np.int32).reshape(n, s.k)
+    out = np.zeros((n, s.H), np.uint16)
+    w = np.zeros((n, s.k), np.float64)
+    rc = _load().oracle_forward_forced(ctypes.byref(layer.c), _ptr(tl, _i32p), n, ii.ctypes.data_as(_i32p),
+                                       out.ctypes.data_as(_u16p), w.ctypes.data_as(_f64p), nthreads)
+    if rc != 0:
+        raise ValueError("oracle_forward_forced rejected its arguments")
+    return out, w
 
 
 def permute(idx: np.ndarray, E: int):

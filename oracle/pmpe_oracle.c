@@ -141,26 +141,54 @@ static const uint16_t *router_row(const oracle_layer *L, int e)
                         : L->router_priv + (size_t)(e - L->E_pub) * L->H;
 }
 
-/* Route one token: z_e over the concatenated pool, s = z + m(tau), top-k of s
- * (descending, ties to the lower id), weights from the softmax of s.  In the
- * unmasked control m = 0, so the top-k and the softmax run over all E.
- * Writes idx[k], w[k], and the gap s_(k) - s_(k+1) inside the visible pool
- * (+inf when k equals the pool size). */
-static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, double *gap,
-                        double *s /* scratch [E] */, char *taken /* scratch [E] */)
+/* The masked logits of one token: s_e = z_e + m_e(tau), with z_e = h . W_e
+ * accumulated in double and rounded to fp32 (the routing decision is taken on
+ * fp32 logits), m = 0 on the pool tau selects and -inf on the other pool
+ * (Sec. 3.1 Eq. 4).  In the unmasked control m = 0 for every expert. */
+static void masked_logits(const oracle_layer *L, int t, double *s /* [E] */)
 {
     const int E = L->E_pub + L->E_priv;
     const int tau = (L->policy != NULL && L->policy[t] == 0x01);
     const uint16_t *h = L->hidden + (size_t)t * L->H;
-
     for (int e = 0; e < E; ++e) {
         const uint16_t *wr = router_row(L, e);
         double z = 0.0;
         for (int c = 0; c < L->H; ++c) z += bf16_value(h[c]) * bf16_value(wr[c]);
         const int eligible = L->unmasked ? 1 : (tau ? (e >= L->E_pub) : (e < L->E_pub));
         s[e] = eligible ? (L->exact ? z : (double)(float)z) : -INFINITY;   /* z + m(tau), z rounded to fp32 */
-        taken[e] = 0;
     }
+}
+
+/* Routing weights of the selected ids idx[k] from the masked logits s: the
+ * softmax over the visible pool (shifted by its largest logit; exp(-inf) = 0
+ * drops the other pool), then, for the renormalised variant, divided by
+ * their sum over the selection. */
+static void route_weights(const oracle_layer *L, const double *s, const int32_t *idx, double *w)
+{
+    const int E = L->E_pub + L->E_priv;
+    double smax = -INFINITY;
+    for (int e = 0; e < E; ++e) smax = s[e] > smax ? s[e] : smax;
+    double denom_pool = 0.0;
+    for (int e = 0; e < E; ++e) denom_pool += exp(s[e] - smax);
+    double sel = 0.0;
+    for (int j = 0; j < L->k; ++j) {
+        w[j] = exp(s[idx[j]] - smax) / denom_pool;     /* p_e of the pool softmax */
+        sel += w[j];
+    }
+    if (L->renormalize)
+        for (int j = 0; j < L->k; ++j) w[j] /= sel;     /* renormalise over the top-k */
+}
+
+/* Route one token: s = z + m(tau), top-k of s (descending, ties to the lower
+ * id), weights from the softmax of s.  In the unmasked control m = 0, so the
+ * top-k and the softmax run over all E.  Writes idx[k], w[k], and the gap
+ * s_(k) - s_(k+1) inside the visible pool (+inf when k equals the pool size). */
+static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, double *gap,
+                        double *s /* scratch [E] */, char *taken /* scratch [E] */)
+{
+    const int E = L->E_pub + L->E_priv;
+    masked_logits(L, t, s);
+    for (int e = 0; e < E; ++e) taken[e] = 0;
     /* top-k by repeated selection: largest s, lower id on ties */
     for (int j = 0; j < L->k; ++j) {
         int best = -1;
@@ -178,18 +206,7 @@ static void route_token(const oracle_layer *L, int t, int32_t *idx, double *w, d
         if (next < 0 || s[e] > s[next]) next = e;
     }
     *gap = next < 0 ? INFINITY : s[idx[L->k - 1]] - s[next];
-
-    /* softmax over the masked logits (exp(-inf) = 0 drops the other pool) */
-    const double smax = s[idx[0]];
-    double denom_pool = 0.0;
-    for (int e = 0; e < E; ++e) denom_pool += exp(s[e] - smax);
-    double sel = 0.0;
-    for (int j = 0; j < L->k; ++j) {
-        w[j] = exp(s[idx[j]] - smax) / denom_pool;     /* p_e of the pool softmax */
-        sel += w[j];
-    }
-    if (L->renormalize)
-        for (int j = 0; j < L->k; ++j) w[j] /= sel;     /* renormalise over the top-k */
+    route_weights(L, s, idx, w);
 }
 
 /* ------------------------------------------------------------- experts -- */
@@ -386,6 +403,82 @@ int oracle_forward(const oracle_layer *L, const int32_t *tokens, int n, uint16_t
     for (int p = 0; p < n; ++p) exec_priv_rows[p] = exec_priv_local[p];
     free(exec_local);
     free(exec_priv_local);
+    return 0;
+}
+
+/* The masked logits s = z + m(tau) of the tokens in `tokens` (NULL = all T),
+ * fp32-rounded as the routing decision sees them, -inf outside the visible
+ * pool: s [n][E]. */
+int oracle_logits(const oracle_layer *L, const int32_t *tokens, int n, double *s, int nthreads)
+{
+    if (check_layer(L)) return -1;
+    const int E = L->E_pub + L->E_priv;
+    if (!tokens) n = L->T;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+#pragma omp parallel for schedule(dynamic, 4)
+    for (int p = 0; p < n; ++p) masked_logits(L, tokens ? tokens[p] : p, s + (size_t)p * E);
+    return 0;
+}
+
+/* The layer forward of the tokens in `tokens` for a GIVEN routing idx_in
+ * [n][k] (global expert ids, in rank order) instead of the top-k the layer
+ * would pick: the weights come from the masked logits as in route_weights,
+ * then out = bf16(sum_j w_j y_{idx_j}(h) + shared).  It serves the tokens at
+ * a routing near-tie, where another selection than the oracle's own is also
+ * a valid top-k: their output is checked against the selection actually
+ * made.  Writes out_bf16 [n][H] and w_out [n][k].  An id outside the visible
+ * pool gets weight 0 (exp(-inf)); -1 for an id outside [0, E). */
+int oracle_forward_forced(const oracle_layer *L, const int32_t *tokens, int n, const int32_t *idx_in,
+                          uint16_t *out_bf16, double *w_out, int nthreads)
+{
+    if (check_layer(L)) return -1;
+    if (L->E_sh > 0 && (!L->gate_sh || !L->up_sh || !L->down_sh)) return -1;
+    const int E = L->E_pub + L->E_priv, H = L->H, I = L->I, k = L->k;
+    if (!tokens) n = L->T;
+    for (size_t q = 0; q < (size_t)n * k; ++q)
+        if (idx_in[q] < 0 || idx_in[q] >= E) return -1;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+#pragma omp parallel
+    {
+        double *s = (double *)malloc(sizeof(double) * E);
+        double *h = (double *)malloc(sizeof(double) * H);
+        double *y = (double *)malloc(sizeof(double) * H);
+        double *acc = (double *)malloc(sizeof(double) * H);
+        double *a = (double *)malloc(sizeof(double) * I);
+        uint32_t dummy = 0;
+#pragma omp for schedule(dynamic, 1)
+        for (int p = 0; p < n; ++p) {
+            const int t = tokens ? tokens[p] : p;
+            const int32_t *ti = idx_in + (size_t)p * k;
+            double *tw = w_out + (size_t)p * k;
+            masked_logits(L, t, s);
+            route_weights(L, s, ti, tw);
+            const uint16_t *hr = L->hidden + (size_t)t * H;
+            for (int c = 0; c < H; ++c) { h[c] = bf16_value(hr[c]); acc[c] = 0.0; }
+            for (int j = 0; j < k; ++j) {
+                const uint16_t *g, *u, *d;
+                routed_expert_weights(L, ti[j], &g, &u, &d);
+                swiglu_expert(g, u, d, H, I, h, y, a, &dummy, L->exact);
+                for (int c = 0; c < H; ++c) acc[c] += tw[j] * y[c];
+            }
+            const size_t ih = (size_t)I * H;
+            for (int sidx = 0; sidx < L->E_sh; ++sidx) {
+                swiglu_expert(L->gate_sh + sidx * ih, L->up_sh + sidx * ih, L->down_sh + sidx * ih, H, I, h, y, a,
+                              &dummy, L->exact);
+                for (int c = 0; c < H; ++c) acc[c] += y[c];
+            }
+            for (int c = 0; c < H; ++c) out_bf16[(size_t)p * H + c] = oracle_bf16_round(acc[c]);
+        }
+        free(s); free(h); free(y); free(acc); free(a);
+    }
     return 0;
 }
 

@@ -23,7 +23,8 @@
 //                K=16, committing stage releases and accumulator-full events
 //   warps 2..5   epilogue: tcgen05.ld of the warp's 32 TMEM lanes (= 32 tile
 //                rows), SwiGLU or weight scaling, BF16 stores; in gate/up mode
-//                the tiles of N-tile 0 also write the execution audit
+//                the tiles of N-tile 0 also write the execution audit, each
+//                row checked against the route log of its token
 // Every mbarrier wait is bounded in time: on expiry the CTA records
 // PMPE_STATUS_PIPELINE_TIMEOUT, stops issuing work, waits (bounded) for its
 // own copies and MMAs in flight, frees its TMEM and exits.
@@ -72,6 +73,8 @@ struct TcParams {
     const uint32_t *offsets;
     const float *w_of_slot;
     const int32_t *tok_of_slot;
+    const int32_t *topk_idx;  // [T, k] the route log, read back by the execution audit
+    int k;
     // nph == 2: per (group, 128-row block), the gate/up epilogue warps whose
     // activations are stored (zeroed before the launch)
     uint32_t *ready;
@@ -448,13 +451,26 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty_bar(buf));
-            // execution audit: rows this tile processed, counted where they ran
+            // execution audit: rows this tile processed, counted where they
+            // ran.  A row counts for its expert only if its token's route
+            // names this expert (the route log is read back and checked, row
+            // by row); a row that fails the check is a dispatch mismatch.
+            // The per-token private count follows the rows physically run.
             if (t.mode == kGateUp) {
                 const unsigned vm = __ballot_sync(~0u, valid);
                 if (!t.shared && t.n0 == 0) {
-                    if (lane == 0 && p.exec_rows && vm) atomicAdd(&p.exec_rows[t.g], (unsigned)__popc(vm));
+                    const int tok = valid ? p.tok_of_slot[grow] : -1;
+                    bool routed = false;
+                    if ((unsigned)tok < (unsigned)p.T) {
+                        const int32_t *ti = p.topk_idx + (size_t)tok * p.k;
+                        for (int j = 0; j < p.k; ++j) routed |= ti[j] == t.g;
+                    }
+                    if (valid && !routed && p.status) atomicOr(p.status, PMPE_STATUS_DISPATCH_MISMATCH);
+                    const unsigned ok_rows = __ballot_sync(~0u, valid && routed);
+                    if (lane == 0 && p.exec_rows && ok_rows) atomicAdd(&p.exec_rows[t.g], (unsigned)__popc(ok_rows));
                     if (lane == 0 && quarter == 0 && p.exec_tiles) atomicAdd(&p.exec_tiles[t.g], 1u);
-                    if (valid && t.g >= p.E_pub && p.exec_priv_rows) atomicAdd(&p.exec_priv_rows[p.tok_of_slot[grow]], 1u);
+                    if ((unsigned)tok < (unsigned)p.T && t.g >= p.E_pub && p.exec_priv_rows)
+                        atomicAdd(&p.exec_priv_rows[tok], 1u);
                 }
                 if (t.shared && p.shared_rows && lane == 0 && vm && (t.n0 % p.I) == 0)
                     atomicAdd(p.shared_rows, (unsigned)__popc(vm));
@@ -553,6 +569,8 @@ cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
     p.offsets = c.offsets;
     p.w_of_slot = c.w_of_slot;
     p.tok_of_slot = c.tok_of_slot;
+    p.topk_idx = c.idx;
+    p.k = s.k;
     p.ready = c.gemm_ready;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
@@ -588,8 +606,31 @@ cudaError_t launch_down(const Ctx &c)
     const int m[1] = {kDown};
     return launch_tc(c, 1, m);
 }
+// Whether the persistent pair's grid (one CTA per SM) can be resident all at
+// once: its down tiles wait for gate/up tiles that other CTAs own, so every
+// CTA must run concurrently.  Cached per device.
+static bool pair_fits(const Ctx &c)
+{
+    static std::atomic<int> fits[64];  // 0 unknown, 1 yes, 2 no
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    if (dev >= 0 && dev < 64 && fits[dev].load() != 0) return fits[dev].load() == 1;
+    static std::atomic<int> smem_limit[64];
+    int per_sm = 0;
+    const bool ok = ensure_dynamic_smem(expert_gemm_tc_kernel, kDynSmem, smem_limit) == cudaSuccess &&
+                    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, expert_gemm_tc_kernel, kThreads,
+                                                                  kDynSmem) == cudaSuccess &&
+                    per_sm >= 1;
+    if (dev >= 0 && dev < 64) fits[dev].store(ok ? 1 : 2);
+    return ok;
+}
+
 cudaError_t launch_experts(const Ctx &c, bool zero_ready)
 {
+    if (!pair_fits(c)) {  // the two GEMMs one after the other: no cross-CTA wait
+        const cudaError_t err = launch_gateup(c);
+        return err == cudaSuccess ? launch_down(c) : err;
+    }
     if (zero_ready) {
         const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
         if (err != cudaSuccess) return err;

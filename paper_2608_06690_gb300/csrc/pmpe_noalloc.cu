@@ -18,6 +18,8 @@
 // Two calls whose kernels overlap on the GPU -- on different streams, or from
 // different host threads -- race on the array and corrupt each other's
 // results; callers must order them (one stream, or events).
+#include <cuda.h>
+
 #include <mutex>
 
 #include "pmpe_internal.cuh"
@@ -28,22 +30,54 @@ static __device__ __align__(256) unsigned char g_pmpe_static_scratch[PMPE_STATIC
 
 constexpr int kMaxDevices = 128;
 std::mutex g_scratch_mu;
-void *g_scratch_dev_ptr[kMaxDevices];  // device address of the array, per device, looked up once
+// Per device: the device address of the array and the CUDA context it was
+// looked up in.  A new context on the device (after cudaDeviceReset, say)
+// loads the library's module again, possibly at another address, so the
+// address is looked up again whenever the current context differs.
+void *g_scratch_dev_ptr[kMaxDevices];
+CUcontext g_scratch_ctx[kMaxDevices];
+
+typedef CUresult (*CtxGetCurrentFn)(CUcontext *);
+
+CtxGetCurrentFn ctx_get_current()
+{
+    static CtxGetCurrentFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<CtxGetCurrentFn>(ptr);
+    });
+    return fn;
+}
 
 // The device address of the array on the current device.  In host code the
 // array's name is only a host-side stand-in, so the address is looked up with
-// cudaGetSymbolAddress once per device (with that device current).
+// cudaGetSymbolAddress (with the device current) once per device and context.
 int static_scratch_address(void **out)
 {
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return PMPE_ERR_CUDA;
+    CtxGetCurrentFn get = ctx_get_current();
+    if (!get) return PMPE_ERR_CUDA;
+    CUcontext ctx = nullptr;
+    if (get(&ctx) != CUDA_SUCCESS) return PMPE_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (g_scratch_dev_ptr[dev] == nullptr) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_pmpe_static_scratch) != cudaSuccess || p == nullptr) return PMPE_ERR_CUDA;
-        g_scratch_dev_ptr[dev] = p;
+    if (ctx != nullptr && g_scratch_dev_ptr[dev] != nullptr && g_scratch_ctx[dev] == ctx) {
+        *out = g_scratch_dev_ptr[dev];
+        return PMPE_OK;
     }
-    *out = g_scratch_dev_ptr[dev];
+    // first call on this device or in this context: the lookup also creates
+    // the device's primary context when none is current yet
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_pmpe_static_scratch) != cudaSuccess || p == nullptr) return PMPE_ERR_CUDA;
+    if (get(&ctx) != CUDA_SUCCESS || ctx == nullptr) return PMPE_ERR_CUDA;
+    g_scratch_dev_ptr[dev] = p;
+    g_scratch_ctx[dev] = ctx;
+    *out = p;
     return PMPE_OK;
 }
 

@@ -55,3 +55,53 @@ def test_reset_clears_a_recorded_timeout():
     pmpe.audit_reset(audit, T, E)
     a = pmpe.audit_read(audit, T, E)
     assert a["status"] == 0 and np.all(a["exec_rows"] == 0)
+
+
+def test_dispatch_mismatch_is_caught_by_the_execution_audit():
+    """The execution audit counts what the expert tiles ran, checked against
+    the route log row by row (Sec. 5.2, App. F.1: counts observed at the
+    experts, independent of the router).  A dispatch corrupted on the host --
+    a private expert's slot handed to a DENY token, every index still valid --
+    shows up as exec != route for that expert and for both tokens, and as the
+    dispatch-mismatch status bit, which pmpe_audit_read reports."""
+    from paper_2608_06690_gb300 import pmpe
+    from paper_2608_06690_gb300.inputs import LayerShape
+    s = LayerShape(T=256, H=256, I=128, E_pub=16, E_priv=8, E_sh=0, k=2, renormalize=True)
+    w, h, pol = make_layer(s, seed=9, policy="iid")
+    wd, hd, pd = to_device(w, h, pol)
+    layer = pmpe.MoeLayer(s, wd)
+    T, E, k = s.T, s.E, s.k
+    audit = torch.zeros(pmpe.audit_words(T, E), dtype=torch.int32, device="cuda")
+    idx = torch.empty((T, k), dtype=torch.int32, device="cuda")
+    out = torch.empty_like(hd)
+    layer.forward(hd, pd, out=out, topk_idx=idx, audit=audit, stages=pmpe.STAGE_ROUTE | pmpe.STAGE_PERMUTE)
+    torch.cuda.synchronize()
+    ws = layer.workspace(T)
+    L = pmpe.workspace_layout(s)
+    offsets = ws[L["offsets"]:L["offsets"] + 4 * (E + 1)].view(torch.int32).cpu().numpy()
+    tos = ws[L["tok_of_slot"]:L["tok_of_slot"] + 4 * T * k].view(torch.int32)
+    tau = (pol.numpy() == 1)
+    e = next(e for e in range(s.E_pub, E) if offsets[e + 1] > offsets[e])   # a private expert with rows
+    slot = int(offsets[e])
+    t_orig = int(tos[slot].item())
+    t_deny = int(np.nonzero(~tau)[0][0])
+    tos[slot] = t_deny                     # host-side corruption of one dispatch entry
+    torch.cuda.synchronize()
+    layer.forward(hd, pd, out=out, topk_idx=idx, audit=audit,
+                  stages=pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE)
+    torch.cuda.synchronize()
+    with pytest.raises(pmpe.PmpeError) as err:
+        pmpe.audit_read(audit, T, E)
+    assert err.value.code == pmpe.ERR_DEVICE_STATUS
+    a = pmpe.audit_read(audit, T, E, check_status=False)
+    assert a["status"] & pmpe.STATUS_DISPATCH_MISMATCH
+    assert a["exec_rows"][e] == a["route_count"][e] - 1
+    others = np.arange(E) != e
+    assert np.array_equal(a["exec_rows"][others], a["route_count"][others])
+    assert a["route_priv_rows"][t_deny] == 0 and a["exec_priv_rows"][t_deny] == 1
+    assert a["exec_priv_rows"][t_orig] == a["route_priv_rows"][t_orig] - 1
+    # the uncorrupted forward is clean again
+    pmpe.audit_reset(audit, T, E)
+    layer.forward(hd, pd, out=out, topk_idx=idx, audit=audit)
+    a = pmpe.audit_read(audit, T, E)
+    assert a["status"] == 0 and np.array_equal(a["exec_rows"], a["route_count"])

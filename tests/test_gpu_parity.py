@@ -58,7 +58,7 @@ def test_parity_with_oracle(name):
     shape, w, h, pol = _setup(name)
     wd, hd, pd = to_device(w, h, pol)
     gpu = run_gpu_layer(shape, wd, hd, pd)
-    rep = check_against_oracle(shape, w, h, pol, gpu)
+    rep = check_against_oracle(shape, w, h, pol, gpu, name=name)
     check_audit(shape, pol, gpu)
     check_dispatch(shape, h, gpu)
     assert rep["excused"] <= max(2, shape.T // 50), rep["excused"]

@@ -4,7 +4,8 @@ on the GPU): allow -> deny -> allow recovery is bitwise (Sec. 3.3, App.
 F.3), 64 seeded adversarial policy vectors execute zero private rows wherever
 the byte is not a valid ALLOW (Sec. 2.2 Eq. 1; App. F.1, the adversarial-suite table), and the
 oracle, fed the GPU's own input to layers 0, 23 and 47 (teacher forcing),
-matches the layer outputs on sampled tokens."""
+matches the layer: every token of layer 47, 1024 tokens spread over the 64
+requests at layers 0 and 23."""
 import numpy as np
 import pytest
 import torch
@@ -13,7 +14,7 @@ import oracle
 from paper_2608_06690_gb300 import inputs as inp
 from paper_2608_06690_gb300 import pmpe
 from paper_2608_06690_gb300.configs import CONFIGS
-from pmpe_testlib import GAP_EPS, MAX_ABS_REL, MEAN_REL, bf16_bits, oracle_layer, output_errors
+from pmpe_testlib import bf16_bits, check_against_oracle, check_audit, run_gpu_layer
 
 pytestmark = pytest.mark.gpu
 
@@ -100,20 +101,26 @@ def test_adversarial_policy_vectors_execute_no_private_rows(stack):
     assert families == {"all_malformed", "flipped_mid_request", "random_bytes"}
 
 
-def test_teacher_forced_oracle_on_sampled_layers(stack):
+def test_teacher_forced_oracle_on_checked_layers(stack):
+    """The stack runs once with the workload's policy; each checked layer is
+    then re-run alone on the input it saw inside the stack, which must give
+    the in-stack output bit for bit (the layer is deterministic and
+    batch-invariant), and that run is compared with the oracle: every token
+    of the last layer, 1024 tokens (16 per request) of layers 0 and 23."""
     cfg, layers, x0 = stack
     s = cfg.shape
     pol = cfg.policy(s.T)
     _, kept = run_stack(layers, x0, pol.cuda(), keep=CHECK_LAYERS)
-    tau = oracle.resolve(pol.numpy(), s.T)
-    g = np.random.default_rng(5)
-    toks = np.sort(np.concatenate([g.choice(np.nonzero(tau == v)[0], 8, replace=False) for v in (0, 1)]))
-    toks = toks.astype(np.int32)
+    per_req = s.T // cfg.n_requests
+    some = np.array([r * per_req + i for r in range(cfg.n_requests) for i in range(16)], np.int32)
     for l in CHECK_LAYERS:
         x_in, y = kept[l]
+        gpu = run_gpu_layer(s, layers[l].weights, x_in, pol.cuda())
+        assert np.array_equal(gpu["out"], bf16_bits(y)), f"layer {l}: re-run differs from the in-stack output"
+        check_audit(s, pol, gpu)
         w_cpu = {k: (None if v is None else v.cpu()) for k, v in layers[l].weights.items()}
-        r = oracle.forward(oracle_layer(s, w_cpu, x_in.cpu(), pol), tokens=toks)
-        ok = r["gap"] >= GAP_EPS
-        mx, mean = output_errors(bf16_bits(y)[toks][ok], r["out"][ok])
-        assert mx <= MAX_ABS_REL and mean <= MEAN_REL, (l, mx, mean)
-        assert (~ok).sum() <= 1
+        toks = None if l == CHECK_LAYERS[-1] else some
+        rep = check_against_oracle(s, w_cpu, x_in.cpu(), pol, gpu, tokens=toks,
+                                   name=f"qwen3_stack48 layer {l} (teacher-forced)")
+        assert rep["excused"] <= max(2, rep["tokens"] // 100), (l, rep)
+        del gpu

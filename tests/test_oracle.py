@@ -325,6 +325,86 @@ def test_forward_is_weighted_sum_of_routed_plus_shared_experts():
         np.testing.assert_allclose(r["out_f64"][t], acc.numpy(), rtol=0, atol=1e-9 * acc.abs().max().item())
 
 
+@pytest.mark.parametrize("unmasked", [False, True])
+def test_logits_are_the_masked_fp32_matmul_and_reproduce_the_route(unmasked):
+    """oracle.logits: numpy's float64 matmul of the BF16 values rounded to
+    fp32, -inf outside the pool tau selects (none in the unmasked control);
+    a brute-force sort of each row gives the oracle's top-k."""
+    s = LayerShape(T=150, H=128, I=16, E_pub=20, E_priv=8, E_sh=0, k=4, renormalize=True)
+    w, h, pol = make_layer(s, seed=21)
+    L = oracle_layer(s, w, h, pol, unmasked=unmasked)
+    got = oracle.logits(L)
+    R = torch.cat([w["router_pub"], w["router_priv"]]).double().numpy()
+    Z = (h.double().numpy() @ R.T).astype(np.float32).astype(np.float64)
+    allow = (pol.numpy() == 1)[:, None]
+    priv = (np.arange(s.E) >= s.E_pub)[None, :]
+    want = Z if unmasked else np.where(allow == priv, Z, -np.inf)
+    np.testing.assert_allclose(got, want, rtol=1e-6, atol=1e-7)
+    assert np.array_equal(np.isinf(got), np.isinf(want))
+    idx, _, _ = oracle.route(L)
+    for t in range(s.T):
+        assert list(idx[t]) == _expected_topk(list(got[t]), s.k)[0]
+    toks = np.array([149, 3, 77], np.int32)
+    assert np.array_equal(oracle.logits(L, tokens=toks), got[toks])
+
+
+@pytest.mark.parametrize("renorm", [True, False])
+def test_forward_forced_with_the_oracles_own_routing_is_the_forward(renorm):
+    """Given the routing forward takes, forward_forced returns forward's
+    output bits and weights (shared experts included)."""
+    s = LayerShape(T=40, H=64, I=32, E_pub=9, E_priv=5, E_sh=1, k=3, renormalize=renorm)
+    w, h, pol = make_layer(s, seed=22)
+    L = oracle_layer(s, w, h, pol)
+    r = oracle.forward(L)
+    out, wt = oracle.forward_forced(L, r["idx"])
+    assert np.array_equal(out, r["out"])
+    np.testing.assert_array_equal(wt, r["w"])
+    toks = np.array([5, 0, 39], np.int32)
+    out2, _ = oracle.forward_forced(L, r["idx"][toks], tokens=toks)
+    assert np.array_equal(out2, r["out"][toks])
+
+
+def test_forward_forced_other_selections():
+    """Any in-pool selection of identical experts gives that one MLP
+    (renormalised weights sum to 1); with distinct experts a selection that
+    swaps the k-th expert for the (k+1)-th changes the output by exactly the
+    swapped terms, from torch.nn.functional MLPs and the logits' softmax."""
+    s = LayerShape(T=16, H=64, I=32, E_pub=8, E_priv=4, E_sh=0, k=3, renormalize=True)
+    w, h, pol = make_layer(s, seed=23)
+    same = dict(w)
+    for name in ("gate", "up", "down"):
+        base = w[f"{name}_pub"][0]
+        same[f"{name}_pub"] = base.expand(s.E_pub, *base.shape).contiguous()
+        same[f"{name}_priv"] = base.expand(s.E_priv, *base.shape).contiguous()
+    g = np.random.default_rng(4)
+    tau = pol.numpy() == 1
+    idx = np.stack([g.choice(np.arange(s.E_pub, s.E) if tau[t] else np.arange(s.E_pub), s.k, replace=False)
+                    for t in range(s.T)]).astype(np.int32)
+    out, wt = oracle.forward_forced(oracle_layer(s, same, h, pol), idx)
+    np.testing.assert_allclose(wt.sum(1), 1.0, rtol=1e-12)
+    ref = _torch_mlp(h.double(), same["gate_pub"][0].double(), same["up_pub"][0].double(),
+                     same["down_pub"][0].double())
+    assert np.array_equal(out, ref.float().to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16))
+    # distinct experts: replace rank k-1 by the (k+1)-th best
+    L = oracle_layer(s, w, h, pol)
+    z = oracle.logits(L)
+    r = oracle.forward(L)
+    for t in range(s.T):
+        order = _expected_topk(list(z[t]), s.k + 1)[0]
+        sel = order[:s.k - 1] + [order[s.k]]
+        o1, w1 = oracle.forward_forced(L, np.array([sel], np.int32), tokens=np.array([t], np.int32))
+        ex = np.exp(z[t, sel] - z[t, order[0]])
+        np.testing.assert_allclose(w1[0], ex / ex.sum(), rtol=1e-12)
+        acc = torch.zeros(s.H, dtype=torch.float64)
+        for j, e in enumerate(sel):
+            pool, i = ("pub", e) if e < s.E_pub else ("priv", e - s.E_pub)
+            acc += w1[0, j] * _torch_mlp(h[t].double(), w[f"gate_{pool}"][i].double(),
+                                         w[f"up_{pool}"][i].double(), w[f"down_{pool}"][i].double())
+        got = bits_to_f64(o1[0])
+        np.testing.assert_allclose(got, acc.numpy(), rtol=0, atol=8e-3 * acc.abs().max().item())
+        assert not np.array_equal(o1[0], r["out"][t])
+
+
 # ------------------------------------------------------------------ audit
 
 @pytest.mark.parametrize("policy", ["iid", "allow", "deny", "none"])
