@@ -39,10 +39,7 @@ L2_FLUSH_BYTES = 512 << 20   # > 129 MB L2
 # grouped GEMM launches (the persistent gate/up + down pair, and each GEMM
 # launched alone), from ncu captures of the current kernels on the named
 # workload; None where no capture of the current kernels exists.
-NCU_TRAFFIC = {
-    "qwen3_prefill": {"experts": 1.700338e9 + 154.519296e6,
-                      "gateup": 1.145576e9 + 44.352512e6, "down": 0.553868e9 + 103.251456e6},
-}
+NCU_TRAFFIC = {}
 
 
 def _dist():
@@ -228,29 +225,37 @@ def build_workload(cfg, device, seed_offset=0):
 
 
 def algorithmic_work(s, counts: np.ndarray):
-    """FLOPs of the two grouped GEMMs and the byte counts of the HBM-bound
-    stages, for one forward with the given per-expert row counts."""
+    """FLOPs of the two grouped GEMMs and the least DRAM bytes of each stage,
+    for one forward with the given per-expert row counts.  "experts" is the
+    forward's persistent launch: gate/up (rows gathered from the hidden
+    states), down and the combine, whose activations and per-row outputs are
+    internal to it; "pair", "gateup", "down" and "combine" are the pieces run
+    on their own (diagnostics), which pass those intermediates through memory."""
     R = s.T * s.k
     f_gateup = 2.0 * R * s.H * 2 * s.I + 2.0 * s.T * s.H * 2 * s.E_sh * s.I
     f_down = 2.0 * R * s.I * s.H + 2.0 * s.T * s.E_sh * s.I * s.H
     touched = int((counts > 0).sum())
     expert_w = 3 * s.I * s.H * 2
     gemm_weight_bytes = touched * expert_w + s.E_sh * expert_w
-    b_gateup = touched * 2 * s.I * s.H * 2 + s.E_sh * 2 * s.I * s.H * 2 + R * s.H * 2 + R * s.I * 2 \
-        + (s.T * s.H * 2 + s.T * s.E_sh * s.I * 2 if s.E_sh else 0)
-    b_down = touched * s.I * s.H * 2 + s.E_sh * s.I * s.H * 2 + R * s.I * 2 + R * s.H * 2 \
-        + (s.T * s.E_sh * s.I * 2 + s.T * s.H * 2 if s.E_sh else 0)
+    w_gu = (touched + s.E_sh) * 2 * s.I * s.H * 2
+    w_dn = (touched + s.E_sh) * s.I * s.H * 2
+    act = R * s.I * 2 + s.T * s.E_sh * s.I * 2
+    yb = R * s.H * 2 + (s.T * s.H * 2 if s.E_sh else 0)
+    maps = R * 12                                   # tok_of_slot, w_of_slot, slot_of
+    b_gateup = w_gu + s.T * s.H * 2 + act + maps
+    b_down = w_dn + act + yb + maps
+    b_combine = yb + s.T * s.H * 2 + maps
+    b_experts = gemm_weight_bytes + s.T * s.H * 2 + s.T * s.H * 2 + maps
     b_route = s.T * s.H * 2 + (s.E_pub + s.E_priv) * s.H * 2 + s.T * s.k * 8 + s.T
-    # the dispatch's least traffic: each token row read once, each routed row
-    # written once, the slot maps
-    b_permute = s.T * s.H * 2 + R * s.H * 2 + R * 16
-    b_combine = R * s.H * 2 + s.T * s.H * 2 + (s.T * s.H * 2 if s.E_sh else 0)
+    # the dispatch order: route log and tickets in, slot maps out
+    b_permute = R * 12 + R * 12
     # the least DRAM traffic of a whole forward: the touched experts' weights
     # (and the shared experts'), both routers, hidden in and out, the route log
     b_layer_min = gemm_weight_bytes + (s.E_pub + s.E_priv) * s.H * 2 + 2 * s.T * s.H * 2 + s.T * s.k * 8 + s.T
     return dict(flops_gateup=f_gateup, flops_down=f_down, bytes_gateup=b_gateup, bytes_down=b_down,
                 bytes_layer_min=b_layer_min,
-                flops_experts=f_gateup + f_down, bytes_experts=b_gateup + b_down,
+                flops_experts=f_gateup + f_down, bytes_experts=b_experts,
+                flops_pair=f_gateup + f_down, bytes_pair=b_gateup + b_down,
                 bytes_route=b_route, bytes_permute=b_permute, bytes_combine=b_combine,
                 touched_experts=touched, gemm_weight_bytes=gemm_weight_bytes)
 
@@ -368,7 +373,7 @@ def roofline_of(work, stage_avg, pipeline, hbm, tf_burst, peak_src):
     below it; both fractions are given for the GEMMs."""
     dominant = max(pipeline, key=stage_avg.get)
     sec = stage_avg[dominant] / 1e3
-    if dominant in ("experts", "gateup", "down"):
+    if dominant in ("experts", "pair", "gateup", "down"):
         tflops = work[f"flops_{dominant}"] / sec / 1e12
         gbs = work[f"bytes_{dominant}"] / sec / 1e9
         intensity = work[f"flops_{dominant}"] / work[f"bytes_{dominant}"]
@@ -428,12 +433,13 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     # is still busy flushing while the host enqueues the stage (no host gap
     # inside the measured interval); stages run in pipeline order on the
     # workspace the previous stage filled.  "experts" is the persistent
-    # gate/up + down launch the forward runs; the two GEMMs launched one at a
-    # time are reported as diagnostics.
+    # gate/up + down + combine launch the forward runs; the gate/up + down
+    # pair, each GEMM and the combine launched on their own are diagnostics.
     stages = [("route", pmpe.STAGE_ROUTE), ("permute", pmpe.STAGE_PERMUTE),
-              ("experts", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE),
+              ("experts", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE),
+              ("pair", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE),
               ("gateup", pmpe.STAGE_GATEUP), ("down", pmpe.STAGE_DOWN)]
-    pipeline = ("route", "permute", "experts", "combine")
+    pipeline = ("route", "permute", "experts")
     stage_ms = {n: [] for n, _ in stages}
     for _ in range(args.steps):
         evs_s = []
@@ -512,7 +518,7 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     stage_report = {}
     for n, ms in stage_avg.items():
         d = {"ms": ms}
-        if n in ("experts", "gateup", "down"):
+        if n in ("experts", "pair", "gateup", "down"):
             d["tflops"] = work[f"flops_{n}"] / (ms / 1e3) / 1e12
         d["gbs"] = work[f"bytes_{n}"] / (ms / 1e3) / 1e9
         d["hbm_frac"] = d["gbs"] / hbm

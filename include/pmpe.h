@@ -71,10 +71,12 @@ extern "C" {
 
 /* Stage bits for pmpe_moe_forward_stages(). */
 #define PMPE_STAGE_ROUTE 0x01u   /* resolve + masked router + top-k + route log */
-#define PMPE_STAGE_PERMUTE 0x02u /* per-expert dispatch order + row gather */
-#define PMPE_STAGE_GATEUP 0x04u  /* grouped gate/up GEMM with fused silu(g)*u, execution audit */
+#define PMPE_STAGE_PERMUTE 0x02u /* per-expert dispatch order (slot maps) */
+#define PMPE_STAGE_GATEUP 0x04u  /* grouped gate/up GEMM on rows gathered from hidden, fused silu(g)*u,
+                                    execution audit */
 #define PMPE_STAGE_DOWN 0x08u    /* grouped down GEMM, scaled by the routing weight */
-#define PMPE_STAGE_COMBINE 0x10u /* weighted unpermute-combine (+ shared experts) */
+#define PMPE_STAGE_COMBINE 0x10u /* weighted unpermute-combine (+ shared experts); inside the same launch
+                                    as GATEUP | DOWN when those run in the same call */
 #define PMPE_STAGE_ALL 0x1Fu
 
 /* ------------------------------------------------------------ layer desc */
@@ -159,16 +161,22 @@ typedef struct pmpe_workspace_layout {
     size_t tok_of_slot;  /* int32  [T*k]    token of each dispatch row */
     size_t w_of_slot;    /* float  [T*k]    routing weight of each dispatch row */
     size_t router_rows;  /* BF16   [C*128, H]  token rows of each router CTA whose tile is not consecutive */
-    size_t a_perm;       /* BF16   [T*k, H] token rows in dispatch order */
+    size_t a_perm;       /* BF16   [T*k, H] token rows in dispatch order, written by the backward calls
+                          * (the forward's expert kernel gathers them from `hidden` as it goes) */
     size_t act;          /* BF16   [T*k, I] silu(g)*u of each dispatch row */
-    size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row */
+    size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row, by column block:
+                          * with bn = 256 if H % 256 == 0 else 128, columns [cb*bn, (cb+1)*bn) of
+                          * row r at y + (cb*T*k + r)*bn.  Dropped from L2 by the forward's combine
+                          * once summed: its contents after a full forward are undefined */
     size_t act_sh;       /* BF16   [T, E_shared*I] shared-expert activations (0 if none) */
-    size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs (0 if none) */
+    size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs, by column block like y (0 if none) */
     size_t tile_done;    /* uint32 [S]      router CTAs finished per 128-token tile */
     size_t router_lists; /* float2 [C2*128, k] per 32-expert chunk: each token's best k (score, id) */
     size_t router_meta;  /* float4 [C2*128] per chunk: max score, sum exp(score - max), entries */
-    size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1]  gate/up epilogue warps done per
-                          * (expert group, 128-row block), read by the down tiles of the same launch */
+    size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1 + H/128]  gate/up epilogue warps
+                          * done per (expert group, 128-row block), read by the down tiles of the same
+                          * launch; then down epilogue warps done per column block of y, read by the
+                          * combine of the same launch */
     size_t tile_counts;  /* uint32 [E, S4]  rows of expert e in router tile s (S4 = S rounded up to 4).
                           * With the tiles of a pool in ascending token order, slot
                           * offsets[e] + sum_{s' < s} tile_counts[e, s'] + position gives every expert

@@ -1,19 +1,25 @@
-// Stages 2 and 5 of the layer: the dispatch order of the routed rows with
-// the row gather, and the weighted unpermute-combine.
+// Stage 2 of the layer, the dispatch order of the routed rows, and the
+// stand-alone form of stage 5, the weighted unpermute-combine.
 //
 // Dispatch (the grouping any grouped expert execution needs): the routed rows
 // are grouped by expert id -- expert e owns slots [offset[e], offset[e+1]) --
 // and, inside an expert, ordered by token: the router's ticket names the
-// row's 128-token tile and its position among that tile's rows of the expert,
-// and the rows of the earlier tiles (tile_counts) come first.  The tiles of a
-// pool run in ascending token order, so every run gives the same order: the
-// stable (t, j) order.  The same pass copies each token row into its slot
-// with 16-byte vector loads.  An id outside [0, E) is recorded in the status
-// word.
+// row's 128-token tile and its position among that tile's rows of its
+// expert, and the rows of the earlier tiles (tile_counts) come first.  The
+// tiles of a pool run in ascending token order, so every run gives the same
+// order: the stable (t, j) order.  Only the slot maps are written (slot_of,
+// tok_of_slot, w_of_slot): the expert kernel gathers each slot's token row
+// from the hidden states itself.  An id outside [0, E) is recorded in the
+// status word.
 //
 // Combine: out_t = bf16( sum_{j < k} y[slot(t, j)] + y_shared[t] ), summed in
 // FP32 in a fixed order (j ascending, then shared), so the result of a token
-// never depends on the other tokens of the batch.
+// never depends on the other tokens of the batch.  The forward runs it inside
+// the expert kernel (per column block of y, as soon as that block is
+// complete); combine_kernel here is the same sum as a kernel of its own, for
+// the stage-by-stage entry point.  y is stored by column block: block cb of
+// slot r is the bn = column_block(H) values [cb * bn, (cb + 1) * bn) at
+// y + (cb * R + r) * bn (y_shared likewise, with T rows).
 #include <algorithm>
 
 #include "pmpe_internal.cuh"
@@ -30,30 +36,27 @@ struct DispatchParams {
     const uint32_t *counts;
     const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
     int slots4;
-    const bf16 *hidden;
-    int T, H, R, k, E;
-    int groups;  // warps per token: each stores the row to a share of its k slots
+    int T, R, k, E;
     uint32_t *offsets;
     int32_t *slot_of, *tok_of_slot;
     float *w_of_slot;
-    bf16 *a_perm;
     uint32_t *status;
 };
 
-// Slot of routed row (t, j): offset[e] + the rows of expert e in the router
-// tiles before the row's tile + its position in that tile (ticket = 128 *
-// tile + position).  Summing the earlier tiles' counts per row measured
+// Slot of routed row r = (t, j): offset[e] + the rows of expert e in the
+// router tiles before the row's tile + its position in that tile (ticket =
+// 128 * tile + position).  Summing the earlier tiles' counts per row measured
 // faster than building their prefix once, in the router's last CTA or in
-// every dispatch CTA's shared memory.  Records the row in slot_of, tok_of_slot
-// and w_of_slot and returns the slot (-1 for an id outside [0, E) or a slot
+// every dispatch CTA's shared memory.  Records the row in slot_of,
+// tok_of_slot and w_of_slot (nothing for an id outside [0, E) or a slot
 // outside [0, R)).
-__device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint32_t *s_off, int t, int j)
+__device__ __forceinline__ void resolve_slot(const DispatchParams &p, const uint32_t *s_off, int r)
 {
-    const int r = t * p.k + j;
+    const int t = r / p.k;
     const int e = p.idx[r];
     if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
         if (p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
-        return -1;
+        return;
     }
     const int tk = p.ticket[r];
     const int ts = min(tk >> 7, p.slots4 - 1);
@@ -61,19 +64,18 @@ __device__ __forceinline__ int resolve_slot(const DispatchParams &p, const uint3
     uint32_t before = 0;
     for (int s2 = 0; s2 < ts; ++s2) before += __ldg(tc + s2);
     const int slot = (int)(s_off[e] + before) + (tk & 127);
-    if ((unsigned)slot >= (unsigned)p.R) return -1;  // only a corrupt ticket could fail this
+    if ((unsigned)slot >= (unsigned)p.R) return;  // only a corrupt ticket could fail this
     p.slot_of[r] = slot;
     p.tok_of_slot[slot] = t;
     p.w_of_slot[slot] = p.w[r];
-    return slot;
 }
 
-// Dispatch and gather in one pass.  Every CTA forms the experts' offsets
-// (exclusive prefix sum of the router's per-expert counts) in shared memory;
-// routed row r = (t, j) of expert e, in tile s at position q of the tile's
-// rows of e, goes to slot offset[e] + sum_{s' < s} tile_counts[e][s'] + q.
-// One warp per token loads the token's row once and stores it to its k slots.
-__global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const DispatchParams p)
+// The dispatch order.  Every CTA forms the experts' offsets (exclusive
+// prefix sum of the router's per-expert counts) in shared memory; routed row
+// r = (t, j) of expert e, in tile s at position q of the tile's rows of e,
+// goes to slot offset[e] + sum_{s' < s} tile_counts[e][s'] + q.  One thread
+// per routed row.
+__global__ void __launch_bounds__(kDispThreads) dispatch_kernel(const DispatchParams p)
 {
     __shared__ uint32_t s_off[2 * kMaxPool + 1];
     pdl_trigger();
@@ -96,36 +98,38 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_gather_kernel(const Dis
     __syncthreads();
     if (blockIdx.x == 0)
         for (int e = threadIdx.x; e <= p.E; e += kDispThreads) p.offsets[e] = s_off[e];
+    for (int r = blockIdx.x * kDispThreads + threadIdx.x; r < p.R; r += gridDim.x * kDispThreads)
+        resolve_slot(p, s_off, r);
+}
 
-    // one warp per (token, group of its routed rows): the token's row is
-    // loaded once (16-byte vectors, all in flight together) and stored to the
-    // group's slots; lane j resolves row (t, j)
+// The token rows of the dispatch slots [offsets[g0], offsets[g1]) copied into
+// rows[slot] (the dispatched-row matrix the backward's GEMMs read): one warp
+// per slot, eight 16-byte loads in flight per lane.
+__global__ void __launch_bounds__(256) gather_dispatch_rows_kernel(const bf16 *hidden, const int32_t *tok_of_slot,
+                                                                    const uint32_t *offsets, int g0, int g1, int R,
+                                                                    int T, int H, bf16 *rows)
+{
+    const uint32_t p0 = min(offsets[g0], (uint32_t)R), p1 = min(max(offsets[g1], p0), (uint32_t)R);
+    const int nv = H / 8;
     const int lane = threadIdx.x & 31;
-    const int nv = p.H / 8;
-    const int warps = gridDim.x * (kDispThreads / 32);
-    const int per = (p.k + p.groups - 1) / p.groups;
-    for (int wi = blockIdx.x * (kDispThreads / 32) + (threadIdx.x >> 5); wi < p.T * p.groups; wi += warps) {
-        const int t = wi / p.groups, gj = wi - t * p.groups;
-        const int j0 = gj * per, j1 = min(p.k, j0 + per);
-        const uint4 *src = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
-        int my_slot = -1;
-        if (lane >= j0 && lane < j1) my_slot = resolve_slot(p, s_off, t, lane);
-        for (int c0 = 0; c0 < nv; c0 += 32 * 8) {
-            uint4 v[8];
+    const int warps = gridDim.x * (blockDim.x >> 5);
+    constexpr int kU = 8;
+    for (uint32_t r = p0 + blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < p1; r += warps) {
+        const int t = tok_of_slot[r];
+        if ((unsigned)t >= (unsigned)T) continue;  // only a corrupt dispatch could fail this
+        const uint4 *src = reinterpret_cast<const uint4 *>(hidden + (size_t)t * H);
+        uint4 *dst = reinterpret_cast<uint4 *>(rows + (size_t)r * H);
+        for (int c0 = 0; c0 < nv; c0 += 32 * kU) {
+            uint4 v[kU];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
+            for (int u = 0; u < kU; ++u) {
                 const int c = c0 + u * 32 + lane;
                 if (c < nv) v[u] = __ldg(src + c);
             }
-            for (int j = j0; j < j1; ++j) {
-                const int slot = __shfl_sync(~0u, my_slot, j);
-                if (slot < 0) continue;
-                uint4 *dst = reinterpret_cast<uint4 *>(p.a_perm + (size_t)slot * p.H);
 #pragma unroll
-                for (int u = 0; u < 8; ++u) {
-                    const int c = c0 + u * 32 + lane;
-                    if (c < nv) dst[c] = v[u];
-                }
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + u * 32 + lane;
+                if (c < nv) dst[c] = v[u];
             }
         }
     }
@@ -146,9 +150,10 @@ __device__ __forceinline__ void add_bf16x8(float *acc, const uint4 &v)
 // routed rows are loaded in batches of 8 independent 16-byte loads before
 // they are summed (in j order), so the loads overlap instead of forming a
 // chain of dependent memory round trips.  Four resident CTAs per SM (at most
-// 64 registers a thread) keep more of those loads in flight.
+// 64 registers a thread) keep more of those loads in flight.  y and y_sh are
+// stored by column blocks of bn values (see the top of this file).
 __global__ void __launch_bounds__(256, 4) combine_kernel(const bf16 *__restrict__ y, const bf16 *__restrict__ y_sh,
-                                                      const int32_t *__restrict__ slot_of, int T, int H, int k,
+                                                      const int32_t *__restrict__ slot_of, int T, int H, int k, int bn,
                                                       bf16 *__restrict__ out)
 {
     pdl_trigger();
@@ -159,6 +164,7 @@ __global__ void __launch_bounds__(256, 4) combine_kernel(const bf16 *__restrict_
     for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
         const int t = (int)(i / nv), c = (int)(i - (long long)t * nv);
+        const int cb = (c * 8) / bn, cc = c * 8 - cb * bn;
         const int32_t *slots = slot_of + (size_t)t * k;
         float acc[8];
 #pragma unroll
@@ -170,14 +176,14 @@ __global__ void __launch_bounds__(256, 4) combine_kernel(const bf16 *__restrict_
                 if (j0 + u < k) {
                     int slot = __ldg(slots + j0 + u);
                     if ((unsigned)slot >= (unsigned)R) slot = 0;  // only after a dispatch mismatch (status set)
-                    v[u] = __ldg(reinterpret_cast<const uint4 *>(y + (size_t)slot * H) + c);
+                    v[u] = __ldg(reinterpret_cast<const uint4 *>(y + ((size_t)cb * R + slot) * bn + cc));
                 }
             }
 #pragma unroll
             for (int u = 0; u < 8; ++u)
                 if (j0 + u < k) add_bf16x8(acc, v[u]);
         }
-        if (y_sh) add_bf16x8(acc, __ldg(reinterpret_cast<const uint4 *>(y_sh + (size_t)t * H) + c));
+        if (y_sh) add_bf16x8(acc, __ldg(reinterpret_cast<const uint4 *>(y_sh + ((size_t)cb * T + t) * bn + cc)));
         uint4 o;
         o.x = pack_bf16x2(acc[0], acc[1]);
         o.y = pack_bf16x2(acc[2], acc[3]);
@@ -198,24 +204,29 @@ int grid_for(long long work, int num_sms)
 
 }  // namespace
 
+int column_block(int H) { return H % 256 == 0 ? 256 : 128; }
+
 cudaError_t launch_permute(const Ctx &c)
 {
     const Shape &s = c.s;
     const int R = s.T * s.k;
     DispatchParams p;
-    p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts; p.hidden = c.hidden;
+    p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts;
     p.tile_counts = c.tile_counts;
     p.slots4 = router_slots4(c.s.T);
-    p.T = s.T; p.H = s.H; p.R = R; p.k = s.k; p.E = s.E();
+    p.T = s.T; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
-    p.a_perm = c.a_perm;
     p.status = c.audit.status;
-    // enough warps for about one full wave (32 per SM); a token's row is
-    // loaded once per group
-    const long long want = 32LL * c.num_sms;
-    p.groups = (int)std::min<long long>(s.k, std::max<long long>(1, (want + s.T - 1) / s.T));
-    return launch_pdl(dispatch_gather_kernel, dim3(grid_for((long long)s.T * p.groups * 32, c.num_sms)),
-                      dim3(kDispThreads), 0, c.stream, p);
+    const int grid = std::max(1, std::min((R + kDispThreads - 1) / kDispThreads, 4 * c.num_sms));
+    return launch_pdl(dispatch_kernel, dim3(grid), dim3(kDispThreads), 0, c.stream, p);
+}
+
+cudaError_t launch_gather_dispatch_rows(const Ctx &c, int g0, int g1)
+{
+    const Shape &s = c.s;
+    gather_dispatch_rows_kernel<<<c.num_sms * 8, 256, 0, c.stream>>>(c.hidden, c.tok_of_slot, c.offsets, g0, g1,
+                                                                     s.T * s.k, s.T, s.H, c.a_perm);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_combine(const Ctx &c)
@@ -223,7 +234,7 @@ cudaError_t launch_combine(const Ctx &c)
     const Shape &s = c.s;
     return launch_pdl(combine_kernel, dim3(grid_for((long long)s.T * (s.H / 8), c.num_sms)), dim3(256), 0, c.stream,
                       (const bf16 *)c.y, (const bf16 *)(s.E_sh > 0 ? c.y_sh : nullptr), (const int32_t *)c.slot_of, s.T,
-                      s.H, s.k, c.out);
+                      s.H, s.k, column_block(s.H), c.out);
 }
 
 }  // namespace pmpe

@@ -1,9 +1,11 @@
-// Stages 3 and 4 of the layer on the 5th-generation tensor cores: grouped
+// Stages 3 to 5 of the layer on the 5th-generation tensor cores: grouped
 // BF16 expert GEMMs with tcgen05.mma accumulating in tensor memory (TMEM),
-// operands staged by TMA into 128-byte-swizzled shared memory.
+// operands staged into 128-byte-swizzled shared memory, and the weighted
+// combine of their outputs.
 //
 //   gate/up:  act = bf16(silu(A_e W_gate,e^T) * (A_e W_up,e^T))    (SwiGLU fused)
 //   down:     y   = bf16(w_row * (act_e W_down,e^T))
+//   combine:  out_t = bf16(sum_j y[slot(t, j)] + y_shared[t])       (j ascending)
 //
 // Groups are the routed experts (rows of the dispatch order) plus, with
 // shared experts, one dense group over all T tokens (gate/up weights of the
@@ -12,11 +14,26 @@
 // built on the device from the dispatch offsets: no host sync, and empty
 // experts contribute no tile.
 //
-// CTA roles (192 threads):
+// The routed gate/up tiles read their A rows straight from the hidden states:
+// the row of dispatch slot r is hidden[tok_of_slot[r]], gathered into shared
+// memory by four warps with 16-byte cp.async copies (the hidden states, read
+// by every expert a token routes to, stay in L2), so the dispatched rows are
+// never written out.  The down tiles run column block by column block (bn
+// output columns of every expert, then the next bn), writing y block by block;
+// once every down tile of a column block is stored, the same four warps sum
+// that block of y into the output, reading it back from L2.
+//
+// Tile list: every gate/up tile (group by group, n-tile major), then the down
+// tiles of column block 0, then, for cb = 1 .. nb-1, the down tiles of block cb
+// followed by the combine items of block cb - 1, and last the combine items of
+// block nb - 1.  CTA c takes tiles c, c + grid, c + 2 grid, ... in order.
+//
+// CTA roles (320 threads):
 //   warp 0       three lanes issue the TMA loads of a 4-stage ring, one
-//                operand box each (A: 128 rows x 64 K; B: 256 rows x 64 K,
-//                i.e. 128 gate + 128 up rows, or 256 / 128 output columns of
-//                the down projection in two halves)
+//                operand box each (A: 128 rows x 64 K of the activations or,
+//                for the shared group, of the hidden states; B: 256 rows x
+//                64 K, i.e. 128 gate + 128 up rows, or 256 / 128 output
+//                columns of the down projection in two halves)
 //   warp 1       allocates 512 TMEM columns (two 128 x 256 FP32
 //                accumulators, so the epilogue of one tile overlaps the MMAs
 //                of the next) and one thread issues tcgen05.mma M=128 N=256
@@ -25,7 +42,9 @@
 //                rows), SwiGLU or weight scaling, BF16 stores; in gate/up mode
 //                the tiles of N-tile 0 also write the execution audit, each
 //                row checked against the route log of its token
-// Every mbarrier wait is bounded in time: on expiry the CTA records
+//   warps 6..9   the A-row gather of the routed gate/up tiles (cp.async into
+//                the ring), then the combine items
+// Every wait is bounded in time: on expiry the CTA records
 // PMPE_STATUS_PIPELINE_TIMEOUT, stops issuing work, waits (bounded) for its
 // own copies and MMAs in flight, frees its TMEM and exits.
 #include <cuda.h>
@@ -48,8 +67,12 @@ constexpr int kBBytes = 256 * BK * 2;         // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kAccCols = 256;                 // FP32 TMEM columns per accumulator
 constexpr int kTmemCols = 2 * kAccCols;
-constexpr int kThreads = 192;
+constexpr int kGatherWarps = 4;               // warps 6..9
+constexpr int kThreads = 192 + 32 * kGatherWarps;
 constexpr int kLoaders = 3;                   // TMA-issuing lanes of warp 0
+constexpr int kFullArrivals = kLoaders + kGatherWarps;  // per ring stage
+constexpr int kGatherDepth = kStages - 1;     // stages a gather warp keeps in flight
+constexpr int kCombTokens = 32;               // tokens per combine item (8 per gather warp)
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
 constexpr int kOutBufBytes = kOutBox * kOutBox * 2;
@@ -57,27 +80,35 @@ constexpr int kOutBytes = 4 * 2 * kOutBufBytes;  // 4 epilogue warps x 2 buffers
 constexpr int kDynSmem = kStages * kStageBytes + kOutBytes + 1024 /* alignment slack */;
 
 enum { kGateUp = 0, kDown = 1 };
+enum { kTileGU = 0, kTileDown = 1, kTileComb = 2 };
 
 // One GEMM of the layer: gate/up (SwiGLU fused) or down (routing weight fused).
 struct TcPhase {
-    int mode;
     int bn;           // output columns per tile (gate/up: 128 activation columns; down: 256 or 128)
     uint32_t idesc;   // tcgen05 instruction descriptor (BF16 x BF16 -> FP32, M = 128, N = MMA width)
     bf16 *C_routed, *C_shared;
 };
 
 struct TcParams {
-    int nph;          // 1: the GEMM of ph[0]; 2: gate/up (ph[0]) then down (ph[1]) in one persistent grid
-    TcPhase ph[2];
-    int E, E_pub, E_sh, T, H, I, R;
+    // which parts this launch runs: the gate/up tiles, the down tiles, the
+    // combine items (only together with the down tiles)
+    int has_gu, has_down, has_comb;
+    TcPhase ph[2];    // [kGateUp], [kDown]
+    int E, E_pub, E_sh, T, H, I, R, k;
+    int nb;           // column blocks of the down output: H / ph[kDown].bn
     const uint32_t *offsets;
     const float *w_of_slot;
     const int32_t *tok_of_slot;
+    const int32_t *slot_of;
     const int32_t *topk_idx;  // [T, k] the route log, read back by the execution audit
-    int k;
-    // nph == 2: per (group, 128-row block), the gate/up epilogue warps whose
-    // activations are stored (zeroed before the launch)
+    const bf16 *hidden;       // the gather source of the routed gate/up tiles
+    // has_gu && has_down: per (group, 128-row block), the gate/up epilogue
+    // warps whose activations are stored (zeroed before the launch)
     uint32_t *ready;
+    // has_comb: per column block, the down epilogue warps whose y is stored
+    // (zeroed before the launch)
+    uint32_t *done_cb;
+    bf16 *out;                // has_comb: the layer output [T, H]
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
     // optional FP32: the gate and up accumulators saved for the backward,
     // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
@@ -97,13 +128,13 @@ struct TcMaps {  // [phase]
 // ------------------------------------------------------------- tile list
 
 struct Tile {
-    int ph, mode, bn, g, m_tile, m0, n0, rows, row_base, nkb;
+    int kind, ph, bn, g, m_tile, m0, n0, rows, row_base, nkb, cb, t0;
     bool shared;
 };
 
 struct TileTable {
-    int prefix[2][kMaxGroups + 1];  // tiles of the groups before g, per phase
-    int mpre[kMaxGroups + 1];       // 128-row blocks of the groups before g
+    int prefix[kMaxGroups + 1];  // gate/up tiles of the groups before g
+    int mpre[kMaxGroups + 1];    // 128-row blocks of the groups before g
     int rows[kMaxGroups];
     int base[kMaxGroups];
 };
@@ -117,34 +148,118 @@ __device__ __forceinline__ int group_k(const TcParams &p, int mode, bool shared)
     return mode == kGateUp ? p.H : (shared ? p.E_sh * p.I : p.I);
 }
 
-// Tile `tile` of the list: the tiles of phase 0 (all groups), then those of
-// phase 1; inside a phase, group by group, n-tile major.
-__device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &tt, int G, int tile)
+// The last group g with arr[g] <= x (arr ascending from arr[0] = 0).
+__device__ __forceinline__ int find_group(const int *arr, int G, int x)
 {
-    Tile t;
-    t.ph = (p.nph == 2 && tile >= tt.prefix[0][G]) ? 1 : 0;
-    const int local_all = tile - (t.ph ? tt.prefix[0][G] : 0);
-    const int *pre = tt.prefix[t.ph];
-    int lo = 0, hi = G - 1;  // last group with prefix <= local_all
+    int lo = 0, hi = G - 1;
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
-        if (pre[mid] <= local_all) lo = mid; else hi = mid - 1;
+        if (arr[mid] <= x) lo = mid; else hi = mid - 1;
     }
-    t.mode = p.ph[t.ph].mode;
-    t.bn = p.ph[t.ph].bn;
-    t.g = lo;
-    t.shared = lo >= p.E;
-    const int rows = tt.rows[lo];
-    const int mt = (rows + BM - 1) / BM;
-    const int local = local_all - pre[lo];
-    const int n_tile = local / mt;
-    t.m_tile = local - n_tile * mt;
-    t.m0 = t.m_tile * BM;
-    t.n0 = n_tile * t.bn;
-    t.rows = min(BM, rows - t.m0);
-    t.row_base = tt.base[lo];
-    t.nkb = group_k(p, t.mode, t.shared) / BK;
+    return lo;
+}
+
+__device__ __forceinline__ int comb_items(const TcParams &p) { return (p.T + kCombTokens - 1) / kCombTokens; }
+
+__device__ __forceinline__ int total_tiles(const TcParams &p, const TileTable &tt, int G)
+{
+    return (p.has_gu ? tt.prefix[G] : 0) + (p.has_down ? p.nb * tt.mpre[G] : 0) +
+           (p.has_comb ? p.nb * comb_items(p) : 0);
+}
+
+__device__ __forceinline__ void fill_rows(const TcParams &p, const TileTable &tt, Tile &t, int g, int m_tile)
+{
+    t.g = g;
+    t.shared = g >= p.E;
+    t.m_tile = m_tile;
+    t.m0 = m_tile * BM;
+    t.rows = min(BM, tt.rows[g] - t.m0);
+    t.row_base = tt.base[g];
+}
+
+__device__ __forceinline__ Tile down_tile(const TcParams &p, const TileTable &tt, int G, int cb, int j)
+{
+    Tile t;
+    t.kind = kTileDown;
+    t.ph = kDown;
+    t.bn = p.ph[kDown].bn;
+    const int g = find_group(tt.mpre, G, j);
+    fill_rows(p, tt, t, g, j - tt.mpre[g]);
+    t.cb = cb;
+    t.n0 = cb * t.bn;
+    t.nkb = group_k(p, kDown, t.shared) / BK;
+    t.t0 = 0;
     return t;
+}
+
+__device__ __forceinline__ Tile comb_tile(int cb, int item)
+{
+    Tile t;
+    t.kind = kTileComb;
+    t.ph = kDown;
+    t.cb = cb;
+    t.t0 = item * kCombTokens;
+    t.nkb = 0;
+    t.bn = t.g = t.m_tile = t.m0 = t.n0 = t.rows = t.row_base = 0;
+    t.shared = false;
+    return t;
+}
+
+// Tile `tile` of the list described at the top of this file.
+__device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &tt, int G, int tile)
+{
+    const int n_gu = p.has_gu ? tt.prefix[G] : 0;
+    if (tile < n_gu) {
+        Tile t;
+        t.kind = kTileGU;
+        t.ph = kGateUp;
+        t.bn = p.ph[kGateUp].bn;
+        const int g = find_group(tt.prefix, G, tile);
+        const int mt = (tt.rows[g] + BM - 1) / BM;
+        const int local = tile - tt.prefix[g];
+        const int n_tile = local / mt;
+        fill_rows(p, tt, t, g, local - n_tile * mt);
+        t.n0 = n_tile * t.bn;
+        t.nkb = group_k(p, kGateUp, t.shared) / BK;
+        t.cb = 0;
+        t.t0 = 0;
+        return t;
+    }
+    const int u = tile - n_gu;
+    const int dn = tt.mpre[G];  // down tiles per column block
+    if (!p.has_comb) return down_tile(p, tt, G, u / dn, u - (u / dn) * dn);
+    if (u < dn) return down_tile(p, tt, G, 0, u);
+    const int u2 = u - dn, round = dn + comb_items(p);
+    if (u2 < (p.nb - 1) * round) {
+        const int r = u2 / round, rem = u2 - r * round;
+        return rem < dn ? down_tile(p, tt, G, r + 1, rem) : comb_tile(r, rem - dn);
+    }
+    return comb_tile(p.nb - 1, u2 - (p.nb - 1) * round);
+}
+
+// 16-byte async copy global -> shared with an explicit source size (0: the
+// 16 bytes are zero-filled and nothing is read).
+__device__ __forceinline__ void cp_async16_zfill(uint32_t dst, const void *src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+
+// Drop a 128-byte line from L2 without writing it back (its data is not read
+// again before it is rewritten).
+__device__ __forceinline__ void discard_l2_line(const void *p)
+{
+    asm volatile("discard.global.L2 [%0], 128;\n" ::"l"(p) : "memory");
+}
+
+__device__ __forceinline__ void add_bf16x8(float *acc, const uint4 &v)
+{
+    const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(b[i]);
+        acc[2 * i] += f.x;
+        acc[2 * i + 1] += f.y;
+    }
 }
 
 // ---------------------------------------------------------------- kernel
@@ -170,7 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     pdl_trigger();
 
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), kLoaders); mbar_init(empty_bar(s), 1); }
+        for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), kFullArrivals); mbar_init(empty_bar(s), 1); }
         for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
         mbar_init(done_bar, 1);
         s_abort = 0;
@@ -181,7 +296,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                      "r"(kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
     }
-    pdl_wait();  // the dispatch offsets and the A operand come from the previous kernels
+    pdl_wait();  // the dispatch offsets and slot maps come from the previous kernel
     // tile list: rows and tiles per group, prefixes over groups
     for (int g = tid; g < G; g += kThreads) {
         const bool shared = g >= p.E;
@@ -198,12 +313,11 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         tt.rows[g] = rows;
         tt.base[g] = base;
         tt.mpre[g + 1] = mt;
-        for (int ph = 0; ph < 2; ++ph)
-            tt.prefix[ph][g + 1] = ph < p.nph ? mt * (group_n(p, p.ph[ph].mode, shared) / p.ph[ph].bn) : 0;
+        tt.prefix[g + 1] = mt * (group_n(p, kGateUp, shared) / p.ph[kGateUp].bn);
     }
     __syncthreads();
-    if (warp < 3) {  // three inclusive scans, one per warp: tiles of phase 0, of phase 1, row blocks
-        int *arr = warp == 2 ? tt.mpre : tt.prefix[warp];
+    if (warp < 2) {  // two inclusive scans, one per warp: gate/up tiles, row blocks
+        int *arr = warp == 1 ? tt.mpre : tt.prefix;
         int carry = 0;
         for (int b = 0; b < G; b += 32) {
             int v = b + lane < G ? arr[b + lane + 1] : 0;
@@ -223,14 +337,18 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
-    const int total = tt.prefix[0][G] + (p.nph == 2 ? tt.prefix[1][G] : 0);
+    const int total = total_tiles(p, tt, G);
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
         // Three lanes, one operand box each: a single thread's TMA boxes are
         // processed one after another, so spreading a stage's boxes over
         // three issuing threads triples the ring's fill rate.
-        //   lane 0: A tile (128 rows x 64 K)
+        //   lane 0: the A tile (128 rows x 64 K) when A comes through TMA (the
+        //           activations, or the hidden states of the shared group), and
+        //           then also the arrivals of the gather warps, which have
+        //           nothing to copy; in a routed gate/up tile the gather warps
+        //           fill A and lane 0 only arrives
         //   lane 1: gate rows (gate/up) or B rows [0, bn/2) (down)
         //   lane 2: up rows (gate/up)   or B rows [bn/2, bn) (down)
         int stage = 0;
@@ -238,18 +356,21 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         uint32_t filled = 0, last_parity = 0;  // per-stage bits, for the drain below
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
+            if (t.kind == kTileComb) continue;
+            const bool gather = t.kind == kTileGU && !t.shared;
             const int q = t.shared ? 2 : (t.g < p.E_pub ? 0 : 1);
             const int ei = t.shared ? 0 : (q == 0 ? t.g : t.g - p.E_pub);
             const CUtensorMap *amap = t.shared ? &maps.a_shared[t.ph] : &maps.a_routed[t.ph];
             const int arow = t.row_base + t.m0;
-            const uint32_t my_tx = lane == 0 ? (uint32_t)kABytes
-                                             : (t.mode == kGateUp ? (uint32_t)(BM * 128) : (uint32_t)(t.bn / 2 * 128));
+            const uint32_t my_tx = lane == 0 ? (gather ? 0u : (uint32_t)kABytes)
+                                             : (t.ph == kGateUp ? (uint32_t)(BM * 128) : (uint32_t)(t.bn / 2 * 128));
             bool ok = true;
-            if (t.ph == 1 && lane == 0) {
-                // a down tile of the persistent pair: its activation rows are
-                // complete once every gate/up epilogue warp of their row block
-                // has stored its part (bounded wait; the weights are loaded meanwhile)
-                const uint32_t need = 4u * (uint32_t)(group_n(p, kGateUp, t.shared) / p.ph[0].bn);
+            if (t.kind == kTileDown && p.has_gu && lane == 0) {
+                // a down tile after the gate/up tiles of the same launch: its
+                // activation rows are complete once every gate/up epilogue
+                // warp of their row block has stored its part (bounded wait;
+                // the weights are loaded meanwhile)
+                const uint32_t need = 4u * (uint32_t)(group_n(p, kGateUp, t.shared) / p.ph[kGateUp].bn);
                 const uint32_t *rp = p.ready + tt.mpre[t.g] + t.m_tile;
                 const unsigned long long t0 = globaltimer_ns();
                 while (ld_acquire_gpu(rp) < need) {
@@ -271,8 +392,11 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 mbar_expect_tx(full_bar(stage), my_tx);
                 const int kx = kb * BK;
                 if (lane == 0) {
-                    tma_load_2d(sA, amap, full_bar(stage), kx, arow);
-                } else if (t.mode == kGateUp) {
+                    if (!gather) {
+                        tma_load_2d(sA, amap, full_bar(stage), kx, arow);
+                        mbar_arrive_count(full_bar(stage), kGatherWarps);
+                    }
+                } else if (t.ph == kGateUp) {
                     const int brow = ei * p.I + t.n0;  // shared: n0 spans E_sh * I rows
                     tma_load_2d(sB + (lane - 1) * BM * 128, lane == 1 ? &maps.b0[t.ph][q] : &maps.b1[t.ph][q],
                                 full_bar(stage), kx, brow);
@@ -303,11 +427,13 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         // ------------------------------------------------ MMA issuer
         int stage = 0, it = 0;
         uint32_t phase = 0;
-        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x, ++it) {
+        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
+            if (t.kind == kTileComb) continue;
             const uint32_t idesc = p.ph[t.ph].idesc;
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            ++it;
             if (!mbar_wait(tempty_bar(buf), use ^ 1u, &s_abort, p.status)) break;
             tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kAccCols);
@@ -333,16 +459,18 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             while (!mbar_try_wait(done_bar, 0))
                 if (globaltimer_ns() - t0 > kWaitLimitNs) break;
         }
-    } else if (warp >= 2) {
+    } else if (warp >= 2 && warp < 6) {
         // ------------------------------------------------ epilogue
         const int quarter = warp & 3;  // TMEM lanes this warp may access
         const uint32_t out_base = sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * 2 * kOutBufBytes);
         int out_parity = 0;
         int it = 0;
-        for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+        for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
+            if (t.kind == kTileComb) continue;
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
+            ++it;
             // one lane waits, the warp follows: tcgen05.ld below is warp-collective
             int ok = 1;
             if (lane == 0) ok = mbar_wait(tfull_bar(buf), use, &s_abort, p.status) ? 1 : 0;
@@ -351,23 +479,28 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             __syncwarp();
             tc_fence_after();
             const TcPhase &ph = p.ph[t.ph];
+            const bool gu = t.kind == kTileGU;
             const int r = quarter * 32 + lane;  // tile row of this thread
             const bool valid = r < t.rows;
             const int grow = t.row_base + t.m0 + r;
             const uint32_t taddr = tmem_base + (uint32_t)(buf * kAccCols) + ((uint32_t)(quarter * 32) << 16);
             // Whole 32-row blocks go out through shared memory and TMA stores;
             // the block holding a tile's last rows is written row by row so that
-            // it never touches the next expert's rows.
+            // it never touches the next expert's rows.  Down outputs are stored
+            // by column block: row r of block cb at (cb * rows_total + r) * bn.
             const bool full_block = (t.rows - quarter * 32) >= 32;
-            const int ldc = t.mode == kGateUp ? (t.shared ? p.E_sh * p.I : p.I) : p.H;
-            bf16 *crow = (t.shared ? ph.C_shared : ph.C_routed) + (size_t)grow * ldc + t.n0;
+            const int rows_total = t.shared ? p.T : p.R;
+            const int out_row0 = gu ? t.row_base + t.m0 : t.cb * rows_total + t.row_base + t.m0;
+            const int ldc = gu ? (t.shared ? p.E_sh * p.I : p.I) : t.bn;
+            const int col0 = gu ? t.n0 : 0;
+            bf16 *crow = (t.shared ? ph.C_shared : ph.C_routed) + (size_t)(out_row0 + r) * ldc + col0;
             const CUtensorMap *cmap = t.shared ? &maps.c_shared[t.ph] : &maps.c_routed[t.ph];
-            const int nchunks = t.mode == kGateUp ? BM / 32 : t.bn / 32;
-            const float sc = (t.mode == kGateUp || t.shared) ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
+            const int nchunks = gu ? BM / 32 : t.bn / 32;
+            const float sc = (gu || t.shared) ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
 #pragma unroll 1
             for (int c = 0; c < nchunks; ++c) {
                 uint32_t pk[16];
-                if (t.mode == kGateUp) {
+                if (gu) {
                     float gv[32], uv[32];
                     tmem_ld32(taddr + c * 32, gv);
                     tmem_ld32(taddr + 128 + c * 32, uv);
@@ -438,7 +571,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tma_store_2d(cmap, sbuf, t.n0 + c * 32, t.row_base + t.m0 + quarter * 32);
+                        tma_store_2d(cmap, sbuf, col0 + c * 32, out_row0 + quarter * 32);
                         bulk_commit();
                     }
                     out_parity ^= 1;
@@ -456,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             // names this expert (the route log is read back and checked, row
             // by row); a row that fails the check is a dispatch mismatch.
             // The per-token private count follows the rows physically run.
-            if (t.mode == kGateUp) {
+            if (gu) {
                 const unsigned vm = __ballot_sync(~0u, valid);
                 if (!t.shared && t.n0 == 0) {
                     const int tok = valid ? p.tok_of_slot[grow] : -1;
@@ -475,22 +608,170 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 if (t.shared && p.shared_rows && lane == 0 && vm && (t.n0 % p.I) == 0)
                     atomicAdd(p.shared_rows, (unsigned)__popc(vm));
             }
-            if (p.nph == 2 && t.ph == 0) {
-                // release this warp's activation rows to the down tiles that read
-                // them: the row stores (generic) and the TMA stores (async proxy,
-                // complete after wait_group 0) are ordered before the count
+            uint32_t *release = nullptr;
+            if (gu && p.has_down) release = p.ready + tt.mpre[t.g] + t.m_tile;
+            if (!gu && p.has_comb) release = p.done_cb + t.cb;
+            if (release) {
+                // release this warp's rows to the tiles that read them (down
+                // tiles: the activations; combine items: this column block of
+                // y): the row stores (generic) and the TMA stores (async
+                // proxy, complete after wait_group 0) are ordered before the count
                 __threadfence();
                 __syncwarp();
                 if (lane == 0) {
                     bulk_wait_all();
                     asm volatile("fence.proxy.async.global;\n" ::: "memory");
                     __threadfence();
-                    atomicAdd(p.ready + tt.mpre[t.g] + t.m_tile, 1u);
+                    atomicAdd(release, 1u);
                 }
                 __syncwarp();
             }
         }
         if (lane == 0) bulk_wait_all();  // this warp's TMA stores are complete before the CTA exits
+    } else if (warp >= 6) {
+        // ------------------------------------------------ A-row gather, combine
+        // Gather: thread i of the 128 copies 16-byte chunk (i & 7) of tile rows
+        // (i >> 3) + 16 j, j = 0..7, every stage, into the 128-byte-swizzled A
+        // slot of the stage (chunk c of row r at chunk c ^ (r & 7)); a warp
+        // instruction covers four whole 128-byte rows.  Rows past the tile's
+        // rows are zero-filled.  Each warp keeps kGatherDepth stages in flight:
+        // after issuing a stage it waits for the oldest one's copies, makes
+        // them visible to the async proxy (the tensor cores read through it)
+        // and arrives on that stage's full barrier.
+        const int gi = tid - 192;            // 0 .. 127
+        const int chunk = gi & 7, row0 = gi >> 3;
+        uint32_t sc = 0;                     // ring stages passed so far (the ring position)
+        uint32_t pend_first = 0;             // oldest stage with copies not yet released
+        int npend = 0;
+        bool ok = true;
+        auto release_oldest = [&]() {
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(full_bar((int)(pend_first % kStages)));
+            ++pend_first;
+            --npend;
+        };
+        auto drain = [&]() {
+            cp_async_wait<0>();
+            while (npend > 0) release_oldest();
+        };
+        for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+            const Tile t = decode_tile(p, tt, G, tile);
+            if (t.kind == kTileComb) {
+                drain();
+                // ---- combine item: tokens [t0, t0 + 32) of column block cb,
+                // once every down tile of the block has stored its y
+                const uint32_t need = 4u * (uint32_t)tt.mpre[G];
+                int waited = 1;
+                if (lane == 0) {
+                    const unsigned long long t0 = globaltimer_ns();
+                    while (ld_acquire_gpu(p.done_cb + t.cb) < need) {
+                        if (s_abort || globaltimer_ns() - t0 > kWaitLimitNs) {
+                            if (!s_abort && p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
+                            s_abort = 1;
+                            waited = 0;
+                            break;
+                        }
+                        __nanosleep(256);
+                    }
+                }
+                waited = __shfl_sync(~0u, waited, 0);
+                if (!waited) { ok = false; break; }
+                const int bn = p.ph[kDown].bn, nch = bn / 8, per = 32 / nch;  // chunks per row, tokens per pass
+                const int sub = lane / nch, cc = (lane - sub * nch) * 8;      // this lane's token and columns
+                const bf16 *ycb = p.ph[kDown].C_routed + (size_t)t.cb * p.R * bn;
+                const bf16 *yshcb = p.E_sh > 0 ? p.ph[kDown].C_shared + (size_t)t.cb * p.T * bn : nullptr;
+                const int tw0 = t.t0 + (warp - 6) * (kCombTokens / kGatherWarps);
+                for (int i0 = 0; i0 < kCombTokens / kGatherWarps; i0 += per) {
+                    const int tok = tw0 + i0 + sub;
+                    const bool live = tok < p.T;
+                    const int32_t *slots = p.slot_of + (size_t)(live ? tok : 0) * p.k;
+                    float acc[8];
+#pragma unroll
+                    for (int q2 = 0; q2 < 8; ++q2) acc[q2] = 0.f;
+                    for (int j0 = 0; j0 < p.k; j0 += 8) {
+                        uint4 v[8];
+                        int sl[8];
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) {
+                            sl[u] = -1;
+                            if (live && j0 + u < p.k) {
+                                int slot = __ldg(slots + j0 + u);
+                                if ((unsigned)slot >= (unsigned)p.R) slot = 0;  // only after a dispatch mismatch
+                                sl[u] = slot;
+                                v[u] = *reinterpret_cast<const uint4 *>(ycb + (size_t)slot * bn + cc);
+                            }
+                        }
+#pragma unroll
+                        for (int u = 0; u < 8; ++u)
+                            if (sl[u] >= 0) add_bf16x8(acc, v[u]);
+                        // these rows of y are not read again: drop them from L2
+                        // without a write-back, one lane per 128-byte line, once
+                        // every lane's load of the line has returned
+                        __syncwarp();
+                        if ((cc & 63) == 0) {
+#pragma unroll
+                            for (int u = 0; u < 8; ++u)
+                                if (sl[u] >= 0) discard_l2_line(ycb + (size_t)sl[u] * bn + cc);
+                        }
+                    }
+                    if (yshcb) {
+                        const bf16 *src = yshcb + (size_t)(live ? tok : 0) * bn + cc;
+                        if (live) add_bf16x8(acc, *reinterpret_cast<const uint4 *>(src));
+                        __syncwarp();
+                        if (live && (cc & 63) == 0) discard_l2_line(src);
+                    }
+                    if (live) {
+                        uint4 o;
+                        o.x = pack_bf16x2(acc[0], acc[1]);
+                        o.y = pack_bf16x2(acc[2], acc[3]);
+                        o.z = pack_bf16x2(acc[4], acc[5]);
+                        o.w = pack_bf16x2(acc[6], acc[7]);
+                        *reinterpret_cast<uint4 *>(p.out + (size_t)tok * p.H + t.cb * bn + cc) = o;
+                    }
+                }
+                continue;
+            }
+            if (t.kind != kTileGU || t.shared) {  // A comes through TMA: only follow the ring
+                drain();
+                sc += (uint32_t)t.nkb;
+                pend_first = sc;
+                continue;
+            }
+            // this thread's 8 rows: their token rows in the hidden states
+            const bf16 *src[8];
+            uint32_t nbytes[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int r = row0 + 16 * j;
+                const int tok = r < t.rows ? p.tok_of_slot[t.row_base + t.m0 + r] : -1;
+                const bool in = (unsigned)tok < (unsigned)p.T;
+                src[j] = p.hidden + (in ? (size_t)tok * p.H : 0) + chunk * 8;
+                nbytes[j] = in ? 16u : 0u;
+            }
+            if (npend == 0) pend_first = sc;
+            for (int kb = 0; kb < t.nkb; ++kb, ++sc) {
+                const int stage = (int)(sc % kStages);
+                const uint32_t phase = (sc / kStages) & 1u;
+                int free_ = 1;
+                if (lane == 0) free_ = mbar_wait(empty_bar(stage), phase ^ 1u, &s_abort, p.status) ? 1 : 0;
+                free_ = __shfl_sync(~0u, free_, 0);
+                if (!free_) { ok = false; break; }
+                const uint32_t sA = sbase + stage * kStageBytes;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const int r = row0 + 16 * j;
+                    cp_async16_zfill(sA + r * 128 + ((chunk ^ (r & 7)) << 4), src[j] + kb * BK, nbytes[j]);
+                }
+                cp_async_commit();
+                ++npend;
+                if (npend > kGatherDepth) {
+                    cp_async_wait<kGatherDepth>();
+                    release_oldest();
+                }
+            }
+        }
+        drain();
     }
 
     // every warp reconverges before the block barrier: __syncthreads is a
@@ -507,79 +788,88 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
 
 // ------------------------------------------------------------ host side
 
-// Parameters and tensor maps of one GEMM (`mode`) as phase `ph` of a launch.
-bool fill_phase(const Ctx &c, int mode, int ph, TcParams &p, TcMaps &maps)
+// Parameters and tensor maps of one GEMM (`mode`) of a launch.
+bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
 {
     const Shape &s = c.s;
     const uint64_t R = (uint64_t)s.T * s.k, T = (uint64_t)s.T;
-    TcPhase &f = p.ph[ph];
-    f.mode = mode;
+    TcPhase &f = p.ph[mode];
     bool ok = true;
     if (mode == kGateUp) {
-        f.bn = 128;
-        f.idesc = make_idesc(BM, 256);
         f.C_routed = c.act;
         f.C_shared = c.act_sh;
-        ok &= encode_2d_box(&maps.c_routed[ph], c.act, s.I, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        ok &= encode_2d_box(&maps.c_routed[mode], c.act, s.I, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
         if (s.E_sh > 0)
-            ok &= encode_2d_box(&maps.c_shared[ph], c.act_sh, (uint64_t)s.E_sh * s.I, T, kOutBox, kOutBox,
+            ok &= encode_2d_box(&maps.c_shared[mode], c.act_sh, (uint64_t)s.E_sh * s.I, T, kOutBox, kOutBox,
                                 CU_TENSOR_MAP_SWIZZLE_64B);
-        ok &= encode_2d(&maps.a_routed[ph], c.a_perm, s.H, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.I;
-            ok &= encode_2d(&maps.b0[ph][q], c.gate[q], s.H, n, 128);
-            ok &= encode_2d(&maps.b1[ph][q], c.up[q], s.H, n, 128);
+            ok &= encode_2d(&maps.b0[mode][q], c.gate[q], s.H, n, 128);
+            ok &= encode_2d(&maps.b1[mode][q], c.up[q], s.H, n, 128);
         }
         if (s.E_sh > 0) {
-            ok &= encode_2d(&maps.a_shared[ph], c.hidden, s.H, T, BM);
-            ok &= encode_2d(&maps.b0[ph][2], c.gate[2], s.H, (uint64_t)s.E_sh * s.I, 128);
-            ok &= encode_2d(&maps.b1[ph][2], c.up[2], s.H, (uint64_t)s.E_sh * s.I, 128);
+            ok &= encode_2d(&maps.a_shared[mode], c.hidden, s.H, T, BM);
+            ok &= encode_2d(&maps.b0[mode][2], c.gate[2], s.H, (uint64_t)s.E_sh * s.I, 128);
+            ok &= encode_2d(&maps.b1[mode][2], c.up[2], s.H, (uint64_t)s.E_sh * s.I, 128);
         }
     } else {
-        f.bn = (s.H % 256 == 0) ? 256 : 128;
-        f.idesc = make_idesc(BM, f.bn);
+        const uint64_t nb = (uint64_t)p.nb;
         f.C_routed = c.y;
         f.C_shared = c.y_sh;
-        ok &= encode_2d_box(&maps.c_routed[ph], c.y, s.H, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        // y and y_sh by column block: [nb * rows][bn]
+        ok &= encode_2d_box(&maps.c_routed[mode], c.y, f.bn, nb * R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
         if (s.E_sh > 0)
-            ok &= encode_2d_box(&maps.c_shared[ph], c.y_sh, s.H, T, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
-        ok &= encode_2d(&maps.a_routed[ph], c.act, s.I, R, BM);
+            ok &= encode_2d_box(&maps.c_shared[mode], c.y_sh, f.bn, nb * T, kOutBox, kOutBox,
+                                CU_TENSOR_MAP_SWIZZLE_64B);
+        ok &= encode_2d(&maps.a_routed[mode], c.act, s.I, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
-            ok &= encode_2d(&maps.b0[ph][q], c.down[q], s.I, n, f.bn / 2);
+            ok &= encode_2d(&maps.b0[mode][q], c.down[q], s.I, n, f.bn / 2);
         }
         if (s.E_sh > 0) {
-            ok &= encode_2d(&maps.a_shared[ph], c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
-            ok &= encode_2d(&maps.b0[ph][2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, f.bn / 2);
+            ok &= encode_2d(&maps.a_shared[mode], c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
+            ok &= encode_2d(&maps.b0[mode][2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, f.bn / 2);
         }
     }
     return ok;
 }
 
-// One persistent launch running the GEMMs of `modes` in order (one or two).
-cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
+// One persistent launch: the gate/up tiles, the down tiles and the combine
+// items, as selected (the combine items only with the down tiles).
+cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool comb)
 {
     const Shape &s = c.s;
     TcParams p;
     TcMaps maps;
     memset(&p, 0, sizeof(p));
     memset(&maps, 0, sizeof(maps));
-    p.nph = nph;
-    p.E = s.E(); p.E_pub = s.E_pub; p.E_sh = s.E_sh; p.T = s.T; p.H = s.H; p.I = s.I; p.R = s.T * s.k;
+    p.has_gu = gu;
+    p.has_down = down;
+    p.has_comb = down && comb;
+    p.E = s.E(); p.E_pub = s.E_pub; p.E_sh = s.E_sh; p.T = s.T; p.H = s.H; p.I = s.I; p.R = s.T * s.k; p.k = s.k;
+    p.ph[kGateUp].bn = 128;
+    p.ph[kGateUp].idesc = make_idesc(BM, 256);
+    p.ph[kDown].bn = column_block(s.H);
+    p.ph[kDown].idesc = make_idesc(BM, p.ph[kDown].bn);
+    p.nb = s.H / p.ph[kDown].bn;
     p.offsets = c.offsets;
     p.w_of_slot = c.w_of_slot;
     p.tok_of_slot = c.tok_of_slot;
+    p.slot_of = c.slot_of;
     p.topk_idx = c.idx;
-    p.k = s.k;
+    p.hidden = c.hidden;
     p.ready = c.gemm_ready;
+    p.done_cb = c.gemm_ready + gemm_ready_blocks(s);
+    p.out = c.out;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
     p.exec_priv_rows = c.audit.exec_priv_rows;
     p.shared_rows = c.audit.shared_rows;
     p.status = c.audit.status;
     bool ok = true;
-    for (int ph = 0; ph < nph; ++ph) ok &= fill_phase(c, modes[ph], ph, p, maps);
-    if (c.saved_gu && modes[0] == kGateUp) {
+    if (gu) ok &= fill_phase(c, kGateUp, p, maps);
+    if (down) ok &= fill_phase(c, kDown, p, maps);
+    if (c.saved_gu && gu) {
         p.saved_gu = c.saved_gu;
         ok &= encode_2d_f32(&maps.gu_save, c.saved_gu, 2 * (uint64_t)s.I, (uint64_t)s.T * s.k, 16, 32,
                             CU_TENSOR_MAP_SWIZZLE_64B);
@@ -594,22 +884,10 @@ cudaError_t launch_tc(const Ctx &c, int nph, const int *modes)
     return launch_pdl(expert_gemm_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
 }
 
-}  // namespace
-
-cudaError_t launch_gateup(const Ctx &c)
-{
-    const int m[1] = {kGateUp};
-    return launch_tc(c, 1, m);
-}
-cudaError_t launch_down(const Ctx &c)
-{
-    const int m[1] = {kDown};
-    return launch_tc(c, 1, m);
-}
-// Whether the persistent pair's grid (one CTA per SM) can be resident all at
-// once: its down tiles wait for gate/up tiles that other CTAs own, so every
-// CTA must run concurrently.  Cached per device.
-static bool pair_fits(const Ctx &c)
+// Whether the persistent grid (one CTA per SM) can be resident all at once:
+// its down tiles wait for gate/up tiles and its combine items for down tiles
+// that other CTAs own, so every CTA must run concurrently.  Cached per device.
+static bool grid_fits(const Ctx &c)
 {
     static std::atomic<int> fits[64];  // 0 unknown, 1 yes, 2 no
     int dev = 0;
@@ -625,18 +903,24 @@ static bool pair_fits(const Ctx &c)
     return ok;
 }
 
-cudaError_t launch_experts(const Ctx &c, bool zero_ready)
+}  // namespace
+
+cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, true, false, false); }
+cudaError_t launch_down(const Ctx &c) { return launch_tc(c, false, true, false); }
+
+cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool with_combine)
 {
-    if (!pair_fits(c)) {  // the two GEMMs one after the other: no cross-CTA wait
-        const cudaError_t err = launch_gateup(c);
-        return err == cudaSuccess ? launch_down(c) : err;
+    if (!grid_fits(c)) {  // one stage after the other: no cross-CTA wait
+        cudaError_t err = launch_gateup(c);
+        if (err == cudaSuccess) err = launch_down(c);
+        if (err == cudaSuccess && with_combine) err = launch_combine(c);
+        return err;
     }
     if (zero_ready) {
         const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
         if (err != cudaSuccess) return err;
     }
-    const int m[2] = {kGateUp, kDown};
-    return launch_tc(c, 2, m);
+    return launch_tc(c, true, true, with_combine);
 }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()

@@ -12,11 +12,12 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Each routed group adds at most one partial 128-row block beyond R/128; the
 // shared-expert group covers the T tokens.
-size_t gemm_ready_words(const Shape &s)
+size_t gemm_ready_blocks(const Shape &s)
 {
     const size_t R = (size_t)s.T * (size_t)s.k;
     return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 1;
 }
+size_t gemm_ready_words(const Shape &s) { return gemm_ready_blocks(s) + (size_t)s.H / 128; }
 
 static bool shape_ok(const Shape &s)
 {
@@ -216,14 +217,16 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     if (err == cudaSuccess && (stages & PMPE_STAGE_ROUTE)) err = launch_route(c);
     if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE)) err = launch_permute(c);
     if ((stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN)) {
-        // one persistent launch; its readiness counters are cleared by the
-        // router's memset when the router runs in this call
-        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_ROUTE));
+        // one persistent launch, with the combine when it is asked for too;
+        // its readiness counters are cleared by the router's memset when the
+        // router runs in this call
+        if (err == cudaSuccess)
+            err = launch_experts(c, !(stages & PMPE_STAGE_ROUTE), (stages & PMPE_STAGE_COMBINE) != 0);
     } else {
         if (err == cudaSuccess && (stages & PMPE_STAGE_GATEUP)) err = launch_gateup(c);
         if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c);
+        if (err == cudaSuccess && (stages & PMPE_STAGE_COMBINE)) err = launch_combine(c);
     }
-    if (err == cudaSuccess && (stages & PMPE_STAGE_COMBINE)) err = launch_combine(c);
     return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
 }
 
@@ -262,6 +265,9 @@ int pmpe_moe_backward_private(const pmpe_moe_desc *d, const void *dout, float *d
         if (err == cudaSuccess) err = cudaMemsetAsync(d_down_priv, 0, ih, st);
         return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
     }
+    // the forward gathers its rows on the fly; the backward's GEMMs read the
+    // private experts' dispatched rows as one matrix
+    if (launch_gather_dispatch_rows(c, s.E_pub, s.E()) != cudaSuccess) return PMPE_ERR_CUDA;
     return launch_backward_private(c, (const bf16 *)dout, d_router_priv, d_gate_priv, d_up_priv, d_down_priv,
                                    (uint8_t *)bwd_workspace) == cudaSuccess
                ? PMPE_OK
@@ -292,6 +298,7 @@ int pmpe_moe_backward_input(const pmpe_moe_desc *d, const void *dout, float *d_h
     const int rc = make_ctx(d, stream, &c);
     if (rc != PMPE_OK) return rc;
     if (s.T == 0) return PMPE_OK;  // no tokens: nothing to write
+    if (launch_gather_dispatch_rows(c, 0, s.E()) != cudaSuccess) return PMPE_ERR_CUDA;
     return launch_backward_input(c, (const bf16 *)dout, d_hidden, (uint8_t *)bwd_workspace) == cudaSuccess
                ? PMPE_OK
                : PMPE_ERR_CUDA;
@@ -339,6 +346,7 @@ int pmpe_moe_backward_step(const pmpe_moe_desc *d, const void *dout, float *d_ro
         if (err == cudaSuccess) err = cudaMemsetAsync(d_down_priv, 0, ih, st);
         return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
     }
+    if (launch_gather_dispatch_rows(c, 0, s.E()) != cudaSuccess) return PMPE_ERR_CUDA;
     return launch_backward_step(c, (const bf16 *)dout, d_router_priv, d_gate_priv, d_up_priv, d_down_priv, d_hidden,
                                 (uint8_t *)bwd_workspace) == cudaSuccess
                ? PMPE_OK

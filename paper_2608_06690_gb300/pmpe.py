@@ -42,15 +42,15 @@ STAGE_COMBINE = 0x10
 STAGE_ALL = 0x1F
 
 # Kernels one full forward launches: router/top-k (with the policy resolve),
-# dispatch + row gather, the gate/up and down GEMMs (one persistent launch),
-# combine (plus one memset of the per-expert counters, which is not a kernel
-# of this library).
-KERNELS_PER_FORWARD = 4
-# kernels one private-branch backward launches: dout row gather, the dL/da
-# GEMM, the gate/up recompute GEMM with the SwiGLU backward, router gradient,
-# router weight-gradient partials and their reduction, the expert
-# weight-gradient GEMM
-KERNELS_PER_BACKWARD = 7
+# the dispatch order, and one persistent launch of the gate/up GEMM (rows
+# gathered from the hidden states), the down GEMM and the combine (plus one
+# memset of the per-expert counters, which is not a kernel of this library).
+KERNELS_PER_FORWARD = 3
+# kernels one private-branch backward launches: the dispatched rows of the
+# private experts, dout row gather, the dL/da GEMM, the gate/up recompute GEMM
+# with the SwiGLU backward, router gradient, router weight-gradient partials
+# and their reduction, the expert weight-gradient GEMM
+KERNELS_PER_BACKWARD = 8
 
 
 def kernels_per_backward_private(shape) -> int:
@@ -60,22 +60,24 @@ def kernels_per_backward_private(shape) -> int:
 
 
 def kernels_per_backward_input(shape) -> int:
-    """Kernels one input-gradient backward launches: the dout row gather, Z,
+    """Kernels one input-gradient backward launches: the dispatched rows, the
+    dout row gather, Z,
     the gate/up recompute with the SwiGLU backward and dA over the routed
     experts (the same three again over the shared experts, if any), the
     router's softmax gradient and the per-token sum; for the pool softmax
     also the pool token lists, the logits GEMM and the router-term GEMM."""
-    return 6 + (3 if shape.E_sh > 0 else 0) + (0 if shape.renormalize else 3)
+    return 7 + (3 if shape.E_sh > 0 else 0) + (0 if shape.renormalize else 3)
 
 
 def kernels_per_backward_step(shape) -> int:
-    """Kernels one combined backward launches: the dout row gather, Z, the
+    """Kernels one combined backward launches: the dispatched rows, the dout
+    row gather, Z, the
     gate/up recompute and dA over the routed experts (the same three over the
     shared experts, if any), the router's dz, its weight-gradient partials
     and their sum, the expert weight-gradient GEMM and the per-token sum; for
     the pool softmax also the pool token lists, the logits GEMM and the
     router-term GEMM."""
-    return 8 + (3 if shape.E_sh > 0 else 0) + (0 if shape.renormalize else 3)
+    return 9 + (3 if shape.E_sh > 0 else 0) + (0 if shape.renormalize else 3)
 
 EXPORTED = ("pmpe_moe_workspace_size", "pmpe_moe_workspace_layout", "pmpe_audit_words", "pmpe_policy_resolve",
             "pmpe_moe_forward", "pmpe_moe_forward_stages", "pmpe_audit_reset", "pmpe_audit_read",

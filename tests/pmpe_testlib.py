@@ -97,8 +97,6 @@ def run_gpu_layer(shape: LayerShape, w: dict, h, pol, audit_reset=True, stages=N
                 offsets=region("offsets", torch.int32, E + 1).numpy().view(np.uint32),
                 slot_of=region("slot_of", torch.int32, R).numpy().reshape(T, k),
                 tok_of_slot=region("tok_of_slot", torch.int32, R).numpy(),
-                a_perm=(region("a_perm", torch.bfloat16, R * shape.H).view(torch.int16).numpy().view(np.uint16)
-                        .reshape(R, shape.H) if R * shape.H <= (1 << 24) else None),
                 layer=layer)
 
 
@@ -206,7 +204,8 @@ def check_dispatch(shape: LayerShape, h_cpu, gpu: dict):
     GPU's own route log, bit for bit: the expert offsets, and the stable slot
     order (expert-major, then token, then rank) in slot_of and tok_of_slot;
     plus the structure (slot_of a bijection onto [0, T*k) that tok_of_slot
-    inverts) and every gathered row equal to its token's row."""
+    inverts).  The expert kernel gathers each slot's row from the hidden
+    states through tok_of_slot, so these maps are what it runs on."""
     import oracle
     counts, offsets, slot_of_ref, tok_of_slot_ref = oracle.permute(gpu["idx"], shape.E)
     assert np.array_equal(gpu["offsets"], offsets)
@@ -222,5 +221,3 @@ def check_dispatch(shape: LayerShape, h_cpu, gpu: dict):
         assert np.array_equal(np.sort(tos[lo:hi]), tok_of_slot_ref[lo:hi]), f"expert {e} holds other tokens"
         mine = gpu["idx"] == e
         assert np.all((so[mine] >= lo) & (so[mine] < hi)), f"a row of expert {e} sits outside its slots"
-    if gpu.get("a_perm") is not None:
-        assert np.array_equal(gpu["a_perm"], bf16_bits(h_cpu)[tos])
