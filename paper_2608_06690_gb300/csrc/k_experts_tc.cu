@@ -70,8 +70,8 @@ constexpr int kTmemCols = 2 * kAccCols;
 constexpr int kGatherWarps = 4;               // warps 6..9
 constexpr int kThreads = 192 + 32 * kGatherWarps;
 constexpr int kLoaders = 3;                   // TMA-issuing lanes of warp 0
-constexpr int kFullArrivals = kLoaders + kGatherWarps;  // per ring stage
-constexpr int kGatherDepth = kStages - 1;     // stages a gather warp keeps in flight
+constexpr int kGatherThreads = 32 * kGatherWarps;
+constexpr int kFullArrivals = kLoaders + kGatherThreads;  // per ring stage
 constexpr int kCombTokens = 32;               // tokens per combine item (8 per gather warp)
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
@@ -237,13 +237,6 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
     return comb_tile(p.nb - 1, u2 - (p.nb - 1) * round);
 }
 
-// 16-byte async copy global -> shared with an explicit source size (0: the
-// 16 bytes are zero-filled and nothing is read).
-__device__ __forceinline__ void cp_async16_zfill(uint32_t dst, const void *src, uint32_t src_bytes)
-{
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-
 // Drop a 128-byte line from L2 without writing it back (its data is not read
 // again before it is rewritten).
 __device__ __forceinline__ void discard_l2_line(const void *p)
@@ -282,6 +275,10 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
 
     const int G = p.E + (p.E_sh > 0 ? 1 : 0);
+    // expert weights stream through L2 once (evict first); the hidden states,
+    // activations and per-row outputs are read again by other tiles of this
+    // launch (evict last)
+    const uint64_t pol_stream = l2_policy_evict_first(), pol_keep = l2_policy_evict_last();
     pdl_trigger();
 
     if (tid == 0) {
@@ -393,21 +390,22 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 const int kx = kb * BK;
                 if (lane == 0) {
                     if (!gather) {
-                        tma_load_2d(sA, amap, full_bar(stage), kx, arow);
-                        mbar_arrive_count(full_bar(stage), kGatherWarps);
+                        tma_load_2d_hint(sA, amap, full_bar(stage), kx, arow, pol_keep);
+                        mbar_arrive_count(full_bar(stage), kGatherThreads);
                     }
                 } else if (t.ph == kGateUp) {
                     const int brow = ei * p.I + t.n0;  // shared: n0 spans E_sh * I rows
-                    tma_load_2d(sB + (lane - 1) * BM * 128, lane == 1 ? &maps.b0[t.ph][q] : &maps.b1[t.ph][q],
-                                full_bar(stage), kx, brow);
+                    tma_load_2d_hint(sB + (lane - 1) * BM * 128, lane == 1 ? &maps.b0[t.ph][q] : &maps.b1[t.ph][q],
+                                     full_bar(stage), kx, brow, pol_stream);
                 } else {
                     const int half = (lane - 1) * (t.bn / 2);
                     if (t.shared) {
                         const int sidx = kx / p.I;
-                        tma_load_2d(sB + half * 128, &maps.b0[t.ph][2], full_bar(stage), kx - sidx * p.I,
-                                    sidx * p.H + t.n0 + half);
+                        tma_load_2d_hint(sB + half * 128, &maps.b0[t.ph][2], full_bar(stage), kx - sidx * p.I,
+                                         sidx * p.H + t.n0 + half, pol_stream);
                     } else {
-                        tma_load_2d(sB + half * 128, &maps.b0[t.ph][q], full_bar(stage), kx, ei * p.H + t.n0 + half);
+                        tma_load_2d_hint(sB + half * 128, &maps.b0[t.ph][q], full_bar(stage), kx,
+                                         ei * p.H + t.n0 + half, pol_stream);
                     }
                 }
                 filled |= 1u << stage;
@@ -441,6 +439,10 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             for (int kb = 0; kb < t.nkb; ++kb) {
                 if (!mbar_wait(full_bar(stage), phase, &s_abort, p.status)) { ok = false; break; }
                 tc_fence_after();
+                // rows the gather warps copied (generic proxy, complete when
+                // the barrier's phase completed) are read by the tensor cores
+                // through the async proxy
+                fence_proxy_async_smem();
                 const uint32_t sA = sbase + stage * kStageBytes, sB = sA + kABytes;
                 const uint64_t ad = sw128_desc(sA), bd = sw128_desc(sB);
 #pragma unroll
@@ -571,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tma_store_2d(cmap, sbuf, col0 + c * 32, out_row0 + quarter * 32);
+                        tma_store_2d_hint(cmap, sbuf, col0 + c * 32, out_row0 + quarter * 32, pol_keep);
                         bulk_commit();
                     }
                     out_parity ^= 1;
@@ -634,31 +636,19 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         // (i >> 3) + 16 j, j = 0..7, every stage, into the 128-byte-swizzled A
         // slot of the stage (chunk c of row r at chunk c ^ (r & 7)); a warp
         // instruction covers four whole 128-byte rows.  Rows past the tile's
-        // rows are zero-filled.  Each warp keeps kGatherDepth stages in flight:
-        // after issuing a stage it waits for the oldest one's copies, makes
-        // them visible to the async proxy (the tensor cores read through it)
-        // and arrives on that stage's full barrier.
+        // rows are zero-filled.  Each thread's copies of a stage arrive on the
+        // stage's full barrier when they complete (cp.async.mbarrier.arrive),
+        // so the threads never wait for their own copies: up to the whole ring
+        // is in flight.  The MMA thread fences the async proxy after the
+        // barrier before the tensor cores read the rows.
         const int gi = tid - 192;            // 0 .. 127
         const int chunk = gi & 7, row0 = gi >> 3;
         uint32_t sc = 0;                     // ring stages passed so far (the ring position)
-        uint32_t pend_first = 0;             // oldest stage with copies not yet released
-        int npend = 0;
         bool ok = true;
-        auto release_oldest = [&]() {
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(full_bar((int)(pend_first % kStages)));
-            ++pend_first;
-            --npend;
-        };
-        auto drain = [&]() {
-            cp_async_wait<0>();
-            while (npend > 0) release_oldest();
-        };
+        auto drain = [&]() { cp_async_wait<0>(); };
         for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
             if (t.kind == kTileComb) {
-                drain();
                 // ---- combine item: tokens [t0, t0 + 32) of column block cb,
                 // once every down tile of the block has stored its y
                 const uint32_t need = 4u * (uint32_t)tt.mpre[G];
@@ -733,9 +723,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 continue;
             }
             if (t.kind != kTileGU || t.shared) {  // A comes through TMA: only follow the ring
-                drain();
                 sc += (uint32_t)t.nkb;
-                pend_first = sc;
                 continue;
             }
             // this thread's 8 rows: their token rows in the hidden states
@@ -749,7 +737,6 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 src[j] = p.hidden + (in ? (size_t)tok * p.H : 0) + chunk * 8;
                 nbytes[j] = in ? 16u : 0u;
             }
-            if (npend == 0) pend_first = sc;
             for (int kb = 0; kb < t.nkb; ++kb, ++sc) {
                 const int stage = (int)(sc % kStages);
                 const uint32_t phase = (sc / kStages) & 1u;
@@ -761,14 +748,9 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
                     const int r = row0 + 16 * j;
-                    cp_async16_zfill(sA + r * 128 + ((chunk ^ (r & 7)) << 4), src[j] + kb * BK, nbytes[j]);
+                    cp_async16_zfill(sA + r * 128 + ((chunk ^ (r & 7)) << 4), src[j] + kb * BK, nbytes[j], pol_keep);
                 }
-                cp_async_commit();
-                ++npend;
-                if (npend > kGatherDepth) {
-                    cp_async_wait<kGatherDepth>();
-                    release_oldest();
-                }
+                cp_async_arrive_noinc(full_bar(stage));
             }
         }
         drain();
