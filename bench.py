@@ -228,9 +228,9 @@ def algorithmic_work(s, counts: np.ndarray):
     """FLOPs of the two grouped GEMMs and the least DRAM bytes of each stage,
     for one forward with the given per-expert row counts.  "experts" is the
     forward's persistent launch: gate/up (rows gathered from the hidden
-    states), down and the combine, whose activations and per-row outputs are
-    internal to it; "pair", "gateup", "down" and "combine" are the pieces run
-    on their own (diagnostics), which pass those intermediates through memory."""
+    states), down and the combine, whose activations and per-row outputs stay
+    inside it; "gateup" and "down" (with the combine) are its two GEMMs run on
+    their own (diagnostics), which pass the activations through memory."""
     R = s.T * s.k
     f_gateup = 2.0 * R * s.H * 2 * s.I + 2.0 * s.T * s.H * 2 * s.E_sh * s.I
     f_down = 2.0 * R * s.I * s.H + 2.0 * s.T * s.E_sh * s.I * s.H
@@ -240,11 +240,9 @@ def algorithmic_work(s, counts: np.ndarray):
     w_gu = (touched + s.E_sh) * 2 * s.I * s.H * 2
     w_dn = (touched + s.E_sh) * s.I * s.H * 2
     act = R * s.I * 2 + s.T * s.E_sh * s.I * 2
-    yb = R * s.H * 2 + (s.T * s.H * 2 if s.E_sh else 0)
-    maps = R * 12                                   # tok_of_slot, w_of_slot, slot_of
+    maps = R * 8                                    # tok_of_slot, w_of_slot
     b_gateup = w_gu + s.T * s.H * 2 + act + maps
-    b_down = w_dn + act + yb + maps
-    b_combine = yb + s.T * s.H * 2 + maps
+    b_down = w_dn + act + s.T * s.H * 2 + maps
     b_experts = gemm_weight_bytes + s.T * s.H * 2 + s.T * s.H * 2 + maps
     b_route = s.T * s.H * 2 + (s.E_pub + s.E_priv) * s.H * 2 + s.T * s.k * 8 + s.T
     # the dispatch order: route log and tickets in, slot maps out
@@ -255,8 +253,7 @@ def algorithmic_work(s, counts: np.ndarray):
     return dict(flops_gateup=f_gateup, flops_down=f_down, bytes_gateup=b_gateup, bytes_down=b_down,
                 bytes_layer_min=b_layer_min,
                 flops_experts=f_gateup + f_down, bytes_experts=b_experts,
-                flops_pair=f_gateup + f_down, bytes_pair=b_gateup + b_down,
-                bytes_route=b_route, bytes_permute=b_permute, bytes_combine=b_combine,
+                bytes_route=b_route, bytes_permute=b_permute,
                 touched_experts=touched, gemm_weight_bytes=gemm_weight_bytes)
 
 
@@ -373,7 +370,7 @@ def roofline_of(work, stage_avg, pipeline, hbm, tf_burst, peak_src):
     below it; both fractions are given for the GEMMs."""
     dominant = max(pipeline, key=stage_avg.get)
     sec = stage_avg[dominant] / 1e3
-    if dominant in ("experts", "pair", "gateup", "down"):
+    if dominant in ("experts", "gateup", "down"):
         tflops = work[f"flops_{dominant}"] / sec / 1e12
         gbs = work[f"bytes_{dominant}"] / sec / 1e9
         intensity = work[f"flops_{dominant}"] / work[f"bytes_{dominant}"]
@@ -433,12 +430,11 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     # is still busy flushing while the host enqueues the stage (no host gap
     # inside the measured interval); stages run in pipeline order on the
     # workspace the previous stage filled.  "experts" is the persistent
-    # gate/up + down + combine launch the forward runs; the gate/up + down
-    # pair, each GEMM and the combine launched on their own are diagnostics.
+    # gate/up + down + combine launch the forward runs; the gate/up GEMM and
+    # the down GEMM with the combine, launched on their own, are diagnostics.
     stages = [("route", pmpe.STAGE_ROUTE), ("permute", pmpe.STAGE_PERMUTE),
               ("experts", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE),
-              ("pair", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE),
-              ("gateup", pmpe.STAGE_GATEUP), ("down", pmpe.STAGE_DOWN)]
+              ("gateup", pmpe.STAGE_GATEUP), ("down", pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE)]
     pipeline = ("route", "permute", "experts")
     stage_ms = {n: [] for n, _ in stages}
     for _ in range(args.steps):
@@ -518,7 +514,7 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     stage_report = {}
     for n, ms in stage_avg.items():
         d = {"ms": ms}
-        if n in ("experts", "pair", "gateup", "down"):
+        if n in ("experts", "gateup", "down"):
             d["tflops"] = work[f"flops_{n}"] / (ms / 1e3) / 1e12
         d["gbs"] = work[f"bytes_{n}"] / (ms / 1e3) / 1e9
         d["hbm_frac"] = d["gbs"] / hbm

@@ -4,29 +4,34 @@
 // combine of their outputs.
 //
 //   gate/up:  act = bf16(silu(A_e W_gate,e^T) * (A_e W_up,e^T))    (SwiGLU fused)
-//   down:     y   = bf16(w_row * (act_e W_down,e^T))
-//   combine:  out_t = bf16(sum_j y[slot(t, j)] + y_shared[t])       (j ascending)
+//   down:     y   = w_row * (act_e W_down,e^T)                       (FP32, never stored)
+//   combine:  out_t = bf16(sum over t's experts in ascending id of y + y_shared[t])
 //
 // Groups are the routed experts (rows of the dispatch order) plus, with
 // shared experts, one dense group over all T tokens (gate/up weights of the
 // E_sh experts side by side; the down projection sums the E_sh experts in
 // one accumulator).  A persistent grid (one CTA per SM) walks a tile list
 // built on the device from the dispatch offsets: no host sync, and empty
-// experts contribute no tile.
+// experts contribute no tile.  The list holds every gate/up tile, then every
+// down tile, group by group (experts in ascending id, the shared group last),
+// n-tile major inside a group; CTA c takes tiles c, c + grid, ... in order.
 //
 // The routed gate/up tiles read their A rows straight from the hidden states:
 // the row of dispatch slot r is hidden[tok_of_slot[r]], gathered into shared
 // memory by four warps with 16-byte cp.async copies (the hidden states, read
 // by every expert a token routes to, stay in L2), so the dispatched rows are
-// never written out.  The down tiles run column block by column block (bn
-// output columns of every expert, then the next bn), writing y block by block;
-// once every down tile of a column block is stored, the same four warps sum
-// that block of y into the output, reading it back from L2.
+// never written out.
 //
-// Tile list: every gate/up tile (group by group, n-tile major), then the down
-// tiles of column block 0, then, for cb = 1 .. nb-1, the down tiles of block cb
-// followed by the combine items of block cb - 1, and last the combine items of
-// block nb - 1.  CTA c takes tiles c, c + grid, c + 2 grid, ... in order.
+// The combine runs in the down epilogue.  Each (token, column block of the
+// output) gets its contributions in ascending expert id -- the order of the
+// down tiles in the list -- then the shared experts': a contribution waits
+// until the token's counter for that block equals its rank, adds its FP32
+// values into an FP32 accumulator row (which stays in L2), and advances the
+// counter; the last one writes the BF16 output row instead.  The order is
+// fixed, so the output is deterministic and does not depend on the other
+// tokens of the batch, and the per-row outputs never go through memory.
+// Every wait is for a tile earlier in the list, and every CTA runs its tiles
+// in list order, so with all CTAs resident every wait ends.
 //
 // CTA roles (320 threads):
 //   warp 0       three lanes issue the TMA loads of a 4-stage ring, one
@@ -39,11 +44,12 @@
 //                of the next) and one thread issues tcgen05.mma M=128 N=256
 //                K=16, committing stage releases and accumulator-full events
 //   warps 2..5   epilogue: tcgen05.ld of the warp's 32 TMEM lanes (= 32 tile
-//                rows), SwiGLU or weight scaling, BF16 stores; in gate/up mode
-//                the tiles of N-tile 0 also write the execution audit, each
-//                row checked against the route log of its token
+//                rows); gate/up: SwiGLU, BF16 TMA stores and, in the tiles of
+//                N-tile 0, the execution audit (each row checked against the
+//                route log of its token); down: the routing weight and the
+//                ordered combine
 //   warps 6..9   the A-row gather of the routed gate/up tiles (cp.async into
-//                the ring), then the combine items
+//                the ring)
 // Every wait is bounded in time: on expiry the CTA records
 // PMPE_STATUS_PIPELINE_TIMEOUT, stops issuing work, waits (bounded) for its
 // own copies and MMAs in flight, frees its TMEM and exits.
@@ -72,7 +78,6 @@ constexpr int kThreads = 192 + 32 * kGatherWarps;
 constexpr int kLoaders = 3;                   // TMA-issuing lanes of warp 0
 constexpr int kGatherThreads = 32 * kGatherWarps;
 constexpr int kFullArrivals = kLoaders + kGatherThreads;  // per ring stage
-constexpr int kCombTokens = 32;               // tokens per combine item (8 per gather warp)
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
 constexpr int kOutBufBytes = kOutBox * kOutBox * 2;
@@ -80,7 +85,7 @@ constexpr int kOutBytes = 4 * 2 * kOutBufBytes;  // 4 epilogue warps x 2 buffers
 constexpr int kDynSmem = kStages * kStageBytes + kOutBytes + 1024 /* alignment slack */;
 
 enum { kGateUp = 0, kDown = 1 };
-enum { kTileGU = 0, kTileDown = 1, kTileComb = 2 };
+enum { kTileGU = 0, kTileDown = 1 };
 
 // One GEMM of the layer: gate/up (SwiGLU fused) or down (routing weight fused).
 struct TcPhase {
@@ -90,25 +95,24 @@ struct TcPhase {
 };
 
 struct TcParams {
-    // which parts this launch runs: the gate/up tiles, the down tiles, the
-    // combine items (only together with the down tiles)
-    int has_gu, has_down, has_comb;
+    // which GEMMs this launch runs: the gate/up tiles, the down tiles (with the combine)
+    int has_gu, has_down;
     TcPhase ph[2];    // [kGateUp], [kDown]
     int E, E_pub, E_sh, T, H, I, R, k;
-    int nb;           // column blocks of the down output: H / ph[kDown].bn
+    int nb;           // column blocks of the output: H / ph[kDown].bn
     const uint32_t *offsets;
     const float *w_of_slot;
     const int32_t *tok_of_slot;
-    const int32_t *slot_of;
-    const int32_t *topk_idx;  // [T, k] the route log, read back by the execution audit
+    const int32_t *topk_idx;  // [T, k] the route log: the execution audit and the combine's ranks
     const bf16 *hidden;       // the gather source of the routed gate/up tiles
     // has_gu && has_down: per (group, 128-row block), the gate/up epilogue
     // warps whose activations are stored (zeroed before the launch)
     uint32_t *ready;
-    // has_comb: per column block, the down epilogue warps whose y is stored
-    // (zeroed before the launch)
-    uint32_t *done_cb;
-    bf16 *out;                // has_comb: the layer output [T, H]
+    // has_down: per (token, column block), the contributions combined so far
+    // (zeroed before the launch), the FP32 partial sums [T, H] and the output
+    uint32_t *comb_cnt;
+    float *acc;
+    bf16 *out;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
     // optional FP32: the gate and up accumulators saved for the backward,
     // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
@@ -128,13 +132,13 @@ struct TcMaps {  // [phase]
 // ------------------------------------------------------------- tile list
 
 struct Tile {
-    int kind, ph, bn, g, m_tile, m0, n0, rows, row_base, nkb, cb, t0;
+    int kind, ph, bn, g, m_tile, m0, n0, rows, row_base, nkb, cb;
     bool shared;
 };
 
 struct TileTable {
-    int prefix[kMaxGroups + 1];  // gate/up tiles of the groups before g
-    int mpre[kMaxGroups + 1];    // 128-row blocks of the groups before g
+    int prefix[2][kMaxGroups + 1];  // tiles of the groups before g, per GEMM
+    int mpre[kMaxGroups + 1];       // 128-row blocks of the groups before g
     int rows[kMaxGroups];
     int base[kMaxGroups];
 };
@@ -148,111 +152,41 @@ __device__ __forceinline__ int group_k(const TcParams &p, int mode, bool shared)
     return mode == kGateUp ? p.H : (shared ? p.E_sh * p.I : p.I);
 }
 
-// The last group g with arr[g] <= x (arr ascending from arr[0] = 0).
-__device__ __forceinline__ int find_group(const int *arr, int G, int x)
-{
-    int lo = 0, hi = G - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (arr[mid] <= x) lo = mid; else hi = mid - 1;
-    }
-    return lo;
-}
-
-__device__ __forceinline__ int comb_items(const TcParams &p) { return (p.T + kCombTokens - 1) / kCombTokens; }
-
 __device__ __forceinline__ int total_tiles(const TcParams &p, const TileTable &tt, int G)
 {
-    return (p.has_gu ? tt.prefix[G] : 0) + (p.has_down ? p.nb * tt.mpre[G] : 0) +
-           (p.has_comb ? p.nb * comb_items(p) : 0);
+    return (p.has_gu ? tt.prefix[kGateUp][G] : 0) + (p.has_down ? tt.prefix[kDown][G] : 0);
 }
 
-__device__ __forceinline__ void fill_rows(const TcParams &p, const TileTable &tt, Tile &t, int g, int m_tile)
-{
-    t.g = g;
-    t.shared = g >= p.E;
-    t.m_tile = m_tile;
-    t.m0 = m_tile * BM;
-    t.rows = min(BM, tt.rows[g] - t.m0);
-    t.row_base = tt.base[g];
-}
-
-__device__ __forceinline__ Tile down_tile(const TcParams &p, const TileTable &tt, int G, int cb, int j)
-{
-    Tile t;
-    t.kind = kTileDown;
-    t.ph = kDown;
-    t.bn = p.ph[kDown].bn;
-    const int g = find_group(tt.mpre, G, j);
-    fill_rows(p, tt, t, g, j - tt.mpre[g]);
-    t.cb = cb;
-    t.n0 = cb * t.bn;
-    t.nkb = group_k(p, kDown, t.shared) / BK;
-    t.t0 = 0;
-    return t;
-}
-
-__device__ __forceinline__ Tile comb_tile(int cb, int item)
-{
-    Tile t;
-    t.kind = kTileComb;
-    t.ph = kDown;
-    t.cb = cb;
-    t.t0 = item * kCombTokens;
-    t.nkb = 0;
-    t.bn = t.g = t.m_tile = t.m0 = t.n0 = t.rows = t.row_base = 0;
-    t.shared = false;
-    return t;
-}
-
-// Tile `tile` of the list described at the top of this file.
+// Tile `tile` of the list: the gate/up tiles (when this launch runs them),
+// then the down tiles; inside a GEMM, group by group, n-tile major.
 __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &tt, int G, int tile)
 {
-    const int n_gu = p.has_gu ? tt.prefix[G] : 0;
-    if (tile < n_gu) {
-        Tile t;
-        t.kind = kTileGU;
-        t.ph = kGateUp;
-        t.bn = p.ph[kGateUp].bn;
-        const int g = find_group(tt.prefix, G, tile);
-        const int mt = (tt.rows[g] + BM - 1) / BM;
-        const int local = tile - tt.prefix[g];
-        const int n_tile = local / mt;
-        fill_rows(p, tt, t, g, local - n_tile * mt);
-        t.n0 = n_tile * t.bn;
-        t.nkb = group_k(p, kGateUp, t.shared) / BK;
-        t.cb = 0;
-        t.t0 = 0;
-        return t;
+    Tile t;
+    const int n_gu = p.has_gu ? tt.prefix[kGateUp][G] : 0;
+    t.ph = tile < n_gu ? kGateUp : kDown;
+    t.kind = t.ph == kGateUp ? kTileGU : kTileDown;
+    const int local_all = tile - (t.ph == kDown ? n_gu : 0);
+    const int *pre = tt.prefix[t.ph];
+    int lo = 0, hi = G - 1;  // last group with prefix <= local_all
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (pre[mid] <= local_all) lo = mid; else hi = mid - 1;
     }
-    const int u = tile - n_gu;
-    const int dn = tt.mpre[G];  // down tiles per column block
-    if (!p.has_comb) return down_tile(p, tt, G, u / dn, u - (u / dn) * dn);
-    if (u < dn) return down_tile(p, tt, G, 0, u);
-    const int u2 = u - dn, round = dn + comb_items(p);
-    if (u2 < (p.nb - 1) * round) {
-        const int r = u2 / round, rem = u2 - r * round;
-        return rem < dn ? down_tile(p, tt, G, r + 1, rem) : comb_tile(r, rem - dn);
-    }
-    return comb_tile(p.nb - 1, u2 - (p.nb - 1) * round);
-}
-
-// Drop a 128-byte line from L2 without writing it back (its data is not read
-// again before it is rewritten).
-__device__ __forceinline__ void discard_l2_line(const void *p)
-{
-    asm volatile("discard.global.L2 [%0], 128;\n" ::"l"(p) : "memory");
-}
-
-__device__ __forceinline__ void add_bf16x8(float *acc, const uint4 &v)
-{
-    const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float2 f = __bfloat1622float2(b[i]);
-        acc[2 * i] += f.x;
-        acc[2 * i + 1] += f.y;
-    }
+    t.bn = p.ph[t.ph].bn;
+    t.g = lo;
+    t.shared = lo >= p.E;
+    const int rows = tt.rows[lo];
+    const int mt = (rows + BM - 1) / BM;
+    const int local = local_all - pre[lo];
+    const int n_tile = local / mt;
+    t.m_tile = local - n_tile * mt;
+    t.m0 = t.m_tile * BM;
+    t.n0 = n_tile * t.bn;
+    t.cb = n_tile;
+    t.rows = min(BM, rows - t.m0);
+    t.row_base = tt.base[lo];
+    t.nkb = group_k(p, t.ph == kGateUp ? kGateUp : kDown, t.shared) / BK;
+    return t;
 }
 
 // ---------------------------------------------------------------- kernel
@@ -310,11 +244,11 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         tt.rows[g] = rows;
         tt.base[g] = base;
         tt.mpre[g + 1] = mt;
-        tt.prefix[g + 1] = mt * (group_n(p, kGateUp, shared) / p.ph[kGateUp].bn);
+        for (int ph = 0; ph < 2; ++ph) tt.prefix[ph][g + 1] = mt * (group_n(p, ph, shared) / p.ph[ph].bn);
     }
     __syncthreads();
-    if (warp < 2) {  // two inclusive scans, one per warp: gate/up tiles, row blocks
-        int *arr = warp == 1 ? tt.mpre : tt.prefix;
+    if (warp < 3) {  // three inclusive scans, one per warp: tiles of each GEMM, row blocks
+        int *arr = warp == 2 ? tt.mpre : tt.prefix[warp];
         int carry = 0;
         for (int b = 0; b < G; b += 32) {
             int v = b + lane < G ? arr[b + lane + 1] : 0;
@@ -353,7 +287,6 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         uint32_t filled = 0, last_parity = 0;  // per-stage bits, for the drain below
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
-            if (t.kind == kTileComb) continue;
             const bool gather = t.kind == kTileGU && !t.shared;
             const int q = t.shared ? 2 : (t.g < p.E_pub ? 0 : 1);
             const int ei = t.shared ? 0 : (q == 0 ? t.g : t.g - p.E_pub);
@@ -427,7 +360,6 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         uint32_t phase = 0;
         for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
-            if (t.kind == kTileComb) continue;
             const uint32_t idesc = p.ph[t.ph].idesc;
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
@@ -469,7 +401,6 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         int it = 0;
         for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
-            if (t.kind == kTileComb) continue;
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
             ++it;
@@ -486,23 +417,17 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             const bool valid = r < t.rows;
             const int grow = t.row_base + t.m0 + r;
             const uint32_t taddr = tmem_base + (uint32_t)(buf * kAccCols) + ((uint32_t)(quarter * 32) << 16);
-            // Whole 32-row blocks go out through shared memory and TMA stores;
-            // the block holding a tile's last rows is written row by row so that
-            // it never touches the next expert's rows.  Down outputs are stored
-            // by column block: row r of block cb at (cb * rows_total + r) * bn.
-            const bool full_block = (t.rows - quarter * 32) >= 32;
-            const int rows_total = t.shared ? p.T : p.R;
-            const int out_row0 = gu ? t.row_base + t.m0 : t.cb * rows_total + t.row_base + t.m0;
-            const int ldc = gu ? (t.shared ? p.E_sh * p.I : p.I) : t.bn;
-            const int col0 = gu ? t.n0 : 0;
-            bf16 *crow = (t.shared ? ph.C_shared : ph.C_routed) + (size_t)(out_row0 + r) * ldc + col0;
-            const CUtensorMap *cmap = t.shared ? &maps.c_shared[t.ph] : &maps.c_routed[t.ph];
-            const int nchunks = gu ? BM / 32 : t.bn / 32;
-            const float sc = (gu || t.shared) ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
+            if (gu) {
+                // Whole 32-row blocks go out through shared memory and TMA
+                // stores; the block holding a tile's last rows is written row
+                // by row so that it never touches the next expert's rows.
+                const bool full_block = (t.rows - quarter * 32) >= 32;
+                const int ldc = t.shared ? p.E_sh * p.I : p.I;
+                bf16 *crow = (t.shared ? ph.C_shared : ph.C_routed) + (size_t)grow * ldc + t.n0;
+                const CUtensorMap *cmap = t.shared ? &maps.c_shared[t.ph] : &maps.c_routed[t.ph];
 #pragma unroll 1
-            for (int c = 0; c < nchunks; ++c) {
-                uint32_t pk[16];
-                if (gu) {
+                for (int c = 0; c < BM / 32; ++c) {
+                    uint32_t pk[16];
                     float gv[32], uv[32];
                     tmem_ld32(taddr + c * 32, gv);
                     tmem_ld32(taddr + 128 + c * 32, uv);
@@ -550,37 +475,115 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                             }
                         }
                     }
-                } else {
+                    if (full_block) {
+                        const uint32_t sbuf = out_base + (uint32_t)(out_parity * kOutBufBytes);
+                        if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+                        __syncwarp();
+                        // 64-byte rows, 16-byte chunk j of row r at chunk j ^ ((r >> 1) & 3): the
+                        // TMA 64-byte swizzle, and conflict-free for these 16-byte writes
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[4 * j]),
+                                         "r"(pk[4 * j + 1]), "r"(pk[4 * j + 2]), "r"(pk[4 * j + 3])
+                                         : "memory");
+                        }
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d_hint(cmap, sbuf, t.n0 + c * 32, t.row_base + t.m0 + quarter * 32, pol_keep);
+                            bulk_commit();
+                        }
+                        out_parity ^= 1;
+                    } else if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                    }
+                }
+            } else {
+                // ---- down: w * (act W_down^T), combined into the output in the
+                // fixed order.  This row's token, its rank among the token's
+                // contributions to this column block (the number of its experts
+                // with a lower id; k for the shared experts), and whether it is
+                // the last contribution.
+                int tok = -1, rank = 0;
+                bool live = false;
+                if (valid) {
+                    if (t.shared) {
+                        tok = grow;  // the shared group's rows are the tokens
+                        rank = p.k;
+                        live = tok < p.T;
+                    } else {
+                        tok = p.tok_of_slot[grow];
+                        if ((unsigned)tok < (unsigned)p.T) {
+                            const int32_t *ti = p.topk_idx + (size_t)tok * p.k;
+                            bool found = false;
+                            for (int j = 0; j < p.k; ++j) {
+                                const int e = ti[j];
+                                rank += e < t.g;
+                                found |= e == t.g;
+                            }
+                            live = found;  // a row whose token does not route here is a dispatch mismatch
+                        }
+                    }
+                }
+                const bool last = t.shared || (rank == p.k - 1 && p.E_sh == 0);
+                const float sc = t.shared ? 1.f : (live ? p.w_of_slot[grow] : 0.f);
+                uint32_t *cnt = live ? p.comb_cnt + (size_t)tok * p.nb + t.cb : nullptr;
+                if (live) {
+                    // the token's contributions of lower rank to this block are in
+                    const unsigned long long w0 = globaltimer_ns();
+                    while (ld_acquire_gpu(cnt) != (uint32_t)rank) {
+                        if (s_abort || globaltimer_ns() - w0 > kWaitLimitNs) {
+                            if (!s_abort && p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
+                            s_abort = 1;
+                            live = false;
+                            break;
+                        }
+                        __nanosleep(64);
+                    }
+                }
+                __syncwarp();
+                float *arow = p.acc + (size_t)(live ? tok : 0) * p.H + t.n0;
+                bf16 *orow = p.out + (size_t)(live ? tok : 0) * p.H + t.n0;
+#pragma unroll 1
+                for (int c = 0; c < t.bn / 32; ++c) {
                     float v[32];
                     tmem_ld32(taddr + c * 32, v);
                     tmem_ld_wait();
+                    if (!live) continue;
+                    float4 *a4 = reinterpret_cast<float4 *>(arow + c * 32);
+                    float acc[32];
+                    if (rank > 0) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(v[2 * i] * sc, v[2 * i + 1] * sc);
+                        for (int i = 0; i < 8; ++i) {
+                            const float4 q = __ldcg(a4 + i);
+                            acc[4 * i] = q.x; acc[4 * i + 1] = q.y; acc[4 * i + 2] = q.z; acc[4 * i + 3] = q.w;
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+                    }
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) acc[i] += v[i] * sc;
+                    if (last) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            dst[i] = make_uint4(pack_bf16x2(acc[8 * i], acc[8 * i + 1]), pack_bf16x2(acc[8 * i + 2], acc[8 * i + 3]),
+                                                pack_bf16x2(acc[8 * i + 4], acc[8 * i + 5]), pack_bf16x2(acc[8 * i + 6], acc[8 * i + 7]));
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            __stcg(a4 + i, make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]));
+                    }
                 }
-                if (full_block) {
-                    const uint32_t sbuf = out_base + (uint32_t)(out_parity * kOutBufBytes);
-                    if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
-                    __syncwarp();
-                    // 64-byte rows, 16-byte chunk j of row r at chunk j ^ ((r >> 1) & 3): the
-                    // TMA 64-byte swizzle, and conflict-free for these 16-byte writes
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[4 * j]),
-                                     "r"(pk[4 * j + 1]), "r"(pk[4 * j + 2]), "r"(pk[4 * j + 3])
-                                     : "memory");
-                    }
-                    fence_proxy_async_smem();
-                    __syncwarp();
-                    if (lane == 0) {
-                        tma_store_2d_hint(cmap, sbuf, col0 + c * 32, out_row0 + quarter * 32, pol_keep);
-                        bulk_commit();
-                    }
-                    out_parity ^= 1;
-                } else if (valid) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+                if (live) {
+                    // this contribution is in: release the next rank
+                    __threadfence();
+                    atomicAdd(cnt, 1u);
                 }
             }
             tc_fence_before();
@@ -610,13 +613,9 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 if (t.shared && p.shared_rows && lane == 0 && vm && (t.n0 % p.I) == 0)
                     atomicAdd(p.shared_rows, (unsigned)__popc(vm));
             }
-            uint32_t *release = nullptr;
-            if (gu && p.has_down) release = p.ready + tt.mpre[t.g] + t.m_tile;
-            if (!gu && p.has_comb) release = p.done_cb + t.cb;
-            if (release) {
-                // release this warp's rows to the tiles that read them (down
-                // tiles: the activations; combine items: this column block of
-                // y): the row stores (generic) and the TMA stores (async
+            if (gu && p.has_down) {
+                // release this warp's activation rows to the down tiles that
+                // read them: the row stores (generic) and the TMA stores (async
                 // proxy, complete after wait_group 0) are ordered before the count
                 __threadfence();
                 __syncwarp();
@@ -624,14 +623,14 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                     bulk_wait_all();
                     asm volatile("fence.proxy.async.global;\n" ::: "memory");
                     __threadfence();
-                    atomicAdd(release, 1u);
+                    atomicAdd(p.ready + tt.mpre[t.g] + t.m_tile, 1u);
                 }
                 __syncwarp();
             }
         }
         if (lane == 0) bulk_wait_all();  // this warp's TMA stores are complete before the CTA exits
     } else if (warp >= 6) {
-        // ------------------------------------------------ A-row gather, combine
+        // ------------------------------------------------ A-row gather
         // Gather: thread i of the 128 copies 16-byte chunk (i & 7) of tile rows
         // (i >> 3) + 16 j, j = 0..7, every stage, into the 128-byte-swizzled A
         // slot of the stage (chunk c of row r at chunk c ^ (r & 7)); a warp
@@ -648,80 +647,6 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         auto drain = [&]() { cp_async_wait<0>(); };
         for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
             const Tile t = decode_tile(p, tt, G, tile);
-            if (t.kind == kTileComb) {
-                // ---- combine item: tokens [t0, t0 + 32) of column block cb,
-                // once every down tile of the block has stored its y
-                const uint32_t need = 4u * (uint32_t)tt.mpre[G];
-                int waited = 1;
-                if (lane == 0) {
-                    const unsigned long long t0 = globaltimer_ns();
-                    while (ld_acquire_gpu(p.done_cb + t.cb) < need) {
-                        if (s_abort || globaltimer_ns() - t0 > kWaitLimitNs) {
-                            if (!s_abort && p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
-                            s_abort = 1;
-                            waited = 0;
-                            break;
-                        }
-                        __nanosleep(256);
-                    }
-                }
-                waited = __shfl_sync(~0u, waited, 0);
-                if (!waited) { ok = false; break; }
-                const int bn = p.ph[kDown].bn, nch = bn / 8, per = 32 / nch;  // chunks per row, tokens per pass
-                const int sub = lane / nch, cc = (lane - sub * nch) * 8;      // this lane's token and columns
-                const bf16 *ycb = p.ph[kDown].C_routed + (size_t)t.cb * p.R * bn;
-                const bf16 *yshcb = p.E_sh > 0 ? p.ph[kDown].C_shared + (size_t)t.cb * p.T * bn : nullptr;
-                const int tw0 = t.t0 + (warp - 6) * (kCombTokens / kGatherWarps);
-                for (int i0 = 0; i0 < kCombTokens / kGatherWarps; i0 += per) {
-                    const int tok = tw0 + i0 + sub;
-                    const bool live = tok < p.T;
-                    const int32_t *slots = p.slot_of + (size_t)(live ? tok : 0) * p.k;
-                    float acc[8];
-#pragma unroll
-                    for (int q2 = 0; q2 < 8; ++q2) acc[q2] = 0.f;
-                    for (int j0 = 0; j0 < p.k; j0 += 8) {
-                        uint4 v[8];
-                        int sl[8];
-#pragma unroll
-                        for (int u = 0; u < 8; ++u) {
-                            sl[u] = -1;
-                            if (live && j0 + u < p.k) {
-                                int slot = __ldg(slots + j0 + u);
-                                if ((unsigned)slot >= (unsigned)p.R) slot = 0;  // only after a dispatch mismatch
-                                sl[u] = slot;
-                                v[u] = *reinterpret_cast<const uint4 *>(ycb + (size_t)slot * bn + cc);
-                            }
-                        }
-#pragma unroll
-                        for (int u = 0; u < 8; ++u)
-                            if (sl[u] >= 0) add_bf16x8(acc, v[u]);
-                        // these rows of y are not read again: drop them from L2
-                        // without a write-back, one lane per 128-byte line, once
-                        // every lane's load of the line has returned
-                        __syncwarp();
-                        if ((cc & 63) == 0) {
-#pragma unroll
-                            for (int u = 0; u < 8; ++u)
-                                if (sl[u] >= 0) discard_l2_line(ycb + (size_t)sl[u] * bn + cc);
-                        }
-                    }
-                    if (yshcb) {
-                        const bf16 *src = yshcb + (size_t)(live ? tok : 0) * bn + cc;
-                        if (live) add_bf16x8(acc, *reinterpret_cast<const uint4 *>(src));
-                        __syncwarp();
-                        if (live && (cc & 63) == 0) discard_l2_line(src);
-                    }
-                    if (live) {
-                        uint4 o;
-                        o.x = pack_bf16x2(acc[0], acc[1]);
-                        o.y = pack_bf16x2(acc[2], acc[3]);
-                        o.z = pack_bf16x2(acc[4], acc[5]);
-                        o.w = pack_bf16x2(acc[6], acc[7]);
-                        *reinterpret_cast<uint4 *>(p.out + (size_t)tok * p.H + t.cb * bn + cc) = o;
-                    }
-                }
-                continue;
-            }
             if (t.kind != kTileGU || t.shared) {  // A comes through TMA: only follow the ring
                 sc += (uint32_t)t.nkb;
                 continue;
@@ -775,9 +700,9 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
 {
     const Shape &s = c.s;
     const uint64_t R = (uint64_t)s.T * s.k, T = (uint64_t)s.T;
-    TcPhase &f = p.ph[mode];
     bool ok = true;
     if (mode == kGateUp) {
+        TcPhase &f = p.ph[mode];
         f.C_routed = c.act;
         f.C_shared = c.act_sh;
         ok &= encode_2d_box(&maps.c_routed[mode], c.act, s.I, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
@@ -795,30 +720,23 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
             ok &= encode_2d(&maps.b1[mode][2], c.up[2], s.H, (uint64_t)s.E_sh * s.I, 128);
         }
     } else {
-        const uint64_t nb = (uint64_t)p.nb;
-        f.C_routed = c.y;
-        f.C_shared = c.y_sh;
-        // y and y_sh by column block: [nb * rows][bn]
-        ok &= encode_2d_box(&maps.c_routed[mode], c.y, f.bn, nb * R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
-        if (s.E_sh > 0)
-            ok &= encode_2d_box(&maps.c_shared[mode], c.y_sh, f.bn, nb * T, kOutBox, kOutBox,
-                                CU_TENSOR_MAP_SWIZZLE_64B);
+        const int bn = p.ph[mode].bn;
         ok &= encode_2d(&maps.a_routed[mode], c.act, s.I, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
-            ok &= encode_2d(&maps.b0[mode][q], c.down[q], s.I, n, f.bn / 2);
+            ok &= encode_2d(&maps.b0[mode][q], c.down[q], s.I, n, bn / 2);
         }
         if (s.E_sh > 0) {
             ok &= encode_2d(&maps.a_shared[mode], c.act_sh, (uint64_t)s.E_sh * s.I, T, BM);
-            ok &= encode_2d(&maps.b0[mode][2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, f.bn / 2);
+            ok &= encode_2d(&maps.b0[mode][2], c.down[2], s.I, (uint64_t)s.E_sh * s.H, bn / 2);
         }
     }
     return ok;
 }
 
-// One persistent launch: the gate/up tiles, the down tiles and the combine
-// items, as selected (the combine items only with the down tiles).
-cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool comb)
+// One persistent launch of the gate/up tiles, the down tiles (which also
+// combine the output), or both.
+cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
 {
     const Shape &s = c.s;
     TcParams p;
@@ -827,7 +745,6 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool comb)
     memset(&maps, 0, sizeof(maps));
     p.has_gu = gu;
     p.has_down = down;
-    p.has_comb = down && comb;
     p.E = s.E(); p.E_pub = s.E_pub; p.E_sh = s.E_sh; p.T = s.T; p.H = s.H; p.I = s.I; p.R = s.T * s.k; p.k = s.k;
     p.ph[kGateUp].bn = 128;
     p.ph[kGateUp].idesc = make_idesc(BM, 256);
@@ -837,11 +754,11 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool comb)
     p.offsets = c.offsets;
     p.w_of_slot = c.w_of_slot;
     p.tok_of_slot = c.tok_of_slot;
-    p.slot_of = c.slot_of;
     p.topk_idx = c.idx;
     p.hidden = c.hidden;
     p.ready = c.gemm_ready;
-    p.done_cb = c.gemm_ready + gemm_ready_blocks(s);
+    p.comb_cnt = c.gemm_ready + gemm_ready_blocks(s);
+    p.acc = c.comb_acc;
     p.out = c.out;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
@@ -867,7 +784,7 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool comb)
 }
 
 // Whether the persistent grid (one CTA per SM) can be resident all at once:
-// its down tiles wait for gate/up tiles and its combine items for down tiles
+// its down tiles wait for gate/up tiles, and its combine for down tiles,
 // that other CTAs own, so every CTA must run concurrently.  Cached per device.
 static bool grid_fits(const Ctx &c)
 {
@@ -887,22 +804,26 @@ static bool grid_fits(const Ctx &c)
 
 }  // namespace
 
-cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, true, false, false); }
-cudaError_t launch_down(const Ctx &c) { return launch_tc(c, false, true, false); }
+cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, true, false); }
 
-cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool with_combine)
+cudaError_t launch_down(const Ctx &c, bool zero_counts)
 {
-    if (!grid_fits(c)) {  // one stage after the other: no cross-CTA wait
-        cudaError_t err = launch_gateup(c);
-        if (err == cudaSuccess) err = launch_down(c);
-        if (err == cudaSuccess && with_combine) err = launch_combine(c);
-        return err;
-    }
-    if (zero_ready) {
+    if (!grid_fits(c)) return cudaErrorCooperativeLaunchTooLarge;
+    if (zero_counts) {
         const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
         if (err != cudaSuccess) return err;
     }
-    return launch_tc(c, true, true, with_combine);
+    return launch_tc(c, false, true);
+}
+
+cudaError_t launch_experts(const Ctx &c, bool zero_counts)
+{
+    if (!grid_fits(c)) return cudaErrorCooperativeLaunchTooLarge;
+    if (zero_counts) {
+        const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
+        if (err != cudaSuccess) return err;
+    }
+    return launch_tc(c, true, true);
 }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()

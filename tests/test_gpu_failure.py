@@ -62,8 +62,9 @@ def test_dispatch_mismatch_is_caught_by_the_execution_audit():
     the route log row by row (Sec. 5.2, App. F.1: counts observed at the
     experts, independent of the router).  A dispatch corrupted on the host --
     a private expert's slot handed to a DENY token, every index still valid --
-    shows up as exec != route for that expert and for both tokens, and as the
-    dispatch-mismatch status bit, which pmpe_audit_read reports."""
+    makes the gate/up tiles run that token's row through the private expert;
+    the audit shows it as exec != route for that expert and for both tokens,
+    and as the dispatch-mismatch status bit, which pmpe_audit_read reports."""
     from paper_2608_06690_gb300 import pmpe
     from paper_2608_06690_gb300.inputs import LayerShape
     s = LayerShape(T=256, H=256, I=128, E_pub=16, E_priv=8, E_sh=0, k=2, renormalize=True)
@@ -87,8 +88,8 @@ def test_dispatch_mismatch_is_caught_by_the_execution_audit():
     t_deny = int(np.nonzero(~tau)[0][0])
     tos[slot] = t_deny                     # host-side corruption of one dispatch entry
     torch.cuda.synchronize()
-    layer.forward(hd, pd, out=out, topk_idx=idx, audit=audit,
-                  stages=pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE)
+    # the gate/up tiles gather the rows named by tok_of_slot and count them
+    layer.forward(hd, pd, out=out, topk_idx=idx, audit=audit, stages=pmpe.STAGE_GATEUP)
     torch.cuda.synchronize()
     with pytest.raises(pmpe.PmpeError) as err:
         pmpe.audit_read(audit, T, E)
