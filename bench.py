@@ -226,11 +226,9 @@ def build_workload(cfg, device, seed_offset=0):
 
 def algorithmic_work(s, counts: np.ndarray):
     """FLOPs of the two grouped GEMMs and the least DRAM bytes of each stage,
-    for one forward with the given per-expert row counts.  "experts" is the
-    forward's persistent launch: gate/up (rows gathered from the hidden
-    states), down and the combine, whose activations and per-row outputs stay
-    inside it; "gateup" and "down" (with the combine) are its two GEMMs run on
-    their own (diagnostics), which pass the activations through memory."""
+    for one forward with the given per-expert row counts.  The gate/up tiles
+    gather their rows from the hidden states (read once from DRAM; the other
+    k - 1 reads of a row hit L2)."""
     R = s.T * s.k
     f_gateup = 2.0 * R * s.H * 2 * s.I + 2.0 * s.T * s.H * 2 * s.E_sh * s.I
     f_down = 2.0 * R * s.I * s.H + 2.0 * s.T * s.E_sh * s.I * s.H
@@ -240,10 +238,10 @@ def algorithmic_work(s, counts: np.ndarray):
     w_gu = (touched + s.E_sh) * 2 * s.I * s.H * 2
     w_dn = (touched + s.E_sh) * s.I * s.H * 2
     act = R * s.I * 2 + s.T * s.E_sh * s.I * 2
-    maps = R * 8                                    # tok_of_slot, w_of_slot
-    b_gateup = w_gu + s.T * s.H * 2 + act + maps
-    b_down = w_dn + act + s.T * s.H * 2 + maps
-    b_experts = gemm_weight_bytes + s.T * s.H * 2 + s.T * s.H * 2 + maps
+    yb = R * s.H * 2 + (s.T * s.H * 2 if s.E_sh else 0)
+    b_gateup = w_gu + s.T * s.H * 2 + act + R * 4
+    b_down = w_dn + act + yb + R * 4
+    b_combine = yb + s.T * s.H * 2 + R * 4
     b_route = s.T * s.H * 2 + (s.E_pub + s.E_priv) * s.H * 2 + s.T * s.k * 8 + s.T
     # the dispatch order: route log and tickets in, slot maps out
     b_permute = R * 12 + R * 12
@@ -252,8 +250,8 @@ def algorithmic_work(s, counts: np.ndarray):
     b_layer_min = gemm_weight_bytes + (s.E_pub + s.E_priv) * s.H * 2 + 2 * s.T * s.H * 2 + s.T * s.k * 8 + s.T
     return dict(flops_gateup=f_gateup, flops_down=f_down, bytes_gateup=b_gateup, bytes_down=b_down,
                 bytes_layer_min=b_layer_min,
-                flops_experts=f_gateup + f_down, bytes_experts=b_experts,
-                bytes_route=b_route, bytes_permute=b_permute,
+                flops_experts=f_gateup + f_down, bytes_experts=b_gateup + b_down,
+                bytes_route=b_route, bytes_permute=b_permute, bytes_combine=b_combine,
                 touched_experts=touched, gemm_weight_bytes=gemm_weight_bytes)
 
 
@@ -430,12 +428,12 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     # is still busy flushing while the host enqueues the stage (no host gap
     # inside the measured interval); stages run in pipeline order on the
     # workspace the previous stage filled.  "experts" is the persistent
-    # gate/up + down + combine launch the forward runs; the gate/up GEMM and
-    # the down GEMM with the combine, launched on their own, are diagnostics.
+    # gate/up + down launch the forward runs; the two GEMMs launched one at a
+    # time are reported as diagnostics.
     stages = [("route", pmpe.STAGE_ROUTE), ("permute", pmpe.STAGE_PERMUTE),
-              ("experts", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE),
-              ("gateup", pmpe.STAGE_GATEUP), ("down", pmpe.STAGE_DOWN | pmpe.STAGE_COMBINE)]
-    pipeline = ("route", "permute", "experts")
+              ("experts", pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN), ("combine", pmpe.STAGE_COMBINE),
+              ("gateup", pmpe.STAGE_GATEUP), ("down", pmpe.STAGE_DOWN)]
+    pipeline = ("route", "permute", "experts", "combine")
     stage_ms = {n: [] for n, _ in stages}
     for _ in range(args.steps):
         evs_s = []

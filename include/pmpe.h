@@ -74,10 +74,8 @@ extern "C" {
 #define PMPE_STAGE_PERMUTE 0x02u /* per-expert dispatch order (slot maps) */
 #define PMPE_STAGE_GATEUP 0x04u  /* grouped gate/up GEMM on rows gathered from hidden, fused silu(g)*u,
                                     execution audit */
-#define PMPE_STAGE_DOWN 0x08u    /* grouped down GEMM, scaled by the routing weight, and the weighted
-                                    unpermute-combine (+ shared experts) of its outputs into `out` */
-#define PMPE_STAGE_COMBINE 0x10u /* the combine: it runs inside PMPE_STAGE_DOWN's launch, so this bit
-                                    adds nothing of its own (kept for the stage order) */
+#define PMPE_STAGE_DOWN 0x08u    /* grouped down GEMM, scaled by the routing weight */
+#define PMPE_STAGE_COMBINE 0x10u /* weighted unpermute-combine (+ shared experts) */
 #define PMPE_STAGE_ALL 0x1Fu
 
 /* ------------------------------------------------------------ layer desc */
@@ -165,17 +163,14 @@ typedef struct pmpe_workspace_layout {
     size_t a_perm;       /* BF16   [T*k, H] token rows in dispatch order, written by the backward calls
                           * (the forward's expert kernel gathers them from `hidden` as it goes) */
     size_t act;          /* BF16   [T*k, I] silu(g)*u of each dispatch row */
-    size_t y;            /* FP32   [T, H]   the combine's partial sums: each token's expert outputs
-                          * (times the routing weights) added in ascending expert id */
+    size_t y;            /* BF16   [T*k, H] w * expert output of each dispatch row */
     size_t act_sh;       /* BF16   [T, E_shared*I] shared-expert activations (0 if none) */
-    size_t y_sh;         /* 0: unused (the shared experts' output goes straight into the combine) */
+    size_t y_sh;         /* BF16   [T, H] summed shared-expert outputs (0 if none) */
     size_t tile_done;    /* uint32 [S]      router CTAs finished per 128-token tile */
     size_t router_lists; /* float2 [C2*128, k] per 32-expert chunk: each token's best k (score, id) */
     size_t router_meta;  /* float4 [C2*128] per chunk: max score, sum exp(score - max), entries */
-    size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1 + T*H/128]  gate/up epilogue warps
-                          * done per (expert group, 128-row block), read by the down tiles of the same
-                          * launch; then, per (token, column block of the output), the contributions
-                          * the combine has added so far */
+    size_t gemm_ready;   /* uint32 [(T*k+127)/128 + E + (T+127)/128 + 1]  gate/up epilogue warps done per
+                          * (expert group, 128-row block), read by the down tiles of the same launch */
     size_t tile_counts;  /* uint32 [E, S4]  rows of expert e in router tile s (S4 = S rounded up to 4).
                           * With the tiles of a pool in ascending token order, slot
                           * offsets[e] + sum_{s' < s} tile_counts[e, s'] + position gives every expert

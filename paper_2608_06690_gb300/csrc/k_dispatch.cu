@@ -1,4 +1,5 @@
-// Stage 2 of the layer, the dispatch order of the routed rows.
+// Stages 2 and 5 of the layer: the dispatch order of the routed rows, and
+// the weighted unpermute-combine.
 //
 // Dispatch (the grouping any grouped expert execution needs): the routed rows
 // are grouped by expert id -- expert e owns slots [offset[e], offset[e+1]) --
@@ -11,6 +12,10 @@
 // from the hidden states itself.  An id outside [0, E) is recorded in the
 // status word.  The backward, which reads the dispatched rows as one matrix,
 // fills it with gather_dispatch_rows_kernel.
+//
+// Combine: out_t = bf16( sum_{j < k} y[slot(t, j)] + y_shared[t] ), summed in
+// FP32 in a fixed order (j ascending, then shared), so the result of a token
+// never depends on the other tokens of the batch.
 #include <algorithm>
 
 #include "pmpe_internal.cuh"
@@ -126,6 +131,71 @@ __global__ void __launch_bounds__(256) gather_dispatch_rows_kernel(const bf16 *h
     }
 }
 
+__device__ __forceinline__ void add_bf16x8(float *acc, const uint4 &v)
+{
+    const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(b[i]);
+        acc[2 * i] += f.x;
+        acc[2 * i + 1] += f.y;
+    }
+}
+
+// Combine: one thread per (token, 16-byte chunk of the output row).  The k
+// routed rows are loaded in batches of 8 independent 16-byte loads before
+// they are summed (in j order), so the loads overlap instead of forming a
+// chain of dependent memory round trips.  Four resident CTAs per SM (at most
+// 64 registers a thread) keep more of those loads in flight.
+__global__ void __launch_bounds__(256, 4) combine_kernel(const bf16 *__restrict__ y, const bf16 *__restrict__ y_sh,
+                                                      const int32_t *__restrict__ slot_of, int T, int H, int k,
+                                                      bf16 *__restrict__ out)
+{
+    pdl_trigger();
+    pdl_wait();
+    const int nv = H / 8;
+    const int R = T * k;
+    const long long total = (long long)T * nv;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int t = (int)(i / nv), c = (int)(i - (long long)t * nv);
+        const int32_t *slots = slot_of + (size_t)t * k;
+        float acc[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+        for (int j0 = 0; j0 < k; j0 += 8) {
+            uint4 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                if (j0 + u < k) {
+                    int slot = __ldg(slots + j0 + u);
+                    if ((unsigned)slot >= (unsigned)R) slot = 0;  // only after a dispatch mismatch (status set)
+                    v[u] = __ldg(reinterpret_cast<const uint4 *>(y + (size_t)slot * H) + c);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                if (j0 + u < k) add_bf16x8(acc, v[u]);
+        }
+        if (y_sh) add_bf16x8(acc, __ldg(reinterpret_cast<const uint4 *>(y_sh + (size_t)t * H) + c));
+        uint4 o;
+        o.x = pack_bf16x2(acc[0], acc[1]);
+        o.y = pack_bf16x2(acc[2], acc[3]);
+        o.z = pack_bf16x2(acc[4], acc[5]);
+        o.w = pack_bf16x2(acc[6], acc[7]);
+        reinterpret_cast<uint4 *>(out + (size_t)t * H)[c] = o;
+    }
+}
+
+// Grid for a grid-stride loop over `work` items of 256-thread blocks: enough
+// blocks to cover the work once, capped at 8 resident blocks per SM.
+int grid_for(long long work, int num_sms)
+{
+    const long long blocks = (work + 255) / 256;
+    const long long cap = 8LL * num_sms;
+    return (int)(blocks < cap ? (blocks > 0 ? blocks : 1) : cap);
+}
+
 }  // namespace
 
 int column_block(int H) { return H % 256 == 0 ? 256 : 128; }
@@ -143,6 +213,14 @@ cudaError_t launch_permute(const Ctx &c)
     p.status = c.audit.status;
     const int grid = std::max(1, std::min((R + kDispThreads - 1) / kDispThreads, 4 * c.num_sms));
     return launch_pdl(dispatch_kernel, dim3(grid), dim3(kDispThreads), 0, c.stream, p);
+}
+
+cudaError_t launch_combine(const Ctx &c)
+{
+    const Shape &s = c.s;
+    return launch_pdl(combine_kernel, dim3(grid_for((long long)s.T * (s.H / 8), c.num_sms)), dim3(256), 0, c.stream,
+                      (const bf16 *)c.y, (const bf16 *)(s.E_sh > 0 ? c.y_sh : nullptr), (const int32_t *)c.slot_of, s.T,
+                      s.H, s.k, c.out);
 }
 
 cudaError_t launch_gather_dispatch_rows(const Ctx &c, int g0, int g1)

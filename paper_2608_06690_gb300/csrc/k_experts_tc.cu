@@ -1,11 +1,9 @@
-// Stages 3 to 5 of the layer on the 5th-generation tensor cores: grouped
+// Stages 3 and 4 of the layer on the 5th-generation tensor cores: grouped
 // BF16 expert GEMMs with tcgen05.mma accumulating in tensor memory (TMEM),
-// operands staged into 128-byte-swizzled shared memory, and the weighted
-// combine of their outputs.
+// operands staged into 128-byte-swizzled shared memory.
 //
 //   gate/up:  act = bf16(silu(A_e W_gate,e^T) * (A_e W_up,e^T))    (SwiGLU fused)
-//   down:     y   = w_row * (act_e W_down,e^T)                       (FP32, never stored)
-//   combine:  out_t = bf16(sum over t's experts in ascending id of y + y_shared[t])
+//   down:     y   = bf16(w_row * (act_e W_down,e^T))
 //
 // Groups are the routed experts (rows of the dispatch order) plus, with
 // shared experts, one dense group over all T tokens (gate/up weights of the
@@ -13,25 +11,18 @@
 // one accumulator).  A persistent grid (one CTA per SM) walks a tile list
 // built on the device from the dispatch offsets: no host sync, and empty
 // experts contribute no tile.  The list holds every gate/up tile, then every
-// down tile, group by group (experts in ascending id, the shared group last),
-// n-tile major inside a group; CTA c takes tiles c, c + grid, ... in order.
+// down tile, group by group, n-tile major inside a group; CTA c takes tiles
+// c, c + grid, ... in order.  A down tile waits (bounded) until the gate/up
+// tiles of its activation rows have stored them.
 //
 // The routed gate/up tiles read their A rows straight from the hidden states:
 // the row of dispatch slot r is hidden[tok_of_slot[r]], gathered into shared
 // memory by four warps with 16-byte cp.async copies (the hidden states, read
 // by every expert a token routes to, stay in L2), so the dispatched rows are
-// never written out.
-//
-// The combine runs in the down epilogue.  Each (token, column block of the
-// output) gets its contributions in ascending expert id -- the order of the
-// down tiles in the list -- then the shared experts': a contribution waits
-// until the token's counter for that block equals its rank, adds its FP32
-// values into an FP32 accumulator row (which stays in L2), and advances the
-// counter; the last one writes the BF16 output row instead.  The order is
-// fixed, so the output is deterministic and does not depend on the other
-// tokens of the batch, and the per-row outputs never go through memory.
-// Every wait is for a tile earlier in the list, and every CTA runs its tiles
-// in list order, so with all CTAs resident every wait ends.
+// never written out.  The gather warps never wait for their own copies: each
+// thread's copies of a stage arrive on the stage's full barrier when they
+// complete (cp.async.mbarrier.arrive), and the MMA thread fences the async
+// proxy after that barrier, before the tensor cores read the rows.
 //
 // CTA roles (320 threads):
 //   warp 0       three lanes issue the TMA loads of a 4-stage ring, one
@@ -44,12 +35,14 @@
 //                of the next) and one thread issues tcgen05.mma M=128 N=256
 //                K=16, committing stage releases and accumulator-full events
 //   warps 2..5   epilogue: tcgen05.ld of the warp's 32 TMEM lanes (= 32 tile
-//                rows); gate/up: SwiGLU, BF16 TMA stores and, in the tiles of
-//                N-tile 0, the execution audit (each row checked against the
-//                route log of its token); down: the routing weight and the
-//                ordered combine
+//                rows), SwiGLU or weight scaling, BF16 stores; in gate/up mode
+//                the tiles of N-tile 0 also write the execution audit, each
+//                row checked against the route log of its token
 //   warps 6..9   the A-row gather of the routed gate/up tiles (cp.async into
 //                the ring)
+// Expert weights stream through L2 once and are loaded with an evict-first
+// policy; the hidden states and activations, read again by other tiles of
+// the launch, with evict-last.
 // Every wait is bounded in time: on expiry the CTA records
 // PMPE_STATUS_PIPELINE_TIMEOUT, stops issuing work, waits (bounded) for its
 // own copies and MMAs in flight, frees its TMEM and exits.
@@ -95,24 +88,18 @@ struct TcPhase {
 };
 
 struct TcParams {
-    // which GEMMs this launch runs: the gate/up tiles, the down tiles (with the combine)
+    // which GEMMs this launch runs: the gate/up tiles, the down tiles
     int has_gu, has_down;
     TcPhase ph[2];    // [kGateUp], [kDown]
     int E, E_pub, E_sh, T, H, I, R, k;
-    int nb;           // column blocks of the output: H / ph[kDown].bn
     const uint32_t *offsets;
     const float *w_of_slot;
     const int32_t *tok_of_slot;
-    const int32_t *topk_idx;  // [T, k] the route log: the execution audit and the combine's ranks
+    const int32_t *topk_idx;  // [T, k] the route log, read back by the execution audit
     const bf16 *hidden;       // the gather source of the routed gate/up tiles
     // has_gu && has_down: per (group, 128-row block), the gate/up epilogue
     // warps whose activations are stored (zeroed before the launch)
     uint32_t *ready;
-    // has_down: per (token, column block), the contributions combined so far
-    // (zeroed before the launch), the FP32 partial sums [T, H] and the output
-    uint32_t *comb_cnt;
-    float *acc;
-    bf16 *out;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
     // optional FP32: the gate and up accumulators saved for the backward,
     // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
@@ -503,87 +490,45 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                     }
                 }
             } else {
-                // ---- down: w * (act W_down^T), combined into the output in the
-                // fixed order.  This row's token, its rank among the token's
-                // contributions to this column block (the number of its experts
-                // with a lower id; k for the shared experts), and whether it is
-                // the last contribution.
-                int tok = -1, rank = 0;
-                bool live = false;
-                if (valid) {
-                    if (t.shared) {
-                        tok = grow;  // the shared group's rows are the tokens
-                        rank = p.k;
-                        live = tok < p.T;
-                    } else {
-                        tok = p.tok_of_slot[grow];
-                        if ((unsigned)tok < (unsigned)p.T) {
-                            const int32_t *ti = p.topk_idx + (size_t)tok * p.k;
-                            bool found = false;
-                            for (int j = 0; j < p.k; ++j) {
-                                const int e = ti[j];
-                                rank += e < t.g;
-                                found |= e == t.g;
-                            }
-                            live = found;  // a row whose token does not route here is a dispatch mismatch
-                        }
-                    }
-                }
-                const bool last = t.shared || (rank == p.k - 1 && p.E_sh == 0);
-                const float sc = t.shared ? 1.f : (live ? p.w_of_slot[grow] : 0.f);
-                uint32_t *cnt = live ? p.comb_cnt + (size_t)tok * p.nb + t.cb : nullptr;
-                if (live) {
-                    // the token's contributions of lower rank to this block are in
-                    const unsigned long long w0 = globaltimer_ns();
-                    while (ld_acquire_gpu(cnt) != (uint32_t)rank) {
-                        if (s_abort || globaltimer_ns() - w0 > kWaitLimitNs) {
-                            if (!s_abort && p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
-                            s_abort = 1;
-                            live = false;
-                            break;
-                        }
-                        __nanosleep(64);
-                    }
-                }
-                __syncwarp();
-                float *arow = p.acc + (size_t)(live ? tok : 0) * p.H + t.n0;
-                bf16 *orow = p.out + (size_t)(live ? tok : 0) * p.H + t.n0;
+                // ---- down: y = w * (act W_down^T), BF16, one row per thread;
+                // whole 32-row blocks through shared memory and TMA stores, a
+                // tile's last partial block row by row
+                const bool full_block = (t.rows - quarter * 32) >= 32;
+                bf16 *crow = (t.shared ? ph.C_shared : ph.C_routed) + (size_t)grow * p.H + t.n0;
+                const CUtensorMap *cmap = t.shared ? &maps.c_shared[t.ph] : &maps.c_routed[t.ph];
+                const float sc = t.shared ? 1.f : (valid ? p.w_of_slot[grow] : 0.f);
 #pragma unroll 1
                 for (int c = 0; c < t.bn / 32; ++c) {
+                    uint32_t pk[16];
                     float v[32];
                     tmem_ld32(taddr + c * 32, v);
                     tmem_ld_wait();
-                    if (!live) continue;
-                    float4 *a4 = reinterpret_cast<float4 *>(arow + c * 32);
-                    float acc[32];
-                    if (rank > 0) {
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const float4 q = __ldcg(a4 + i);
-                            acc[4 * i] = q.x; acc[4 * i + 1] = q.y; acc[4 * i + 2] = q.z; acc[4 * i + 3] = q.w;
+                    for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(v[2 * i] * sc, v[2 * i + 1] * sc);
+                    if (full_block) {
+                        const uint32_t sbuf = out_base + (uint32_t)(out_parity * kOutBufBytes);
+                        if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+                        __syncwarp();
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const uint32_t addr = sbuf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4);
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[4 * j]),
+                                         "r"(pk[4 * j + 1]), "r"(pk[4 * j + 2]), "r"(pk[4 * j + 3])
+                                         : "memory");
                         }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-                    }
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) acc[i] += v[i] * sc;
-                    if (last) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(orow + c * 32);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(cmap, sbuf, t.n0 + c * 32, t.row_base + t.m0 + quarter * 32);
+                            bulk_commit();
+                        }
+                        out_parity ^= 1;
+                    } else if (valid) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(crow + c * 32);
 #pragma unroll
                         for (int i = 0; i < 4; ++i)
-                            dst[i] = make_uint4(pack_bf16x2(acc[8 * i], acc[8 * i + 1]), pack_bf16x2(acc[8 * i + 2], acc[8 * i + 3]),
-                                                pack_bf16x2(acc[8 * i + 4], acc[8 * i + 5]), pack_bf16x2(acc[8 * i + 6], acc[8 * i + 7]));
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            __stcg(a4 + i, make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]));
+                            dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
                     }
-                }
-                if (live) {
-                    // this contribution is in: release the next rank
-                    __threadfence();
-                    atomicAdd(cnt, 1u);
                 }
             }
             tc_fence_before();
@@ -721,6 +666,12 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
         }
     } else {
         const int bn = p.ph[mode].bn;
+        TcPhase &f = p.ph[mode];
+        f.C_routed = c.y;
+        f.C_shared = c.y_sh;
+        ok &= encode_2d_box(&maps.c_routed[mode], c.y, s.H, R, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
+        if (s.E_sh > 0)
+            ok &= encode_2d_box(&maps.c_shared[mode], c.y_sh, s.H, T, kOutBox, kOutBox, CU_TENSOR_MAP_SWIZZLE_64B);
         ok &= encode_2d(&maps.a_routed[mode], c.act, s.I, R, BM);
         for (int q = 0; q < 2; ++q) {
             const uint64_t n = (uint64_t)(q ? s.E_priv : s.E_pub) * s.H;
@@ -734,8 +685,7 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
     return ok;
 }
 
-// One persistent launch of the gate/up tiles, the down tiles (which also
-// combine the output), or both.
+// One persistent launch of the gate/up tiles, the down tiles, or both.
 cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
 {
     const Shape &s = c.s;
@@ -750,16 +700,12 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
     p.ph[kGateUp].idesc = make_idesc(BM, 256);
     p.ph[kDown].bn = column_block(s.H);
     p.ph[kDown].idesc = make_idesc(BM, p.ph[kDown].bn);
-    p.nb = s.H / p.ph[kDown].bn;
     p.offsets = c.offsets;
     p.w_of_slot = c.w_of_slot;
     p.tok_of_slot = c.tok_of_slot;
     p.topk_idx = c.idx;
     p.hidden = c.hidden;
     p.ready = c.gemm_ready;
-    p.comb_cnt = c.gemm_ready + gemm_ready_blocks(s);
-    p.acc = c.comb_acc;
-    p.out = c.out;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
     p.exec_priv_rows = c.audit.exec_priv_rows;
@@ -784,8 +730,8 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
 }
 
 // Whether the persistent grid (one CTA per SM) can be resident all at once:
-// its down tiles wait for gate/up tiles, and its combine for down tiles,
-// that other CTAs own, so every CTA must run concurrently.  Cached per device.
+// the down tiles of the gate/up + down launch wait for gate/up tiles that
+// other CTAs own, so every CTA must run concurrently.  Cached per device.
 static bool grid_fits(const Ctx &c)
 {
     static std::atomic<int> fits[64];  // 0 unknown, 1 yes, 2 no
@@ -806,20 +752,15 @@ static bool grid_fits(const Ctx &c)
 
 cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, true, false); }
 
-cudaError_t launch_down(const Ctx &c, bool zero_counts)
-{
-    if (!grid_fits(c)) return cudaErrorCooperativeLaunchTooLarge;
-    if (zero_counts) {
-        const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
-        if (err != cudaSuccess) return err;
-    }
-    return launch_tc(c, false, true);
-}
+cudaError_t launch_down(const Ctx &c) { return launch_tc(c, false, true); }
 
-cudaError_t launch_experts(const Ctx &c, bool zero_counts)
+cudaError_t launch_experts(const Ctx &c, bool zero_ready)
 {
-    if (!grid_fits(c)) return cudaErrorCooperativeLaunchTooLarge;
-    if (zero_counts) {
+    if (!grid_fits(c)) {  // the two GEMMs one after the other: no cross-CTA wait
+        const cudaError_t err = launch_gateup(c);
+        return err == cudaSuccess ? launch_down(c) : err;
+    }
+    if (zero_ready) {
         const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
         if (err != cudaSuccess) return err;
     }

@@ -12,12 +12,11 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Each routed group adds at most one partial 128-row block beyond R/128; the
 // shared-expert group covers the T tokens.
-size_t gemm_ready_blocks(const Shape &s)
+size_t gemm_ready_words(const Shape &s)
 {
     const size_t R = (size_t)s.T * (size_t)s.k;
     return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 1;
 }
-size_t gemm_ready_words(const Shape &s) { return gemm_ready_blocks(s) + (size_t)s.T * ((size_t)s.H / 128); }
 
 static bool shape_ok(const Shape &s)
 {
@@ -57,9 +56,9 @@ int compute_layout(const Shape &s, pmpe_workspace_layout *L)
     L->router_rows = take(2 * rctas * 128 * (size_t)s.H, 1024);
     L->a_perm = take(2 * R * s.H, 1024);
     L->act = take(2 * R * s.I, 1024);
-    L->y = take(4 * T * s.H, 1024);
+    L->y = take(2 * R * s.H, 1024);
     L->act_sh = s.E_sh > 0 ? take(2 * T * s.E_sh * s.I, 1024) : 0;
-    L->y_sh = 0;
+    L->y_sh = s.E_sh > 0 ? take(2 * T * s.H, 1024) : 0;
     L->total = align_up(o, 1024);
     return PMPE_OK;
 }
@@ -147,8 +146,9 @@ static int make_ctx(const pmpe_moe_desc *d, void *stream, Ctx *c)
     c->router_rows = (bf16 *)(ws + L.router_rows);
     c->a_perm = (bf16 *)(ws + L.a_perm);
     c->act = (bf16 *)(ws + L.act);
-    c->comb_acc = (float *)(ws + L.y);
+    c->y = (bf16 *)(ws + L.y);
     c->act_sh = s.E_sh > 0 ? (bf16 *)(ws + L.act_sh) : nullptr;
+    c->y_sh = s.E_sh > 0 ? (bf16 *)(ws + L.y_sh) : nullptr;
     c->stream = (cudaStream_t)stream;
     c->unmasked = d->unmasked_control;
     c->saved_gu = d->saved_gu;
@@ -215,16 +215,15 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     cudaError_t err = cudaSuccess;
     if (err == cudaSuccess && (stages & PMPE_STAGE_ROUTE)) err = launch_route(c);
     if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE)) err = launch_permute(c);
-    // the combine runs inside the down launch (PMPE_STAGE_COMBINE adds
-    // nothing of its own); the kernel's counters are cleared by the router's
-    // memset when the router runs in this call
-    const bool zero = !(stages & PMPE_STAGE_ROUTE);
     if ((stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN)) {
-        if (err == cudaSuccess) err = launch_experts(c, zero);
+        // one persistent launch; its readiness counters are cleared by the
+        // router's memset when the router runs in this call
+        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_ROUTE));
     } else {
         if (err == cudaSuccess && (stages & PMPE_STAGE_GATEUP)) err = launch_gateup(c);
-        if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c, zero);
+        if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c);
     }
+    if (err == cudaSuccess && (stages & PMPE_STAGE_COMBINE)) err = launch_combine(c);
     return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
 }
 

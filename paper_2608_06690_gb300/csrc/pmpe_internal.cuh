@@ -58,8 +58,7 @@ struct Ctx {
     float4 *router_meta;  // [router CTAs * 128] per-chunk softmax partials
     bf16 *router_rows;  // [router CTAs * 128, H] copied token rows of non-contiguous router tiles
     bf16 *a_perm;  // [T*k, H] dispatched rows: filled only by the backward (the forward gathers on the fly)
-    bf16 *act, *act_sh;
-    float *comb_acc;  // [T, H] FP32 partial sums of the combine
+    bf16 *act, *y, *act_sh, *y_sh;
     cudaStream_t stream;
     int num_sms;
     int unmasked;  // the soft-router control: no hard mask (a negative control, not the method)
@@ -72,20 +71,17 @@ int router_chunks(int pool_size);
 int router_slots(int T);
 // router_slots rounded up to a multiple of 4 (the row pitch of tile_counts).
 int router_slots4(int T);
-// Counters of the persistent expert kernel: one per (group, 128-row block),
-// an upper bound over all routings (gemm_ready_blocks), then the combine's
-// one per (token, column block of the output) (T * H / 128 words at most);
-// gemm_ready_words counts both.
-size_t gemm_ready_blocks(const Shape &s);
+// Readiness counters of the persistent expert GEMMs: one per (group, 128-row
+// block), an upper bound over all routings.
 size_t gemm_ready_words(const Shape &s);
-// Output columns per down tile (a column block of the output): 256 when H allows, else 128.
+// Output columns per down tile: 256 when H allows, else 128.
 int column_block(int H);
 
 // Launchers (one per stage); each returns the launch's cudaError_t.
 cudaError_t launch_route(const Ctx &c);
 cudaError_t launch_permute(const Ctx &c);
 cudaError_t launch_gateup(const Ctx &c);
-cudaError_t launch_down(const Ctx &c, bool zero_counts);
+cudaError_t launch_down(const Ctx &c);
 // Backward of the private branch (k_backward.cu): scratch bytes and launch.
 size_t backward_workspace_bytes(const Shape &s);
 cudaError_t launch_backward_private(const Ctx &c, const bf16 *dout, float *d_router, float *d_gate, float *d_up,
@@ -144,14 +140,11 @@ cudaError_t launch_rows_da(const Ctx &c, const RowsGroups &g, const bf16 *dgu, b
 // all routed experts (`all`) and dout_rows indexed by dispatch slot.
 cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf16 *dgu, const bf16 *wact,
                                   float *d_gate, float *d_up, float *d_down, const RowsGroups *all = nullptr);
-// The expert kernel: gate/up alone, down with the combine (down tiles wait
-// for earlier contributions of their tokens), or both in one persistent
-// launch (down tiles also wait for their activation rows).  zero_counts
-// clears the kernel's counters first (the router's memset clears them when
-// the router runs in the same call).  The down launches need all their CTAs
-// resident at once and return cudaErrorCooperativeLaunchTooLarge when the
-// device cannot host one CTA per SM.
-cudaError_t launch_experts(const Ctx &c, bool zero_counts);
+// Gate/up and down in one persistent launch (down tiles wait for their
+// activation rows); zero_ready clears the readiness counters first.  When the
+// device cannot host one CTA per SM at once, the two GEMMs run as two launches.
+cudaError_t launch_experts(const Ctx &c, bool zero_ready);
+cudaError_t launch_combine(const Ctx &c);
 // The token rows of the dispatch slots of groups g0 .. g1 - 1 copied from the
 // hidden states into the workspace's dispatched-row matrix (a_perm), which the
 // backward's GEMMs read.

@@ -42,10 +42,11 @@ STAGE_COMBINE = 0x10
 STAGE_ALL = 0x1F
 
 # Kernels one full forward launches: router/top-k (with the policy resolve),
-# the dispatch order, and one persistent launch of the gate/up GEMM (rows
-# gathered from the hidden states), the down GEMM and the combine (plus one
-# memset of the per-expert counters, which is not a kernel of this library).
-KERNELS_PER_FORWARD = 3
+# the dispatch order, one persistent launch of the gate/up GEMM (rows
+# gathered from the hidden states) and the down GEMM, and the combine (plus
+# one memset of the per-expert counters, which is not a kernel of this
+# library).
+KERNELS_PER_FORWARD = 4
 # kernels one private-branch backward launches: the dispatched rows of the
 # private experts, dout row gather, the dL/da GEMM, the gate/up recompute GEMM
 # with the SwiGLU backward, router gradient, router weight-gradient partials
