@@ -29,10 +29,12 @@ struct DispatchParams {
     const int32_t *idx;
     const int32_t *ticket;
     const float *w;
-    const uint32_t *counts;
+    uint32_t *counts;             // [E] written: the rows of each expert
     const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
-    int slots4;
+    int slots, slots4;            // router tile slots, and the row pitch of tile_counts
     int T, R, k, E;
+    uint32_t *gemm_ready;         // the expert kernel's readiness counters, cleared here
+    int gemm_ready_words;
     uint32_t *offsets;
     int32_t *slot_of, *tok_of_slot;
     float *w_of_slot;
@@ -66,21 +68,33 @@ __device__ __forceinline__ void resolve_slot(const DispatchParams &p, const uint
     p.w_of_slot[slot] = p.w[r];
 }
 
-// The dispatch order.  Every CTA forms the experts' offsets (exclusive
-// prefix sum of the router's per-expert counts) in shared memory; routed row
+// The dispatch order.  Every CTA forms the experts' row counts (the column
+// sums of tile_counts) and offsets (their exclusive prefix sum) in shared
+// memory; CTA 0 also writes both out and clears the expert kernel's
+// readiness counters, which that kernel reads after this one; routed row
 // r = (t, j) of expert e, in tile s at position q of the tile's rows of e,
 // goes to slot offset[e] + sum_{s' < s} tile_counts[e][s'] + q.  One thread
 // per routed row.
 __global__ void __launch_bounds__(kDispThreads) dispatch_kernel(const DispatchParams p)
 {
     __shared__ uint32_t s_off[2 * kMaxPool + 1];
+    __shared__ uint32_t s_cnt[2 * kMaxPool];
     pdl_trigger();
     pdl_wait();
+    // the rows of each expert: its column sums of tile_counts (every slot's
+    // column is written by the router, zeros included)
+    for (int e = threadIdx.x; e < p.E; e += kDispThreads) {
+        const uint32_t *tc = p.tile_counts + (size_t)e * p.slots4;
+        uint32_t tot = 0;
+        for (int s2 = 0; s2 < p.slots; ++s2) tot += __ldg(tc + s2);
+        s_cnt[e] = tot;
+    }
+    __syncthreads();
     if (threadIdx.x < 32) {
         uint32_t carry = 0;
         const int lane = threadIdx.x;
         for (int b = 0; b < p.E; b += 32) {
-            uint32_t v = b + lane < p.E ? p.counts[b + lane] : 0u;
+            uint32_t v = b + lane < p.E ? s_cnt[b + lane] : 0u;
 #pragma unroll
             for (int off = 1; off < 32; off <<= 1) {
                 const uint32_t y = __shfl_up_sync(~0u, v, off);
@@ -92,8 +106,11 @@ __global__ void __launch_bounds__(kDispThreads) dispatch_kernel(const DispatchPa
         if (lane == 0) s_off[0] = 0;
     }
     __syncthreads();
-    if (blockIdx.x == 0)
+    if (blockIdx.x == 0) {
         for (int e = threadIdx.x; e <= p.E; e += kDispThreads) p.offsets[e] = s_off[e];
+        for (int e = threadIdx.x; e < p.E; e += kDispThreads) p.counts[e] = s_cnt[e];
+        for (int i = threadIdx.x; i < p.gemm_ready_words; i += kDispThreads) p.gemm_ready[i] = 0u;
+    }
     for (int r = blockIdx.x * kDispThreads + threadIdx.x; r < p.R; r += gridDim.x * kDispThreads)
         resolve_slot(p, s_off, r);
 }
@@ -207,7 +224,10 @@ cudaError_t launch_permute(const Ctx &c)
     DispatchParams p;
     p.idx = c.idx; p.ticket = c.ticket; p.w = c.w; p.counts = c.counts;
     p.tile_counts = c.tile_counts;
+    p.slots = router_slots(c.s.T);
     p.slots4 = router_slots4(c.s.T);
+    p.gemm_ready = c.gemm_ready;
+    p.gemm_ready_words = (int)gemm_ready_words(s);
     p.T = s.T; p.R = R; p.k = s.k; p.E = s.E();
     p.offsets = c.offsets; p.slot_of = c.slot_of; p.tok_of_slot = c.tok_of_slot; p.w_of_slot = c.w_of_slot;
     p.status = c.audit.status;

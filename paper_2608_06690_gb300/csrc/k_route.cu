@@ -566,6 +566,458 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
     }
 }
 
+// ---------------------------------------------------------------------------
+// router_cluster_kernel: the same routing with the reduction over H split
+// across a cluster of nq CTAs (nq = 4, or 2 when H is not a multiple of 256)
+// and no cross-CTA traffic through global memory.
+//
+// Each cluster takes one pool-homogeneous 128-token tile (the tile assignment
+// of router_tc_kernel).  CTA q of the cluster multiplies the tile's token rows
+// by the pool's router over the q-th 1/nq of H: tcgen05.mma with the router
+// rows as M (128 experts per MMA, one or two MMAs for pools up to 256; rows
+// past the pool read as zeros) and the 128 tokens as N, so the CTA reads
+// H/nq of each token row and of each router row.  The partial logits go from
+// tensor memory to shared memory; after a cluster barrier, CTA q owns the
+// tokens [q 128/nq, (q+1) 128/nq) of the tile and sums their partial logits
+// over the nq CTAs in CTA order (distributed shared memory), masks, selects
+// the top-k in 32-expert chunks and merges the chunk lists per token.  The
+// rank of each row among the tile's rows of its expert comes from the tile's
+// 128-bit token mask per expert, whose words the CTAs of the cluster exchange
+// after a second cluster barrier.  CTA 0 writes the tile's column of
+// tile_counts for every expert (zero for the other pool), so nothing has to
+// be cleared before the launch; a cluster whose slot holds no tile writes
+// zeros there.  The dispatch sums the columns into the per-expert counts.
+//
+// Every CTA of a cluster reaches every cluster barrier: the waits before them
+// are bounded, and a CTA that gave up skips work, not barriers.
+constexpr int kCThreads = 192;       // warp 0 TMA, warp 1 TMEM + MMA, warps 2..5 gather / epilogue / finalize
+constexpr int kCTile = 128;          // tokens per tile (MMA N)
+constexpr int kCRingBytes = 192 * 1024;
+constexpr int kCMaxStages = 6;
+constexpr int kCMaxChunks = kMaxPool / kChunk;  // 32-expert chunks of one pool
+
+struct ClusterRouterParams {
+    int T, H, E_pub, E_priv, k, renorm;
+    int nq;              // CTAs per cluster: H is split into nq ranges
+    int slots4;
+    uint32_t idesc;      // M = 128, N = 128
+    const uint8_t *policy;
+    const bf16 *hidden;
+    uint8_t *tau;
+    int32_t *idx;
+    float *w;
+    int32_t *ticket;     // [T, k] 128 * tile slot + position among the tile's rows of its expert
+    uint32_t *tile_counts;  // [E][slots4] rows of each expert per tile (a column per tile slot)
+    uint32_t *route_count, *route_priv_rows, *status;
+};
+
+struct ClusterRouterMaps {
+    CUtensorMap hidden;     // [T, H], box 64 x 128 (tiles of consecutive tokens)
+    CUtensorMap router[2];  // [E_pool, H], box 64 x 128
+};
+
+// Shared-memory bytes of router_cluster_kernel for a pool of P experts (the
+// larger pool), top-k k and nq CTAs per cluster: the ring, and after it the
+// partial logits [128][P rounded to 128 + 4] FP32 with the chunk lists.
+static int cluster_router_smem(int P, int k, int nq)
+{
+    const int pp = (P + 127) / 128 * 128;
+    const int tpc = kCTile / nq;
+    const int nc = (P + kChunk - 1) / kChunk;
+    const int partial = kCTile * (pp + 4) * 4;
+    const int lists = tpc * nc * k * 8 + tpc * nc * 16;
+    const int after = partial + lists;
+    return (after > kCRingBytes ? after : kCRingBytes) + 1024;
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync_all()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ uint32_t dsmem_addr(uint32_t local, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(local), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ float4 dsmem_ld_f4(uint32_t addr)
+{
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];\n"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
+}
+__device__ __forceinline__ uint32_t dsmem_ld_u32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];\n" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+
+__global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const ClusterRouterParams p,
+                                                                       const __grid_constant__ ClusterRouterMaps maps)
+{
+    extern __shared__ uint8_t dsmem[];
+    __shared__ int s_tok[kCTile];
+    __shared__ int warp_tot[kCThreads / 32];
+    __shared__ __align__(8) uint64_t bars[2 * kCMaxStages + 2];
+    __shared__ uint32_t s_tmem;
+    __shared__ volatile int s_abort;
+    __shared__ uint32_t smask[kMaxPool * 4];  // this CTA's tokens of the tile, per pool expert, 4 x 32 bits
+    __shared__ uint32_t sfull[kMaxPool * 4];  // the whole tile's mask (OR over the cluster)
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int q = (int)cluster_ctarank();
+    const int slot = blockIdx.x / p.nq;
+    pdl_trigger();
+    pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
+
+    // ---- tile assignment (as router_tc_kernel): resolve and rank in one pass
+    const int per = ((p.T + kCThreads - 1) / kCThreads + 15) & ~15;
+    const int t0 = min(p.T, tid * per), t1 = min(p.T, t0 + per);
+    const int a = count_allow(p.policy, t0, t1);
+    int na;
+    const int a_before = block_scan(a, warp_tot, na);
+    const int nd = p.T - na;
+    const int tiles_d = (nd + kCTile - 1) / kCTile;
+    int pool, m0;
+    bool has_tile = true;
+    if (slot < tiles_d) {
+        pool = 0;
+        m0 = slot * kCTile;
+    } else {
+        pool = 1;
+        m0 = (slot - tiles_d) * kCTile;
+        has_tile = m0 < na;
+    }
+    const int E = p.E_pub + p.E_priv;
+    if (!has_tile) {  // uniform over the cluster: no tile for this slot
+        if (q == 0)
+            for (int e = tid; e < E; e += kCThreads) p.tile_counts[(size_t)e * p.slots4 + slot] = 0u;
+        return;
+    }
+    const int rows = min(kCTile, (pool ? na : nd) - m0);
+    if ((pool ? a_before : t0 - a_before) < m0 + rows && (pool ? a_before + a : t1 - a_before - a) > m0) {
+        int ra = a_before, rd = t0 - a_before;
+        for (int t = t0; t < t1; ++t) {
+            const bool al = is_allow(p.policy, t);
+            const int rank = al ? ra++ : rd++;
+            if ((al ? 1 : 0) == pool && rank >= m0 && rank < m0 + rows) s_tok[rank - m0] = t;
+        }
+    }
+    __syncthreads();
+    for (int r = rows + tid; r < kCTile; r += kCThreads) s_tok[r] = s_tok[0];
+    const int contiguous = __syncthreads_and(tid >= rows || s_tok[tid < kCTile ? tid : 0] == s_tok[0] + tid);
+
+    const int P = pool ? p.E_priv : p.E_pub;
+    const int base = pool ? p.E_pub : 0;
+    const int nm = (P + 127) / 128;                 // MMAs of 128 experts
+    const int pp = nm * 128;
+    const int nc = (P + kChunk - 1) / kChunk;       // 32-expert chunks
+    const int kq = p.H / p.nq, k0 = q * kq, nkb = kq / 64;
+    const uint32_t a_bytes = (uint32_t)nm * 16384u, stage_bytes = a_bytes + 16384u;
+    const int stages = min(kCMaxStages, kCRingBytes / (int)stage_bytes);
+    const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
+    uint8_t *sgen = dsmem + (sbase - smem_u32(dsmem));
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int st) { return bar0 + 8u * st; };
+    auto empty_bar = [&](int st) { return bar0 + 8u * (kCMaxStages + st); };
+    const uint32_t tfull_bar = bar0 + 8u * (2 * kCMaxStages);
+    const uint32_t done_bar = bar0 + 8u * (2 * kCMaxStages + 1);
+    if (tid == 0) {
+        for (int st = 0; st < stages; ++st) {
+            mbar_init(full_bar(st), contiguous ? 1 : 1 + 128);
+            mbar_init(empty_bar(st), 1);
+        }
+        mbar_init(tfull_bar, 1);
+        mbar_init(done_bar, 1);
+        s_abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    for (int i = tid; i < kMaxPool * 4; i += kCThreads) smask[i] = 0u;
+    if (warp == 1) tmem_alloc(smem_u32(&s_tmem), 256);
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---- TMA: the router rows of this CTA's range of H (and the token
+            // rows, when the tile's tokens are consecutive)
+            const uint32_t tx = a_bytes + (contiguous ? 16384u : 0u);
+            uint32_t filled = 0, last_parity = 0;
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int st = kb % stages;
+                const uint32_t ph = (uint32_t)(kb / stages) & 1u;
+                if (!mbar_wait(empty_bar(st), ph ^ 1u, &s_abort, p.status)) break;
+                const uint32_t sA = sbase + st * stage_bytes, sB = sA + a_bytes;
+                mbar_expect_tx(full_bar(st), tx);
+                for (int mi = 0; mi < nm; ++mi)
+                    tma_load_2d(sA + mi * 16384u, &maps.router[pool], full_bar(st), k0 + kb * 64, mi * 128);
+                if (contiguous) tma_load_2d(sB, &maps.hidden, full_bar(st), k0 + kb * 64, s_tok[0]);
+                filled |= 1u << st;
+                last_parity = (last_parity & ~(1u << st)) | (ph << st);
+            }
+            for (int st = 0; st < stages; ++st)
+                if ((filled >> st) & 1u) {
+                    const unsigned long long w0 = globaltimer_ns();
+                    while (!mbar_try_wait(full_bar(st), (last_parity >> st) & 1u))
+                        if (globaltimer_ns() - w0 > kWaitLimitNs) break;
+                }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---- MMA: logits[128 experts, 128 tokens] += router x rows^T per stage
+            bool ok = true;
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int st = kb % stages;
+                const uint32_t ph = (uint32_t)(kb / stages) & 1u;
+                if (!mbar_wait(full_bar(st), ph, &s_abort, p.status)) { ok = false; break; }
+                tc_fence_after();
+                fence_proxy_async_smem();  // gathered rows (generic proxy) read by the tensor cores
+                const uint32_t sA = sbase + st * stage_bytes, sB = sA + a_bytes;
+                const uint64_t bd = sw128_desc(sB);
+                for (int mi = 0; mi < nm; ++mi) {
+                    const uint64_t ad = sw128_desc(sA + mi * 16384u);
+#pragma unroll
+                    for (int k4 = 0; k4 < 4; ++k4)
+                        tc_mma(tmem + (uint32_t)(mi * 128), ad + 2 * k4, bd + 2 * k4, p.idesc, (kb | k4) != 0);
+                }
+                tc_commit(empty_bar(st));
+            }
+            if (ok) tc_commit(tfull_bar);
+            tc_commit(done_bar);
+            const unsigned long long w0 = globaltimer_ns();
+            while (!mbar_try_wait(done_bar, 0))
+                if (globaltimer_ns() - w0 > kWaitLimitNs) break;
+        }
+    } else {
+        // ---- gather (tiles of non-consecutive tokens): thread gi copies 16-byte
+        // chunk (gi & 7) of tile rows (gi >> 3) + 16 j, swizzled as TMA would
+        const int gi = tid - 64;
+        if (!contiguous) {
+            const int chunk = gi & 7, row0 = gi >> 3;
+            const bf16 *src[8];
+            uint32_t nbytes[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int r = row0 + 16 * j;
+                const bool in = r < rows;
+                src[j] = p.hidden + (in ? (size_t)s_tok[r] * p.H : 0) + k0 + chunk * 8;
+                nbytes[j] = in ? 16u : 0u;
+            }
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int st = kb % stages;
+                const uint32_t ph = (uint32_t)(kb / stages) & 1u;
+                int free_ = 1;
+                if (lane == 0) free_ = mbar_wait(empty_bar(st), ph ^ 1u, &s_abort, p.status) ? 1 : 0;
+                free_ = __shfl_sync(~0u, free_, 0);
+                if (!free_) break;
+                const uint32_t sB = sbase + st * stage_bytes + a_bytes;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const int r = row0 + 16 * j;
+                    cp_async16(sB + r * 128 + ((chunk ^ (r & 7)) << 4), src[j] + kb * 64, (int)nbytes[j]);
+                }
+                cp_async_arrive_noinc(full_bar(st));
+            }
+            cp_async_wait<0>();
+        }
+        // ---- epilogue: partial logits to shared memory, [token][expert] FP32
+        // (the ring is free once every MMA has completed)
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait(tfull_bar, 0, &s_abort, p.status) ? 1 : 0;
+        ok = __shfl_sync(~0u, ok, 0);
+        if (ok) {
+            __syncwarp();
+            tc_fence_after();
+            const int quarter = warp & 3;
+            float *S = reinterpret_cast<float *>(sgen);
+            const int pitch = pp + 4;
+            for (int mi = 0; mi < nm; ++mi) {
+                const int e = mi * 128 + quarter * 32 + lane;
+                for (int cc = 0; cc < kCTile / 32; ++cc) {
+                    float v[32];
+                    tmem_ld32(tmem + (uint32_t)(mi * 128 + cc * 32) + ((uint32_t)(quarter * 32) << 16), v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) S[(cc * 32 + i) * pitch + e] = v[i];
+                }
+            }
+        }
+    }
+    __syncwarp();
+    tc_fence_before();
+    cluster_sync_all();  // #1: every CTA's partial logits are in its shared memory
+
+    // ---- finalize this CTA's tokens: sum the partials over the cluster in CTA
+    // order, top-k per 32-expert chunk, then the merge per token
+    const int tpc = kCTile / p.nq;
+    const int ntok = max(0, min(rows - q * tpc, tpc));
+    const int K = p.k;
+    const int pitch = pp + 4;
+    float *lv = reinterpret_cast<float *>(sgen + (size_t)kCTile * pitch * 4);  // [tpc][nc][K] scores
+    int *le = reinterpret_cast<int *>(lv + (size_t)tpc * nc * K);               // [tpc][nc][K] ids
+    float4 *lmeta = reinterpret_cast<float4 *>(le + (size_t)tpc * nc * K);       // [tpc][nc]
+    const uint32_t S_local = sbase;
+    if (warp >= 2 && !s_abort) {
+        for (int pi = tid - 64; pi < ntok * nc; pi += 128) {
+            const int tl = pi / nc, c = pi - tl * nc;
+            const int tt = q * tpc + tl;  // token index inside the tile
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+            const uint32_t off = (uint32_t)((tt * pitch + c * 32) * 4);
+            for (int qq = 0; qq < p.nq; ++qq) {  // fixed order: deterministic
+                const uint32_t ra = dsmem_addr(S_local + off, (uint32_t)qq);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float4 x = dsmem_ld_f4(ra + 16u * i);
+                    v[4 * i] += x.x; v[4 * i + 1] += x.y; v[4 * i + 2] += x.z; v[4 * i + 3] += x.w;
+                }
+            }
+            const int nvalid = min(kChunk, P - c * kChunk);
+            int e[32];
+            float mx = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                float x = v[i];
+                if (x != x) x = -INFINITY;  // NaN never outranks a number
+                const bool in_pool = i < nvalid;
+                v[i] = in_pool ? x : -INFINITY;
+                e[i] = in_pool ? c * kChunk + i : 0x7fffffff;
+                mx = in_pool ? fmaxf(mx, x) : mx;
+            }
+            float ssum = 0.f;
+            if (!p.renorm) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (i < nvalid) ssum += expf(v[i] - mx);
+            }
+            const int cnt = min(K, nvalid);
+            float *dv = lv + ((size_t)tl * nc + c) * K;
+            int *de = le + ((size_t)tl * nc + c) * K;
+            if (K <= 8) {
+                uint32_t taken = nvalid >= 32 ? 0u : ~((1u << nvalid) - 1u);
+                for (int j = 0; j < cnt; ++j) {
+                    float bv;
+                    int be;
+                    const int bi = best_untaken(v, e, taken, bv, be);
+                    taken |= 1u << bi;
+                    dv[j] = bv;
+                    de[j] = be;
+                }
+            } else {
+                sort32(v, e);
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j < cnt) {
+                        dv[j] = v[j];
+                        de[j] = e[j];
+                    }
+            }
+            lmeta[tl * nc + c] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
+        }
+    }
+    __syncthreads();
+    // merge the chunk lists of token tl in chunk order (one thread per token)
+    float sel_v[kMaxTopK];
+    int sel_e[kMaxTopK];
+    float top = 0.f, Ssum = 0.f;
+    const int tl = tid;
+    const bool mine = tl < ntok && !s_abort;
+    if (mine) {
+        int head[kCMaxChunks], n[kCMaxChunks];
+#pragma unroll
+        for (int u = 0; u < kCMaxChunks; ++u) {
+            head[u] = 0;
+            n[u] = u < nc ? __float_as_int(lmeta[tl * nc + u].z) : 0;
+        }
+        for (int j = 0; j < K; ++j) {
+            int bu = -1, be = 0;
+            float bv = 0.f;
+#pragma unroll
+            for (int u = 0; u < kCMaxChunks; ++u) {
+                if (head[u] < n[u]) {
+                    const size_t o = ((size_t)tl * nc + u) * K + head[u];
+                    const float x = lv[o];
+                    const int ee = le[o];
+                    if (bu < 0 || ranks_above(x, ee, bv, be)) { bu = u; bv = x; be = ee; }
+                }
+            }
+            if (bu < 0) break;  // unreachable for k <= pool size
+#pragma unroll
+            for (int u = 0; u < kCMaxChunks; ++u) head[u] += (u == bu) ? 1 : 0;
+            sel_v[j] = bv;
+            sel_e[j] = be;
+            if (j == 0) top = bv;
+            const int tt = q * tpc + tl;
+            atomicOr(&smask[be * 4 + (tt >> 5)], 1u << (tt & 31));
+        }
+        if (p.renorm) {
+            for (int j = 0; j < K; ++j) Ssum += expf(sel_v[j] - top);
+        } else {
+            for (int u = 0; u < nc; ++u) {  // fixed order: deterministic
+                const float4 m = lmeta[tl * nc + u];
+                if (__float_as_int(m.z) > 0) Ssum += m.y * expf(m.x - top);
+            }
+        }
+    }
+    __syncthreads();
+    cluster_sync_all();  // #2: every CTA's token masks are in its shared memory
+
+    // ---- the tile's mask per expert (OR over the cluster), its counts, and
+    // each row's position among the tile's rows of its expert (token order)
+    for (int i = tid; i < P * 4; i += kCThreads) {
+        uint32_t m = 0u;
+        for (int qq = 0; qq < p.nq; ++qq) m |= dsmem_ld_u32(dsmem_addr(smem_u32(&smask[i]), (uint32_t)qq));
+        sfull[i] = m;
+    }
+    __syncthreads();
+    if (q == 0) {
+        for (int eg = tid; eg < E; eg += kCThreads) {
+            const int i = eg - base;
+            uint32_t c = 0u;
+            if (i >= 0 && i < P)
+                c = __popc(sfull[i * 4]) + __popc(sfull[i * 4 + 1]) + __popc(sfull[i * 4 + 2]) + __popc(sfull[i * 4 + 3]);
+            p.tile_counts[(size_t)eg * p.slots4 + slot] = c;
+            if (c && p.route_count) atomicAdd(&p.route_count[eg], c);
+        }
+    }
+    if (mine) {
+        const int tt = q * tpc + tl;
+        const int t = s_tok[tt];
+        const int wd = tt >> 5;
+        const uint32_t below = (1u << (tt & 31)) - 1u;
+        for (int j = 0; j < K; ++j) {
+            const int be = sel_e[j];
+            int rank = (int)__popc(sfull[be * 4 + wd] & below);
+            for (int w2 = 0; w2 < wd; ++w2) rank += (int)__popc(sfull[be * 4 + w2]);
+            p.idx[(size_t)t * K + j] = base + be;
+            p.ticket[(size_t)t * K + j] = (int32_t)(slot * kCTile + rank);
+            p.w[(size_t)t * K + j] = expf(sel_v[j] - top) / Ssum;
+        }
+        p.tau[t] = pool ? 1 : 0;
+        if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], pool ? (unsigned)K : 0u);
+    }
+    __syncthreads();
+    cluster_sync_all();  // #3: no CTA leaves while another still reads its shared memory
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 256);
+    }
+}
+
 // Per-request policy bytes to per-token bytes, in one CTA: the offsets are
 // checked first (cu[0] == 0, non-decreasing, cu[n] <= T); any violation is
 // malformed metadata and every token becomes DENY.  Otherwise token t takes
@@ -606,7 +1058,10 @@ int router_chunks(int pool_size) { return (pool_size + kChunk - 1) / kChunk; }
 int router_slots(int T) { return (T + kTileRows - 1) / kTileRows + 1; }
 int router_slots4(int T) { return (router_slots(T) + 3) & ~3; }
 
-cudaError_t launch_route(const Ctx &c)
+// The router of the unmasked control, and of shapes whose merge scratch does
+// not fit router_cluster_kernel: one CTA per (tile, 32-expert chunk), the
+// chunk lists merged by the tile's last CTA through global memory.
+static cudaError_t launch_route_chunked(const Ctx &c)
 {
     const Shape &s = c.s;
     RouterParams p;
@@ -668,6 +1123,66 @@ cudaError_t launch_route(const Ctx &c)
     cudaError_t err = ensure_dynamic_smem(router_tc_kernel, smem, smem_limit);
     if (err != cudaSuccess) return err;
     return launch_pdl(router_tc_kernel, dim3(grid), dim3(kRThreads), smem, c.stream, p, maps);
+}
+
+// CTAs per cluster of router_cluster_kernel for hidden size H.
+static int cluster_router_nq(int H) { return H % 256 == 0 ? 4 : 2; }
+// Dynamic shared memory the cluster router may take beside its static arrays.
+constexpr int kCMaxDynSmem = 208 * 1024;
+
+bool route_uses_cluster_kernel(const Shape &s, int unmasked)
+{
+    if (unmasked) return false;
+    const int P = s.E_pub > s.E_priv ? s.E_pub : s.E_priv;
+    return cluster_router_smem(P, s.k, cluster_router_nq(s.H)) <= kCMaxDynSmem;
+}
+
+cudaError_t launch_route(const Ctx &c)
+{
+    const Shape &s = c.s;
+    if (!route_uses_cluster_kernel(s, c.unmasked)) return launch_route_chunked(c);
+    ClusterRouterParams p;
+    ClusterRouterMaps maps;
+    memset(&p, 0, sizeof(p));
+    memset(&maps, 0, sizeof(maps));
+    p.T = s.T; p.H = s.H; p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.k = s.k; p.renorm = s.renorm;
+    p.nq = cluster_router_nq(s.H);
+    p.slots4 = router_slots4(s.T);
+    p.idesc = make_idesc(128, kCTile);
+    p.policy = c.policy;
+    p.hidden = c.hidden;
+    p.tau = c.tau;
+    p.idx = c.idx;
+    p.w = c.w;
+    p.ticket = c.ticket;
+    p.tile_counts = c.tile_counts;
+    p.route_count = c.audit.route_count;
+    p.route_priv_rows = c.audit.route_priv_rows;
+    p.status = c.audit.status;
+    bool ok = encode_2d(&maps.hidden, c.hidden, s.H, s.T, kCTile);
+    ok &= encode_2d(&maps.router[0], c.router_pub, s.H, s.E_pub, 128);
+    ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, 128);
+    if (!ok) return cudaErrorInvalidValue;
+    const int P = s.E_pub > s.E_priv ? s.E_pub : s.E_priv;
+    const int smem = cluster_router_smem(P, s.k, p.nq);
+    static std::atomic<int> smem_limit[64];
+    cudaError_t err = ensure_dynamic_smem(router_cluster_kernel, smem, smem_limit);
+    if (err != cudaSuccess) return err;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(router_slots(s.T) * p.nq);
+    cfg.blockDim = dim3(kCThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = c.stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = p.nq;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, router_cluster_kernel, p, maps);
 }
 
 cudaError_t launch_policy_from_requests(const uint8_t *req_policy, const int32_t *cu_seqlens, int n_req, int T,

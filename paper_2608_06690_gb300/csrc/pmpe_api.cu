@@ -217,8 +217,8 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE)) err = launch_permute(c);
     if ((stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN)) {
         // one persistent launch; its readiness counters are cleared by the
-        // router's memset when the router runs in this call
-        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_ROUTE));
+        // dispatch when the dispatch runs in this call
+        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_PERMUTE));
     } else {
         if (err == cudaSuccess && (stages & PMPE_STAGE_GATEUP)) err = launch_gateup(c);
         if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c);
