@@ -568,8 +568,9 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
 
 // ---------------------------------------------------------------------------
 // router_cluster_kernel: the same routing with the reduction over H split
-// across a cluster of nq CTAs (nq = 4, or 2 when H is not a multiple of 256)
-// and no cross-CTA traffic through global memory.
+// across a cluster of nq CTAs (4, or 2 when H is not a multiple of 256, or 8
+// for batches small enough to fit the GPU in clusters of 8) and no cross-CTA
+// traffic through global memory.
 //
 // Each cluster takes one pool-homogeneous 128-token tile (the tile assignment
 // of router_tc_kernel).  CTA q of the cluster multiplies the tile's token rows
@@ -651,14 +652,13 @@ __device__ __forceinline__ float4 dsmem_ld_f4(uint32_t addr)
     float4 v;
     asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];\n"
                  : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(addr)
-                 : "memory");
+                 : "r"(addr));
     return v;
 }
 __device__ __forceinline__ uint32_t dsmem_ld_u32(uint32_t addr)
 {
     uint32_t v;
-    asm volatile("ld.shared::cluster.u32 %0, [%1];\n" : "=r"(v) : "r"(addr) : "memory");
+    asm volatile("ld.shared::cluster.u32 %0, [%1];\n" : "=r"(v) : "r"(addr));
     return v;
 }
 
@@ -878,12 +878,29 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = 0.f;
             const uint32_t off = (uint32_t)((tt * pitch + c * 32) * 4);
-            for (int qq = 0; qq < p.nq; ++qq) {  // fixed order: deterministic
-                const uint32_t ra = dsmem_addr(S_local + off, (uint32_t)qq);
+            // every CTA's partials of these 32 logits, half a chunk at a time:
+            // all loads of a half are issued before any is used, then summed
+            // in CTA order (fixed: deterministic)
+            for (int q0 = 0; q0 < p.nq; q0 += 4) {
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const float4 x = dsmem_ld_f4(ra + 16u * i);
-                    v[4 * i] += x.x; v[4 * i + 1] += x.y; v[4 * i + 2] += x.z; v[4 * i + 3] += x.w;
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    float4 x[4][4];
+#pragma unroll
+                    for (int qq = 0; qq < 4; ++qq)
+                        if (q0 + qq < p.nq) {
+                            const uint32_t ra = dsmem_addr(S_local + off + 64u * h2, (uint32_t)(q0 + qq));
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) x[qq][i] = dsmem_ld_f4(ra + 16u * i);
+                        }
+#pragma unroll
+                    for (int qq = 0; qq < 4; ++qq)
+                        if (q0 + qq < p.nq) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                float *d = v + 16 * h2 + 4 * i;
+                                d[0] += x[qq][i].x; d[1] += x[qq][i].y; d[2] += x[qq][i].z; d[3] += x[qq][i].w;
+                            }
+                        }
                 }
             }
             const int nvalid = min(kChunk, P - c * kChunk);
@@ -978,10 +995,23 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
 
     // ---- the tile's mask per expert (OR over the cluster), its counts, and
     // each row's position among the tile's rows of its expert (token order)
-    for (int i = tid; i < P * 4; i += kCThreads) {
-        uint32_t m = 0u;
-        for (int qq = 0; qq < p.nq; ++qq) m |= dsmem_ld_u32(dsmem_addr(smem_u32(&smask[i]), (uint32_t)qq));
-        sfull[i] = m;
+    for (int i0 = tid; i0 < P * 4; i0 += 2 * kCThreads) {  // up to 16 remote loads in flight per thread
+        uint32_t m[2][8];
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+#pragma unroll
+            for (int qq = 0; qq < 8; ++qq)
+                m[u][qq] = (qq < p.nq && i0 + u * kCThreads < P * 4)
+                               ? dsmem_ld_u32(dsmem_addr(smem_u32(&smask[i0 + u * kCThreads]), (uint32_t)qq))
+                               : 0u;
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+            if (i0 + u * kCThreads < P * 4) {
+                uint32_t o = 0u;
+#pragma unroll
+                for (int qq = 0; qq < 8; ++qq) o |= m[u][qq];
+                sfull[i0 + u * kCThreads] = o;
+            }
     }
     __syncthreads();
     if (q == 0) {
@@ -1125,28 +1155,35 @@ static cudaError_t launch_route_chunked(const Ctx &c)
     return launch_pdl(router_tc_kernel, dim3(grid), dim3(kRThreads), smem, c.stream, p, maps);
 }
 
-// CTAs per cluster of router_cluster_kernel for hidden size H.
-static int cluster_router_nq(int H) { return H % 256 == 0 ? 4 : 2; }
+// CTAs per cluster of router_cluster_kernel for hidden size H and T tokens:
+// 4 (2 when H is not a multiple of 256), and 8 when H allows and the
+// clusters of 8 still fit on the GPU at once, so that each CTA's share of H
+// fits its ring in one round.
+static int cluster_router_nq(int H, int T, int num_sms)
+{
+    if (H % 512 == 0 && router_slots(T) * 8 <= num_sms) return 8;
+    return H % 256 == 0 ? 4 : 2;
+}
 // Dynamic shared memory the cluster router may take beside its static arrays.
 constexpr int kCMaxDynSmem = 208 * 1024;
 
-bool route_uses_cluster_kernel(const Shape &s, int unmasked)
+bool route_uses_cluster_kernel(const Shape &s, int unmasked, int num_sms)
 {
     if (unmasked) return false;
     const int P = s.E_pub > s.E_priv ? s.E_pub : s.E_priv;
-    return cluster_router_smem(P, s.k, cluster_router_nq(s.H)) <= kCMaxDynSmem;
+    return cluster_router_smem(P, s.k, cluster_router_nq(s.H, s.T, num_sms)) <= kCMaxDynSmem;
 }
 
 cudaError_t launch_route(const Ctx &c)
 {
     const Shape &s = c.s;
-    if (!route_uses_cluster_kernel(s, c.unmasked)) return launch_route_chunked(c);
+    if (!route_uses_cluster_kernel(s, c.unmasked, c.num_sms)) return launch_route_chunked(c);
     ClusterRouterParams p;
     ClusterRouterMaps maps;
     memset(&p, 0, sizeof(p));
     memset(&maps, 0, sizeof(maps));
     p.T = s.T; p.H = s.H; p.E_pub = s.E_pub; p.E_priv = s.E_priv; p.k = s.k; p.renorm = s.renorm;
-    p.nq = cluster_router_nq(s.H);
+    p.nq = cluster_router_nq(s.H, s.T, c.num_sms);
     p.slots4 = router_slots4(s.T);
     p.idesc = make_idesc(128, kCTile);
     p.policy = c.policy;

@@ -81,7 +81,7 @@ int column_block(int H);
 cudaError_t launch_route(const Ctx &c);
 // Whether launch_route takes the cluster router (no memset before it; the
 // dispatch derives the per-expert counts from tile_counts) or the chunked one.
-bool route_uses_cluster_kernel(const Shape &s, int unmasked);
+bool route_uses_cluster_kernel(const Shape &s, int unmasked, int num_sms);
 cudaError_t launch_permute(const Ctx &c);
 cudaError_t launch_gateup(const Ctx &c);
 cudaError_t launch_down(const Ctx &c);
