@@ -580,8 +580,8 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
 // H/nq of each token row and of each router row.  The partial logits go from
 // tensor memory to shared memory; after a cluster barrier, CTA q owns the
 // tokens [q 128/nq, (q+1) 128/nq) of the tile and sums their partial logits
-// over the nq CTAs in CTA order (distributed shared memory), one warp per
-// token, and masks them; k rounds of a warp-wide argmax select the top-k.  The
+// over the nq CTAs in CTA order (distributed shared memory), masks, selects
+// the top-k in 32-expert chunks and merges the chunk lists per token.  The
 // rank of each row among the tile's rows of its expert comes from the tile's
 // 128-bit token mask per expert, whose words the CTAs of the cluster exchange
 // after a second cluster barrier.  CTA 0 writes the tile's column of
@@ -624,9 +624,10 @@ static int cluster_router_smem(int P, int k, int nq)
 {
     const int pp = (P + 127) / 128 * 128;
     const int tpc = kCTile / nq;
+    const int nc = (P + kChunk - 1) / kChunk;
     const int partial = kCTile * (pp + 4) * 4;
-    const int picks = tpc * k * 8;
-    const int after = partial + picks;
+    const int lists = tpc * nc * k * 8 + tpc * nc * 16;
+    const int after = partial + lists;
     return (after > kCRingBytes ? after : kCRingBytes) + 1024;
 }
 
@@ -863,104 +864,133 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     tc_fence_before();
     cluster_sync_all();  // #1: every CTA's partial logits are in its shared memory
 
-    // ---- finalize this CTA's tokens, one warp per token: lane l holds the
-    // logits of experts 4l .. 4l+3 (and 128 + 4l .. for pools above 128),
-    // each the sum of the cluster's partials in CTA order (deterministic);
-    // then k rounds of a warp argmax (larger logit, ties to the lower id)
+    // ---- finalize this CTA's tokens: sum the partials over the cluster in CTA
+    // order, top-k per 32-expert chunk, then the merge per token
     const int tpc = kCTile / p.nq;
     const int ntok = max(0, min(rows - q * tpc, tpc));
     const int K = p.k;
     const int pitch = pp + 4;
-    float *sel_v = reinterpret_cast<float *>(sgen + (size_t)kCTile * pitch * 4);  // [tpc][K]
-    int *sel_e = reinterpret_cast<int *>(sel_v + (size_t)tpc * K);                // [tpc][K]
+    float *lv = reinterpret_cast<float *>(sgen + (size_t)kCTile * pitch * 4);  // [tpc][nc][K] scores
+    int *le = reinterpret_cast<int *>(lv + (size_t)tpc * nc * K);               // [tpc][nc][K] ids
+    float4 *lmeta = reinterpret_cast<float4 *>(le + (size_t)tpc * nc * K);       // [tpc][nc]
     const uint32_t S_local = sbase;
     if (warp >= 2 && !s_abort) {
-        for (int tl = warp - 2; tl < ntok; tl += 4) {
+        for (int pi = tid - 64; pi < ntok * nc; pi += 128) {
+            const int tl = pi / nc, c = pi - tl * nc;
             const int tt = q * tpc + tl;  // token index inside the tile
-            float v[8];
-            int e[8];
+            float v[32];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = 0.f;
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+            const uint32_t off = (uint32_t)((tt * pitch + c * 32) * 4);
+            // every CTA's partials of these 32 logits, half a chunk at a time:
+            // all loads of a half are issued before any is used, then summed
+            // in CTA order (fixed: deterministic)
             for (int q0 = 0; q0 < p.nq; q0 += 4) {
-                float4 x[4][2];
 #pragma unroll
-                for (int qq = 0; qq < 4; ++qq)
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    float4 x[4][4];
 #pragma unroll
-                    for (int h = 0; h < 2; ++h)
-                        if (q0 + qq < p.nq && h < nm)
-                            x[qq][h] = dsmem_ld_f4(
-                                dsmem_addr(S_local + (uint32_t)((tt * pitch + h * 128 + 4 * lane) * 4), (uint32_t)(q0 + qq)));
+                    for (int qq = 0; qq < 4; ++qq)
+                        if (q0 + qq < p.nq) {
+                            const uint32_t ra = dsmem_addr(S_local + off + 64u * h2, (uint32_t)(q0 + qq));
 #pragma unroll
-                for (int qq = 0; qq < 4; ++qq)
-#pragma unroll
-                    for (int h = 0; h < 2; ++h)
-                        if (q0 + qq < p.nq && h < nm) {
-                            v[4 * h] += x[qq][h].x; v[4 * h + 1] += x[qq][h].y;
-                            v[4 * h + 2] += x[qq][h].z; v[4 * h + 3] += x[qq][h].w;
+                            for (int i = 0; i < 4; ++i) x[qq][i] = dsmem_ld_f4(ra + 16u * i);
                         }
+#pragma unroll
+                    for (int qq = 0; qq < 4; ++qq)
+                        if (q0 + qq < p.nq) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                float *d = v + 16 * h2 + 4 * i;
+                                d[0] += x[qq][i].x; d[1] += x[qq][i].y; d[2] += x[qq][i].z; d[3] += x[qq][i].w;
+                            }
+                        }
+                }
             }
+            const int nvalid = min(kChunk, P - c * kChunk);
+            int e[32];
             float mx = -INFINITY;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int ei = (i >> 2) * 128 + 4 * lane + (i & 3);
+            for (int i = 0; i < 32; ++i) {
                 float x = v[i];
                 if (x != x) x = -INFINITY;  // NaN never outranks a number
-                const bool in_pool = (i >> 2) < nm && ei < P;
+                const bool in_pool = i < nvalid;
                 v[i] = in_pool ? x : -INFINITY;
-                e[i] = in_pool ? ei : 0x7fffffff;  // past the pool: below every expert
+                e[i] = in_pool ? c * kChunk + i : 0x7fffffff;
                 mx = in_pool ? fmaxf(mx, x) : mx;
             }
-            float pool_sum = 0.f;
-            if (!p.renorm) {  // the pool softmax denominator, shifted by the pool's largest logit
+            float ssum = 0.f;
+            if (!p.renorm) {
 #pragma unroll
-                for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(~0u, mx, off));
-#pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    if (e[i] != 0x7fffffff) pool_sum += expf(v[i] - mx);
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) pool_sum += __shfl_xor_sync(~0u, pool_sum, off);
+                for (int i = 0; i < 32; ++i)
+                    if (i < nvalid) ssum += expf(v[i] - mx);
             }
-            uint32_t taken = 0u;  // bit i: v[i] already selected
-            float my_v = 0.f;
-            int my_e = 0;
-            float top = 0.f;
-            for (int j = 0; j < K; ++j) {
-                float bv = -INFINITY;
-                int be = 0x7fffffff, bi = -1;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const bool better = !((taken >> i) & 1u) && e[i] != 0x7fffffff &&
-                                        (bi < 0 || ranks_above(v[i], e[i], bv, be));
-                    bv = better ? v[i] : bv;
-                    be = better ? e[i] : be;
-                    bi = better ? i : bi;
+            const int cnt = min(K, nvalid);
+            float *dv = lv + ((size_t)tl * nc + c) * K;
+            int *de = le + ((size_t)tl * nc + c) * K;
+            if (K <= 8) {
+                uint32_t taken = nvalid >= 32 ? 0u : ~((1u << nvalid) - 1u);
+                for (int j = 0; j < cnt; ++j) {
+                    float bv;
+                    int be;
+                    const int bi = best_untaken(v, e, taken, bv, be);
+                    taken |= 1u << bi;
+                    dv[j] = bv;
+                    de[j] = be;
                 }
-                // the warp's best (every lane ends with the same pair)
+            } else {
+                sort32(v, e);
 #pragma unroll
-                for (int off = 16; off > 0; off >>= 1) {
-                    const float ov = __shfl_xor_sync(~0u, bv, off);
-                    const int oe = __shfl_xor_sync(~0u, be, off);
-                    const bool take = oe != 0x7fffffff && (be == 0x7fffffff || ranks_above(ov, oe, bv, be));
-                    bv = take ? ov : bv;
-                    be = take ? oe : be;
+                for (int j = 0; j < 32; ++j)
+                    if (j < cnt) {
+                        dv[j] = v[j];
+                        de[j] = e[j];
+                    }
+            }
+            lmeta[tl * nc + c] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
+        }
+    }
+    __syncthreads();
+    // merge the chunk lists of token tl in chunk order (one thread per token)
+    float sel_v[kMaxTopK];
+    int sel_e[kMaxTopK];
+    float top = 0.f, Ssum = 0.f;
+    const int tl = tid;
+    const bool mine = tl < ntok && !s_abort;
+    if (mine) {
+        int head[kCMaxChunks], n[kCMaxChunks];
+#pragma unroll
+        for (int u = 0; u < kCMaxChunks; ++u) {
+            head[u] = 0;
+            n[u] = u < nc ? __float_as_int(lmeta[tl * nc + u].z) : 0;
+        }
+        for (int j = 0; j < K; ++j) {
+            int bu = -1, be = 0;
+            float bv = 0.f;
+#pragma unroll
+            for (int u = 0; u < kCMaxChunks; ++u) {
+                if (head[u] < n[u]) {
+                    const size_t o = ((size_t)tl * nc + u) * K + head[u];
+                    const float x = lv[o];
+                    const int ee = le[o];
+                    if (bu < 0 || ranks_above(x, ee, bv, be)) { bu = u; bv = x; be = ee; }
                 }
-                if (bi >= 0 && e[bi] == be) taken |= 1u << bi;  // the owning lane marks it
-                if (lane == j) { my_v = bv; my_e = be; }
-                if (j == 0) top = bv;
             }
-            // routing weights: softmax over the k selected logits, or the pool
-            // softmax probabilities; lane j holds pick j
-            float ex = lane < K ? expf(my_v - top) : 0.f;
-            float denom = pool_sum;
-            if (p.renorm) {
-                denom = ex;
+            if (bu < 0) break;  // unreachable for k <= pool size
 #pragma unroll
-                for (int off = 16; off > 0; off >>= 1) denom += __shfl_xor_sync(~0u, denom, off);
-            }
-            if (lane < K) {
-                sel_v[tl * K + lane] = ex / denom;
-                sel_e[tl * K + lane] = my_e;
-                atomicOr(&smask[my_e * 4 + (tt >> 5)], 1u << (tt & 31));
+            for (int u = 0; u < kCMaxChunks; ++u) head[u] += (u == bu) ? 1 : 0;
+            sel_v[j] = bv;
+            sel_e[j] = be;
+            if (j == 0) top = bv;
+            const int tt = q * tpc + tl;
+            atomicOr(&smask[be * 4 + (tt >> 5)], 1u << (tt & 31));
+        }
+        if (p.renorm) {
+            for (int j = 0; j < K; ++j) Ssum += expf(sel_v[j] - top);
+        } else {
+            for (int u = 0; u < nc; ++u) {  // fixed order: deterministic
+                const float4 m = lmeta[tl * nc + u];
+                if (__float_as_int(m.z) > 0) Ssum += m.y * expf(m.x - top);
             }
         }
     }
@@ -998,23 +1028,21 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             if (c && p.route_count) atomicAdd(&p.route_count[eg], c);
         }
     }
-    if (!s_abort) {
-        for (int pi = tid; pi < ntok * K; pi += kCThreads) {
-            const int tl = pi / K, j = pi - tl * K;
-            const int tt = q * tpc + tl;
-            const int t = s_tok[tt];
-            const int be = sel_e[tl * K + j];
-            const int wd = tt >> 5;
-            int rank = (int)__popc(sfull[be * 4 + wd] & ((1u << (tt & 31)) - 1u));
+    if (mine) {
+        const int tt = q * tpc + tl;
+        const int t = s_tok[tt];
+        const int wd = tt >> 5;
+        const uint32_t below = (1u << (tt & 31)) - 1u;
+        for (int j = 0; j < K; ++j) {
+            const int be = sel_e[j];
+            int rank = (int)__popc(sfull[be * 4 + wd] & below);
             for (int w2 = 0; w2 < wd; ++w2) rank += (int)__popc(sfull[be * 4 + w2]);
             p.idx[(size_t)t * K + j] = base + be;
             p.ticket[(size_t)t * K + j] = (int32_t)(slot * kCTile + rank);
-            p.w[(size_t)t * K + j] = sel_v[tl * K + j];
-            if (j == 0) {
-                p.tau[t] = pool ? 1 : 0;
-                if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], pool ? (unsigned)K : 0u);
-            }
+            p.w[(size_t)t * K + j] = expf(sel_v[j] - top) / Ssum;
         }
+        p.tau[t] = pool ? 1 : 0;
+        if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], pool ? (unsigned)K : 0u);
     }
     __syncthreads();
     cluster_sync_all();  // #3: no CTA leaves while another still reads its shared memory

@@ -40,10 +40,10 @@ CASES = {
     # k > 8 takes the router's sorting-network path; 40 public experts span two chunks
     "k12_two_chunks_pool_softmax": (LayerShape(T=150, H=256, I=128, E_pub=40, E_priv=16, E_sh=0, k=12,
                                                renormalize=False), 44, "iid"),
-    # a 256-expert pool (two MMAs of 128 experts, eight logits a lane) with
-    # k = 24 warp-argmax rounds, at H = 128 (clusters of 2)
-    "k24_pool_256": (LayerShape(T=200, H=128, I=128, E_pub=256, E_priv=64, E_sh=0, k=24, renormalize=True), 47,
-                     "iid"),
+    # a 256-expert pool with k = 24 at H = 128: the chunk lists do not fit the
+    # cluster router's shared memory, so the chunked router runs the method
+    "k24_pool_256_chunked_router": (LayerShape(T=200, H=128, I=128, E_pub=256, E_priv=64, E_sh=0, k=24,
+                                               renormalize=True), 47, "iid"),
 }
 
 
