@@ -1159,13 +1159,16 @@ static cudaError_t launch_route_chunked(const Ctx &c)
     return launch_pdl(router_tc_kernel, dim3(grid), dim3(kRThreads), smem, c.stream, p, maps);
 }
 
-// CTAs per cluster of router_cluster_kernel for hidden size H and T tokens:
-// 4 (2 when H is not a multiple of 256), and 8 when H allows and the
-// clusters of 8 still fit on the GPU at once, so that each CTA's share of H
-// fits its ring in one round.
+// CTAs per cluster of router_cluster_kernel for hidden size H and T tokens
+// (one CTA per SM): 8 when H allows and the clusters of 8 fit on the GPU at
+// once, so that each CTA's share of H fits its ring in one round; else 4 (2
+// when H is not a multiple of 256); and 2 when clusters of 4 would not fit
+// the GPU in one wave (one wave of clusters of 2 measured faster than two
+// waves of clusters of 4: 35 vs 57 us at T = 8192).
 static int cluster_router_nq(int H, int T, int num_sms)
 {
     if (H % 512 == 0 && router_slots(T) * 8 <= num_sms) return 8;
+    if (router_slots(T) * 4 > num_sms) return 2;
     return H % 256 == 0 ? 4 : 2;
 }
 // Dynamic shared memory the cluster router may take beside its static arrays.
