@@ -34,6 +34,16 @@ from paper_2608_06690_gb300.configs import CONFIGS  # noqa: E402
 
 METRIC = "MoE-layer tokens/s (mixed allow/deny)"
 L2_FLUSH_BYTES = 512 << 20   # > 129 MB L2
+# After each L2 flush the GPU also spins this many cycles (~0.1 ms) before
+# the timed interval opens, so the host has always enqueued the timed work
+# by the time the GPU reaches it: no host gap inside a measured interval,
+# also for the first interval after a synchronisation.
+GPU_LEAD_CYCLES = 200_000
+
+
+def flush_l2(flush):
+    flush.zero_()
+    torch.cuda._sleep(GPU_LEAD_CYCLES)
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
 # grouped GEMM launches (the persistent gate/up + down pair, and each GEMM
@@ -412,7 +422,7 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     torch.cuda.synchronize(dev)
     t_wall0 = time.perf_counter()
     for e0, e1 in evs:
-        flush.zero_()
+        flush_l2(flush)
         e0.record(stream)
         step()
         e1.record(stream)
@@ -438,7 +448,7 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
     for _ in range(args.steps):
         evs_s = []
         for n, bit in stages:
-            flush.zero_()
+            flush_l2(flush)
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(stream)
             layer.forward(h, pol, out=out, stages=bit)
@@ -541,7 +551,7 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
         "config": {"workload": cfg.name, "T": s.T, "H": s.H, "I": s.I, "E_pub": s.E_pub, "E_priv": s.E_priv,
                    "E_shared": s.E_sh, "k": s.k, "renormalize": s.renormalize, "requests": cfg.n_requests,
                    "allow_tokens": int((pol == 1).sum().item()),
-                   "l2": "flushed (512 MB write) before every step", "parallelism": f"replicas x{ws_n}"},
+                   "l2": "flushed (512 MB write) before every step, then a 0.1 ms GPU spin outside the timed interval", "parallelism": f"replicas x{ws_n}"},
     }
     return rep, layer, counts
 
@@ -561,7 +571,7 @@ def measure_backward(pmpe, cfg, layer, h, pol, dev, args, flush, counts):
     def timed(fn, n):
         evs = []
         for _ in range(n):
-            flush.zero_()
+            flush_l2(flush)
             a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a_ev.record(stream)
             fn()

@@ -200,6 +200,14 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     // activations and per-row outputs are read again by other tiles of this
     // launch (evict last)
     const uint64_t pol_stream = l2_policy_evict_first(), pol_keep = l2_policy_evict_last();
+    if (warp == 0 && lane < 2) {  // the weight maps of this launch's GEMMs, ahead of their first loads
+        const int ph = lane == 0 ? kGateUp : kDown;
+        if (ph == kGateUp ? p.has_gu : p.has_down)
+            for (int q = 0; q < (p.E_sh > 0 ? 3 : 2); ++q) {
+                prefetch_tmap(&maps.b0[ph][q]);
+                if (ph == kGateUp) prefetch_tmap(&maps.b1[ph][q]);
+            }
+    }
     pdl_trigger();
 
     if (tid == 0) {

@@ -577,14 +577,18 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
 // by the pool's router over the q-th 1/nq of H: tcgen05.mma with the router
 // rows as M (128 experts per MMA, one or two MMAs for pools up to 256; rows
 // past the pool read as zeros) and the 128 tokens as N, so the CTA reads
-// H/nq of each token row and of each router row.  The partial logits go from
-// tensor memory to shared memory; after a cluster barrier, CTA q owns the
-// tokens [q 128/nq, (q+1) 128/nq) of the tile and sums their partial logits
-// over the nq CTAs in CTA order (distributed shared memory), masks, selects
-// the top-k in 32-expert chunks and merges the chunk lists per token.  The
+// H/nq of each token row and of each router row.  CTA q owns the tokens
+// [q 128/nq, (q+1) 128/nq) of the tile.  Once every CTA of the cluster has
+// finished its MMAs (a cluster barrier: the rings are then free), each CTA
+// pushes its partial logits straight from tensor memory into the owner's
+// shared memory with remote stores (distributed shared memory), one slot per
+// source CTA; after a second barrier, the owner sums them in CTA order from
+// its own shared memory (deterministic), masks, sorts each 32-expert chunk's
+// best candidates with a bitonic network and merges the chunk lists of a
+// token by lane shuffles.  The
 // rank of each row among the tile's rows of its expert comes from the tile's
 // 128-bit token mask per expert, whose words the CTAs of the cluster exchange
-// after a second cluster barrier.  CTA 0 writes the tile's column of
+// after a third cluster barrier.  CTA 0 writes the tile's column of
 // tile_counts for every expert (zero for the other pool), so nothing has to
 // be cleared before the launch; a cluster whose slot holds no tile writes
 // zeros there.  The dispatch sums the columns into the per-expert counts.
@@ -595,7 +599,6 @@ constexpr int kCThreads = 192;       // warp 0 TMA, warp 1 TMEM + MMA, warps 2..
 constexpr int kCTile = 128;          // tokens per tile (MMA N)
 constexpr int kCRingBytes = 192 * 1024;
 constexpr int kCMaxStages = 6;
-constexpr int kCMaxChunks = kMaxPool / kChunk;  // 32-expert chunks of one pool
 
 struct ClusterRouterParams {
     int T, H, E_pub, E_priv, k, renorm;
@@ -624,10 +627,9 @@ static int cluster_router_smem(int P, int k, int nq)
 {
     const int pp = (P + 127) / 128 * 128;
     const int tpc = kCTile / nq;
-    const int nc = (P + kChunk - 1) / kChunk;
-    const int partial = kCTile * (pp + 4) * 4;
-    const int lists = tpc * nc * k * 8 + tpc * nc * 16;
-    const int after = partial + lists;
+    const int partial = kCTile * (pp + 4) * 4;  // staged partials, then the receive buffer
+    const int lists = tpc * k * 8 + tpc * 8;
+    const int after = 2 * partial + lists;
     return (after > kCRingBytes ? after : kCRingBytes) + 1024;
 }
 
@@ -647,19 +649,177 @@ __device__ __forceinline__ uint32_t dsmem_addr(uint32_t local, uint32_t rank)
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(local), "r"(rank));
     return r;
 }
-__device__ __forceinline__ float4 dsmem_ld_f4(uint32_t addr)
-{
-    float4 v;
-    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];\n"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(addr));
-    return v;
-}
 __device__ __forceinline__ uint32_t dsmem_ld_u32(uint32_t addr)
 {
     uint32_t v;
     asm volatile("ld.shared::cluster.u32 %0, [%1];\n" : "=r"(v) : "r"(addr));
     return v;
+}
+
+// Bulk copy of `bytes` (a multiple of 16, both addresses 16-byte aligned)
+// from this CTA's shared memory to a shared::cluster address of another CTA
+// of the cluster, completing as transaction bytes on that CTA's mbarrier.
+__device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
+                 "r"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+// Selection key of a logit of pool-local expert `id` (< 256): the logit's
+// order-preserving 32-bit image with its low 8 bits replaced by 255 - id.
+// Keys are unique and nonzero, compare like (logit desc, id asc) except
+// between logits in the same 256-ulp bucket (key >> 8), and carry the id.
+__device__ __forceinline__ uint32_t logit_key(float x, int id)
+{
+    x = x == 0.f ? 0.f : x;  // -0 and +0 are equal logits
+    const uint32_t b = __float_as_uint(x);
+    const uint32_t m = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return (m & 0xffffff00u) | (uint32_t)(255 - id);
+}
+
+// A summed logit as the mask treats it: NaN never outranks a number.
+__device__ __forceinline__ float clean_logit(float x) { return x != x ? -INFINITY : x; }
+
+// Finalize of the tile's tokens [q tpc, q tpc + ntok) owned by this CTA, by
+// all threads of the CTA (a warp-uniform loop; the code is kept compact,
+// since each CTA runs it once, from a cold instruction cache).
+//
+// Thread pair (token tl, chunk c) sums the chunk's 32 partial logits over
+// the cluster's CTAs in CTA order (rcv[src][tl][expert]; the sums replace
+// slot 0), stores their selection keys in slot 1 and records the chunk's
+// softmax partial (max, sum of exp(x - max)); experts past the pool have no
+// key.  The ncp lanes of a token (ncp = chunks rounded up to a power of two;
+// padding lanes hold no key) then take k + 1 passes: the group's largest key
+// left (a max over the lane's keys, then over the lanes by shuffles), which
+// its owner removes.  The keys of the passes are the candidates in key
+// order; they are the exact top k in the exact order whenever no two
+// consecutive ones of the first k + 1 share a bucket.  Otherwise (near-equal
+// logits) the warp repeats the selection with the exact comparison of
+// (logit, id).  The token's k pool-local ids go to sel_e, the logits to
+// sel_v, its top logit and the softmax denominator (over the k selected
+// logits, or over the whole pool from the chunk partials in chunk order) to
+// tmeta, and every selected (expert, token) sets its bit in the CTA's mask.
+__device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pitch, int q, int tpc,
+                                int ntok, int nc, int P, float *sel_v, int *sel_e, float2 *tmeta,
+                                uint32_t *smask)
+{
+    const int ncp = nc <= 1 ? 1 : (nc <= 2 ? 2 : (nc <= 4 ? 4 : 8));
+    const int lg = ncp == 1 ? 0 : (ncp == 2 ? 1 : (ncp == 4 ? 2 : 3));
+    const int npairs = tpc * ncp;
+    const int K = p.k;
+    for (int pb = 0; pb < npairs; pb += kCThreads) {  // the same trip count in every lane
+        const int pi = pb + (int)threadIdx.x;
+        const int tl = pi >> lg, c = pi & (ncp - 1);
+        const bool tok_ok = pi < npairs && tl < ntok;
+        const int nvalid = (tok_ok && c < nc) ? min(kChunk, P - c * kChunk) : 0;
+        float *row = rcv + (size_t)(tok_ok ? tl : 0) * pitch;  // slot 0: the token's summed logits
+        float *sum = row + c * kChunk;
+        uint32_t *key = reinterpret_cast<uint32_t *>(rcv + (size_t)tpc * pitch) + (sum - rcv);  // slot 1
+        float mx = -INFINITY, ssum = 0.f;
+        if (nvalid > 0) {
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+            for (int s2 = 0; s2 < p.nq; ++s2) {
+                const float4 *r4 = reinterpret_cast<const float4 *>(sum + (size_t)s2 * tpc * pitch);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float4 x = r4[i];
+                    v[4 * i] += x.x;
+                    v[4 * i + 1] += x.y;
+                    v[4 * i + 2] += x.z;
+                    v[4 * i + 3] += x.w;
+                }
+            }
+            float4 *w4 = reinterpret_cast<float4 *>(sum);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+#pragma unroll 4
+            for (int i = 0; i < 32; ++i) {
+                const float x = clean_logit(sum[i]);
+                key[i] = i < nvalid ? logit_key(x, c * kChunk + i) : 0u;
+                mx = i < nvalid ? fmaxf(mx, x) : mx;
+            }
+            if (!p.renorm)
+                for (int i = 0; i < nvalid; ++i) ssum += expf(clean_logit(sum[i]) - mx);
+        }
+        __syncwarp();
+        // ---- fast path: k + 1 passes over the keys
+        bool amb = false;
+        uint32_t prev = 0u;
+        for (int j = 0; j <= K; ++j) {
+            uint32_t m = 0u;
+            if (nvalid > 0) {
+                uint32_t m4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                for (int i = 0; i < 32; i += 4) {
+                    const uint4 k4 = *reinterpret_cast<const uint4 *>(key + i);
+                    m4[0] = max(m4[0], k4.x);
+                    m4[1] = max(m4[1], k4.y);
+                    m4[2] = max(m4[2], k4.z);
+                    m4[3] = max(m4[3], k4.w);
+                }
+                m = max(max(m4[0], m4[1]), max(m4[2], m4[3]));
+            }
+            for (int d = 1; d < ncp; d <<= 1) m = max(m, __shfl_xor_sync(~0u, m, d));
+            const int id = 255 - (int)(m & 255u);
+            if (m != 0u && nvalid > 0 && (id >> 5) == c) key[id & 31] = 0u;  // the owner removes the winner
+            if (j > 0) amb |= (m >> 8) == (prev >> 8);
+            if (j < K && c == 0 && tok_ok) sel_e[tl * K + j] = id;
+            prev = m;
+            __syncwarp();
+        }
+        amb &= tok_ok;
+        if (__any_sync(~0u, amb)) {
+            // ---- exact path for the whole warp: k passes with the exact
+            // comparison of (logit, id), ties to the lower id
+            uint32_t taken = 0u;
+            for (int j = 0; j < K; ++j) {
+                float bv = -INFINITY;
+                int be = 0x7fffffff;
+                for (int i = 0; i < nvalid; ++i) {
+                    const float x = clean_logit(sum[i]);
+                    const int e = c * kChunk + i;
+                    if (!((taken >> i) & 1u) && ranks_above(x, e, bv, be)) {
+                        bv = x;
+                        be = e;
+                    }
+                }
+                for (int d = 1; d < ncp; d <<= 1) {
+                    const float ov = __shfl_xor_sync(~0u, bv, d);
+                    const int oe = __shfl_xor_sync(~0u, be, d);
+                    if (ranks_above(ov, oe, bv, be)) {
+                        bv = ov;
+                        be = oe;
+                    }
+                }
+                if (nvalid > 0 && (be >> 5) == c) taken |= 1u << (be & 31);
+                if (c == 0 && tok_ok) sel_e[tl * K + j] = be;
+            }
+            __syncwarp();
+        }
+        // ---- the selected logits, the mask bits, top and denominator
+        float top = 0.f, den = 0.f;
+        if (tok_ok) {
+            const int tt = q * tpc + tl;
+            for (int j = c; j < K; j += ncp) {
+                const int e = sel_e[tl * K + j];
+                sel_v[tl * K + j] = clean_logit(row[e]);
+                atomicOr(&smask[e * 4 + (tt >> 5)], 1u << (tt & 31));
+            }
+            top = clean_logit(row[sel_e[tl * K]]);
+            if (p.renorm)
+                for (int j = 0; j < K; ++j) den += expf(clean_logit(row[sel_e[tl * K + j]]) - top);
+        }
+        if (!p.renorm) {
+            const int g0 = (int)(threadIdx.x & 31) & ~(ncp - 1);
+            for (int u = 0; u < ncp; ++u) {  // chunk order: deterministic
+                const float mu = __shfl_sync(~0u, mx, g0 + u), su = __shfl_sync(~0u, ssum, g0 + u);
+                if (u < nc) den += su * expf(mu - top);
+            }
+        }
+        if (tok_ok && c == 0) tmeta[tl] = make_float2(top, den);
+    }
 }
 
 __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const ClusterRouterParams p,
@@ -668,7 +828,7 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     extern __shared__ uint8_t dsmem[];
     __shared__ int s_tok[kCTile];
     __shared__ int warp_tot[kCThreads / 32];
-    __shared__ __align__(8) uint64_t bars[2 * kCMaxStages + 2];
+    __shared__ __align__(8) uint64_t bars[2 * kCMaxStages + 3];
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
     __shared__ uint32_t smask[kMaxPool * 4];  // this CTA's tokens of the tile, per pool expert, 4 x 32 bits
@@ -677,6 +837,11 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int q = (int)cluster_ctarank();
     const int slot = blockIdx.x / p.nq;
+    if (tid == 0) {
+        prefetch_tmap(&maps.hidden);
+        prefetch_tmap(&maps.router[0]);
+        prefetch_tmap(&maps.router[1]);
+    }
     pdl_trigger();
     pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
 
@@ -732,6 +897,11 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     auto empty_bar = [&](int st) { return bar0 + 8u * (kCMaxStages + st); };
     const uint32_t tfull_bar = bar0 + 8u * (2 * kCMaxStages);
     const uint32_t done_bar = bar0 + 8u * (2 * kCMaxStages + 1);
+    const uint32_t rcv_bar = bar0 + 8u * (2 * kCMaxStages + 2);  // partial logits received from the cluster
+    const int tpc = kCTile / p.nq;
+    const int pitch = pp + 4;
+    const uint32_t slice_bytes = (uint32_t)(tpc * pitch * 4);  // one source CTA's partials of this CTA's tokens
+    const uint32_t part_bytes = (uint32_t)(kCTile * pitch * 4);
     if (tid == 0) {
         for (int st = 0; st < stages; ++st) {
             mbar_init(full_bar(st), contiguous ? 2 : 1 + 128);
@@ -739,6 +909,8 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
         }
         mbar_init(tfull_bar, 1);
         mbar_init(done_bar, 1);
+        mbar_init(rcv_bar, 1);
+        mbar_expect_tx(rcv_bar, (uint32_t)p.nq * slice_bytes);
         s_abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
@@ -837,8 +1009,8 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             }
             cp_async_wait<0>();
         }
-        // ---- epilogue: partial logits to shared memory, [token][expert] FP32
-        // (the ring is free once every MMA has completed)
+        // ---- epilogue: the partial logits to shared memory, [token][expert]
+        // FP32 (pitch pp + 4; the ring is free once every MMA has completed)
         int ok = 1;
         if (lane == 0) ok = mbar_wait(tfull_bar, 0, &s_abort, p.status) ? 1 : 0;
         ok = __shfl_sync(~0u, ok, 0);
@@ -847,7 +1019,6 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             tc_fence_after();
             const int quarter = warp & 3;
             float *S = reinterpret_cast<float *>(sgen);
-            const int pitch = pp + 4;
             for (int mi = 0; mi < nm; ++mi) {
                 const int e = mi * 128 + quarter * 32 + lane;
                 for (int cc = 0; cc < kCTile / 32; ++cc) {
@@ -858,141 +1029,54 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
                     for (int i = 0; i < 32; ++i) S[(cc * 32 + i) * pitch + e] = v[i];
                 }
             }
+            fence_proxy_async_smem();  // the bulk copies below read these rows
         }
     }
     __syncwarp();
     tc_fence_before();
-    cluster_sync_all();  // #1: every CTA's partial logits are in its shared memory
+    // #1: every CTA of the cluster has staged its partial logits, and every
+    // ring is free to receive the others'
+    cluster_sync_all();
+    tc_fence_after();
 
-    // ---- finalize this CTA's tokens: sum the partials over the cluster in CTA
-    // order, top-k per 32-expert chunk, then the merge per token
-    const int tpc = kCTile / p.nq;
-    const int ntok = max(0, min(rows - q * tpc, tpc));
-    const int K = p.k;
-    const int pitch = pp + 4;
-    float *lv = reinterpret_cast<float *>(sgen + (size_t)kCTile * pitch * 4);  // [tpc][nc][K] scores
-    int *le = reinterpret_cast<int *>(lv + (size_t)tpc * nc * K);               // [tpc][nc][K] ids
-    float4 *lmeta = reinterpret_cast<float4 *>(le + (size_t)tpc * nc * K);       // [tpc][nc]
-    const uint32_t S_local = sbase;
-    if (warp >= 2 && !s_abort) {
-        for (int pi = tid - 64; pi < ntok * nc; pi += 128) {
-            const int tl = pi / nc, c = pi - tl * nc;
-            const int tt = q * tpc + tl;  // token index inside the tile
-            float v[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-            const uint32_t off = (uint32_t)((tt * pitch + c * 32) * 4);
-            // every CTA's partials of these 32 logits, half a chunk at a time:
-            // all loads of a half are issued before any is used, then summed
-            // in CTA order (fixed: deterministic)
-            for (int q0 = 0; q0 < p.nq; q0 += 4) {
-#pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    float4 x[4][4];
-#pragma unroll
-                    for (int qq = 0; qq < 4; ++qq)
-                        if (q0 + qq < p.nq) {
-                            const uint32_t ra = dsmem_addr(S_local + off + 64u * h2, (uint32_t)(q0 + qq));
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) x[qq][i] = dsmem_ld_f4(ra + 16u * i);
-                        }
-#pragma unroll
-                    for (int qq = 0; qq < 4; ++qq)
-                        if (q0 + qq < p.nq) {
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                float *d = v + 16 * h2 + 4 * i;
-                                d[0] += x[qq][i].x; d[1] += x[qq][i].y; d[2] += x[qq][i].z; d[3] += x[qq][i].w;
-                            }
-                        }
-                }
+    // ---- exchange: CTA q sends the rows of owner o's tokens [o tpc, (o + 1)
+    // tpc) to slot q of o's receive buffer (after the staging rows) with one
+    // bulk copy per owner, completing on o's rcv_bar; every CTA then waits
+    // for its nq slots.  The wait is bounded but ignores the abort flag: no
+    // copy into this CTA's shared memory may still be in flight at its exit.
+    if (tid == 0) {
+        for (int o = 0; o < p.nq; ++o)
+            bulk_copy_to_peer(dsmem_addr(sbase + part_bytes + (uint32_t)q * slice_bytes, (uint32_t)o),
+                              sbase + (uint32_t)o * slice_bytes, slice_bytes, dsmem_addr(rcv_bar, (uint32_t)o));
+    }
+    bool received = true;
+    {
+        const unsigned long long w0 = globaltimer_ns();
+        while (!mbar_try_wait(rcv_bar, 0))
+            if (globaltimer_ns() - w0 > kWaitLimitNs) {
+                received = false;
+                break;
             }
-            const int nvalid = min(kChunk, P - c * kChunk);
-            int e[32];
-            float mx = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                float x = v[i];
-                if (x != x) x = -INFINITY;  // NaN never outranks a number
-                const bool in_pool = i < nvalid;
-                v[i] = in_pool ? x : -INFINITY;
-                e[i] = in_pool ? c * kChunk + i : 0x7fffffff;
-                mx = in_pool ? fmaxf(mx, x) : mx;
-            }
-            float ssum = 0.f;
-            if (!p.renorm) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (i < nvalid) ssum += expf(v[i] - mx);
-            }
-            const int cnt = min(K, nvalid);
-            float *dv = lv + ((size_t)tl * nc + c) * K;
-            int *de = le + ((size_t)tl * nc + c) * K;
-            if (K <= 8) {
-                uint32_t taken = nvalid >= 32 ? 0u : ~((1u << nvalid) - 1u);
-                for (int j = 0; j < cnt; ++j) {
-                    float bv;
-                    int be;
-                    const int bi = best_untaken(v, e, taken, bv, be);
-                    taken |= 1u << bi;
-                    dv[j] = bv;
-                    de[j] = be;
-                }
-            } else {
-                sort32(v, e);
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (j < cnt) {
-                        dv[j] = v[j];
-                        de[j] = e[j];
-                    }
-            }
-            lmeta[tl * nc + c] = make_float4(mx, ssum, __int_as_float(cnt), 0.f);
-        }
+    }
+    if (!received && tid == 0) {
+        s_abort = 1;
+        if (p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
     }
     __syncthreads();
-    // merge the chunk lists of token tl in chunk order (one thread per token)
-    float sel_v[kMaxTopK];
-    int sel_e[kMaxTopK];
-    float top = 0.f, Ssum = 0.f;
-    const int tl = tid;
-    const bool mine = tl < ntok && !s_abort;
-    if (mine) {
-        int head[kCMaxChunks], n[kCMaxChunks];
-#pragma unroll
-        for (int u = 0; u < kCMaxChunks; ++u) {
-            head[u] = 0;
-            n[u] = u < nc ? __float_as_int(lmeta[tl * nc + u].z) : 0;
-        }
-        for (int j = 0; j < K; ++j) {
-            int bu = -1, be = 0;
-            float bv = 0.f;
-#pragma unroll
-            for (int u = 0; u < kCMaxChunks; ++u) {
-                if (head[u] < n[u]) {
-                    const size_t o = ((size_t)tl * nc + u) * K + head[u];
-                    const float x = lv[o];
-                    const int ee = le[o];
-                    if (bu < 0 || ranks_above(x, ee, bv, be)) { bu = u; bv = x; be = ee; }
-                }
-            }
-            if (bu < 0) break;  // unreachable for k <= pool size
-#pragma unroll
-            for (int u = 0; u < kCMaxChunks; ++u) head[u] += (u == bu) ? 1 : 0;
-            sel_v[j] = bv;
-            sel_e[j] = be;
-            if (j == 0) top = bv;
-            const int tt = q * tpc + tl;
-            atomicOr(&smask[be * 4 + (tt >> 5)], 1u << (tt & 31));
-        }
-        if (p.renorm) {
-            for (int j = 0; j < K; ++j) Ssum += expf(sel_v[j] - top);
-        } else {
-            for (int u = 0; u < nc; ++u) {  // fixed order: deterministic
-                const float4 m = lmeta[tl * nc + u];
-                if (__float_as_int(m.z) > 0) Ssum += m.y * expf(m.x - top);
-            }
-        }
+
+    // ---- finalize this CTA's tokens: per (token, 32-expert chunk) one thread
+    // sums the chunk's partials over the cluster in CTA order, sorts its best
+    // KP candidates (a bitonic network), and the ncp lanes of a token merge
+    // their lists by shuffles into the token's top k
+    const int ntok = max(0, min(rows - q * tpc, tpc));
+    const int K = p.k;
+    const bool abort_now = s_abort != 0;
+    float *rcv = reinterpret_cast<float *>(sgen + part_bytes);                   // [nq][tpc][pitch]
+    float *sel_v = reinterpret_cast<float *>(sgen + 2 * (size_t)part_bytes);     // [tpc][K] scores
+    int *sel_e = reinterpret_cast<int *>(sel_v + (size_t)tpc * K);                // [tpc][K] pool-local ids
+    float2 *tmeta = reinterpret_cast<float2 *>(sel_e + (size_t)tpc * K);          // [tpc] (top, denominator)
+    if (!abort_now) {
+        finalize_tokens(p, rcv, pitch, q, tpc, ntok, nc, P, sel_v, sel_e, tmeta, smask);
     }
     __syncthreads();
     cluster_sync_all();  // #2: every CTA's token masks are in its shared memory
@@ -1028,21 +1112,26 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             if (c && p.route_count) atomicAdd(&p.route_count[eg], c);
         }
     }
-    if (mine) {
-        const int tt = q * tpc + tl;
-        const int t = s_tok[tt];
-        const int wd = tt >> 5;
-        const uint32_t below = (1u << (tt & 31)) - 1u;
-        for (int j = 0; j < K; ++j) {
-            const int be = sel_e[j];
+    // one thread per routed row (token, j) of this CTA's tokens
+    if (!abort_now) {
+        for (int wi = tid; wi < ntok * K; wi += kCThreads) {
+            const int tl = wi / K, j = wi - tl * K;
+            const int tt = q * tpc + tl;
+            const int t = s_tok[tt];
+            const int wd = tt >> 5;
+            const uint32_t below = (1u << (tt & 31)) - 1u;
+            const int be = sel_e[wi];
             int rank = (int)__popc(sfull[be * 4 + wd] & below);
             for (int w2 = 0; w2 < wd; ++w2) rank += (int)__popc(sfull[be * 4 + w2]);
+            const float2 m = tmeta[tl];
             p.idx[(size_t)t * K + j] = base + be;
             p.ticket[(size_t)t * K + j] = (int32_t)(slot * kCTile + rank);
-            p.w[(size_t)t * K + j] = expf(sel_v[j] - top) / Ssum;
+            p.w[(size_t)t * K + j] = expf(sel_v[wi] - m.x) / m.y;
+            if (j == 0) {
+                p.tau[t] = pool ? 1 : 0;
+                if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], pool ? (unsigned)K : 0u);
+            }
         }
-        p.tau[t] = pool ? 1 : 0;
-        if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], pool ? (unsigned)K : 0u);
     }
     __syncthreads();
     cluster_sync_all();  // #3: no CTA leaves while another still reads its shared memory

@@ -204,6 +204,12 @@ __device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap *map
 
 // Make this thread's completed generic-proxy shared-memory writes (e.g. from
 // cp.async) visible to the async proxy that tcgen05.mma reads through.
+// Fetch a tensor map (a kernel parameter) into the TMA unit's descriptor
+// cache ahead of its first use.
+__device__ __forceinline__ void prefetch_tmap(const void *map)
+{
+    asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
 __device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
 
 __device__ __forceinline__ void tmem_alloc(uint32_t slot_smem_addr, uint32_t ncols)
