@@ -11,9 +11,16 @@
 // one accumulator).  A persistent grid (one CTA per SM) walks a tile list
 // built on the device from the dispatch offsets: no host sync, and empty
 // experts contribute no tile.  The list holds every gate/up tile, then every
-// down tile, group by group, n-tile major inside a group; CTA c takes tiles
-// c, c + grid, ... in order.  A down tile waits (bounded) until the gate/up
-// tiles of its activation rows have stored them.
+// down tile, group by group, n-tile major inside a group.  The CTAs take the
+// tiles in list order: in waves (CTA c: tiles c, c + grid, ...) when a group
+// has several 128-row blocks, so that the m-tiles sharing weights run
+// together, and otherwise dynamically, each CTA the next tile when its loader
+// is ready for one (an atomic counter), which evens out tiles of unequal
+// cost.  Warp 0 hands each tile index to the CTA's other roles through a
+// small queue in shared memory.  A down tile waits (bounded) until the
+// gate/up tiles of its activation rows have stored them; every one of those
+// was handed out earlier to a running CTA, and no gate/up tile ever waits,
+// so the wait ends.
 //
 // The routed gate/up tiles read their A rows straight from the hidden states:
 // the row of dispatch slot r is hidden[tok_of_slot[r]], gathered into shared
@@ -72,6 +79,8 @@ constexpr int kLoaders = 3;                   // TMA-issuing lanes of warp 0
 constexpr int kGatherThreads = 32 * kGatherWarps;
 constexpr int kFullArrivals = kLoaders + kGatherThreads;  // per ring stage
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
+constexpr int kTQ = 8;                        // tile queue entries (tile indices handed to the CTA's roles)
+constexpr int kTQConsumers = 1 + 4 + kGatherWarps;  // MMA thread, epilogue warps, gather warps (one lane each)
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
 constexpr int kOutBufBytes = kOutBox * kOutBox * 2;
 constexpr int kOutBytes = 4 * 2 * kOutBufBytes;  // 4 epilogue warps x 2 buffers
@@ -100,6 +109,9 @@ struct TcParams {
     // has_gu && has_down: per (group, 128-row block), the gate/up epilogue
     // warps whose activations are stored (zeroed before the launch)
     uint32_t *ready;
+    // the next tile of the list to hand out (zeroed before the launch): CTAs
+    // take tiles in list order, each when it is ready for one
+    uint32_t *tile_ctr;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
     // optional FP32: the gate and up accumulators saved for the backward,
     // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
@@ -182,9 +194,10 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
 {
     extern __shared__ uint8_t dsmem[];
     __shared__ TileTable tt;
-    __shared__ __align__(8) uint64_t bars[2 * kStages + 5];
+    __shared__ __align__(8) uint64_t bars[2 * kStages + 5 + 2 * kTQ];
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
+    __shared__ volatile int s_tq[kTQ];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
@@ -194,6 +207,24 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
     auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
     const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
+    auto tq_full_bar = [&](int i) { return bar0 + 8u * (2 * kStages + 5 + i); };
+    auto tq_empty_bar = [&](int i) { return bar0 + 8u * (2 * kStages + 5 + kTQ + i); };
+    // Entry i of the CTA's tile sequence, for a consumer role (one thread):
+    // -1 at the end of the list or after an abort.  In wave order every role
+    // computes it; dynamically, warp 0 hands it out through the tile queue.
+    bool dyn = false;
+    int total = 0;
+    auto next_tile = [&](int i) -> int {
+        if (!dyn) {
+            const long long st = (long long)blockIdx.x + (long long)i * gridDim.x;
+            return (st < total && !s_abort) ? (int)st : -1;
+        }
+        const int slot = i % kTQ;
+        if (!mbar_wait(tq_full_bar(slot), (uint32_t)(i / kTQ) & 1u, &s_abort, p.status)) return -1;
+        const int t = s_tq[slot];
+        mbar_arrive(tq_empty_bar(slot));
+        return t;
+    };
 
     const int G = p.E + (p.E_sh > 0 ? 1 : 0);
     // expert weights stream through L2 once (evict first); the hidden states,
@@ -214,6 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         for (int s = 0; s < kStages; ++s) { mbar_init(full_bar(s), kFullArrivals); mbar_init(empty_bar(s), 1); }
         for (int b = 0; b < 2; ++b) { mbar_init(tfull_bar(b), 1); mbar_init(tempty_bar(b), 4); }
         mbar_init(done_bar, 1);
+        for (int i = 0; i < kTQ; ++i) { mbar_init(tq_full_bar(i), 1); mbar_init(tq_empty_bar(i), kTQConsumers); }
         s_abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
@@ -224,6 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     }
     pdl_wait();  // the dispatch offsets and slot maps come from the previous kernel
     // tile list: rows and tiles per group, prefixes over groups
+    int multi = 0;  // some group has more than one 128-row block
     for (int g = tid; g < G; g += kThreads) {
         const bool shared = g >= p.E;
         int rows, base;
@@ -236,12 +269,14 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             base = b;
         }
         const int mt = (rows + BM - 1) / BM;
+        multi |= mt > 1 ? 1 : 0;
         tt.rows[g] = rows;
         tt.base[g] = base;
         tt.mpre[g + 1] = mt;
         for (int ph = 0; ph < 2; ++ph) tt.prefix[ph][g + 1] = mt * (group_n(p, ph, shared) / p.ph[ph].bn);
     }
-    __syncthreads();
+    // the same value in every thread of every CTA (all read the same offsets)
+    multi = __syncthreads_or(multi);
     if (warp < 3) {  // three inclusive scans, one per warp: tiles of each GEMM, row blocks
         int *arr = warp == 2 ? tt.mpre : tt.prefix[warp];
         int carry = 0;
@@ -263,7 +298,8 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
-    const int total = total_tiles(p, tt, G);
+    total = total_tiles(p, tt, G);
+    dyn = multi == 0;
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
@@ -280,7 +316,34 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         int stage = 0;
         uint32_t phase = 0;
         uint32_t filled = 0, last_parity = 0;  // per-stage bits, for the drain below
-        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
+        // Lane 0 picks the tiles and hands each to the CTA's other roles
+        // through the tile queue.  When a group has several 128-row blocks,
+        // its m-tiles share weights: they sit next to each other in the list
+        // and the CTAs take the list in waves (CTA c: tiles c, c + grid, ...),
+        // so those m-tiles run at the same moment and one DRAM read of the
+        // weights serves them all.  When no group has (decode), nothing is
+        // shared, and the tiles go out dynamically, the next one to whichever
+        // CTA is ready (an atomic counter, taken one tile ahead), which
+        // evens out tiles of unequal cost.
+        uint32_t ahead = (lane == 0 && dyn) ? atomicAdd(p.tile_ctr, 1u) : 0u;
+        for (int qi = 0;; ++qi) {
+            int tile = -1;
+            if (!dyn) {
+                tile = next_tile(qi);
+            } else {
+                if (lane == 0) {
+                    const int slot = qi % kTQ;
+                    if (mbar_wait(tq_empty_bar(slot), ((uint32_t)(qi / kTQ) & 1u) ^ 1u, &s_abort, p.status) &&
+                        !s_abort && ahead < (uint32_t)total) {
+                        tile = (int)ahead;
+                        ahead = atomicAdd(p.tile_ctr, 1u);
+                    }
+                    s_tq[slot] = tile;
+                    mbar_arrive(tq_full_bar(slot));
+                }
+                tile = __shfl_sync((1u << kLoaders) - 1u, tile, 0);
+            }
+            if (tile < 0) break;
             const Tile t = decode_tile(p, tt, G, tile);
             const bool gather = t.kind == kTileGU && !t.shared;
             const int q = t.shared ? 2 : (t.g < p.E_pub ? 0 : 1);
@@ -353,7 +416,9 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         // ------------------------------------------------ MMA issuer
         int stage = 0, it = 0;
         uint32_t phase = 0;
-        for (int tile = blockIdx.x; tile < total && !s_abort; tile += gridDim.x) {
+        for (int qi = 0;; ++qi) {
+            const int tile = next_tile(qi);
+            if (tile < 0) break;
             const Tile t = decode_tile(p, tt, G, tile);
             const uint32_t idesc = p.ph[t.ph].idesc;
             const int buf = it & 1;
@@ -394,7 +459,11 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         const uint32_t out_base = sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * 2 * kOutBufBytes);
         int out_parity = 0;
         int it = 0;
-        for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+        for (int qi = 0;; ++qi) {
+            int tile = 0;
+            if (lane == 0) tile = next_tile(qi);
+            tile = __shfl_sync(~0u, tile, 0);
+            if (tile < 0) break;
             const Tile t = decode_tile(p, tt, G, tile);
             const int buf = it & 1;
             const uint32_t use = (uint32_t)(it >> 1) & 1u;
@@ -598,7 +667,11 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         uint32_t sc = 0;                     // ring stages passed so far (the ring position)
         bool ok = true;
         auto drain = [&]() { cp_async_wait<0>(); };
-        for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
+        for (int qi = 0; ok; ++qi) {
+            int tile = 0;
+            if (lane == 0) tile = next_tile(qi);
+            tile = __shfl_sync(~0u, tile, 0);
+            if (tile < 0) break;
             const Tile t = decode_tile(p, tt, G, tile);
             if (t.kind != kTileGU || t.shared) {  // A comes through TMA: only follow the ring
                 sc += (uint32_t)t.nkb;
@@ -714,6 +787,7 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
     p.topk_idx = c.idx;
     p.hidden = c.hidden;
     p.ready = c.gemm_ready;
+    p.tile_ctr = c.gemm_ready + gemm_ready_words(s) - 1;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
     p.exec_priv_rows = c.audit.exec_priv_rows;
@@ -758,9 +832,19 @@ static bool grid_fits(const Ctx &c)
 
 }  // namespace
 
-cudaError_t launch_gateup(const Ctx &c) { return launch_tc(c, true, false); }
+// The two GEMMs in separate launches (diagnostics, and the fallback when the
+// persistent grid cannot be resident at once): each starts from tile 0.
+cudaError_t launch_gateup(const Ctx &c)
+{
+    const cudaError_t err = cudaMemsetAsync(c.gemm_ready + gemm_ready_words(c.s) - 1, 0, sizeof(uint32_t), c.stream);
+    return err == cudaSuccess ? launch_tc(c, true, false) : err;
+}
 
-cudaError_t launch_down(const Ctx &c) { return launch_tc(c, false, true); }
+cudaError_t launch_down(const Ctx &c)
+{
+    const cudaError_t err = cudaMemsetAsync(c.gemm_ready + gemm_ready_words(c.s) - 1, 0, sizeof(uint32_t), c.stream);
+    return err == cudaSuccess ? launch_tc(c, false, true) : err;
+}
 
 cudaError_t launch_experts(const Ctx &c, bool zero_ready)
 {

@@ -11,11 +11,12 @@ namespace pmpe {
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Each routed group adds at most one partial 128-row block beyond R/128; the
-// shared-expert group covers the T tokens.
+// shared-expert group covers the T tokens.  The last word is the expert
+// kernel's tile counter (the next tile of its list to hand out).
 size_t gemm_ready_words(const Shape &s)
 {
     const size_t R = (size_t)s.T * (size_t)s.k;
-    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 1;
+    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 2;
 }
 
 static bool shape_ok(const Shape &s)
