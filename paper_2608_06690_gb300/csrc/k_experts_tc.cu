@@ -113,6 +113,27 @@ struct TcParams {
     // take tiles in list order, each when it is ready for one
     uint32_t *tile_ctr;
     uint32_t *exec_rows, *exec_tiles, *exec_priv_rows, *shared_rows, *status;
+    // fused dispatch (the launch follows the router directly): the CTAs first
+    // derive the dispatch order from the router's per-tile counts and route
+    // log, write the slot maps, clear the counters above, and meet at a grid
+    // barrier (grid_bar, zeroed by the router) before the first tile
+    int fuse_dispatch;
+    const int32_t *ticket;      // [T, k] 128 * router tile + position among the tile's rows of its expert
+    const float *w_route;       // [T, k] routing weights
+    const uint32_t *tile_counts;  // [E][slots4] rows of each expert per router tile
+    int slots, slots4;
+    uint32_t *counts_w, *offsets_w;  // written: rows and first slot of each expert
+    int32_t *slot_of_w, *tok_of_slot_w;
+    float *w_of_slot_w;
+    uint32_t *grid_bar;
+    int clear_words;            // readiness counters and the tile counter, from `ready`
+    // small batches (every expert at most one 128-row block): the first
+    // `prefetch_tiles` gate/up tiles of the list of all experts have their
+    // weights prefetched into L2 by the CTA of the same index, before the
+    // launch waits for the routing (the weights are inputs, not results of
+    // the kernels before); 0 = off
+    int prefetch_tiles;
+    const bf16 *gate_w[2], *up_w[2];  // [E_pool * I, H] public / private
     // optional FP32: the gate and up accumulators saved for the backward,
     // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
     // experts (gu_save / gu_save_sh maps for whole 32-row blocks)
@@ -190,6 +211,39 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
 
 // ---------------------------------------------------------------- kernel
 
+// Every CTA of the grid arrives, then waits (bounded) until `target`
+// arrivals are counted.  The grid is resident all at once (checked before the
+// launch), so the wait ends.  Writes before the barrier, by any thread of any
+// CTA, are visible after it.  Returns false, with the timeout recorded, when
+// the wait expired.
+__device__ bool grid_barrier(uint32_t *ctr, uint32_t target, uint32_t *status)
+{
+    __shared__ int s_ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int ok = 1;
+        __threadfence();
+        atomicAdd(ctr, 1u);
+        const unsigned long long t0 = globaltimer_ns();
+        while (ld_acquire_gpu(ctr) < target) {
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                if (status) atomicOr(status, PMPE_STATUS_PIPELINE_TIMEOUT);
+                ok = 0;
+                break;
+            }
+            __nanosleep(32);
+        }
+        __threadfence();
+        s_ok = ok;
+    }
+    __syncthreads();
+    return s_ok != 0;
+}
+
+// Shared-memory bytes the fused dispatch needs for its per-expert prefix of
+// the router tiles' counts ([E][slots + 1] words, inside the ring).
+constexpr size_t fused_dispatch_smem(int E, int slots) { return (size_t)E * (size_t)(slots + 1) * 4u; }
+
 __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcParams p, const __grid_constant__ TcMaps maps)
 {
     extern __shared__ uint8_t dsmem[];
@@ -254,7 +308,84 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                      "r"(kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
     }
-    pdl_wait();  // the dispatch offsets and slot maps come from the previous kernel
+    if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles) {
+        // weights of gate/up tile blockIdx.x of the list of all experts: 128
+        // gate rows and 128 up rows, each block contiguous (bulk L2 prefetch)
+        const int nt = p.I / 128;
+        const int e = (int)blockIdx.x / nt, n = (int)blockIdx.x - e * nt;
+        if (e < p.E) {
+            const int q = e < p.E_pub ? 0 : 1;
+            const size_t row0 = (size_t)(q ? e - p.E_pub : e) * p.I + (size_t)n * 128;
+            const uint32_t bytes = (uint32_t)(128u * (uint32_t)p.H * 2u);
+            bulk_prefetch_l2(p.gate_w[q] + row0 * p.H, bytes);
+            bulk_prefetch_l2(p.up_w[q] + row0 * p.H, bytes);
+        }
+    }
+    pdl_wait();  // the dispatch offsets and slot maps (or the route log) come from the previous kernel
+    if (p.fuse_dispatch) {
+        // ---- the dispatch order, as dispatch_kernel derives it.  pre[e][s]:
+        // rows of expert e in the router tiles before tile s (in the ring,
+        // which no load has touched yet), its total = the expert's rows
+        uint32_t *pre = reinterpret_cast<uint32_t *>(dsmem + (sbase - smem_u32(dsmem)));
+        const int sp = p.slots + 1;
+        for (int g = tid; g < p.E; g += kThreads) {
+            const uint32_t *tc = p.tile_counts + (size_t)g * p.slots4;
+            uint32_t acc = 0;
+            int s2 = 0;
+            for (; s2 + 4 <= p.slots; s2 += 4) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(tc + s2);  // slots4: rows 16-byte aligned
+                pre[g * sp + s2] = acc; acc += v.x;
+                pre[g * sp + s2 + 1] = acc; acc += v.y;
+                pre[g * sp + s2 + 2] = acc; acc += v.z;
+                pre[g * sp + s2 + 3] = acc; acc += v.w;
+            }
+            for (; s2 < p.slots; ++s2) { pre[g * sp + s2] = acc; acc += tc[s2]; }
+            pre[g * sp + p.slots] = acc;
+            tt.rows[g] = (int)acc;
+        }
+        __syncthreads();
+        if (warp == 0) {  // exclusive prefix over the experts: their first slots
+            int carry = 0;
+            for (int b = 0; b < p.E; b += 32) {
+                const int v0 = b + lane < p.E ? tt.rows[b + lane] : 0;
+                int v = v0;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int y = __shfl_up_sync(~0u, v, off);
+                    if (lane >= off) v += y;
+                }
+                if (b + lane < p.E) tt.base[b + lane] = carry + v - v0;
+                carry += __shfl_sync(~0u, v, 31);
+            }
+        }
+        __syncthreads();
+        if (blockIdx.x == 0) {
+            for (int g = tid; g < p.E; g += kThreads) {
+                p.offsets_w[g] = (uint32_t)tt.base[g];
+                p.counts_w[g] = (uint32_t)tt.rows[g];
+            }
+            if (tid == 0) p.offsets_w[p.E] = (uint32_t)(tt.base[p.E - 1] + tt.rows[p.E - 1]);
+            for (int i = tid; i < p.clear_words; i += kThreads) p.ready[i] = 0u;
+        }
+        // this CTA's share of the routed rows r = (t, j): slot = first slot of
+        // its expert + the expert's rows in earlier router tiles + its
+        // position in its tile (ticket = 128 * tile + position)
+        for (int r = blockIdx.x * kThreads + tid; r < p.R; r += gridDim.x * kThreads) {
+            const int e = p.topk_idx[r];
+            if ((unsigned)e >= (unsigned)p.E) {  // never produced by the router
+                if (p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+                continue;
+            }
+            const int tk = p.ticket[r];
+            const int ts = min(tk >> 7, p.slots);
+            const int slot = tt.base[e] + (int)pre[e * sp + ts] + (tk & 127);
+            if ((unsigned)slot >= (unsigned)p.R) continue;  // only a corrupt ticket could fail this
+            p.slot_of_w[r] = slot;
+            p.tok_of_slot_w[slot] = r / p.k;
+            p.w_of_slot_w[slot] = p.w_route[r];
+        }
+        if (!grid_barrier(p.grid_bar, gridDim.x, p.status)) s_abort = 1;
+    }
     // tile list: rows and tiles per group, prefixes over groups
     int multi = 0;  // some group has more than one 128-row block
     for (int g = tid; g < G; g += kThreads) {
@@ -263,6 +394,9 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         if (shared) {
             rows = p.T;
             base = 0;
+        } else if (p.fuse_dispatch) {  // derived above
+            rows = min(tt.rows[g], p.R);
+            base = min(tt.base[g], p.R - rows);
         } else {  // clamped to [0, R): only a corrupt workspace could make this matter
             const int b = min((int)p.offsets[g], p.R), e = min(max((int)p.offsets[g + 1], b), p.R);
             rows = e - b;
@@ -766,8 +900,9 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
     return ok;
 }
 
-// One persistent launch of the gate/up tiles, the down tiles, or both.
-cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
+// One persistent launch of the gate/up tiles, the down tiles, or both (and,
+// with fuse_dispatch, the dispatch before them).
+cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = false)
 {
     const Shape &s = c.s;
     TcParams p;
@@ -787,12 +922,35 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down)
     p.topk_idx = c.idx;
     p.hidden = c.hidden;
     p.ready = c.gemm_ready;
-    p.tile_ctr = c.gemm_ready + gemm_ready_words(s) - 1;
+    if (gu && s.T <= BM && s.I % 128 == 0) {
+        // at most T rows per expert: no expert has a second 128-row block
+        p.prefetch_tiles = std::min(s.E() * (s.I / 128), 96);
+        for (int q = 0; q < 2; ++q) {
+            p.gate_w[q] = c.gate[q];
+            p.up_w[q] = c.up[q];
+        }
+    }
+    p.tile_ctr = c.gemm_ready + gemm_ready_words(s) - 2;
     p.exec_rows = c.audit.exec_rows;
     p.exec_tiles = c.audit.exec_tiles;
     p.exec_priv_rows = c.audit.exec_priv_rows;
     p.shared_rows = c.audit.shared_rows;
     p.status = c.audit.status;
+    if (fuse_dispatch) {
+        p.fuse_dispatch = 1;
+        p.ticket = c.ticket;
+        p.w_route = c.w;
+        p.tile_counts = c.tile_counts;
+        p.slots = router_slots(s.T);
+        p.slots4 = router_slots4(s.T);
+        p.counts_w = c.counts;
+        p.offsets_w = c.offsets;
+        p.slot_of_w = c.slot_of;
+        p.tok_of_slot_w = c.tok_of_slot;
+        p.w_of_slot_w = c.w_of_slot;
+        p.grid_bar = c.gemm_ready + gemm_ready_words(s) - 1;
+        p.clear_words = (int)gemm_ready_words(s) - 1;
+    }
     bool ok = true;
     if (gu) ok &= fill_phase(c, kGateUp, p, maps);
     if (down) ok &= fill_phase(c, kDown, p, maps);
@@ -836,27 +994,35 @@ static bool grid_fits(const Ctx &c)
 // persistent grid cannot be resident at once): each starts from tile 0.
 cudaError_t launch_gateup(const Ctx &c)
 {
-    const cudaError_t err = cudaMemsetAsync(c.gemm_ready + gemm_ready_words(c.s) - 1, 0, sizeof(uint32_t), c.stream);
+    const cudaError_t err = cudaMemsetAsync(c.gemm_ready + gemm_ready_words(c.s) - 2, 0, sizeof(uint32_t), c.stream);
     return err == cudaSuccess ? launch_tc(c, true, false) : err;
 }
 
 cudaError_t launch_down(const Ctx &c)
 {
-    const cudaError_t err = cudaMemsetAsync(c.gemm_ready + gemm_ready_words(c.s) - 1, 0, sizeof(uint32_t), c.stream);
+    const cudaError_t err = cudaMemsetAsync(c.gemm_ready + gemm_ready_words(c.s) - 2, 0, sizeof(uint32_t), c.stream);
     return err == cudaSuccess ? launch_tc(c, false, true) : err;
 }
 
-cudaError_t launch_experts(const Ctx &c, bool zero_ready)
+// The dispatch can run inside the persistent launch when that launch's grid
+// is resident at once (its grid barrier) and the prefix table of the router
+// tiles' counts fits its ring.
+bool experts_fuse_dispatch(const Ctx &c)
+{
+    return grid_fits(c) && fused_dispatch_smem(c.s.E(), router_slots(c.s.T)) <= (size_t)(kStages * kStageBytes);
+}
+
+cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool fuse_dispatch)
 {
     if (!grid_fits(c)) {  // the two GEMMs one after the other: no cross-CTA wait
         const cudaError_t err = launch_gateup(c);
         return err == cudaSuccess ? launch_down(c) : err;
     }
-    if (zero_ready) {
+    if (zero_ready && !fuse_dispatch) {
         const cudaError_t err = cudaMemsetAsync(c.gemm_ready, 0, sizeof(uint32_t) * gemm_ready_words(c.s), c.stream);
         if (err != cudaSuccess) return err;
     }
-    return launch_tc(c, true, true);
+    return launch_tc(c, true, true, fuse_dispatch);
 }
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn()

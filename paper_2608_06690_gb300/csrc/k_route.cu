@@ -613,6 +613,7 @@ struct ClusterRouterParams {
     int32_t *ticket;     // [T, k] 128 * tile slot + position among the tile's rows of its expert
     uint32_t *tile_counts;  // [E][slots4] rows of each expert per tile (a column per tile slot)
     uint32_t *route_count, *route_priv_rows, *status;
+    uint32_t *gemm_bar;  // the expert launch's grid barrier counter, zeroed here
 };
 
 struct ClusterRouterMaps {
@@ -844,6 +845,7 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     }
     pdl_trigger();
     pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
+    if (blockIdx.x == 0 && tid == 0 && p.gemm_bar) *p.gemm_bar = 0u;  // read by the expert launch after this grid
 
     // ---- tile assignment (as router_tc_kernel): resolve and rank in one pass
     const int per = ((p.T + kCThreads - 1) / kCThreads + 15) & ~15;
@@ -1292,6 +1294,7 @@ cudaError_t launch_route(const Ctx &c)
     p.route_count = c.audit.route_count;
     p.route_priv_rows = c.audit.route_priv_rows;
     p.status = c.audit.status;
+    p.gemm_bar = c.gemm_ready + gemm_ready_words(s) - 1;
     bool ok = encode_2d(&maps.hidden, c.hidden, s.H, s.T, kCTile);
     ok &= encode_2d(&maps.router[0], c.router_pub, s.H, s.E_pub, 128);
     ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, 128);

@@ -11,12 +11,13 @@ namespace pmpe {
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Each routed group adds at most one partial 128-row block beyond R/128; the
-// shared-expert group covers the T tokens.  The last word is the expert
-// kernel's tile counter (the next tile of its list to hand out).
+// shared-expert group covers the T tokens.  The last two words are the expert
+// kernel's tile counter (the next tile of its list to hand out) and its grid
+// barrier counter.
 size_t gemm_ready_words(const Shape &s)
 {
     const size_t R = (size_t)s.T * (size_t)s.k;
-    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 2;
+    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 3;
 }
 
 static bool shape_ok(const Shape &s)
@@ -214,12 +215,16 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     if (c.s.T == 0 || stages == 0) return PMPE_OK;
     if (stages & ~PMPE_STAGE_ALL) return PMPE_ERR_INVALID_ARG;
     cudaError_t err = cudaSuccess;
+    // The dispatch runs inside the persistent expert launch when that launch
+    // follows the router in this call (the router zeroes its grid barrier).
+    const bool fuse = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && (stages & PMPE_STAGE_GATEUP) &&
+                      (stages & PMPE_STAGE_DOWN) && experts_fuse_dispatch(c);
     if (err == cudaSuccess && (stages & PMPE_STAGE_ROUTE)) err = launch_route(c);
-    if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE)) err = launch_permute(c);
+    if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE) && !fuse) err = launch_permute(c);
     if ((stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN)) {
         // one persistent launch; its readiness counters are cleared by the
-        // dispatch when the dispatch runs in this call
-        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_PERMUTE));
+        // dispatch when the dispatch runs in this call (inside it, when fused)
+        if (err == cudaSuccess) err = launch_experts(c, !(stages & PMPE_STAGE_PERMUTE), fuse);
     } else {
         if (err == cudaSuccess && (stages & PMPE_STAGE_GATEUP)) err = launch_gateup(c);
         if (err == cudaSuccess && (stages & PMPE_STAGE_DOWN)) err = launch_down(c);

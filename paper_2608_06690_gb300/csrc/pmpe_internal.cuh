@@ -146,7 +146,11 @@ cudaError_t launch_backward_wgrad(const Ctx &c, const bf16 *dout_rows, const bf1
 // Gate/up and down in one persistent launch (down tiles wait for their
 // activation rows); zero_ready clears the readiness counters first.  When the
 // device cannot host one CTA per SM at once, the two GEMMs run as two launches.
-cudaError_t launch_experts(const Ctx &c, bool zero_ready);
+// The persistent gate/up + down launch.  With fuse_dispatch (the router ran
+// just before in the same call, and experts_fuse_dispatch holds) the launch
+// also derives the dispatch order itself, in place of launch_permute.
+cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool fuse_dispatch);
+bool experts_fuse_dispatch(const Ctx &c);
 cudaError_t launch_combine(const Ctx &c);
 // The token rows of the dispatch slots of groups g0 .. g1 - 1 copied from the
 // hidden states into the workspace's dispatched-row matrix (a_perm), which the

@@ -204,6 +204,12 @@ __device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap *map
 
 // Make this thread's completed generic-proxy shared-memory writes (e.g. from
 // cp.async) visible to the async proxy that tcgen05.mma reads through.
+// Prefetch [ptr, ptr + bytes) into L2 (16-byte aligned, a multiple of 16 bytes).
+__device__ __forceinline__ void bulk_prefetch_l2(const void *ptr, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(ptr), "r"(bytes) : "memory");
+}
+
 // Fetch a tensor map (a kernel parameter) into the TMA unit's descriptor
 // cache ahead of its first use.
 __device__ __forceinline__ void prefetch_tmap(const void *map)
