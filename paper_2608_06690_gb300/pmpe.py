@@ -41,12 +41,12 @@ STAGE_DOWN = 0x08
 STAGE_COMBINE = 0x10
 STAGE_ALL = 0x1F
 
-# Kernels one full forward launches: router/top-k (with the policy resolve),
-# the dispatch order, one persistent launch of the gate/up GEMM (rows
-# gathered from the hidden states) and the down GEMM, and the combine (plus
-# one memset of the per-expert counters, which is not a kernel of this
-# library).
-KERNELS_PER_FORWARD = 4
+# Kernels one full forward launches: the router/top-k (with the policy
+# resolve), one persistent launch that derives the dispatch order and runs the
+# gate/up GEMM (rows gathered from the hidden states) and the down GEMM, and
+# the combine; no memset.  (Where the persistent grid cannot be resident at
+# once, the dispatch is a kernel of its own and the GEMMs two launches: 5.)
+KERNELS_PER_FORWARD = 3
 # kernels one private-branch backward launches: the dispatched rows of the
 # private experts, dout row gather, the dL/da GEMM, the gate/up recompute GEMM
 # with the SwiGLU backward, router gradient, router weight-gradient partials
