@@ -543,7 +543,7 @@ def measure_forward(pmpe, cfg, w, h, pol, dev, args, ws_n, barrier, nvml, flush)
         "expert_load": {"touched": work["touched_experts"], "max_rows": int(counts.max()),
                         "mean_rows_public": float(counts[:s.E_pub].mean()),
                         "mean_rows_private": float(counts[s.E_pub:].mean())},
-        "gpu_launches": pmpe.KERNELS_PER_FORWARD * args.steps,
+        "gpu_launches": pmpe.kernels_per_forward(s) * args.steps,
         "clocks": clocks,
         "wall_s_timed_region": t_wall,
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h.numel() * 2 + pol.numel(),

@@ -79,6 +79,7 @@ constexpr int kLoaders = 3;                   // TMA-issuing lanes of warp 0
 constexpr int kGatherThreads = 32 * kGatherWarps;
 constexpr int kFullArrivals = kLoaders + kGatherThreads;  // per ring stage
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
+constexpr int kPrefetchTiles = 96;            // gate/up tiles (1 MB of weights each) prefetched into L2 at small batches
 constexpr int kTQ = 8;                        // tile queue entries (tile indices handed to the CTA's roles)
 constexpr int kTQConsumers = 1 + 4 + kGatherWarps;  // MMA thread, epilogue warps, gather warps (one lane each)
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
@@ -922,9 +923,11 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = fal
     p.topk_idx = c.idx;
     p.hidden = c.hidden;
     p.ready = c.gemm_ready;
-    if (gu && s.T <= BM && s.I % 128 == 0) {
+    if (gu && s.T <= BM && s.I % 128 == 0 && (long long)s.H * s.I >= (1ll << 20)) {
         // at most T rows per expert: no expert has a second 128-row block
-        p.prefetch_tiles = std::min(s.E() * (s.I / 128), 96);
+        // (small experts, as in the tiny layer: the launch is too short to
+        // gain from it)
+        p.prefetch_tiles = std::min(s.E() * (s.I / 128), kPrefetchTiles);
         for (int q = 0; q < 2; ++q) {
             p.gate_w[q] = c.gate[q];
             p.up_w[q] = c.up[q];
@@ -1006,10 +1009,13 @@ cudaError_t launch_down(const Ctx &c)
 
 // The dispatch can run inside the persistent launch when that launch's grid
 // is resident at once (its grid barrier) and the prefix table of the router
-// tiles' counts fits its ring.
+// tiles' counts fits its ring.  For small experts (fewer than 2^20 weights a
+// projection: the tiny test layer) the launch is short and the grid barrier
+// costs more than the dispatch kernel it saves (40.1 vs 38.2 us a step).
 bool experts_fuse_dispatch(const Ctx &c)
 {
-    return grid_fits(c) && fused_dispatch_smem(c.s.E(), router_slots(c.s.T)) <= (size_t)(kStages * kStageBytes);
+    return (long long)c.s.H * c.s.I >= (1ll << 20) && grid_fits(c) &&
+           fused_dispatch_smem(c.s.E(), router_slots(c.s.T)) <= (size_t)(kStages * kStageBytes);
 }
 
 cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool fuse_dispatch)

@@ -687,12 +687,12 @@ __device__ __forceinline__ float clean_logit(float x) { return x != x ? -INFINIT
 //
 // Thread pair (token tl, chunk c) sums the chunk's 32 partial logits over
 // the cluster's CTAs in CTA order (rcv[src][tl][expert]; the sums replace
-// slot 0), stores their selection keys in slot 1 and records the chunk's
-// softmax partial (max, sum of exp(x - max)); experts past the pool have no
-// key.  The ncp lanes of a token (ncp = chunks rounded up to a power of two;
-// padding lanes hold no key) then take k + 1 passes: the group's largest key
-// left (a max over the lane's keys, then over the lanes by shuffles), which
-// its owner removes.  The keys of the passes are the candidates in key
+// slot 0), turns them into selection keys held in registers and records the
+// chunk's softmax partial (max, sum of exp(x - max)); experts past the pool
+// have no key.  The ncp lanes of a token (ncp = chunks rounded up to a power
+// of two; padding lanes hold no key) then take k + 1 passes: the group's
+// largest key left (a max over the lane's keys, then over the lanes by
+// shuffles), which its owner removes.  The keys of the passes are the candidates in key
 // order; they are the exact top k in the exact order whenever no two
 // consecutive ones of the first k + 1 share a bucket.  Otherwise (near-equal
 // logits) the warp repeats the selection with the exact comparison of
@@ -715,8 +715,10 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
         const int nvalid = (tok_ok && c < nc) ? min(kChunk, P - c * kChunk) : 0;
         float *row = rcv + (size_t)(tok_ok ? tl : 0) * pitch;  // slot 0: the token's summed logits
         float *sum = row + c * kChunk;
-        uint32_t *key = reinterpret_cast<uint32_t *>(rcv + (size_t)tpc * pitch) + (sum - rcv);  // slot 1
         float mx = -INFINITY, ssum = 0.f;
+        uint32_t key[32];  // this lane's selection keys (0: no candidate)
+#pragma unroll
+        for (int i = 0; i < 32; ++i) key[i] = 0u;
         if (nvalid > 0) {
             float v[32];
 #pragma unroll
@@ -735,9 +737,9 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
             float4 *w4 = reinterpret_cast<float4 *>(sum);
 #pragma unroll
             for (int i = 0; i < 8; ++i) w4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-#pragma unroll 4
+#pragma unroll
             for (int i = 0; i < 32; ++i) {
-                const float x = clean_logit(sum[i]);
+                const float x = clean_logit(v[i]);
                 key[i] = i < nvalid ? logit_key(x, c * kChunk + i) : 0u;
                 mx = i < nvalid ? fmaxf(mx, x) : mx;
             }
@@ -745,31 +747,24 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
                 for (int i = 0; i < nvalid; ++i) ssum += expf(clean_logit(sum[i]) - mx);
         }
         __syncwarp();
-        // ---- fast path: k + 1 passes over the keys
+        // ---- fast path: k + 1 passes over the keys, held in registers
         bool amb = false;
         uint32_t prev = 0u;
         for (int j = 0; j <= K; ++j) {
-            uint32_t m = 0u;
-            if (nvalid > 0) {
-                uint32_t m4[4] = {0u, 0u, 0u, 0u};
+            uint32_t m8[8];
 #pragma unroll
-                for (int i = 0; i < 32; i += 4) {
-                    const uint4 k4 = *reinterpret_cast<const uint4 *>(key + i);
-                    m4[0] = max(m4[0], k4.x);
-                    m4[1] = max(m4[1], k4.y);
-                    m4[2] = max(m4[2], k4.z);
-                    m4[3] = max(m4[3], k4.w);
-                }
-                m = max(max(m4[0], m4[1]), max(m4[2], m4[3]));
-            }
+            for (int i = 0; i < 8; ++i) m8[i] = max(max(key[4 * i], key[4 * i + 1]), max(key[4 * i + 2], key[4 * i + 3]));
+            uint32_t m = max(max(max(m8[0], m8[1]), max(m8[2], m8[3])), max(max(m8[4], m8[5]), max(m8[6], m8[7])));
             for (int d = 1; d < ncp; d <<= 1) m = max(m, __shfl_xor_sync(~0u, m, d));
+            // keys are unique: the lane holding the winner removes it
+#pragma unroll
+            for (int i = 0; i < 32; ++i) key[i] = key[i] == m ? 0u : key[i];
             const int id = 255 - (int)(m & 255u);
-            if (m != 0u && nvalid > 0 && (id >> 5) == c) key[id & 31] = 0u;  // the owner removes the winner
             if (j > 0) amb |= (m >> 8) == (prev >> 8);
             if (j < K && c == 0 && tok_ok) sel_e[tl * K + j] = id;
             prev = m;
-            __syncwarp();
         }
+        __syncwarp();
         amb &= tok_ok;
         if (__any_sync(~0u, amb)) {
             // ---- exact path for the whole warp: k passes with the exact

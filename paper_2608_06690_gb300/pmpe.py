@@ -44,9 +44,17 @@ STAGE_ALL = 0x1F
 # Kernels one full forward launches: the router/top-k (with the policy
 # resolve), one persistent launch that derives the dispatch order and runs the
 # gate/up GEMM (rows gathered from the hidden states) and the down GEMM, and
-# the combine; no memset.  (Where the persistent grid cannot be resident at
-# once, the dispatch is a kernel of its own and the GEMMs two launches: 5.)
+# the combine; no memset.  For small experts (H * I < 2^20, the tiny test
+# layer) the dispatch is a kernel of its own: 4.  (Where the persistent grid
+# cannot be resident at once, the GEMMs take two launches as well.)
 KERNELS_PER_FORWARD = 3
+
+
+def kernels_per_forward(shape) -> int:
+    """Kernels of this library one full forward of `shape` launches on a GPU
+    where the persistent expert grid is resident at once (the rule the
+    library applies when it launches the forward)."""
+    return 3 if shape.H * shape.I >= (1 << 20) else 4
 # kernels one private-branch backward launches: the dispatched rows of the
 # private experts, dout row gather, the dL/da GEMM, the gate/up recompute GEMM
 # with the SwiGLU backward, router gradient, router weight-gradient partials
