@@ -81,6 +81,7 @@ constexpr int kFullArrivals = kLoaders + kGatherThreads;  // per ring stage
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
 constexpr int kPrefetchTiles = 96;            // gate/up tiles (1 MB of weights each) prefetched into L2 at small batches
 constexpr int kTQ = 8;                        // tile queue entries (tile indices handed to the CTA's roles)
+constexpr int kTailWaves = 2;                 // waves of tiles at the list's end handed out dynamically
 constexpr int kTQConsumers = 1 + 4 + kGatherWarps;  // MMA thread, epilogue warps, gather warps (one lane each)
 constexpr int kOutBox = 32;                   // output staged and stored as 32 x 32 BF16 boxes (2 KB)
 constexpr int kOutBufBytes = kOutBox * kOutBox * 2;
@@ -267,15 +268,13 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     // Entry i of the CTA's tile sequence, for a consumer role (one thread):
     // -1 at the end of the list or after an abort.  In wave order every role
     // computes it; dynamically, warp 0 hands it out through the tile queue.
-    bool dyn = false;
-    int total = 0;
+    // The list's tiles [0, tail) go out in waves (CTA c: c, c + grid, ...,
+    // n_wave of them), the rest [tail, total) dynamically, through the queue.
+    int total = 0, tail = 0, n_wave = 0;
     auto next_tile = [&](int i) -> int {
-        if (!dyn) {
-            const long long st = (long long)blockIdx.x + (long long)i * gridDim.x;
-            return (st < total && !s_abort) ? (int)st : -1;
-        }
-        const int slot = i % kTQ;
-        if (!mbar_wait(tq_full_bar(slot), (uint32_t)(i / kTQ) & 1u, &s_abort, p.status)) return -1;
+        if (i < n_wave) return s_abort ? -1 : (int)blockIdx.x + i * (int)gridDim.x;
+        const int d = i - n_wave, slot = d % kTQ;
+        if (!mbar_wait(tq_full_bar(slot), (uint32_t)(d / kTQ) & 1u, &s_abort, p.status)) return -1;
         const int t = s_tq[slot];
         mbar_arrive(tq_empty_bar(slot));
         return t;
@@ -434,7 +433,12 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     tc_fence_after();
     const uint32_t tmem_base = s_tmem;
     total = total_tiles(p, tt, G);
-    dyn = multi == 0;
+    // waves keep an expert's m-tiles (which share weights) running together;
+    // the last kTailWaves waves, and every tile when no group has a second
+    // 128-row block (nothing to share), go out dynamically, so that the CTAs
+    // finish together
+    tail = multi == 0 ? 0 : max(0, total - kTailWaves * (int)gridDim.x);
+    n_wave = (int)blockIdx.x < tail ? (tail - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
     if (warp == 0 && lane < kLoaders) {
         // ------------------------------------------------ TMA producers
@@ -460,18 +464,19 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         // shared, and the tiles go out dynamically, the next one to whichever
         // CTA is ready (an atomic counter, taken one tile ahead), which
         // evens out tiles of unequal cost.
-        uint32_t ahead = (lane == 0 && dyn) ? atomicAdd(p.tile_ctr, 1u) : 0u;
+        uint32_t ahead = 0u;  // lane 0: the next dynamic tile, taken one ahead
         for (int qi = 0;; ++qi) {
             int tile = -1;
-            if (!dyn) {
+            if (qi < n_wave) {
                 tile = next_tile(qi);
             } else {
                 if (lane == 0) {
-                    const int slot = qi % kTQ;
-                    if (mbar_wait(tq_empty_bar(slot), ((uint32_t)(qi / kTQ) & 1u) ^ 1u, &s_abort, p.status) &&
+                    const int d = qi - n_wave, slot = d % kTQ;
+                    if (d == 0) ahead = (uint32_t)tail + atomicAdd(p.tile_ctr, 1u);
+                    if (mbar_wait(tq_empty_bar(slot), ((uint32_t)(d / kTQ) & 1u) ^ 1u, &s_abort, p.status) &&
                         !s_abort && ahead < (uint32_t)total) {
                         tile = (int)ahead;
-                        ahead = atomicAdd(p.tile_ctr, 1u);
+                        ahead = (uint32_t)tail + atomicAdd(p.tile_ctr, 1u);
                     }
                     s_tq[slot] = tile;
                     mbar_arrive(tq_full_bar(slot));
