@@ -614,6 +614,14 @@ struct ClusterRouterParams {
     uint32_t *tile_counts;  // [E][slots4] rows of each expert per tile (a column per tile slot)
     uint32_t *route_count, *route_priv_rows, *status;
     uint32_t *gemm_bar;  // the expert launch's grid barrier counter, zeroed here
+    // With dispatch != 0 (T <= 128: each pool fills at most one tile) the
+    // router also writes the dispatch order, and clears the expert launch's
+    // gemm_ready_words readiness counters, so that no dispatch step follows.
+    int dispatch;
+    uint32_t *offsets, *counts, *gemm_ready;
+    int gemm_ready_words;
+    int32_t *slot_of, *tok_of_slot;
+    float *w_of_slot;
 };
 
 struct ClusterRouterMaps {
@@ -841,6 +849,10 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     pdl_trigger();
     pdl_wait();  // the caller's hidden states / policy may come from the previous kernel
     if (blockIdx.x == 0 && tid == 0 && p.gemm_bar) *p.gemm_bar = 0u;  // read by the expert launch after this grid
+    if (p.dispatch && blockIdx.x == 0) {
+        for (int i = tid; i < p.gemm_ready_words; i += kCThreads) p.gemm_ready[i] = 0u;
+        if (tid == 0) p.offsets[p.E_pub + p.E_priv] = (uint32_t)(p.T * p.k);
+    }
 
     // ---- tile assignment (as router_tc_kernel): resolve and rank in one pass
     const int per = ((p.T + kCThreads - 1) / kCThreads + 15) & ~15;
@@ -862,8 +874,16 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     }
     const int E = p.E_pub + p.E_priv;
     if (!has_tile) {  // uniform over the cluster: no tile for this slot
-        if (q == 0)
+        if (q == 0) {
             for (int e = tid; e < E; e += kCThreads) p.tile_counts[(size_t)e * p.slots4 + slot] = 0u;
+            if (p.dispatch) {  // a pool without tokens: its experts have no rows
+                for (int e = tid; e < E; e += kCThreads)
+                    if (e < p.E_pub ? nd == 0 : na == 0) {
+                        p.offsets[e] = e < p.E_pub ? 0u : (uint32_t)(nd * p.k);
+                        p.counts[e] = 0u;
+                    }
+            }
+        }
         return;
     }
     const int rows = min(kCTile, (pool ? na : nd) - m0);
@@ -1109,6 +1129,38 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             if (c && p.route_count) atomicAdd(&p.route_count[eg], c);
         }
     }
+    // Dispatch order (when the tile is its pool's only one): the pool's rows
+    // start after every earlier pool's (the public pool's nd tokens, k rows
+    // each), its experts' rows follow one another in id order, and a row's
+    // slot adds its position among its expert's rows of the tile, i.e. the
+    // order offset[e] + (rows of e in earlier tiles, none) + position.
+    uint32_t *s_first = reinterpret_cast<uint32_t *>(sgen);  // [P] first slot per pool expert (ring, free again)
+    if (p.dispatch) {
+        if (warp == 0) {
+            uint32_t carry = pool ? (uint32_t)(nd * K) : 0u;
+            for (int b = 0; b < P; b += 32) {
+                const int i = b + lane;
+                const uint32_t c =
+                    i < P ? __popc(sfull[i * 4]) + __popc(sfull[i * 4 + 1]) + __popc(sfull[i * 4 + 2]) + __popc(sfull[i * 4 + 3])
+                          : 0u;
+                uint32_t v = c;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const uint32_t y = __shfl_up_sync(~0u, v, off);
+                    if (lane >= off) v += y;
+                }
+                if (i < P) {
+                    s_first[i] = carry + v - c;
+                    if (q == 0) {
+                        p.offsets[base + i] = carry + v - c;
+                        p.counts[base + i] = c;
+                    }
+                }
+                carry += __shfl_sync(~0u, v, 31);
+            }
+        }
+        __syncthreads();
+    }
     // one thread per routed row (token, j) of this CTA's tokens
     if (!abort_now) {
         for (int wi = tid; wi < ntok * K; wi += kCThreads) {
@@ -1121,9 +1173,18 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             int rank = (int)__popc(sfull[be * 4 + wd] & below);
             for (int w2 = 0; w2 < wd; ++w2) rank += (int)__popc(sfull[be * 4 + w2]);
             const float2 m = tmeta[tl];
+            const float wt = expf(sel_v[wi] - m.x) / m.y;
             p.idx[(size_t)t * K + j] = base + be;
             p.ticket[(size_t)t * K + j] = (int32_t)(slot * kCTile + rank);
-            p.w[(size_t)t * K + j] = expf(sel_v[wi] - m.x) / m.y;
+            p.w[(size_t)t * K + j] = wt;
+            if (p.dispatch) {
+                const uint32_t sl = s_first[be] + (uint32_t)rank;
+                if (sl < (uint32_t)(p.T * K)) {  // only a lost cluster exchange could fail this
+                    p.slot_of[(size_t)t * K + j] = (int32_t)sl;
+                    p.tok_of_slot[sl] = t;
+                    p.w_of_slot[sl] = wt;
+                }
+            }
             if (j == 0) {
                 p.tau[t] = pool ? 1 : 0;
                 if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], pool ? (unsigned)K : 0u);
@@ -1267,10 +1328,15 @@ bool route_uses_cluster_kernel(const Shape &s, int unmasked, int num_sms)
     return cluster_router_smem(P, s.k, cluster_router_nq(s.H, s.T, num_sms)) <= kCMaxDynSmem;
 }
 
-cudaError_t launch_route(const Ctx &c)
+bool route_writes_dispatch(const Ctx &c)
+{
+    return c.s.T <= kCTile && route_uses_cluster_kernel(c.s, c.unmasked, c.num_sms);
+}
+
+cudaError_t launch_route(const Ctx &c, bool write_dispatch)
 {
     const Shape &s = c.s;
-    if (!route_uses_cluster_kernel(s, c.unmasked, c.num_sms)) return launch_route_chunked(c);
+    if (!route_uses_cluster_kernel(s, c.unmasked, c.num_sms)) return write_dispatch ? cudaErrorInvalidValue : launch_route_chunked(c);
     ClusterRouterParams p;
     ClusterRouterMaps maps;
     memset(&p, 0, sizeof(p));
@@ -1290,6 +1356,17 @@ cudaError_t launch_route(const Ctx &c)
     p.route_priv_rows = c.audit.route_priv_rows;
     p.status = c.audit.status;
     p.gemm_bar = c.gemm_ready + gemm_ready_words(s) - 1;
+    if (write_dispatch) {
+        if (s.T > kCTile) return cudaErrorInvalidValue;
+        p.dispatch = 1;
+        p.offsets = c.offsets;
+        p.counts = c.counts;
+        p.gemm_ready = c.gemm_ready;
+        p.gemm_ready_words = (int)gemm_ready_words(s);
+        p.slot_of = c.slot_of;
+        p.tok_of_slot = c.tok_of_slot;
+        p.w_of_slot = c.w_of_slot;
+    }
     bool ok = encode_2d(&maps.hidden, c.hidden, s.H, s.T, kCTile);
     ok &= encode_2d(&maps.router[0], c.router_pub, s.H, s.E_pub, 128);
     ok &= encode_2d(&maps.router[1], c.router_priv, s.H, s.E_priv, 128);

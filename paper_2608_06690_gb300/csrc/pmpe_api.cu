@@ -215,12 +215,15 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     if (c.s.T == 0 || stages == 0) return PMPE_OK;
     if (stages & ~PMPE_STAGE_ALL) return PMPE_ERR_INVALID_ARG;
     cudaError_t err = cudaSuccess;
-    // The dispatch runs inside the persistent expert launch when that launch
-    // follows the router in this call (the router zeroes its grid barrier).
-    const bool fuse = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && (stages & PMPE_STAGE_GATEUP) &&
-                      (stages & PMPE_STAGE_DOWN) && experts_fuse_dispatch(c);
-    if (err == cudaSuccess && (stages & PMPE_STAGE_ROUTE)) err = launch_route(c);
-    if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE) && !fuse) err = launch_permute(c);
+    // With both the router and the dispatch in this call, the router writes
+    // the dispatch order itself at T <= 128; otherwise the dispatch runs
+    // inside the persistent expert launch when that launch follows the router
+    // in this call (the router zeroes its grid barrier), else as a kernel.
+    const bool route_disp = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && route_writes_dispatch(c);
+    const bool fuse = !route_disp && (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) &&
+                      (stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN) && experts_fuse_dispatch(c);
+    if (err == cudaSuccess && (stages & PMPE_STAGE_ROUTE)) err = launch_route(c, route_disp);
+    if (err == cudaSuccess && (stages & PMPE_STAGE_PERMUTE) && !fuse && !route_disp) err = launch_permute(c);
     if ((stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN)) {
         // one persistent launch; its readiness counters are cleared by the
         // dispatch when the dispatch runs in this call (inside it, when fused)

@@ -78,7 +78,13 @@ size_t gemm_ready_words(const Shape &s);
 int column_block(int H);
 
 // Launchers (one per stage); each returns the launch's cudaError_t.
-cudaError_t launch_route(const Ctx &c);
+// The router; with write_dispatch (only where route_writes_dispatch holds)
+// it also writes the dispatch order and clears the expert launch's
+// readiness counters, in place of the dispatch step.
+cudaError_t launch_route(const Ctx &c, bool write_dispatch);
+// Whether the router can write the dispatch order itself: T <= 128 (each
+// pool fills at most one router tile) and the cluster router runs.
+bool route_writes_dispatch(const Ctx &c);
 // Whether launch_route takes the cluster router (no memset before it; the
 // dispatch derives the per-expert counts from tile_counts) or the chunked one.
 bool route_uses_cluster_kernel(const Shape &s, int unmasked, int num_sms);

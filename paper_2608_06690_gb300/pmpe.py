@@ -53,8 +53,11 @@ KERNELS_PER_FORWARD = 3
 def kernels_per_forward(shape) -> int:
     """Kernels of this library one full forward of `shape` launches on a GPU
     where the persistent expert grid is resident at once (the rule the
-    library applies when it launches the forward)."""
-    return 3 if shape.H * shape.I >= (1 << 20) else 4
+    library applies when it launches the forward): the router, the expert
+    GEMMs and the combine, plus a dispatch kernel where neither the router
+    (at most 128 tokens) nor the expert launch (experts of at least 2^20
+    weights a projection) derives the dispatch order."""
+    return 3 if shape.T <= 128 or shape.H * shape.I >= (1 << 20) else 4
 # kernels one private-branch backward launches: the dispatched rows of the
 # private experts, dout row gather, the dL/da GEMM, the gate/up recompute GEMM
 # with the SwiGLU backward, router gradient, router weight-gradient partials
