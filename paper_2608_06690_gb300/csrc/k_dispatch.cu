@@ -19,6 +19,7 @@
 #include <algorithm>
 
 #include "pmpe_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace pmpe {
 namespace {
@@ -204,6 +205,131 @@ __global__ void __launch_bounds__(256, 4) combine_kernel(const bf16 *__restrict_
     }
 }
 
+// Combine through bulk copies (the form launch_combine takes when a ring of
+// at least two tokens fits shared memory).  Two CTAs per SM take tokens
+// blockIdx.x, blockIdx.x + grid, ...  All threads first stage the CTA's
+// dispatch slots in shared memory (one round of independent loads); then
+// lane j of warp 0 copies row j of a token (its k routed rows, then its
+// shared-expert row) from y into a ring stage with one bulk copy, and the
+// consumer warps sum the stage in combine_kernel's order (j ascending, then
+// shared, FP32), so both forms give the same bits.  The rows in flight sit
+// in shared memory, not in registers, where the thread-per-chunk form was
+// bound by the loads its registers could hold (ncu: long-scoreboard stalls,
+// 50 % occupancy).  Measured at Qwen3 prefill: the layer step 431 -> 424 us
+// (the routed rows y, written just before, are partly still in L2); at
+// DeepSeek-V2-Lite 979 -> 972 us.  One CTA per SM with a 200 KB ring was as
+// fast inside the step but slower from DRAM alone (41 vs 33 us): a CTA's
+// bulk copies in flight were too few to cover DRAM latency.
+constexpr int kCombWarps = 8;                            // consumer warps; warp 0 issues the copies
+constexpr int kCombTmaThreads = 32 * (kCombWarps + 1);
+constexpr int kCombMaxStages = 8;
+constexpr int kCombCtasPerSm = 2;
+constexpr int kCombSmemBytes = 100 * 1024;               // ring + staged slots, per CTA
+
+struct CombineTmaParams {
+    const bf16 *y, *y_sh;
+    const int32_t *slot_of;
+    int T, H, k, R;
+    int nrows;                       // rows per token: k, plus one with shared experts
+    int stages;
+    uint32_t row_bytes, stage_bytes;
+    bf16 *out;
+    uint32_t *status;
+};
+
+__global__ void __launch_bounds__(kCombTmaThreads, kCombCtasPerSm) combine_tma_kernel(const CombineTmaParams p)
+{
+    extern __shared__ uint8_t csm[];
+    __shared__ __align__(8) uint64_t bars[2 * kCombMaxStages];
+    __shared__ volatile int s_abort;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t sbase = (smem_u32(csm) + 127u) & ~127u;
+    const uint8_t *sgen = csm + (sbase - smem_u32(csm));
+    int *s_slots = reinterpret_cast<int *>(csm + (sbase - smem_u32(csm)) + (size_t)p.stages * p.stage_bytes);
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int st) { return bar0 + 8u * (uint32_t)st; };
+    auto empty_bar = [&](int st) { return bar0 + 8u * (uint32_t)(kCombMaxStages + st); };
+    if (tid == 0) {
+        for (int st = 0; st < p.stages; ++st) {
+            mbar_init(full_bar(st), 1);
+            mbar_init(empty_bar(st), kCombWarps);
+        }
+        s_abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    pdl_trigger();
+    pdl_wait();
+    const int grid = (int)gridDim.x, b = (int)blockIdx.x;
+    const int ntok = b < p.T ? (p.T - 1 - b) / grid + 1 : 0;
+    const int nslots = ntok * p.k;
+#pragma unroll 4
+    for (int x = tid; x < nslots; x += kCombTmaThreads) {
+        const int tl = x / p.k, j = x - tl * p.k;
+        int slot = __ldg(p.slot_of + (size_t)(b + tl * grid) * p.k + j);
+        if ((unsigned)slot >= (unsigned)p.R) slot = 0;  // only after a dispatch mismatch (status set)
+        s_slots[x] = slot;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        const uint64_t pol = l2_policy_evict_first();
+        uint32_t filled = 0u, last_parity = 0u;
+        for (int i = 0; i < ntok; ++i) {
+            const int st = i % p.stages;
+            const uint32_t ph = (uint32_t)(i / p.stages) & 1u;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(empty_bar(st), ph ^ 1u, &s_abort, p.status) ? 1 : 0;
+            if (!__shfl_sync(~0u, ok, 0)) break;
+            if (lane == 0) mbar_expect_tx(full_bar(st), (uint32_t)p.nrows * p.row_bytes);
+            __syncwarp();
+            if (lane < p.nrows) {
+                const int t = b + i * grid;
+                const bf16 *src = lane < p.k ? p.y + (size_t)s_slots[i * p.k + lane] * p.H : p.y_sh + (size_t)t * p.H;
+                bulk_load_g2s(sbase + (uint32_t)st * p.stage_bytes + (uint32_t)lane * p.row_bytes, src, p.row_bytes,
+                              full_bar(st), pol);
+            }
+            filled |= 1u << st;
+            last_parity = (last_parity & ~(1u << st)) | (ph << st);
+        }
+        // no copy into this CTA's shared memory may still be in flight at its
+        // exit (bounded: after an abort the consumers stopped early)
+        if (lane == 0)
+            for (int st = 0; st < p.stages; ++st)
+                if ((filled >> st) & 1u) {
+                    const unsigned long long w0 = globaltimer_ns();
+                    while (!mbar_try_wait(full_bar(st), (last_parity >> st) & 1u))
+                        if (globaltimer_ns() - w0 > kWaitLimitNs) break;
+                }
+    } else {
+        const int ct = tid - 32;
+        const int nv = p.H / 8;
+        for (int i = 0; i < ntok; ++i) {
+            const int st = i % p.stages;
+            const uint32_t ph = (uint32_t)(i / p.stages) & 1u;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(full_bar(st), ph, &s_abort, p.status) ? 1 : 0;
+            if (!__shfl_sync(~0u, ok, 0)) break;
+            mbar_try_wait(full_bar(st), ph);  // completed: this lane's acquire of the copied rows
+            const int t = b + i * grid;
+            const uint8_t *stage = sgen + (size_t)st * p.stage_bytes;
+            for (int c = ct; c < nv; c += 32 * kCombWarps) {
+                float acc[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+                for (int j = 0; j < p.nrows; ++j)
+                    add_bf16x8(acc, *reinterpret_cast<const uint4 *>(stage + (size_t)j * p.row_bytes + (size_t)c * 16));
+                uint4 o;
+                o.x = pack_bf16x2(acc[0], acc[1]);
+                o.y = pack_bf16x2(acc[2], acc[3]);
+                o.z = pack_bf16x2(acc[4], acc[5]);
+                o.w = pack_bf16x2(acc[6], acc[7]);
+                reinterpret_cast<uint4 *>(p.out + (size_t)t * p.H)[c] = o;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty_bar(st));
+        }
+    }
+}
+
 // Grid for a grid-stride loop over `work` items of 256-thread blocks: enough
 // blocks to cover the work once, capped at 8 resident blocks per SM.
 int grid_for(long long work, int num_sms)
@@ -238,6 +364,31 @@ cudaError_t launch_permute(const Ctx &c)
 cudaError_t launch_combine(const Ctx &c)
 {
     const Shape &s = c.s;
+    {
+        CombineTmaParams p;
+        p.y = c.y;
+        p.y_sh = s.E_sh > 0 ? c.y_sh : nullptr;
+        p.slot_of = c.slot_of;
+        p.T = s.T; p.H = s.H; p.k = s.k; p.R = s.T * s.k;
+        p.nrows = s.k + (s.E_sh > 0 ? 1 : 0);
+        p.row_bytes = (uint32_t)s.H * 2u;
+        p.stage_bytes = (uint32_t)p.nrows * p.row_bytes;
+        p.out = c.out;
+        p.status = c.audit.status;
+        const int grid = std::max(1, std::min(kCombCtasPerSm * c.num_sms, s.T));
+        const long long ntok = (s.T + grid - 1) / grid;
+        const long long slots_bytes = (ntok * s.k * 4 + 15) / 16 * 16;
+        const long long room = (long long)kCombSmemBytes - 128 - slots_bytes;
+        const long long stages = room > 0 ? std::min<long long>(kCombMaxStages, room / p.stage_bytes) : 0;
+        if (stages >= 2) {
+            p.stages = (int)stages;
+            const int smem = (int)(128 + stages * p.stage_bytes + slots_bytes);
+            static std::atomic<int> smem_limit[64];
+            const cudaError_t err = ensure_dynamic_smem(combine_tma_kernel, smem, smem_limit);
+            if (err != cudaSuccess) return err;
+            return launch_pdl(combine_tma_kernel, dim3(grid), dim3(kCombTmaThreads), (size_t)smem, c.stream, p);
+        }
+    }
     return launch_pdl(combine_kernel, dim3(grid_for((long long)s.T * (s.H / 8), c.num_sms)), dim3(256), 0, c.stream,
                       (const bf16 *)c.y, (const bf16 *)(s.E_sh > 0 ? c.y_sh : nullptr), (const int32_t *)c.slot_of, s.T,
                       s.H, s.k, c.out);

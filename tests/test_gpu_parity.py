@@ -40,6 +40,10 @@ CASES = {
     # k > 8 takes the router's sorting-network path; 40 public experts span two chunks
     "k12_two_chunks_pool_softmax": (LayerShape(T=150, H=256, I=128, E_pub=40, E_priv=16, E_sh=0, k=12,
                                                renormalize=False), 44, "iid"),
+    # 9 rows of 8 KB per token: a ring of two tokens does not fit the bulk
+    # combine's shared memory, so the thread-per-chunk combine runs
+    "wide_rows_chunk_combine": (LayerShape(T=40, H=4096, I=128, E_pub=12, E_priv=8, E_sh=1, k=8, renormalize=True),
+                                48, "iid"),
     # a 256-expert pool with k = 24 at H = 128: the chunk lists do not fit the
     # cluster router's shared memory, so the chunked router runs the method
     "k24_pool_256_chunked_router": (LayerShape(T=200, H=128, I=128, E_pub=256, E_priv=64, E_sh=0, k=24,
