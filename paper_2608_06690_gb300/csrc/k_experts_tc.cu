@@ -213,35 +213,6 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
 
 // ---------------------------------------------------------------- kernel
 
-// Every CTA of the grid arrives, then waits (bounded) until `target`
-// arrivals are counted.  The grid is resident all at once (checked before the
-// launch), so the wait ends.  Writes before the barrier, by any thread of any
-// CTA, are visible after it.  Returns false, with the timeout recorded, when
-// the wait expired.
-__device__ bool grid_barrier(uint32_t *ctr, uint32_t target, uint32_t *status)
-{
-    __shared__ int s_ok;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int ok = 1;
-        __threadfence();
-        atomicAdd(ctr, 1u);
-        const unsigned long long t0 = globaltimer_ns();
-        while (ld_acquire_gpu(ctr) < target) {
-            if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                if (status) atomicOr(status, PMPE_STATUS_PIPELINE_TIMEOUT);
-                ok = 0;
-                break;
-            }
-            __nanosleep(32);
-        }
-        __threadfence();
-        s_ok = ok;
-    }
-    __syncthreads();
-    return s_ok != 0;
-}
-
 // Shared-memory bytes the fused dispatch needs for its per-expert prefix of
 // the router tiles' counts ([E][slots + 1] words, inside the ring).
 constexpr size_t fused_dispatch_smem(int E, int slots) { return (size_t)E * (size_t)(slots + 1) * 4u; }
@@ -384,8 +355,34 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             p.tok_of_slot_w[slot] = r / p.k;
             p.w_of_slot_w[slot] = p.w_route[r];
         }
-        if (!grid_barrier(p.grid_bar, gridDim.x, p.status)) s_abort = 1;
+        // arrive at the grid barrier (an arrival counter the router zeroed);
+        // each role waits for every CTA's arrival (wait_dispatch) only before
+        // it first reads what other CTAs wrote here, so that the tile table,
+        // the first weight loads and the other CTAs' arrivals overlap
+        __syncthreads();
+        if (tid == 0) {
+            __threadfence();
+            atomicAdd(p.grid_bar, 1u);
+        }
     }
+    // Until every CTA has arrived: the slot maps (tok_of_slot, w_of_slot) and
+    // the readiness and tile counters (cleared by CTA 0) are not yet final.
+    // Every lane that calls this acquires the arrivals itself (bounded wait;
+    // the grid is resident all at once, checked before the launch).
+    auto wait_dispatch = [&]() -> bool {
+        if (!p.fuse_dispatch) return true;
+        const unsigned long long t0 = globaltimer_ns();
+        while (ld_acquire_gpu(p.grid_bar) < gridDim.x) {
+            if (s_abort) return false;
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                s_abort = 1;
+                if (p.status) atomicOr(p.status, PMPE_STATUS_PIPELINE_TIMEOUT);
+                return false;
+            }
+            __nanosleep(32);
+        }
+        return true;
+    };
     // tile list: rows and tiles per group, prefixes over groups
     int multi = 0;  // some group has more than one 128-row block
     for (int g = tid; g < G; g += kThreads) {
@@ -465,6 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         // CTA is ready (an atomic counter, taken one tile ahead), which
         // evens out tiles of unequal cost.
         uint32_t ahead = 0u;  // lane 0: the next dynamic tile, taken one ahead
+        bool synced = false;  // lane 0: wait_dispatch has returned
         for (int qi = 0;; ++qi) {
             int tile = -1;
             if (qi < n_wave) {
@@ -472,7 +470,10 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             } else {
                 if (lane == 0) {
                     const int d = qi - n_wave, slot = d % kTQ;
-                    if (d == 0) ahead = (uint32_t)tail + atomicAdd(p.tile_ctr, 1u);
+                    if (d == 0) {
+                        if (!synced) synced = wait_dispatch();
+                        ahead = synced ? (uint32_t)tail + atomicAdd(p.tile_ctr, 1u) : (uint32_t)total;
+                    }
                     if (mbar_wait(tq_empty_bar(slot), ((uint32_t)(d / kTQ) & 1u) ^ 1u, &s_abort, p.status) &&
                         !s_abort && ahead < (uint32_t)total) {
                         tile = (int)ahead;
@@ -500,8 +501,10 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 // the weights are loaded meanwhile)
                 const uint32_t need = 4u * (uint32_t)(group_n(p, kGateUp, t.shared) / p.ph[kGateUp].bn);
                 const uint32_t *rp = p.ready + tt.mpre[t.g] + t.m_tile;
+                if (!synced) synced = wait_dispatch();
+                if (!synced) ok = false;
                 const unsigned long long t0 = globaltimer_ns();
-                while (ld_acquire_gpu(rp) < need) {
+                while (ok && ld_acquire_gpu(rp) < need) {
                     if (s_abort) { ok = false; break; }
                     if (globaltimer_ns() - t0 > kWaitLimitNs) {
                         s_abort = 1;
@@ -599,6 +602,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         const uint32_t out_base = sbase + kStages * kStageBytes + (uint32_t)((warp - 2) * 2 * kOutBufBytes);
         int out_parity = 0;
         int it = 0;
+        bool synced = false;  // wait_dispatch has returned (every lane acquires)
         for (int qi = 0;; ++qi) {
             int tile = 0;
             if (lane == 0) tile = next_tile(qi);
@@ -613,6 +617,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
             if (lane == 0) ok = mbar_wait(tfull_bar(buf), use, &s_abort, p.status) ? 1 : 0;
             ok = __shfl_sync(~0u, ok, 0);
             if (!ok) break;
+            if (!synced && !(synced = wait_dispatch())) break;
             __syncwarp();
             tc_fence_after();
             const TcPhase &ph = p.ph[t.ph];
@@ -806,6 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         const int chunk = gi & 7, row0 = gi >> 3;
         uint32_t sc = 0;                     // ring stages passed so far (the ring position)
         bool ok = true;
+        bool synced = false;                 // wait_dispatch has returned (every lane acquires)
         auto drain = [&]() { cp_async_wait<0>(); };
         for (int qi = 0; ok; ++qi) {
             int tile = 0;
@@ -817,6 +823,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                 sc += (uint32_t)t.nkb;
                 continue;
             }
+            if (!synced && !(synced = wait_dispatch())) break;
             // this thread's 8 rows: their token rows in the hidden states
             const bf16 *src[8];
             uint32_t nbytes[8];
