@@ -775,20 +775,38 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
         __syncwarp();
         amb &= tok_ok;
         if (__any_sync(~0u, amb)) {
-            // ---- exact path for the whole warp: k passes with the exact
-            // comparison of (logit, id), ties to the lower id
-            uint32_t taken = 0u;
+            // ---- exact path for the whole warp: the chunk's logits in
+            // registers (an entry taken, or past the pool, reads as (-inf, no
+            // id), which never outranks a candidate); per pass a pairwise tree
+            // of the exact comparison of (logit, id), ties to the lower id,
+            // then the maximum over the token's lanes, whose owner removes it
+            float xv[32];
+            int xe[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const bool in = i < nvalid;
+                xv[i] = in ? clean_logit(sum[i]) : -INFINITY;
+                xe[i] = in ? c * kChunk + i : 0x7fffffff;
+            }
             for (int j = 0; j < K; ++j) {
-                float bv = -INFINITY;
-                int be = 0x7fffffff;
-                for (int i = 0; i < nvalid; ++i) {
-                    const float x = clean_logit(sum[i]);
-                    const int e = c * kChunk + i;
-                    if (!((taken >> i) & 1u) && ranks_above(x, e, bv, be)) {
-                        bv = x;
-                        be = e;
-                    }
+                float tv[16];
+                int te[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const bool hi = ranks_above(xv[2 * i + 1], xe[2 * i + 1], xv[2 * i], xe[2 * i]);
+                    tv[i] = hi ? xv[2 * i + 1] : xv[2 * i];
+                    te[i] = hi ? xe[2 * i + 1] : xe[2 * i];
                 }
+#pragma unroll
+                for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+                    for (int i = 0; i < w; ++i) {
+                        const bool hi = ranks_above(tv[i + w], te[i + w], tv[i], te[i]);
+                        tv[i] = hi ? tv[i + w] : tv[i];
+                        te[i] = hi ? te[i + w] : te[i];
+                    }
+                float bv = tv[0];
+                int be = te[0];
                 for (int d = 1; d < ncp; d <<= 1) {
                     const float ov = __shfl_xor_sync(~0u, bv, d);
                     const int oe = __shfl_xor_sync(~0u, be, d);
@@ -797,7 +815,12 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
                         be = oe;
                     }
                 }
-                if (nvalid > 0 && (be >> 5) == c) taken |= 1u << (be & 31);
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (xe[i] == be) {
+                        xv[i] = -INFINITY;
+                        xe[i] = 0x7fffffff;
+                    }
                 if (c == 0 && tok_ok) sel_e[tl * K + j] = be;
             }
             __syncwarp();

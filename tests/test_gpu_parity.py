@@ -100,6 +100,39 @@ def test_expert_loads_0_1_and_152_rows():
     assert counts[3] >= 152 and counts[shape.E_pub + 2] == 1 and (counts == 0).any()
 
 
+def test_exact_logit_ties_take_the_lower_id():
+    """Exactly equal logits (Sec. 3.1 takes the top k after the mask; at an
+    exact tie the lower expert id ranks first, the reading both sides
+    implement): router rows duplicated in pairs, so every token's selection
+    meets ties and the router takes its exact selection path, and every fifth
+    token with a zero hidden state, whose logits are all 0."""
+    shape = LayerShape(T=150, H=256, I=128, E_pub=24, E_priv=8, E_sh=0, k=4, renormalize=True)
+    w, h, pol = make_layer(shape, 49)
+    for key in ("router_pub", "router_priv"):
+        r = w[key].clone()
+        r[1::2] = r[0::2]  # row 2i + 1 equals row 2i
+        w[key] = r
+    h = h.clone()
+    h[::5] = 0
+    wd, hd, pd = to_device(w, h, pol)
+    gpu = run_gpu_layer(shape, wd, hd, pd)
+    check_against_oracle(shape, w, h, pol, gpu)
+    idx = gpu["idx"]
+    base = np.where(gpu["tau"][:, None] == 1, shape.E_pub, 0)
+    loc = idx - base
+    # all-zero tokens: the pool's first k experts, in id order
+    assert np.array_equal(loc[::5], np.tile(np.arange(shape.k), (len(loc[::5]), 1)))
+    # twins (equal logits): 2i + 1 comes right after 2i, which is missing
+    # from the selection only when 2i falls in the k-th place
+    for t in range(shape.T):
+        sel = list(loc[t])
+        for j, e in enumerate(sel):
+            if e % 2 == 1:
+                assert j > 0 and sel[j - 1] == e - 1, (t, sel)
+            elif j < len(sel) - 1:
+                assert sel[j + 1] == e + 1, (t, sel)
+
+
 def test_zero_tokens_is_a_noop():
     from paper_2608_06690_gb300 import pmpe
     shape = LayerShape(T=0, H=256, I=128, E_pub=8, E_priv=4, E_sh=0, k=2, renormalize=True)
