@@ -598,6 +598,11 @@ __global__ void __launch_bounds__(kRThreads, 1) router_tc_kernel(const RouterPar
 constexpr int kCThreads = 192;       // warp 0 TMA, warp 1 TMEM + MMA, warps 2..5 gather / epilogue / finalize
 constexpr int kCTile = 128;          // tokens per tile (MMA N)
 constexpr int kCRingBytes = 192 * 1024;
+// Staged partial logits: a token's row holds its 32-expert chunks at a stride
+// of 36 floats, so that the lanes of a token, one chunk each, read different
+// shared-memory banks in the selection (a stride of 32 put them all on one).
+constexpr int kChunkPitch = 36;
+__device__ __forceinline__ int chunk_pos(int e) { return (e >> 5) * kChunkPitch + (e & 31); }
 constexpr int kCMaxStages = 6;
 
 struct ClusterRouterParams {
@@ -636,7 +641,7 @@ static int cluster_router_smem(int P, int k, int nq)
 {
     const int pp = (P + 127) / 128 * 128;
     const int tpc = kCTile / nq;
-    const int partial = kCTile * (pp + 4) * 4;  // staged partials, then the receive buffer
+    const int partial = kCTile * (pp / kChunk * kChunkPitch) * 4;  // staged partials, then the receive buffer
     const int lists = tpc * k * 8 + tpc * 8;
     const int after = 2 * partial + lists;
     return (after > kCRingBytes ? after : kCRingBytes) + 1024;
@@ -722,7 +727,7 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
         const bool tok_ok = pi < npairs && tl < ntok;
         const int nvalid = (tok_ok && c < nc) ? min(kChunk, P - c * kChunk) : 0;
         float *row = rcv + (size_t)(tok_ok ? tl : 0) * pitch;  // slot 0: the token's summed logits
-        float *sum = row + c * kChunk;
+        float *sum = row + c * kChunkPitch;
         float mx = -INFINITY, ssum = 0.f;
         uint32_t key[32];  // this lane's selection keys (0: no candidate)
 #pragma unroll
@@ -831,12 +836,12 @@ __device__ void finalize_tokens(const ClusterRouterParams &p, float *rcv, int pi
             const int tt = q * tpc + tl;
             for (int j = c; j < K; j += ncp) {
                 const int e = sel_e[tl * K + j];
-                sel_v[tl * K + j] = clean_logit(row[e]);
+                sel_v[tl * K + j] = clean_logit(row[chunk_pos(e)]);
                 atomicOr(&smask[e * 4 + (tt >> 5)], 1u << (tt & 31));
             }
-            top = clean_logit(row[sel_e[tl * K]]);
+            top = clean_logit(row[chunk_pos(sel_e[tl * K])]);
             if (p.renorm)
-                for (int j = 0; j < K; ++j) den += expf(clean_logit(row[sel_e[tl * K + j]]) - top);
+                for (int j = 0; j < K; ++j) den += expf(clean_logit(row[chunk_pos(sel_e[tl * K + j])]) - top);
         }
         if (!p.renorm) {
             const int g0 = (int)(threadIdx.x & 31) & ~(ncp - 1);
@@ -939,7 +944,7 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
     const uint32_t done_bar = bar0 + 8u * (2 * kCMaxStages + 1);
     const uint32_t rcv_bar = bar0 + 8u * (2 * kCMaxStages + 2);  // partial logits received from the cluster
     const int tpc = kCTile / p.nq;
-    const int pitch = pp + 4;
+    const int pitch = pp / kChunk * kChunkPitch;  // floats per token row of partial logits
     const uint32_t slice_bytes = (uint32_t)(tpc * pitch * 4);  // one source CTA's partials of this CTA's tokens
     const uint32_t part_bytes = (uint32_t)(kCTile * pitch * 4);
     if (tid == 0) {
@@ -1050,7 +1055,8 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
             cp_async_wait<0>();
         }
         // ---- epilogue: the partial logits to shared memory, [token][expert]
-        // FP32 (pitch pp + 4; the ring is free once every MMA has completed)
+        // FP32 (chunks of 32 experts at a stride of kChunkPitch; the ring is
+        // free once every MMA has completed)
         int ok = 1;
         if (lane == 0) ok = mbar_wait(tfull_bar, 0, &s_abort, p.status) ? 1 : 0;
         ok = __shfl_sync(~0u, ok, 0);
@@ -1066,7 +1072,7 @@ __global__ void __launch_bounds__(kCThreads, 1) router_cluster_kernel(const Clus
                     tmem_ld32(tmem + (uint32_t)(mi * 128 + cc * 32) + ((uint32_t)(quarter * 32) << 16), v);
                     tmem_ld_wait();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) S[(cc * 32 + i) * pitch + e] = v[i];
+                    for (int i = 0; i < 32; ++i) S[(cc * 32 + i) * pitch + chunk_pos(e)] = v[i];
                 }
             }
             fence_proxy_async_smem();  // the bulk copies below read these rows
