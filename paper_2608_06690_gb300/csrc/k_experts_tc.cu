@@ -129,6 +129,22 @@ struct TcParams {
     float *w_of_slot_w;
     uint32_t *grid_bar;
     int clear_words;            // readiness counters and the tile counter, from `ready`
+    // routing in the launch (T <= 128, nothing launched before this kernel
+    // but the clearing of `ready`, the tile counter and the barriers): the
+    // CTAs compute the masked router's logits, the top k, the routing weights
+    // and the route log, then the dispatch order (route_in_launch)
+    int fuse_route;
+    int renorm;
+    const uint8_t *policy;           // [T] policy bytes, or NULL (every token DENY)
+    const bf16 *router_w[2];         // [E_pub, H] public, [E_priv, H] private router
+    float *z;                        // [T][zpitch] logits of each token's pool (scratch)
+    int zpitch;
+    int32_t *idx_w, *ticket_w;       // [T, k] route log written
+    float *w_w;                      // [T, k] routing weights written
+    uint8_t *tau_w;                  // [T]
+    uint32_t *tile_counts_w;         // [E][slots4]
+    uint32_t *route_count, *route_priv_rows;
+    uint32_t *bar_a, *bar_b;         // grid barriers after the logits and after the selection
     // small batches (every expert at most one 128-row block): the first
     // `prefetch_tiles` gate/up tiles of the list of all experts have their
     // weights prefetched into L2 by the CTA of the same index, before the
@@ -213,6 +229,334 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
 
 // ---------------------------------------------------------------- kernel
 
+// Weights of gate/up tile blockIdx.x of the list of all experts (the first
+// wave when every expert has at most one 128-row block): 128 gate rows and
+// 128 up rows, each block contiguous, prefetched into L2 by one thread.
+__device__ __forceinline__ void prefetch_first_wave(const TcParams &p)
+{
+    const int nt = p.I / 128;
+    const int e = (int)blockIdx.x / nt, n = (int)blockIdx.x - e * nt;
+    if (e < p.E) {
+        const int q = e < p.E_pub ? 0 : 1;
+        const size_t row0 = (size_t)(q ? e - p.E_pub : e) * p.I + (size_t)n * 128;
+        const uint32_t bytes = (uint32_t)(128u * (uint32_t)p.H * 2u);
+        bulk_prefetch_l2(p.gate_w[q] + row0 * p.H, bytes);
+        bulk_prefetch_l2(p.up_w[q] + row0 * p.H, bytes);
+    }
+}
+
+// Every CTA of the grid arrives (after all of its threads' writes), then
+// waits, bounded, until `target` arrivals are counted; writes before the
+// barrier, by any thread of any CTA, are visible after it.  The grid is
+// resident all at once (checked before the launch).  False after a timeout
+// or an abort.
+__device__ bool grid_barrier(uint32_t *ctr, uint32_t target, volatile int *abort_flag, uint32_t *status)
+{
+    __shared__ int s_ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int ok = 1;
+        __threadfence();
+        atomicAdd(ctr, 1u);
+        const unsigned long long t0 = globaltimer_ns();
+        while (ld_acquire_gpu(ctr) < target) {
+            if (*abort_flag) { ok = 0; break; }
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                *abort_flag = 1;
+                if (status) atomicOr(status, PMPE_STATUS_PIPELINE_TIMEOUT);
+                ok = 0;
+                break;
+            }
+            __nanosleep(32);
+        }
+        __threadfence();
+        s_ok = ok;
+    }
+    __syncthreads();
+    return s_ok != 0;
+}
+
+constexpr int kRouteMaxTokens = 128;   // routing in the launch: one selection CTA per token
+constexpr int kRouteMaxH = 2048;       // a 32-expert block of router rows (128 KB) plus the token row fit the ring
+constexpr int kRouteXChunks = kRouteMaxH / 256;  // 16-byte pieces of the token row per lane
+
+__device__ __forceinline__ float dot8_bf16(const uint4 &a, const uint4 &b, float acc)
+{
+    const __nv_bfloat162 *x = reinterpret_cast<const __nv_bfloat162 *>(&a);
+    const __nv_bfloat162 *y = reinterpret_cast<const __nv_bfloat162 *>(&b);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 u = __bfloat1622float2(x[i]), v = __bfloat1622float2(y[i]);
+        acc = fmaf(u.x, v.x, acc);
+        acc = fmaf(u.y, v.y, acc);
+    }
+    return acc;
+}
+
+// Exact ranking of two candidates (logit, pool-local id): the larger logit,
+// at equal logits the lower id (NaN was cleaned to -inf before).
+__device__ __forceinline__ bool route_above(float x, int e, float bx, int be)
+{
+    return (x > bx) | ((x == bx) & (e < be));
+}
+
+// Routing inside the persistent launch, for T <= 128 tokens (Sec. 3.1 Eq. 4
+// and App. B.1), in three steps separated by grid barriers:
+//   1. logits: work items (token t, block c of t's pool), spread over the
+//      CTAs, at most one each; each warp of a CTA forms the dot products of its
+//      experts with the token row (FP32: a lane's 16-byte pieces in order,
+//      then a butterfly), into z[t][e].  A token meets only its own pool's
+//      router rows.
+//   2. selection: CTA t < T, one warp: the top k of z[t] by k passes of an
+//      exact (logit, id) maximum, ties to the lower id; the weights (softmax
+//      over the k, or over the pool); the route log.
+//   3. dispatch: every CTA forms per expert the mask of the tokens that
+//      picked it, the counts and first slots (experts in id order, tokens in
+//      order), and resolves its share of the routed rows (slot = first slot
+//      + rank of the token among the expert's tokens).  The tile table takes
+//      the counts and first slots; the caller then arrives at grid_bar.
+// Returns false after an abort (a barrier timed out).
+__device__ bool route_in_launch(const TcParams &p, uint8_t *ring, TileTable &tt, volatile int *s_abort)
+{
+    __shared__ int s_item[kRouteMaxTokens + 1];  // items of the tokens before t
+    __shared__ uint8_t s_tau[kRouteMaxTokens];
+    __shared__ int s_nd;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    constexpr int kWarps = kThreads / 32;
+    const int T = p.T, K = p.k, E = p.E, E_priv = p.E - p.E_pub, R = p.R;
+    // ---- tau per token (Sec. 2.1) and the logit work items: (token, block
+    // of bs experts of its pool), bs the least size from 32 up that gives
+    // every CTA at most one item (a CTA's item is a chain of dependent load
+    // rounds, so two items on one CTA would double the step)
+    __shared__ int s_bs;
+    if (warp == 0) {
+        int nd = 0;
+        for (int b0 = 0; b0 < T; b0 += 32) {
+            const int t = b0 + lane;
+            const int tau = (t < T && p.policy) ? (p.policy[t] == 0x01 ? 1 : 0) : 0;
+            if (t < T) s_tau[t] = (uint8_t)tau;
+            nd += __popc(__ballot_sync(~0u, t < T && tau == 0));
+        }
+        const int na = T - nd;
+        int bs = 256;  // one item per token always fits (T <= the grid)
+        for (int b1 = 32; b1 < 256; b1 += 32) {  // the lanes test 32 sizes at a time
+            const int c = b1 + lane;
+            const bool fits = nd * ((p.E_pub + c - 1) / c) + na * ((E_priv + c - 1) / c) <= (int)gridDim.x;
+            const unsigned m = __ballot_sync(~0u, fits);
+            if (m) {
+                bs = b1 + __ffs(m) - 1;
+                break;
+            }
+        }
+        int carry = 0;
+        for (int b0 = 0; b0 < T; b0 += 32) {
+            const int t = b0 + lane;
+            const int v0 = t < T ? ((s_tau[t] ? E_priv : p.E_pub) + bs - 1) / bs : 0;
+            int v = v0;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(~0u, v, off);
+                if (lane >= off) v += y;
+            }
+            if (t < T) s_item[t] = carry + v - v0;
+            carry += __shfl_sync(~0u, v, 31);
+        }
+        if (lane == 0) {
+            s_item[T] = carry;
+            s_nd = nd;
+            s_bs = bs;
+        }
+    }
+    __syncthreads();
+    const int nitems = s_item[T], nd = s_nd, bs = s_bs;
+    const int nch = p.H / 8;  // 16-byte pieces of a row
+    // ---- 1. logits (loads straight into registers: each warp takes its
+    // experts two at a time, so that a lane has 16 loads of 16 bytes in
+    // flight; bulk copies of the block into shared memory were slower)
+    for (int i = (int)blockIdx.x; i < nitems; i += (int)gridDim.x) {
+        int lo = 0, hi = T - 1;  // the token of item i: the last t with s_item[t] <= i
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_item[mid] <= i) lo = mid; else hi = mid - 1;
+        }
+        const int t = lo, tau = s_tau[t];
+        const int e0 = (i - s_item[t]) * bs;
+        const int ne = min(bs, (tau ? E_priv : p.E_pub) - e0);
+        const uint4 *xrow = reinterpret_cast<const uint4 *>(p.hidden + (size_t)t * p.H);
+        const uint4 *wblk = reinterpret_cast<const uint4 *>(p.router_w[tau] + (size_t)e0 * p.H);
+        uint4 xr[kRouteXChunks];
+#pragma unroll
+        for (int q = 0; q < kRouteXChunks; ++q) {
+            const int ch = lane + 32 * q;
+            xr[q] = ch < nch ? __ldg(xrow + ch) : make_uint4(0u, 0u, 0u, 0u);
+        }
+        for (int e = warp; e < ne; e += 2 * kWarps) {
+            const int e2 = e + kWarps;  // the second expert of the pair (absent past the block)
+            uint4 wa[kRouteXChunks], wb[kRouteXChunks];
+#pragma unroll
+            for (int q = 0; q < kRouteXChunks; ++q) {
+                const int ch = lane + 32 * q;
+                wa[q] = ch < nch ? __ldg(wblk + (size_t)e * nch + ch) : make_uint4(0u, 0u, 0u, 0u);
+                wb[q] = (ch < nch && e2 < ne) ? __ldg(wblk + (size_t)e2 * nch + ch) : make_uint4(0u, 0u, 0u, 0u);
+            }
+            float acc_a = 0.f, acc_b = 0.f;
+#pragma unroll
+            for (int q = 0; q < kRouteXChunks; ++q) {
+                if (lane + 32 * q < nch) {
+                    acc_a = dot8_bf16(wa[q], xr[q], acc_a);
+                    acc_b = dot8_bf16(wb[q], xr[q], acc_b);
+                }
+            }
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) {
+                acc_a += __shfl_xor_sync(~0u, acc_a, off);
+                acc_b += __shfl_xor_sync(~0u, acc_b, off);
+            }
+            if (lane == 0) {
+                p.z[(size_t)t * p.zpitch + e0 + e] = acc_a;
+                if (e2 < ne) p.z[(size_t)t * p.zpitch + e0 + e2] = acc_b;
+            }
+        }
+    }
+    if (!grid_barrier(p.bar_a, gridDim.x, s_abort, p.status)) return false;
+    // the first wave's weights into L2 while the selection and the dispatch
+    // run (not earlier: the prefetch would delay the router rows)
+    if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles) prefetch_first_wave(p);
+    // ---- 2. selection, one warp per token
+    if ((int)blockIdx.x < T && warp == 0) {
+        const int t = (int)blockIdx.x, tau = s_tau[t];
+        const int P = tau ? E_priv : p.E_pub, base = tau ? p.E_pub : 0;
+        const float *zt = p.z + (size_t)t * p.zpitch;
+        float v[8], vo[8];
+        int id[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int e = lane + 32 * q;
+            const float x = e < P ? zt[e] : -INFINITY;
+            vo[q] = v[q] = x != x ? -INFINITY : x;  // NaN never outranks a number
+            id[q] = e < P ? e : 0x7fffffff;
+        }
+        float my_v = 0.f, top = 0.f;
+        int my_e = 0;
+        for (int j = 0; j < K; ++j) {
+            float bv = v[0];
+            int be = id[0];
+#pragma unroll
+            for (int q = 1; q < 8; ++q)
+                if (route_above(v[q], id[q], bv, be)) {
+                    bv = v[q];
+                    be = id[q];
+                }
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) {
+                const float ov = __shfl_xor_sync(~0u, bv, off);
+                const int oe = __shfl_xor_sync(~0u, be, off);
+                if (route_above(ov, oe, bv, be)) {
+                    bv = ov;
+                    be = oe;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (id[q] == be) {
+                    v[q] = -INFINITY;
+                    id[q] = 0x7fffffff;
+                }
+            if (lane == j) {
+                my_v = bv;
+                my_e = be;
+            }
+            if (j == 0) top = bv;
+        }
+        float den = 0.f;
+        if (p.renorm) {  // softmax over the k selected logits, in rank order
+            for (int j = 0; j < K; ++j) den += expf(__shfl_sync(~0u, my_v, j) - top);
+        } else {         // softmax over the pool
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (lane + 32 * q < P) den += expf(vo[q] - top);
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) den += __shfl_xor_sync(~0u, den, off);
+        }
+        if (lane < K) {
+            p.idx_w[(size_t)t * K + lane] = base + my_e;
+            p.w_w[(size_t)t * K + lane] = expf(my_v - top) / den;
+            if (p.route_count) atomicAdd(&p.route_count[base + my_e], 1u);
+        }
+        if (lane == 0) {
+            p.tau_w[t] = (uint8_t)tau;
+            if (p.route_priv_rows) atomicAdd(&p.route_priv_rows[t], tau ? (unsigned)K : 0u);
+        }
+    }
+    if (!grid_barrier(p.bar_b, gridDim.x, s_abort, p.status)) return false;
+    // ---- 3. dispatch order: per expert the mask of its tokens (4 x 32 bits)
+    uint32_t *smask = reinterpret_cast<uint32_t *>(ring);
+    int *sfirst = reinterpret_cast<int *>(smask + (size_t)E * 4);
+    int *scount = sfirst + E;
+    for (int i = tid; i < E * 4; i += kThreads) smask[i] = 0u;
+    __syncthreads();
+    for (int r = tid; r < R; r += kThreads) {
+        const int e = p.idx_w[r], t = r / K;
+        if ((unsigned)e < (unsigned)E) atomicOr(&smask[e * 4 + (t >> 5)], 1u << (t & 31));
+    }
+    __syncthreads();
+    if (warp == 0) {  // rows per expert and their exclusive prefix: the first slots
+        int carry = 0;
+        for (int b0 = 0; b0 < E; b0 += 32) {
+            const int g = b0 + lane;
+            const int v0 = g < E ? __popc(smask[g * 4]) + __popc(smask[g * 4 + 1]) + __popc(smask[g * 4 + 2]) +
+                                       __popc(smask[g * 4 + 3])
+                                 : 0;
+            int v = v0;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int y = __shfl_up_sync(~0u, v, off);
+                if (lane >= off) v += y;
+            }
+            if (g < E) {
+                sfirst[g] = carry + v - v0;
+                scount[g] = v0;
+            }
+            carry += __shfl_sync(~0u, v, 31);
+        }
+    }
+    __syncthreads();
+    // the router tile of a pool's tokens (the cluster router's numbering:
+    // the DENY tile first when there are DENY tokens)
+    auto tile_of = [&](int g) { return g < p.E_pub ? 0 : (nd > 0 ? 1 : 0); };
+    if (blockIdx.x == 0) {
+        for (int g = tid; g < E; g += kThreads) {
+            p.offsets_w[g] = (uint32_t)sfirst[g];
+            p.counts_w[g] = (uint32_t)scount[g];
+            for (int sl = 0; sl < p.slots; ++sl)
+                p.tile_counts_w[(size_t)g * p.slots4 + sl] = sl == tile_of(g) ? (uint32_t)scount[g] : 0u;
+        }
+        if (tid == 0) p.offsets_w[E] = (uint32_t)R;
+    }
+    for (int r = (int)blockIdx.x * kThreads + tid; r < R; r += (int)gridDim.x * kThreads) {
+        const int e = p.idx_w[r], t = r / K;
+        if ((unsigned)e >= (unsigned)E) {  // never produced by the selection
+            if (p.status) atomicOr(p.status, PMPE_STATUS_BAD_EXPERT_ID);
+            continue;
+        }
+        const int wd = t >> 5;
+        int rank = __popc(smask[e * 4 + wd] & ((1u << (t & 31)) - 1u));
+        for (int w2 = 0; w2 < wd; ++w2) rank += __popc(smask[e * 4 + w2]);
+        const int slot = sfirst[e] + rank;
+        if ((unsigned)slot >= (unsigned)R) continue;
+        p.slot_of_w[r] = slot;
+        p.tok_of_slot_w[slot] = t;
+        p.w_of_slot_w[slot] = p.w_w[r];
+        p.ticket_w[r] = tile_of(e) * 128 + rank;
+    }
+    for (int g = tid; g < E; g += kThreads) {
+        tt.rows[g] = scount[g];
+        tt.base[g] = sfirst[g];
+    }
+    fence_proxy_async_smem();  // this thread's use of the ring, before the GEMM's copies land there
+    return true;
+}
+
 // Shared-memory bytes the fused dispatch needs for its per-expert prefix of
 // the router tiles' counts ([E][slots + 1] words, inside the ring).
 constexpr size_t fused_dispatch_smem(int E, int slots) { return (size_t)E * (size_t)(slots + 1) * 4u; }
@@ -279,20 +623,20 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                      "r"(kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
     }
-    if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles) {
-        // weights of gate/up tile blockIdx.x of the list of all experts: 128
-        // gate rows and 128 up rows, each block contiguous (bulk L2 prefetch)
-        const int nt = p.I / 128;
-        const int e = (int)blockIdx.x / nt, n = (int)blockIdx.x - e * nt;
-        if (e < p.E) {
-            const int q = e < p.E_pub ? 0 : 1;
-            const size_t row0 = (size_t)(q ? e - p.E_pub : e) * p.I + (size_t)n * 128;
-            const uint32_t bytes = (uint32_t)(128u * (uint32_t)p.H * 2u);
-            bulk_prefetch_l2(p.gate_w[q] + row0 * p.H, bytes);
-            bulk_prefetch_l2(p.up_w[q] + row0 * p.H, bytes);
+    // weights of the first wave into L2 while the routing is computed (in
+    // this launch: after this CTA's router rows have landed, which the
+    // prefetch would otherwise delay)
+    if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles && !p.fuse_route) prefetch_first_wave(p);
+    pdl_wait();  // the dispatch offsets and slot maps (or the route log, or cleared counters) come from the previous kernel
+    if (p.fuse_route) {
+        const bool ok = route_in_launch(p, dsmem + (sbase - smem_u32(dsmem)), tt, &s_abort);
+        if (!ok && tid == 0) s_abort = 1;
+        __syncthreads();
+        if (tid == 0) {  // arrive at the grid barrier; the roles wait for it (wait_dispatch)
+            __threadfence();
+            atomicAdd(p.grid_bar, 1u);
         }
     }
-    pdl_wait();  // the dispatch offsets and slot maps (or the route log) come from the previous kernel
     if (p.fuse_dispatch) {
         // ---- the dispatch order, as dispatch_kernel derives it.  pre[e][s]:
         // rows of expert e in the router tiles before tile s (in the ring,
@@ -370,7 +714,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     // Every lane that calls this acquires the arrivals itself (bounded wait;
     // the grid is resident all at once, checked before the launch).
     auto wait_dispatch = [&]() -> bool {
-        if (!p.fuse_dispatch) return true;
+        if (!p.fuse_dispatch && !p.fuse_route) return true;
         const unsigned long long t0 = globaltimer_ns();
         while (ld_acquire_gpu(p.grid_bar) < gridDim.x) {
             if (s_abort) return false;
@@ -391,7 +735,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         if (shared) {
             rows = p.T;
             base = 0;
-        } else if (p.fuse_dispatch) {  // derived above
+        } else if (p.fuse_dispatch || p.fuse_route) {  // derived above
             rows = min(tt.rows[g], p.R);
             base = min(tt.base[g], p.R - rows);
         } else {  // clamped to [0, R): only a corrupt workspace could make this matter
@@ -915,7 +1259,7 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
 
 // One persistent launch of the gate/up tiles, the down tiles, or both (and,
 // with fuse_dispatch, the dispatch before them).
-cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = false)
+cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = false, bool fuse_route = false)
 {
     const Shape &s = c.s;
     TcParams p;
@@ -965,6 +1309,32 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = fal
         p.w_of_slot_w = c.w_of_slot;
         p.grid_bar = c.gemm_ready + gemm_ready_words(s) - 1;
         p.clear_words = (int)gemm_ready_words(s) - 1;
+    }
+    if (fuse_route) {  // every counter cleared by clear_counters_kernel before this launch
+        p.fuse_route = 1;
+        p.renorm = s.renorm;
+        p.policy = c.policy;
+        p.router_w[0] = c.router_pub;
+        p.router_w[1] = c.router_priv;
+        p.z = reinterpret_cast<float *>(c.router_rows);  // the chunked router's scratch, unused here
+        p.zpitch = std::max(s.E_pub, s.E_priv);
+        p.idx_w = c.idx;
+        p.ticket_w = c.ticket;
+        p.w_w = c.w;
+        p.tau_w = c.tau;
+        p.tile_counts_w = c.tile_counts;
+        p.route_count = c.audit.route_count;
+        p.route_priv_rows = c.audit.route_priv_rows;
+        p.slots = router_slots(s.T);
+        p.slots4 = router_slots4(s.T);
+        p.counts_w = c.counts;
+        p.offsets_w = c.offsets;
+        p.slot_of_w = c.slot_of;
+        p.tok_of_slot_w = c.tok_of_slot;
+        p.w_of_slot_w = c.w_of_slot;
+        p.bar_a = c.gemm_ready + gemm_ready_words(s) - 4;
+        p.bar_b = c.gemm_ready + gemm_ready_words(s) - 3;
+        p.grid_bar = c.gemm_ready + gemm_ready_words(s) - 1;
     }
     bool ok = true;
     if (gu) ok &= fill_phase(c, kGateUp, p, maps);
@@ -1028,6 +1398,36 @@ bool experts_fuse_dispatch(const Ctx &c)
 {
     return (long long)c.s.H * c.s.I >= (1ll << 20) && grid_fits(c) &&
            fused_dispatch_smem(c.s.E(), router_slots(c.s.T)) <= (size_t)(kStages * kStageBytes);
+}
+
+// Routing in the expert launch: at most 128 tokens (one selection CTA each,
+// all resident with the persistent grid), the masked router of the method
+// (not the unmasked control), pools of at most 256 experts (8 logits a lane
+// in the selection), H <= 2048 (a block of 32 router rows and the token row
+// fit the ring), and the dispatch's per-expert masks fit the ring too.
+bool experts_fuse_route(const Ctx &c)
+{
+    const Shape &s = c.s;
+    return s.T >= 1 && s.T <= kRouteMaxTokens && s.T <= c.num_sms && !c.unmasked && s.H <= kRouteMaxH &&
+           s.E_pub <= 256 && s.E_priv <= 256 && (size_t)s.E() * 24u <= (size_t)(kStages * kStageBytes) &&
+           grid_fits(c);
+}
+
+__global__ void clear_counters_kernel(uint32_t *w, int n)
+{
+    pdl_trigger();
+    pdl_wait();  // the previous forward on this workspace has finished with them
+    for (int i = threadIdx.x; i < n; i += blockDim.x) w[i] = 0u;
+}
+
+// The forward's launches when the expert launch routes: the counters
+// (readiness, tile, barriers) cleared by a one-block kernel, then the
+// persistent launch (routing, dispatch order, gate/up and down).
+cudaError_t launch_experts_routed(const Ctx &c)
+{
+    const cudaError_t err =
+        launch_pdl(clear_counters_kernel, dim3(1), dim3(256), 0, c.stream, c.gemm_ready, (int)gemm_ready_words(c.s));
+    return err == cudaSuccess ? launch_tc(c, true, true, false, true) : err;
 }
 
 cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool fuse_dispatch)

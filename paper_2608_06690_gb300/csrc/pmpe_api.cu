@@ -17,7 +17,7 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 size_t gemm_ready_words(const Shape &s)
 {
     const size_t R = (size_t)s.T * (size_t)s.k;
-    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 3;
+    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 5;
 }
 
 static bool shape_ok(const Shape &s)
@@ -215,10 +215,19 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     if (c.s.T == 0 || stages == 0) return PMPE_OK;
     if (stages & ~PMPE_STAGE_ALL) return PMPE_ERR_INVALID_ARG;
     cudaError_t err = cudaSuccess;
-    // With both the router and the dispatch in this call, the router writes
-    // the dispatch order itself at T <= 128; otherwise the dispatch runs
-    // inside the persistent expert launch when that launch follows the router
-    // in this call (the router zeroes its grid barrier), else as a kernel.
+    // The whole forward at T <= 128: the persistent expert launch routes the
+    // tokens and derives the dispatch order itself.  Otherwise, with both the
+    // router and the dispatch in this call, the router writes the dispatch
+    // order at T <= 128; else the dispatch runs inside the persistent expert
+    // launch when that launch follows the router in this call (the router
+    // zeroes its grid barrier), else as a kernel.
+    const bool all = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && (stages & PMPE_STAGE_GATEUP) &&
+                     (stages & PMPE_STAGE_DOWN);
+    if (all && experts_fuse_route(c)) {
+        err = launch_experts_routed(c);
+        if (err == cudaSuccess && (stages & PMPE_STAGE_COMBINE)) err = launch_combine(c);
+        return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
+    }
     const bool route_disp = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && route_writes_dispatch(c);
     const bool fuse = !route_disp && (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) &&
                       (stages & PMPE_STAGE_GATEUP) && (stages & PMPE_STAGE_DOWN) && experts_fuse_dispatch(c);

@@ -100,13 +100,15 @@ def test_expert_loads_0_1_and_152_rows():
     assert counts[3] >= 152 and counts[shape.E_pub + 2] == 1 and (counts == 0).any()
 
 
-def test_exact_logit_ties_take_the_lower_id():
+@pytest.mark.parametrize("T", [150, 100])
+def test_exact_logit_ties_take_the_lower_id(T):
     """Exactly equal logits (Sec. 3.1 takes the top k after the mask; at an
     exact tie the lower expert id ranks first, the reading both sides
     implement): router rows duplicated in pairs, so every token's selection
-    meets ties and the router takes its exact selection path, and every fifth
+    meets ties (at T = 150 the cluster router takes its exact selection path;
+    at T = 100 the expert launch routes the tokens itself), and every fifth
     token with a zero hidden state, whose logits are all 0."""
-    shape = LayerShape(T=150, H=256, I=128, E_pub=24, E_priv=8, E_sh=0, k=4, renormalize=True)
+    shape = LayerShape(T=T, H=256, I=128, E_pub=24, E_priv=8, E_sh=0, k=4, renormalize=True)
     w, h, pol = make_layer(shape, 49)
     for key in ("router_pub", "router_priv"):
         r = w[key].clone()
