@@ -561,6 +561,9 @@ __device__ bool route_in_launch(const TcParams &p, uint8_t *ring, TileTable &tt,
 // the router tiles' counts ([E][slots + 1] words, inside the ring).
 constexpr size_t fused_dispatch_smem(int E, int slots) { return (size_t)E * (size_t)(slots + 1) * 4u; }
 
+// kRoute: the instantiation that can route the tokens itself (p.fuse_route);
+// the other one carries none of that code (fewer registers, a smaller body).
+template <bool kRoute>
 __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcParams p, const __grid_constant__ TcMaps maps)
 {
     extern __shared__ uint8_t dsmem[];
@@ -628,7 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     // prefetch would otherwise delay)
     if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles && !p.fuse_route) prefetch_first_wave(p);
     pdl_wait();  // the dispatch offsets and slot maps (or the route log, or cleared counters) come from the previous kernel
-    if (p.fuse_route) {
+    if (kRoute && p.fuse_route) {
         const bool ok = route_in_launch(p, dsmem + (sbase - smem_u32(dsmem)), tt, &s_abort);
         if (!ok && tid == 0) s_abort = 1;
         __syncthreads();
@@ -1257,6 +1260,14 @@ bool fill_phase(const Ctx &c, int mode, TcParams &p, TcMaps &maps)
     return ok;
 }
 
+// The dynamic shared-memory limit of one instantiation, raised once per device.
+template <bool kRoute>
+cudaError_t ensure_tc_smem()
+{
+    static std::atomic<int> smem_limit[64];
+    return ensure_dynamic_smem(expert_gemm_tc_kernel<kRoute>, kDynSmem, smem_limit);
+}
+
 // One persistent launch of the gate/up tiles, the down tiles, or both (and,
 // with fuse_dispatch, the dispatch before them).
 cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = false, bool fuse_route = false)
@@ -1348,10 +1359,11 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = fal
                                 2 * (uint64_t)s.E_sh * s.I, (uint64_t)s.T, 16, 32, CU_TENSOR_MAP_SWIZZLE_64B);
     }
     if (!ok) return cudaErrorInvalidValue;
-    static std::atomic<int> smem_limit[64];
-    cudaError_t err = ensure_dynamic_smem(expert_gemm_tc_kernel, kDynSmem, smem_limit);
+    const cudaError_t err = fuse_route ? ensure_tc_smem<true>() : ensure_tc_smem<false>();
     if (err != cudaSuccess) return err;
-    return launch_pdl(expert_gemm_tc_kernel, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
+    if (fuse_route)
+        return launch_pdl(expert_gemm_tc_kernel<true>, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
+    return launch_pdl(expert_gemm_tc_kernel<false>, dim3(c.num_sms), dim3(kThreads), kDynSmem, c.stream, p, maps);
 }
 
 // Whether the persistent grid (one CTA per SM) can be resident all at once:
@@ -1363,12 +1375,13 @@ static bool grid_fits(const Ctx &c)
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return false;
     if (dev >= 0 && dev < 64 && fits[dev].load() != 0) return fits[dev].load() == 1;
-    static std::atomic<int> smem_limit[64];
-    int per_sm = 0;
-    const bool ok = ensure_dynamic_smem(expert_gemm_tc_kernel, kDynSmem, smem_limit) == cudaSuccess &&
-                    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, expert_gemm_tc_kernel, kThreads,
+    int per_sm = 0, per_sm_r = 0;
+    const bool ok = ensure_tc_smem<false>() == cudaSuccess && ensure_tc_smem<true>() == cudaSuccess &&
+                    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, expert_gemm_tc_kernel<false>, kThreads,
                                                                   kDynSmem) == cudaSuccess &&
-                    per_sm >= 1;
+                    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_r, expert_gemm_tc_kernel<true>, kThreads,
+                                                                  kDynSmem) == cudaSuccess &&
+                    per_sm >= 1 && per_sm_r >= 1;
     if (dev >= 0 && dev < 64) fits[dev].store(ok ? 1 : 2);
     return ok;
 }
