@@ -80,6 +80,13 @@ constexpr int kGatherThreads = 32 * kGatherWarps;
 constexpr int kFullArrivals = kLoaders + kGatherThreads;  // per ring stage
 constexpr int kMaxGroups = 2 * kMaxPool + 1;
 constexpr int kPrefetchTiles = 96;            // gate/up tiles (1 MB of weights each) prefetched into L2 at small batches
+// Large batches, the launch following the router: the gate and up weights of
+// the list's first experts (at most 96 MiB, at most 16 experts) prefetched
+// into L2 while the router runs, by the CTAs that start early, after a delay
+// that lets the router's own reads of the token rows go first.
+constexpr size_t kPrefillPrefetchBytes = 96ull << 20;
+constexpr int kPrefillPrefetchExperts = 16;
+constexpr unsigned long long kPrefillPrefetchDelayNs = 14000;
 constexpr int kTQ = 8;                        // tile queue entries (tile indices handed to the CTA's roles)
 constexpr int kTailWaves = 2;                 // waves of tiles at the list's end handed out dynamically
 constexpr int kTQConsumers = 1 + 4 + kGatherWarps;  // MMA thread, epilogue warps, gather warps (one lane each)
@@ -151,6 +158,7 @@ struct TcParams {
     // launch waits for the routing (the weights are inputs, not results of
     // the kernels before); 0 = off
     int prefetch_tiles;
+    int prefetch_experts;      // large batches: CTA e < this prefetches expert e's gate and up rows
     const bf16 *gate_w[2], *up_w[2];  // [E_pool * I, H] public / private
     // optional FP32: the gate and up accumulators saved for the backward,
     // [R][2I] G | U of the routed rows, then [T][2 E_sh I] of the shared
@@ -630,6 +638,21 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     // this launch: after this CTA's router rows have landed, which the
     // prefetch would otherwise delay)
     if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles && !p.fuse_route) prefetch_first_wave(p);
+    if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_experts) {
+        // the list starts with expert 0's tiles, then expert 1's, ...: the
+        // first wave's weights (bounded spin: a fixed delay)
+        const unsigned long long t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < kPrefillPrefetchDelayNs) {
+        }
+        const int e = (int)blockIdx.x;
+        const int q = e < p.E_pub ? 0 : 1;
+        const size_t row0 = (size_t)(q ? e - p.E_pub : e) * p.I;
+        for (int r = 0; r < p.I; r += 128) {
+            const uint32_t bytes = (uint32_t)min(128, p.I - r) * (uint32_t)p.H * 2u;
+            bulk_prefetch_l2(p.gate_w[q] + (row0 + r) * p.H, bytes);
+            bulk_prefetch_l2(p.up_w[q] + (row0 + r) * p.H, bytes);
+        }
+    }
     pdl_wait();  // the dispatch offsets and slot maps (or the route log, or cleared counters) come from the previous kernel
     if (kRoute && p.fuse_route) {
         const bool ok = route_in_launch(p, dsmem + (sbase - smem_u32(dsmem)), tt, &s_abort);
@@ -1308,6 +1331,14 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = fal
     p.status = c.audit.status;
     if (fuse_dispatch) {
         p.fuse_dispatch = 1;
+        const size_t gu_bytes = (size_t)2 * s.I * s.H * 2;  // one expert's gate and up rows
+        p.prefetch_experts = (int)std::min<size_t>(std::min<size_t>(kPrefillPrefetchBytes / gu_bytes,
+                                                                    (size_t)kPrefillPrefetchExperts),
+                                                   (size_t)s.E());
+        for (int q = 0; q < 2; ++q) {
+            p.gate_w[q] = c.gate[q];
+            p.up_w[q] = c.up[q];
+        }
         p.ticket = c.ticket;
         p.w_route = c.w;
         p.tile_counts = c.tile_counts;
