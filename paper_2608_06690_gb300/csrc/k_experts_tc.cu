@@ -580,6 +580,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_abort;
     __shared__ volatile int s_tq[kTQ];
+    __shared__ volatile int s_pdl_done;  // thread 0 has passed griddepcontrol.wait
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t sbase = (smem_u32(dsmem) + 1023u) & ~1023u;
@@ -627,6 +628,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         mbar_init(done_bar, 1);
         for (int i = 0; i < kTQ; ++i) { mbar_init(tq_full_bar(i), 1); mbar_init(tq_empty_bar(i), kTQConsumers); }
         s_abort = 0;
+        s_pdl_done = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 1) {
@@ -634,15 +636,17 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
                      "r"(kTmemCols));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::);
     }
+    __syncthreads();  // s_pdl_done and s_abort are initialised
     // weights of the first wave into L2 while the routing is computed (in
     // this launch: after this CTA's router rows have landed, which the
     // prefetch would otherwise delay)
     if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_tiles && !p.fuse_route) prefetch_first_wave(p);
     if (warp == 2 && lane == 0 && (int)blockIdx.x < p.prefetch_experts) {
         // the list starts with expert 0's tiles, then expert 1's, ...: the
-        // first wave's weights (bounded spin: a fixed delay)
+        // first wave's weights, after the delay, or at once when the router
+        // has already finished (thread 0 passed its wait; bounded spin)
         const unsigned long long t0 = globaltimer_ns();
-        while (globaltimer_ns() - t0 < kPrefillPrefetchDelayNs) {
+        while (globaltimer_ns() - t0 < kPrefillPrefetchDelayNs && !s_pdl_done) {
         }
         const int e = (int)blockIdx.x;
         const int q = e < p.E_pub ? 0 : 1;
@@ -654,6 +658,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         }
     }
     pdl_wait();  // the dispatch offsets and slot maps (or the route log, or cleared counters) come from the previous kernel
+    if (tid == 0) s_pdl_done = 1;
     if (kRoute && p.fuse_route) {
         const bool ok = route_in_launch(p, dsmem + (sbase - smem_u32(dsmem)), tt, &s_abort);
         if (!ok && tid == 0) s_abort = 1;
