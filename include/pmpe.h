@@ -290,7 +290,13 @@ PMPE_API int pmpe_policy_from_requests(const uint8_t *req_policy, const int32_t 
                                        uint8_t *policy_out, void *stream);
 
 /* The whole layer forward (all stages) on `stream`.  No host synchronisation;
- * expert row counts stay on the device. */
+ * expert row counts stay on the device.  The expert launch is persistent, one
+ * CTA per SM, and its CTAs wait for one another (grid barriers, readiness
+ * counters): it assumes the whole grid is resident at once, which the library
+ * checks for this device before it takes that form.  If other work on the GPU
+ * holds SMs for longer than the bounded waits (4 s), the waits expire, the
+ * kernel sets PMPE_STATUS_PIPELINE_TIMEOUT in the status word and returns;
+ * the outputs of that call are then not valid. */
 PMPE_API int pmpe_moe_forward(const pmpe_moe_desc *d, void *stream);
 
 /* Run a subset of the stages (PMPE_STAGE_* bits), in pipeline order.  Each
