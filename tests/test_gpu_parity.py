@@ -40,6 +40,18 @@ CASES = {
     # k > 8 takes the router's sorting-network path; 40 public experts span two chunks
     "k12_two_chunks_pool_softmax": (LayerShape(T=150, H=256, I=128, E_pub=40, E_priv=16, E_sh=0, k=12,
                                                renormalize=False), 44, "iid"),
+    # the expert launch's own routing (T <= 128) on a DeepSeek-like layer:
+    # pool softmax, 64-expert public pool, shared experts, k = 6
+    "small_batch_pool_softmax_shared": (LayerShape(T=96, H=256, I=128, E_pub=64, E_priv=16, E_sh=2, k=6,
+                                                   renormalize=False), 50, "iid"),
+    # the batch sizes on both sides of the in-launch routing's limit
+    "t128_routed_in_launch": (LayerShape(T=128, H=256, I=128, E_pub=16, E_priv=8, E_sh=0, k=2, renormalize=True),
+                              51, "iid"),
+    "t129_cluster_router": (LayerShape(T=129, H=256, I=128, E_pub=16, E_priv=8, E_sh=0, k=2, renormalize=True),
+                            52, "iid"),
+    # H = 384: the routing lanes hold one or two 16-byte pieces of a row
+    "h384_small_batch": (LayerShape(T=50, H=384, I=128, E_pub=24, E_priv=8, E_sh=0, k=4, renormalize=True), 53,
+                         "iid"),
     # 9 rows of 8 KB per token: a ring of two tokens does not fit the bulk
     # combine's shared memory, so the thread-per-chunk combine runs
     "wide_rows_chunk_combine": (LayerShape(T=40, H=4096, I=128, E_pub=12, E_priv=8, E_sh=1, k=8, renormalize=True),
