@@ -157,13 +157,16 @@ def test_zero_tokens_is_a_noop():
     torch.cuda.synchronize()
 
 
-def test_determinism_recovery_and_batch_invariance():
+@pytest.mark.parametrize("T", [256, 96])
+def test_determinism_recovery_and_batch_invariance(T):
     """Allow -> deny -> allow on the same inputs: the recovery pass is
     bitwise identical to the first allow pass (Sec. 3.3, App. F.3); a row's
     output is bitwise unchanged when other rows' policies flip (App. F.1,
-    mixed-policy batches)."""
+    mixed-policy batches).  The forwards run back to back on one workspace
+    with no host synchronisation, with the cluster router (T = 256) and with
+    the routing inside the expert launch (T = 96)."""
     from paper_2608_06690_gb300 import pmpe
-    shape = LayerShape(T=256, H=256, I=256, E_pub=16, E_priv=8, E_sh=1, k=3, renormalize=True)
+    shape = LayerShape(T=T, H=256, I=256, E_pub=16, E_priv=8, E_sh=1, k=3, renormalize=True)
     w, h, _ = make_layer(shape, 43)
     wd, hd, _ = to_device(w, h, None)
     layer = pmpe.MoeLayer(shape, wd)
