@@ -285,7 +285,7 @@ __device__ bool grid_barrier(uint32_t *ctr, uint32_t target, volatile int *abort
 }
 
 constexpr int kRouteMaxTokens = 128;   // routing in the launch: one selection CTA per token
-constexpr int kRouteMaxH = 2048;       // a 32-expert block of router rows (128 KB) plus the token row fit the ring
+constexpr int kRouteMaxH = 2048;       // the logits hold a row's 16-byte pieces in registers, 8 a lane at most
 constexpr int kRouteXChunks = kRouteMaxH / 256;  // 16-byte pieces of the token row per lane
 
 __device__ __forceinline__ float dot8_bf16(const uint4 &a, const uint4 &b, float acc)
@@ -1452,8 +1452,9 @@ bool experts_fuse_dispatch(const Ctx &c)
 // Routing in the expert launch: at most 128 tokens (one selection CTA each,
 // all resident with the persistent grid), the masked router of the method
 // (not the unmasked control), pools of at most 256 experts (8 logits a lane
-// in the selection), H <= 2048 (a block of 32 router rows and the token row
-// fit the ring), and the dispatch's per-expert masks fit the ring too.
+// in the selection), H <= 2048 (a lane holds at most 8 16-byte pieces of a
+// row in registers for the logits), and the dispatch's per-expert masks fit
+// the ring.
 bool experts_fuse_route(const Ctx &c)
 {
     const Shape &s = c.s;
