@@ -152,6 +152,11 @@ struct TcParams {
     uint32_t *tile_counts_w;         // [E][slots4]
     uint32_t *route_count, *route_priv_rows;
     uint32_t *bar_a, *bar_b;         // grid barriers after the logits and after the selection
+    // with fuse_route: the weighted combine too, after a last grid barrier
+    // (bar_d) once every CTA's down tiles are stored
+    int fuse_combine;
+    uint32_t *bar_d;
+    bf16 *out;                       // [T, H]
     // small batches (every expert at most one 128-row block): the first
     // `prefetch_tiles` gate/up tiles of the list of all experts have their
     // weights prefetched into L2 by the CTA of the same index, before the
@@ -1239,6 +1244,56 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base), "r"(kTmemCols));
     }
+    if (kRoute && p.fuse_combine) {
+        // ---- the weighted combine (Sec. 3.1), as combine_kernel sums it:
+        // j ascending, then the shared experts, in FP32.  Every epilogue
+        // warp's stores are complete (wait_group 0 above); they are made
+        // visible, then every CTA meets at the last grid barrier.
+        if (warp >= 2 && warp < 6 && lane == 0) {
+            asm volatile("fence.proxy.async.global;\n" ::: "memory");
+            __threadfence();
+        }
+        if (grid_barrier(p.bar_d, gridDim.x, &s_abort, p.status)) {
+            const bf16 *y = p.ph[kDown].C_routed;
+            const bf16 *y_sh = p.E_sh > 0 ? p.ph[kDown].C_shared : nullptr;
+            const int nv = p.H / 8;
+            for (int t = (int)blockIdx.x; t < p.T; t += (int)gridDim.x) {
+                for (int c = tid; c < nv; c += kThreads) {
+                    float acc[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+                    for (int j = 0; j < p.k; ++j) {
+                        int slot = p.slot_of_w[(size_t)t * p.k + j];
+                        if ((unsigned)slot >= (unsigned)p.R) slot = 0;  // only after a dispatch mismatch (status set)
+                        const uint4 v = *reinterpret_cast<const uint4 *>(y + (size_t)slot * p.H + (size_t)c * 8);
+                        const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const float2 f = __bfloat1622float2(b[q]);
+                            acc[2 * q] += f.x;
+                            acc[2 * q + 1] += f.y;
+                        }
+                    }
+                    if (y_sh) {
+                        const uint4 v = *reinterpret_cast<const uint4 *>(y_sh + (size_t)t * p.H + (size_t)c * 8);
+                        const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const float2 f = __bfloat1622float2(b[q]);
+                            acc[2 * q] += f.x;
+                            acc[2 * q + 1] += f.y;
+                        }
+                    }
+                    uint4 o;
+                    o.x = pack_bf16x2(acc[0], acc[1]);
+                    o.y = pack_bf16x2(acc[2], acc[3]);
+                    o.z = pack_bf16x2(acc[4], acc[5]);
+                    o.w = pack_bf16x2(acc[6], acc[7]);
+                    reinterpret_cast<uint4 *>(p.out + (size_t)t * p.H)[c] = o;
+                }
+            }
+        }
+    }
 }
 
 // ------------------------------------------------------------ host side
@@ -1298,7 +1353,8 @@ cudaError_t ensure_tc_smem()
 
 // One persistent launch of the gate/up tiles, the down tiles, or both (and,
 // with fuse_dispatch, the dispatch before them).
-cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = false, bool fuse_route = false)
+cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = false, bool fuse_route = false,
+                      bool fuse_combine = false)
 {
     const Shape &s = c.s;
     TcParams p;
@@ -1382,6 +1438,11 @@ cudaError_t launch_tc(const Ctx &c, bool gu, bool down, bool fuse_dispatch = fal
         p.bar_a = c.gemm_ready + gemm_ready_words(s) - 4;
         p.bar_b = c.gemm_ready + gemm_ready_words(s) - 3;
         p.grid_bar = c.gemm_ready + gemm_ready_words(s) - 1;
+        if (fuse_combine) {
+            p.fuse_combine = 1;
+            p.bar_d = c.gemm_ready + gemm_ready_words(s) - 5;
+            p.out = c.out;
+        }
     }
     bool ok = true;
     if (gu) ok &= fill_phase(c, kGateUp, p, maps);
@@ -1473,11 +1534,11 @@ __global__ void clear_counters_kernel(uint32_t *w, int n)
 // The forward's launches when the expert launch routes: the counters
 // (readiness, tile, barriers) cleared by a one-block kernel, then the
 // persistent launch (routing, dispatch order, gate/up and down).
-cudaError_t launch_experts_routed(const Ctx &c)
+cudaError_t launch_experts_routed(const Ctx &c, bool combine)
 {
     const cudaError_t err =
         launch_pdl(clear_counters_kernel, dim3(1), dim3(256), 0, c.stream, c.gemm_ready, (int)gemm_ready_words(c.s));
-    return err == cudaSuccess ? launch_tc(c, true, true, false, true) : err;
+    return err == cudaSuccess ? launch_tc(c, true, true, false, true, combine) : err;
 }
 
 cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool fuse_dispatch)

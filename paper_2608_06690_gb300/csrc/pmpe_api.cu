@@ -17,7 +17,7 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 size_t gemm_ready_words(const Shape &s)
 {
     const size_t R = (size_t)s.T * (size_t)s.k;
-    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 5;
+    return (R + 127) / 128 + (size_t)s.E() + ((size_t)s.T + 127) / 128 + 6;
 }
 
 static bool shape_ok(const Shape &s)
@@ -223,9 +223,8 @@ int pmpe_moe_forward_stages(const pmpe_moe_desc *d, unsigned stages, void *strea
     // zeroes its grid barrier), else as a kernel.
     const bool all = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && (stages & PMPE_STAGE_GATEUP) &&
                      (stages & PMPE_STAGE_DOWN);
-    if (all && experts_fuse_route(c)) {
-        err = launch_experts_routed(c);
-        if (err == cudaSuccess && (stages & PMPE_STAGE_COMBINE)) err = launch_combine(c);
+    if (all && experts_fuse_route(c)) {  // the combine too, when asked for
+        err = launch_experts_routed(c, (stages & PMPE_STAGE_COMBINE) != 0);
         return err == cudaSuccess ? PMPE_OK : PMPE_ERR_CUDA;
     }
     const bool route_disp = (stages & PMPE_STAGE_ROUTE) && (stages & PMPE_STAGE_PERMUTE) && route_writes_dispatch(c);

@@ -159,10 +159,11 @@ cudaError_t launch_experts(const Ctx &c, bool zero_ready, bool fuse_dispatch);
 bool experts_fuse_dispatch(const Ctx &c);
 // Whether the expert launch can route the tokens itself (T <= 128, the
 // masked router, pools of at most 256 experts, H <= 2048, a resident grid),
-// and that form of the forward's first launches: a kernel clearing the
-// counters, then the persistent launch (routing, dispatch, both GEMMs).
+// and that form of the forward: a kernel clearing the counters, then the
+// persistent launch (routing, dispatch, both GEMMs and, with `combine`, the
+// weighted combine).
 bool experts_fuse_route(const Ctx &c);
-cudaError_t launch_experts_routed(const Ctx &c);
+cudaError_t launch_experts_routed(const Ctx &c, bool combine);
 cudaError_t launch_combine(const Ctx &c);
 // The token rows of the dispatch slots of groups g0 .. g1 - 1 copied from the
 // hidden states into the workspace's dispatched-row matrix (a_perm), which the

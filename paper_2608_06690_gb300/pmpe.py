@@ -55,12 +55,12 @@ def kernels_per_forward(shape) -> int:
     where the persistent expert grid is resident at once (the rule the
     library applies when it launches the forward).  At most 128 tokens (H
     up to 2048, pools of at most 256 experts): a kernel clearing the expert
-    launch's counters, the expert launch (routing, dispatch order, both
-    GEMMs) and the combine.  Otherwise the router, the expert GEMMs and the
+    launch's counters and the expert launch (routing, dispatch order, both
+    GEMMs, combine).  Otherwise the router, the expert GEMMs and the
     combine, plus a dispatch kernel unless the expert launch derives the
     dispatch order (experts of at least 2^20 weights a projection)."""
     if shape.T <= 128 and shape.H <= 2048 and max(shape.E_pub, shape.E_priv) <= 256:
-        return 3
+        return 2
     return 3 if shape.H * shape.I >= (1 << 20) else 4
 # kernels one private-branch backward launches: the dispatched rows of the
 # private experts, dout row gather, the dL/da GEMM, the gate/up recompute GEMM

@@ -80,7 +80,7 @@ def test_workspace_size_and_layout(pmpe):
                     ticket=4 * R, tok_of_slot=4 * R, w_of_slot=4 * R, tile_done=4 * slots,
                     router_lists=8 * ctas_all * 128 * sh.k, router_meta=16 * ctas_all * 128,
                     # readiness counters, then the expert kernel's tile and grid-barrier counters
-                    gemm_ready=4 * ((R + 127) // 128 + E + (T + 127) // 128 + 5),
+                    gemm_ready=4 * ((R + 127) // 128 + E + (T + 127) // 128 + 6),
                     router_rows=2 * ctas * 128 * sh.H, a_perm=2 * R * sh.H, act=2 * R * sh.I, y=2 * R * sh.H,
                     act_sh=2 * T * sh.E_sh * sh.I, y_sh=2 * T * sh.H if sh.E_sh else 0,
                     tile_counts=4 * E * ((slots + 3) // 4 * 4))
@@ -91,7 +91,7 @@ def test_workspace_size_and_layout(pmpe):
         assert LL["router_meta"] % 16 == 0 and LL["router_lists"] % 8 == 0 and LL["router_rows"] % 1024 == 0
         assert LL["tile_done"] == LL["counts"] + 4 * E  # one memset clears these three
         assert LL["gemm_ready"] == LL["tile_done"] + 4 * slots
-        gr_end = LL["gemm_ready"] + 4 * ((R + 127) // 128 + E + (T + 127) // 128 + 5)
+        gr_end = LL["gemm_ready"] + 4 * ((R + 127) // 128 + E + (T + 127) // 128 + 6)
         assert LL["tile_counts"] % 16 == 0 and gr_end <= LL["tile_counts"] <= gr_end + 12
     assert pmpe.workspace_size(LayerShape(64, 200, 128, 8, 4, 0, 2, True)) == 0    # H % 128
     assert pmpe.workspace_size(LayerShape(64, 256, 128, 8, 4, 0, 9, True)) == 0    # k > pool
