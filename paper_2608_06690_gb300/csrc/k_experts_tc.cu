@@ -208,8 +208,29 @@ __device__ __forceinline__ int total_tiles(const TcParams &p, const TileTable &t
     return (p.has_gu ? tt.prefix[kGateUp][G] : 0) + (p.has_down ? tt.prefix[kDown][G] : 0);
 }
 
+// The down GEMM's order of the groups: with shared experts their group sits
+// after the first half of the routed experts, so that the list ends with
+// routed down tiles (K = I) instead of the shared group's (K = E_sh I, the
+// launch's longest tiles), which otherwise made the last wave uneven; there
+// the shared group's gate/up tiles, the last of the gate/up list, are long
+// finished.  The gate/up GEMM keeps the groups in id order (the copy warps
+// fill no stage after one whose A comes through TMA).  down_place inverts it.
+__device__ __forceinline__ int down_group(const TcParams &p, int L)
+{
+    if (p.E_sh == 0) return L;
+    const int h = p.E / 2;
+    return L < h ? L : (L == h ? p.E : L - 1);
+}
+__device__ __forceinline__ int down_place(const TcParams &p, int g)
+{
+    if (p.E_sh == 0) return g;
+    const int h = p.E / 2;
+    return g < h ? g : (g == p.E ? h : g + 1);
+}
+
 // Tile `tile` of the list: the gate/up tiles (when this launch runs them),
-// then the down tiles; inside a GEMM, group by group, n-tile major.
+// then the down tiles; inside a GEMM, group by group (the down GEMM in
+// down_group order), n-tile major.
 __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &tt, int G, int tile)
 {
     Tile t;
@@ -224,9 +245,10 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
         if (pre[mid] <= local_all) lo = mid; else hi = mid - 1;
     }
     t.bn = p.ph[t.ph].bn;
-    t.g = lo;
-    t.shared = lo >= p.E;
-    const int rows = tt.rows[lo];
+    const int g = t.ph == kDown ? down_group(p, lo) : lo;
+    t.g = g;
+    t.shared = g >= p.E;
+    const int rows = tt.rows[g];
     const int mt = (rows + BM - 1) / BM;
     const int local = local_all - pre[lo];
     const int n_tile = local / mt;
@@ -235,7 +257,7 @@ __device__ __forceinline__ Tile decode_tile(const TcParams &p, const TileTable &
     t.n0 = n_tile * t.bn;
     t.cb = n_tile;
     t.rows = min(BM, rows - t.m0);
-    t.row_base = tt.base[lo];
+    t.row_base = tt.base[g];
     t.nkb = group_k(p, t.ph == kGateUp ? kGateUp : kDown, t.shared) / BK;
     return t;
 }
@@ -784,7 +806,8 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         tt.rows[g] = rows;
         tt.base[g] = base;
         tt.mpre[g + 1] = mt;
-        for (int ph = 0; ph < 2; ++ph) tt.prefix[ph][g + 1] = mt * (group_n(p, ph, shared) / p.ph[ph].bn);
+        tt.prefix[kGateUp][g + 1] = mt * (group_n(p, kGateUp, shared) / p.ph[kGateUp].bn);
+        tt.prefix[kDown][down_place(p, g) + 1] = mt * (group_n(p, kDown, shared) / p.ph[kDown].bn);
     }
     // the same value in every thread of every CTA (all read the same offsets)
     multi = __syncthreads_or(multi);
