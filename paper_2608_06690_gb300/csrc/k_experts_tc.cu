@@ -280,19 +280,28 @@ __device__ __forceinline__ void prefetch_first_wave(const TcParams &p)
     }
 }
 
+// Arrival at a grid barrier: a release add, so that the writes the CTA
+// barrier before it ordered (every thread's) are visible to whoever
+// acquires the count.
+__device__ __forceinline__ void grid_arrive(uint32_t *ctr)
+{
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;\n" ::"l"(ctr) : "memory");
+}
+
 // Every CTA of the grid arrives (after all of its threads' writes), then
-// waits, bounded, until `target` arrivals are counted; writes before the
-// barrier, by any thread of any CTA, are visible after it.  The grid is
-// resident all at once (checked before the launch).  False after a timeout
-// or an abort.
+// waits, bounded, until `target` arrivals are counted (acquire loads; the CTA
+// barrier after them orders the other threads); writes before the barrier,
+// by any thread of any CTA, are visible after it.  The grid is resident all
+// at once (checked before the launch).  False after a timeout or an abort.
+// (A release add and a tight acquire spin measured 0.5 us faster a decode
+// step than a full fence, a relaxed add and a spin with back-off.)
 __device__ bool grid_barrier(uint32_t *ctr, uint32_t target, volatile int *abort_flag, uint32_t *status)
 {
     __shared__ int s_ok;
     __syncthreads();
     if (threadIdx.x == 0) {
         int ok = 1;
-        __threadfence();
-        atomicAdd(ctr, 1u);
+        grid_arrive(ctr);
         const unsigned long long t0 = globaltimer_ns();
         while (ld_acquire_gpu(ctr) < target) {
             if (*abort_flag) { ok = 0; break; }
@@ -302,9 +311,7 @@ __device__ bool grid_barrier(uint32_t *ctr, uint32_t target, volatile int *abort
                 ok = 0;
                 break;
             }
-            __nanosleep(32);
         }
-        __threadfence();
         s_ok = ok;
     }
     __syncthreads();
@@ -690,10 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         const bool ok = route_in_launch(p, dsmem + (sbase - smem_u32(dsmem)), tt, &s_abort);
         if (!ok && tid == 0) s_abort = 1;
         __syncthreads();
-        if (tid == 0) {  // arrive at the grid barrier; the roles wait for it (wait_dispatch)
-            __threadfence();
-            atomicAdd(p.grid_bar, 1u);
-        }
+        if (tid == 0) grid_arrive(p.grid_bar);  // the roles wait for it (wait_dispatch)
     }
     if (p.fuse_dispatch) {
         // ---- the dispatch order, as dispatch_kernel derives it.  pre[e][s]:
@@ -762,10 +766,7 @@ __global__ void __launch_bounds__(kThreads, 1) expert_gemm_tc_kernel(const TcPar
         // it first reads what other CTAs wrote here, so that the tile table,
         // the first weight loads and the other CTAs' arrivals overlap
         __syncthreads();
-        if (tid == 0) {
-            __threadfence();
-            atomicAdd(p.grid_bar, 1u);
-        }
+        if (tid == 0) grid_arrive(p.grid_bar);
     }
     // Until every CTA has arrived: the slot maps (tok_of_slot, w_of_slot) and
     // the readiness and tile counters (cleared by CTA 0) are not yet final.
