@@ -52,7 +52,7 @@ def flush_l2(flush):
 # DRAM read + write bytes per launch of the dominant kernel (the persistent
 # expert GEMM pair), from one ncu capture of the current kernel per workload:
 # profiles/expert_gemm_tc_qwen3_prefill.md and ..._qwen3_decode.md.
-NCU_TRAFFIC = {"qwen3_prefill": {"experts": 1.7952e9}, "qwen3_decode": {"experts": 1.3547e9}}
+NCU_TRAFFIC = {"qwen3_prefill": {"experts": 1.7942e9}, "qwen3_decode": {"experts": 1.3541e9}}
 
 
 def _dist():
