@@ -69,9 +69,10 @@ def to_device(w: dict, h, pol, device="cuda"):
     return wd, h.to(device).contiguous(), (None if pol is None else pol.to(device).contiguous())
 
 
-def run_gpu_layer(shape: LayerShape, w: dict, h, pol, audit_reset=True, stages=None):
+def run_gpu_layer(shape: LayerShape, w: dict, h, pol, audit_reset=True, stages=None, stage_seq=None):
     """Run the layer through the C ABI; return outputs, the route log, the
-    audit counters and the dispatch intermediates, all on the host."""
+    audit counters and the dispatch intermediates, all on the host.  With
+    ``stage_seq``, one call per listed stage mask on the same workspace."""
     from paper_2608_06690_gb300 import pmpe
     layer = pmpe.MoeLayer(shape, w)
     T, k, E = shape.T, shape.k, shape.E
@@ -79,8 +80,8 @@ def run_gpu_layer(shape: LayerShape, w: dict, h, pol, audit_reset=True, stages=N
     wt = torch.full((T, k), float("nan"), dtype=torch.float32, device="cuda")
     audit = torch.zeros(pmpe.audit_words(T, E), dtype=torch.int32, device="cuda")
     out = torch.full((T, shape.H), float("nan"), dtype=torch.bfloat16, device="cuda")
-    layer.forward(h, pol, out=out, topk_idx=idx, topk_w=wt, audit=audit,
-                  stages=pmpe.STAGE_ALL if stages is None else stages)
+    for st in (stage_seq if stage_seq is not None else [pmpe.STAGE_ALL if stages is None else stages]):
+        layer.forward(h, pol, out=out, topk_idx=idx, topk_w=wt, audit=audit, stages=st)
     torch.cuda.synchronize()
     a = pmpe.audit_read(audit, T, E, check_status=False)
     ws = layer.workspace(T)

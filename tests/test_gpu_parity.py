@@ -147,6 +147,23 @@ def test_exact_logit_ties_take_the_lower_id(T):
                 assert sel[j + 1] == e + 1, (t, sel)
 
 
+@pytest.mark.parametrize("T", [96, 300])
+def test_stage_by_stage_calls_match_the_oracle(T):
+    """The layer run one stage per call on one workspace (route + dispatch,
+    gate/up + down, combine): at T <= 128 the cluster router then writes the
+    dispatch order itself; above, the dispatch kernel runs.  Outputs, route
+    log, audit and dispatch order against the oracle."""
+    from paper_2608_06690_gb300 import pmpe
+    shape = LayerShape(T=T, H=256, I=256, E_pub=24, E_priv=8, E_sh=1, k=4, renormalize=True)
+    w, h, pol = make_layer(shape, 54)
+    wd, hd, pd = to_device(w, h, pol)
+    seq = [pmpe.STAGE_ROUTE | pmpe.STAGE_PERMUTE, pmpe.STAGE_GATEUP | pmpe.STAGE_DOWN, pmpe.STAGE_COMBINE]
+    gpu = run_gpu_layer(shape, wd, hd, pd, stage_seq=seq)
+    check_against_oracle(shape, w, h, pol, gpu)
+    check_audit(shape, pol, gpu)
+    check_dispatch(shape, h, gpu)
+
+
 def test_zero_tokens_is_a_noop():
     from paper_2608_06690_gb300 import pmpe
     shape = LayerShape(T=0, H=256, I=128, E_pub=8, E_priv=4, E_sh=0, k=2, renormalize=True)
